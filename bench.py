@@ -1,0 +1,418 @@
+"""Benchmark of the grouped multi-tenant step on GB300.
+
+One step = one pass of the whole hot path over one group: host plan (timed
+separately), packer, all backbone blocks over the packed varlen batch,
+final norm + pool, every tenant's head forward, L2 loss and head backward.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload llama7b]
+    python bench.py --impl reference ...   # the fp64 CPU oracle, timed
+
+Prints ONE JSON line (rank 0).  `value` is whole-job tokens/s with inputs
+resident in HBM; `e2e` is the same metric through the C ABI with the step's
+inputs copied from pinned host memory and its losses / predictions read back
+inside the timed region.  With N > 1 (torchrun) every rank runs its own
+group (independent replicas, weak scaling, no data-path collective).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "grouped fwd+head-bwd tokens/s on 1 GB300; % bf16 tensor peak; speedup vs per-tenant"
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"],
+                    bf16_sustained=d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                    source="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
+
+
+def workload_desc(w):
+    b = w.backbone
+    return (f"{w.name}: {len(w.tenants)} tenants, {len(w.samples)} samples, "
+            f"{w.n_tokens} packed tokens; {b.n_layers} blocks d={b.d} {b.n_heads}x{b.head_dim} "
+            f"heads ({b.n_kv_heads} kv), FFN {b.d_ff} {'SwiGLU' if b.glu == 0 else 'GeGLU'}")
+
+
+def oracle_requests(w):
+    return [dict(tenant=r.tenant, schema=r.schema,
+                 samples=[dict(n_img=s.n_img, text_len=s.text_len, vision_row=s.vision_row,
+                               text_pos=s.text_pos, target_off=s.target_off) for s in r.samples])
+            for r in w.requests]
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (the reference arm and the cpu_baseline key)
+# ---------------------------------------------------------------------------
+
+def oracle_sample_run(w, n_layers, bw_np=None, inp_np=None):
+    """Time the fp64 oracle on one sample of the workload through `n_layers`
+    blocks.  Returns (seconds, tokens, description)."""
+    import synth
+    from oracle import model as M
+    bb = M.backbone_dict(w)
+    if bw_np is None:
+        bw_np = synth.to_numpy_tree(synth.make_backbone_weights(w, device="cpu")) \
+            if w.backbone.n_layers * w.backbone.d < 10000 else None
+    s = min(w.samples, key=lambda s: s.length(w.backbone.vision_tokens))
+    t0 = time.perf_counter()
+    x = M.sample_embeddings(bb, vars(s), inp_np["vision"], inp_np["text_ids"],
+                            bw_np["text_table"])
+    h = M.backbone_sample(bb, bw_np, x, n_layers=n_layers)
+    M.mean_pool(h)
+    dt = time.perf_counter() - t0
+    L = x.shape[0]
+    return dt, L, (f"1 sample ({L} tokens) through {n_layers} of {w.backbone.n_layers} blocks "
+                   f"+ final norm/pool; tokens/s scaled by {n_layers}/{w.backbone.n_layers}")
+
+
+def host_numpy_inputs(w, bw, inp, n_layers):
+    """Host copies (bf16 bit patterns) of what one oracle sample needs."""
+    import synth
+    bw_np = dict(layers=[synth.to_numpy_tree(L) for L in bw["layers"][:n_layers]],
+                 final_norm=synth.bf16_bits(bw["final_norm"]),
+                 text_table=synth.bf16_bits(bw["text_table"]))
+    return bw_np, synth.to_numpy_tree(inp)
+
+
+# ---------------------------------------------------------------------------
+# clocks
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{gpu_index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.f,
+                stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                rows.append(parts)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v == "Active"})
+        loaded = [v for v in sm if mx and v > 0.3 * max(mx)] or sm
+        return dict(sm_mhz=float(np.median(loaded)) if loaded else None,
+                    sm_max_mhz=max(mx) if mx else None, reasons=reasons, samples=len(rows))
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+
+    import synth
+    from paper_2607_16074_gb300 import build as B
+    from paper_2607_16074_gb300 import jnx as J
+    from paper_2607_16074_gb300 import runtime as R
+
+    B.build()
+    J.lib()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = synth.make_workload(args.workload)
+    # each rank owns an independent group (same shapes, its own inputs)
+    w.seed = w.seed + 1000 * rank if rank else w.seed
+    bw = synth.make_backbone_weights(w, device=dev)
+    hw = synth.make_head_weights(w, device=dev)
+    inp = synth.make_inputs(w, device=dev)
+    inp_host = {k: v.cpu().pin_memory() for k, v in inp.items()}
+
+    reqs = oracle_requests(w)
+    t0 = time.perf_counter()
+    plan = J.jnx_group_plan(w.schemas(), reqs, len(w.tenants), w.max_samples, w.max_tokens)
+    plan_ms = (time.perf_counter() - t0) * 1e3
+    group = R.DeviceGroup(plan, device=dev)
+    backbone = R.DeviceBackbone(w.backbone, bw, n_tenants=len(w.tenants))
+    heads = R.DeviceHeads(w.tenants, w.backbone.d, hw, device=dev)
+    step = R.GroupedStep(backbone, heads, group, device=dev)
+    preds = torch.zeros_like(inp["targets"])
+    stream = torch.cuda.current_stream()
+
+    def one_step():
+        step.run(inp["vision"], inp["text_ids"], inp["targets"], preds)
+
+    for _ in range(args.warmup):
+        one_step()
+    R.check_status(step.ws_bb)
+    R.check_status(step.ws_h)
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    # ---- device-resident timed region, every launch traced ----------------
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    cap = 4096 * max(1, args.steps)
+    barrier()
+    torch.cuda.synchronize()
+    J.jnx_trace_enable(cap)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        one_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = J.jnx_trace_count()
+    kinds, ms, work = J.jnx_trace_read(cap)
+    J.jnx_trace_disable()
+    clk = clocks.stop()
+    t_ms = e0.elapsed_time(e1)
+    if world > 1:
+        tt = torch.tensor([t_ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        t_ms = float(tt.item())
+    tokens = plan.n_tokens
+    value = tokens * world * args.steps / (t_ms / 1e3)
+
+    # ---- end to end through the C ABI from pinned host memory --------------
+    vis_d, tid_d, tgt_d = inp["vision"], inp["text_ids"], inp["targets"]
+    loss_h = torch.empty(step.loss.shape, dtype=torch.float32).pin_memory()
+    preds_h = torch.empty(preds.shape, dtype=torch.float32).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in inp_host.values())
+    d2h = loss_h.numel() * 4 + preds_h.numel() * 4
+
+    def e2e_step():
+        vis_d.copy_(inp_host["vision"], non_blocking=True)
+        tid_d.copy_(inp_host["text_ids"], non_blocking=True)
+        tgt_d.copy_(inp_host["targets"], non_blocking=True)
+        p = J.jnx_group_plan(w.schemas(), reqs, len(w.tenants), w.max_samples, w.max_tokens)
+        g = R.DeviceGroup(p, device=dev, non_blocking=True)
+        step.group = g
+        step.run(vis_d, tid_d, tgt_d, preds)
+        loss_h.copy_(step.loss, non_blocking=True)
+        preds_h.copy_(preds, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+        return g
+
+    keep = e2e_step()
+    barrier()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        keep = e2e_step()
+    torch.cuda.synchronize()
+    barrier()
+    e2e_ms = (time.perf_counter() - t0) * 1e3
+    if world > 1:
+        tt = torch.tensor([e2e_ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    step.group = group
+    e2e_plan_bytes = sum(a.nbytes for a in (plan.cu_seqlens, plan.sample_slot, plan.sample_target,
+                                            plan.seg_offsets, plan.gather_src, plan.pos_ids))
+
+    # ---- per-tenant isolated execution (the speedup's baseline) -----------
+    speed = None
+    if not args.no_per_tenant:
+        iso = []
+        for t in range(len(w.tenants)):
+            sub = w.subset([t])
+            p = J.jnx_group_plan(sub.schemas(), oracle_requests(sub), len(w.tenants),
+                                 w.max_samples, w.max_tokens)
+            if p.n_samples == 0:
+                continue
+            iso.append(R.GroupedStep(backbone, heads, R.DeviceGroup(p, device=dev), device=dev))
+        for st in iso:  # warm
+            st.run(inp["vision"], inp["text_ids"], inp["targets"], preds)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for st in iso:
+            st.run(inp["vision"], inp["text_ids"], inp["targets"], preds)
+        b.record(stream)
+        torch.cuda.synchronize()
+        t_iso = a.elapsed_time(b)
+        speed = dict(per_tenant_ms=round(t_iso, 3), grouped_ms=round(t_ms / args.steps, 3),
+                     speedup=round(t_iso / (t_ms / args.steps), 4),
+                     per_tenant_tokens_per_s=round(tokens / (t_iso / 1e3), 1))
+        del iso
+
+    # ---- roofline of the dominant kernel (all backbone GEMM launches) ------
+    peaks = load_peaks()
+    gemm_mask = np.isin(kinds, (3, 5, 6, 7))
+    g_flops, g_ms = float(work[gemm_mask].sum()), float(ms[gemm_mask].sum())
+    g_tf = g_flops / (g_ms / 1e3) / 1e12 if g_ms > 0 else 0.0
+    per_kernel = {}
+    tot_ms = float(ms.sum())
+    for k in sorted(set(kinds.tolist())):
+        m = kinds == k
+        name = J.KERNEL_NAMES.get(k, str(k))
+        kms = float(ms[m].sum())
+        wk = float(work[m].sum())
+        rate = wk / (kms / 1e3) if kms > 0 else 0.0
+        per_kernel[name] = dict(launches=int(m.sum()), ms=round(kms, 3),
+                                share=round(kms / tot_ms, 4) if tot_ms else None,
+                                **({"tflops": round(rate / 1e12, 1)} if k in J.TENSOR_KERNELS
+                                   else {"gbs": round(rate / 1e9, 1)}))
+    step_flops = float(work[np.isin(kinds, J.TENSOR_KERNELS + (10, 11))].sum()) / args.steps
+    step_tf = step_flops / (t_ms / args.steps / 1e3) / 1e12
+    roofline = dict(kernel="k_gemm (tcgen05; all backbone GEMM launches: QKV+RoPE, O+residual, "
+                           "gate/up+GLU, down+residual)",
+                    bound="tensor", achieved=round(g_tf, 1), peak=peaks["bf16_sustained"],
+                    unit="TFLOP/s", frac=round(g_tf / peaks["bf16_sustained"], 4),
+                    frac_of_burst=round(g_tf / peaks["bf16"], 4),
+                    peak_note=f"bf16_tflops_sustained of {peaks['source']} peaks "
+                              "(kernel timed inside a long step)",
+                    traffic=None)
+
+    # ---- CPU oracle baseline (rank 0, N = 1 only) --------------------------
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        nl = min(args.oracle_layers, w.backbone.n_layers)
+        bw_np, inp_np = host_numpy_inputs(w, bw, inp, nl)
+        dt, L, desc = oracle_sample_run(w, nl, bw_np, inp_np)
+        cpu = dict(value=round(L / (dt * w.backbone.n_layers / nl), 3), unit="tokens/s",
+                   cores=os.cpu_count(), kind="oracle", sample=desc, seconds=round(dt, 2))
+
+    out = dict(
+        metric=METRIC, value=round(value, 1), unit="tokens/s", n_gpus=world, steps=args.steps,
+        warmup=args.warmup, ms_per_step=round(t_ms / args.steps, 3), higher_is_better=True,
+        scaling="weak", vs_baseline=None, dtype="bf16", data="synthetic",
+        config=dict(workload=workload_desc(w), global_batch=tokens * world,
+                    seq_len=int(plan.max_seqlen), parallelism=f"replicas{world}",
+                    tenants=len(w.tenants), samples=plan.n_samples,
+                    l2="inputs larger than L2 (weights 13 GB, activations > 1 GB per step)"),
+        clocks=clk,
+        e2e=dict(value=round(tokens * world * args.steps / (e2e_ms / 1e3), 1), unit="tokens/s",
+                 h2d_bytes_per_step=int(h2d + e2e_plan_bytes), d2h_bytes_per_step=int(d2h)),
+        gpu_launches=int(launches),
+        roofline=roofline,
+        step_tensor=dict(achieved=round(step_tf, 1), unit="TFLOP/s",
+                         frac_of_burst=round(step_tf / peaks["bf16"], 4),
+                         frac_of_sustained=round(step_tf / peaks["bf16_sustained"], 4),
+                         note="all tensor-core algorithmic FLOPs of one step / step time"),
+        per_tenant=speed,
+        plan_ms=round(plan_ms, 3),
+        kernels=per_kernel,
+        cpu_baseline=cpu,
+    )
+    return out
+
+
+def run_reference(args, rank, world):
+    """The fp64 CPU oracle, as it stands, timed on the host cores."""
+    import synth
+    w = synth.make_workload(args.workload)
+    nl = min(args.reference_layers, w.backbone.n_layers)
+    import torch
+    bw = synth.make_backbone_weights(dataclass_layers(w, nl), device="cpu")
+    inp = synth.make_inputs(w, device="cpu")
+    bw_np, inp_np = host_numpy_inputs(w, bw, inp, nl)
+    for _ in range(args.warmup):
+        oracle_sample_run(w, nl, bw_np, inp_np)
+    tot, toks = 0.0, 0
+    desc = ""
+    for _ in range(args.steps):
+        dt, L, desc = oracle_sample_run(w, nl, bw_np, inp_np)
+        tot += dt
+        toks += L
+    scaled_s = tot * w.backbone.n_layers / nl
+    v = toks / scaled_s
+    return dict(metric=METRIC, value=round(v, 3), unit="tokens/s", n_gpus=world,
+                steps=args.steps, warmup=args.warmup,
+                ms_per_step=round(scaled_s / args.steps * 1e3, 1), higher_is_better=True,
+                scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
+                config=dict(workload=workload_desc(w), parallelism="cpu"),
+                impl="reference",
+                cpu_baseline=dict(value=round(v, 3), unit="tokens/s", cores=os.cpu_count(),
+                                  kind="oracle", sample=desc),
+                e2e=dict(value=round(v, 3), unit="tokens/s", h2d_bytes_per_step=0,
+                         d2h_bytes_per_step=0))
+
+
+def dataclass_layers(w, n_layers):
+    """The workload with only its first n_layers blocks (weights of the other
+    blocks are not needed by a bounded oracle sample)."""
+    import dataclasses
+    return dataclasses.replace(w, backbone=dataclasses.replace(w.backbone, n_layers=n_layers))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama7b")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-per-tenant", action="store_true")
+    ap.add_argument("--oracle-layers", type=int, default=2)
+    ap.add_argument("--reference-layers", type=int, default=1)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        print(json.dumps(run_reference(args, rank, world)), flush=True)
+        return
+
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    out = run_ours(args, rank, world, local_rank)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

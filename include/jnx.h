@@ -1,0 +1,334 @@
+/*
+ * jnx — grouped multi-tenant backbone forward with tenant-private action heads.
+ *
+ * C ABI of the GB300 (sm_103a) library libjnx.so.  The calls follow the
+ * paper's statement of group batching:
+ *
+ *   jnx_group_plan        collect the largest FIFO-compatible prefix of
+ *                         requests and canonicalise it into one packed varlen
+ *                         batch with its slices (App. A, "Inference Queue
+ *                         Composition"; §3.3, "Multi-Tenant Group Batching").
+ *   jnx_backbone_forward  one shared frozen backbone forward over the packed
+ *                         batch (the `encode` of App. A; §4.2 group execution).
+ *   jnx_heads_forward     split the features by the recorded slices and run
+ *                         each tenant's own action head and L2 loss on that
+ *                         tenant's samples only (App. A `split`/`decode`;
+ *                         §4.2 tenant-private loss).
+ *   jnx_heads_backward    gradients of each tenant's loss into that tenant's
+ *                         slot only; nothing is summed across tenants
+ *                         (App. A, "Actor Consumption and Version
+ *                         Consistency"; §4.2 tenant-private backward).
+ *
+ * Conventions for every call:
+ *   - All pointers are borrowed.  The library allocates no device memory and
+ *     frees nothing; scratch space is the caller's `workspace`.
+ *   - Device calls are asynchronous on `stream` (a cudaStream_t passed as
+ *     void*; NULL = the legacy default stream).
+ *   - Arguments the host can check are checked before any launch; on error
+ *     nothing is written and a message is available from jnx_last_error().
+ *   - Errors a kernel detects (an index outside its buffer) set a status word
+ *     at the start of the workspace instead of faulting; the offending access
+ *     is skipped.  jnx_check_status() reads and clears it.
+ *   - bf16 arrays are passed as uint16_t bit patterns; all matrices are
+ *     row-major, projections stored [out, in].
+ */
+#ifndef JNX_H
+#define JNX_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t jnx_status;
+
+#define JNX_OK 0
+#define JNX_ERR_INVALID_ARG (-1)
+#define JNX_ERR_CAPACITY (-3)
+#define JNX_ERR_OVERFLOW (-5)
+#define JNX_ERR_CUDA (-6)
+#define JNX_ERR_DEVICE_BOUNDS (-7)
+#define JNX_ERR_TIMEOUT (-8)
+#define JNX_ERR_UNSUPPORTED (-9)
+#define JNX_ERR_WORKSPACE (-10)
+
+/* Message describing the last error returned on this thread ("" if none). */
+const char* jnx_last_error(void);
+
+/* Library ABI version (increments on any struct or signature change). */
+int32_t jnx_version(void);
+
+/* ------------------------------------------------------------------------
+ * Plan (host only; callable without a GPU)
+ * ------------------------------------------------------------------------ */
+
+/* A tenant schema.  The first six fields are the shared-prefix signature:
+ * two requests are compatible iff these are equal ("compatibility is
+ * determined at the shared frozen-prefix boundary rather than by tenant
+ * identity", App. A).  max_images and action_width describe the tenant's
+ * own input limit and output structure and do not affect compatibility. */
+typedef struct {
+    int32_t backbone_id;
+    int32_t d_model;
+    int32_t vision_tokens;  /* rows per image */
+    int32_t embed_dtype;    /* 0 = bf16 */
+    int32_t vocab_id;
+    int32_t rope_id;
+    int32_t max_images;     /* per sample */
+    int32_t action_width;   /* C * D_t floats per sample (targets, predictions) */
+} jnx_schema;
+
+/* One sample (observation) of a request.  Its vision rows are
+ * vision[vision_row .. vision_row + n_img*vision_tokens), its text ids
+ * text_ids[text_pos .. text_pos + text_len), its targets / predictions
+ * targets[target_off .. target_off + action_width). */
+typedef struct {
+    int32_t n_img;
+    int32_t text_len;
+    int64_t vision_row;
+    int64_t text_pos;
+    int64_t target_off;
+} jnx_sample;
+
+/* One inference request in arrival order (App. A `InferenceRequest`). */
+typedef struct {
+    int32_t tenant;      /* tenant slot, 0 <= tenant < n_tenants */
+    int32_t schema;      /* index into the schema array */
+    int32_t n_samples;   /* >= 1 */
+    int32_t reserved;
+    const jnx_sample* samples;  /* [n_samples] */
+} jnx_request;
+
+typedef struct {
+    int32_t max_samples;  /* batch limit in samples */
+    int32_t max_tokens;   /* batch limit in packed tokens */
+} jnx_limits;
+
+/* Plan output: caller-owned host arrays with their capacities.
+ *   cu_seqlens[S+1]   token offset of each packed sample
+ *   sample_slot[S]    group slot (0..n_slots-1) of each packed sample
+ *   sample_req[S]     index of the accepted request it came from
+ *   sample_target[S]  its target/prediction offset (from jnx_sample)
+ *   sample_width[S]   its action width (from its schema)
+ *   seg_offsets[G+1]  packed-sample offsets of each group slot
+ *   slot_tenant[G]    tenant of each group slot
+ *   gather_src[N]     per packed token: vision row (>= 0) or
+ *                     -(text position + 1) (< 0)
+ *   pos_ids[N]        per packed token: position inside its sample
+ * Packed order: tenants by first appearance, their requests in arrival
+ * order, each request's samples in order; in a sample the vision rows of
+ * its images first, then its text tokens.  Positions restart at 0. */
+typedef struct {
+    int32_t cap_samples, cap_tokens, cap_slots;  /* in */
+    int32_t n_requests;                          /* out: accepted prefix length */
+    int32_t n_samples, n_tokens, n_slots, max_seqlen;  /* out */
+    int32_t* cu_seqlens;
+    int32_t* sample_slot;
+    int32_t* sample_req;
+    int32_t* sample_target;
+    int32_t* sample_width;
+    int32_t* seg_offsets;
+    int32_t* slot_tenant;
+    int32_t* gather_src;
+    int32_t* pos_ids;
+} jnx_plan;
+
+/* Collect the largest FIFO-compatible prefix of `reqs` and canonicalise it.
+ * Scanning stops at the first request whose prefix signature differs from
+ * the first request's, or that would push the batch over `lim` (whole
+ * requests; the first request is always accepted so the queue drains).
+ * Errors: JNX_ERR_INVALID_ARG (bad tenant/schema index, n_samples < 1, a
+ * sample with n_img outside [0, max_images], text_len < 0 or no token),
+ * JNX_ERR_OVERFLOW (a row, position or offset outside int32),
+ * JNX_ERR_CAPACITY (arrays too small: the required n_samples, n_tokens and
+ * n_slots are written back, nothing else).  n_reqs == 0 gives an empty plan. */
+jnx_status jnx_group_plan(const jnx_schema* schemas, int32_t n_schemas,
+                          const jnx_request* reqs, int32_t n_reqs, int32_t n_tenants,
+                          const jnx_limits* lim, jnx_plan* out);
+
+/* ------------------------------------------------------------------------
+ * Device-side view of a plan
+ * ------------------------------------------------------------------------ */
+
+/* The plan arrays copied to the device (the caller copies them), plus the
+ * host copies the launcher reads to shape its launches. */
+typedef struct {
+    int32_t n_samples, n_tokens, n_slots, max_seqlen;
+    const int32_t* cu_seqlens;     /* device [n_samples + 1] */
+    const int32_t* sample_slot;    /* device [n_samples] */
+    const int32_t* sample_target;  /* device [n_samples] */
+    const int32_t* seg_offsets;    /* device [n_slots + 1] */
+    const int32_t* gather_src;     /* device [n_tokens] */
+    const int32_t* pos_ids;        /* device [n_tokens] */
+    const int32_t* h_cu_seqlens;   /* host   [n_samples + 1] */
+    const int32_t* h_seg_offsets;  /* host   [n_slots + 1] */
+    const int32_t* h_slot_tenant;  /* host   [n_slots] */
+} jnx_group;
+
+/* ------------------------------------------------------------------------
+ * Shared frozen backbone
+ * ------------------------------------------------------------------------ */
+
+#define JNX_GLU_SWIGLU 0     /* act = SiLU */
+#define JNX_GLU_GEGLU_TANH 1 /* act = tanh-approximated GELU */
+
+/* One pre-norm decoder block (device pointers, bf16):
+ *   n1 = RMSNorm(x) * attn_norm;  [q|k|v] = n1 W_qkv^T; RoPE on q, k;
+ *   x += W_o Attn(q, k, v);  n2 = RMSNorm(x) * ffn_norm;
+ *   x += W_down (act(n2 W_g^T) * (n2 W_u^T)).
+ * w_qkv  [(H + 2 Hkv) hd, d]: rows of W_q, then W_k, then W_v.
+ * w_gu   [2 F, d]: 128-row blocks alternating gate and up rows, i.e. block
+ *        2j holds gate rows 128j..128j+127 and block 2j+1 the matching up
+ *        rows (jnx_pack_gate_up builds it from W_g and W_u).
+ * LoRA (lora_rank r > 0): for each of q, k, v, o, per-tenant adapters
+ *   lora_a_* [n_tenants, r, in] and lora_b_* [n_tenants, out, r];
+ *   y += (x A_t^T) B_t^T for the rows of tenant t.  NULL when r == 0. */
+typedef struct {
+    const uint16_t* attn_norm;  /* [d] */
+    const uint16_t* w_qkv;
+    const uint16_t* w_o;        /* [d, H hd] */
+    const uint16_t* ffn_norm;   /* [d] */
+    const uint16_t* w_gu;
+    const uint16_t* w_down;     /* [d, F] */
+    const uint16_t* lora_a_q; const uint16_t* lora_b_q;
+    const uint16_t* lora_a_k; const uint16_t* lora_b_k;
+    const uint16_t* lora_a_v; const uint16_t* lora_b_v;
+    const uint16_t* lora_a_o; const uint16_t* lora_b_o;
+} jnx_layer;
+
+typedef struct {
+    int32_t n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ff;
+    int32_t glu;           /* JNX_GLU_* */
+    int32_t lora_rank;     /* 0 = no adapters */
+    int32_t n_tenants;     /* rows of the LoRA adapter arrays */
+    int32_t vocab;
+    int32_t vision_tokens;
+    float eps;             /* RMSNorm epsilon */
+    float rope_theta;
+    const uint16_t* text_table;  /* device [vocab, d] */
+    const uint16_t* final_norm;  /* device [d] */
+    const jnx_layer* layers;     /* HOST array [n_layers] of device pointers */
+} jnx_backbone;
+
+/* Workspace bytes jnx_backbone_forward needs for a batch of n_tokens. */
+size_t jnx_backbone_workspace_bytes(const jnx_backbone* bb, int32_t n_tokens);
+
+/* Pack the batch (vision rows / text-embedding rows by gather_src), run all
+ * blocks over it with attention confined to each sample, apply the final
+ * RMSNorm and write the features:
+ *   pooled [n_samples, d] fp32: the mean of each sample's final normed rows
+ *          (features for MLP heads), or NULL;
+ *   hidden [n_tokens, d] bf16: the final normed rows (features for query
+ *          heads), or NULL.
+ * vision [n_vision_rows, d] bf16 and text_ids [n_text] int32 are the
+ * caller's observation buffers that gather_src indexes.  A gather index
+ * outside them, or a text id outside [0, vocab), sets
+ * JNX_ERR_DEVICE_BOUNDS in the status word and the row is zero-filled. */
+jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_group* g,
+                                const uint16_t* vision, int64_t n_vision_rows,
+                                const int32_t* text_ids, int64_t n_text,
+                                float* pooled, uint16_t* hidden,
+                                void* workspace, size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Tenant-private action heads (one slot per tenant)
+ * ------------------------------------------------------------------------ */
+
+#define JNX_HEAD_MLP 0    /* y = SiLU(p W1^T + b1) W2^T + b2 on the pooled feature p */
+#define JNX_HEAD_XATTN 1  /* y = flatten(softmax(Q k^T/sqrt(dq)) v) Wout^T + bout,
+                             k = X Wk^T, v = X Wv^T over the sample's hidden rows X */
+
+typedef struct {
+    int32_t kind;       /* JNX_HEAD_* */
+    int32_t d_in;       /* backbone width d */
+    int32_t d_hidden;   /* MLP hidden width */
+    int32_t n_queries;  /* query head: learned queries */
+    int32_t q_dim;      /* query head: attention width */
+    int32_t width;      /* outputs per sample, C * D_t */
+    /* MLP (device, bf16): w1 [d_hidden, d_in], b1 [d_hidden], w2 [width, d_hidden], b2 [width] */
+    const uint16_t *w1, *b1, *w2, *b2;
+    /* query head (device, bf16): q [n_queries, q_dim], wk/wv [q_dim, d_in],
+       wout [width, n_queries*q_dim], bout [width] */
+    const uint16_t *q, *wk, *wv, *wout, *bout;
+} jnx_head;
+
+/* Per-slot fp32 gradient buffers, same shapes as the parameters. */
+typedef struct {
+    float *w1, *b1, *w2, *b2;
+    float *q, *wk, *wv, *wout, *bout;
+} jnx_head_grads;
+
+/* Workspace bytes jnx_heads_forward / jnx_heads_backward need. */
+size_t jnx_heads_workspace_bytes(const jnx_head* heads, int32_t n_tenants, const jnx_group* g);
+
+/* Each group slot's head on that tenant's samples only.  heads[] is a HOST
+ * array indexed by tenant.  Writes preds at each sample's target offset
+ * (arrival layout, fp32) and loss[tenant] = mean squared error over the
+ * tenant's samples and outputs, for the tenants in the group only.  The
+ * activations the backward needs are kept in `workspace`. */
+jnx_status jnx_heads_forward(const jnx_head* heads, int32_t n_tenants, const jnx_group* g,
+                             const float* pooled, const uint16_t* hidden,
+                             const float* targets, float* preds, float* loss,
+                             void* workspace, size_t ws_bytes, void* stream);
+
+/* Gradients of each group tenant's loss w.r.t. that tenant's head
+ * parameters, written (overwritten, fp32) into grads[tenant] only; slots of
+ * tenants outside the group are not touched.  Must follow jnx_heads_forward
+ * on the same stream with the same group, features, targets and workspace:
+ * it reads the activations that call stored there.  No feature gradient is
+ * produced (the backbone is frozen). */
+jnx_status jnx_heads_backward(const jnx_head* heads, int32_t n_tenants, const jnx_group* g,
+                              const float* pooled, const uint16_t* hidden,
+                              const float* targets, const jnx_head_grads* grads,
+                              void* workspace, size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Status and helpers
+ * ------------------------------------------------------------------------ */
+
+/* Synchronise `stream`, read and clear the device status word at the start
+ * of `workspace`; returns JNX_OK or the first error a kernel recorded. */
+jnx_status jnx_check_status(void* workspace, void* stream);
+
+/* Build the interleaved w_gu layout from W_g [F, d] and W_u [F, d]
+ * (F a multiple of 128).  out [2F, d]. */
+jnx_status jnx_pack_gate_up(const uint16_t* w_gate, const uint16_t* w_up, int32_t F, int32_t d,
+                            uint16_t* out, void* stream);
+
+
+/* ------------------------------------------------------------------------
+ * Kernel tracing (host thread local)
+ * ------------------------------------------------------------------------ */
+
+/* Kernel ids reported by the tracer. */
+#define JNX_K_PACK 1       /* work = HBM bytes */
+#define JNX_K_RMSNORM 2    /* work = HBM bytes */
+#define JNX_K_GEMM_QKV 3   /* work = FLOPs */
+#define JNX_K_ATTN 4       /* work = FLOPs (within-sample only) */
+#define JNX_K_GEMM_O 5     /* work = FLOPs */
+#define JNX_K_GEMM_GU 6    /* work = FLOPs */
+#define JNX_K_GEMM_DOWN 7  /* work = FLOPs */
+#define JNX_K_POOL 8       /* work = HBM bytes */
+#define JNX_K_ROPE_TABLE 9 /* work = bytes written */
+#define JNX_K_HEADS_FWD 10 /* work = FLOPs */
+#define JNX_K_HEADS_BWD 11 /* work = FLOPs */
+#define JNX_K_GEMM 12      /* jnx_op_gemm; work = FLOPs */
+
+/* While enabled on the calling thread, each kernel launch of the library is
+ * bracketed by two CUDA events on its stream (up to `capacity` launches are
+ * kept; later ones are only counted).  Enabling resets the record. */
+jnx_status jnx_trace_enable(int32_t capacity);
+jnx_status jnx_trace_disable(void);
+/* Launches seen since the last enable (including those past capacity). */
+int32_t jnx_trace_count(void);
+/* Waits for the recorded events and returns, per recorded launch, its kernel
+ * id, its duration in ms and its algorithmic work; *n_out = entries written. */
+jnx_status jnx_trace_read(int32_t* kinds, float* ms, double* work, int32_t cap, int32_t* n_out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* JNX_H */

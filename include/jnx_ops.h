@@ -1,0 +1,71 @@
+/*
+ * Stage-level entry points of libjnx.so: each step of jnx_backbone_forward
+ * on its own, for stage-wise parity tests and per-kernel measurement.  The
+ * conventions of jnx.h apply (borrowed pointers, asynchronous on `stream`,
+ * host-checked arguments, bf16 as uint16_t bit patterns, row-major).
+ */
+#ifndef JNX_OPS_H
+#define JNX_OPS_H
+
+#include "jnx.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Epilogues of jnx_op_gemm. */
+#define JNX_EPI_BF16 0  /* out bf16 [M, ldo] = C */
+#define JNX_EPI_F32 1   /* out fp32 [M, ldo] = C */
+#define JNX_EPI_RESID 2 /* out fp32 [M, ldo] += C (residual stream update) */
+#define JNX_EPI_GLU 3   /* W holds 128-row blocks alternating gate / up rows;
+                           out bf16 [M, ldo] columns j < N/2 = act(C_gate) * C_up */
+#define JNX_EPI_ROPE 4  /* out bf16 [M, ldo] = C with rotate-half RoPE at
+                           position pos[row] on columns < rope_cols */
+
+/* The canonical packing step (§3.3: the VLAFeature is where the tenants'
+ * samples are concatenated): x[t, :] = fp32 of vision[gather_src[t]] or of
+ * text_table[text_ids[-gather_src[t] - 1]].  x is [n_tokens, d] fp32.  A
+ * source index outside its buffer or a text id outside [0, vocab) writes a
+ * zero row and JNX_ERR_DEVICE_BOUNDS to *status (device int, may be NULL). */
+jnx_status jnx_op_pack(const jnx_group* g, const uint16_t* vision, int64_t n_vision_rows,
+                       const int32_t* text_ids, int64_t n_text, const uint16_t* text_table,
+                       int32_t vocab, int32_t d, float* x, int32_t* status, void* stream);
+
+/* out[M, d] bf16 = x / sqrt(mean(x^2) + eps) * gamma, fp32 statistics;
+ * d in {256, 512, 1024, 2048, 4096}. */
+jnx_status jnx_op_rmsnorm(const float* x, const uint16_t* gamma, float eps, int32_t M, int32_t d,
+                          uint16_t* out, void* stream);
+
+/* Workspace bytes of jnx_op_gemm with JNX_EPI_ROPE for positions < max_pos. */
+size_t jnx_op_gemm_workspace_bytes(int32_t max_pos, int32_t head_dim);
+
+/* C[M, N] = A[M, K] W[N, K]^T on the tcgen05 tensor cores, fp32 accumulate,
+ * then the epilogue.  N % 256 == 0, K % 64 == 0, A/W rows 16-byte aligned.
+ * pos/max_pos/rope_cols/head_dim/rope_theta are read for JNX_EPI_ROPE only
+ * (workspace then holds the status word and the RoPE table); act
+ * (JNX_GLU_*) for JNX_EPI_GLU only.  workspace may be NULL otherwise. */
+jnx_status jnx_op_gemm(const uint16_t* A, const uint16_t* W, int32_t M, int32_t N, int32_t K,
+                       int32_t epilogue, void* out, int32_t ldo, const int32_t* pos,
+                       int32_t max_pos, int32_t rope_cols, int32_t head_dim, float rope_theta,
+                       int32_t act, void* workspace, size_t ws_bytes, void* stream);
+
+/* Attention confined to each sample: for every sample s, head h,
+ * out[t] = softmax(q_t K_s^T / sqrt(hd)) V_s over the sample's own tokens.
+ * qkv [n_tokens, (H + 2 Hkv) hd] bf16 (q heads, then k heads, then v heads),
+ * out [n_tokens, H hd] bf16; head_dim in {64, 128, 256}. */
+jnx_status jnx_op_attention(const uint16_t* qkv, int32_t n_heads, int32_t n_kv_heads,
+                            int32_t head_dim, const int32_t* cu_seqlens, int32_t n_samples,
+                            int32_t max_seqlen, uint16_t* out, void* stream);
+
+/* Final RMSNorm and per-sample mean: pooled[s] = gamma * mean over the
+ * sample's rows of x_t / sqrt(mean(x_t^2) + eps) (fp32), hidden[t] = bf16
+ * of the normed row.  Either output may be NULL. */
+jnx_status jnx_op_final_pool(const float* x, const uint16_t* gamma, float eps,
+                             const int32_t* cu_seqlens, int32_t n_samples, int32_t d,
+                             float* pooled, uint16_t* hidden, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* JNX_OPS_H */

@@ -1,0 +1,524 @@
+// C-ABI entry points: the shared backbone forward, the tenant heads, status
+// and helpers, plus the stage-level entry points of jnx_ops.h.
+#include <algorithm>
+#include <vector>
+
+#include "../../include/jnx_ops.h"
+#include "jnx_dev.cuh"
+#include "jnx_heads.h"
+#include "jnx_kernels.h"
+#include "jnx_trace.h"
+
+using namespace jnx;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+constexpr size_t kStatusBytes = 256;
+
+size_t up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
+
+// Workspace carve-up of jnx_backbone_forward.
+struct BackboneWs {
+    int* status;
+    float* x;         // residual stream [N, d] fp32
+    uint16_t* nrm;    // normed activations [N, d] bf16
+    uint16_t* qkv;    // [N, (H + 2 Hkv) hd] bf16
+    uint16_t* att;    // [N, H hd] bf16
+    uint16_t* u;      // [N, F] bf16
+    float2* rope;     // [max_pos, hd / 2]
+    size_t bytes;
+};
+
+constexpr int kMaxRopePos = 1 << 16;  // longest sample the workspace reserves RoPE rows for
+
+BackboneWs carve_backbone(const jnx_backbone* bb, int64_t N, void* base) {
+    uint8_t* p = static_cast<uint8_t*>(base);
+    BackboneWs w{};
+    const int64_t d = bb->d_model, qkvw = (int64_t)(bb->n_heads + 2 * bb->n_kv_heads) * bb->head_dim;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        uint8_t* r = p ? p + off : nullptr;
+        off += up(bytes);
+        return r;
+    };
+    w.status = reinterpret_cast<int*>(take(kStatusBytes));
+    w.x = reinterpret_cast<float*>(take((size_t)N * d * 4));
+    w.nrm = reinterpret_cast<uint16_t*>(take((size_t)N * d * 2));
+    w.qkv = reinterpret_cast<uint16_t*>(take((size_t)N * qkvw * 2));
+    w.att = reinterpret_cast<uint16_t*>(take((size_t)N * bb->n_heads * bb->head_dim * 2));
+    w.u = reinterpret_cast<uint16_t*>(take((size_t)N * bb->d_ff * 2));
+    w.rope = reinterpret_cast<float2*>(take((size_t)kMaxRopePos * (bb->head_dim / 2) * 8));
+    w.bytes = off;
+    return w;
+}
+
+jnx_status check_backbone(const jnx_backbone* bb) {
+    if (!bb || !bb->layers || !bb->text_table || !bb->final_norm)
+        return fail(JNX_ERR_INVALID_ARG, "backbone: null descriptor field");
+    if (bb->n_layers < 0 || bb->n_heads <= 0 || bb->n_kv_heads <= 0 ||
+        bb->n_heads % bb->n_kv_heads)
+        return fail(JNX_ERR_INVALID_ARG, "backbone: bad head counts");
+    if (bb->head_dim != 64 && bb->head_dim != 128 && bb->head_dim != 256)
+        return fail(JNX_ERR_UNSUPPORTED, "backbone: head_dim %d not in {64,128,256}", bb->head_dim);
+    const int d = bb->d_model;
+    if (d != 256 && d != 512 && d != 1024 && d != 2048 && d != 4096)
+        return fail(JNX_ERR_UNSUPPORTED, "backbone: d_model %d not in {256..4096}", d);
+    const int qkvw = (bb->n_heads + 2 * bb->n_kv_heads) * bb->head_dim;
+    jnx_status st;
+    if ((st = gemm_check(1, qkvw, d)) || (st = gemm_check(1, d, bb->n_heads * bb->head_dim)) ||
+        (st = gemm_check(1, 2 * bb->d_ff, d)) || (st = gemm_check(1, d, bb->d_ff)))
+        return st;
+    if (bb->glu != JNX_GLU_SWIGLU && bb->glu != JNX_GLU_GEGLU_TANH)
+        return fail(JNX_ERR_INVALID_ARG, "backbone: unknown glu %d", bb->glu);
+    if (bb->lora_rank != 0) return fail(JNX_ERR_UNSUPPORTED, "backbone: LoRA not built yet");
+    for (int l = 0; l < bb->n_layers; ++l) {
+        const jnx_layer& L = bb->layers[l];
+        if (!L.attn_norm || !L.w_qkv || !L.w_o || !L.ffn_norm || !L.w_gu || !L.w_down)
+            return fail(JNX_ERR_INVALID_ARG, "backbone: layer %d has a null weight", l);
+    }
+    return JNX_OK;
+}
+
+jnx_status check_group(const jnx_group* g) {
+    if (!g) return fail(JNX_ERR_INVALID_ARG, "group: null");
+    if (g->n_samples < 0 || g->n_tokens < 0 || g->n_slots < 0 || g->max_seqlen < 0)
+        return fail(JNX_ERR_INVALID_ARG, "group: negative count");
+    if (g->n_samples > 0 && (!g->cu_seqlens || !g->sample_slot || !g->sample_target ||
+                             !g->h_cu_seqlens))
+        return fail(JNX_ERR_INVALID_ARG, "group: null sample array");
+    if (g->n_tokens > 0 && (!g->gather_src || !g->pos_ids))
+        return fail(JNX_ERR_INVALID_ARG, "group: null token array");
+    if (g->n_slots > 0 && (!g->seg_offsets || !g->h_seg_offsets || !g->h_slot_tenant))
+        return fail(JNX_ERR_INVALID_ARG, "group: null slot array");
+    if (g->max_seqlen > kMaxRopePos)
+        return fail(JNX_ERR_UNSUPPORTED, "group: sample longer than %d tokens", kMaxRopePos);
+    return JNX_OK;
+}
+
+jnx_status cuda_status(const char* what) {
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+}  // namespace
+
+extern "C" size_t jnx_backbone_workspace_bytes(const jnx_backbone* bb, int32_t n_tokens) {
+    if (!bb || n_tokens < 0) return 0;
+    return carve_backbone(bb, n_tokens, nullptr).bytes;
+}
+
+extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_group* g,
+                                           const uint16_t* vision, int64_t n_vision_rows,
+                                           const int32_t* text_ids, int64_t n_text, float* pooled,
+                                           uint16_t* hidden, void* workspace, size_t ws_bytes,
+                                           void* stream) {
+    clear_error();
+    jnx_status st;
+    if ((st = check_backbone(bb)) || (st = check_group(g))) return st;
+    if (!workspace) return fail(JNX_ERR_INVALID_ARG, "backbone: null workspace");
+    const int N = g->n_tokens, d = bb->d_model, H = bb->n_heads, Hkv = bb->n_kv_heads,
+              hd = bb->head_dim, F = bb->d_ff;
+    BackboneWs w = carve_backbone(bb, N, workspace);
+    if (ws_bytes < w.bytes)
+        return fail(JNX_ERR_WORKSPACE, "backbone: workspace %zu < %zu bytes", ws_bytes, w.bytes);
+    if (N == 0) return JNX_OK;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int qkvw = (H + 2 * Hkv) * hd;
+
+    const double Nd = (double)N * d;
+    {
+        TraceScope ts(JNX_K_PACK, Nd * 6.0, s);
+        if ((st = pack_launch(g, vision, n_vision_rows, text_ids, n_text, bb->text_table,
+                              bb->vocab, d, w.x, w.status, s)))
+            return st;
+    }
+    {
+        TraceScope ts(JNX_K_ROPE_TABLE, (double)g->max_seqlen * hd * 4.0, s);
+        if ((st = rope_table_launch(w.rope, g->max_seqlen, hd, bb->rope_theta, s))) return st;
+    }
+    // within-sample attention FLOPs: QK^T and PV over each sample's own tokens
+    double attn_flops = 0.0;
+    for (int i = 0; i < g->n_samples; ++i) {
+        const double L = g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i];
+        attn_flops += 4.0 * L * L * H * hd;
+    }
+
+    for (int l = 0; l < bb->n_layers; ++l) {
+        const jnx_layer& L = bb->layers[l];
+        // attention sub-block
+        {
+            TraceScope ts(JNX_K_RMSNORM, Nd * 6.0, s);
+            if ((st = rmsnorm_launch(w.x, L.attn_norm, bb->eps, N, d, w.nrm, s))) return st;
+        }
+        GemmParams p{};
+        p.M = N;
+        p.N = qkvw;
+        p.K = d;
+        p.epi = EPI_ROPE;
+        p.out = w.qkv;
+        p.ldo = qkvw;
+        p.pos = g->pos_ids;
+        p.rope = w.rope;
+        p.rope_cols = (H + Hkv) * hd;
+        p.hd = hd;
+        p.status = w.status;
+        {
+            TraceScope ts(JNX_K_GEMM_QKV, 2.0 * N * qkvw * d, s);
+            if ((st = gemm_launch(w.nrm, d, L.w_qkv, d, p, s))) return st;
+        }
+        {
+            TraceScope ts(JNX_K_ATTN, attn_flops, s);
+            if ((st = attention_launch(w.qkv, qkvw, H, Hkv, hd, g->cu_seqlens, g->n_samples,
+                                       g->max_seqlen, w.att, H * hd, s)))
+                return st;
+        }
+        p = GemmParams{};
+        p.M = N;
+        p.N = d;
+        p.K = H * hd;
+        p.epi = EPI_RESID;
+        p.resid = w.x;
+        p.ldr = d;
+        p.status = w.status;
+        {
+            TraceScope ts(JNX_K_GEMM_O, 2.0 * N * d * H * hd, s);
+            if ((st = gemm_launch(w.att, H * hd, L.w_o, H * hd, p, s))) return st;
+        }
+        // feed-forward sub-block
+        {
+            TraceScope ts(JNX_K_RMSNORM, Nd * 6.0, s);
+            if ((st = rmsnorm_launch(w.x, L.ffn_norm, bb->eps, N, d, w.nrm, s))) return st;
+        }
+        p = GemmParams{};
+        p.M = N;
+        p.N = 2 * F;
+        p.K = d;
+        p.epi = EPI_GLU;
+        p.out = w.u;
+        p.ldo = F;
+        p.act = bb->glu;
+        p.status = w.status;
+        {
+            TraceScope ts(JNX_K_GEMM_GU, 2.0 * N * 2.0 * F * d, s);
+            if ((st = gemm_launch(w.nrm, d, L.w_gu, d, p, s))) return st;
+        }
+        p = GemmParams{};
+        p.M = N;
+        p.N = d;
+        p.K = F;
+        p.epi = EPI_RESID;
+        p.resid = w.x;
+        p.ldr = d;
+        p.status = w.status;
+        {
+            TraceScope ts(JNX_K_GEMM_DOWN, 2.0 * N * d * F, s);
+            if ((st = gemm_launch(w.u, F, L.w_down, F, p, s))) return st;
+        }
+    }
+    TraceScope ts(JNX_K_POOL, Nd * 4.0 + (hidden ? Nd * 2.0 : 0.0) +
+                                  (pooled ? (double)g->n_samples * d * 4.0 : 0.0), s);
+    return final_pool_launch(w.x, bb->final_norm, bb->eps, g->cu_seqlens, g->n_samples, d, pooled,
+                             hidden, s);
+}
+
+// ---------------------------------------------------------------------------
+// heads
+// ---------------------------------------------------------------------------
+namespace {
+
+struct HeadsWs {
+    int* status;
+    HeadScratch sc;
+    size_t bytes;
+};
+
+int heads_ld(const jnx_head* heads, const jnx_group* g) {
+    int ld = 8;
+    for (int i = 0; i < g->n_slots; ++i) {
+        const jnx_head& h = heads[g->h_slot_tenant[i]];
+        ld = std::max(ld, std::max(h.d_hidden, h.width));
+    }
+    return (ld + 7) / 8 * 8;
+}
+
+HeadsWs carve_heads(const jnx_head* heads, const jnx_group* g, void* base) {
+    uint8_t* p = static_cast<uint8_t*>(base);
+    HeadsWs w{};
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        uint8_t* r = p ? p + off : nullptr;
+        off += up(bytes);
+        return r;
+    };
+    const int ld = heads_ld(heads, g);
+    const size_t arr = (size_t)std::max(g->n_samples, 1) * ld * 4;
+    w.status = reinterpret_cast<int*>(take(kStatusBytes));
+    w.sc.z = reinterpret_cast<float*>(take(arr));
+    w.sc.a = reinterpret_cast<float*>(take(arr));
+    w.sc.y = reinterpret_cast<float*>(take(arr));
+    w.sc.dy = reinterpret_cast<float*>(take(arr));
+    w.sc.dz = reinterpret_cast<float*>(take(arr));
+    w.sc.ld = ld;
+    w.bytes = off;
+    return w;
+}
+
+jnx_status check_heads(const jnx_head* heads, int32_t n_tenants, const jnx_group* g,
+                       bool need_grads, const jnx_head_grads* grads) {
+    jnx_status st;
+    if ((st = check_group(g))) return st;
+    if (!heads && g->n_slots > 0) return fail(JNX_ERR_INVALID_ARG, "heads: null head table");
+    for (int i = 0; i < g->n_slots; ++i) {
+        const int t = g->h_slot_tenant[i];
+        if (t < 0 || t >= n_tenants)
+            return fail(JNX_ERR_INVALID_ARG, "heads: group slot %d tenant %d out of range", i, t);
+        const jnx_head& h = heads[t];
+        if (h.kind != JNX_HEAD_MLP)
+            return fail(JNX_ERR_UNSUPPORTED, "heads: tenant %d head kind %d not built yet", t,
+                        h.kind);
+        if (h.d_in % 8 || h.d_hidden % 8 || h.d_hidden <= 0 || h.width <= 0 || h.d_in <= 0)
+            return fail(JNX_ERR_UNSUPPORTED, "heads: tenant %d widths must be multiples of 8", t);
+        if (!h.w1 || !h.b1 || !h.w2 || !h.b2)
+            return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null parameter", t);
+        if (need_grads) {
+            const jnx_head_grads& gr = grads[t];
+            if (!gr.w1 || !gr.b1 || !gr.w2 || !gr.b2)
+                return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null gradient buffer", t);
+        }
+        const int s0 = g->h_seg_offsets[i], s1 = g->h_seg_offsets[i + 1];
+        if (s0 < 0 || s1 <= s0 || s1 > g->n_samples)
+            return fail(JNX_ERR_INVALID_ARG, "heads: bad segment of group slot %d", i);
+    }
+    return JNX_OK;
+}
+
+// Fill the per-slot table for group slots [g0, g0 + n).
+void fill_table(HeadTable& tab, const jnx_head* heads, const jnx_head_grads* grads,
+                const jnx_group* g, int g0, int n, int& max_hidden, int& max_width, int& max_din) {
+    max_hidden = max_width = max_din = 0;
+    for (int i = 0; i < n; ++i) {
+        const int t = g->h_slot_tenant[g0 + i];
+        const jnx_head& h = heads[t];
+        HeadSlot& hs = tab.slot[i];
+        hs.w1 = h.w1;
+        hs.b1 = h.b1;
+        hs.w2 = h.w2;
+        hs.b2 = h.b2;
+        if (grads) {
+            hs.g_w1 = grads[t].w1;
+            hs.g_b1 = grads[t].b1;
+            hs.g_w2 = grads[t].w2;
+            hs.g_b2 = grads[t].b2;
+        }
+        hs.s0 = g->h_seg_offsets[g0 + i];
+        hs.s1 = g->h_seg_offsets[g0 + i + 1];
+        hs.d_in = h.d_in;
+        hs.d_hidden = h.d_hidden;
+        hs.width = h.width;
+        hs.tenant = t;
+        max_hidden = std::max(max_hidden, h.d_hidden);
+        max_width = std::max(max_width, h.width);
+        max_din = std::max(max_din, h.d_in);
+    }
+}
+
+}  // namespace
+
+extern "C" size_t jnx_heads_workspace_bytes(const jnx_head* heads, int32_t n_tenants,
+                                            const jnx_group* g) {
+    if (!g || (g->n_slots > 0 && (!heads || !g->h_slot_tenant))) return 0;
+    for (int i = 0; i < g->n_slots; ++i)
+        if (g->h_slot_tenant[i] < 0 || g->h_slot_tenant[i] >= n_tenants) return 0;
+    return carve_heads(heads, g, nullptr).bytes;
+}
+
+extern "C" jnx_status jnx_heads_forward(const jnx_head* heads, int32_t n_tenants,
+                                        const jnx_group* g, const float* pooled,
+                                        const uint16_t* hidden, const float* targets, float* preds,
+                                        float* loss, void* workspace, size_t ws_bytes,
+                                        void* stream) {
+    clear_error();
+    jnx_status st;
+    if ((st = check_heads(heads, n_tenants, g, false, nullptr))) return st;
+    if (g->n_slots == 0) return JNX_OK;
+    if (!pooled || !targets || !preds || !loss || !workspace)
+        return fail(JNX_ERR_INVALID_ARG, "heads forward: null buffer");
+    HeadsWs w = carve_heads(heads, g, workspace);
+    if (ws_bytes < w.bytes)
+        return fail(JNX_ERR_WORKSPACE, "heads: workspace %zu < %zu bytes", ws_bytes, w.bytes);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    HeadTable tab;
+    for (int g0 = 0; g0 < g->n_slots; g0 += kMaxSlots) {
+        const int n = std::min(kMaxSlots, g->n_slots - g0);
+        int mh, mw, md;
+        fill_table(tab, heads, nullptr, g, g0, n, mh, mw, md);
+        double fl = 0.0;
+        for (int i = 0; i < n; ++i)
+            fl += 2.0 * (tab.slot[i].s1 - tab.slot[i].s0) *
+                  ((double)tab.slot[i].d_in * tab.slot[i].d_hidden +
+                   (double)tab.slot[i].d_hidden * tab.slot[i].width);
+        TraceScope ts(JNX_K_HEADS_FWD, fl, s);
+        if ((st = mlp_heads_forward(tab, n, mh, mw, pooled, heads[g->h_slot_tenant[g0]].d_in,
+                                    g->sample_target, targets, preds, loss, w.sc, s)))
+            return st;
+    }
+    return JNX_OK;
+}
+
+extern "C" jnx_status jnx_heads_backward(const jnx_head* heads, int32_t n_tenants,
+                                         const jnx_group* g, const float* pooled,
+                                         const uint16_t* hidden, const float* targets,
+                                         const jnx_head_grads* grads, void* workspace,
+                                         size_t ws_bytes, void* stream) {
+    clear_error();
+    jnx_status st;
+    if (!grads && g && g->n_slots > 0) return fail(JNX_ERR_INVALID_ARG, "heads backward: null grads");
+    if ((st = check_heads(heads, n_tenants, g, true, grads))) return st;
+    if (g->n_slots == 0) return JNX_OK;
+    if (!pooled || !workspace) return fail(JNX_ERR_INVALID_ARG, "heads backward: null buffer");
+    HeadsWs w = carve_heads(heads, g, workspace);
+    if (ws_bytes < w.bytes)
+        return fail(JNX_ERR_WORKSPACE, "heads: workspace %zu < %zu bytes", ws_bytes, w.bytes);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    HeadTable tab;
+    for (int g0 = 0; g0 < g->n_slots; g0 += kMaxSlots) {
+        const int n = std::min(kMaxSlots, g->n_slots - g0);
+        int mh, mw, md;
+        fill_table(tab, heads, grads, g, g0, n, mh, mw, md);
+        double fl = 0.0;
+        for (int i = 0; i < n; ++i)
+            fl += 2.0 * (tab.slot[i].s1 - tab.slot[i].s0) *
+                  ((double)tab.slot[i].d_in * tab.slot[i].d_hidden +
+                   2.0 * tab.slot[i].d_hidden * tab.slot[i].width);
+        TraceScope ts(JNX_K_HEADS_BWD, fl, s);
+        if ((st = mlp_heads_backward(tab, n, mh, mw, md, pooled, heads[g->h_slot_tenant[g0]].d_in,
+                                     w.sc, s)))
+            return st;
+    }
+    return JNX_OK;
+}
+
+// ---------------------------------------------------------------------------
+// status and helpers
+// ---------------------------------------------------------------------------
+
+extern "C" jnx_status jnx_check_status(void* workspace, void* stream) {
+    clear_error();
+    if (!workspace) return fail(JNX_ERR_INVALID_ARG, "check_status: null workspace");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int v = 0;
+    if (cudaMemcpyAsync(&v, workspace, sizeof v, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaMemsetAsync(workspace, 0, sizeof v, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return fail(JNX_ERR_CUDA, "check_status: %s", cudaGetErrorString(cudaGetLastError()));
+    if (v != 0) return fail(v, "a kernel reported status %d", v);
+    return JNX_OK;
+}
+
+__global__ void k_pack_gate_up(const uint16_t* __restrict__ wg, const uint16_t* __restrict__ wu,
+                               int F, int d, uint16_t* __restrict__ out) {
+    const int64_t row = blockIdx.x;  // output row in [0, 2F)
+    const int blk = (int)(row / 128), r = (int)(row % 128);
+    const int src = (blk / 2) * 128 + r;
+    const uint16_t* in = (blk & 1) ? wu : wg;
+    const uint4* a = reinterpret_cast<const uint4*>(in + (size_t)src * d);
+    uint4* b = reinterpret_cast<uint4*>(out + (size_t)row * d);
+    for (int c = threadIdx.x; c < d / 8; c += blockDim.x) b[c] = a[c];
+}
+
+extern "C" jnx_status jnx_pack_gate_up(const uint16_t* w_gate, const uint16_t* w_up, int32_t F,
+                                       int32_t d, uint16_t* out, void* stream) {
+    clear_error();
+    if (!w_gate || !w_up || !out || F <= 0 || d <= 0 || F % 128 || d % 8)
+        return fail(JNX_ERR_INVALID_ARG, "pack_gate_up: need F %% 128 == 0 and d %% 8 == 0");
+    k_pack_gate_up<<<2 * F, 128, 0, static_cast<cudaStream_t>(stream)>>>(w_gate, w_up, F, d, out);
+    return cuda_status("pack_gate_up");
+}
+
+// ---------------------------------------------------------------------------
+// stage-level entry points (jnx_ops.h)
+// ---------------------------------------------------------------------------
+
+extern "C" jnx_status jnx_op_pack(const jnx_group* g, const uint16_t* vision,
+                                  int64_t n_vision_rows, const int32_t* text_ids, int64_t n_text,
+                                  const uint16_t* text_table, int32_t vocab, int32_t d, float* x,
+                                  int32_t* status, void* stream) {
+    clear_error();
+    jnx_status st;
+    if ((st = check_group(g))) return st;
+    return pack_launch(g, vision, n_vision_rows, text_ids, n_text, text_table, vocab, d, x, status,
+                       static_cast<cudaStream_t>(stream));
+}
+
+extern "C" jnx_status jnx_op_rmsnorm(const float* x, const uint16_t* gamma, float eps, int32_t M,
+                                     int32_t d, uint16_t* out, void* stream) {
+    clear_error();
+    if (M < 0 || !x || !gamma || !out) return fail(JNX_ERR_INVALID_ARG, "rmsnorm: bad argument");
+    return rmsnorm_launch(x, gamma, eps, M, d, out, static_cast<cudaStream_t>(stream));
+}
+
+extern "C" size_t jnx_op_gemm_workspace_bytes(int32_t max_pos, int32_t head_dim) {
+    return kStatusBytes + up((size_t)std::max(max_pos, 1) * std::max(head_dim / 2, 1) * 8);
+}
+
+extern "C" jnx_status jnx_op_gemm(const uint16_t* A, const uint16_t* W, int32_t M, int32_t N,
+                                  int32_t K, int32_t epilogue, void* out, int32_t ldo,
+                                  const int32_t* pos, int32_t max_pos, int32_t rope_cols,
+                                  int32_t head_dim, float rope_theta, int32_t act,
+                                  void* workspace, size_t ws_bytes, void* stream) {
+    clear_error();
+    if (!A || !W || !out || M < 0) return fail(JNX_ERR_INVALID_ARG, "gemm: null argument");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    GemmParams p{};
+    p.M = M;
+    p.N = N;
+    p.K = K;
+    p.epi = epilogue;
+    p.out = out;
+    p.ldo = ldo;
+    p.act = act;
+    if (epilogue == EPI_RESID) {
+        p.resid = static_cast<float*>(out);
+        p.ldr = ldo;
+    }
+    if (epilogue == EPI_ROPE) {
+        if (!pos || !workspace || (head_dim != 64 && head_dim != 128 && head_dim != 256) ||
+            max_pos <= 0)
+            return fail(JNX_ERR_INVALID_ARG, "gemm rope: need pos, workspace, head_dim");
+        if (ws_bytes < jnx_op_gemm_workspace_bytes(max_pos, head_dim))
+            return fail(JNX_ERR_WORKSPACE, "gemm rope: workspace too small");
+        float2* tab = reinterpret_cast<float2*>(static_cast<uint8_t*>(workspace) + kStatusBytes);
+        jnx_status st = rope_table_launch(tab, max_pos, head_dim, rope_theta, s);
+        if (st) return st;
+        p.pos = pos;
+        p.rope = tab;
+        p.rope_cols = rope_cols;
+        p.hd = head_dim;
+    }
+    if (workspace) p.status = static_cast<int*>(workspace);
+    TraceScope ts(JNX_K_GEMM, 2.0 * M * N * K, s);
+    return gemm_launch(A, K, W, K, p, s);
+}
+
+extern "C" jnx_status jnx_op_attention(const uint16_t* qkv, int32_t n_heads, int32_t n_kv_heads,
+                                       int32_t head_dim, const int32_t* cu_seqlens,
+                                       int32_t n_samples, int32_t max_seqlen, uint16_t* out,
+                                       void* stream) {
+    clear_error();
+    if (!qkv || !out || (n_samples > 0 && !cu_seqlens))
+        return fail(JNX_ERR_INVALID_ARG, "attention: null argument");
+    const int ldq = (n_heads + 2 * n_kv_heads) * head_dim;
+    return attention_launch(qkv, ldq, n_heads, n_kv_heads, head_dim, cu_seqlens, n_samples,
+                            max_seqlen, out, n_heads * head_dim, static_cast<cudaStream_t>(stream));
+}
+
+extern "C" jnx_status jnx_op_final_pool(const float* x, const uint16_t* gamma, float eps,
+                                        const int32_t* cu_seqlens, int32_t n_samples, int32_t d,
+                                        float* pooled, uint16_t* hidden, void* stream) {
+    clear_error();
+    if (!x || !gamma || (n_samples > 0 && !cu_seqlens))
+        return fail(JNX_ERR_INVALID_ARG, "final_pool: null argument");
+    return final_pool_launch(x, gamma, eps, cu_seqlens, n_samples, d, pooled, hidden,
+                             static_cast<cudaStream_t>(stream));
+}

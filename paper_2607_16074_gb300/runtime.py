@@ -1,0 +1,172 @@
+"""Device-side plumbing around the C ABI: PyTorch holds the device memory and
+the stream; these classes only fill the C structs with its addresses and
+call the library.  No arithmetic of the method happens here.
+"""
+from __future__ import annotations
+
+import ctypes as C
+from typing import Dict, List, Optional, Sequence
+
+import numpy as np
+import torch
+
+from . import jnx as J
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream: Optional[torch.cuda.Stream]) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+class DeviceGroup:
+    """A plan's arrays copied to the device, wrapped in a jnx_group."""
+
+    DEV = ("cu_seqlens", "sample_slot", "sample_target", "seg_offsets", "gather_src", "pos_ids")
+
+    def __init__(self, plan: J.Plan, device="cuda", non_blocking: bool = False):
+        self.plan = plan
+        self.h = {k: np.ascontiguousarray(getattr(plan, k), dtype=np.int32)
+                  for k in ("cu_seqlens", "seg_offsets", "slot_tenant")}
+        self.d = {}
+        for k in self.DEV:
+            a = torch.from_numpy(np.ascontiguousarray(getattr(plan, k), dtype=np.int32))
+            if non_blocking:
+                a = a.pin_memory()
+            self.d[k] = a.to(device, non_blocking=non_blocking)
+        hp = lambda k: self.h[k].ctypes.data_as(J.P32)
+        self.struct = J.jnx_group(
+            plan.n_samples, plan.n_tokens, plan.n_slots, plan.max_seqlen,
+            *[self.d[k].data_ptr() or None for k in self.DEV],
+            hp("cu_seqlens"), hp("seg_offsets"), hp("slot_tenant"))
+
+    @property
+    def ref(self):
+        return C.byref(self.struct)
+
+
+class DeviceBackbone:
+    """Frozen backbone weights on the device in the library's layout: the
+    fused [W_q; W_k; W_v] rows and the 128-row interleaved gate/up matrix
+    (built by jnx_pack_gate_up)."""
+
+    def __init__(self, cfg, weights: Dict, n_tenants: int = 1, stream=None):
+        self.cfg = cfg
+        L = J.lib()
+        self.keep: List[torch.Tensor] = []
+        self.layers = (J.jnx_layer * max(1, cfg.n_layers))()
+        s = _stream(stream)
+        for i, lw in enumerate(weights["layers"]):
+            w_qkv = torch.cat([lw["wq"], lw["wk"], lw["wv"]], dim=0).contiguous()
+            w_gu = torch.empty((2 * cfg.d_ff, cfg.d), dtype=torch.bfloat16, device=w_qkv.device)
+            J.check(L.jnx_pack_gate_up(lw["wg"].data_ptr(), lw["wu"].data_ptr(), cfg.d_ff, cfg.d,
+                                       w_gu.data_ptr(), s))
+            ent = dict(attn_norm=lw["attn_norm"], w_qkv=w_qkv, w_o=lw["wo"],
+                       ffn_norm=lw["ffn_norm"], w_gu=w_gu, w_down=lw["wd"])
+            self.keep += list(ent.values())
+            self.layers[i] = J.jnx_layer(*[ent[k].data_ptr() for k in
+                                           ("attn_norm", "w_qkv", "w_o", "ffn_norm", "w_gu",
+                                            "w_down")])
+        self.text_table = weights["text_table"]
+        self.final_norm = weights["final_norm"]
+        self.struct = J.jnx_backbone(cfg.n_layers, cfg.d, cfg.n_heads, cfg.n_kv_heads,
+                                     cfg.head_dim, cfg.d_ff, cfg.glu, cfg.lora_rank, n_tenants,
+                                     cfg.vocab, cfg.vision_tokens, cfg.eps, cfg.rope_theta,
+                                     self.text_table.data_ptr(), self.final_norm.data_ptr(),
+                                     C.cast(self.layers, C.POINTER(J.jnx_layer)))
+
+    def workspace_bytes(self, n_tokens: int) -> int:
+        return J.lib().jnx_backbone_workspace_bytes(C.byref(self.struct), n_tokens)
+
+    def forward(self, group: DeviceGroup, vision: torch.Tensor, text_ids: torch.Tensor,
+                pooled: Optional[torch.Tensor], hidden: Optional[torch.Tensor],
+                ws: torch.Tensor, stream=None) -> None:
+        J.check(J.lib().jnx_backbone_forward(
+            C.byref(self.struct), group.ref, vision.data_ptr(), vision.shape[0],
+            text_ids.data_ptr(), text_ids.shape[0], _ptr(pooled), _ptr(hidden),
+            ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)))
+
+
+class DeviceHeads:
+    """One head slot per tenant (bf16 parameters) and fp32 gradient slots."""
+
+    def __init__(self, tenants: Sequence, d: int, heads: List[Dict], device="cuda"):
+        n = len(tenants)
+        self.n = n
+        self.arr = (J.jnx_head * max(1, n))()
+        self.garr = (J.jnx_head_grads * max(1, n))()
+        self.grads: List[Dict[str, torch.Tensor]] = []
+        self.keep = []
+        for t, (tn, hw) in enumerate(zip(tenants, heads)):
+            if tn.head_kind == J.JNX_HEAD_MLP:
+                self.arr[t] = J.jnx_head(tn.head_kind, d, tn.d_hidden, 0, 0, tn.width,
+                                         hw["w1"].data_ptr(), hw["b1"].data_ptr(),
+                                         hw["w2"].data_ptr(), hw["b2"].data_ptr(),
+                                         None, None, None, None, None)
+                g = {k: torch.zeros(hw[k].shape, dtype=torch.float32, device=device)
+                     for k in ("w1", "b1", "w2", "b2")}
+                self.garr[t] = J.jnx_head_grads(*[g[k].data_ptr() for k in ("w1", "b1", "w2",
+                                                                             "b2")],
+                                                None, None, None, None, None)
+            else:
+                self.arr[t] = J.jnx_head(tn.head_kind, d, 0, tn.n_queries, tn.q_dim, tn.width,
+                                         None, None, None, None, hw["q"].data_ptr(),
+                                         hw["wk"].data_ptr(), hw["wv"].data_ptr(),
+                                         hw["wout"].data_ptr(), hw["bout"].data_ptr())
+                g = {k: torch.zeros(hw[k].shape, dtype=torch.float32, device=device)
+                     for k in ("q", "wk", "wv", "wout", "bout")}
+                self.garr[t] = J.jnx_head_grads(None, None, None, None,
+                                                *[g[k].data_ptr() for k in ("q", "wk", "wv",
+                                                                            "wout", "bout")])
+            self.grads.append(g)
+            self.keep.append(hw)
+
+    def workspace_bytes(self, group: DeviceGroup) -> int:
+        return J.lib().jnx_heads_workspace_bytes(self.arr, self.n, group.ref)
+
+    def forward(self, group: DeviceGroup, pooled, hidden, targets, preds, loss, ws,
+                stream=None) -> None:
+        J.check(J.lib().jnx_heads_forward(
+            self.arr, self.n, group.ref, _ptr(pooled), _ptr(hidden), targets.data_ptr(),
+            preds.data_ptr(), loss.data_ptr(), ws.data_ptr(), ws.numel() * ws.element_size(),
+            _stream(stream)))
+
+    def backward(self, group: DeviceGroup, pooled, hidden, targets, ws, stream=None) -> None:
+        J.check(J.lib().jnx_heads_backward(
+            self.arr, self.n, group.ref, _ptr(pooled), _ptr(hidden), targets.data_ptr(),
+            self.garr, ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def check_status(ws: torch.Tensor, stream=None) -> None:
+    J.check(J.lib().jnx_check_status(ws.data_ptr(), _stream(stream)))
+
+
+class GroupedStep:
+    """One grouped step through the C ABI: backbone forward over the packed
+    batch, then every group tenant's head forward, loss and backward."""
+
+    def __init__(self, backbone: DeviceBackbone, heads: DeviceHeads, group: DeviceGroup,
+                 device="cuda"):
+        self.bb, self.heads, self.group = backbone, heads, group
+        cfg = backbone.cfg
+        S, N = group.plan.n_samples, group.plan.n_tokens
+        self.need_hidden = any(heads.arr[t].kind == J.JNX_HEAD_XATTN
+                               for t in group.plan.slot_tenant.tolist())
+        self.pooled = torch.zeros((max(S, 1), cfg.d), dtype=torch.float32, device=device)
+        self.hidden = (torch.zeros((max(N, 1), cfg.d), dtype=torch.bfloat16, device=device)
+                       if self.need_hidden else None)
+        self.ws_bb = torch.zeros(max(backbone.workspace_bytes(N), 256), dtype=torch.uint8,
+                                 device=device)
+        self.ws_h = torch.zeros(max(heads.workspace_bytes(group), 256), dtype=torch.uint8,
+                                device=device)
+        self.loss = torch.full((max(heads.n, 1),), float("nan"), dtype=torch.float32, device=device)
+
+    def run(self, vision, text_ids, targets, preds, stream=None) -> None:
+        self.bb.forward(self.group, vision, text_ids,
+                        None if self.need_hidden else self.pooled, self.hidden, self.ws_bb, stream)
+        self.heads.forward(self.group, self.pooled, self.hidden, targets, preds, self.loss,
+                           self.ws_h, stream)
+        self.heads.backward(self.group, self.pooled, self.hidden, targets, self.ws_h, stream)

@@ -1,0 +1,115 @@
+"""CPU tests of the C-ABI library: it loads, exports every symbol the
+headers declare, and its host-side plan matches the oracle bit for bit."""
+import ctypes as C
+import os
+import random
+import re
+
+import numpy as np
+import pytest
+
+import synth
+from oracle import plan as OP
+from paper_2607_16074_gb300 import build as B
+from paper_2607_16074_gb300 import jnx as J
+from tests.helpers import oracle_requests
+from tests.test_oracle_plan import _random_queue
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    B.build()
+
+
+def declared_functions():
+    names = set()
+    for h in ("jnx.h", "jnx_ops.h"):
+        src = open(os.path.join(ROOT, "include", h)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names |= set(re.findall(r"\b(jnx_\w+)\s*\(", src))
+    return names
+
+
+def test_library_exports_every_declared_symbol():
+    L = J.lib()
+    names = declared_functions()
+    assert len(names) >= 16
+    for n in names:
+        assert hasattr(L, n), n
+    assert set(J.EXPORTS) == names
+    assert J.jnx_version() == 1
+
+
+def _cmp(plan, ref):
+    for k in J.Plan.FIELDS:
+        assert getattr(plan, k).tolist() == ref[k], k
+    for k in ("n_requests", "n_samples", "n_tokens", "n_slots", "max_seqlen"):
+        assert getattr(plan, k) == ref[k], k
+
+
+@pytest.mark.parametrize("name", synth.WORKLOADS)
+def test_plan_bit_exact_vs_oracle_on_every_workload(name):
+    w = synth.make_workload(name)
+    reqs = oracle_requests(w)
+    for ms, mt in ((1 << 30, 1 << 30), (100, 30000), (3, 1)):
+        ref = OP.group_plan(w.schemas(), reqs, len(w.tenants), ms, mt)
+        got = J.jnx_group_plan(w.schemas(), reqs, len(w.tenants), ms, mt)
+        _cmp(got, ref)
+
+
+def test_plan_bit_exact_vs_oracle_random_queues():
+    rng = random.Random(5)
+    for _ in range(300):
+        schemas, reqs, T = _random_queue(rng, rng.randint(0, 7))
+        ms, mt = rng.randint(1, 9), rng.randint(1, 60)
+        _cmp(J.jnx_group_plan(schemas, reqs, T, ms, mt, caps=(1, 1, 1)),
+             OP.group_plan(schemas, reqs, T, ms, mt))
+
+
+def test_plan_errors_write_nothing_and_explain():
+    w = synth.make_workload("tiny")
+    reqs = oracle_requests(w)
+    bad = [dict(r) for r in reqs]
+    bad[1] = dict(bad[1], tenant=7)
+    with pytest.raises(J.JnxError) as e:
+        J.jnx_group_plan(w.schemas(), bad, 2, 100, 1000)
+    assert e.value.code == J.JNX_ERR_INVALID_ARG and "tenant" in str(e.value)
+    bad = [dict(r) for r in reqs]
+    bad[0] = dict(bad[0], samples=[dict(bad[0]["samples"][0], text_len=0, n_img=0)])
+    with pytest.raises(J.JnxError):
+        J.jnx_group_plan(w.schemas(), bad, 2, 100, 1000)
+    bad = [dict(r) for r in reqs]
+    bad[0] = dict(bad[0], samples=[dict(bad[0]["samples"][0], vision_row=2**31)])
+    with pytest.raises(J.JnxError) as e:
+        J.jnx_group_plan(w.schemas(), bad, 2, 100, 1000)
+    assert e.value.code == J.JNX_ERR_OVERFLOW
+
+
+def test_plan_capacity_two_call_pattern():
+    w = synth.make_workload("small")
+    L = J.lib()
+    sch = J.make_schemas(w.schemas())
+    req, keep = J.make_requests(oracle_requests(w))
+    lim = J.jnx_limits(1 << 30, 1 << 30)
+    raw = J.jnx_plan(4, 16, 2, 0, 0, 0, 0, 0, *([None] * 9))
+    rc = L.jnx_group_plan(sch, len(w.tenants), req, len(w.requests), len(w.tenants),
+                          C.byref(lim), C.byref(raw))
+    assert rc == J.JNX_ERR_CAPACITY
+    assert raw.n_samples == len(w.samples) and raw.n_tokens == w.n_tokens and raw.n_slots == 8
+
+
+def test_empty_queue_gives_empty_plan():
+    p = J.jnx_group_plan(synth.make_workload("tiny").schemas(), [], 2, 10, 10)
+    assert p.n_samples == 0 and p.n_tokens == 0 and p.cu_seqlens.tolist() == [0]
+
+
+def test_gpu_calls_reject_bad_arguments_without_a_gpu():
+    L = J.lib()
+    # a null backbone descriptor is rejected on the host before any launch
+    rc = L.jnx_backbone_forward(None, None, None, 0, None, 0, None, None, None, 0, None)
+    assert rc == J.JNX_ERR_INVALID_ARG
+    assert "backbone" in J.jnx_last_error()
+    rc = L.jnx_op_gemm(None, None, 1, 256, 64, 0, None, 256, None, 0, 0, 0, 0.0, 0, None, 0, None)
+    assert rc == J.JNX_ERR_INVALID_ARG
