@@ -370,6 +370,81 @@ def run_reference(args, rank, world):
                          d2h_bytes_per_step=0))
 
 
+def run_kernel(args):
+    """One library kernel alone through the stage-level C ABI on the 7B-class
+    shapes with `--tokens` packed rows (samples of 272..320 tokens): a small,
+    self-contained case for profilers and per-kernel timing."""
+    import torch
+
+    from paper_2607_16074_gb300 import build as B
+    from paper_2607_16074_gb300 import jnx as J
+    B.build()
+    L = J.lib()
+    dev = torch.device("cuda", 0)
+    M, d, F, H, hd = args.tokens, 4096, 11008, 32, 128
+    g = torch.Generator(device=dev).manual_seed(7)
+    rnd = lambda *s, std=1.0: (torch.randn(*s, generator=g, device=dev) * std).to(torch.bfloat16)
+    s = torch.cuda.current_stream()
+    rng = np.random.default_rng(7)
+    lens = []
+    while sum(lens) < M:
+        lens.append(int(min(rng.integers(272, 321), M - sum(lens))))
+    cu = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
+    pos = torch.cat([torch.arange(l, dtype=torch.int32) for l in lens]).to(dev)
+    ws = torch.zeros(L.jnx_op_gemm_workspace_bytes(1024, hd), dtype=torch.uint8, device=dev)
+    k = args.kernel
+    if k == "gemm_gu":
+        A, W = rnd(M, d), rnd(2 * F, d, std=0.02)
+        out = torch.empty(M, F, dtype=torch.bfloat16, device=dev)
+        call = lambda: L.jnx_op_gemm(A.data_ptr(), W.data_ptr(), M, 2 * F, d, J.JNX_EPI_GLU,
+                                     out.data_ptr(), F, None, 0, 0, 0, 0.0, 0, None, 0, s.cuda_stream)
+        work, unit = 2.0 * M * 2 * F * d, "TFLOP/s"
+    elif k == "gemm_qkv":
+        A, W = rnd(M, d), rnd(3 * d, d, std=0.02)
+        out = torch.empty(M, 3 * d, dtype=torch.bfloat16, device=dev)
+        call = lambda: L.jnx_op_gemm(A.data_ptr(), W.data_ptr(), M, 3 * d, d, J.JNX_EPI_ROPE,
+                                     out.data_ptr(), 3 * d, pos.data_ptr(), 1024, 2 * d, hd,
+                                     10000.0, 0, ws.data_ptr(), ws.numel(), s.cuda_stream)
+        work, unit = 2.0 * M * 3 * d * d, "TFLOP/s"
+    elif k in ("gemm_o", "gemm_down"):
+        K = d if k == "gemm_o" else F
+        A, W = rnd(M, K), rnd(d, K, std=0.02)
+        x = torch.zeros(M, d, dtype=torch.float32, device=dev)
+        call = lambda: L.jnx_op_gemm(A.data_ptr(), W.data_ptr(), M, d, K, J.JNX_EPI_RESID,
+                                     x.data_ptr(), d, None, 0, 0, 0, 0.0, 0, None, 0, s.cuda_stream)
+        work, unit = 2.0 * M * d * K, "TFLOP/s"
+    elif k == "attention":
+        qkv = rnd(M, 3 * d)
+        out = torch.empty(M, d, dtype=torch.bfloat16, device=dev)
+        call = lambda: L.jnx_op_attention(qkv.data_ptr(), H, H, hd, cu.data_ptr(), len(lens),
+                                          max(lens), out.data_ptr(), s.cuda_stream)
+        work, unit = sum(4.0 * l * l * H * hd for l in lens), "TFLOP/s"
+    elif k == "rmsnorm":
+        x = torch.randn(M, d, generator=g, device=dev)
+        gam = rnd(d)
+        out = torch.empty(M, d, dtype=torch.bfloat16, device=dev)
+        call = lambda: L.jnx_op_rmsnorm(x.data_ptr(), gam.data_ptr(), 1e-6, M, d, out.data_ptr(),
+                                        s.cuda_stream)
+        work, unit = M * d * 6.0, "GB/s"
+    else:
+        raise SystemExit(f"unknown kernel {k}")
+    for _ in range(args.warmup):
+        J.check(call())
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(args.steps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(s)
+        J.check(call())
+        b.record(s)
+        torch.cuda.synchronize()
+        times.append(a.elapsed_time(b))
+    med = float(np.median(times))
+    rate = work / (med / 1e3) / (1e12 if unit == "TFLOP/s" else 1e9)
+    return dict(kernel=k, tokens=M, median_ms=round(med, 4), rate=round(rate, 1), unit=unit,
+                times_ms=[round(t, 4) for t in times])
+
+
 def dataclass_layers(w, n_layers):
     """The workload with only its first n_layers blocks (weights of the other
     blocks are not needed by a bounded oracle sample)."""
@@ -388,7 +463,14 @@ def main():
     ap.add_argument("--no-per-tenant", action="store_true")
     ap.add_argument("--oracle-layers", type=int, default=2)
     ap.add_argument("--reference-layers", type=int, default=1)
+    ap.add_argument("--kernel", default=None,
+                    help="time one kernel alone (gemm_gu, gemm_qkv, gemm_o, gemm_down, "
+                         "attention, rmsnorm) on 7B-class shapes with --tokens rows")
+    ap.add_argument("--tokens", type=int, default=8192)
     args = ap.parse_args()
+    if args.kernel:
+        print(json.dumps(run_kernel(args)), flush=True)
+        return
     args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
 
     rank = int(os.environ.get("RANK", "0"))

@@ -10,7 +10,7 @@ from oracle import model as M
 from paper_2607_16074_gb300 import jnx as J
 from paper_2607_16074_gb300 import runtime as R
 from tests.gpu_helpers import f64
-from tests.helpers import BF16_TOL, GROUPED_TOL, oracle_requests, rel_err
+from tests.helpers import BF16_TOL, GROUPED_TOL, deep_tol, oracle_requests, rel_err
 
 pytestmark = pytest.mark.gpu
 
@@ -176,4 +176,54 @@ def test_llama7b_full_size_sampled_sample():
     npi = synth.to_numpy_tree(s.inp)
     x = M.sample_embeddings(bb, vars(smp), npi["vision"], npi["text_ids"], np_bw["text_table"])
     ref = M.mean_pool(M.backbone_sample(bb, np_bw, x))
-    assert rel_err(f64(step.pooled[si]), ref) < BF16_TOL
+    e = rel_err(f64(step.pooled[si]), ref)
+    assert e < deep_tol(w.backbone.n_layers), e
+
+
+def test_llama7b_shapes_two_blocks_whole_tenants():
+    """Every kernel at the 7B-class widths and the full packed length
+    (~65.8k tokens, 32 tenants), two blocks deep so the benchmark spec's 2e-2 bound
+    applies to the whole path; the two smallest tenants are checked end to
+    end (features, loss, predictions, head gradients)."""
+    w = synth.make_workload("llama7b", n_layers=2)
+    s = Setup(w, gen_device="cuda")
+    plan, step, preds = s.run()
+    counts = {t: sum(len(r.samples) for r in w.requests if r.tenant == t) for t in range(32)}
+    pick = sorted(counts, key=lambda t: (counts[t], t))[:2]
+    _compare(s, plan, step, preds, s.oracle(tenants=pick))
+
+
+@pytest.mark.parametrize("name", ["small", "llama7b"])
+def test_heads_stage_on_synthetic_features(name):
+    """The head stage alone at the workload's head shapes, on seeded random
+    pooled features (inputs from the generator, not from the backbone)."""
+    w = synth.make_workload(name)
+    hw = synth.make_head_weights(w)
+    inp = synth.make_inputs(w)
+    plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), len(w.tenants), 1 << 30, 1 << 30)
+    g = R.DeviceGroup(plan)
+    pooled = torch.randn((plan.n_samples, w.backbone.d),
+                         generator=torch.Generator().manual_seed(3)).cuda()
+    heads = R.DeviceHeads(w.tenants, w.backbone.d, [{k: v.cuda() for k, v in h.items()} for h in hw])
+    ws = torch.zeros(heads.workspace_bytes(g), dtype=torch.uint8, device="cuda")
+    tg = inp["targets"].cuda()
+    preds = torch.full_like(tg, float("nan"))
+    loss = torch.full((len(w.tenants),), float("nan"), device="cuda")
+    heads.forward(g, pooled, None, tg, preds, loss, ws)
+    heads.backward(g, pooled, None, tg, ws)
+    torch.cuda.synchronize()
+    P = f64(pooled)
+    npT = synth.to_numpy_tree(inp)["targets"]
+    seg = plan.seg_offsets
+    for gi, t in enumerate(plan.slot_tenant.tolist()):
+        tn = w.tenants[t]
+        samples = [s for q in w.requests if q.tenant == t for s in q.samples]
+        T = np.stack([npT[s.target_off:s.target_off + tn.width] for s in samples])
+        feats = list(P[seg[gi]:seg[gi + 1]])
+        lo, Y, gr = M.tenant_step(0, synth.to_numpy_tree(hw[t]), feats, T)
+        assert abs(float(loss[t]) - lo) < 1e-4 * abs(lo)
+        got = np.stack([f64(preds[s.target_off:s.target_off + tn.width]) for s in samples])
+        assert rel_err(got, Y) < 1e-4
+        for k, v in gr.items():
+            e = rel_err(f64(heads.grads[t][k]), v)
+            assert e < 1e-4, (t, k, e)
