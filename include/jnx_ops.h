@@ -64,6 +64,26 @@ jnx_status jnx_op_final_pool(const float* x, const uint16_t* gamma, float eps,
                              const int32_t* cu_seqlens, int32_t n_samples, int32_t d,
                              float* pooled, uint16_t* hidden, void* stream);
 
+/* The fused QKV projection + RoPE of jnx_op_gemm (JNX_EPI_ROPE) for callers
+ * that cannot allocate device memory — e.g. a plugin in a serving process
+ * whose pool owns every device allocation, or a batching worker that must
+ * not call cudaMalloc between requests because it can stall the device.
+ * The paper has no counterpart: this is a deployment variant of the library.
+ * The caller passes inputs and outputs only; the status word and the RoPE
+ * table live in a fixed file-scope device array inside the library (every
+ * GPU that loads the library holds it until exit; nothing is allocated).
+ * Limits: max_pos * head_dim / 2 <= JNX_NOALLOC_MAX_ROPE_ENTRIES, otherwise
+ * JNX_ERR_UNSUPPORTED before any launch; positions must be < max_pos.
+ * The first call on a device looks up the array's address (make it before
+ * any stream capture).  All calls on a device share the array: each clears
+ * the status word and rewrites the table it reads, and calls that overlap on
+ * the GPU race.  Arguments and results otherwise as jnx_op_gemm. */
+#define JNX_NOALLOC_MAX_ROPE_ENTRIES (1 << 19)
+jnx_status jnx_op_gemm_rope_noalloc(const uint16_t* A, const uint16_t* W, int32_t M, int32_t N,
+                                    int32_t K, uint16_t* out, int32_t ldo, const int32_t* pos,
+                                    int32_t max_pos, int32_t rope_cols, int32_t head_dim,
+                                    float rope_theta, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -25,6 +25,7 @@ JNX_ERR_UNSUPPORTED, JNX_ERR_WORKSPACE = -9, -10
 JNX_GLU_SWIGLU, JNX_GLU_GEGLU_TANH = 0, 1
 JNX_HEAD_MLP, JNX_HEAD_XATTN = 0, 1
 JNX_EPI_BF16, JNX_EPI_F32, JNX_EPI_RESID, JNX_EPI_GLU, JNX_EPI_ROPE = 0, 1, 2, 3, 4
+JNX_NOALLOC_MAX_ROPE_ENTRIES = 1 << 19
 
 
 class JnxError(RuntimeError):
@@ -109,7 +110,7 @@ EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_work
            "jnx_heads_backward", "jnx_check_status", "jnx_pack_gate_up", "jnx_op_pack",
            "jnx_op_rmsnorm", "jnx_op_gemm_workspace_bytes", "jnx_op_gemm", "jnx_op_attention",
            "jnx_op_final_pool", "jnx_trace_enable", "jnx_trace_disable", "jnx_trace_count",
-           "jnx_trace_read")
+           "jnx_trace_read", "jnx_op_gemm_rope_noalloc")
 
 
 def lib() -> C.CDLL:
@@ -148,6 +149,8 @@ def lib() -> C.CDLL:
         "jnx_trace_disable": (i32, []),
         "jnx_trace_count": (i32, []),
         "jnx_trace_read": (i32, [vp, vp, vp, i32, P32]),
+        "jnx_op_gemm_rope_noalloc": (i32, [vp, vp, i32, i32, i32, vp, i32, vp, i32, i32, i32, f32,
+                                           vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
