@@ -315,6 +315,7 @@ jnx_status jnx_pack_gate_up(const uint16_t* w_gate, const uint16_t* w_up, int32_
 #define JNX_K_HEADS_FWD 10 /* work = FLOPs */
 #define JNX_K_HEADS_BWD 11 /* work = FLOPs */
 #define JNX_K_GEMM 12      /* jnx_op_gemm; work = FLOPs */
+#define JNX_K_LORA 13      /* LoRA row tenants / down-projections; work = FLOPs */
 
 /* While enabled on the calling thread, each kernel launch of the library is
  * bracketed by two CUDA events on its stream (up to `capacity` launches are

@@ -27,6 +27,9 @@ struct BackboneWs {
     uint16_t* att;    // [N, H hd] bf16
     uint16_t* u;      // [N, F] bf16
     float2* rope;     // [max_pos, hd / 2]
+    int* row_tenant;  // LoRA: tenant of each packed row [N]
+    float* t_qkv;     // LoRA: n1 [A_q | A_k | A_v]^T  [N, 3r]
+    float* t_o;       // LoRA: attention output A_o^T  [N, r]
     size_t bytes;
 };
 
@@ -49,6 +52,11 @@ BackboneWs carve_backbone(const jnx_backbone* bb, int64_t N, void* base) {
     w.att = reinterpret_cast<uint16_t*>(take((size_t)N * bb->n_heads * bb->head_dim * 2));
     w.u = reinterpret_cast<uint16_t*>(take((size_t)N * bb->d_ff * 2));
     w.rope = reinterpret_cast<float2*>(take((size_t)kMaxRopePos * (bb->head_dim / 2) * 8));
+    if (bb->lora_rank) {
+        w.row_tenant = reinterpret_cast<int*>(take((size_t)N * 4));
+        w.t_qkv = reinterpret_cast<float*>(take((size_t)N * 3 * kLoraRank * 4));
+        w.t_o = reinterpret_cast<float*>(take((size_t)N * kLoraRank * 4));
+    }
     w.bytes = off;
     return w;
 }
@@ -71,11 +79,18 @@ jnx_status check_backbone(const jnx_backbone* bb) {
         return st;
     if (bb->glu != JNX_GLU_SWIGLU && bb->glu != JNX_GLU_GEGLU_TANH)
         return fail(JNX_ERR_INVALID_ARG, "backbone: unknown glu %d", bb->glu);
-    if (bb->lora_rank != 0) return fail(JNX_ERR_UNSUPPORTED, "backbone: LoRA not built yet");
+    if (bb->lora_rank != 0 && bb->lora_rank != kLoraRank)
+        return fail(JNX_ERR_UNSUPPORTED, "backbone: LoRA rank %d (built for %d)", bb->lora_rank,
+                    kLoraRank);
+    if (bb->lora_rank && (bb->n_tenants <= 0 || d % 64 || (bb->n_heads * bb->head_dim) % 64))
+        return fail(JNX_ERR_INVALID_ARG, "backbone: LoRA needs n_tenants > 0 and widths %% 64");
     for (int l = 0; l < bb->n_layers; ++l) {
         const jnx_layer& L = bb->layers[l];
         if (!L.attn_norm || !L.w_qkv || !L.w_o || !L.ffn_norm || !L.w_gu || !L.w_down)
             return fail(JNX_ERR_INVALID_ARG, "backbone: layer %d has a null weight", l);
+        if (bb->lora_rank && (!L.lora_a_q || !L.lora_b_q || !L.lora_a_k || !L.lora_b_k ||
+                              !L.lora_a_v || !L.lora_b_v || !L.lora_a_o || !L.lora_b_o))
+            return fail(JNX_ERR_INVALID_ARG, "backbone: layer %d has a null LoRA adapter", l);
     }
     return JNX_OK;
 }
@@ -123,6 +138,11 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
     if (ws_bytes < w.bytes)
         return fail(JNX_ERR_WORKSPACE, "backbone: workspace %zu < %zu bytes", ws_bytes, w.bytes);
     if (N == 0) return JNX_OK;
+    const bool lora = bb->lora_rank != 0;
+    for (int i = 0; lora && i < g->n_slots; ++i)
+        if (g->h_slot_tenant[i] < 0 || g->h_slot_tenant[i] >= bb->n_tenants)
+            return fail(JNX_ERR_INVALID_ARG, "backbone: tenant %d has no LoRA adapter",
+                        g->h_slot_tenant[i]);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const int qkvw = (H + 2 * Hkv) * hd;
 
@@ -136,6 +156,10 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
     {
         TraceScope ts(JNX_K_ROPE_TABLE, (double)g->max_seqlen * hd * 4.0, s);
         if ((st = rope_table_launch(w.rope, g->max_seqlen, hd, bb->rope_theta, s))) return st;
+    }
+    if (lora) {
+        TraceScope ts(JNX_K_LORA, (double)N * 4.0, s);
+        if ((st = lora_row_tenant_launch(g, w.row_tenant, s))) return st;
     }
     // within-sample attention FLOPs: QK^T and PV over each sample's own tokens
     double attn_flops = 0.0;
@@ -163,6 +187,23 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
         p.rope_cols = (H + Hkv) * hd;
         p.hd = hd;
         p.status = w.status;
+        if (lora) {
+            {
+                TraceScope ts(JNX_K_LORA, 2.0 * N * d * 3 * kLoraRank, s);
+                const uint16_t* a3[3] = {L.lora_a_q, L.lora_a_k, L.lora_a_v};
+                if ((st = lora_down_launch(g, w.nrm, d, d, 3, a3, w.t_qkv, 3 * kLoraRank, s)))
+                    return st;
+            }
+            p.lora_t = w.t_qkv;
+            p.ldt = 3 * kLoraRank;
+            p.row_tenant = w.row_tenant;
+            p.lora_b[0] = L.lora_b_q;
+            p.lora_b[1] = L.lora_b_k;
+            p.lora_b[2] = L.lora_b_v;
+            p.lora_cols[0] = H * hd;
+            p.lora_cols[1] = Hkv * hd;
+            p.lora_cols[2] = Hkv * hd;
+        }
         {
             TraceScope ts(JNX_K_GEMM_QKV, 2.0 * N * qkvw * d, s);
             if ((st = gemm_launch(w.nrm, d, L.w_qkv, d, p, s))) return st;
@@ -181,6 +222,19 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
         p.resid = w.x;
         p.ldr = d;
         p.status = w.status;
+        if (lora) {
+            {
+                TraceScope ts(JNX_K_LORA, 2.0 * N * H * hd * kLoraRank, s);
+                const uint16_t* a1[1] = {L.lora_a_o};
+                if ((st = lora_down_launch(g, w.att, H * hd, H * hd, 1, a1, w.t_o, kLoraRank, s)))
+                    return st;
+            }
+            p.lora_t = w.t_o;
+            p.ldt = kLoraRank;
+            p.row_tenant = w.row_tenant;
+            p.lora_b[0] = L.lora_b_o;
+            p.lora_cols[0] = d;
+        }
         {
             TraceScope ts(JNX_K_GEMM_O, 2.0 * N * d * H * hd, s);
             if ((st = gemm_launch(w.att, H * hd, L.w_o, H * hd, p, s))) return st;
@@ -233,13 +287,32 @@ struct HeadsWs {
     size_t bytes;
 };
 
-int heads_ld(const jnx_head* heads, const jnx_group* g) {
-    int ld = 8;
+struct HeadDims {
+    int ld_h = 8, ld_y = 8, ldkv = 256, nq = 4;
+    bool any_mlp = false, any_x = false;
+};
+
+int head_hid(const jnx_head& h) {
+    return h.kind == JNX_HEAD_MLP ? h.d_hidden : h.n_queries * h.q_dim;
+}
+
+HeadDims head_dims(const jnx_head* heads, const jnx_group* g) {
+    HeadDims d;
     for (int i = 0; i < g->n_slots; ++i) {
         const jnx_head& h = heads[g->h_slot_tenant[i]];
-        ld = std::max(ld, std::max(h.d_hidden, h.width));
+        d.ld_h = std::max(d.ld_h, head_hid(h));
+        d.ld_y = std::max(d.ld_y, h.width);
+        if (h.kind == JNX_HEAD_XATTN) {
+            d.any_x = true;
+            d.ldkv = std::max(d.ldkv, h.q_dim);
+            d.nq = h.n_queries;
+        } else {
+            d.any_mlp = true;
+        }
     }
-    return (ld + 7) / 8 * 8;
+    d.ld_h = (d.ld_h + 7) / 8 * 8;
+    d.ld_y = (d.ld_y + 7) / 8 * 8;
+    return d;
 }
 
 HeadsWs carve_heads(const jnx_head* heads, const jnx_group* g, void* base) {
@@ -249,42 +322,71 @@ HeadsWs carve_heads(const jnx_head* heads, const jnx_group* g, void* base) {
     auto take = [&](size_t bytes) {
         uint8_t* r = p ? p + off : nullptr;
         off += up(bytes);
-        return r;
+        return reinterpret_cast<float*>(r);
     };
-    const int ld = heads_ld(heads, g);
-    const size_t arr = (size_t)std::max(g->n_samples, 1) * ld * 4;
+    const HeadDims hd = head_dims(heads, g);
+    const size_t S = (size_t)std::max(g->n_samples, 1), N = (size_t)std::max(g->n_tokens, 1);
     w.status = reinterpret_cast<int*>(take(kStatusBytes));
-    w.sc.z = reinterpret_cast<float*>(take(arr));
-    w.sc.a = reinterpret_cast<float*>(take(arr));
-    w.sc.y = reinterpret_cast<float*>(take(arr));
-    w.sc.dy = reinterpret_cast<float*>(take(arr));
-    w.sc.dz = reinterpret_cast<float*>(take(arr));
-    w.sc.ld = ld;
+    w.sc.ld_h = hd.ld_h;
+    w.sc.ld_y = hd.ld_y;
+    w.sc.z = take(S * hd.ld_h * 4);
+    w.sc.h = take(S * hd.ld_h * 4);
+    w.sc.dh = take(S * hd.ld_h * 4);
+    w.sc.y = take(S * hd.ld_y * 4);
+    w.sc.dy = take(S * hd.ld_y * 4);
+    w.sc.ldkv = hd.ldkv;
+    if (hd.any_x) {
+        w.sc.kbuf = take(N * hd.ldkv * 4);
+        w.sc.vbuf = take(N * hd.ldkv * 4);
+        w.sc.dk = take(N * hd.ldkv * 4);
+        w.sc.dv = take(N * hd.ldkv * 4);
+        w.sc.P = take(N * hd.nq * 4);
+        w.sc.dS = take(N * hd.nq * 4);
+        w.sc.dQs = take(S * hd.ld_h * 4);
+    }
     w.bytes = off;
     return w;
 }
 
 jnx_status check_heads(const jnx_head* heads, int32_t n_tenants, const jnx_group* g,
-                       bool need_grads, const jnx_head_grads* grads) {
+                       bool need_grads, const jnx_head_grads* grads, const float* pooled,
+                       const uint16_t* hidden) {
     jnx_status st;
     if ((st = check_group(g))) return st;
     if (!heads && g->n_slots > 0) return fail(JNX_ERR_INVALID_ARG, "heads: null head table");
+    int nq = -1;
     for (int i = 0; i < g->n_slots; ++i) {
         const int t = g->h_slot_tenant[i];
         if (t < 0 || t >= n_tenants)
             return fail(JNX_ERR_INVALID_ARG, "heads: group slot %d tenant %d out of range", i, t);
         const jnx_head& h = heads[t];
-        if (h.kind != JNX_HEAD_MLP)
-            return fail(JNX_ERR_UNSUPPORTED, "heads: tenant %d head kind %d not built yet", t,
-                        h.kind);
-        if (h.d_in % 8 || h.d_hidden % 8 || h.d_hidden <= 0 || h.width <= 0 || h.d_in <= 0)
-            return fail(JNX_ERR_UNSUPPORTED, "heads: tenant %d widths must be multiples of 8", t);
-        if (!h.w1 || !h.b1 || !h.w2 || !h.b2)
-            return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null parameter", t);
-        if (need_grads) {
-            const jnx_head_grads& gr = grads[t];
-            if (!gr.w1 || !gr.b1 || !gr.w2 || !gr.b2)
+        if (h.width <= 0 || h.d_in <= 0 || h.d_in % 64)
+            return fail(JNX_ERR_UNSUPPORTED, "heads: tenant %d needs width > 0, d_in %% 64 == 0", t);
+        if (h.kind == JNX_HEAD_MLP) {
+            if (h.d_hidden <= 0 || h.d_hidden % 8)
+                return fail(JNX_ERR_UNSUPPORTED, "heads: tenant %d d_hidden %% 8 != 0", t);
+            if (!h.w1 || !h.b1 || !h.w2 || !h.b2)
+                return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null parameter", t);
+            if (!pooled) return fail(JNX_ERR_INVALID_ARG, "heads: MLP heads need pooled features");
+            if (need_grads && (!grads[t].w1 || !grads[t].b1 || !grads[t].w2 || !grads[t].b2))
                 return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null gradient buffer", t);
+        } else if (h.kind == JNX_HEAD_XATTN) {
+            if (h.n_queries <= 0 || h.n_queries > 32 || h.n_queries % 4 || h.q_dim % 256 ||
+                h.q_dim > 512 || h.q_dim <= 0)
+                return fail(JNX_ERR_UNSUPPORTED,
+                            "heads: tenant %d query head needs n_queries in {4,8,..,32} and "
+                            "q_dim in {256, 512}", t);
+            if (nq >= 0 && nq != h.n_queries)
+                return fail(JNX_ERR_UNSUPPORTED, "heads: query heads of one group differ in n_queries");
+            nq = h.n_queries;
+            if (!h.q || !h.wk || !h.wv || !h.wout || !h.bout)
+                return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null parameter", t);
+            if (!hidden) return fail(JNX_ERR_INVALID_ARG, "heads: query heads need hidden rows");
+            if (need_grads && (!grads[t].q || !grads[t].wk || !grads[t].wv || !grads[t].wout ||
+                               !grads[t].bout))
+                return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null gradient buffer", t);
+        } else {
+            return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d unknown head kind %d", t, h.kind);
         }
         const int s0 = g->h_seg_offsets[i], s1 = g->h_seg_offsets[i + 1];
         if (s0 < 0 || s1 <= s0 || s1 > g->n_samples)
@@ -293,34 +395,81 @@ jnx_status check_heads(const jnx_head* heads, int32_t n_tenants, const jnx_group
     return JNX_OK;
 }
 
-// Fill the per-slot table for group slots [g0, g0 + n).
-void fill_table(HeadTable& tab, const jnx_head* heads, const jnx_head_grads* grads,
-                const jnx_group* g, int g0, int n, int& max_hidden, int& max_width, int& max_din) {
-    max_hidden = max_width = max_din = 0;
+// Fill the per-slot table for group slots [g0, g0 + n) and describe the batch.
+HeadBatch fill_table(HeadTable& tab, const jnx_head* heads, const jnx_head_grads* grads,
+                     const jnx_group* g, int g0, int n) {
+    HeadBatch b{};
+    b.g0 = g0;
+    b.n = n;
+    b.sample0 = g->h_seg_offsets[g0];
+    b.sample1 = g->h_seg_offsets[g0 + n];
     for (int i = 0; i < n; ++i) {
         const int t = g->h_slot_tenant[g0 + i];
         const jnx_head& h = heads[t];
         HeadSlot& hs = tab.slot[i];
-        hs.w1 = h.w1;
-        hs.b1 = h.b1;
-        hs.w2 = h.w2;
-        hs.b2 = h.b2;
-        if (grads) {
-            hs.g_w1 = grads[t].w1;
-            hs.g_b1 = grads[t].b1;
-            hs.g_w2 = grads[t].w2;
-            hs.g_b2 = grads[t].b2;
-        }
+        hs = HeadSlot{};
+        hs.kind = h.kind;
+        hs.tenant = t;
         hs.s0 = g->h_seg_offsets[g0 + i];
         hs.s1 = g->h_seg_offsets[g0 + i + 1];
+        hs.r0 = g->h_cu_seqlens[hs.s0];
+        hs.r1 = g->h_cu_seqlens[hs.s1];
         hs.d_in = h.d_in;
-        hs.d_hidden = h.d_hidden;
+        hs.hid = head_hid(h);
         hs.width = h.width;
-        hs.tenant = t;
-        max_hidden = std::max(max_hidden, h.d_hidden);
-        max_width = std::max(max_width, h.width);
-        max_din = std::max(max_din, h.d_in);
+        if (h.kind == JNX_HEAD_MLP) {
+            hs.w1 = h.w1;
+            hs.b1 = h.b1;
+            hs.w2 = h.w2;
+            hs.b2 = h.b2;
+            if (grads) {
+                hs.g_w1 = grads[t].w1;
+                hs.g_b1 = grads[t].b1;
+                hs.g_w2 = grads[t].w2;
+                hs.g_b2 = grads[t].b2;
+            }
+            b.any_mlp = true;
+            b.max_mlp_hid = std::max(b.max_mlp_hid, hs.hid);
+        } else {
+            hs.nq = h.n_queries;
+            hs.dq = h.q_dim;
+            hs.w2 = h.wout;
+            hs.b2 = h.bout;
+            hs.q = h.q;
+            hs.wk = h.wk;
+            hs.wv = h.wv;
+            if (grads) {
+                hs.g_w2 = grads[t].wout;
+                hs.g_b2 = grads[t].bout;
+                hs.g_q = grads[t].q;
+                hs.g_wk = grads[t].wk;
+                hs.g_wv = grads[t].wv;
+            }
+            b.any_xattn = true;
+            b.max_nq = std::max(b.max_nq, hs.nq);
+            b.max_dq = std::max(b.max_dq, hs.dq);
+        }
+        b.max_hid = std::max(b.max_hid, hs.hid);
+        b.max_width = std::max(b.max_width, hs.width);
     }
+    return b;
+}
+
+double heads_flops(const HeadTable& tab, int n, bool backward) {
+    double fl = 0.0;
+    for (int i = 0; i < n; ++i) {
+        const HeadSlot& h = tab.slot[i];
+        const double ns = h.s1 - h.s0, nr = h.r1 - h.r0;
+        if (h.kind == JNX_HEAD_MLP) {
+            fl += 2.0 * ns * ((double)h.d_in * h.hid + (backward ? 2.0 : 1.0) * h.hid * h.width);
+        } else {
+            const double kv = 2.0 * nr * h.d_in * 2.0 * h.dq;
+            const double att = 4.0 * h.nq * h.dq * nr;
+            const double out = 2.0 * ns * h.hid * h.width;
+            fl += backward ? (kv + 2.0 * att + 2.0 * out) : (kv + att + out);
+        }
+    }
+    return fl;
 }
 
 }  // namespace
@@ -340,27 +489,40 @@ extern "C" jnx_status jnx_heads_forward(const jnx_head* heads, int32_t n_tenants
                                         void* stream) {
     clear_error();
     jnx_status st;
-    if ((st = check_heads(heads, n_tenants, g, false, nullptr))) return st;
+    if ((st = check_heads(heads, n_tenants, g, false, nullptr, pooled, hidden))) return st;
     if (g->n_slots == 0) return JNX_OK;
-    if (!pooled || !targets || !preds || !loss || !workspace)
+    if (!targets || !preds || !loss || !workspace)
         return fail(JNX_ERR_INVALID_ARG, "heads forward: null buffer");
     HeadsWs w = carve_heads(heads, g, workspace);
     if (ws_bytes < w.bytes)
         return fail(JNX_ERR_WORKSPACE, "heads: workspace %zu < %zu bytes", ws_bytes, w.bytes);
+    if ((st = heads_set_smem())) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int d = heads[g->h_slot_tenant[0]].d_in;
     HeadTable tab;
     for (int g0 = 0; g0 < g->n_slots; g0 += kMaxSlots) {
         const int n = std::min(kMaxSlots, g->n_slots - g0);
-        int mh, mw, md;
-        fill_table(tab, heads, nullptr, g, g0, n, mh, mw, md);
-        double fl = 0.0;
-        for (int i = 0; i < n; ++i)
-            fl += 2.0 * (tab.slot[i].s1 - tab.slot[i].s0) *
-                  ((double)tab.slot[i].d_in * tab.slot[i].d_hidden +
-                   (double)tab.slot[i].d_hidden * tab.slot[i].width);
-        TraceScope ts(JNX_K_HEADS_FWD, fl, s);
-        if ((st = mlp_heads_forward(tab, n, mh, mw, pooled, heads[g->h_slot_tenant[g0]].d_in,
-                                    g->sample_target, targets, preds, loss, w.sc, s)))
+        HeadBatch b = fill_table(tab, heads, nullptr, g, g0, n);
+        TraceScope ts(JNX_K_HEADS_FWD, heads_flops(tab, n, false), s);
+        for (int i = 0; i < n && b.any_xattn; ++i) {
+            const HeadSlot& hs = tab.slot[i];
+            if (hs.kind != JNX_HEAD_XATTN || hs.r1 == hs.r0) continue;
+            for (int which = 0; which < 2; ++which) {
+                GemmParams p{};
+                p.M = hs.r1 - hs.r0;
+                p.N = hs.dq;
+                p.K = d;
+                p.epi = EPI_F32;
+                p.out = (which ? w.sc.vbuf : w.sc.kbuf) + (size_t)hs.r0 * w.sc.ldkv;
+                p.ldo = w.sc.ldkv;
+                p.status = w.status;
+                if ((st = gemm_launch(hidden + (size_t)hs.r0 * d, d, which ? hs.wv : hs.wk, d, p,
+                                      s)))
+                    return st;
+            }
+        }
+        if ((st = heads_forward_launch(tab, b, w.sc, pooled, d, g->cu_seqlens, g->sample_slot,
+                                       g->sample_target, targets, preds, loss, s)))
             return st;
     }
     return JNX_OK;
@@ -373,27 +535,24 @@ extern "C" jnx_status jnx_heads_backward(const jnx_head* heads, int32_t n_tenant
                                          size_t ws_bytes, void* stream) {
     clear_error();
     jnx_status st;
-    if (!grads && g && g->n_slots > 0) return fail(JNX_ERR_INVALID_ARG, "heads backward: null grads");
-    if ((st = check_heads(heads, n_tenants, g, true, grads))) return st;
+    if (!grads && g && g->n_slots > 0)
+        return fail(JNX_ERR_INVALID_ARG, "heads backward: null grads");
+    if ((st = check_heads(heads, n_tenants, g, true, grads, pooled, hidden))) return st;
     if (g->n_slots == 0) return JNX_OK;
-    if (!pooled || !workspace) return fail(JNX_ERR_INVALID_ARG, "heads backward: null buffer");
+    if (!workspace) return fail(JNX_ERR_INVALID_ARG, "heads backward: null workspace");
     HeadsWs w = carve_heads(heads, g, workspace);
     if (ws_bytes < w.bytes)
         return fail(JNX_ERR_WORKSPACE, "heads: workspace %zu < %zu bytes", ws_bytes, w.bytes);
+    if ((st = heads_set_smem())) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int d = heads[g->h_slot_tenant[0]].d_in;
     HeadTable tab;
     for (int g0 = 0; g0 < g->n_slots; g0 += kMaxSlots) {
         const int n = std::min(kMaxSlots, g->n_slots - g0);
-        int mh, mw, md;
-        fill_table(tab, heads, grads, g, g0, n, mh, mw, md);
-        double fl = 0.0;
-        for (int i = 0; i < n; ++i)
-            fl += 2.0 * (tab.slot[i].s1 - tab.slot[i].s0) *
-                  ((double)tab.slot[i].d_in * tab.slot[i].d_hidden +
-                   2.0 * tab.slot[i].d_hidden * tab.slot[i].width);
-        TraceScope ts(JNX_K_HEADS_BWD, fl, s);
-        if ((st = mlp_heads_backward(tab, n, mh, mw, md, pooled, heads[g->h_slot_tenant[g0]].d_in,
-                                     w.sc, s)))
+        HeadBatch b = fill_table(tab, heads, grads, g, g0, n);
+        TraceScope ts(JNX_K_HEADS_BWD, heads_flops(tab, n, true), s);
+        if ((st = heads_backward_launch(tab, b, w.sc, pooled, d, hidden, g->cu_seqlens,
+                                        g->sample_slot, s)))
             return st;
     }
     return JNX_OK;
@@ -401,6 +560,7 @@ extern "C" jnx_status jnx_heads_backward(const jnx_head* heads, int32_t n_tenant
 
 // ---------------------------------------------------------------------------
 // status and helpers
+
 // ---------------------------------------------------------------------------
 
 extern "C" jnx_status jnx_check_status(void* workspace, void* stream) {

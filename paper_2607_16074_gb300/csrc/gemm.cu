@@ -59,10 +59,53 @@ __device__ __forceinline__ float act_fn(float g, int act) {
     return 0.5f * g * (1.0f + tanhf(c * (g + 0.044715f * g * g * g)));
 }
 
-template <int EPI>
+// LoRA up-projection for 32 consecutive columns [col, col + 32) of one row:
+// v[e] += t[row, part r..] . B_part[tenant][col + e - part start, :].  The
+// 32 columns never straddle two parts (part widths are multiples of 64).
+__device__ __forceinline__ void lora_chunk(float (&v)[32], int row, int tenant, int col,
+                                           const GemmParams& p) {
+    constexpr int R = kLoraRank;
+    int part = 0, c = col;
+    while (part < 2 && c >= p.lora_cols[part]) {
+        c -= p.lora_cols[part];
+        ++part;
+    }
+    const float4* tr = reinterpret_cast<const float4*>(p.lora_t + (size_t)row * p.ldt + part * R);
+    float t[R];
+#pragma unroll
+    for (int i = 0; i < R / 4; ++i) {
+        const float4 q = tr[i];
+        t[4 * i] = q.x;
+        t[4 * i + 1] = q.y;
+        t[4 * i + 2] = q.z;
+        t[4 * i + 3] = q.w;
+    }
+    const uint4* b = reinterpret_cast<const uint4*>(
+        p.lora_b[part] + ((size_t)tenant * p.lora_cols[part] + c) * R);
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+        float acc = 0.f;
+#pragma unroll
+        for (int h = 0; h < R / 8; ++h) {
+            const uint4 w = __ldg(b + (R / 8) * e + h);
+            acc += t[8 * h + 0] * __uint_as_float(w.x << 16) +
+                   t[8 * h + 1] * __uint_as_float(w.x & 0xFFFF0000u) +
+                   t[8 * h + 2] * __uint_as_float(w.y << 16) +
+                   t[8 * h + 3] * __uint_as_float(w.y & 0xFFFF0000u) +
+                   t[8 * h + 4] * __uint_as_float(w.z << 16) +
+                   t[8 * h + 5] * __uint_as_float(w.z & 0xFFFF0000u) +
+                   t[8 * h + 6] * __uint_as_float(w.w << 16) +
+                   t[8 * h + 7] * __uint_as_float(w.w & 0xFFFF0000u);
+        }
+        v[e] += acc;
+    }
+}
+
+template <int EPI, bool LORA>
 __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int n0,
                                               const GemmParams& p) {
     const bool valid = row < p.M;
+    const int tenant = (LORA && valid) ? p.row_tenant[row] : 0;
     if constexpr (EPI == EPI_BF16 || EPI == EPI_F32 || EPI == EPI_RESID) {
 #pragma unroll 1
         for (int c = 0; c < 8; ++c) {
@@ -71,6 +114,14 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int n0,
             tmem_ld_wait();
             if (!valid) continue;
             const int col = n0 + c * 32;
+            if constexpr (LORA) {
+                float f[32];
+#pragma unroll
+                for (int e = 0; e < 32; ++e) f[e] = __uint_as_float(r[e]);
+                lora_chunk(f, row, tenant, col, p);
+#pragma unroll
+                for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(f[e]);
+            }
             if constexpr (EPI == EPI_BF16) {
                 uint4* dst = reinterpret_cast<uint4*>(static_cast<bf16_t*>(p.out) +
                                                       (size_t)row * p.ldo + col);
@@ -149,6 +200,10 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int n0,
                 a[e] = __uint_as_float(lo[e]);
                 b[e] = __uint_as_float(hi[e]);
             }
+            if constexpr (LORA) {
+                lora_chunk(a, row, tenant, col, p);
+                lora_chunk(b, row, tenant, col + half, p);
+            }
             if (col < p.rope_cols) {
                 const float2* cs = p.rope + (size_t)pos * half + hchunk * 32;
 #pragma unroll
@@ -180,7 +235,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int n0,
     }
 }
 
-template <int EPI>
+template <int EPI, bool LORA>
 __global__ void __launch_bounds__(192, 1)
     k_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
            GemmParams p) {
@@ -321,7 +376,8 @@ __global__ void __launch_bounds__(192, 1)
             }
             tc_fence_after();
             const int row = mb * BM + q * 32 + lane;
-            epilogue_tile<EPI>(tmem_base + acc * BN + ((uint32_t)(q * 32) << 16), row, nb * BN, p);
+            epilogue_tile<EPI, LORA>(tmem_base + acc * BN + ((uint32_t)(q * 32) << 16), row,
+                                     nb * BN, p);
             tc_fence_before();
             mbar_arrive(&tempty[acc]);
         }
@@ -385,17 +441,17 @@ int num_sms() {
     return n > 0 ? n : 1;
 }
 
-template <int EPI>
+template <int EPI, bool LORA = false>
 static cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const GemmParams& p,
                               int grid, cudaStream_t s) {
     static bool attr_done = false;  // per instantiation; idempotent if raced
     if (!attr_done) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             gemm::SMEM_BYTES);
+        cudaError_t e = cudaFuncSetAttribute(
+            k_gemm<EPI, LORA>, cudaFuncAttributeMaxDynamicSharedMemorySize, gemm::SMEM_BYTES);
         if (e != cudaSuccess) return e;
         attr_done = true;
     }
-    k_gemm<EPI><<<grid, 192, gemm::SMEM_BYTES, s>>>(ta, tb, p);
+    k_gemm<EPI, LORA><<<grid, 192, gemm::SMEM_BYTES, s>>>(ta, tb, p);
     return cudaGetLastError();
 }
 
@@ -421,6 +477,16 @@ jnx_status gemm_launch(const uint16_t* A, int lda, const uint16_t* B, int ldb, G
     if (tiles < grid) grid = tiles;
     if (p.group_m <= 0) p.group_m = 16;
     cudaError_t e;
+    if (p.lora_t) {
+        if (p.epi == EPI_ROPE)
+            e = launch_epi<EPI_ROPE, true>(ta, tb, p, grid, s);
+        else if (p.epi == EPI_RESID)
+            e = launch_epi<EPI_RESID, true>(ta, tb, p, grid, s);
+        else
+            return fail(JNX_ERR_UNSUPPORTED, "gemm: LoRA only with the RoPE or residual epilogue");
+        if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));
+        return JNX_OK;
+    }
     switch (p.epi) {
         case EPI_BF16: e = launch_epi<EPI_BF16>(ta, tb, p, grid, s); break;
         case EPI_F32: e = launch_epi<EPI_F32>(ta, tb, p, grid, s); break;

@@ -7,13 +7,22 @@
 
 namespace jnx {
 
-// One group slot: the tenant's head parameters and gradient buffers, and the
-// packed-sample range [s0, s1) of that tenant.
+// One group slot: the tenant's head parameters and gradient buffers, its
+// packed samples [s0, s1) and token rows [r0, r1).
 struct HeadSlot {
-    const uint16_t *w1, *b1, *w2, *b2;
-    float *g_w1, *g_b1, *g_w2, *g_b2;
+    int kind;        // JNX_HEAD_MLP or JNX_HEAD_XATTN
+    int tenant;
     int s0, s1;
-    int d_in, d_hidden, width, tenant;
+    int r0, r1;
+    int d_in;        // backbone width
+    int hid;         // input width of the output layer: MLP d_hidden, query head nq * dq
+    int width;       // outputs per sample
+    int nq, dq;      // query head
+    int pad_;
+    const uint16_t *w1, *b1;   // MLP first layer
+    const uint16_t *w2, *b2;   // output layer: MLP W2/b2 or query-head Wout/bout
+    const uint16_t *q, *wk, *wv;
+    float *g_w1, *g_b1, *g_w2, *g_b2, *g_q, *g_wk, *g_wv;
 };
 
 // Slots passed by value in kernel parameter space (up to kMaxSlots at once).
@@ -22,19 +31,33 @@ struct HeadTable {
     HeadSlot slot[kMaxSlots];
 };
 
-// Head activations kept in the workspace between forward and backward;
-// every array is [n_samples, ld] fp32 with ld >= max(d_hidden, width).
-struct HeadScratch {
-    float *z, *a, *y, *dy, *dz;
-    int ld;
+// What one launch batch of slots holds.
+struct HeadBatch {
+    int g0, n;                 // group slots [g0, g0 + n)
+    int sample0, sample1;      // their packed samples
+    int max_hid, max_mlp_hid, max_width, max_nq, max_dq;
+    bool any_mlp, any_xattn;
 };
 
-jnx_status mlp_heads_forward(const HeadTable& tab, int n, int max_hidden, int max_width,
-                             const float* pooled, int d, const int* sample_target,
-                             const float* targets, float* preds, float* loss, HeadScratch ws,
-                             cudaStream_t s);
-jnx_status mlp_heads_backward(const HeadTable& tab, int n, int max_hidden, int max_width,
-                              int max_din, const float* pooled, int d, HeadScratch ws,
-                              cudaStream_t s);
+// Head activations kept in the workspace between forward and backward.
+struct HeadScratch {
+    float *z, *h, *dh;   // [n_samples, ld_h]
+    float *y, *dy;       // [n_samples, ld_y]
+    int ld_h, ld_y;
+    // query heads
+    float *kbuf, *vbuf, *dk, *dv;  // [n_tokens, ldkv]
+    int ldkv;
+    float *P, *dS;                 // [nq * n_tokens], key-major per sample
+    float* dQs;                    // [n_samples, ld_h]
+};
+
+jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const HeadScratch& ws,
+                                const float* pooled, int d, const int* cu, const int* sample_slot,
+                                const int* sample_target, const float* targets, float* preds,
+                                float* loss, cudaStream_t s);
+jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const HeadScratch& ws,
+                                 const float* pooled, int d, const uint16_t* hidden,
+                                 const int* cu, const int* sample_slot, cudaStream_t s);
+jnx_status heads_set_smem();
 
 }  // namespace jnx

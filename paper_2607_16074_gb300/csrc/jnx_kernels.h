@@ -24,7 +24,33 @@ struct GemmParams {
     int act;              // EPI_GLU: JNX_GLU_*
     int group_m;          // tile-order group size (row blocks)
     int* status;          // device status word
+    // LoRA up-projection (EPI_ROPE / EPI_RESID): when lora_t is set, the
+    // epilogue adds t[row, p*r .. p*r+r) . B_p[tenant(row)][col', :] to each
+    // column of part p before its own op.  Parts are consecutive column
+    // ranges of lora_cols[p] columns; B_p is [n_tenants, lora_cols[p], r].
+    const float* lora_t;  // [M, ldt] fp32
+    int ldt;
+    const int* row_tenant;
+    const uint16_t* lora_b[3];
+    int lora_cols[3];
 };
+
+// LoRA: rank and the number of tenant segments one launch describes.
+constexpr int kLoraRank = 16;
+constexpr int kLoraMaxSlots = 256;
+struct LoraSlots {
+    int g0, n, sample0, pad_;
+    int tenant[kLoraMaxSlots];
+    int r0[kLoraMaxSlots], r1[kLoraMaxSlots], tile_start[kLoraMaxSlots];
+};
+struct LoraDown {
+    const uint16_t* a[3];  // per part: [n_tenants, r, K]
+};
+// row_tenant[r] for every packed row.
+jnx_status lora_row_tenant_launch(const jnx_group* g, int* row_tenant, cudaStream_t s);
+// t[row, :] = x[row, :] . [A_0 | .. | A_{n_parts-1}][tenant(row)]^T, fp32.
+jnx_status lora_down_launch(const jnx_group* g, const uint16_t* x, int ldx, int K, int n_parts,
+                            const uint16_t* const* a, float* t, int ldt, cudaStream_t s);
 
 // GEMM C = A . B^T with A [M, K] (row stride lda), B [N, K] (row stride ldb).
 jnx_status gemm_check(int M, int N, int K);

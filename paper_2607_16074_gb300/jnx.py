@@ -257,8 +257,8 @@ def jnx_group_plan(schemas: Sequence[dict], requests: Sequence[dict], n_tenants:
 # ---------------------------------------------------------------------------
 KERNEL_NAMES = {1: "pack", 2: "rmsnorm", 3: "gemm_qkv_rope", 4: "attention", 5: "gemm_o_resid",
                 6: "gemm_gate_up_glu", 7: "gemm_down_resid", 8: "final_norm_pool",
-                9: "rope_table", 10: "heads_fwd", 11: "heads_bwd", 12: "gemm"}
-TENSOR_KERNELS = (3, 4, 5, 6, 7, 12)
+                9: "rope_table", 10: "heads_fwd", 11: "heads_bwd", 12: "gemm", 13: "lora_down"}
+TENSOR_KERNELS = (3, 4, 5, 6, 7, 12, 13)
 
 
 def jnx_trace_enable(capacity: int) -> None:

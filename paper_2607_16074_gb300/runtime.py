@@ -66,10 +66,14 @@ class DeviceBackbone:
                                        w_gu.data_ptr(), s))
             ent = dict(attn_norm=lw["attn_norm"], w_qkv=w_qkv, w_o=lw["wo"],
                        ffn_norm=lw["ffn_norm"], w_gu=w_gu, w_down=lw["wd"])
+            names = ["attn_norm", "w_qkv", "w_o", "ffn_norm", "w_gu", "w_down"]
+            if cfg.lora_rank:
+                for p in ("q", "k", "v", "o"):
+                    ent["lora_a_" + p] = lw["lora_a_" + p].contiguous()
+                    ent["lora_b_" + p] = lw["lora_b_" + p].contiguous()
+                    names += ["lora_a_" + p, "lora_b_" + p]
             self.keep += list(ent.values())
-            self.layers[i] = J.jnx_layer(*[ent[k].data_ptr() for k in
-                                           ("attn_norm", "w_qkv", "w_o", "ffn_norm", "w_gu",
-                                            "w_down")])
+            self.layers[i] = J.jnx_layer(**{k: ent[k].data_ptr() for k in names})
         self.text_table = weights["text_table"]
         self.final_norm = weights["final_norm"]
         self.struct = J.jnx_backbone(cfg.n_layers, cfg.d, cfg.n_heads, cfg.n_kv_heads,
@@ -153,8 +157,9 @@ class GroupedStep:
         self.bb, self.heads, self.group = backbone, heads, group
         cfg = backbone.cfg
         S, N = group.plan.n_samples, group.plan.n_tokens
-        self.need_hidden = any(heads.arr[t].kind == J.JNX_HEAD_XATTN
-                               for t in group.plan.slot_tenant.tolist())
+        kinds = {heads.arr[t].kind for t in group.plan.slot_tenant.tolist()}
+        self.need_hidden = J.JNX_HEAD_XATTN in kinds
+        self.need_pooled = J.JNX_HEAD_MLP in kinds or not kinds
         self.pooled = torch.zeros((max(S, 1), cfg.d), dtype=torch.float32, device=device)
         self.hidden = (torch.zeros((max(N, 1), cfg.d), dtype=torch.bfloat16, device=device)
                        if self.need_hidden else None)
@@ -166,7 +171,7 @@ class GroupedStep:
 
     def run(self, vision, text_ids, targets, preds, stream=None) -> None:
         self.bb.forward(self.group, vision, text_ids,
-                        None if self.need_hidden else self.pooled, self.hidden, self.ws_bb, stream)
+                        self.pooled if self.need_pooled else None, self.hidden, self.ws_bb, stream)
         self.heads.forward(self.group, self.pooled, self.hidden, targets, preds, self.loss,
                            self.ws_h, stream)
         self.heads.backward(self.group, self.pooled, self.hidden, targets, self.ws_h, stream)
