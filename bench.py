@@ -49,6 +49,15 @@ def workload_desc(w):
             f"heads ({b.n_kv_heads} kv), FFN {b.d_ff} {'SwiGLU' if b.glu == 0 else 'GeGLU'}")
 
 
+def make_bench_workload(args):
+    import synth
+    over = {"n_layers": args.layers} if getattr(args, "layers", 0) else {}
+    w = synth.make_workload(args.workload, **over)
+    if getattr(args, "subset", 0):
+        w = w.subset(list(range(args.subset)))
+    return w
+
+
 def oracle_requests(w):
     return [dict(tenant=r.tenant, schema=r.schema,
                  samples=[dict(n_img=s.n_img, text_len=s.text_len, vision_row=s.vision_row,
@@ -156,7 +165,7 @@ def run_ours(args, rank, world, local_rank):
     J.lib()
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    w = synth.make_workload(args.workload)
+    w = make_bench_workload(args)
     # each rank owns an independent group (same shapes, its own inputs)
     w.seed = w.seed + 1000 * rank if rank else w.seed
     bw = synth.make_backbone_weights(w, device=dev)
@@ -467,6 +476,9 @@ def main():
                     help="time one kernel alone (gemm_gu, gemm_qkv, gemm_o, gemm_down, "
                          "attention, rmsnorm) on 7B-class shapes with --tokens rows")
     ap.add_argument("--tokens", type=int, default=8192)
+    ap.add_argument("--subset", type=int, default=0,
+                    help="keep only the first K tenants' requests (a smaller case for profilers)")
+    ap.add_argument("--layers", type=int, default=0, help="override the number of blocks")
     args = ap.parse_args()
     if args.kernel:
         print(json.dumps(run_kernel(args)), flush=True)

@@ -188,12 +188,22 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int n0,
         for (int c = 0; c < 8; ++c) {
             const int hchunk = c % (2 * hc);
             if (hchunk >= hc) continue;  // handled with its lower partner
+            const int col = n0 + c * 32;
+            const bool rot = valid && col < p.rope_cols;
+            // (cos, sin) of this row's position, 16-byte loads issued before
+            // the TMEM read so their latency overlaps it
+            float4 cs[16];
+            if (rot) {
+                const float4* src =
+                    reinterpret_cast<const float4*>(p.rope + (size_t)pos * half + hchunk * 32);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) cs[e] = __ldg(src + e);
+            }
             uint32_t lo[32], hi[32];
             tmem_ld32(tbase + c * 32, lo);
             tmem_ld32(tbase + (c + hc) * 32, hi);
             tmem_ld_wait();
             if (!valid) continue;
-            const int col = n0 + c * 32;
             float a[32], b[32];
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
@@ -204,14 +214,14 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int n0,
                 lora_chunk(a, row, tenant, col, p);
                 lora_chunk(b, row, tenant, col + half, p);
             }
-            if (col < p.rope_cols) {
-                const float2* cs = p.rope + (size_t)pos * half + hchunk * 32;
+            if (rot) {
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
-                    const float2 t = cs[e];
+                    const float cr = (e & 1) ? cs[e >> 1].z : cs[e >> 1].x;
+                    const float sr = (e & 1) ? cs[e >> 1].w : cs[e >> 1].y;
                     const float x0 = a[e], x1 = b[e];
-                    a[e] = x0 * t.x - x1 * t.y;
-                    b[e] = x1 * t.x + x0 * t.y;
+                    a[e] = x0 * cr - x1 * sr;
+                    b[e] = x1 * cr + x0 * sr;
                 }
             }
             bf16_t* base = static_cast<bf16_t*>(p.out) + (size_t)row * p.ldo;
@@ -369,13 +379,13 @@ __global__ void __launch_bounds__(192, 1)
             const uint32_t acc_phase = (local >> 1) & 1;
             int mb, nb;
             tile_coords(tile, num_m, num_n, p.group_m, mb, nb);
+            const int row = mb * BM + q * 32 + lane;
             if (!mbar_wait(&tfull[acc], acc_phase) || *abort_flag) {
                 *abort_flag = 1;
                 report(p.status, JNX_ERR_TIMEOUT);
                 break;
             }
             tc_fence_after();
-            const int row = mb * BM + q * 32 + lane;
             epilogue_tile<EPI, LORA>(tmem_base + acc * BN + ((uint32_t)(q * 32) << 16), row,
                                      nb * BN, p);
             tc_fence_before();
