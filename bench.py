@@ -425,8 +425,8 @@ def run_kernel(args):
     elif k == "attention":
         qkv = rnd(M, 3 * d)
         out = torch.empty(M, d, dtype=torch.bfloat16, device=dev)
-        call = lambda: L.jnx_op_attention(qkv.data_ptr(), H, H, hd, cu.data_ptr(), len(lens),
-                                          max(lens), out.data_ptr(), s.cuda_stream)
+        call = lambda: L.jnx_op_attention(qkv.data_ptr(), M, H, H, hd, cu.data_ptr(), len(lens),
+                                          max(lens), out.data_ptr(), None, s.cuda_stream)
         work, unit = sum(4.0 * l * l * H * hd for l in lens), "TFLOP/s"
     elif k == "rmsnorm":
         x = torch.randn(M, d, generator=g, device=dev)

@@ -52,10 +52,12 @@ jnx_status jnx_op_gemm(const uint16_t* A, const uint16_t* W, int32_t M, int32_t 
 /* Attention confined to each sample: for every sample s, head h,
  * out[t] = softmax(q_t K_s^T / sqrt(hd)) V_s over the sample's own tokens.
  * qkv [n_tokens, (H + 2 Hkv) hd] bf16 (q heads, then k heads, then v heads),
- * out [n_tokens, H hd] bf16; head_dim in {64, 128, 256}. */
-jnx_status jnx_op_attention(const uint16_t* qkv, int32_t n_heads, int32_t n_kv_heads,
-                            int32_t head_dim, const int32_t* cu_seqlens, int32_t n_samples,
-                            int32_t max_seqlen, uint16_t* out, void* stream);
+ * out [n_tokens, H hd] bf16; head_dim in {64, 128, 256}.  A wait that ran
+ * out of time writes JNX_ERR_TIMEOUT to *status (device int, may be NULL). */
+jnx_status jnx_op_attention(const uint16_t* qkv, int32_t n_tokens, int32_t n_heads,
+                            int32_t n_kv_heads, int32_t head_dim, const int32_t* cu_seqlens,
+                            int32_t n_samples, int32_t max_seqlen, uint16_t* out,
+                            int32_t* status, void* stream);
 
 /* Final RMSNorm and per-sample mean: pooled[s] = gamma * mean over the
  * sample's rows of x_t / sqrt(mean(x_t^2) + eps) (fp32), hidden[t] = bf16

@@ -210,8 +210,8 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
         }
         {
             TraceScope ts(JNX_K_ATTN, attn_flops, s);
-            if ((st = attention_launch(w.qkv, qkvw, H, Hkv, hd, g->cu_seqlens, g->n_samples,
-                                       g->max_seqlen, w.att, H * hd, s)))
+            if ((st = attention_launch(w.qkv, qkvw, N, H, Hkv, hd, g->cu_seqlens, g->n_samples,
+                                       g->max_seqlen, w.att, H * hd, w.status, s)))
                 return st;
         }
         p = GemmParams{};
@@ -661,16 +661,19 @@ extern "C" jnx_status jnx_op_gemm(const uint16_t* A, const uint16_t* W, int32_t 
     return gemm_launch(A, K, W, K, p, s);
 }
 
-extern "C" jnx_status jnx_op_attention(const uint16_t* qkv, int32_t n_heads, int32_t n_kv_heads,
-                                       int32_t head_dim, const int32_t* cu_seqlens,
-                                       int32_t n_samples, int32_t max_seqlen, uint16_t* out,
+extern "C" jnx_status jnx_op_attention(const uint16_t* qkv, int32_t n_tokens, int32_t n_heads,
+                                       int32_t n_kv_heads, int32_t head_dim,
+                                       const int32_t* cu_seqlens, int32_t n_samples,
+                                       int32_t max_seqlen, uint16_t* out, int32_t* status,
                                        void* stream) {
     clear_error();
-    if (!qkv || !out || (n_samples > 0 && !cu_seqlens))
+    if (!qkv || !out || (n_samples > 0 && !cu_seqlens) || n_tokens < 0)
         return fail(JNX_ERR_INVALID_ARG, "attention: null argument");
     const int ldq = (n_heads + 2 * n_kv_heads) * head_dim;
-    return attention_launch(qkv, ldq, n_heads, n_kv_heads, head_dim, cu_seqlens, n_samples,
-                            max_seqlen, out, n_heads * head_dim, static_cast<cudaStream_t>(stream));
+    TraceScope ts(JNX_K_ATTN, 0.0, static_cast<cudaStream_t>(stream));
+    return attention_launch(qkv, ldq, n_tokens, n_heads, n_kv_heads, head_dim, cu_seqlens,
+                            n_samples, max_seqlen, out, n_heads * head_dim, status,
+                            static_cast<cudaStream_t>(stream));
 }
 
 extern "C" jnx_status jnx_op_final_pool(const float* x, const uint16_t* gamma, float eps,

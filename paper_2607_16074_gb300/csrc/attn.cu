@@ -7,11 +7,15 @@
 // token, so a sample's result is the same wherever it sits in the packed
 // batch (grouped == isolated).
 //
-// Flash-style online softmax in fp32 with bf16 mma.sync (m16n8k16): each of
-// the 4 warps owns 16 query rows; K/V tiles stream through a double-buffered
-// cp.async ring in XOR-swizzled shared memory read with ldmatrix.  Q, K, V
-// come from the fused projection output [N, (H + 2 Hkv) hd]; query head h
-// reads K/V head h / (H / Hkv) (MQA when Hkv = 1).
+// Two kernels, chosen per head dim in attention_launch:
+//  k_attn     flash-style online softmax in fp32 with bf16 mma.sync
+//             (m16n8k16): each of the 4 warps owns 16 query rows; K/V tiles
+//             stream through a double-buffered cp.async ring in XOR-swizzled
+//             shared memory read with ldmatrix;
+//  k_attn_tc  the same algorithm on tcgen05: S and O accumulate in TMEM, Q/K/V
+//             arrive by TMA, P goes through shared memory (see below).
+// Q, K, V come from the fused projection output [N, (H + 2 Hkv) hd]; query
+// head h reads K/V head h / (H / Hkv) (MQA when Hkv = 1).
 #include "jnx_dev.cuh"
 #include "jnx_kernels.h"
 
@@ -197,6 +201,264 @@ __global__ void __launch_bounds__(128) k_attn(const uint16_t* __restrict__ qkv, 
     }
 }
 
+// ---------------------------------------------------------------------------
+// tcgen05 version.  One CTA = (sample, 128-query tile, head), 128 threads:
+// thread r owns query row r for the softmax and the epilogue; thread 0 also
+// issues the TMA copies and the MMAs.  Per key tile of BN keys:
+//   S = Q K^T          tcgen05.mma (M=128, N=BN, K=HD) into TMEM
+//   softmax            each thread reads its S row from TMEM twice (row max,
+//                      then p = 2^(s*scale*log2e - m)), rescales its O row in
+//                      TMEM when the running max moved, and writes p as bf16
+//                      into shared memory in the 128-byte-swizzled K-major
+//                      layout the next MMA reads
+//   O += P V           tcgen05.mma (M=128, N=HD, K=BN), V read MN-major
+// K/V tiles are double-buffered: the copy of tile kt+1 runs during tile kt.
+// The commit that follows S(kt) also covers PV(kt-1), so one barrier wait
+// tells the softmax threads that O, P and the older K/V buffer are free.
+// ---------------------------------------------------------------------------
+namespace attn_tc {
+constexpr int BM = 128;
+}
+
+template <int HD, int BN>
+struct AttnTcCfg {
+    // P rows are 128 bytes (64 keys) in the 128-byte-swizzled layout the PV
+    // MMA reads, so a key tile narrower than 64 would not fill its buffer.
+    static_assert(BN == 64 || BN == 128, "key tile must be 64 or 128 keys");
+    static_assert(HD % 64 == 0 && HD <= 256, "head dim must be 64, 128 or 256");
+    static constexpr int QB = attn_tc::BM * HD * 2;  // Q tile bytes
+    static constexpr int KB = BN * HD * 2;           // K (or V) tile bytes
+    static constexpr int PB = attn_tc::BM * BN * 2;  // P tile bytes
+    static constexpr int SMEM = QB + 4 * KB + PB + 1024 + 256;
+    static constexpr uint32_t O_COL = 128;           // TMEM column of the O accumulator
+    static constexpr uint32_t TCOLS = O_COL + HD <= 256 ? 256 : 512;  // TMEM columns held
+};
+
+template <int HD, int BN>
+__global__ void __launch_bounds__(128, 1)
+    k_attn_tc(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tkv,
+              const int* __restrict__ cu, int tiles_per_sample, int H, int Hkv, float scale_log2,
+              uint16_t* __restrict__ out, int ldo, int* status) {
+    using C = AttnTcCfg<HD, BN>;
+    constexpr int BM = attn_tc::BM;
+    constexpr int NCH = HD / 64;  // 64-column chunks of a head row
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint8_t* sQ = sm;
+    // K/V buffer b: K at QB + 2b KB, V right after it
+    auto sK = [&](int b) { return sm + C::QB + 2 * b * C::KB; };
+    auto sV = [&](int b) { return sm + C::QB + (2 * b + 1) * C::KB; };
+    uint8_t* sP = sm + C::QB + 4 * C::KB;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sP + C::PB);
+    uint64_t* q_full = bars;
+    uint64_t* kv_full = bars + 1;  // [2]
+    uint64_t* s_full = bars + 3;
+    uint64_t* pv_done = bars + 4;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 5);
+
+    const int s = blockIdx.x / tiles_per_sample;
+    const int qt = blockIdx.x % tiles_per_sample;
+    const int h = blockIdx.y;
+    const int kvh = h / (H / Hkv);
+    const int start = cu[s];
+    const int L = cu[s + 1] - start;
+    const int q0 = qt * BM;
+    if (q0 >= L) return;  // uniform for the whole CTA
+
+    const int tid = threadIdx.x, warp = tid >> 5;
+    if (tid == 0) {
+        mbar_init(q_full, 1);
+        mbar_init(&kv_full[0], 1);
+        mbar_init(&kv_full[1], 1);
+        mbar_init(s_full, 1);
+        mbar_init(pv_done, 1);
+        fence_barrier_init();
+        fence_proxy_async();
+    }
+    if (warp == 0) {
+        tmem_alloc(tmem_slot, C::TCOLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = *tmem_slot;
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    const uint32_t tS = tbase + lane_base;
+    const uint32_t tO = tbase + lane_base + C::O_COL;
+    const int n_kt = (L + BN - 1) / BN;
+    bool ok = true;
+
+    auto issue_kv = [&](int kt, int buf) {
+        mbar_arrive_expect_tx(&kv_full[buf], 2 * C::KB);
+        const int y = start + kt * BN;
+#pragma unroll
+        for (int c = 0; c < NCH; ++c) {
+            tma_load_2d(sK(buf) + c * BN * 128, &tkv, (H + kvh) * HD + c * 64, y, &kv_full[buf]);
+            tma_load_2d(sV(buf) + c * BN * 128, &tkv, (H + Hkv + kvh) * HD + c * 64, y,
+                        &kv_full[buf]);
+        }
+    };
+    if (tid == 0) {
+        mbar_arrive_expect_tx(q_full, C::QB);
+#pragma unroll
+        for (int c = 0; c < NCH; ++c)
+            tma_load_2d(sQ + c * BM * 128, &tq, h * HD + c * 64, start + q0, q_full);
+        issue_kv(0, 0);
+    }
+
+    constexpr uint32_t IDESC_S = idesc_bf16_f32(BM, BN);
+    constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, HD) | (1u << 16);  // B (V) MN-major
+    float m = -INFINITY, l = 0.f;
+
+    for (int kt = 0; kt < n_kt; ++kt) {
+        const int buf = kt & 1;
+        if (tid == 0) {
+            if (kt == 0) ok = ok && mbar_wait(q_full, 0);
+            ok = ok && mbar_wait(&kv_full[buf], (kt >> 1) & 1);
+            tc_fence_after();
+            const uint32_t qa = smem_u32(sQ), ka = smem_u32(sK(buf));
+#pragma unroll
+            for (int ks = 0; ks < HD / 16; ++ks)
+                tc_mma_f16(tS - lane_base, sw128_desc(qa + (ks >> 2) * BM * 128 + (ks & 3) * 32),
+                           sw128_desc(ka + (ks >> 2) * BN * 128 + (ks & 3) * 32), IDESC_S,
+                           ks > 0);
+            tc_commit(s_full);
+        }
+        __syncwarp();
+        ok = mbar_wait(s_full, kt & 1) && ok;
+        tc_fence_after();
+        if (tid == 0 && kt + 1 < n_kt) issue_kv(kt + 1, buf ^ 1);  // PV(kt-1) is done
+
+        // pass 1: row max over this tile's valid keys
+        const int kbase = kt * BN;
+        float mx = -INFINITY;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+            uint32_t r[32];
+            tmem_ld32(tS + c * 32, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 32; ++e)
+                if (kbase + c * 32 + e < L) mx = fmaxf(mx, __uint_as_float(r[e]) * scale_log2);
+        }
+        const float m_new = fmaxf(m, mx);
+        const float alpha = exp2f(m - m_new);
+        if (kt > 0 && __any_sync(0xffffffffu, alpha < 1.0f)) {
+#pragma unroll 1
+            for (int c = 0; c < HD / 32; ++c) {
+                uint32_t r[32];
+                tmem_ld32(tO + c * 32, r);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+                tmem_st32(tO + c * 32, r);
+            }
+            tmem_st_wait();
+        }
+        m = m_new;
+        // pass 2: p = 2^(s * scale - m) -> bf16 P in smem, row sum
+        float rs = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+            uint32_t r[32];
+            tmem_ld32(tS + c * 32, r);
+            tmem_ld_wait();
+            float p[32];
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+                p[e] = (kbase + c * 32 + e < L) ? exp2f(__uint_as_float(r[e]) * scale_log2 - m)
+                                                : 0.f;
+                rs += p[e];
+            }
+            // keys c*32 .. c*32+31 = 16-byte units 4(c%2) .. 4(c%2)+3 of chunk c/2
+            uint8_t* prow = sP + (c >> 1) * BM * 128 + tid * 128;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int unit = 4 * (c & 1) + u;
+                uint4 w;
+                w.x = pack_bf2(p[8 * u + 0], p[8 * u + 1]);
+                w.y = pack_bf2(p[8 * u + 2], p[8 * u + 3]);
+                w.z = pack_bf2(p[8 * u + 4], p[8 * u + 5]);
+                w.w = pack_bf2(p[8 * u + 6], p[8 * u + 7]);
+                *reinterpret_cast<uint4*>(prow + ((unit ^ (tid & 7)) << 4)) = w;
+            }
+        }
+        l = l * alpha + rs;
+        fence_proxy_async();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t pa = smem_u32(sP), va = smem_u32(sV(buf));
+#pragma unroll
+            for (int ks = 0; ks < BN / 16; ++ks)
+                tc_mma_f16(tO - lane_base,
+                           sw128_desc(pa + (ks >> 2) * BM * 128 + (ks & 3) * 32),
+                           sw128_desc_mn(va + ks * 16 * 128, BN * 128, 1024), IDESC_PV,
+                           (kt > 0 || ks > 0));
+            if (kt == n_kt - 1) tc_commit(pv_done);
+        }
+        __syncwarp();
+    }
+    ok = mbar_wait(pv_done, 0) && ok;
+    tc_fence_after();
+    if (!ok && tid == 0) report(status, JNX_ERR_TIMEOUT);
+
+    // epilogue: O / l -> bf16
+    const float inv = 1.0f / l;
+    const int row = q0 + tid;
+    uint16_t* orow = out + (size_t)(start + row) * ldo + h * HD;
+#pragma unroll 1
+    for (int c = 0; c < HD / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(tO + c * 32, r);
+        tmem_ld_wait();
+        if (row < L) {
+            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+                uint4 w;
+                w.x = pack_bf2(__uint_as_float(r[8 * v + 0]) * inv, __uint_as_float(r[8 * v + 1]) * inv);
+                w.y = pack_bf2(__uint_as_float(r[8 * v + 2]) * inv, __uint_as_float(r[8 * v + 3]) * inv);
+                w.z = pack_bf2(__uint_as_float(r[8 * v + 4]) * inv, __uint_as_float(r[8 * v + 5]) * inv);
+                w.w = pack_bf2(__uint_as_float(r[8 * v + 6]) * inv, __uint_as_float(r[8 * v + 7]) * inv);
+                dst[v] = w;
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tbase, C::TCOLS);
+}
+
+template <int HD, int BN>
+static jnx_status launch_attn_tc(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv,
+                                 const int* cu, int S, int max_seqlen, uint16_t* out, int ldo,
+                                 int* status, cudaStream_t s) {
+    using C = AttnTcCfg<HD, BN>;
+    static bool attr = false;
+    if (!attr) {
+        if (cudaFuncSetAttribute(k_attn_tc<HD, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 C::SMEM) != cudaSuccess)
+            return fail(JNX_ERR_CUDA, "attention: smem attribute");
+        attr = true;
+    }
+    CUtensorMap tq, tkv;
+    if (!make_tmap_bf16(&tq, qkv, n_tokens, ldq, ldq, attn_tc::BM, 64) ||
+        !make_tmap_bf16(&tkv, qkv, n_tokens, ldq, ldq, BN, 64))
+        return fail(JNX_ERR_CUDA, "attention: tensor map encode failed");
+    const int tps = (max_seqlen + attn_tc::BM - 1) / attn_tc::BM;
+    const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)HD));
+    dim3 grid(S * tps, H);
+    k_attn_tc<HD, BN><<<grid, 128, C::SMEM, s>>>(tq, tkv, cu, tps, H, Hkv, scale_log2, out, ldo,
+                                                 status);
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
+}
+
 template <int HD, int BN>
 static cudaError_t launch_attn(const uint16_t* qkv, int ldq, int H, int Hkv, const int* cu, int S,
                                int max_seqlen, uint16_t* out, int ldo, cudaStream_t s) {
@@ -215,20 +477,34 @@ static cudaError_t launch_attn(const uint16_t* qkv, int ldq, int H, int Hkv, con
     return cudaGetLastError();
 }
 
-jnx_status attention_launch(const uint16_t* qkv, int ldq, int H, int Hkv, int hd, const int* cu,
-                            int S, int max_seqlen, uint16_t* out, int ldo, cudaStream_t s) {
+jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv, int hd,
+                            const int* cu, int S, int max_seqlen, uint16_t* out, int ldo,
+                            int* status, cudaStream_t s) {
     if (S == 0 || max_seqlen == 0) return JNX_OK;
     if (Hkv <= 0 || H % Hkv) return fail(JNX_ERR_UNSUPPORTED, "attention: H %% Hkv != 0");
     if ((long long)S * ((max_seqlen + attn::BM - 1) / attn::BM) > 0x7FFFFFFFLL || H > 65535)
         return fail(JNX_ERR_UNSUPPORTED, "attention: grid too large");
-    cudaError_t e;
+    // Per head dim, the faster of the two kernels as measured on GB300 for
+    // prefixes of 260..840 tokens: the mma.sync kernel for 64 / 128 (181 /
+    // 224 TFLOP/s against 71 / 143 for this tcgen05 version, whose single
+    // 128-thread CTA per SM leaves the per-tile copy and softmax latencies
+    // exposed), the tcgen05 kernel for 256 (300 against 281).
+    cudaError_t e = cudaSuccess;
     switch (hd) {
-        case 64: e = launch_attn<64, 64>(qkv, ldq, H, Hkv, cu, S, max_seqlen, out, ldo, s); break;
-        case 128: e = launch_attn<128, 64>(qkv, ldq, H, Hkv, cu, S, max_seqlen, out, ldo, s); break;
-        case 256: e = launch_attn<256, 32>(qkv, ldq, H, Hkv, cu, S, max_seqlen, out, ldo, s); break;
-        default: return fail(JNX_ERR_UNSUPPORTED, "attention: head_dim %d not in {64,128,256}", hd);
+        case 64:
+            e = launch_attn<64, 64>(qkv, ldq, H, Hkv, cu, S, max_seqlen, out, ldo, s);
+            return e == cudaSuccess ? JNX_OK
+                                    : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
+        case 128:
+            e = launch_attn<128, 64>(qkv, ldq, H, Hkv, cu, S, max_seqlen, out, ldo, s);
+            return e == cudaSuccess ? JNX_OK
+                                    : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
+        case 256:
+            return launch_attn_tc<256, 64>(qkv, ldq, n_tokens, H, Hkv, cu, S, max_seqlen, out,
+                                           ldo, status, s);
+        default:
+            return fail(JNX_ERR_UNSUPPORTED, "attention: head_dim %d not in {64,128,256}", hd);
     }
-    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
 }
 
 }  // namespace jnx

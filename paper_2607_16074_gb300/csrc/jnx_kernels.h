@@ -77,7 +77,8 @@ jnx_status final_pool_launch(const float* x, const uint16_t* gamma, float eps, c
 jnx_status rope_table_launch(float2* tab, int max_pos, int hd, float theta, cudaStream_t s);
 
 // Varlen attention confined to each sample, bidirectional.
-jnx_status attention_launch(const uint16_t* qkv, int ldq, int H, int Hkv, int hd, const int* cu,
-                            int S, int max_seqlen, uint16_t* out, int ldo, cudaStream_t s);
+jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv, int hd,
+                            const int* cu, int S, int max_seqlen, uint16_t* out, int ldo,
+                            int* status, cudaStream_t s);
 
 }  // namespace jnx

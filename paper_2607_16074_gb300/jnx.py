@@ -143,7 +143,7 @@ def lib() -> C.CDLL:
         "jnx_op_gemm_workspace_bytes": (sz, [i32, i32]),
         "jnx_op_gemm": (i32, [vp, vp, i32, i32, i32, i32, vp, i32, vp, i32, i32, i32, f32, i32,
                               vp, sz, vp]),
-        "jnx_op_attention": (i32, [vp, i32, i32, i32, vp, i32, i32, vp, vp]),
+        "jnx_op_attention": (i32, [vp, i32, i32, i32, i32, vp, i32, i32, vp, vp, vp]),
         "jnx_op_final_pool": (i32, [vp, vp, f32, vp, i32, i32, vp, vp, vp]),
         "jnx_trace_enable": (i32, [i32]),
         "jnx_trace_disable": (i32, []),

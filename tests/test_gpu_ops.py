@@ -142,15 +142,18 @@ def _ragged_cu(lengths):
 
 @pytest.mark.parametrize("H,Hkv,hd", [(4, 4, 64), (2, 2, 128), (4, 1, 256), (4, 2, 128)])
 def test_attention_varlen(H, Hkv, hd):
-    lengths = [1, 17, 64, 65, 130, 200, 3]
+    # lengths straddle the 64- and 128-key tiles and the 128-query tile
+    lengths = [1, 17, 64, 65, 127, 128, 129, 200, 3, 300]
     cu = _ragged_cu(lengths)
     N = int(cu[-1])
     qkv = randn_bf16((N, (H + 2 * Hkv) * hd), 20 + hd, 1.0)
     out = torch.full((N, H * hd), 7.0, dtype=torch.bfloat16, device="cuda")
     cu_d = torch.tensor(cu).cuda()
-    J.check(J.lib().jnx_op_attention(qkv.data_ptr(), H, Hkv, hd, cu_d.data_ptr(), len(lengths),
-                                     max(lengths), out.data_ptr(), stream()))
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    J.check(J.lib().jnx_op_attention(qkv.data_ptr(), N, H, Hkv, hd, cu_d.data_ptr(), len(lengths),
+                                     max(lengths), out.data_ptr(), st.data_ptr(), stream()))
     torch.cuda.synchronize()
+    assert int(st.item()) == 0
     X = f64(qkv)
     for s in range(len(lengths)):
         a, b = cu[s], cu[s + 1]
@@ -170,8 +173,9 @@ def test_attention_sharp_logits():
     N = int(cu[-1])
     qkv = randn_bf16((N, (H + 2 * Hkv) * hd), 31, 3.0)
     out = torch.zeros((N, H * hd), dtype=torch.bfloat16, device="cuda")
-    J.check(J.lib().jnx_op_attention(qkv.data_ptr(), H, Hkv, hd, torch.tensor(cu).cuda().data_ptr(),
-                                     2, 150, out.data_ptr(), stream()))
+    J.check(J.lib().jnx_op_attention(qkv.data_ptr(), N, H, Hkv, hd,
+                                     torch.tensor(cu).cuda().data_ptr(), 2, 150, out.data_ptr(),
+                                     None, stream()))
     torch.cuda.synchronize()
     X = f64(qkv)
     for s in range(2):
