@@ -27,9 +27,8 @@ struct BackboneWs {
     uint16_t* att;    // [N, H hd] bf16
     uint16_t* u;      // [N, F] bf16
     float2* rope;     // [max_pos, hd / 2]
-    int* row_tenant;  // LoRA: tenant of each packed row [N]
-    float* t_qkv;     // LoRA: n1 [A_q | A_k | A_v]^T  [N, 3r]
-    float* t_o;       // LoRA: attention output A_o^T  [N, r]
+    uint16_t* t_qkv;  // LoRA: n1 [A_q | A_k | A_v]^T  [N, 3r] bf16
+    uint16_t* t_o;    // LoRA: attention output A_o^T  [N, r] bf16
     size_t bytes;
 };
 
@@ -53,9 +52,8 @@ BackboneWs carve_backbone(const jnx_backbone* bb, int64_t N, void* base) {
     w.u = reinterpret_cast<uint16_t*>(take((size_t)N * bb->d_ff * 2));
     w.rope = reinterpret_cast<float2*>(take((size_t)kMaxRopePos * (bb->head_dim / 2) * 8));
     if (bb->lora_rank) {
-        w.row_tenant = reinterpret_cast<int*>(take((size_t)N * 4));
-        w.t_qkv = reinterpret_cast<float*>(take((size_t)N * 3 * kLoraRank * 4));
-        w.t_o = reinterpret_cast<float*>(take((size_t)N * kLoraRank * 4));
+        w.t_qkv = reinterpret_cast<uint16_t*>(take((size_t)N * 3 * kLoraRank * 2));
+        w.t_o = reinterpret_cast<uint16_t*>(take((size_t)N * kLoraRank * 2));
     }
     w.bytes = off;
     return w;
@@ -157,9 +155,34 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
         TraceScope ts(JNX_K_ROPE_TABLE, (double)g->max_seqlen * hd * 4.0, s);
         if ((st = rope_table_launch(w.rope, g->max_seqlen, hd, bb->rope_theta, s))) return st;
     }
+    // LoRA: one segment per group tenant (its contiguous packed rows)
+    std::vector<int> seg_r0, seg_r1;
+    LoraSpec lq{}, lo{};
     if (lora) {
-        TraceScope ts(JNX_K_LORA, (double)N * 4.0, s);
-        if ((st = lora_row_tenant_launch(g, w.row_tenant, s))) return st;
+        if (g->n_slots > kLoraMaxSlots)
+            return fail(JNX_ERR_UNSUPPORTED, "backbone: LoRA groups hold at most %d tenants",
+                        kLoraMaxSlots);
+        for (int i = 0; i < g->n_slots; ++i) {
+            seg_r0.push_back(g->h_cu_seqlens[g->h_seg_offsets[i]]);
+            seg_r1.push_back(g->h_cu_seqlens[g->h_seg_offsets[i + 1]]);
+        }
+        lq.t = w.t_qkv;
+        lq.ldt = 3 * kLoraRank;
+        lq.n_parts = 3;
+        lq.cols[0] = H * hd;
+        lq.cols[1] = Hkv * hd;
+        lq.cols[2] = Hkv * hd;
+        lo.t = w.t_o;
+        lo.ldt = kLoraRank;
+        lo.n_parts = 1;
+        lo.cols[0] = d;
+        for (LoraSpec* ls : {&lq, &lo}) {
+            ls->n_tenants = bb->n_tenants;
+            ls->n_seg = g->n_slots;
+            ls->seg_r0 = seg_r0.data();
+            ls->seg_r1 = seg_r1.data();
+            ls->seg_tenant = g->h_slot_tenant;
+        }
     }
     // within-sample attention FLOPs: QK^T and PV over each sample's own tokens
     double attn_flops = 0.0;
@@ -194,17 +217,12 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
                 if ((st = lora_down_launch(g, w.nrm, d, d, 3, a3, w.t_qkv, 3 * kLoraRank, s)))
                     return st;
             }
-            p.lora_t = w.t_qkv;
-            p.ldt = 3 * kLoraRank;
-            p.row_tenant = w.row_tenant;
-            p.lora_b[0] = L.lora_b_q;
-            p.lora_b[1] = L.lora_b_k;
-            p.lora_b[2] = L.lora_b_v;
-            p.lora_cols[0] = H * hd;
-            p.lora_cols[1] = Hkv * hd;
-            p.lora_cols[2] = Hkv * hd;
-        }
-        {
+            lq.b[0] = L.lora_b_q;
+            lq.b[1] = L.lora_b_k;
+            lq.b[2] = L.lora_b_v;
+            TraceScope ts(JNX_K_GEMM_QKV, 2.0 * N * qkvw * d, s);
+            if ((st = gemm_launch_lora(w.nrm, d, L.w_qkv, d, p, lq, s))) return st;
+        } else {
             TraceScope ts(JNX_K_GEMM_QKV, 2.0 * N * qkvw * d, s);
             if ((st = gemm_launch(w.nrm, d, L.w_qkv, d, p, s))) return st;
         }
@@ -229,13 +247,10 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
                 if ((st = lora_down_launch(g, w.att, H * hd, H * hd, 1, a1, w.t_o, kLoraRank, s)))
                     return st;
             }
-            p.lora_t = w.t_o;
-            p.ldt = kLoraRank;
-            p.row_tenant = w.row_tenant;
-            p.lora_b[0] = L.lora_b_o;
-            p.lora_cols[0] = d;
-        }
-        {
+            lo.b[0] = L.lora_b_o;
+            TraceScope ts(JNX_K_GEMM_O, 2.0 * N * d * H * hd, s);
+            if ((st = gemm_launch_lora(w.att, H * hd, L.w_o, H * hd, p, lo, s))) return st;
+        } else {
             TraceScope ts(JNX_K_GEMM_O, 2.0 * N * d * H * hd, s);
             if ((st = gemm_launch(w.att, H * hd, L.w_o, H * hd, p, s))) return st;
         }

@@ -24,6 +24,7 @@
 // or where the row sits, so packed (grouped) and per-tenant runs agree
 // bit for bit.
 #include <mutex>
+#include <type_traits>
 
 #include "jnx_dev.cuh"
 #include "jnx_kernels.h"
@@ -38,7 +39,34 @@ constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 512;  // two 256-column fp32 accumulators
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
 constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
+// LoRA operands of one tile (K = 16, 32-byte rows): t rows and B rows, a
+// 2-deep ring after the main stages.
+constexpr int LT_BYTES = BM * 16 * 2;
+constexpr int LB_BYTES = BN * 16 * 2;
+constexpr int LSTAGE = LT_BYTES + LB_BYTES;
+constexpr int SMEM_BYTES_LORA = SMEM_BYTES + 2 * LSTAGE;
 }  // namespace gemm
+
+// Descriptor of a K-major bf16 tile with 32-byte rows (K = 16) stored with
+// the 32-byte swizzle: 8-row atoms of 256 bytes.
+__device__ __forceinline__ uint64_t sw32_desc(uint32_t smem_addr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((smem_addr & 0x3FFFF) >> 4);
+    d |= (uint64_t)1 << 16;              // leading byte offset (unused: K fits one row)
+    d |= (uint64_t)(256 >> 4) << 32;     // stride byte offset: next 8-row atom
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)6 << 61;              // layout: 32-byte swizzle
+    return d;
+}
+
+struct NoLora {};
+
+// Rows [row0, row_end) and column block nb of one output tile.  Without
+// LoRA, tiles are plain 128-row blocks of M; with LoRA they are laid out per
+// tenant segment so every tile belongs to one tenant (`seg`).
+struct TileGeo {
+    int row0, row_end, nb, seg;
+};
 
 // Tile order: groups of `group_m` row-blocks, N fastest inside a group, so
 // the CTAs resident at one time share a few A row-blocks and a band of B.
@@ -59,53 +87,10 @@ __device__ __forceinline__ float act_fn(float g, int act) {
     return 0.5f * g * (1.0f + tanhf(c * (g + 0.044715f * g * g * g)));
 }
 
-// LoRA up-projection for 32 consecutive columns [col, col + 32) of one row:
-// v[e] += t[row, part r..] . B_part[tenant][col + e - part start, :].  The
-// 32 columns never straddle two parts (part widths are multiples of 64).
-__device__ __forceinline__ void lora_chunk(float (&v)[32], int row, int tenant, int col,
-                                           const GemmParams& p) {
-    constexpr int R = kLoraRank;
-    int part = 0, c = col;
-    while (part < 2 && c >= p.lora_cols[part]) {
-        c -= p.lora_cols[part];
-        ++part;
-    }
-    const float4* tr = reinterpret_cast<const float4*>(p.lora_t + (size_t)row * p.ldt + part * R);
-    float t[R];
-#pragma unroll
-    for (int i = 0; i < R / 4; ++i) {
-        const float4 q = tr[i];
-        t[4 * i] = q.x;
-        t[4 * i + 1] = q.y;
-        t[4 * i + 2] = q.z;
-        t[4 * i + 3] = q.w;
-    }
-    const uint4* b = reinterpret_cast<const uint4*>(
-        p.lora_b[part] + ((size_t)tenant * p.lora_cols[part] + c) * R);
-#pragma unroll
-    for (int e = 0; e < 32; ++e) {
-        float acc = 0.f;
-#pragma unroll
-        for (int h = 0; h < R / 8; ++h) {
-            const uint4 w = __ldg(b + (R / 8) * e + h);
-            acc += t[8 * h + 0] * __uint_as_float(w.x << 16) +
-                   t[8 * h + 1] * __uint_as_float(w.x & 0xFFFF0000u) +
-                   t[8 * h + 2] * __uint_as_float(w.y << 16) +
-                   t[8 * h + 3] * __uint_as_float(w.y & 0xFFFF0000u) +
-                   t[8 * h + 4] * __uint_as_float(w.z << 16) +
-                   t[8 * h + 5] * __uint_as_float(w.z & 0xFFFF0000u) +
-                   t[8 * h + 6] * __uint_as_float(w.w << 16) +
-                   t[8 * h + 7] * __uint_as_float(w.w & 0xFFFF0000u);
-        }
-        v[e] += acc;
-    }
-}
-
-template <int EPI, bool LORA>
-__device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int n0,
+template <int EPI>
+__device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int row_end, int n0,
                                               const GemmParams& p) {
-    const bool valid = row < p.M;
-    const int tenant = (LORA && valid) ? p.row_tenant[row] : 0;
+    const bool valid = row < row_end;
     if constexpr (EPI == EPI_BF16 || EPI == EPI_F32 || EPI == EPI_RESID) {
 #pragma unroll 1
         for (int c = 0; c < 8; ++c) {
@@ -114,14 +99,6 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int n0,
             tmem_ld_wait();
             if (!valid) continue;
             const int col = n0 + c * 32;
-            if constexpr (LORA) {
-                float f[32];
-#pragma unroll
-                for (int e = 0; e < 32; ++e) f[e] = __uint_as_float(r[e]);
-                lora_chunk(f, row, tenant, col, p);
-#pragma unroll
-                for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(f[e]);
-            }
             if constexpr (EPI == EPI_BF16) {
                 uint4* dst = reinterpret_cast<uint4*>(static_cast<bf16_t*>(p.out) +
                                                       (size_t)row * p.ldo + col);
@@ -210,10 +187,6 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int n0,
                 a[e] = __uint_as_float(lo[e]);
                 b[e] = __uint_as_float(hi[e]);
             }
-            if constexpr (LORA) {
-                lora_chunk(a, row, tenant, col, p);
-                lora_chunk(b, row, tenant, col + half, p);
-            }
             if (rot) {
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
@@ -245,22 +218,59 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int n0,
     }
 }
 
+template <bool LORA, class LG>
+__device__ __forceinline__ TileGeo tile_geo(int tile, int num_m, int num_n, const GemmParams& p,
+                                            const LG& lg) {
+    int mb, nb;
+    tile_coords(tile, num_m, num_n, p.group_m, mb, nb);
+    TileGeo g;
+    g.nb = nb;
+    if constexpr (LORA) {
+        int sg = 0;
+        while (sg + 1 < lg.n_seg && lg.seg_tile0[sg + 1] <= mb) ++sg;
+        g.seg = sg;
+        g.row0 = lg.seg_r0[sg] + (mb - lg.seg_tile0[sg]) * gemm::BM;
+        g.row_end = min(g.row0 + gemm::BM, lg.seg_r1[sg]);
+    } else {
+        g.seg = 0;
+        g.row0 = mb * gemm::BM;
+        g.row_end = min(g.row0 + gemm::BM, p.M);
+    }
+    return g;
+}
+
+// The LoRA part holding column block nb, and the block's first column in it.
+__device__ __forceinline__ void lora_part(const LoraGemm& lg, int nb, int& part, int& c0) {
+    int c = nb * gemm::BN;
+    part = 0;
+    while (part + 1 < lg.n_parts && c >= lg.part_cols[part]) {
+        c -= lg.part_cols[part];
+        ++part;
+    }
+    c0 = c;
+}
+
 template <int EPI, bool LORA>
 __global__ void __launch_bounds__(192, 1)
     k_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
+           const __grid_constant__ typename std::conditional<LORA, LoraGemm, NoLora>::type lg,
            GemmParams p) {
     using namespace gemm;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+    uint8_t* lsm = smem + STAGES * STAGE_BYTES;  // LoRA ring (LORA only)
+    uint64_t* full = reinterpret_cast<uint64_t*>(lsm + (LORA ? 2 * LSTAGE : 0));
     uint64_t* empty = full + STAGES;
     uint64_t* tfull = empty + STAGES;
     uint64_t* tempty = tfull + 2;
     uint64_t* drain = tempty + 2;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    uint64_t* lfull = drain + 1;   // [2]
+    uint64_t* lempty = lfull + 2;  // [2]
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(lempty + 2);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     volatile int* consumed = abort_flag + 1;
+    volatile int* lconsumed = abort_flag + 2;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -273,10 +283,13 @@ __global__ void __launch_bounds__(192, 1)
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
             mbar_init(&tempty[a], 128);
+            mbar_init(&lfull[a], 1);
+            mbar_init(&lempty[a], 1);
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
         *consumed = 0;
+        *lconsumed = 0;
         fence_barrier_init();
         fence_proxy_async();
     }
@@ -293,19 +306,24 @@ __global__ void __launch_bounds__(192, 1)
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
-    const int num_m = (p.M + BM - 1) / BM;
+    int num_m;
+    if constexpr (LORA)
+        num_m = lg.seg_tile0[lg.n_seg];
+    else
+        num_m = (p.M + BM - 1) / BM;
     const int num_n = p.N / BN;
     const int num_k = p.K / BK;
     const int num_tiles = num_m * num_n;
-    int issued = 0;
+    int issued = 0, l_issued = 0;
 
     if (warp == 0) {
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
+            int lj = 0;
+            uint32_t lphase = 0;
             for (int tile = blockIdx.x; tile < num_tiles && !*abort_flag; tile += gridDim.x) {
-                int mb, nb;
-                tile_coords(tile, num_m, num_n, p.group_m, mb, nb);
+                const TileGeo g = tile_geo<LORA>(tile, num_m, num_n, p, lg);
                 for (int kb = 0; kb < num_k; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1)) {
                         *abort_flag = 1;
@@ -314,12 +332,33 @@ __global__ void __launch_bounds__(192, 1)
                     }
                     mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
                     uint8_t* sa = smem + stage * STAGE_BYTES;
-                    tma_load_2d(sa, &ta, kb * BK, mb * BM, &full[stage]);
-                    tma_load_2d(sa + A_BYTES, &tb, kb * BK, nb * BN, &full[stage]);
+                    tma_load_2d(sa, &ta, kb * BK, g.row0, &full[stage]);
+                    tma_load_2d(sa + A_BYTES, &tb, kb * BK, g.nb * BN, &full[stage]);
                     ++issued;
                     if (++stage == STAGES) {
                         stage = 0;
                         phase ^= 1;
+                    }
+                }
+                if constexpr (LORA) {
+                    if (*abort_flag) break;
+                    // this tile's t rows (its part) and its tenant's B rows
+                    if (!mbar_wait(&lempty[lj], lphase ^ 1)) {
+                        *abort_flag = 1;
+                        report(p.status, JNX_ERR_TIMEOUT);
+                        break;
+                    }
+                    int part, c0;
+                    lora_part(lg, g.nb, part, c0);
+                    uint8_t* lt = lsm + lj * LSTAGE;
+                    mbar_arrive_expect_tx(&lfull[lj], LSTAGE);
+                    tma_load_2d(lt, &lg.tt, part * 16, g.row0, &lfull[lj]);
+                    tma_load_2d(lt + LT_BYTES, &lg.tb[part], 0,
+                                lg.seg_tenant[g.seg] * lg.part_cols[part] + c0, &lfull[lj]);
+                    ++l_issued;
+                    if (++lj == 2) {
+                        lj = 0;
+                        lphase ^= 1;
                     }
                 }
             }
@@ -329,6 +368,8 @@ __global__ void __launch_bounds__(192, 1)
             int stage = 0;
             uint32_t phase = 0;
             int local = 0;
+            int lj = 0;
+            uint32_t lphase = 0;
             for (int tile = blockIdx.x; tile < num_tiles && !*abort_flag;
                  tile += gridDim.x, ++local) {
                 const int acc = local & 1;
@@ -360,6 +401,21 @@ __global__ void __launch_bounds__(192, 1)
                         phase ^= 1;
                     }
                 }
+                if constexpr (LORA) {
+                    // D += t[rows, part] . B_part[tenant][cols]^T (one K = 16 step)
+                    if (ok && !mbar_wait(&lfull[lj], lphase)) ok = false;
+                    if (ok) {
+                        *lconsumed = *lconsumed + 1;
+                        tc_fence_after();
+                        const uint32_t la = smem_u32(lsm + lj * LSTAGE);
+                        tc_mma_f16(d, sw32_desc(la), sw32_desc(la + LT_BYTES), IDESC, 1);
+                        tc_commit(&lempty[lj]);
+                        if (++lj == 2) {
+                            lj = 0;
+                            lphase ^= 1;
+                        }
+                    }
+                }
                 if (!ok) {
                     *abort_flag = 1;
                     report(p.status, JNX_ERR_TIMEOUT);
@@ -377,17 +433,16 @@ __global__ void __launch_bounds__(192, 1)
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
             const int acc = local & 1;
             const uint32_t acc_phase = (local >> 1) & 1;
-            int mb, nb;
-            tile_coords(tile, num_m, num_n, p.group_m, mb, nb);
-            const int row = mb * BM + q * 32 + lane;
+            const TileGeo g = tile_geo<LORA>(tile, num_m, num_n, p, lg);
+            const int row = g.row0 + q * 32 + lane;
             if (!mbar_wait(&tfull[acc], acc_phase) || *abort_flag) {
                 *abort_flag = 1;
                 report(p.status, JNX_ERR_TIMEOUT);
                 break;
             }
             tc_fence_after();
-            epilogue_tile<EPI, LORA>(tmem_base + acc * BN + ((uint32_t)(q * 32) << 16), row,
-                                     nb * BN, p);
+            epilogue_tile<EPI>(tmem_base + acc * BN + ((uint32_t)(q * 32) << 16), row, g.row_end,
+                               g.nb * BN, p);
             tc_fence_before();
             mbar_arrive(&tempty[acc]);
         }
@@ -400,6 +455,8 @@ __global__ void __launch_bounds__(192, 1)
         // wait (bounded) for TMA copies this CTA issued but nobody consumed
         for (int i = *consumed; i < issued; ++i)
             mbar_wait(&full[i % STAGES], (i / STAGES) & 1, 100000000LL);
+        for (int i = *lconsumed; i < l_issued; ++i)
+            mbar_wait(&lfull[i & 1], (i >> 1) & 1, 100000000LL);
     }
     __syncwarp();
     if (warp == 1) tmem_dealloc(tmem_base, TMEM_COLS);
@@ -430,17 +487,21 @@ static PFN_tmapEncodeTiled encode_fn() {
 }
 
 bool make_tmap_bf16(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols,
-                    uint64_t row_stride_elems, uint32_t box_rows, uint32_t box_cols) {
+                    uint64_t row_stride_elems, uint32_t box_rows, uint32_t box_cols,
+                    int swizzle_bytes) {
     PFN_tmapEncodeTiled fn = encode_fn();
     if (!fn) return false;
     if ((reinterpret_cast<uintptr_t>(ptr) & 15) || ((row_stride_elems * 2) & 15)) return false;
+    if (box_cols * 2 > (uint32_t)swizzle_bytes) return false;  // a box row within one swizzle span
     cuuint64_t dims[2] = {cols, rows};
     cuuint64_t strides[1] = {row_stride_elems * 2};
     cuuint32_t box[2] = {box_cols, box_rows};
     cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle sw = swizzle_bytes == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                                  : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                        : CU_TENSOR_MAP_SWIZZLE_32B;
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
-              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-              CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -451,17 +512,18 @@ int num_sms() {
     return n > 0 ? n : 1;
 }
 
-template <int EPI, bool LORA = false>
-static cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const GemmParams& p,
-                              int grid, cudaStream_t s) {
+template <int EPI, bool LORA, class LG>
+static cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const LG& lg,
+                              const GemmParams& p, int grid, cudaStream_t s) {
+    constexpr int smem = LORA ? gemm::SMEM_BYTES_LORA : gemm::SMEM_BYTES;
     static bool attr_done = false;  // per instantiation; idempotent if raced
     if (!attr_done) {
-        cudaError_t e = cudaFuncSetAttribute(
-            k_gemm<EPI, LORA>, cudaFuncAttributeMaxDynamicSharedMemorySize, gemm::SMEM_BYTES);
+        cudaError_t e = cudaFuncSetAttribute(k_gemm<EPI, LORA>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         attr_done = true;
     }
-    k_gemm<EPI, LORA><<<grid, 192, gemm::SMEM_BYTES, s>>>(ta, tb, p);
+    k_gemm<EPI, LORA><<<grid, 192, smem, s>>>(ta, tb, lg, p);
     return cudaGetLastError();
 }
 
@@ -487,24 +549,69 @@ jnx_status gemm_launch(const uint16_t* A, int lda, const uint16_t* B, int ldb, G
     if (tiles < grid) grid = tiles;
     if (p.group_m <= 0) p.group_m = 16;
     cudaError_t e;
-    if (p.lora_t) {
-        if (p.epi == EPI_ROPE)
-            e = launch_epi<EPI_ROPE, true>(ta, tb, p, grid, s);
-        else if (p.epi == EPI_RESID)
-            e = launch_epi<EPI_RESID, true>(ta, tb, p, grid, s);
-        else
-            return fail(JNX_ERR_UNSUPPORTED, "gemm: LoRA only with the RoPE or residual epilogue");
-        if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));
-        return JNX_OK;
-    }
+    const NoLora none{};
     switch (p.epi) {
-        case EPI_BF16: e = launch_epi<EPI_BF16>(ta, tb, p, grid, s); break;
-        case EPI_F32: e = launch_epi<EPI_F32>(ta, tb, p, grid, s); break;
-        case EPI_RESID: e = launch_epi<EPI_RESID>(ta, tb, p, grid, s); break;
-        case EPI_GLU: e = launch_epi<EPI_GLU>(ta, tb, p, grid, s); break;
-        case EPI_ROPE: e = launch_epi<EPI_ROPE>(ta, tb, p, grid, s); break;
+        case EPI_BF16: e = launch_epi<EPI_BF16, false>(ta, tb, none, p, grid, s); break;
+        case EPI_F32: e = launch_epi<EPI_F32, false>(ta, tb, none, p, grid, s); break;
+        case EPI_RESID: e = launch_epi<EPI_RESID, false>(ta, tb, none, p, grid, s); break;
+        case EPI_GLU: e = launch_epi<EPI_GLU, false>(ta, tb, none, p, grid, s); break;
+        case EPI_ROPE: e = launch_epi<EPI_ROPE, false>(ta, tb, none, p, grid, s); break;
         default: return fail(JNX_ERR_INVALID_ARG, "gemm: unknown epilogue %d", p.epi);
     }
+    if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));
+    return JNX_OK;
+}
+
+jnx_status gemm_launch_lora(const uint16_t* A, int lda, const uint16_t* B, int ldb, GemmParams p,
+                            const LoraSpec& ls, cudaStream_t s) {
+    jnx_status st = gemm_check(p.M, p.N, p.K);
+    if (st != JNX_OK) return st;
+    if (p.epi != EPI_ROPE && p.epi != EPI_RESID)
+        return fail(JNX_ERR_UNSUPPORTED, "gemm: LoRA only with the RoPE or residual epilogue");
+    if (ls.n_seg < 0 || ls.n_seg > kLoraMaxSlots || ls.n_parts < 1 || ls.n_parts > 3 ||
+        (ls.ldt * 2) % 16 || ls.ldt < 16 * ls.n_parts)
+        return fail(JNX_ERR_UNSUPPORTED, "gemm: bad LoRA description");
+    int cols = 0;
+    for (int i = 0; i < ls.n_parts; ++i) {
+        if (ls.cols[i] <= 0 || ls.cols[i] % gemm::BN)
+            return fail(JNX_ERR_UNSUPPORTED, "gemm: LoRA part widths must be multiples of 256");
+        cols += ls.cols[i];
+    }
+    if (cols != p.N) return fail(JNX_ERR_INVALID_ARG, "gemm: LoRA parts do not cover N");
+    if (p.M == 0 || ls.n_seg == 0) return JNX_OK;
+    static thread_local LoraGemm lg;  // staging of the kernel argument (copied at launch)
+    lg = LoraGemm{};
+    lg.n_parts = ls.n_parts;
+    lg.n_seg = ls.n_seg;
+    int tiles = 0;
+    for (int i = 0; i < ls.n_seg; ++i) {
+        if (ls.seg_r0[i] < 0 || ls.seg_r1[i] < ls.seg_r0[i] || ls.seg_r1[i] > p.M ||
+            ls.seg_tenant[i] < 0 || ls.seg_tenant[i] >= ls.n_tenants)
+            return fail(JNX_ERR_INVALID_ARG, "gemm: bad LoRA segment %d", i);
+        lg.seg_r0[i] = ls.seg_r0[i];
+        lg.seg_r1[i] = ls.seg_r1[i];
+        lg.seg_tenant[i] = ls.seg_tenant[i];
+        lg.seg_tile0[i] = tiles;
+        tiles += (ls.seg_r1[i] - ls.seg_r0[i] + gemm::BM - 1) / gemm::BM;
+    }
+    lg.seg_tile0[ls.n_seg] = tiles;
+    CUtensorMap ta, tb;
+    bool ok = make_tmap_bf16(&ta, A, p.M, p.K, lda, gemm::BM, gemm::BK) &&
+              make_tmap_bf16(&tb, B, p.N, p.K, ldb, gemm::BN, gemm::BK) &&
+              make_tmap_bf16(&lg.tt, ls.t, p.M, ls.ldt, ls.ldt, gemm::BM, 16, 32);
+    for (int i = 0; i < ls.n_parts && ok; ++i) {
+        lg.part_cols[i] = ls.cols[i];
+        ok = make_tmap_bf16(&lg.tb[i], ls.b[i], (uint64_t)ls.n_tenants * ls.cols[i], kLoraRank,
+                            kLoraRank, gemm::BN, 16, 32);
+    }
+    if (!ok) return fail(JNX_ERR_CUDA, "gemm: LoRA tensor map encode failed");
+    const int total = tiles * (p.N / gemm::BN);
+    if (total == 0) return JNX_OK;
+    int grid = num_sms();
+    if (total < grid) grid = total;
+    if (p.group_m <= 0) p.group_m = 16;
+    cudaError_t e = p.epi == EPI_ROPE ? launch_epi<EPI_ROPE, true>(ta, tb, lg, p, grid, s)
+                                      : launch_epi<EPI_RESID, true>(ta, tb, lg, p, grid, s);
     if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));
     return JNX_OK;
 }

@@ -24,20 +24,42 @@ struct GemmParams {
     int act;              // EPI_GLU: JNX_GLU_*
     int group_m;          // tile-order group size (row blocks)
     int* status;          // device status word
-    // LoRA up-projection (EPI_ROPE / EPI_RESID): when lora_t is set, the
-    // epilogue adds t[row, p*r .. p*r+r) . B_p[tenant(row)][col', :] to each
-    // column of part p before its own op.  Parts are consecutive column
-    // ranges of lora_cols[p] columns; B_p is [n_tenants, lora_cols[p], r].
-    const float* lora_t;  // [M, ldt] fp32
-    int ldt;
-    const int* row_tenant;
-    const uint16_t* lora_b[3];
-    int lora_cols[3];
 };
 
 // LoRA: rank and the number of tenant segments one launch describes.
 constexpr int kLoraRank = 16;
 constexpr int kLoraMaxSlots = 256;
+
+// Per-tenant LoRA up-projection done on the tensor core inside a projection
+// GEMM (EPI_ROPE or EPI_RESID): the GEMM's 128-row tiles are laid out per
+// tenant segment (a tile never holds two tenants), and after the K loop of a
+// tile one more K = 16 MMA adds t[rows, part] . B_part[tenant][cols]^T, where
+// the tile's 256 output columns lie in one part (Q, K or V for the fused
+// projection, the single part for O).
+struct LoraGemm {
+    CUtensorMap tt;          // t [M, ldt] bf16, box 16 x 128, 32-byte swizzle
+    CUtensorMap tb[3];       // B_p viewed as [n_tenants * cols_p, 16], box 16 x 256
+    int part_cols[3];        // output columns of each part (multiples of 256)
+    int n_parts, n_seg;
+    int seg_r0[kLoraMaxSlots], seg_r1[kLoraMaxSlots], seg_tenant[kLoraMaxSlots];
+    int seg_tile0[kLoraMaxSlots + 1];  // first 128-row tile of each segment
+};
+
+// Host description of a LoRA up-projection for gemm_launch_lora.
+struct LoraSpec {
+    const uint16_t* t;       // [M, ldt] bf16 down-projected rows
+    int ldt;
+    const uint16_t* b[3];    // per part: [n_tenants, cols_p, r] bf16
+    int cols[3];
+    int n_parts, n_tenants;
+    int n_seg;
+    const int* seg_r0;       // host arrays [n_seg]: token rows of each tenant segment
+    const int* seg_r1;
+    const int* seg_tenant;
+};
+
+jnx_status gemm_launch_lora(const uint16_t* A, int lda, const uint16_t* B, int ldb, GemmParams p,
+                            const LoraSpec& ls, cudaStream_t s);
 struct LoraSlots {
     int g0, n, sample0, pad_;
     int tenant[kLoraMaxSlots];
@@ -46,18 +68,17 @@ struct LoraSlots {
 struct LoraDown {
     const uint16_t* a[3];  // per part: [n_tenants, r, K]
 };
-// row_tenant[r] for every packed row.
-jnx_status lora_row_tenant_launch(const jnx_group* g, int* row_tenant, cudaStream_t s);
-// t[row, :] = x[row, :] . [A_0 | .. | A_{n_parts-1}][tenant(row)]^T, fp32.
+// t[row, :] = bf16(x[row, :] . [A_0 | .. | A_{n_parts-1}][tenant(row)]^T).
 jnx_status lora_down_launch(const jnx_group* g, const uint16_t* x, int ldx, int K, int n_parts,
-                            const uint16_t* const* a, float* t, int ldt, cudaStream_t s);
+                            const uint16_t* const* a, uint16_t* t, int ldt, cudaStream_t s);
 
 // GEMM C = A . B^T with A [M, K] (row stride lda), B [N, K] (row stride ldb).
 jnx_status gemm_check(int M, int N, int K);
 jnx_status gemm_launch(const uint16_t* A, int lda, const uint16_t* B, int ldb, GemmParams p,
                        cudaStream_t s, int max_ctas = 0);
 bool make_tmap_bf16(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols,
-                    uint64_t row_stride_elems, uint32_t box_rows, uint32_t box_cols);
+                    uint64_t row_stride_elems, uint32_t box_rows, uint32_t box_cols,
+                    int swizzle_bytes = 128);
 int num_sms();
 
 // Packer: x[N, d] fp32 = widened gather of vision rows / text-embedding rows.

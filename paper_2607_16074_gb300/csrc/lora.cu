@@ -2,26 +2,19 @@
 // workload): y += (x A_t^T) B_t^T for the rows of tenant t, rank r = 16.
 //
 // The low-rank update is split in two:
-//   down  t = x A_t^T  [rows, parts * r] fp32   -- this file: a segmented
+//   down  t = x A_t^T  [rows, parts * r] bf16   -- this file: a segmented
 //         mma.sync kernel whose 64-row tiles never straddle two tenants
 //         (tiles start at each tenant's first row), so each tile applies one
 //         tenant's A;
-//   up    t B_t^T is added inside the projection GEMM's epilogue (gemm.cu),
-//         before RoPE for Q/K/V and before the residual add for O, using the
-//         per-row tenant index built here.
+//   up    t B_t^T is one more K = 16 tcgen05 MMA into the projection GEMM's
+//         accumulator (gemm.cu, gemm_launch_lora), before RoPE for Q/K/V and
+//         before the residual add for O; that GEMM lays its tiles out per
+//         tenant segment too.
 // Rows of one tenant are contiguous because the plan packs tenant by tenant.
 #include "jnx_dev.cuh"
 #include "jnx_kernels.h"
 
 namespace jnx {
-
-// row_tenant[r] = tenant of the sample that owns packed row r.
-__global__ void k_row_tenant(const int* __restrict__ cu, const int* __restrict__ sample_slot,
-                             const __grid_constant__ LoraSlots ls, int* __restrict__ row_tenant) {
-    const int s = ls.sample0 + blockIdx.x;
-    const int t = ls.tenant[sample_slot[s] - ls.g0];
-    for (int r = cu[s] + threadIdx.x; r < cu[s + 1]; r += blockDim.x) row_tenant[r] = t;
-}
 
 namespace lora {
 constexpr int BM = 64, BK = 64;
@@ -39,7 +32,7 @@ template <int NP>
 __global__ void __launch_bounds__(128) k_lora_down(const uint16_t* __restrict__ x, int ldx, int K,
                                                    const __grid_constant__ LoraSlots ls,
                                                    const __grid_constant__ LoraDown ld,
-                                                   float* __restrict__ t, int ldt) {
+                                                   uint16_t* __restrict__ t, int ldt) {
     using lora::BK;
     using lora::BM;
     constexpr int R = kLoraRank;
@@ -113,28 +106,14 @@ __global__ void __launch_bounds__(128) k_lora_down(const uint16_t* __restrict__ 
     for (int i = 0; i < NT; ++i) {
         const int col = i * 8 + 2 * tq;
         if (ra < r1)
-            *reinterpret_cast<float2*>(t + (size_t)ra * ldt + col) = make_float2(acc[i][0], acc[i][1]);
+            *reinterpret_cast<uint32_t*>(t + (size_t)ra * ldt + col) = pack_bf2(acc[i][0], acc[i][1]);
         if (rb < r1)
-            *reinterpret_cast<float2*>(t + (size_t)rb * ldt + col) = make_float2(acc[i][2], acc[i][3]);
+            *reinterpret_cast<uint32_t*>(t + (size_t)rb * ldt + col) = pack_bf2(acc[i][2], acc[i][3]);
     }
-}
-
-jnx_status lora_row_tenant_launch(const jnx_group* g, int* row_tenant, cudaStream_t s) {
-    for (int g0 = 0; g0 < g->n_slots; g0 += kLoraMaxSlots) {
-        LoraSlots ls{};
-        ls.g0 = g0;
-        ls.n = g->n_slots - g0 < kLoraMaxSlots ? g->n_slots - g0 : kLoraMaxSlots;
-        for (int i = 0; i < ls.n; ++i) ls.tenant[i] = g->h_slot_tenant[g0 + i];
-        ls.sample0 = g->h_seg_offsets[g0];
-        const int ns = g->h_seg_offsets[g0 + ls.n] - ls.sample0;
-        if (ns > 0) k_row_tenant<<<ns, 256, 0, s>>>(g->cu_seqlens, g->sample_slot, ls, row_tenant);
-    }
-    cudaError_t e = cudaGetLastError();
-    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "row tenant: %s", cudaGetErrorString(e));
 }
 
 jnx_status lora_down_launch(const jnx_group* g, const uint16_t* x, int ldx, int K, int n_parts,
-                            const uint16_t* const* a, float* t, int ldt, cudaStream_t s) {
+                            const uint16_t* const* a, uint16_t* t, int ldt, cudaStream_t s) {
     if (K % lora::BK) return fail(JNX_ERR_UNSUPPORTED, "lora: K %% 64 != 0");
     LoraDown ld{};
     for (int p = 0; p < n_parts; ++p) ld.a[p] = a[p];
