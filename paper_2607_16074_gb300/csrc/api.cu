@@ -397,6 +397,8 @@ jnx_status check_heads(const jnx_head* heads, int32_t n_tenants, const jnx_group
             if (!h.q || !h.wk || !h.wv || !h.wout || !h.bout)
                 return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null parameter", t);
             if (!hidden) return fail(JNX_ERR_INVALID_ARG, "heads: query heads need hidden rows");
+            if (h.d_in % 128)
+                return fail(JNX_ERR_UNSUPPORTED, "heads: query heads need d_in %% 128 == 0");
             if (need_grads && (!grads[t].q || !grads[t].wk || !grads[t].wv || !grads[t].wout ||
                                !grads[t].bout))
                 return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null gradient buffer", t);

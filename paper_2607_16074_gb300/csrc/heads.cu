@@ -417,53 +417,150 @@ __global__ void __launch_bounds__(256) k_xattn_dq(const __grid_constant__ HeadTa
 }
 
 // dW[c, e] = sum over the slot's token rows r of g[r, c] * X[r, e], for
-// g = dk (-> dWk) and g = dv (-> dWv).  64 x 64 output tile per CTA, rows in
-// chunks of 32 through shared memory, 4 x 4 outputs per thread, fixed order.
-__global__ void __launch_bounds__(256) k_xattn_wgrad(const __grid_constant__ HeadTable tab,
+// g = dk (-> dWk) and g = dv (-> dWv): a GEMM whose reduction runs over the
+// tenant's rows, on bf16 mma.sync (m16n8k16) with fp32 accumulation.  One
+// CTA per 64 x 128 output tile, 4 warps in a 2 x 2 layout (32 x 64 each);
+// rows stream through shared memory in chunks of 32.  The fp32 g is split
+// while staged into g_hi = bf16(g) and g_lo = bf16(g - g_hi) and both are
+// multiplied (X is exact in bf16), which keeps the result at fp32 accuracy;
+// both operands are row-major in r (MN-major) and are read with
+// ldmatrix.trans; X arrives by cp.async.  Fixed reduction order.
+namespace wg {
+constexpr int BMC = 64, BNE = 128, BR = 32;
+}
+
+__global__ void __launch_bounds__(128) k_xattn_wgrad(const __grid_constant__ HeadTable tab,
                                                      const float* __restrict__ dk,
                                                      const float* __restrict__ dv, int ldkv,
                                                      const uint16_t* __restrict__ X, int ldx) {
+    using namespace wg;
     const HeadSlot& hs = tab.slot[blockIdx.x];
     if (hs.kind != JNX_HEAD_XATTN) return;
     const int which = blockIdx.z & 1;
-    const int ctile = blockIdx.y;                 // 64-row block of the dq axis
-    const int etile = blockIdx.z >> 1;            // 64-column block of the d axis
-    if (ctile * 64 >= hs.dq || etile * 64 >= hs.d_in) return;
+    const int c0 = blockIdx.y * BMC;            // dq rows of the tile
+    const int e0 = (blockIdx.z >> 1) * BNE;     // d columns of the tile
+    if (c0 >= hs.dq || e0 >= hs.d_in) return;
     const float* G = which ? dv : dk;
     float* out = which ? hs.g_wv : hs.g_wk;
-    __shared__ float As[32][64 + 4];
-    __shared__ float Bs[32][64 + 4];
-    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-    float acc[4][4] = {};
-    for (int r = hs.r0; r < hs.r1; r += 32) {
-        const int nr = min(32, hs.r1 - r);
-        for (int i = threadIdx.x; i < 32 * 64; i += 256) {
-            const int rr = i / 64, cc = i % 64;
-            const bool ok = rr < nr;
-            As[rr][cc] = ok ? G[(size_t)(r + rr) * ldkv + ctile * 64 + cc] : 0.f;
-            Bs[rr][cc] = ok ? bf2f(X[(size_t)(r + rr) * ldx + etile * 64 + cc]) : 0.f;
-        }
-        __syncthreads();
-#pragma unroll 8
-        for (int rr = 0; rr < 32; ++rr) {
-            float a[4], b[4];
+    __shared__ __align__(128) uint8_t sA[2][2][BR * BMC * 2];  // [buf][hi/lo][r][c] bf16
+    __shared__ __align__(128) uint8_t sB[2][BR * BNE * 2];  // [r][e] bf16, 256-byte rows
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int wm = warp & 1, wn = warp >> 1;
+    const uint32_t aA = smem_u32(sA), aB = smem_u32(sB);
+    // row r, 16-byte chunk ch of a tile with `cpr` chunks per row, XOR-swizzled
+    auto swz = [](int r, int ch, int cpr) { return (uint32_t)(r * cpr * 16 + ((ch ^ (r & 7)) << 4)); };
+
+    float acc[2][8][4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                a[i] = As[rr][ty * 4 + i];
-                b[i] = Bs[rr][tx * 4 + i];
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j][0] = acc[i][j][1] = acc[i][j][2] = acc[i][j][3] = 0.f;
+
+    // A staging: thread -> (row = tid / 4, 16 consecutive c at (tid % 4) * 16)
+    const int ar = tid >> 2, ac = (tid & 3) * 16;
+    float4 areg[4];
+    auto load_a = [&](int r) {
+        const bool ok = r + ar < hs.r1;
+        const float4* src = reinterpret_cast<const float4*>(G + (size_t)(r + ar) * ldkv + c0 + ac);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) areg[i] = ok ? src[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    };
+    auto store_a = [&](int buf) {
+        uint8_t* hi_base = sA[buf][0];
+        uint8_t* lo_base = sA[buf][1];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const float v[8] = {areg[2 * h].x,     areg[2 * h].y,     areg[2 * h].z,
+                                areg[2 * h].w,     areg[2 * h + 1].x, areg[2 * h + 1].y,
+                                areg[2 * h + 1].z, areg[2 * h + 1].w};
+            uint32_t hw[4], lw[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                hw[q] = pack_bf2(v[2 * q], v[2 * q + 1]);
+                const float h0 = __uint_as_float(hw[q] << 16);
+                const float h1 = __uint_as_float(hw[q] & 0xFFFF0000u);
+                lw[q] = pack_bf2(v[2 * q] - h0, v[2 * q + 1] - h1);
             }
+            const uint32_t off = swz(ar, ac / 8 + h, BMC / 8);
+            *reinterpret_cast<uint4*>(hi_base + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+            *reinterpret_cast<uint4*>(lo_base + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+        }
+    };
+    auto load_b = [&](int r, int buf) {
+        for (int i = tid; i < BR * (BNE / 8); i += 128) {
+            const int rr = i / (BNE / 8), ch = i % (BNE / 8);
+            const bool ok = r + rr < hs.r1;
+            cp_async16(aB + buf * BR * BNE * 2 + swz(rr, ch, BNE / 8),
+                       ok ? (const void*)(X + (size_t)(r + rr) * ldx + e0 + ch * 8)
+                          : (const void*)X,
+                       ok);
+        }
+    };
+
+    const int mi = lane >> 3, rr8 = lane & 7;
+    int buf = 0;
+    if (hs.r0 < hs.r1) {
+        load_a(hs.r0);
+        load_b(hs.r0, 0);
+        cp_async_commit();
+        store_a(0);
+    }
+    for (int r = hs.r0; r < hs.r1; r += BR) {
+        const bool more = r + BR < hs.r1;
+        if (more) {
+            load_a(r + BR);
+            load_b(r + BR, buf ^ 1);
+        }
+        cp_async_commit();
+        cp_async_wait<1>();
+        __syncthreads();
+        const uint32_t a_base = aA + buf * 2 * BR * BMC * 2, b_base = aB + buf * BR * BNE * 2;
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
+        for (int ks = 0; ks < BR / 16; ++ks) {
+            uint32_t af[2][2][4];  // [hi/lo][m-tile][regs]
 #pragma unroll
-                for (int k = 0; k < 4; ++k) acc[i][k] += a[i] * b[k];
+            for (int part = 0; part < 2; ++part)
+#pragma unroll
+                for (int im = 0; im < 2; ++im) {
+                    // matrices (m 0-7, k 0-7), (m 8-15, k 0-7), (m 0-7, k 8-15), (m 8-15, k 8-15)
+                    const int kr = ks * 16 + rr8 + 8 * (mi >> 1);
+                    const int mch = (wm * 32 + im * 16) / 8 + (mi & 1);
+                    ldsm_x4_t(a_base + part * BR * BMC * 2 + swz(kr, mch, BMC / 8),
+                              af[part][im][0], af[part][im][1], af[part][im][2], af[part][im][3]);
+                }
+#pragma unroll
+            for (int np = 0; np < 4; ++np) {
+                // matrices (k 0-7, n 0-7), (k 8-15, n 0-7), (k 0-7, n 8-15), (k 8-15, n 8-15)
+                const int kr = ks * 16 + rr8 + 8 * (mi & 1);
+                const int nch = (wn * 64 + np * 16) / 8 + (mi >> 1);
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4_t(b_base + swz(kr, nch, BNE / 8), b0, b1, b2, b3);
+#pragma unroll
+                for (int part = 0; part < 2; ++part)
+#pragma unroll
+                    for (int im = 0; im < 2; ++im) {
+                        const uint32_t* a = af[part][im];
+                        mma_bf16(acc[im][2 * np], a[0], a[1], a[2], a[3], b0, b1);
+                        mma_bf16(acc[im][2 * np + 1], a[0], a[1], a[2], a[3], b2, b3);
+                    }
+            }
         }
         __syncthreads();
+        if (more) store_a(buf ^ 1);
+        buf ^= 1;
     }
+    const int g = lane >> 2, t = lane & 3;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        float4* o = reinterpret_cast<float4*>(out + (size_t)(ctile * 64 + ty * 4 + i) * hs.d_in +
-                                              etile * 64 + tx * 4);
-        *o = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+    for (int im = 0; im < 2; ++im) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int c = c0 + wm * 32 + im * 16 + g;
+            const int e = e0 + wn * 64 + j * 8 + 2 * t;
+            *reinterpret_cast<float2*>(out + (size_t)c * hs.d_in + e) =
+                make_float2(acc[im][j][0], acc[im][j][1]);
+            *reinterpret_cast<float2*>(out + (size_t)(c + 8) * hs.d_in + e) =
+                make_float2(acc[im][j][2], acc[im][j][3]);
+        }
     }
 }
 
@@ -514,8 +611,8 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
             ws.ld_h, ws.dk, ws.dv, ws.dQs);
         k_xattn_dq<<<dim3(b.n, (b.max_nq * b.max_dq + 255) / 256), 256, 0, s>>>(tab, ws.dQs,
                                                                                  ws.ld_h);
-        k_xattn_wgrad<<<dim3(b.n, b.max_dq / 64, 2 * (d / 64)), 256, 0, s>>>(tab, ws.dk, ws.dv,
-                                                                             ws.ldkv, hidden, d);
+        k_xattn_wgrad<<<dim3(b.n, b.max_dq / wg::BMC, 2 * (d / wg::BNE)), 128, 0, s>>>(
+            tab, ws.dk, ws.dv, ws.ldkv, hidden, d);
     }
     return cuda_ok("heads backward");
 }
