@@ -91,7 +91,7 @@ template <int EPI>
 __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int row_end, int n0,
                                               const GemmParams& p) {
     const bool valid = row < row_end;
-    if constexpr (EPI == EPI_BF16 || EPI == EPI_F32 || EPI == EPI_RESID) {
+    if constexpr (EPI == EPI_BF16 || EPI == EPI_F32) {
 #pragma unroll 1
         for (int c = 0; c < 8; ++c) {
             uint32_t r[32];
@@ -119,16 +119,39 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int row_e
                     dst[v] = make_float4(__uint_as_float(r[4 * v]), __uint_as_float(r[4 * v + 1]),
                                          __uint_as_float(r[4 * v + 2]),
                                          __uint_as_float(r[4 * v + 3]));
-            } else {
-                float4* dst = reinterpret_cast<float4*>(p.resid + (size_t)row * p.ldr + col);
+            }
+        }
+    } else if constexpr (EPI == EPI_RESID) {
+        // x[row, n0 .. n0+256) += C: the residual row is read two 32-column
+        // chunks ahead of its use so its latency overlaps the TMEM reads and
+        // the stores of the chunks before it
+        float4* xrow = reinterpret_cast<float4*>(p.resid + (size_t)(valid ? row : 0) * p.ldr + n0);
+        float4 xa[8], xb[8];
+        if (valid) {
+#pragma unroll
+            for (int v = 0; v < 8; ++v) {
+                xa[v] = xrow[v];
+                xb[v] = xrow[8 + v];
+            }
+        }
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            uint32_t r[32];
+            tmem_ld32(tbase + c * 32, r);
+            tmem_ld_wait();
+            float4(&cur)[8] = (c & 1) ? xb : xa;
+            if (valid) {
 #pragma unroll
                 for (int v = 0; v < 8; ++v) {
-                    float4 x = dst[v];
-                    x.x += __uint_as_float(r[4 * v]);
-                    x.y += __uint_as_float(r[4 * v + 1]);
-                    x.z += __uint_as_float(r[4 * v + 2]);
-                    x.w += __uint_as_float(r[4 * v + 3]);
-                    dst[v] = x;
+                    cur[v].x += __uint_as_float(r[4 * v]);
+                    cur[v].y += __uint_as_float(r[4 * v + 1]);
+                    cur[v].z += __uint_as_float(r[4 * v + 2]);
+                    cur[v].w += __uint_as_float(r[4 * v + 3]);
+                    xrow[8 * c + v] = cur[v];
+                }
+                if (c + 2 < 8) {
+#pragma unroll
+                    for (int v = 0; v < 8; ++v) cur[v] = xrow[8 * (c + 2) + v];
                 }
             }
         }
