@@ -49,6 +49,28 @@ def workload_desc(w):
             f"heads ({b.n_kv_heads} kv), FFN {b.d_ff} {'SwiGLU' if b.glu == 0 else 'GeGLU'}")
 
 
+def replica_seed(base_seed: int, rank: int) -> int:
+    """With N > 1 every rank runs its own independent group: the same shapes,
+    its own seeded inputs and weights (no data-path collective)."""
+    return base_seed + 1000 * rank
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """The job's time is its slowest rank's (barrier-bracketed region)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(tokens_per_rank: int, world: int, steps: int, t_ms: float) -> float:
+    """Whole-job throughput: the tokens all ranks processed over the job time."""
+    return tokens_per_rank * world * steps / (t_ms / 1e3)
+
+
 def make_bench_workload(args):
     import synth
     over = {"n_layers": args.layers} if getattr(args, "layers", 0) else {}
@@ -167,7 +189,7 @@ def run_ours(args, rank, world, local_rank):
     dev = torch.device("cuda", local_rank)
     w = make_bench_workload(args)
     # each rank owns an independent group (same shapes, its own inputs)
-    w.seed = w.seed + 1000 * rank if rank else w.seed
+    w.seed = replica_seed(w.seed, rank)
     bw = synth.make_backbone_weights(w, device=dev)
     hw = synth.make_head_weights(w, device=dev)
     inp = synth.make_inputs(w, device=dev)
@@ -215,13 +237,9 @@ def run_ours(args, rank, world, local_rank):
     kinds, ms, work = J.jnx_trace_read(cap)
     J.jnx_trace_disable()
     clk = clocks.stop()
-    t_ms = e0.elapsed_time(e1)
-    if world > 1:
-        tt = torch.tensor([t_ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        t_ms = float(tt.item())
+    t_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
     tokens = plan.n_tokens
-    value = tokens * world * args.steps / (t_ms / 1e3)
+    value = job_tokens_per_s(tokens, world, args.steps, t_ms)
 
     # ---- end to end through the C ABI from pinned host memory --------------
     vis_d, tid_d, tgt_d = inp["vision"], inp["text_ids"], inp["targets"]
@@ -251,11 +269,7 @@ def run_ours(args, rank, world, local_rank):
         keep = e2e_step()
     torch.cuda.synchronize()
     barrier()
-    e2e_ms = (time.perf_counter() - t0) * 1e3
-    if world > 1:
-        tt = torch.tensor([e2e_ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
+    e2e_ms = max_over_ranks((time.perf_counter() - t0) * 1e3, world, dev)
     step.group = group
     e2e_plan_bytes = sum(a.nbytes for a in (plan.cu_seqlens, plan.sample_slot, plan.sample_target,
                                             plan.seg_offsets, plan.gather_src, plan.pos_ids))
@@ -332,7 +346,8 @@ def run_ours(args, rank, world, local_rank):
                     tenants=len(w.tenants), samples=plan.n_samples,
                     l2="inputs larger than L2 (weights 13 GB, activations > 1 GB per step)"),
         clocks=clk,
-        e2e=dict(value=round(tokens * world * args.steps / (e2e_ms / 1e3), 1), unit="tokens/s",
+        e2e=dict(value=round(job_tokens_per_s(tokens, world, args.steps, e2e_ms), 1),
+                 unit="tokens/s",
                  h2d_bytes_per_step=int(h2d + e2e_plan_bytes), d2h_bytes_per_step=int(d2h)),
         gpu_launches=int(launches),
         roofline=roofline,

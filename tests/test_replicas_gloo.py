@@ -1,0 +1,58 @@
+"""The N > 1 benchmark path on CPU: two gloo ranks, each an independent
+replica of the grouped step's host side (its own plan over its own seeded
+workload), the job time taken as the slowest rank's, throughput summed over
+ranks.  No data-path collective is involved."""
+import os
+import socket
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+import bench
+import synth
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    p = s.getsockname()[1]
+    s.close()
+    return p
+
+
+def _worker(rank, world, port, out):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        from paper_2607_16074_gb300 import jnx as J
+        w = synth.make_workload("small")
+        w.seed = bench.replica_seed(w.seed, rank)
+        inp = synth.make_inputs(w)
+        plan = J.jnx_group_plan(w.schemas(), bench.oracle_requests(w), len(w.tenants),
+                                w.max_samples, w.max_tokens)
+        local_ms = 10.0 + 5.0 * rank           # a stand-in for each rank's timed region
+        job_ms = bench.max_over_ranks(local_ms, world)
+        tps = bench.job_tokens_per_s(plan.n_tokens, world, 3, job_ms)
+        out[rank] = (job_ms, tps, plan.n_tokens, float(inp["targets"][:4].sum()))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_replicas_weak_scaling():
+    world = 2
+    mgr = mp.Manager()
+    out = mgr.dict()
+    mp.spawn(_worker, args=(world, _free_port(), out), nprocs=world, join=True)
+    (ms0, tps0, n0, t0), (ms1, tps1, n1, t1) = out[0], out[1]
+    assert ms0 == ms1 == 15.0                  # the slowest rank's time
+    assert n0 == n1                            # same shapes on every replica
+    assert t0 != t1                            # but each replica's own inputs
+    assert tps0 == tps1 == pytest.approx(n0 * 2 * 3 / 0.015)
+
+
+def test_single_rank_needs_no_process_group():
+    assert bench.max_over_ranks(7.5, 1) == 7.5
+    assert bench.replica_seed(4, 0) == 4
