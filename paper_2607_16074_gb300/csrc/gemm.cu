@@ -550,6 +550,17 @@ static cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, cons
     return cudaGetLastError();
 }
 
+// Tile-order group height: enough 128-row blocks of A to hold ~40 MB in L2
+// while the group sweeps all column blocks, so each weight band is re-read
+// once per group rather than once per few row blocks.  Measured on GB300 at
+// 65,536 tokens: gate/up (K=4096) 1810 -> ~1870 TFLOP/s going from 16 to 40,
+// QKV best at 32-48, down (K=11008) best at 14-16.
+static int default_group_m(int K) {
+    const double a_block = (double)gemm::BM * K * 2.0;
+    int g = (int)(40.0 * 1024 * 1024 / a_block + 0.5);
+    return g < 8 ? 8 : (g > 48 ? 48 : g);
+}
+
 jnx_status gemm_check(int M, int N, int K) {
     if (M < 0 || N <= 0 || K <= 0 || N % gemm::BN || K % gemm::BK)
         return fail(JNX_ERR_UNSUPPORTED, "gemm: need N %% 256 == 0 and K %% 64 == 0 (M=%d N=%d K=%d)",
@@ -570,7 +581,7 @@ jnx_status gemm_launch(const uint16_t* A, int lda, const uint16_t* B, int ldb, G
     int grid = num_sms();
     if (max_ctas > 0 && max_ctas < grid) grid = max_ctas;
     if (tiles < grid) grid = tiles;
-    if (p.group_m <= 0) p.group_m = 16;
+    if (p.group_m <= 0) p.group_m = default_group_m(p.K);
     cudaError_t e;
     const NoLora none{};
     switch (p.epi) {
@@ -632,7 +643,7 @@ jnx_status gemm_launch_lora(const uint16_t* A, int lda, const uint16_t* B, int l
     if (total == 0) return JNX_OK;
     int grid = num_sms();
     if (total < grid) grid = total;
-    if (p.group_m <= 0) p.group_m = 16;
+    if (p.group_m <= 0) p.group_m = default_group_m(p.K);
     cudaError_t e = p.epi == EPI_ROPE ? launch_epi<EPI_ROPE, true>(ta, tb, lg, p, grid, s)
                                       : launch_epi<EPI_RESID, true>(ta, tb, lg, p, grid, s);
     if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));
