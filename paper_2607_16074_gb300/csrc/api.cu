@@ -29,6 +29,7 @@ struct BackboneWs {
     float2* rope;     // [max_pos, hd / 2]
     uint16_t* t_qkv;  // LoRA: n1 [A_q | A_k | A_v]^T  [N, 3r] bf16
     uint16_t* t_o;    // LoRA: attention output A_o^T  [N, r] bf16
+    int2* attn_items; // attention work items (sample, 128-query tile)
     size_t bytes;
 };
 
@@ -55,6 +56,8 @@ BackboneWs carve_backbone(const jnx_backbone* bb, int64_t N, void* base) {
         w.t_qkv = reinterpret_cast<uint16_t*>(take((size_t)N * 3 * kLoraRank * 2));
         w.t_o = reinterpret_cast<uint16_t*>(take((size_t)N * kLoraRank * 2));
     }
+    // at most one item per sample plus one per 128 tokens
+    w.attn_items = reinterpret_cast<int2*>(take((size_t)(N + N / 128 + 1) * sizeof(int2)));
     w.bytes = off;
     return w;
 }
@@ -190,6 +193,34 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
         const double L = g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i];
         attn_flops += 4.0 * L * L * H * hd;
     }
+    // Attention work items, most expensive first, so that the persistent
+    // attention kernel's round-robin over them ends with the cheap ones
+    // (longest-processing-time-first balance across SMs).  Shared by every
+    // layer: the samples do not change.
+    int n_items = 0;
+    {
+        std::vector<int2> items;
+        std::vector<int> cost;
+        for (int i = 0; i < g->n_samples; ++i) {
+            const int L = g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i];
+            for (int q0 = 0; q0 < L; q0 += 128) {
+                items.push_back(make_int2(i, q0 / 128));
+                cost.push_back((L + 63) / 64);  // key tiles the item walks
+            }
+        }
+        std::vector<int> order(items.size());
+        for (size_t i = 0; i < order.size(); ++i) order[i] = (int)i;
+        std::stable_sort(order.begin(), order.end(),
+                         [&](int a, int b) { return cost[a] > cost[b]; });
+        std::vector<int2> sorted(items.size());
+        for (size_t i = 0; i < order.size(); ++i) sorted[i] = items[order[i]];
+        n_items = (int)sorted.size();
+        if ((size_t)n_items > (size_t)N + N / 128 + 1)
+            return fail(JNX_ERR_INVALID_ARG, "backbone: sample lengths exceed n_tokens");
+        if (n_items && cudaMemcpyAsync(w.attn_items, sorted.data(), sorted.size() * sizeof(int2),
+                                       cudaMemcpyHostToDevice, s) != cudaSuccess)
+            return cuda_status("backbone: attention items");
+    }
 
     for (int l = 0; l < bb->n_layers; ++l) {
         const jnx_layer& L = bb->layers[l];
@@ -229,7 +260,8 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
         {
             TraceScope ts(JNX_K_ATTN, attn_flops, s);
             if ((st = attention_launch(w.qkv, qkvw, N, H, Hkv, hd, g->cu_seqlens, g->n_samples,
-                                       g->max_seqlen, w.att, H * hd, w.status, s)))
+                                       g->max_seqlen, w.attn_items, n_items, w.att, H * hd,
+                                       w.status, s)))
                 return st;
         }
         p = GemmParams{};
@@ -689,7 +721,7 @@ extern "C" jnx_status jnx_op_attention(const uint16_t* qkv, int32_t n_tokens, in
     const int ldq = (n_heads + 2 * n_kv_heads) * head_dim;
     TraceScope ts(JNX_K_ATTN, 0.0, static_cast<cudaStream_t>(stream));
     return attention_launch(qkv, ldq, n_tokens, n_heads, n_kv_heads, head_dim, cu_seqlens,
-                            n_samples, max_seqlen, out, n_heads * head_dim, status,
+                            n_samples, max_seqlen, nullptr, 0, out, n_heads * head_dim, status,
                             static_cast<cudaStream_t>(stream));
 }
 

@@ -1,205 +1,25 @@
 // Varlen attention confined to each sample (block-diagonal, bidirectional).
 //
 // Every sample is one observation prefix; its tokens attend to each other
-// and to nothing else, so the grid only visits (sample, 64-query tile, head)
-// triples inside a sample and the key loop only walks that sample's keys:
-// no cross-sample tile is ever computed.  Tiles start at the sample's first
-// token, so a sample's result is the same wherever it sits in the packed
-// batch (grouped == isolated).
+// and to nothing else, so the kernels only visit (sample, 128-query tile,
+// head) triples inside a sample and the key loop only walks that sample's
+// keys: no cross-sample tile is ever computed.  Tiles start at the sample's
+// first token, so a sample's result is the same wherever it sits in the
+// packed batch (grouped == isolated).
 //
-// Two kernels, chosen per head dim in attention_launch:
-//  k_attn     flash-style online softmax in fp32 with bf16 mma.sync
-//             (m16n8k16): each of the 4 warps owns 16 query rows; K/V tiles
-//             stream through a double-buffered cp.async ring in XOR-swizzled
-//             shared memory read with ldmatrix;
-//  k_attn_tc  the same algorithm on tcgen05: S and O accumulate in TMEM, Q/K/V
-//             arrive by TMA, P goes through shared memory (see below).
+// Two tcgen05 kernels (S and O accumulate in TMEM, Q/K/V arrive by TMA, P
+// goes through shared memory), chosen per head dim in attention_launch:
+//  k_attn_ws  head dims 64 / 128: persistent and warp-specialised, two
+//             independent streams of query tiles per CTA with double-buffered
+//             scores, so softmax, MMA and copies overlap;
+//  k_attn_tc  head dim 256 (whose O accumulator leaves no TMEM for a second
+//             stream): one CTA per (sample, query tile, head).
 // Q, K, V come from the fused projection output [N, (H + 2 Hkv) hd]; query
 // head h reads K/V head h / (H / Hkv) (MQA when Hkv = 1).
 #include "jnx_dev.cuh"
 #include "jnx_kernels.h"
 
 namespace jnx {
-
-namespace attn {
-constexpr int BM = 64;  // query rows per CTA (16 per warp)
-}
-
-// byte offset of 16-byte chunk `ch` of row `r` in a [rows][HD] bf16 tile
-template <int HD>
-__device__ __forceinline__ uint32_t sw_off(int r, int ch) {
-    return (uint32_t)(r * HD * 2 + ((ch ^ (r & 7)) << 4));
-}
-
-template <int HD, int BN>
-__global__ void __launch_bounds__(128) k_attn(const uint16_t* __restrict__ qkv, int ldq, int H,
-                                              int Hkv, const int* __restrict__ cu,
-                                              int tiles_per_sample, float scale_log2,
-                                              uint16_t* __restrict__ out, int ldo) {
-    using attn::BM;
-    constexpr int CH = HD / 8;   // 16-byte chunks per row
-    constexpr int NT = BN / 8;   // S n-tiles per warp
-    constexpr int OT = HD / 8;   // O n-tiles per warp
-    extern __shared__ __align__(128) uint8_t sm[];
-    uint8_t* sQ = sm;
-    uint8_t* sK = sQ + BM * HD * 2;
-    uint8_t* sV = sK + 2 * BN * HD * 2;
-
-    const int s = blockIdx.x / tiles_per_sample;
-    const int qt = blockIdx.x % tiles_per_sample;
-    const int h = blockIdx.y;
-    const int kvh = h / (H / Hkv);
-    const int start = cu[s];
-    const int L = cu[s + 1] - start;
-    const int q0 = qt * BM;
-    if (q0 >= L) return;
-
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const uint16_t* Qg = qkv + (size_t)start * ldq + h * HD;
-    const uint16_t* Kg = qkv + (size_t)start * ldq + (H + kvh) * HD;
-    const uint16_t* Vg = qkv + (size_t)start * ldq + (H + Hkv + kvh) * HD;
-
-    const uint32_t sQa = smem_u32(sQ), sKa = smem_u32(sK), sVa = smem_u32(sV);
-
-    // Q tile (rows beyond the sample are zero)
-    for (int i = tid; i < BM * CH; i += 128) {
-        const int r = i / CH, ch = i % CH;
-        const bool ok = q0 + r < L;
-        cp_async16(sQa + sw_off<HD>(r, ch), ok ? (const void*)(Qg + (size_t)(q0 + r) * ldq + ch * 8)
-                                               : (const void*)qkv,
-                   ok);
-    }
-    auto load_kv = [&](int kt, int buf) {
-        const int k0 = kt * BN;
-        for (int i = tid; i < BN * CH; i += 128) {
-            const int r = i / CH, ch = i % CH;
-            const bool ok = k0 + r < L;
-            const size_t off = (size_t)(k0 + r) * ldq + ch * 8;
-            cp_async16(sKa + buf * BN * HD * 2 + sw_off<HD>(r, ch),
-                       ok ? (const void*)(Kg + off) : (const void*)qkv, ok);
-            cp_async16(sVa + buf * BN * HD * 2 + sw_off<HD>(r, ch),
-                       ok ? (const void*)(Vg + off) : (const void*)qkv, ok);
-        }
-    };
-    const int n_kt = (L + BN - 1) / BN;
-    load_kv(0, 0);
-    cp_async_commit();
-
-    float o[OT][4];
-#pragma unroll
-    for (int i = 0; i < OT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-
-    const int g = lane >> 2, t = lane & 3;
-    const int mi = lane >> 3, rr = lane & 7;
-    const int qrow = warp * 16;
-
-    for (int kt = 0; kt < n_kt; ++kt) {
-        const int buf = kt & 1;
-        if (kt + 1 < n_kt) load_kv(kt + 1, buf ^ 1);
-        cp_async_commit();
-        cp_async_wait<1>();
-        __syncthreads();
-
-        const uint32_t kb = sKa + buf * BN * HD * 2;
-        const uint32_t vb = sVa + buf * BN * HD * 2;
-
-        // S = Q K^T (16 x BN per warp)
-        float sc[NT][4];
-#pragma unroll
-        for (int i = 0; i < NT; ++i) sc[i][0] = sc[i][1] = sc[i][2] = sc[i][3] = 0.f;
-#pragma unroll
-        for (int ks = 0; ks < HD / 16; ++ks) {
-            uint32_t a0, a1, a2, a3;
-            ldsm_x4(sQa + sw_off<HD>(qrow + rr + 8 * (mi & 1), ks * 2 + (mi >> 1)), a0, a1, a2, a3);
-#pragma unroll
-            for (int nb = 0; nb < BN / 16; ++nb) {
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4(kb + sw_off<HD>(nb * 16 + rr + 8 * (mi >> 1), ks * 2 + (mi & 1)), b0, b1,
-                        b2, b3);
-                mma_bf16(sc[2 * nb], a0, a1, a2, a3, b0, b1);
-                mma_bf16(sc[2 * nb + 1], a0, a1, a2, a3, b2, b3);
-            }
-        }
-
-        // scale to log2 domain, mask keys past the sample, online softmax
-        const int kbase = kt * BN;
-        float mx0 = m0, mx1 = m1;
-#pragma unroll
-        for (int i = 0; i < NT; ++i) {
-            const int key = kbase + i * 8 + 2 * t;
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const bool ok = key + (e & 1) < L;
-                sc[i][e] = ok ? sc[i][e] * scale_log2 : -INFINITY;
-            }
-            mx0 = fmaxf(mx0, fmaxf(sc[i][0], sc[i][1]));
-            mx1 = fmaxf(mx1, fmaxf(sc[i][2], sc[i][3]));
-        }
-        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-        const float al0 = exp2f(m0 - mx0), al1 = exp2f(m1 - mx1);
-        m0 = mx0;
-        m1 = mx1;
-        float rs0 = 0.f, rs1 = 0.f;
-#pragma unroll
-        for (int i = 0; i < NT; ++i) {
-            sc[i][0] = exp2f(sc[i][0] - m0);
-            sc[i][1] = exp2f(sc[i][1] - m0);
-            sc[i][2] = exp2f(sc[i][2] - m1);
-            sc[i][3] = exp2f(sc[i][3] - m1);
-            rs0 += sc[i][0] + sc[i][1];
-            rs1 += sc[i][2] + sc[i][3];
-        }
-        l0 = l0 * al0 + rs0;
-        l1 = l1 * al1 + rs1;
-#pragma unroll
-        for (int i = 0; i < OT; ++i) {
-            o[i][0] *= al0;
-            o[i][1] *= al0;
-            o[i][2] *= al1;
-            o[i][3] *= al1;
-        }
-
-        // O += P V
-#pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
-            const uint32_t a0 = pack_bf2(sc[2 * kk][0], sc[2 * kk][1]);
-            const uint32_t a1 = pack_bf2(sc[2 * kk][2], sc[2 * kk][3]);
-            const uint32_t a2 = pack_bf2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-            const uint32_t a3 = pack_bf2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
-#pragma unroll
-            for (int np = 0; np < HD / 16; ++np) {
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4_t(vb + sw_off<HD>(kk * 16 + rr + 8 * (mi & 1), 2 * np + (mi >> 1)), b0, b1,
-                          b2, b3);
-                mma_bf16(o[2 * np], a0, a1, a2, a3, b0, b1);
-                mma_bf16(o[2 * np + 1], a0, a1, a2, a3, b2, b3);
-            }
-        }
-        __syncthreads();
-    }
-
-    l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-    l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-    const float i0 = 1.f / l0, i1 = 1.f / l1;
-    const int r0 = q0 + qrow + g, r1 = r0 + 8;
-    uint16_t* ob = out + (size_t)start * ldo + h * HD;
-#pragma unroll
-    for (int i = 0; i < OT; ++i) {
-        const int col = i * 8 + 2 * t;
-        if (r0 < L)
-            *reinterpret_cast<uint32_t*>(ob + (size_t)r0 * ldo + col) =
-                pack_bf2(o[i][0] * i0, o[i][1] * i0);
-        if (r1 < L)
-            *reinterpret_cast<uint32_t*>(ob + (size_t)r1 * ldo + col) =
-                pack_bf2(o[i][2] * i1, o[i][3] * i1);
-    }
-}
 
 // ---------------------------------------------------------------------------
 // tcgen05 version.  One CTA = (sample, 128-query tile, head), 128 threads:
@@ -434,6 +254,453 @@ __global__ void __launch_bounds__(128, 1)
     if (warp == 0) tmem_dealloc(tbase, C::TCOLS);
 }
 
+// ---------------------------------------------------------------------------
+// Persistent warp-specialised tcgen05 attention (head dims 64 / 128).
+//
+// One CTA per SM runs two independent streams of work items; an item is one
+// 128-query tile of one sample and head, and its key loop walks that
+// sample's keys in BN-key tiles.  Stream t owns
+//   warp t        TMA producer: Q (one buffer, refilled as soon as the
+//                 item's last S MMA has completed), K and V through
+//                 separate 2-deep rings that run on from item to item
+//   warp 2 + t    MMA issuer: S(kt) = Q K(kt)^T into one of two TMEM score
+//                 buffers, O += P(kt) V(kt) into the TMEM accumulator; S runs
+//                 two tiles ahead of PV, so the tensor core computes the next
+//                 scores while the softmax warps work on the current ones
+//   warps 4+4t..  online softmax and epilogue, one query row per thread
+// and TMEM columns [256 t, 256 t + 256): S buffers at +0 and +BN, O at
+// +2 BN.  P (bf16) goes through shared memory as the K-major A operand of
+// the PV MMA; V is read as the MN-major B operand.  The two streams share
+// nothing but the tensor core, so one stream's softmax overlaps the other's
+// MMAs and copies, and a short tail tile costs only its own stream.
+//
+// The running max is lazy: a row raises the max m it subtracts only when a
+// new tile's max exceeds it by more than 8 (log2 units), so O is rarely
+// rescaled; the probabilities stay below 2^8 and O / l does not depend on m.
+//
+// Barriers per stream (each role tracks parities with completion counters):
+//   q_full, q_empty          Q landed / the item's last S MMA completed
+//   k_full[2], k_empty[2]    K ring (a slot frees when its S MMA completes)
+//   v_full[2], v_empty[2]    V ring (a slot frees when its PV MMA completes)
+//   s_full[2]                score buffer b holds a new S
+//   p_full                   P(kt) written and its S read (128 arrivals)
+//   o_done                   a PV MMA completed
+//   o_free                   the epilogue has read O (128 arrivals)
+//   drain                    all MMAs of the stream completed (teardown)
+// ---------------------------------------------------------------------------
+namespace attn_ws {
+constexpr int BM = 128;        // query rows per item
+constexpr float kLazy = 8.0f;  // log2 growth of the max that forces a rescale
+constexpr int kBars = 16;      // barriers per stream
+}  // namespace attn_ws
+
+// Work items: an explicit (sample, query tile) list, or, without one, every
+// (query tile, sample) combination tile-major with the empty ones skipped.
+struct AttnItems {
+    const int2* list;
+    int n;  // entries of `list`, or S * tiles_max
+    int S;
+};
+
+__device__ __forceinline__ bool attn_item(const AttnItems& it, const int* __restrict__ cu, int H,
+                                          int w, int& s, int& qt, int& h) {
+    h = w % H;
+    const int i = w / H;
+    if (it.list) {
+        const int2 e = it.list[i];
+        s = e.x;
+        qt = e.y;
+        return true;
+    }
+    qt = i / it.S;
+    s = i % it.S;
+    return qt * attn_ws::BM < cu[s + 1] - cu[s];
+}
+
+template <int HD, int BN>
+struct AttnWsCfg {
+    static_assert(BN == 64, "key tile of 64 keys");
+    static_assert(HD == 64 || HD == 128, "head dim 64 or 128");
+    static constexpr int BM = attn_ws::BM;
+    static constexpr int QB = BM * HD * 2;  // Q tile
+    static constexpr int KB = BN * HD * 2;  // one K (or V) tile
+    static constexpr int PB = BM * BN * 2;  // P tile
+    static constexpr int OFF_K = QB;
+    static constexpr int OFF_V = OFF_K + 2 * KB;
+    static constexpr int OFF_P = OFF_V + 2 * KB;
+    static constexpr int STREAM = OFF_P + PB;  // bytes per stream (multiple of 1024)
+    static constexpr int OFF_BAR = 2 * STREAM;
+    static constexpr int SMEM = OFF_BAR + 2 * attn_ws::kBars * 8 + 16 + 1024;
+    static_assert(STREAM % 1024 == 0, "128B-swizzled tiles need 1024-byte alignment");
+    static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
+    static constexpr uint32_t O_COL = 2 * BN;  // within the stream's 256 columns
+    static_assert(O_COL + HD <= 256, "TMEM columns per stream");
+};
+
+// Softmax of one 128 x BN score tile for this thread's row: row max (pass
+// 1), then probabilities packed as bf16 pairs (pass 2).  FULL: every key of
+// the tile lies inside the sample (no mask).
+template <int BN, bool FULL>
+__device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float scale_log2,
+                                                bool first, float& m, float& alpha, float& rs,
+                                                uint32_t (&pk)[BN / 2]) {
+    float mx = -INFINITY;
+#pragma unroll
+    for (int c = 0; c < BN / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld32(tS + c * 32, v);
+        tmem_ld_wait();
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+            if (FULL || c * 32 + e < kvalid) mx = fmaxf(mx, __uint_as_float(v[e]));
+    }
+    mx *= scale_log2;
+    alpha = 1.f;
+    if (first) {
+        m = mx;
+    } else if (mx > m + attn_ws::kLazy) {
+        alpha = ex2_approx(m - mx);
+        m = mx;
+    }
+    const float nm = -m;
+    rs = 0.f;
+#pragma unroll
+    for (int c = 0; c < BN / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld32(tS + c * 32, v);
+        tmem_ld_wait();
+#pragma unroll
+        for (int e = 0; e < 32; e += 2) {
+            float p0 = ex2_approx(fmaf(__uint_as_float(v[e]), scale_log2, nm));
+            float p1 = ex2_approx(fmaf(__uint_as_float(v[e + 1]), scale_log2, nm));
+            if (!FULL) {
+                if (c * 32 + e >= kvalid) p0 = 0.f;
+                if (c * 32 + e + 1 >= kvalid) p1 = 0.f;
+            }
+            rs += p0 + p1;
+            pk[c * 16 + e / 2] = pack_bf2(p0, p1);
+        }
+    }
+}
+
+template <int HD, int BN>
+__global__ void __launch_bounds__(384, 1)
+    k_attn_ws(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tkv,
+              const int* __restrict__ cu, AttnItems items, int H, int Hkv, float scale_log2,
+              uint16_t* __restrict__ out, int ldo, int* status) {
+    using C = AttnWsCfg<HD, BN>;
+    constexpr int BM = C::BM;
+    constexpr int NCH = HD / 64;  // 64-column (128-byte) chunks of a Q/K/V row
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + C::OFF_BAR + 2 * attn_ws::kBars * 8);
+    volatile int* fail_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    // stream of this warp: producers 0/1, MMA issuers 2/3, softmax 4-7 / 8-11
+    const int t = warp < 4 ? (warp & 1) : (warp - 4) >> 2;
+    uint8_t* st = sm + t * C::STREAM;
+    uint8_t* sQ = st;
+    auto sK = [&](int b) { return st + C::OFF_K + b * C::KB; };
+    auto sV = [&](int b) { return st + C::OFF_V + b * C::KB; };
+    uint8_t* sP = st + C::OFF_P;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR) + t * attn_ws::kBars;
+    uint64_t* q_full = bars + 0;
+    uint64_t* q_empty = bars + 1;
+    uint64_t* k_full = bars + 2;   // [2]
+    uint64_t* k_empty = bars + 4;  // [2]
+    uint64_t* v_full = bars + 6;   // [2]
+    uint64_t* v_empty = bars + 8;  // [2]
+    uint64_t* s_full = bars + 10;  // [2]
+    uint64_t* p_full = bars + 12;
+    uint64_t* o_done = bars + 13;
+    uint64_t* o_free = bars + 14;
+    uint64_t* drain = bars + 15;
+
+    const int n_work = items.n * H;
+    const int group = H / Hkv;
+    const int w0 = 2 * blockIdx.x + t, dw = 2 * gridDim.x;
+    if (tid == 0) {
+        // both streams' barriers: one arrival each, but p_full and o_free,
+        // which every softmax thread of the stream arrives on
+        uint64_t* all = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR);
+        for (int i = 0; i < 2 * attn_ws::kBars; ++i) {
+            const int k = i % attn_ws::kBars;
+            mbar_init(&all[i], (k == 12 || k == 14) ? BM : 1);
+        }
+        *fail_flag = 0;
+        fence_barrier_init();
+        fence_proxy_async();
+    }
+    if (warp == 2) {
+        tmem_alloc(tmem_slot, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = *tmem_slot + (uint32_t)(t * 256);
+
+    if (warp < 2) {
+        // ---------------- producer of stream t ----------------
+        if (lane == 0) {
+            tma_prefetch_desc(&tq);
+            tma_prefetch_desc(&tkv);
+            bool ok = true;
+            int nq = 0;            // Q tiles loaded
+            uint32_t gk = 0, gv = 0;  // K / V tiles loaded
+            auto load_kv = [&](bool is_v, uint32_t& g, int y, int col) -> bool {
+                const int b = g & 1;
+                uint64_t* full = is_v ? &v_full[b] : &k_full[b];
+                if (!mbar_wait(is_v ? &v_empty[b] : &k_empty[b], ((g >> 1) & 1) ^ 1)) return false;
+                mbar_arrive_expect_tx(full, C::KB);
+                uint8_t* dst = is_v ? sV(b) : sK(b);
+#pragma unroll
+                for (int c = 0; c < NCH; ++c)
+                    tma_load_2d(dst + c * BN * 128, &tkv, col + c * 64, y, full);
+                ++g;
+                return true;
+            };
+            for (int w = w0; w < n_work && ok && !*fail_flag; w += dw) {
+                int s, qt, h;
+                if (!attn_item(items, cu, H, w, s, qt, h)) continue;
+                const int start = cu[s], L = cu[s + 1] - start;
+                const int n_kt = (L + BN - 1) / BN;
+                const int kvh = h / group;
+                if (nq > 0 && !(ok = mbar_wait(q_empty, (nq - 1) & 1))) break;
+                mbar_arrive_expect_tx(q_full, C::QB);
+#pragma unroll
+                for (int c = 0; c < NCH; ++c)
+                    tma_load_2d(sQ + c * BM * 128, &tq, h * HD + c * 64, start + qt * BM, q_full);
+                ++nq;
+                // K runs one tile ahead of V: S(kt + 1) is issued before PV(kt)
+                for (int j = 0; j <= n_kt && ok; ++j) {
+                    if (j < n_kt) ok = load_kv(false, gk, start + j * BN, (H + kvh) * HD);
+                    if (ok && j > 0)
+                        ok = load_kv(true, gv, start + (j - 1) * BN, (H + Hkv + kvh) * HD);
+                }
+            }
+            if (!ok) *fail_flag = 1;
+            // teardown: every copy this thread issued has landed before the
+            // CTA may exit (immediate in a normal run: the MMA warp has
+            // consumed them all)
+            if (nq > 0) mbar_wait(q_full, (nq - 1) & 1);
+            for (uint32_t k = 0; k < 2 && k < gk; ++k)
+                mbar_wait(&k_full[(gk - 1 - k) & 1], ((gk - 1 - k) >> 1) & 1);
+            for (uint32_t k = 0; k < 2 && k < gv; ++k)
+                mbar_wait(&v_full[(gv - 1 - k) & 1], ((gv - 1 - k) >> 1) & 1);
+        }
+    } else if (warp < 4) {
+        // ---------------- MMA issuer of stream t ----------------
+        if (lane == 0) {
+            constexpr uint32_t IDESC_S = idesc_bf16_f32(BM, BN);
+            constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, HD) | (1u << 16);  // B MN-major
+            bool ok = true, issued = false;
+            int nq = 0;                  // Q tiles consumed
+            uint32_t gk = 0, gv = 0;     // K / V tiles consumed
+            uint32_t gs = 0;             // S tiles issued (score buffer gs & 1)
+            uint32_t gp = 0;             // p_full completions consumed
+            int items_done = 0;
+            auto issue_s = [&](const uint32_t qa) -> bool {
+                const int b = gk & 1;
+                if (!mbar_wait(&k_full[b], (gk >> 1) & 1)) return false;
+                tc_fence_after();
+                const uint32_t ka = smem_u32(sK(b));
+                const uint32_t d = tbase + (gs & 1) * BN;
+#pragma unroll
+                for (int ks = 0; ks < HD / 16; ++ks)
+                    tc_mma_f16(d, sw128_desc(qa + (ks >> 2) * BM * 128 + (ks & 3) * 32),
+                               sw128_desc(ka + (ks >> 2) * BN * 128 + (ks & 3) * 32), IDESC_S,
+                               ks > 0);
+                tc_commit(&s_full[gs & 1]);
+                tc_commit(&k_empty[b]);
+                ++gk;
+                ++gs;
+                issued = true;
+                return true;
+            };
+            for (int w = w0; w < n_work && ok && !*fail_flag; w += dw) {
+                int s, qt, h;
+                if (!attn_item(items, cu, H, w, s, qt, h)) continue;
+                const int L = cu[s + 1] - cu[s];
+                const int n_kt = (L + BN - 1) / BN;
+                if (!(ok = mbar_wait(q_full, nq & 1))) break;
+                ++nq;
+                tc_fence_after();
+                const uint32_t qa = smem_u32(sQ);
+                // S(0), S(1): their score buffers were read before the
+                // previous item's last PVs were issued
+                ok = issue_s(qa) && (n_kt < 2 || issue_s(qa));
+                if (ok && n_kt <= 2) tc_commit(q_empty);
+                for (int kt = 0; kt < n_kt && ok; ++kt) {
+                    // P(kt) is out and S(kt) read
+                    if (!(ok = mbar_wait(p_full, gp & 1))) break;
+                    ++gp;
+                    // the first PV of an item overwrites O: the previous
+                    // item's epilogue must have read it
+                    if (kt == 0 && items_done > 0 && !(ok = mbar_wait(o_free, (items_done - 1) & 1)))
+                        break;
+                    const int b = gv & 1;
+                    if (!(ok = mbar_wait(&v_full[b], (gv >> 1) & 1))) break;
+                    tc_fence_after();
+                    const uint32_t pa = smem_u32(sP), va = smem_u32(sV(b));
+#pragma unroll
+                    for (int ks = 0; ks < BN / 16; ++ks)
+                        tc_mma_f16(tbase + C::O_COL,
+                                   sw128_desc(pa + (ks >> 2) * BM * 128 + (ks & 3) * 32),
+                                   sw128_desc_mn(va + ks * 16 * 128, BN * 128, 1024), IDESC_PV,
+                                   kt > 0 || ks > 0);
+                    tc_commit(o_done);
+                    tc_commit(&v_empty[b]);
+                    ++gv;
+                    // S(kt + 2) reuses the score buffer of S(kt)
+                    if (kt + 2 < n_kt) {
+                        ok = issue_s(qa);
+                        if (ok && kt + 3 == n_kt) tc_commit(q_empty);
+                    }
+                }
+                ++items_done;
+            }
+            if (!ok) *fail_flag = 1;
+            if (issued) {
+                tc_commit(drain);
+                mbar_wait(drain, 0);
+            }
+        }
+    } else {
+        // ---------------- softmax + epilogue of stream t ----------------
+        const int quarter = warp & 3;  // TMEM lanes this warp may access
+        const int r = quarter * 32 + lane;
+        const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+        const uint32_t tO = tbase + lane_base + C::O_COL;
+        uint32_t gs = 0, nd = 0;  // S tiles / o_done completions consumed
+        bool ok = true;
+        for (int w = w0; w < n_work && ok; w += dw) {
+            if (__any_sync(0xffffffffu, *fail_flag != 0)) break;
+            int s, qt, h;
+            if (!attn_item(items, cu, H, w, s, qt, h)) continue;
+            const int start = cu[s], L = cu[s + 1] - start;
+            const int n_kt = (L + BN - 1) / BN;
+            float m = 0.f, l = 0.f;
+            for (int kt = 0; kt < n_kt; ++kt) {
+                // waits are made warp-uniform: TMEM loads are warp-collective
+                if (!(ok = __all_sync(0xffffffffu, mbar_wait(&s_full[gs & 1], (gs >> 1) & 1))))
+                    break;
+                tc_fence_after();
+                const uint32_t tS = tbase + lane_base + (gs & 1) * BN;
+                ++gs;
+                const int kvalid = L - kt * BN;  // keys of this tile inside the sample
+                uint32_t pk[BN / 2];
+                float alpha, rs;
+                if (kvalid >= BN)
+                    attn_ws_softmax<BN, true>(tS, kvalid, scale_log2, kt == 0, m, alpha, rs, pk);
+                else
+                    attn_ws_softmax<BN, false>(tS, kvalid, scale_log2, kt == 0, m, alpha, rs, pk);
+                if (kt > 0) {
+                    // PV(kt-1) must be done before O is rescaled and P rewritten
+                    if (!(ok = __all_sync(0xffffffffu, mbar_wait(o_done, nd & 1)))) break;
+                    ++nd;
+                    tc_fence_after();
+                    if (__any_sync(0xffffffffu, alpha < 1.f)) {
+#pragma unroll 1
+                        for (int c = 0; c < HD / 32; ++c) {
+                            uint32_t v[32];
+                            tmem_ld32(tO + c * 32, v);
+                            tmem_ld_wait();
+#pragma unroll
+                            for (int e = 0; e < 32; ++e)
+                                v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+                            tmem_st32(tO + c * 32, v);
+                        }
+                        tmem_st_wait();
+                    }
+                }
+                l = l * alpha + rs;
+                uint8_t* prow = sP + r * 128;
+#pragma unroll
+                for (int u = 0; u < BN / 8; ++u)
+                    *reinterpret_cast<uint4*>(prow + (u >> 3) * BM * 128 +
+                                              (((u & 7) ^ (r & 7)) << 4)) =
+                        make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+                fence_proxy_async();  // P visible to the tensor core
+                tc_fence_before();
+                mbar_arrive(p_full);
+            }
+            if (!ok) break;
+            // epilogue: O / l -> bf16
+            if (!(ok = __all_sync(0xffffffffu, mbar_wait(o_done, nd & 1)))) break;
+            ++nd;
+            tc_fence_after();
+            const float inv = 1.0f / l;
+            uint32_t ob[HD / 2];
+#pragma unroll
+            for (int c = 0; c < HD / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(tO + c * 32, v);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 16; ++e)
+                    ob[c * 16 + e] = pack_bf2(__uint_as_float(v[2 * e]) * inv,
+                                              __uint_as_float(v[2 * e + 1]) * inv);
+            }
+            tc_fence_before();
+            mbar_arrive(o_free);
+            const int row = qt * BM + r;
+            if (row < L) {
+                uint4* dst = reinterpret_cast<uint4*>(out + (size_t)(start + row) * ldo + h * HD);
+#pragma unroll
+                for (int q = 0; q < HD / 8; ++q)
+                    dst[q] = make_uint4(ob[4 * q], ob[4 * q + 1], ob[4 * q + 2], ob[4 * q + 3]);
+            }
+        }
+        if (!ok) *fail_flag = 1;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (*fail_flag && tid == 0) report(status, JNX_ERR_TIMEOUT);
+    if (warp == 2) tmem_dealloc(*tmem_slot, 512);
+}
+
+template <int HD, int BN>
+static jnx_status launch_attn_ws(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv,
+                                 const int* cu, int S, int max_seqlen, const int2* items,
+                                 int n_items, uint16_t* out, int ldo, int* status,
+                                 cudaStream_t s) {
+    using C = AttnWsCfg<HD, BN>;
+    static bool attr = false;
+    if (!attr) {
+        if (cudaFuncSetAttribute(k_attn_ws<HD, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 C::SMEM) != cudaSuccess)
+            return fail(JNX_ERR_CUDA, "attention: smem attribute");
+        attr = true;
+    }
+    CUtensorMap tq, tkv;
+    if (!make_tmap_bf16(&tq, qkv, n_tokens, ldq, ldq, C::BM, 64) ||
+        !make_tmap_bf16(&tkv, qkv, n_tokens, ldq, ldq, BN, 64))
+        return fail(JNX_ERR_CUDA, "attention: tensor map encode failed");
+    AttnItems it;
+    it.S = S;
+    if (items) {
+        it.list = items;
+        it.n = n_items;
+    } else {
+        it.list = nullptr;
+        it.n = S * ((max_seqlen + C::BM - 1) / C::BM);
+    }
+    if ((long long)it.n * H > 0x7FFFFFFFLL)
+        return fail(JNX_ERR_UNSUPPORTED, "attention: too many work items");
+    const int n_work = it.n * H;
+    if (n_work == 0) return JNX_OK;
+    const int grid = std::min((n_work + 1) / 2, num_sms());
+    const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)HD));
+    k_attn_ws<HD, BN><<<grid, 384, C::SMEM, s>>>(tq, tkv, cu, it, H, Hkv, scale_log2, out, ldo,
+                                                 status);
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
+}
+
 template <int HD, int BN>
 static jnx_status launch_attn_tc(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv,
                                  const int* cu, int S, int max_seqlen, uint16_t* out, int ldo,
@@ -459,46 +726,20 @@ static jnx_status launch_attn_tc(const uint16_t* qkv, int ldq, int n_tokens, int
     return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
 }
 
-template <int HD, int BN>
-static cudaError_t launch_attn(const uint16_t* qkv, int ldq, int H, int Hkv, const int* cu, int S,
-                               int max_seqlen, uint16_t* out, int ldo, cudaStream_t s) {
-    constexpr int smem = attn::BM * HD * 2 + 4 * BN * HD * 2;
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e =
-            cudaFuncSetAttribute(k_attn<HD, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e != cudaSuccess) return e;
-        attr = true;
-    }
-    const int tps = (max_seqlen + attn::BM - 1) / attn::BM;
-    const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)HD));
-    dim3 grid(S * tps, H);
-    k_attn<HD, BN><<<grid, 128, smem, s>>>(qkv, ldq, H, Hkv, cu, tps, scale_log2, out, ldo);
-    return cudaGetLastError();
-}
-
 jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv, int hd,
-                            const int* cu, int S, int max_seqlen, uint16_t* out, int ldo,
-                            int* status, cudaStream_t s) {
+                            const int* cu, int S, int max_seqlen, const int2* items, int n_items,
+                            uint16_t* out, int ldo, int* status, cudaStream_t s) {
     if (S == 0 || max_seqlen == 0) return JNX_OK;
     if (Hkv <= 0 || H % Hkv) return fail(JNX_ERR_UNSUPPORTED, "attention: H %% Hkv != 0");
-    if ((long long)S * ((max_seqlen + attn::BM - 1) / attn::BM) > 0x7FFFFFFFLL || H > 65535)
+    if ((long long)S * ((max_seqlen + attn_tc::BM - 1) / attn_tc::BM) > 0x7FFFFFFFLL || H > 65535)
         return fail(JNX_ERR_UNSUPPORTED, "attention: grid too large");
-    // Per head dim, the faster of the two kernels as measured on GB300 for
-    // prefixes of 260..840 tokens: the mma.sync kernel for 64 / 128 (181 /
-    // 224 TFLOP/s against 71 / 143 for this tcgen05 version, whose single
-    // 128-thread CTA per SM leaves the per-tile copy and softmax latencies
-    // exposed), the tcgen05 kernel for 256 (300 against 281).
-    cudaError_t e = cudaSuccess;
     switch (hd) {
         case 64:
-            e = launch_attn<64, 64>(qkv, ldq, H, Hkv, cu, S, max_seqlen, out, ldo, s);
-            return e == cudaSuccess ? JNX_OK
-                                    : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
+            return launch_attn_ws<64, 64>(qkv, ldq, n_tokens, H, Hkv, cu, S, max_seqlen, items,
+                                          n_items, out, ldo, status, s);
         case 128:
-            e = launch_attn<128, 64>(qkv, ldq, H, Hkv, cu, S, max_seqlen, out, ldo, s);
-            return e == cudaSuccess ? JNX_OK
-                                    : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
+            return launch_attn_ws<128, 64>(qkv, ldq, n_tokens, H, Hkv, cu, S, max_seqlen, items,
+                                           n_items, out, ldo, status, s);
         case 256:
             return launch_attn_tc<256, 64>(qkv, ldq, n_tokens, H, Hkv, cu, S, max_seqlen, out,
                                            ldo, status, s);

@@ -24,6 +24,14 @@ __device__ __forceinline__ uint32_t pack_bf2(float a, float b) {
     return (uint32_t)f2bf(a) | ((uint32_t)f2bf(b) << 16);
 }
 
+// 2^x by the hardware's approximate base-2 exponential (ex2.approx.ftz.f32):
+// subnormal results flush to zero.
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 // Record the first device-side error in the status word (never traps).
 __device__ __forceinline__ void report(int* status, int code) {
     if (status) atomicCAS(status, 0, code);

@@ -97,9 +97,11 @@ jnx_status final_pool_launch(const float* x, const uint16_t* gamma, float eps, c
 // (cos, sin) table for positions [0, max_pos) of head dim hd.
 jnx_status rope_table_launch(float2* tab, int max_pos, int hd, float theta, cudaStream_t s);
 
-// Varlen attention confined to each sample, bidirectional.
+// Varlen attention confined to each sample, bidirectional.  `items`
+// (device, optional) lists the (sample, 128-query tile) work items in the
+// order the persistent kernel should take them; null enumerates them.
 jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv, int hd,
-                            const int* cu, int S, int max_seqlen, uint16_t* out, int ldo,
-                            int* status, cudaStream_t s);
+                            const int* cu, int S, int max_seqlen, const int2* items, int n_items,
+                            uint16_t* out, int ldo, int* status, cudaStream_t s);
 
 }  // namespace jnx
