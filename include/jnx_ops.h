@@ -41,6 +41,9 @@ size_t jnx_op_gemm_workspace_bytes(int32_t max_pos, int32_t head_dim);
 
 /* C[M, N] = A[M, K] W[N, K]^T on the tcgen05 tensor cores, fp32 accumulate,
  * then the epilogue.  N % 256 == 0, K % 64 == 0, A/W rows 16-byte aligned.
+ * out has rows of ldo elements (bf16, or fp32 for JNX_EPI_F32 / RESID),
+ * ldo >= the output width (N, or N / 2 for JNX_EPI_GLU), 16-byte aligned
+ * rows and base, else JNX_ERR_INVALID_ARG.
  * pos/max_pos/rope_cols/head_dim/rope_theta are read for JNX_EPI_ROPE only
  * (workspace then holds the status word and the RoPE table); act
  * (JNX_GLU_*) for JNX_EPI_GLU only.  workspace may be NULL otherwise. */

@@ -678,6 +678,15 @@ extern "C" jnx_status jnx_op_gemm(const uint16_t* A, const uint16_t* W, int32_t 
                                   void* workspace, size_t ws_bytes, void* stream) {
     clear_error();
     if (!A || !W || !out || M < 0) return fail(JNX_ERR_INVALID_ARG, "gemm: null argument");
+    if (epilogue < EPI_BF16 || epilogue > EPI_ROPE)
+        return fail(JNX_ERR_INVALID_ARG, "gemm: unknown epilogue %d", epilogue);
+    {
+        // the epilogues write (and the residual one reads) 16-byte vectors
+        const int esz = (epilogue == EPI_F32 || epilogue == EPI_RESID) ? 4 : 2;
+        const int width = epilogue == EPI_GLU ? N / 2 : N;
+        if (ldo < width || ((size_t)ldo * esz) % 16 || reinterpret_cast<uintptr_t>(out) % 16)
+            return fail(JNX_ERR_INVALID_ARG, "gemm: out needs 16-byte aligned rows of >= %d", width);
+    }
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     GemmParams p{};
     p.M = M;

@@ -37,7 +37,8 @@ constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 512;  // two 256-column fp32 accumulators
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+constexpr int STG_BYTES = 4 * 2048;  // epilogue staging, 2 KB per epilogue warp
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/ + STG_BYTES;
 constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 // LoRA operands of one tile (K = 16, 32-byte rows): t rows and B rows, a
 // 2-deep ring after the main stages.
@@ -87,72 +88,122 @@ __device__ __forceinline__ float act_fn(float g, int act) {
     return 0.5f * g * (1.0f + tanhf(c * (g + 0.044715f * g * g * g)));
 }
 
+// Epilogue staging: each epilogue warp turns its 32 rows x 64 bytes from
+// one-row-per-thread (the TMEM layout) into row-contiguous global accesses
+// through a 2 KB shared-memory slot.  Writer: thread `lane` puts row `lane`.
+// Reader: in step i (0..3) thread `lane` takes row 8 i + lane / 4, 16-byte
+// unit lane % 4, so one instruction touches 8 rows x 64 contiguous bytes
+// instead of 32 rows x 16 bytes.  Units are XOR-swizzled by (row / 2) % 4,
+// which keeps both sides free of bank conflicts.
+__device__ __forceinline__ void stg_put(uint8_t* stg, int lane, const uint4 (&v)[4]) {
+    uint8_t* rowp = stg + lane * 64;
+    const int sw = (lane >> 1) & 3;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) *reinterpret_cast<uint4*>(rowp + ((j ^ sw) << 4)) = v[j];
+}
+
+__device__ __forceinline__ uint4 stg_get(const uint8_t* stg, int lane, int i) {
+    const int r = 8 * i + (lane >> 2), j = lane & 3;
+    return *reinterpret_cast<const uint4*>(stg + r * 64 + ((j ^ ((r >> 1) & 3)) << 4));
+}
+
+__device__ __forceinline__ uint4 pack8_bf16(const float* f) {
+    uint4 w;
+    w.x = pack_bf2(f[0], f[1]);
+    w.y = pack_bf2(f[2], f[3]);
+    w.z = pack_bf2(f[4], f[5]);
+    w.w = pack_bf2(f[6], f[7]);
+    return w;
+}
+
+// 32 bf16 per row (64 bytes) from this thread's row to rows row_base + 0..31
+// at column `col` of a bf16 [*, ldo] matrix.
+__device__ __forceinline__ void stg_store_bf16(uint8_t* stg, int lane, const uint4 (&v)[4],
+                                               bf16_t* out, int ldo, int row_base, int row_end,
+                                               int col) {
+    stg_put(stg, lane, v);
+    __syncwarp();
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint4 w = stg_get(stg, lane, i);
+        const int row = row_base + 8 * i + (lane >> 2);
+        if (row < row_end)
+            *reinterpret_cast<uint4*>(out + (size_t)row * ldo + col + (lane & 3) * 8) = w;
+    }
+    __syncwarp();
+}
+
+// The accumulator tile at tbase (this warp's 32 TMEM lanes = rows
+// row_base..row_base+31, 256 fp32 columns) -> the epilogue's output.
 template <int EPI>
-__device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int row_end, int n0,
+__device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int lane,
+                                              int row_base, int row_end, int n0,
                                               const GemmParams& p) {
-    const bool valid = row < row_end;
-    if constexpr (EPI == EPI_BF16 || EPI == EPI_F32) {
+    const int my_row = row_base + lane;
+    const bool valid = my_row < row_end;
+    if constexpr (EPI == EPI_BF16) {
 #pragma unroll 1
         for (int c = 0; c < 8; ++c) {
             uint32_t r[32];
             tmem_ld32(tbase + c * 32, r);
             tmem_ld_wait();
-            if (!valid) continue;
-            const int col = n0 + c * 32;
-            if constexpr (EPI == EPI_BF16) {
-                uint4* dst = reinterpret_cast<uint4*>(static_cast<bf16_t*>(p.out) +
-                                                      (size_t)row * p.ldo + col);
+            uint4 v[4];
 #pragma unroll
-                for (int v = 0; v < 4; ++v) {
-                    uint4 w;
-                    w.x = pack_bf2(__uint_as_float(r[8 * v + 0]), __uint_as_float(r[8 * v + 1]));
-                    w.y = pack_bf2(__uint_as_float(r[8 * v + 2]), __uint_as_float(r[8 * v + 3]));
-                    w.z = pack_bf2(__uint_as_float(r[8 * v + 4]), __uint_as_float(r[8 * v + 5]));
-                    w.w = pack_bf2(__uint_as_float(r[8 * v + 6]), __uint_as_float(r[8 * v + 7]));
-                    dst[v] = w;
-                }
-            } else if constexpr (EPI == EPI_F32) {
-                float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.out) +
-                                                        (size_t)row * p.ldo + col);
-#pragma unroll
-                for (int v = 0; v < 8; ++v)
-                    dst[v] = make_float4(__uint_as_float(r[4 * v]), __uint_as_float(r[4 * v + 1]),
-                                         __uint_as_float(r[4 * v + 2]),
-                                         __uint_as_float(r[4 * v + 3]));
-            }
+            for (int u = 0; u < 4; ++u) v[u] = pack8_bf16(reinterpret_cast<const float*>(r) + 8 * u);
+            stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
+                           n0 + c * 32);
         }
-    } else if constexpr (EPI == EPI_RESID) {
-        // x[row, n0 .. n0+256) += C: the residual row is read two 32-column
-        // chunks ahead of its use so its latency overlaps the TMEM reads and
-        // the stores of the chunks before it
-        float4* xrow = reinterpret_cast<float4*>(p.resid + (size_t)(valid ? row : 0) * p.ldr + n0);
-        float4 xa[8], xb[8];
-        if (valid) {
+    } else if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
+        // 16 fp32 columns (64 bytes) per staging pass; the residual of the
+        // next pass is loaded before this pass is staged
+        float* dst = EPI == EPI_RESID ? p.resid : static_cast<float*>(p.out);
+        const int ld = EPI == EPI_RESID ? p.ldr : p.ldo;
+        float4 xr[2][4];
+        auto load_resid = [&](int pass, float4 (&x)[4]) {
+            const int col = n0 + pass * 16 + (lane & 3) * 4;
 #pragma unroll
-            for (int v = 0; v < 8; ++v) {
-                xa[v] = xrow[v];
-                xb[v] = xrow[8 + v];
+            for (int i = 0; i < 4; ++i) {
+                const int row = row_base + 8 * i + (lane >> 2);
+                x[i] = row < row_end ? *reinterpret_cast<const float4*>(dst + (size_t)row * ld + col)
+                                     : make_float4(0.f, 0.f, 0.f, 0.f);
             }
-        }
+        };
+        if constexpr (EPI == EPI_RESID) load_resid(0, xr[0]);
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
             uint32_t r[32];
             tmem_ld32(tbase + c * 32, r);
             tmem_ld_wait();
-            float4(&cur)[8] = (c & 1) ? xb : xa;
-            if (valid) {
 #pragma unroll
-                for (int v = 0; v < 8; ++v) {
-                    cur[v].x += __uint_as_float(r[4 * v]);
-                    cur[v].y += __uint_as_float(r[4 * v + 1]);
-                    cur[v].z += __uint_as_float(r[4 * v + 2]);
-                    cur[v].w += __uint_as_float(r[4 * v + 3]);
-                    xrow[8 * c + v] = cur[v];
-                }
-                if (c + 2 < 8) {
+            for (int h = 0; h < 2; ++h) {
+                const int pass = 2 * c + h;
+                if constexpr (EPI == EPI_RESID)
+                    if (pass + 1 < 16) load_resid(pass + 1, xr[(pass + 1) & 1]);
+                uint4 v[4];
 #pragma unroll
-                    for (int v = 0; v < 8; ++v) cur[v] = xrow[8 * (c + 2) + v];
+                for (int u = 0; u < 4; ++u)
+                    v[u] = make_uint4(r[16 * h + 4 * u], r[16 * h + 4 * u + 1],
+                                      r[16 * h + 4 * u + 2], r[16 * h + 4 * u + 3]);
+                stg_put(stg, lane, v);
+                __syncwarp();
+                const int col = n0 + pass * 16 + (lane & 3) * 4;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const uint4 w = stg_get(stg, lane, i);
+                    const int row = row_base + 8 * i + (lane >> 2);
+                    float4 o = make_float4(__uint_as_float(w.x), __uint_as_float(w.y),
+                                           __uint_as_float(w.z), __uint_as_float(w.w));
+                    if constexpr (EPI == EPI_RESID) {
+                        const float4 x = xr[pass & 1][i];
+                        o.x += x.x;
+                        o.y += x.y;
+                        o.z += x.z;
+                        o.w += x.w;
+                    }
+                    if (row < row_end)
+                        *reinterpret_cast<float4*>(dst + (size_t)row * ld + col) = o;
                 }
+                __syncwarp();
             }
         }
     } else if constexpr (EPI == EPI_GLU) {
@@ -162,28 +213,23 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int row_e
             tmem_ld32(tbase + c * 32, g);
             tmem_ld32(tbase + (c + 4) * 32, u);
             tmem_ld_wait();
-            if (!valid) continue;
-            uint4* dst = reinterpret_cast<uint4*>(static_cast<bf16_t*>(p.out) +
-                                                  (size_t)row * p.ldo + n0 / 2 + c * 32);
+            uint4 v[4];
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {
+            for (int q = 0; q < 4; ++q) {
                 float o[8];
 #pragma unroll
                 for (int e = 0; e < 8; ++e)
-                    o[e] = act_fn(__uint_as_float(g[8 * v + e]), p.act) *
-                           __uint_as_float(u[8 * v + e]);
-                uint4 w;
-                w.x = pack_bf2(o[0], o[1]);
-                w.y = pack_bf2(o[2], o[3]);
-                w.z = pack_bf2(o[4], o[5]);
-                w.w = pack_bf2(o[6], o[7]);
-                dst[v] = w;
+                    o[e] = act_fn(__uint_as_float(g[8 * q + e]), p.act) *
+                           __uint_as_float(u[8 * q + e]);
+                v[q] = pack8_bf16(o);
             }
+            stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
+                           n0 / 2 + c * 32);
         }
     } else if constexpr (EPI == EPI_ROPE) {
         const int hc = p.hd / 64;  // 32-column chunks in half a head
         const int half = p.hd / 2;
-        const int pos = valid ? p.pos[row] : 0;
+        const int pos = valid ? p.pos[my_row] : 0;
 #pragma unroll 1
         for (int c = 0; c < 8; ++c) {
             const int hchunk = c % (2 * hc);
@@ -203,7 +249,6 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int row_e
             tmem_ld32(tbase + c * 32, lo);
             tmem_ld32(tbase + (c + hc) * 32, hi);
             tmem_ld_wait();
-            if (!valid) continue;
             float a[32], b[32];
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
@@ -220,23 +265,15 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, int row, int row_e
                     b[e] = x1 * cr + x0 * sr;
                 }
             }
-            bf16_t* base = static_cast<bf16_t*>(p.out) + (size_t)row * p.ldo;
-            uint4* d0 = reinterpret_cast<uint4*>(base + col);
-            uint4* d1 = reinterpret_cast<uint4*>(base + col + half);
+            uint4 v[4];
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {
-                uint4 w;
-                w.x = pack_bf2(a[8 * v + 0], a[8 * v + 1]);
-                w.y = pack_bf2(a[8 * v + 2], a[8 * v + 3]);
-                w.z = pack_bf2(a[8 * v + 4], a[8 * v + 5]);
-                w.w = pack_bf2(a[8 * v + 6], a[8 * v + 7]);
-                d0[v] = w;
-                w.x = pack_bf2(b[8 * v + 0], b[8 * v + 1]);
-                w.y = pack_bf2(b[8 * v + 2], b[8 * v + 3]);
-                w.z = pack_bf2(b[8 * v + 4], b[8 * v + 5]);
-                w.w = pack_bf2(b[8 * v + 6], b[8 * v + 7]);
-                d1[v] = w;
-            }
+            for (int q = 0; q < 4; ++q) v[q] = pack8_bf16(a + 8 * q);
+            stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
+                           col);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) v[q] = pack8_bf16(b + 8 * q);
+            stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
+                           col + half);
         }
     }
 }
@@ -452,20 +489,29 @@ __global__ void __launch_bounds__(192, 1)
         }
     } else {
         const int q = warp & 3;  // TMEM lane quarter this warp may access
+        // this warp's staging slot, after the barrier block
+        uint8_t* stg = reinterpret_cast<uint8_t*>(full) + 256 + (warp - 2) * 2048;
         int local = 0;
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
             const int acc = local & 1;
             const uint32_t acc_phase = (local >> 1) & 1;
             const TileGeo g = tile_geo<LORA>(tile, num_m, num_n, p, lg);
-            const int row = g.row0 + q * 32 + lane;
+            const int row_base = g.row0 + q * 32;
+            if constexpr (EPI == EPI_RESID) {
+                // bring this warp's residual rows of the tile into L2 while
+                // the accumulator is still being computed
+                const int row = row_base + lane;
+                if (row < g.row_end)
+                    l2_prefetch_bulk(p.resid + (size_t)row * p.ldr + g.nb * BN, BN * 4);
+            }
             if (!mbar_wait(&tfull[acc], acc_phase) || *abort_flag) {
                 *abort_flag = 1;
                 report(p.status, JNX_ERR_TIMEOUT);
                 break;
             }
             tc_fence_after();
-            epilogue_tile<EPI>(tmem_base + acc * BN + ((uint32_t)(q * 32) << 16), row, g.row_end,
-                               g.nb * BN, p);
+            epilogue_tile<EPI>(tmem_base + acc * BN + ((uint32_t)(q * 32) << 16), stg, lane,
+                               row_base, g.row_end, g.nb * BN, p);
             tc_fence_before();
             mbar_arrive(&tempty[acc]);
         }

@@ -97,6 +97,13 @@ __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)map) : "memory");
 }
 
+// Prefetch `bytes` (multiple of 16) at a 16-byte-aligned global address into
+// L2 (cp.async.bulk.prefetch: no destination, no completion to wait for).
+__device__ __forceinline__ void l2_prefetch_bulk(const void* src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"((uint64_t)src), "r"(bytes)
+                 : "memory");
+}
+
 // 2D tiled load: box at (x = inner element index, y = row) into smem,
 // completion signalled on `bar` as transaction bytes.
 __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, int32_t x,
