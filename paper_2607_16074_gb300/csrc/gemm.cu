@@ -120,15 +120,14 @@ __device__ __forceinline__ uint4 pack8_bf16(const float* f) {
 // at column `col` of a bf16 [*, ldo] matrix.
 __device__ __forceinline__ void stg_store_bf16(uint8_t* stg, int lane, const uint4 (&v)[4],
                                                bf16_t* out, int ldo, int row_base, int row_end,
-                                               int col) {
+                                               int col, uint64_t pol) {
     stg_put(stg, lane, v);
     __syncwarp();
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const uint4 w = stg_get(stg, lane, i);
         const int row = row_base + 8 * i + (lane >> 2);
-        if (row < row_end)
-            *reinterpret_cast<uint4*>(out + (size_t)row * ldo + col + (lane & 3) * 8) = w;
+        if (row < row_end) st_global_u4_hint(out + (size_t)row * ldo + col + (lane & 3) * 8, w, pol);
     }
     __syncwarp();
 }
@@ -141,6 +140,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                                               const GemmParams& p) {
     const int my_row = row_base + lane;
     const bool valid = my_row < row_end;
+    const uint64_t pol = l2_evict_first_policy();  // outputs and residual are streamed
     if constexpr (EPI == EPI_BF16) {
 #pragma unroll 1
         for (int c = 0; c < 8; ++c) {
@@ -151,24 +151,31 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
 #pragma unroll
             for (int u = 0; u < 4; ++u) v[u] = pack8_bf16(reinterpret_cast<const float*>(r) + 8 * u);
             stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
-                           n0 + c * 32);
+                           n0 + c * 32, pol);
         }
     } else if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
-        // 16 fp32 columns (64 bytes) per staging pass; the residual of the
-        // next pass is loaded before this pass is staged
+        // 16 fp32 columns (64 bytes) per staging pass; the residual is
+        // loaded RD - 1 passes ahead of its use, so several passes' loads
+        // are in flight while the accumulator is staged
+        constexpr int RD = 4;
         float* dst = EPI == EPI_RESID ? p.resid : static_cast<float*>(p.out);
         const int ld = EPI == EPI_RESID ? p.ldr : p.ldo;
-        float4 xr[2][4];
+        float4 xr[RD][4];
         auto load_resid = [&](int pass, float4 (&x)[4]) {
             const int col = n0 + pass * 16 + (lane & 3) * 4;
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int row = row_base + 8 * i + (lane >> 2);
-                x[i] = row < row_end ? *reinterpret_cast<const float4*>(dst + (size_t)row * ld + col)
-                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+                uint4 u = make_uint4(0u, 0u, 0u, 0u);
+                if (row < row_end) u = ld_global_u4_hint(dst + (size_t)row * ld + col, pol);
+                x[i] = make_float4(__uint_as_float(u.x), __uint_as_float(u.y),
+                                   __uint_as_float(u.z), __uint_as_float(u.w));
             }
         };
-        if constexpr (EPI == EPI_RESID) load_resid(0, xr[0]);
+        if constexpr (EPI == EPI_RESID) {
+#pragma unroll
+            for (int q = 0; q < RD - 1; ++q) load_resid(q, xr[q]);
+        }
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
             uint32_t r[32];
@@ -178,7 +185,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
             for (int h = 0; h < 2; ++h) {
                 const int pass = 2 * c + h;
                 if constexpr (EPI == EPI_RESID)
-                    if (pass + 1 < 16) load_resid(pass + 1, xr[(pass + 1) & 1]);
+                    if (pass + RD - 1 < 16) load_resid(pass + RD - 1, xr[(pass + RD - 1) % RD]);
                 uint4 v[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u)
@@ -194,14 +201,17 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                     float4 o = make_float4(__uint_as_float(w.x), __uint_as_float(w.y),
                                            __uint_as_float(w.z), __uint_as_float(w.w));
                     if constexpr (EPI == EPI_RESID) {
-                        const float4 x = xr[pass & 1][i];
+                        const float4 x = xr[pass % RD][i];
                         o.x += x.x;
                         o.y += x.y;
                         o.z += x.z;
                         o.w += x.w;
                     }
                     if (row < row_end)
-                        *reinterpret_cast<float4*>(dst + (size_t)row * ld + col) = o;
+                        st_global_u4_hint(dst + (size_t)row * ld + col,
+                                          make_uint4(__float_as_uint(o.x), __float_as_uint(o.y),
+                                                     __float_as_uint(o.z), __float_as_uint(o.w)),
+                                          pol);
                 }
                 __syncwarp();
             }
@@ -224,7 +234,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                 v[q] = pack8_bf16(o);
             }
             stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
-                           n0 / 2 + c * 32);
+                           n0 / 2 + c * 32, pol);
         }
     } else if constexpr (EPI == EPI_ROPE) {
         const int hc = p.hd / 64;  // 32-column chunks in half a head
@@ -269,11 +279,11 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
 #pragma unroll
             for (int q = 0; q < 4; ++q) v[q] = pack8_bf16(a + 8 * q);
             stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
-                           col);
+                           col, pol);
 #pragma unroll
             for (int q = 0; q < 4; ++q) v[q] = pack8_bf16(b + 8 * q);
             stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
-                           col + half);
+                           col + half, pol);
         }
     }
 }
@@ -497,13 +507,6 @@ __global__ void __launch_bounds__(192, 1)
             const uint32_t acc_phase = (local >> 1) & 1;
             const TileGeo g = tile_geo<LORA>(tile, num_m, num_n, p, lg);
             const int row_base = g.row0 + q * 32;
-            if constexpr (EPI == EPI_RESID) {
-                // bring this warp's residual rows of the tile into L2 while
-                // the accumulator is still being computed
-                const int row = row_base + lane;
-                if (row < g.row_end)
-                    l2_prefetch_bulk(p.resid + (size_t)row * p.ldr + g.nb * BN, BN * 4);
-            }
             if (!mbar_wait(&tfull[acc], acc_phase) || *abort_flag) {
                 *abort_flag = 1;
                 report(p.status, JNX_ERR_TIMEOUT);

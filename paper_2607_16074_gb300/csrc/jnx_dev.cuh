@@ -97,10 +97,28 @@ __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)map) : "memory");
 }
 
-// Prefetch `bytes` (multiple of 16) at a 16-byte-aligned global address into
-// L2 (cp.async.bulk.prefetch: no destination, no completion to wait for).
-__device__ __forceinline__ void l2_prefetch_bulk(const void* src, uint32_t bytes) {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"((uint64_t)src), "r"(bytes)
+// L2 eviction policy for data that is touched once (a streamed output, the
+// residual read-modify-write): its lines go first, so they do not push out
+// operand tiles that other CTAs are still reusing.
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+// 16-byte global load / store under an L2 cache policy; the load does not
+// allocate in L1.
+__device__ __forceinline__ uint4 ld_global_u4_hint(const void* p, uint64_t pol) {
+    uint4 v;
+    asm volatile("ld.global.L1::no_allocate.L2::cache_hint.v4.b32 {%0,%1,%2,%3}, [%4], %5;"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"((uint64_t)p), "l"(pol));
+    return v;
+}
+
+__device__ __forceinline__ void st_global_u4_hint(void* p, uint4 v, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.v4.b32 [%0], {%1,%2,%3,%4}, %5;" ::"l"((uint64_t)p),
+                 "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "l"(pol)
                  : "memory");
 }
 
