@@ -54,8 +54,8 @@ def workload_desc(w):
 # command are in profiles/), valid only for the GEMM source it was taken on.
 RECORDED_TRAFFIC = {
     # workload: (sha256 of csrc/gemm.cu, bytes per launch, profile)
-    "llama7b": ("aa55ebbd6ba7c078aa6df5362c97cf4cf77713a19804e1c9c53bda41f98263ce",
-                3.00e9 + 1.44e9, "profiles/gemm_gate_up_glu_llama7b_dram.md"),
+    "llama7b": ("53b6844e9af1004cc4be22948c8c6d683c8c9846040c420e5bae98210ada0a2b",
+                3.01e9 + 1.44e9, "profiles/gemm_gate_up_glu_llama7b_dram.md"),
 }
 
 

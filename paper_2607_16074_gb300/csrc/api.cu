@@ -238,6 +238,7 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
         p.ldo = qkvw;
         p.pos = g->pos_ids;
         p.rope = w.rope;
+        p.rope_ld = g->max_seqlen;
         p.rope_cols = (H + Hkv) * hd;
         p.hd = hd;
         p.status = w.status;
@@ -711,6 +712,7 @@ extern "C" jnx_status jnx_op_gemm(const uint16_t* A, const uint16_t* W, int32_t 
         if (st) return st;
         p.pos = pos;
         p.rope = tab;
+        p.rope_ld = max_pos;
         p.rope_cols = rope_cols;
         p.hd = head_dim;
     }

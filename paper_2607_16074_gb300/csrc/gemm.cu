@@ -246,14 +246,15 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
             if (hchunk >= hc) continue;  // handled with its lower partner
             const int col = n0 + c * 32;
             const bool rot = valid && col < p.rope_cols;
-            // (cos, sin) of this row's position, 16-byte loads issued before
-            // the TMEM read so their latency overlaps it
-            float4 cs[16];
+            // (cos, sin) of this row's position for the chunk's 32
+            // frequencies, loaded before the TMEM read so their latency
+            // overlaps it; the table is frequency-major, so the warp's rows
+            // (mostly consecutive positions) read consecutive entries
+            float2 cs[32];
             if (rot) {
-                const float4* src =
-                    reinterpret_cast<const float4*>(p.rope + (size_t)pos * half + hchunk * 32);
+                const float2* src = p.rope + (size_t)(hchunk * 32) * p.rope_ld + pos;
 #pragma unroll
-                for (int e = 0; e < 16; ++e) cs[e] = __ldg(src + e);
+                for (int e = 0; e < 32; ++e) cs[e] = __ldg(src + (size_t)e * p.rope_ld);
             }
             uint32_t lo[32], hi[32];
             tmem_ld32(tbase + c * 32, lo);
@@ -268,8 +269,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
             if (rot) {
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
-                    const float cr = (e & 1) ? cs[e >> 1].z : cs[e >> 1].x;
-                    const float sr = (e & 1) ? cs[e >> 1].w : cs[e >> 1].y;
+                    const float cr = cs[e].x, sr = cs[e].y;
                     const float x0 = a[e], x1 = b[e];
                     a[e] = x0 * cr - x1 * sr;
                     b[e] = x1 * cr + x0 * sr;

@@ -18,7 +18,8 @@ struct GemmParams {
     float* resid;         // EPI_RESID: fp32 [M, ldr], updated in place
     int ldr;
     const int* pos;       // EPI_ROPE: position of each row
-    const float2* rope;   // EPI_ROPE: (cos, sin) table [max_pos, hd/2]
+    const float2* rope;   // EPI_ROPE: (cos, sin) table [hd/2][rope_ld], frequency-major
+    int rope_ld;          // EPI_ROPE: positions per frequency row of the table (max_pos)
     int rope_cols;        // EPI_ROPE: columns [0, rope_cols) get RoPE
     int hd;               // EPI_ROPE: head dim (64, 128 or 256)
     int act;              // EPI_GLU: JNX_GLU_*

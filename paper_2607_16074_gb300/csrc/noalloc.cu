@@ -100,6 +100,7 @@ extern "C" jnx_status jnx_op_gemm_rope_noalloc(const uint16_t* A, const uint16_t
     p.ldo = ldo;
     p.pos = pos;
     p.rope = table;
+    p.rope_ld = max_pos;
     p.rope_cols = rope_cols;
     p.hd = head_dim;
     p.status = reinterpret_cast<int*>(scratch);

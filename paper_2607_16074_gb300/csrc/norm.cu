@@ -206,10 +206,13 @@ jnx_status final_pool_launch(const float* x, const uint16_t* gamma, float eps, c
 // RoPE table: (cos, sin) of pos * theta^(-2i/hd), evaluated in double and
 // rounded to fp32 once.
 // ---------------------------------------------------------------------------
+// (cos, sin) of position p at frequency i, stored frequency-major
+// (tab[i * max_pos + p]) so that rows of consecutive positions read
+// consecutive entries.
 __global__ void k_rope_table(float2* tab, int max_pos, int half, double theta) {
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= max_pos * half) return;
-    const int p = idx / half, i = idx % half;
+    const int i = idx / max_pos, p = idx % max_pos;
     const double inv = pow(theta, -2.0 * (double)i / (double)(2 * half));
     double sn, cs;
     sincos((double)p * inv, &sn, &cs);
