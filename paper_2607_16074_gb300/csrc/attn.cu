@@ -269,10 +269,14 @@ __global__ void __launch_bounds__(128, 1)
 //                 scores while the softmax warps work on the current ones
 //   warps 4+4t..  online softmax and epilogue, one query row per thread
 // and TMEM columns [256 t, 256 t + 256): S buffers at +0 and +BN, O at
-// +2 BN.  P (bf16) goes through shared memory as the K-major A operand of
-// the PV MMA; V is read as the MN-major B operand.  The two streams share
-// nothing but the tensor core, so one stream's softmax overlaps the other's
-// MMAs and copies, and a short tail tile costs only its own stream.
+// +2 BN.  P (bf16, two per 32-bit column) overwrites the first BN / 2
+// columns of the score buffer it was computed from and is the TMEM A
+// operand of the PV MMA; V is read from shared memory as the MN-major B
+// operand.  With two score buffers P is double-buffered too, so the softmax
+// of tile kt does not wait for PV(kt-1) (only a rare rescale of O does).
+// The two streams share nothing but the tensor core, so one stream's
+// softmax overlaps the other's MMAs and copies, and a short tail tile costs
+// only its own stream.
 //
 // The running max is lazy: a row raises the max m it subtracts only when a
 // new tile's max exceeds it by more than 8 (log2 units), so O is rarely
@@ -283,15 +287,19 @@ __global__ void __launch_bounds__(128, 1)
 //   k_full[2], k_empty[2]    K ring (a slot frees when its S MMA completes)
 //   v_full[2], v_empty[2]    V ring (a slot frees when its PV MMA completes)
 //   s_full[2]                score buffer b holds a new S
-//   p_full                   P(kt) written and its S read (128 arrivals)
-//   o_done                   a PV MMA completed
+//   p_full[2]                P of a tile written over its S in score
+//                            buffer b (128 arrivals)
+//   o_done[2]                PV of a tile with score buffer b completed; a
+//                            softmax thread waits for PV(g-2) before it
+//                            arrives for tile g, so neither barrier runs two
+//                            phases ahead of a waiter
 //   o_free                   the epilogue has read O (128 arrivals)
 //   drain                    all MMAs of the stream completed (teardown)
 // ---------------------------------------------------------------------------
 namespace attn_ws {
 constexpr int BM = 128;        // query rows per item
 constexpr float kLazy = 8.0f;  // log2 growth of the max that forces a rescale
-constexpr int kBars = 16;      // barriers per stream
+constexpr int kBars = 18;      // barriers per stream
 }  // namespace attn_ws
 
 // Work items: an explicit (sample, query tile) list, or, without one, every
@@ -302,19 +310,33 @@ struct AttnItems {
     int S;
 };
 
-__device__ __forceinline__ bool attn_item(const AttnItems& it, const int* __restrict__ cu, int H,
-                                          int w, int& s, int& qt, int& h) {
-    h = w % H;
+// One work item: query tile qt of the sample at packed rows [start,
+// start + L), head h.  Fetched one item ahead by every role so that the
+// list and cu_seqlens loads of the next item overlap the current one.
+struct AttnWork {
+    int qt, h, start, L;
+    bool valid;  // false past the end, or for an empty enumerated item
+};
+
+__device__ __forceinline__ AttnWork attn_fetch(const AttnItems& it, const int* __restrict__ cu,
+                                               int H, int w, int n_work) {
+    AttnWork a{0, 0, 0, 0, false};
+    if (w >= n_work) return a;
+    a.h = w % H;
     const int i = w / H;
+    int s;
     if (it.list) {
         const int2 e = it.list[i];
         s = e.x;
-        qt = e.y;
-        return true;
+        a.qt = e.y;
+    } else {
+        a.qt = i / it.S;
+        s = i % it.S;
     }
-    qt = i / it.S;
-    s = i % it.S;
-    return qt * attn_ws::BM < cu[s + 1] - cu[s];
+    a.start = cu[s];
+    a.L = cu[s + 1] - a.start;
+    a.valid = a.qt * attn_ws::BM < a.L;
+    return a;
 }
 
 template <int HD, int BN>
@@ -324,11 +346,9 @@ struct AttnWsCfg {
     static constexpr int BM = attn_ws::BM;
     static constexpr int QB = BM * HD * 2;  // Q tile
     static constexpr int KB = BN * HD * 2;  // one K (or V) tile
-    static constexpr int PB = BM * BN * 2;  // P tile
     static constexpr int OFF_K = QB;
     static constexpr int OFF_V = OFF_K + 2 * KB;
-    static constexpr int OFF_P = OFF_V + 2 * KB;
-    static constexpr int STREAM = OFF_P + PB;  // bytes per stream (multiple of 1024)
+    static constexpr int STREAM = OFF_V + 2 * KB;  // bytes per stream (multiple of 1024)
     static constexpr int OFF_BAR = 2 * STREAM;
     static constexpr int SMEM = OFF_BAR + 2 * attn_ws::kBars * 8 + 16 + 1024;
     static_assert(STREAM % 1024 == 0, "128B-swizzled tiles need 1024-byte alignment");
@@ -344,7 +364,11 @@ template <int BN, bool FULL>
 __device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float scale_log2,
                                                 bool first, float& m, float& alpha, float& rs,
                                                 uint32_t (&pk)[BN / 2]) {
-    float mx = -INFINITY;
+    // both passes reduce into 4 independent partial results (then a tree),
+    // so the max and the sum are not one 64-long dependent chain
+    float mx4[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) mx4[j] = -INFINITY;
 #pragma unroll
     for (int c = 0; c < BN / 32; ++c) {
         uint32_t v[32];
@@ -352,8 +376,9 @@ __device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float s
         tmem_ld_wait();
 #pragma unroll
         for (int e = 0; e < 32; ++e)
-            if (FULL || c * 32 + e < kvalid) mx = fmaxf(mx, __uint_as_float(v[e]));
+            if (FULL || c * 32 + e < kvalid) mx4[e & 3] = fmaxf(mx4[e & 3], __uint_as_float(v[e]));
     }
+    float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
     mx *= scale_log2;
     alpha = 1.f;
     if (first) {
@@ -363,7 +388,9 @@ __device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float s
         m = mx;
     }
     const float nm = -m;
-    rs = 0.f;
+    float rs4[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) rs4[j] = 0.f;
 #pragma unroll
     for (int c = 0; c < BN / 32; ++c) {
         uint32_t v[32];
@@ -377,10 +404,11 @@ __device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float s
                 if (c * 32 + e >= kvalid) p0 = 0.f;
                 if (c * 32 + e + 1 >= kvalid) p1 = 0.f;
             }
-            rs += p0 + p1;
+            rs4[(e >> 1) & 3] += p0 + p1;
             pk[c * 16 + e / 2] = pack_bf2(p0, p1);
         }
     }
+    rs = (rs4[0] + rs4[1]) + (rs4[2] + rs4[3]);
 }
 
 template <int HD, int BN>
@@ -404,7 +432,6 @@ __global__ void __launch_bounds__(384, 1)
     uint8_t* sQ = st;
     auto sK = [&](int b) { return st + C::OFF_K + b * C::KB; };
     auto sV = [&](int b) { return st + C::OFF_V + b * C::KB; };
-    uint8_t* sP = st + C::OFF_P;
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR) + t * attn_ws::kBars;
     uint64_t* q_full = bars + 0;
     uint64_t* q_empty = bars + 1;
@@ -413,21 +440,21 @@ __global__ void __launch_bounds__(384, 1)
     uint64_t* v_full = bars + 6;   // [2]
     uint64_t* v_empty = bars + 8;  // [2]
     uint64_t* s_full = bars + 10;  // [2]
-    uint64_t* p_full = bars + 12;
-    uint64_t* o_done = bars + 13;
-    uint64_t* o_free = bars + 14;
-    uint64_t* drain = bars + 15;
+    uint64_t* p_full = bars + 12;  // [2]
+    uint64_t* o_done = bars + 14;  // [2]
+    uint64_t* o_free = bars + 16;
+    uint64_t* drain = bars + 17;
 
     const int n_work = items.n * H;
     const int group = H / Hkv;
     const int w0 = 2 * blockIdx.x + t, dw = 2 * gridDim.x;
     if (tid == 0) {
-        // both streams' barriers: one arrival each, but p_full and o_free,
+        // both streams' barriers: one arrival each, but p_full[] and o_free,
         // which every softmax thread of the stream arrives on
         uint64_t* all = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR);
         for (int i = 0; i < 2 * attn_ws::kBars; ++i) {
             const int k = i % attn_ws::kBars;
-            mbar_init(&all[i], (k == 12 || k == 14) ? BM : 1);
+            mbar_init(&all[i], (k == 12 || k == 13 || k == 16) ? BM : 1);
         }
         *fail_flag = 0;
         fence_barrier_init();
@@ -462,10 +489,12 @@ __global__ void __launch_bounds__(384, 1)
                 ++g;
                 return true;
             };
+            AttnWork nxt = attn_fetch(items, cu, H, w0, n_work);
             for (int w = w0; w < n_work && ok && !*fail_flag; w += dw) {
-                int s, qt, h;
-                if (!attn_item(items, cu, H, w, s, qt, h)) continue;
-                const int start = cu[s], L = cu[s + 1] - start;
+                const AttnWork a = nxt;
+                nxt = attn_fetch(items, cu, H, w + dw, n_work);
+                if (!a.valid) continue;
+                const int start = a.start, L = a.L, qt = a.qt, h = a.h;
                 const int n_kt = (L + BN - 1) / BN;
                 const int kvh = h / group;
                 if (nq > 0 && !(ok = mbar_wait(q_empty, (nq - 1) & 1))) break;
@@ -500,7 +529,7 @@ __global__ void __launch_bounds__(384, 1)
             int nq = 0;                  // Q tiles consumed
             uint32_t gk = 0, gv = 0;     // K / V tiles consumed
             uint32_t gs = 0;             // S tiles issued (score buffer gs & 1)
-            uint32_t gp = 0;             // p_full completions consumed
+            uint32_t gp = 0;             // p_full completions consumed = PVs issued
             int items_done = 0;
             auto issue_s = [&](const uint32_t qa) -> bool {
                 const int b = gk & 1;
@@ -520,11 +549,12 @@ __global__ void __launch_bounds__(384, 1)
                 issued = true;
                 return true;
             };
+            AttnWork nxt = attn_fetch(items, cu, H, w0, n_work);
             for (int w = w0; w < n_work && ok && !*fail_flag; w += dw) {
-                int s, qt, h;
-                if (!attn_item(items, cu, H, w, s, qt, h)) continue;
-                const int L = cu[s + 1] - cu[s];
-                const int n_kt = (L + BN - 1) / BN;
+                const AttnWork a = nxt;
+                nxt = attn_fetch(items, cu, H, w + dw, n_work);
+                if (!a.valid) continue;
+                const int n_kt = (a.L + BN - 1) / BN;
                 if (!(ok = mbar_wait(q_full, nq & 1))) break;
                 ++nq;
                 tc_fence_after();
@@ -534,8 +564,9 @@ __global__ void __launch_bounds__(384, 1)
                 ok = issue_s(qa) && (n_kt < 2 || issue_s(qa));
                 if (ok && n_kt <= 2) tc_commit(q_empty);
                 for (int kt = 0; kt < n_kt && ok; ++kt) {
-                    // P(kt) is out and S(kt) read
-                    if (!(ok = mbar_wait(p_full, gp & 1))) break;
+                    // P(kt) is in TMEM, over S(kt) in score buffer gp & 1
+                    const uint32_t pb = gp & 1;
+                    if (!(ok = mbar_wait(&p_full[pb], (gp >> 1) & 1))) break;
                     ++gp;
                     // the first PV of an item overwrites O: the previous
                     // item's epilogue must have read it
@@ -544,17 +575,18 @@ __global__ void __launch_bounds__(384, 1)
                     const int b = gv & 1;
                     if (!(ok = mbar_wait(&v_full[b], (gv >> 1) & 1))) break;
                     tc_fence_after();
-                    const uint32_t pa = smem_u32(sP), va = smem_u32(sV(b));
+                    const uint32_t pa = tbase + pb * BN, va = smem_u32(sV(b));
 #pragma unroll
-                    for (int ks = 0; ks < BN / 16; ++ks)
-                        tc_mma_f16(tbase + C::O_COL,
-                                   sw128_desc(pa + (ks >> 2) * BM * 128 + (ks & 3) * 32),
-                                   sw128_desc_mn(va + ks * 16 * 128, BN * 128, 1024), IDESC_PV,
-                                   kt > 0 || ks > 0);
-                    tc_commit(o_done);
+                    for (int ks = 0; ks < BN / 16; ++ks)  // 16 keys = 8 TMEM columns of P
+                        tc_mma_f16_ts(tbase + C::O_COL, pa + ks * 8,
+                                      sw128_desc_mn(va + ks * 16 * 128, BN * 128, 1024), IDESC_PV,
+                                      kt > 0 || ks > 0);
+                    tc_commit(&o_done[pb]);
                     tc_commit(&v_empty[b]);
                     ++gv;
-                    // S(kt + 2) reuses the score buffer of S(kt)
+                    // S(kt + 2) reuses the score buffer of S(kt) / P(kt): the
+                    // tensor core runs this thread's MMAs in issue order, so
+                    // PV(kt) has read P(kt) before S(kt + 2) lands there
                     if (kt + 2 < n_kt) {
                         ok = issue_s(qa);
                         if (ok && kt + 3 == n_kt) tc_commit(q_empty);
@@ -574,13 +606,26 @@ __global__ void __launch_bounds__(384, 1)
         const int r = quarter * 32 + lane;
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
         const uint32_t tO = tbase + lane_base + C::O_COL;
-        uint32_t gs = 0, nd = 0;  // S tiles / o_done completions consumed
+        uint32_t gs = 0;  // S tiles consumed
+        uint32_t nw = 0;  // PVs this thread has seen complete (in order)
+        // wait until PV(0 .. upto-1) of this stream have completed
+        auto wait_pv = [&](uint32_t upto) -> bool {
+            for (; nw < upto; ++nw)
+                if (!__all_sync(0xffffffffu, mbar_wait(&o_done[nw & 1], (nw >> 1) & 1)))
+                    return false;
+            tc_fence_after();
+            return true;
+        };
         bool ok = true;
+        AttnWork nxt = attn_fetch(items, cu, H, w0, n_work);
         for (int w = w0; w < n_work && ok; w += dw) {
             if (__any_sync(0xffffffffu, *fail_flag != 0)) break;
-            int s, qt, h;
-            if (!attn_item(items, cu, H, w, s, qt, h)) continue;
-            const int start = cu[s], L = cu[s + 1] - start;
+            const AttnWork a = nxt;
+            if (!a.valid) {
+                nxt = attn_fetch(items, cu, H, w + dw, n_work);
+                continue;
+            }
+            const int start = a.start, L = a.L, qt = a.qt, h = a.h;
             const int n_kt = (L + BN - 1) / BN;
             float m = 0.f, l = 0.f;
             for (int kt = 0; kt < n_kt; ++kt) {
@@ -589,7 +634,7 @@ __global__ void __launch_bounds__(384, 1)
                     break;
                 tc_fence_after();
                 const uint32_t tS = tbase + lane_base + (gs & 1) * BN;
-                ++gs;
+                const uint32_t g = gs++;  // stream-wide index of this tile
                 const int kvalid = L - kt * BN;  // keys of this tile inside the sample
                 uint32_t pk[BN / 2];
                 float alpha, rs;
@@ -597,12 +642,10 @@ __global__ void __launch_bounds__(384, 1)
                     attn_ws_softmax<BN, true>(tS, kvalid, scale_log2, kt == 0, m, alpha, rs, pk);
                 else
                     attn_ws_softmax<BN, false>(tS, kvalid, scale_log2, kt == 0, m, alpha, rs, pk);
-                if (kt > 0) {
-                    // PV(kt-1) must be done before O is rescaled and P rewritten
-                    if (!(ok = __all_sync(0xffffffffu, mbar_wait(o_done, nd & 1)))) break;
-                    ++nd;
-                    tc_fence_after();
-                    if (__any_sync(0xffffffffu, alpha < 1.f)) {
+                if (kt > 0 && __any_sync(0xffffffffu, alpha < 1.f)) {
+                    // rescaling O needs every earlier PV of the item done
+                    if (!(ok = wait_pv(g))) break;
+                    {
 #pragma unroll 1
                         for (int c = 0; c < HD / 32; ++c) {
                             uint32_t v[32];
@@ -617,41 +660,48 @@ __global__ void __launch_bounds__(384, 1)
                     }
                 }
                 l = l * alpha + rs;
-                uint8_t* prow = sP + r * 128;
-#pragma unroll
-                for (int u = 0; u < BN / 8; ++u)
-                    *reinterpret_cast<uint4*>(prow + (u >> 3) * BM * 128 +
-                                              (((u & 7) ^ (r & 7)) << 4)) =
-                        make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
-                fence_proxy_async();  // P visible to the tensor core
+                // keeps o_done[b] within one phase of this thread's waits
+                if (g >= 2 && !(ok = wait_pv(g - 1))) break;
+                static_assert(BN / 2 == 32, "P of one row is one 32-column TMEM store");
+                tmem_st32(tS, pk);
+                tmem_st_wait();
                 tc_fence_before();
-                mbar_arrive(p_full);
+                mbar_arrive(&p_full[g & 1]);
             }
             if (!ok) break;
-            // epilogue: O / l -> bf16
-            if (!(ok = __all_sync(0xffffffffu, mbar_wait(o_done, nd & 1)))) break;
-            ++nd;
-            tc_fence_after();
+            // the next item's loads overlap this epilogue (fetched here, not
+            // at the top, so they hold no registers during the key loop)
+            nxt = attn_fetch(items, cu, H, w + dw, n_work);
+            // epilogue: O / l -> bf16 once the item's last PV is done
+            if (!(ok = wait_pv(gs))) break;
             const float inv = 1.0f / l;
-            uint32_t ob[HD / 2];
-#pragma unroll
-            for (int c = 0; c < HD / 32; ++c) {
-                uint32_t v[32];
-                tmem_ld32(tO + c * 32, v);
-                tmem_ld_wait();
-#pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    ob[c * 16 + e] = pack_bf2(__uint_as_float(v[2 * e]) * inv,
-                                              __uint_as_float(v[2 * e + 1]) * inv);
-            }
-            tc_fence_before();
-            mbar_arrive(o_free);
             const int row = qt * BM + r;
-            if (row < L) {
-                uint4* dst = reinterpret_cast<uint4*>(out + (size_t)(start + row) * ldo + h * HD);
+            uint4* dst = reinterpret_cast<uint4*>(out + (size_t)(start + row) * ldo + h * HD);
+            // 64 columns at a time; O is released (o_free) once its last
+            // columns are in registers
 #pragma unroll
-                for (int q = 0; q < HD / 8; ++q)
-                    dst[q] = make_uint4(ob[4 * q], ob[4 * q + 1], ob[4 * q + 2], ob[4 * q + 3]);
+            for (int half = 0; half < HD / 64; ++half) {
+                uint32_t ob[32];
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {
+                    uint32_t v[32];
+                    tmem_ld32(tO + (2 * half + c) * 32, v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int e = 0; e < 16; ++e)
+                        ob[c * 16 + e] = pack_bf2(__uint_as_float(v[2 * e]) * inv,
+                                                  __uint_as_float(v[2 * e + 1]) * inv);
+                }
+                if (half == HD / 64 - 1) {
+                    tc_fence_before();
+                    mbar_arrive(o_free);
+                }
+                if (row < L) {
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        dst[8 * half + q] =
+                            make_uint4(ob[4 * q], ob[4 * q + 1], ob[4 * q + 2], ob[4 * q + 3]);
+                }
             }
         }
         if (!ok) *fail_flag = 1;
