@@ -339,6 +339,21 @@ __device__ __forceinline__ AttnWork attn_fetch(const AttnItems& it, const int* _
     return a;
 }
 
+// Epilogue staging (as in the GEMM epilogue): thread `lane` puts its row's
+// 64 bytes; in step i thread `lane` gets row 8 i + lane / 4, 16-byte unit
+// lane % 4.  Units are XOR-swizzled by (row / 2) % 4 (no bank conflicts).
+__device__ __forceinline__ void attn_stg_put(uint8_t* stg, int lane, const uint4 (&v)[4]) {
+    uint8_t* rowp = stg + lane * 64;
+    const int sw = (lane >> 1) & 3;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) *reinterpret_cast<uint4*>(rowp + ((j ^ sw) << 4)) = v[j];
+}
+
+__device__ __forceinline__ uint4 attn_stg_get(const uint8_t* stg, int lane, int i) {
+    const int r = 8 * i + (lane >> 2), j = lane & 3;
+    return *reinterpret_cast<const uint4*>(stg + r * 64 + ((j ^ ((r >> 1) & 3)) << 4));
+}
+
 template <int HD, int BN>
 struct AttnWsCfg {
     static_assert(BN == 64, "key tile of 64 keys");
@@ -349,7 +364,8 @@ struct AttnWsCfg {
     static constexpr int OFF_K = QB;
     static constexpr int OFF_V = OFF_K + 2 * KB;
     static constexpr int STREAM = OFF_V + 2 * KB;  // bytes per stream (multiple of 1024)
-    static constexpr int OFF_BAR = 2 * STREAM;
+    static constexpr int OFF_STG = 2 * STREAM;   // epilogue staging, 2 KB per softmax warp
+    static constexpr int OFF_BAR = OFF_STG + 8 * 2048;
     static constexpr int SMEM = OFF_BAR + 2 * attn_ws::kBars * 8 + 16 + 1024;
     static_assert(STREAM % 1024 == 0, "128B-swizzled tiles need 1024-byte alignment");
     static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
@@ -360,25 +376,60 @@ struct AttnWsCfg {
 // Softmax of one 128 x BN score tile for this thread's row: row max (pass
 // 1), then probabilities packed as bf16 pairs (pass 2).  FULL: every key of
 // the tile lies inside the sample (no mask).
+// 2^x for a pair of arguments on the FMA pipe instead of the MUFU pipe
+// (range reduction plus a polynomial, as in common libm exp2 designs):
+// j = rint(x) by adding 1.5 * 2^23, f = x - j in [-0.5, 0.5], 2^f by a
+// degree-3 polynomial fitted for minimum maximum relative error on that
+// interval (below 8e-5, under the 2^-9 rounding that P gets in bf16), and
+// j added into the exponent field.  x is clamped at -126 so the exponent
+// cannot wrap; such a p (below 2^-126) is negligible next to the row's
+// largest p (at least 2^-8).
+__device__ __forceinline__ void ex2_poly2(float x0, float x1, float& p0, float& p1) {
+    const uint64_t magic = f2_pack(12582912.f, 12582912.f);
+    const uint64_t nmagic = f2_pack(-12582912.f, -12582912.f);
+    const uint64_t x = f2_pack(fmaxf(x0, -126.f), fmaxf(x1, -126.f));
+    const uint64_t t = f2_add(x, magic);                            // j in the low mantissa bits
+    const uint64_t f = f2_fma(f2_add(t, nmagic), f2_pack(-1.f, -1.f), x);  // x - j
+    uint64_t q = f2_pack(0.055174146f, 0.055174146f);
+    q = f2_fma(q, f, f2_pack(0.24261758f, 0.24261758f));
+    q = f2_fma(q, f, f2_pack(0.69326109f, 0.69326109f));
+    q = f2_fma(q, f, f2_pack(0.99992758f, 0.99992758f));
+    float t0, t1, q0, q1;
+    f2_unpack(t, t0, t1);
+    f2_unpack(q, q0, q1);
+    p0 = __uint_as_float(__float_as_uint(q0) + (__float_as_uint(t0) << 23));
+    p1 = __uint_as_float(__float_as_uint(q1) + (__float_as_uint(t1) << 23));
+}
+
 template <int BN, bool FULL>
 __device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float scale_log2,
                                                 bool first, float& m, float& alpha, float& rs,
                                                 uint32_t (&pk)[BN / 2]) {
-    // both passes reduce into 4 independent partial results (then a tree),
-    // so the max and the sum are not one 64-long dependent chain
+    static_assert(BN == 64, "one S row is two 32-column TMEM loads");
+    // the whole S row in one TMEM round trip
+    uint32_t v[2][32];
+    tmem_ld32(tS, v[0]);
+    tmem_ld32(tS + 32, v[1]);
+    tmem_ld_wait();
+    // row max into 4 independent partial results (then a tree), so it is not
+    // one 64-long dependent chain; full tiles take two keys per instruction
     float mx4[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) mx4[j] = -INFINITY;
 #pragma unroll
-    for (int c = 0; c < BN / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(tS + c * 32, v);
-        tmem_ld_wait();
+    for (int c = 0; c < 2; ++c)
 #pragma unroll
-        for (int e = 0; e < 32; ++e)
-            if (FULL || c * 32 + e < kvalid) mx4[e & 3] = fmaxf(mx4[e & 3], __uint_as_float(v[e]));
-    }
-    float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+        for (int e = 0; e < 32; e += 2) {
+            const float a0 = __uint_as_float(v[c][e]), a1 = __uint_as_float(v[c][e + 1]);
+            float& acc = mx4[(e >> 1) & 3];
+            if (FULL) {
+                acc = fmax3(acc, a0, a1);
+            } else {
+                if (c * 32 + e < kvalid) acc = fmaxf(acc, a0);
+                if (c * 32 + e + 1 < kvalid) acc = fmaxf(acc, a1);
+            }
+        }
+    float mx = fmax3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3]));
     mx *= scale_log2;
     alpha = 1.f;
     if (first) {
@@ -387,28 +438,38 @@ __device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float s
         alpha = ex2_approx(m - mx);
         m = mx;
     }
-    const float nm = -m;
-    float rs4[4];
+    // p = 2^(s scale - m): the argument of two keys per packed FMA, the row
+    // sum in two packed partial sums
+    const uint64_t sc2 = f2_pack(scale_log2, scale_log2), nm2 = f2_pack(-m, -m);
+    uint64_t rs2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
 #pragma unroll
-    for (int j = 0; j < 4; ++j) rs4[j] = 0.f;
-#pragma unroll
-    for (int c = 0; c < BN / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(tS + c * 32, v);
-        tmem_ld_wait();
+    for (int c = 0; c < 2; ++c)
 #pragma unroll
         for (int e = 0; e < 32; e += 2) {
-            float p0 = ex2_approx(fmaf(__uint_as_float(v[e]), scale_log2, nm));
-            float p1 = ex2_approx(fmaf(__uint_as_float(v[e + 1]), scale_log2, nm));
+            float x0, x1;
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(v[c][e]), __uint_as_float(v[c][e + 1])), sc2,
+                             nm2),
+                      x0, x1);
+            float p0, p1;
+            // on full tiles one pair in four goes to the FMA pipe, which
+            // relieves the MUFU pipe the two streams' softmax warps share
+            if (FULL && ((e >> 1) & 3) == 3) {
+                ex2_poly2(x0, x1, p0, p1);
+            } else {
+                p0 = ex2_approx(x0);
+                p1 = ex2_approx(x1);
+            }
             if (!FULL) {
                 if (c * 32 + e >= kvalid) p0 = 0.f;
                 if (c * 32 + e + 1 >= kvalid) p1 = 0.f;
             }
-            rs4[(e >> 1) & 3] += p0 + p1;
+            rs2[(e >> 1) & 1] = f2_add(rs2[(e >> 1) & 1], f2_pack(p0, p1));
             pk[c * 16 + e / 2] = pack_bf2(p0, p1);
         }
-    }
-    rs = (rs4[0] + rs4[1]) + (rs4[2] + rs4[3]);
+    float r0, r1, r2, r3;
+    f2_unpack(rs2[0], r0, r1);
+    f2_unpack(rs2[1], r2, r3);
+    rs = (r0 + r1) + (r2 + r3);
 }
 
 template <int HD, int BN>
@@ -603,7 +664,6 @@ __global__ void __launch_bounds__(384, 1)
     } else {
         // ---------------- softmax + epilogue of stream t ----------------
         const int quarter = warp & 3;  // TMEM lanes this warp may access
-        const int r = quarter * 32 + lane;
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
         const uint32_t tO = tbase + lane_base + C::O_COL;
         uint32_t gs = 0;  // S tiles consumed
@@ -675,33 +735,47 @@ __global__ void __launch_bounds__(384, 1)
             // epilogue: O / l -> bf16 once the item's last PV is done
             if (!(ok = wait_pv(gs))) break;
             const float inv = 1.0f / l;
-            const int row = qt * BM + r;
-            uint4* dst = reinterpret_cast<uint4*>(out + (size_t)(start + row) * ldo + h * HD);
-            // 64 columns at a time; O is released (o_free) once its last
-            // columns are in registers
+            // 32 columns at a time through this warp's staging slot, so each
+            // store instruction writes 8 rows x 64 contiguous bytes; O is
+            // released (o_free) once its last columns are in registers
+            uint8_t* stg = sm + C::OFF_STG + (warp - 4) * 2048;
+            const int row0 = qt * BM + quarter * 32;  // first row of this warp
+            // the TMEM load of chunk c + 1 is in flight while chunk c is
+            // converted and stored
+            uint32_t ov[2][32];
+            tmem_ld32(tO, ov[0]);
 #pragma unroll
-            for (int half = 0; half < HD / 64; ++half) {
-                uint32_t ob[32];
-#pragma unroll
-                for (int c = 0; c < 2; ++c) {
-                    uint32_t v[32];
-                    tmem_ld32(tO + (2 * half + c) * 32, v);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int e = 0; e < 16; ++e)
-                        ob[c * 16 + e] = pack_bf2(__uint_as_float(v[2 * e]) * inv,
-                                                  __uint_as_float(v[2 * e + 1]) * inv);
-                }
-                if (half == HD / 64 - 1) {
+            for (int c = 0; c < HD / 32; ++c) {
+                uint32_t(&v)[32] = ov[c & 1];
+                tmem_ld_wait_regs(v);
+                if (c + 1 < HD / 32) {
+                    tmem_ld32(tO + (c + 1) * 32, ov[(c + 1) & 1]);
+                } else {
                     tc_fence_before();
                     mbar_arrive(o_free);
                 }
-                if (row < L) {
+                uint4 q4[4];
 #pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        dst[8 * half + q] =
-                            make_uint4(ob[4 * q], ob[4 * q + 1], ob[4 * q + 2], ob[4 * q + 3]);
+                for (int u = 0; u < 4; ++u)
+                    q4[u] = make_uint4(pack_bf2(__uint_as_float(v[8 * u]) * inv,
+                                                __uint_as_float(v[8 * u + 1]) * inv),
+                                       pack_bf2(__uint_as_float(v[8 * u + 2]) * inv,
+                                                __uint_as_float(v[8 * u + 3]) * inv),
+                                       pack_bf2(__uint_as_float(v[8 * u + 4]) * inv,
+                                                __uint_as_float(v[8 * u + 5]) * inv),
+                                       pack_bf2(__uint_as_float(v[8 * u + 6]) * inv,
+                                                __uint_as_float(v[8 * u + 7]) * inv));
+                attn_stg_put(stg, lane, q4);
+                __syncwarp();
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int rr = 8 * i + (lane >> 2);
+                    const uint4 w4 = attn_stg_get(stg, lane, i);
+                    if (row0 + rr < L)
+                        *reinterpret_cast<uint4*>(out + (size_t)(start + row0 + rr) * ldo + h * HD +
+                                                  c * 32 + (lane & 3) * 8) = w4;
                 }
+                __syncwarp();
             }
         }
         if (!ok) *fail_flag = 1;
