@@ -273,31 +273,20 @@ def run_ours(args, rank, world, local_rank):
     value = job_tokens_per_s(tokens, world, args.steps, t_ms)
 
     # ---- end to end through the C ABI from pinned host memory --------------
-    vis_d, tid_d, tgt_d = inp["vision"], inp["text_ids"], inp["targets"]
-    loss_h = torch.empty(step.loss.shape, dtype=torch.float32).pin_memory()
-    preds_h = torch.empty(preds.shape, dtype=torch.float32).pin_memory()
+    # Every step plans its group on the host, copies its inputs from pinned
+    # host memory and reads its loss and predictions back; StepPipeline
+    # overlaps step i+1's planning and input copy with step i.
     h2d = sum(t.numel() * t.element_size() for t in inp_host.values())
-    d2h = loss_h.numel() * 4 + preds_h.numel() * 4
-
-    def e2e_step():
-        vis_d.copy_(inp_host["vision"], non_blocking=True)
-        tid_d.copy_(inp_host["text_ids"], non_blocking=True)
-        tgt_d.copy_(inp_host["targets"], non_blocking=True)
-        p = J.jnx_group_plan(w.schemas(), reqs, len(w.tenants), w.max_samples, w.max_tokens)
-        g = R.DeviceGroup(p, device=dev, non_blocking=True)
-        step.group = g
-        step.run(vis_d, tid_d, tgt_d, preds)
-        loss_h.copy_(step.loss, non_blocking=True)
-        preds_h.copy_(preds, non_blocking=True)
-        torch.cuda.current_stream().synchronize()
-        return g
-
-    keep = e2e_step()
+    d2h = step.loss.numel() * 4 + preds.numel() * 4
+    pipe = R.StepPipeline(step, inp["vision"].shape[0], inp["text_ids"].numel(),
+                          tuple(inp["targets"].shape), device=dev)
+    plan_fn = lambda i: J.jnx_group_plan(w.schemas(), reqs, len(w.tenants), w.max_samples,
+                                         w.max_tokens)
+    pipe.run([inp_host] * 2, plan_fn)  # warm-up of the pipeline's own buffers
     barrier()
     torch.cuda.synchronize()
     t0 = time.perf_counter()
-    for _ in range(args.steps):
-        keep = e2e_step()
+    pipe.run([inp_host] * args.steps, plan_fn)
     torch.cuda.synchronize()
     barrier()
     e2e_ms = max_over_ranks((time.perf_counter() - t0) * 1e3, world, dev)

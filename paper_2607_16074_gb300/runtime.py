@@ -175,3 +175,95 @@ class GroupedStep:
         self.heads.forward(self.group, self.pooled, self.hidden, targets, preds, self.loss,
                            self.ws_h, stream)
         self.heads.backward(self.group, self.pooled, self.hidden, targets, self.ws_h, stream)
+
+
+class StepPipeline:
+    """Grouped steps fed from pinned host memory, each step's preparation
+    overlapped with the step before it.
+
+    While step i runs on the compute stream, the host plans step i+1 and a
+    copy stream moves its inputs into the second of two device input
+    buffers; step i+1 waits only for that copy (and its group's plan arrays,
+    which go up on the compute stream behind step i).  Every step's per-slot
+    loss and predictions come back to pinned host memory on the compute
+    stream and are handed to `on_result(i, loss, preds)` once step i is done
+    (while step i+1 is already queued on the GPU).  All steps share the
+    GroupedStep's buffers and workspaces, so each step's group must need no
+    more than the group the GroupedStep was built for."""
+
+    def __init__(self, step: GroupedStep, vision_rows: int, n_text: int, targets_shape,
+                 device="cuda"):
+        self.step = step
+        self.dev = device
+        d = step.bb.cfg.d
+        self.vis = [torch.empty((max(vision_rows, 1), d), dtype=torch.bfloat16, device=device)
+                    for _ in range(2)]
+        self.tid = [torch.empty(max(n_text, 1), dtype=torch.int32, device=device)
+                    for _ in range(2)]
+        self.tgt = [torch.empty(targets_shape, dtype=torch.float32, device=device)
+                    for _ in range(2)]
+        self.preds = torch.zeros(targets_shape, dtype=torch.float32, device=device)
+        self.copy_stream = torch.cuda.Stream(device=device)
+        self.copied = [torch.cuda.Event() for _ in range(2)]
+        self.done = [torch.cuda.Event() for _ in range(2)]
+        self.loss_h = [torch.empty(step.loss.shape, dtype=torch.float32).pin_memory()
+                       for _ in range(2)]
+        self.preds_h = [torch.empty(targets_shape, dtype=torch.float32).pin_memory()
+                        for _ in range(2)]
+        self.groups: List[Optional[DeviceGroup]] = [None, None]
+        self.h2d_bytes = 0
+        self.max_tokens = step.group.plan.n_tokens
+        self.max_samples = step.group.plan.n_samples
+
+    def _fits(self, g: DeviceGroup) -> None:
+        s = self.step
+        if (g.plan.n_tokens > self.max_tokens or g.plan.n_samples > self.max_samples
+                or s.ws_h.numel() < s.heads.workspace_bytes(g)
+                or s.ws_bb.numel() < s.bb.workspace_bytes(g.plan.n_tokens)):
+            raise ValueError("StepPipeline: a step's group is larger than the step's buffers")
+        kinds = {s.heads.arr[t].kind for t in g.plan.slot_tenant.tolist()}
+        if ((J.JNX_HEAD_XATTN in kinds and not s.need_hidden)
+                or (J.JNX_HEAD_MLP in kinds and not s.need_pooled)):
+            raise ValueError("StepPipeline: a step's group has a head kind the step was not built for")
+
+    def _stage(self, i: int, host: Dict[str, torch.Tensor], plan) -> None:
+        b = i & 1
+        g = DeviceGroup(plan, device=self.dev, non_blocking=True)
+        self._fits(g)
+        cs = self.copy_stream
+        cs.wait_event(self.done[b])  # step i-2 has finished reading buffer b
+        with torch.cuda.stream(cs):
+            for dst, k in ((self.vis[b], "vision"), (self.tid[b], "text_ids"),
+                           (self.tgt[b], "targets")):
+                src = host[k]
+                dst.view(-1)[:src.numel()].copy_(src.view(-1), non_blocking=True)
+                self.h2d_bytes += src.numel() * src.element_size()
+        self.copied[b].record(cs)
+        self.groups[b] = g
+
+    def run(self, batches: Sequence[Dict[str, torch.Tensor]], plan_fn, on_result=None) -> None:
+        """batches[i]: pinned host tensors 'vision', 'text_ids', 'targets' of
+        step i; plan_fn(i) returns step i's plan (called on the host while
+        step i-1 runs)."""
+        ks = torch.cuda.current_stream(self.dev)
+        n = len(batches)
+        if n == 0:
+            return
+        self._stage(0, batches[0], plan_fn(0))
+        for i in range(n):
+            b = i & 1
+            ks.wait_event(self.copied[b])
+            self.step.group = self.groups[b]
+            self.step.run(self.vis[b], self.tid[b], self.tgt[b], self.preds, ks)
+            self.loss_h[b].copy_(self.step.loss, non_blocking=True)
+            self.preds_h[b].copy_(self.preds, non_blocking=True)
+            self.done[b].record(ks)
+            if i >= 1:
+                self.done[b ^ 1].synchronize()
+                if on_result is not None:
+                    on_result(i - 1, self.loss_h[b ^ 1], self.preds_h[b ^ 1])
+            if i + 1 < n:
+                self._stage(i + 1, batches[i + 1], plan_fn(i + 1))
+        self.done[(n - 1) & 1].synchronize()
+        if on_result is not None:
+            on_result(n - 1, self.loss_h[(n - 1) & 1], self.preds_h[(n - 1) & 1])

@@ -359,3 +359,46 @@ def test_zipf2b_lora_two_blocks_vs_oracle():
         for k, gref in ref[t]["grads"].items():
             e = rel_err(f64(s.heads.grads[t][k]), gref)
             assert e < gt[k], ("grad", t, k, e, gt[k])
+
+
+def test_step_pipeline_matches_plain_steps():
+    # StepPipeline overlaps each step's planning and input copy with the step
+    # before it; every step must still give exactly what a plain step gives
+    # (same kernels, same order), including a step whose group (one tenant)
+    # differs from the previous one's
+    w = synth.make_workload("tiny")
+    s = Setup(w)
+    _, ref_step, ref_preds = s.run()
+    ref_loss = ref_step.loss.cpu()
+    ref_preds = ref_preds.cpu()
+    wsub = w.subset([0])
+    sub_plan, sub_step, _ = s.run(wsub)
+    sub_loss = sub_step.loss.cpu()
+
+    plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), len(w.tenants), w.max_samples,
+                            w.max_tokens)
+    step = R.GroupedStep(s.bb, s.heads, R.DeviceGroup(plan))
+    host = {k: v.cpu().pin_memory() for k, v in s.inp.items()}
+    pipe = R.StepPipeline(step, s.inp["vision"].shape[0], s.inp["text_ids"].numel(),
+                          tuple(s.inp["targets"].shape))
+    order = ["full", "full", "sub", "full"]
+
+    def plan_fn(i):
+        ww = wsub if order[i] == "sub" else w
+        return J.jnx_group_plan(ww.schemas(), oracle_requests(ww), len(w.tenants),
+                                w.max_samples, w.max_tokens)
+
+    got = {}
+    pipe.run([host] * len(order), plan_fn,
+             on_result=lambda i, loss, preds: got.__setitem__(i, (loss.clone(), preds.clone())))
+    R.check_status(step.ws_bb)
+    R.check_status(step.ws_h)
+    assert sorted(got) == list(range(len(order)))
+    for i, kind in enumerate(order):
+        loss, preds = got[i]
+        if kind == "full":
+            assert torch.equal(loss, ref_loss), i
+            assert torch.equal(preds, ref_preds), i
+        else:
+            for t in set(sub_plan.slot_tenant.tolist()):
+                assert torch.equal(loss[t], sub_loss[t]), (i, t)
