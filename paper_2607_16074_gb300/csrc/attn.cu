@@ -7,13 +7,10 @@
 // first token, so a sample's result is the same wherever it sits in the
 // packed batch (grouped == isolated).
 //
-// Two tcgen05 kernels (S and O accumulate in TMEM, Q/K/V arrive by TMA, P
-// goes through shared memory), chosen per head dim in attention_launch:
-//  k_attn_ws  head dims 64 / 128: persistent and warp-specialised, two
-//             independent streams of query tiles per CTA with double-buffered
-//             scores, so softmax, MMA and copies overlap;
-//  k_attn_tc  head dim 256 (whose O accumulator leaves no TMEM for a second
-//             stream): one CTA per (sample, query tile, head).
+// One tcgen05 kernel, k_attn_ws: S, P and O live in TMEM, Q/K/V arrive by
+// TMA; persistent and warp-specialised, with two independent streams of
+// query tiles per CTA for head dims 64 / 128 and one for head dim 256 (whose
+// O accumulator leaves no TMEM for a second stream).
 // Q, K, V come from the fused projection output [N, (H + 2 Hkv) hd]; query
 // head h reads K/V head h / (H / Hkv) (MQA when Hkv = 1).
 #include "jnx_dev.cuh"
@@ -22,244 +19,12 @@
 namespace jnx {
 
 // ---------------------------------------------------------------------------
-// tcgen05 version.  One CTA = (sample, 128-query tile, head), 128 threads:
-// thread r owns query row r for the softmax and the epilogue; thread 0 also
-// issues the TMA copies and the MMAs.  Per key tile of BN keys:
-//   S = Q K^T          tcgen05.mma (M=128, N=BN, K=HD) into TMEM
-//   softmax            each thread reads its S row from TMEM twice (row max,
-//                      then p = 2^(s*scale*log2e - m)), rescales its O row in
-//                      TMEM when the running max moved, and writes p as bf16
-//                      into shared memory in the 128-byte-swizzled K-major
-//                      layout the next MMA reads
-//   O += P V           tcgen05.mma (M=128, N=HD, K=BN), V read MN-major
-// K/V tiles are double-buffered: the copy of tile kt+1 runs during tile kt.
-// The commit that follows S(kt) also covers PV(kt-1), so one barrier wait
-// tells the softmax threads that O, P and the older K/V buffer are free.
-// ---------------------------------------------------------------------------
-namespace attn_tc {
-constexpr int BM = 128;
-}
-
-template <int HD, int BN>
-struct AttnTcCfg {
-    // P rows are 128 bytes (64 keys) in the 128-byte-swizzled layout the PV
-    // MMA reads, so a key tile narrower than 64 would not fill its buffer.
-    static_assert(BN == 64 || BN == 128, "key tile must be 64 or 128 keys");
-    static_assert(HD % 64 == 0 && HD <= 256, "head dim must be 64, 128 or 256");
-    static constexpr int QB = attn_tc::BM * HD * 2;  // Q tile bytes
-    static constexpr int KB = BN * HD * 2;           // K (or V) tile bytes
-    static constexpr int PB = attn_tc::BM * BN * 2;  // P tile bytes
-    static constexpr int SMEM = QB + 4 * KB + PB + 1024 + 256;
-    static constexpr uint32_t O_COL = 128;           // TMEM column of the O accumulator
-    static constexpr uint32_t TCOLS = O_COL + HD <= 256 ? 256 : 512;  // TMEM columns held
-};
-
-template <int HD, int BN>
-__global__ void __launch_bounds__(128, 1)
-    k_attn_tc(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tkv,
-              const int* __restrict__ cu, int tiles_per_sample, int H, int Hkv, float scale_log2,
-              uint16_t* __restrict__ out, int ldo, int* status) {
-    using C = AttnTcCfg<HD, BN>;
-    constexpr int BM = attn_tc::BM;
-    constexpr int NCH = HD / 64;  // 64-column chunks of a head row
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t* sm = reinterpret_cast<uint8_t*>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    uint8_t* sQ = sm;
-    // K/V buffer b: K at QB + 2b KB, V right after it
-    auto sK = [&](int b) { return sm + C::QB + 2 * b * C::KB; };
-    auto sV = [&](int b) { return sm + C::QB + (2 * b + 1) * C::KB; };
-    uint8_t* sP = sm + C::QB + 4 * C::KB;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sP + C::PB);
-    uint64_t* q_full = bars;
-    uint64_t* kv_full = bars + 1;  // [2]
-    uint64_t* s_full = bars + 3;
-    uint64_t* pv_done = bars + 4;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 5);
-
-    const int s = blockIdx.x / tiles_per_sample;
-    const int qt = blockIdx.x % tiles_per_sample;
-    const int h = blockIdx.y;
-    const int kvh = h / (H / Hkv);
-    const int start = cu[s];
-    const int L = cu[s + 1] - start;
-    const int q0 = qt * BM;
-    if (q0 >= L) return;  // uniform for the whole CTA
-
-    const int tid = threadIdx.x, warp = tid >> 5;
-    if (tid == 0) {
-        mbar_init(q_full, 1);
-        mbar_init(&kv_full[0], 1);
-        mbar_init(&kv_full[1], 1);
-        mbar_init(s_full, 1);
-        mbar_init(pv_done, 1);
-        fence_barrier_init();
-        fence_proxy_async();
-    }
-    if (warp == 0) {
-        tmem_alloc(tmem_slot, C::TCOLS);
-        tmem_relinquish();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tbase = *tmem_slot;
-    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-    const uint32_t tS = tbase + lane_base;
-    const uint32_t tO = tbase + lane_base + C::O_COL;
-    const int n_kt = (L + BN - 1) / BN;
-    bool ok = true;
-
-    auto issue_kv = [&](int kt, int buf) {
-        mbar_arrive_expect_tx(&kv_full[buf], 2 * C::KB);
-        const int y = start + kt * BN;
-#pragma unroll
-        for (int c = 0; c < NCH; ++c) {
-            tma_load_2d(sK(buf) + c * BN * 128, &tkv, (H + kvh) * HD + c * 64, y, &kv_full[buf]);
-            tma_load_2d(sV(buf) + c * BN * 128, &tkv, (H + Hkv + kvh) * HD + c * 64, y,
-                        &kv_full[buf]);
-        }
-    };
-    if (tid == 0) {
-        mbar_arrive_expect_tx(q_full, C::QB);
-#pragma unroll
-        for (int c = 0; c < NCH; ++c)
-            tma_load_2d(sQ + c * BM * 128, &tq, h * HD + c * 64, start + q0, q_full);
-        issue_kv(0, 0);
-    }
-
-    constexpr uint32_t IDESC_S = idesc_bf16_f32(BM, BN);
-    constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, HD) | (1u << 16);  // B (V) MN-major
-    float m = -INFINITY, l = 0.f;
-
-    for (int kt = 0; kt < n_kt; ++kt) {
-        const int buf = kt & 1;
-        if (tid == 0) {
-            if (kt == 0) ok = ok && mbar_wait(q_full, 0);
-            ok = ok && mbar_wait(&kv_full[buf], (kt >> 1) & 1);
-            tc_fence_after();
-            const uint32_t qa = smem_u32(sQ), ka = smem_u32(sK(buf));
-#pragma unroll
-            for (int ks = 0; ks < HD / 16; ++ks)
-                tc_mma_f16(tS - lane_base, sw128_desc(qa + (ks >> 2) * BM * 128 + (ks & 3) * 32),
-                           sw128_desc(ka + (ks >> 2) * BN * 128 + (ks & 3) * 32), IDESC_S,
-                           ks > 0);
-            tc_commit(s_full);
-        }
-        __syncwarp();
-        ok = mbar_wait(s_full, kt & 1) && ok;
-        tc_fence_after();
-        if (tid == 0 && kt + 1 < n_kt) issue_kv(kt + 1, buf ^ 1);  // PV(kt-1) is done
-
-        // pass 1: row max over this tile's valid keys
-        const int kbase = kt * BN;
-        float mx = -INFINITY;
-#pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-            uint32_t r[32];
-            tmem_ld32(tS + c * 32, r);
-            tmem_ld_wait();
-#pragma unroll
-            for (int e = 0; e < 32; ++e)
-                if (kbase + c * 32 + e < L) mx = fmaxf(mx, __uint_as_float(r[e]) * scale_log2);
-        }
-        const float m_new = fmaxf(m, mx);
-        const float alpha = exp2f(m - m_new);
-        if (kt > 0 && __any_sync(0xffffffffu, alpha < 1.0f)) {
-#pragma unroll 1
-            for (int c = 0; c < HD / 32; ++c) {
-                uint32_t r[32];
-                tmem_ld32(tO + c * 32, r);
-                tmem_ld_wait();
-#pragma unroll
-                for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-                tmem_st32(tO + c * 32, r);
-            }
-            tmem_st_wait();
-        }
-        m = m_new;
-        // pass 2: p = 2^(s * scale - m) -> bf16 P in smem, row sum
-        float rs = 0.f;
-#pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-            uint32_t r[32];
-            tmem_ld32(tS + c * 32, r);
-            tmem_ld_wait();
-            float p[32];
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-                p[e] = (kbase + c * 32 + e < L) ? exp2f(__uint_as_float(r[e]) * scale_log2 - m)
-                                                : 0.f;
-                rs += p[e];
-            }
-            // keys c*32 .. c*32+31 = 16-byte units 4(c%2) .. 4(c%2)+3 of chunk c/2
-            uint8_t* prow = sP + (c >> 1) * BM * 128 + tid * 128;
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int unit = 4 * (c & 1) + u;
-                uint4 w;
-                w.x = pack_bf2(p[8 * u + 0], p[8 * u + 1]);
-                w.y = pack_bf2(p[8 * u + 2], p[8 * u + 3]);
-                w.z = pack_bf2(p[8 * u + 4], p[8 * u + 5]);
-                w.w = pack_bf2(p[8 * u + 6], p[8 * u + 7]);
-                *reinterpret_cast<uint4*>(prow + ((unit ^ (tid & 7)) << 4)) = w;
-            }
-        }
-        l = l * alpha + rs;
-        fence_proxy_async();
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0) {
-            tc_fence_after();
-            const uint32_t pa = smem_u32(sP), va = smem_u32(sV(buf));
-#pragma unroll
-            for (int ks = 0; ks < BN / 16; ++ks)
-                tc_mma_f16(tO - lane_base,
-                           sw128_desc(pa + (ks >> 2) * BM * 128 + (ks & 3) * 32),
-                           sw128_desc_mn(va + ks * 16 * 128, BN * 128, 1024), IDESC_PV,
-                           (kt > 0 || ks > 0));
-            if (kt == n_kt - 1) tc_commit(pv_done);
-        }
-        __syncwarp();
-    }
-    ok = mbar_wait(pv_done, 0) && ok;
-    tc_fence_after();
-    if (!ok && tid == 0) report(status, JNX_ERR_TIMEOUT);
-
-    // epilogue: O / l -> bf16
-    const float inv = 1.0f / l;
-    const int row = q0 + tid;
-    uint16_t* orow = out + (size_t)(start + row) * ldo + h * HD;
-#pragma unroll 1
-    for (int c = 0; c < HD / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32(tO + c * 32, r);
-        tmem_ld_wait();
-        if (row < L) {
-            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
-#pragma unroll
-            for (int v = 0; v < 4; ++v) {
-                uint4 w;
-                w.x = pack_bf2(__uint_as_float(r[8 * v + 0]) * inv, __uint_as_float(r[8 * v + 1]) * inv);
-                w.y = pack_bf2(__uint_as_float(r[8 * v + 2]) * inv, __uint_as_float(r[8 * v + 3]) * inv);
-                w.z = pack_bf2(__uint_as_float(r[8 * v + 4]) * inv, __uint_as_float(r[8 * v + 5]) * inv);
-                w.w = pack_bf2(__uint_as_float(r[8 * v + 6]) * inv, __uint_as_float(r[8 * v + 7]) * inv);
-                dst[v] = w;
-            }
-        }
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (warp == 0) tmem_dealloc(tbase, C::TCOLS);
-}
-
-// ---------------------------------------------------------------------------
-// Persistent warp-specialised tcgen05 attention (head dims 64 / 128).
+// Persistent warp-specialised tcgen05 attention (head dims 64 / 128 / 256).
 //
-// One CTA per SM runs two independent streams of work items; an item is one
-// 128-query tile of one sample and head, and its key loop walks that
-// sample's keys in BN-key tiles.  Stream t owns
+// One CTA per SM runs NST independent streams of work items (two for head
+// dims 64 / 128, one for 256); an item is one 128-query tile of one sample
+// and head, and its key loop walks that sample's keys in BN-key tiles.
+// Stream t owns
 //   warp t        TMA producer: Q (one buffer, refilled as soon as the
 //                 item's last S MMA has completed), K and V through
 //                 separate 2-deep rings that run on from item to item
@@ -268,7 +33,7 @@ __global__ void __launch_bounds__(128, 1)
 //                 two tiles ahead of PV, so the tensor core computes the next
 //                 scores while the softmax warps work on the current ones
 //   warps 4+4t..  online softmax and epilogue, one query row per thread
-// and TMEM columns [256 t, 256 t + 256): S buffers at +0 and +BN, O at
+// and TMEM columns from 256 t: S buffers at +0 and +BN, O (HD columns) at
 // +2 BN.  P (bf16, two per 32-bit column) overwrites the first BN / 2
 // columns of the score buffer it was computed from and is the TMEM A
 // operand of the PV MMA; V is read from shared memory as the MN-major B
@@ -303,11 +68,12 @@ constexpr int kBars = 18;      // barriers per stream
 }  // namespace attn_ws
 
 // Work items: an explicit (sample, query tile) list, or, without one, every
-// (query tile, sample) combination tile-major with the empty ones skipped.
+// (sample, query tile) combination sample-major (a sample's query tiles,
+// which read the same K/V, run close together) with the empty ones skipped.
 struct AttnItems {
     const int2* list;
-    int n;  // entries of `list`, or S * tiles_max
-    int S;
+    int n;      // entries of `list`, or S * tiles
+    int tiles;  // query tiles per sample in the enumeration (longest sample)
 };
 
 // One work item: query tile qt of the sample at packed rows [start,
@@ -330,8 +96,8 @@ __device__ __forceinline__ AttnWork attn_fetch(const AttnItems& it, const int* _
         s = e.x;
         a.qt = e.y;
     } else {
-        a.qt = i / it.S;
-        s = i % it.S;
+        a.qt = i % it.tiles;
+        s = i / it.tiles;
     }
     a.start = cu[s];
     a.L = cu[s + 1] - a.start;
@@ -357,20 +123,25 @@ __device__ __forceinline__ uint4 attn_stg_get(const uint8_t* stg, int lane, int 
 template <int HD, int BN>
 struct AttnWsCfg {
     static_assert(BN == 64, "key tile of 64 keys");
-    static_assert(HD == 64 || HD == 128, "head dim 64 or 128");
+    static_assert(HD == 64 || HD == 128 || HD == 256, "head dim 64, 128 or 256");
+    // streams per CTA: a stream holds two BN-column score buffers and an
+    // HD-column O in TMEM (512 columns), so head dim 256 runs one stream
+    static constexpr int NST = HD == 256 ? 1 : 2;
+    static constexpr int THREADS = 128 + 128 * NST;
+    static constexpr uint32_t TSTRIDE = 256;  // TMEM columns between streams
     static constexpr int BM = attn_ws::BM;
     static constexpr int QB = BM * HD * 2;  // Q tile
     static constexpr int KB = BN * HD * 2;  // one K (or V) tile
     static constexpr int OFF_K = QB;
     static constexpr int OFF_V = OFF_K + 2 * KB;
     static constexpr int STREAM = OFF_V + 2 * KB;  // bytes per stream (multiple of 1024)
-    static constexpr int OFF_STG = 2 * STREAM;   // epilogue staging, 2 KB per softmax warp
-    static constexpr int OFF_BAR = OFF_STG + 8 * 2048;
-    static constexpr int SMEM = OFF_BAR + 2 * attn_ws::kBars * 8 + 16 + 1024;
+    static constexpr int OFF_STG = NST * STREAM;  // epilogue staging, 2 KB per softmax warp
+    static constexpr int OFF_BAR = OFF_STG + 4 * NST * 2048;
+    static constexpr int SMEM = OFF_BAR + NST * attn_ws::kBars * 8 + 16 + 1024;
     static_assert(STREAM % 1024 == 0, "128B-swizzled tiles need 1024-byte alignment");
     static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
     static constexpr uint32_t O_COL = 2 * BN;  // within the stream's 256 columns
-    static_assert(O_COL + HD <= 256, "TMEM columns per stream");
+    static_assert(O_COL + HD <= (NST == 2 ? TSTRIDE : 512), "TMEM columns per stream");
 };
 
 // Softmax of one 128 x BN score tile for this thread's row: row max (pass
@@ -473,7 +244,7 @@ __device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float s
 }
 
 template <int HD, int BN>
-__global__ void __launch_bounds__(384, 1)
+__global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
     k_attn_ws(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tkv,
               const int* __restrict__ cu, AttnItems items, int H, int Hkv, float scale_log2,
               uint16_t* __restrict__ out, int ldo, int* status) {
@@ -483,7 +254,7 @@ __global__ void __launch_bounds__(384, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + C::OFF_BAR + 2 * attn_ws::kBars * 8);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + C::OFF_BAR + C::NST * attn_ws::kBars * 8);
     volatile int* fail_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -508,12 +279,12 @@ __global__ void __launch_bounds__(384, 1)
 
     const int n_work = items.n * H;
     const int group = H / Hkv;
-    const int w0 = 2 * blockIdx.x + t, dw = 2 * gridDim.x;
+    const int w0 = C::NST * blockIdx.x + t, dw = C::NST * gridDim.x;
     if (tid == 0) {
         // both streams' barriers: one arrival each, but p_full[] and o_free,
         // which every softmax thread of the stream arrives on
         uint64_t* all = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR);
-        for (int i = 0; i < 2 * attn_ws::kBars; ++i) {
+        for (int i = 0; i < C::NST * attn_ws::kBars; ++i) {
             const int k = i % attn_ws::kBars;
             mbar_init(&all[i], (k == 12 || k == 13 || k == 16) ? BM : 1);
         }
@@ -528,11 +299,11 @@ __global__ void __launch_bounds__(384, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tbase = *tmem_slot + (uint32_t)(t * 256);
+    const uint32_t tbase = *tmem_slot + (uint32_t)t * C::TSTRIDE;
 
     if (warp < 2) {
         // ---------------- producer of stream t ----------------
-        if (lane == 0) {
+        if (lane == 0 && t < C::NST) {
             tma_prefetch_desc(&tq);
             tma_prefetch_desc(&tkv);
             bool ok = true;
@@ -583,7 +354,7 @@ __global__ void __launch_bounds__(384, 1)
         }
     } else if (warp < 4) {
         // ---------------- MMA issuer of stream t ----------------
-        if (lane == 0) {
+        if (lane == 0 && t < C::NST) {
             constexpr uint32_t IDESC_S = idesc_bf16_f32(BM, BN);
             constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, HD) | (1u << 16);  // B MN-major
             bool ok = true, issued = false;
@@ -805,46 +576,21 @@ static jnx_status launch_attn_ws(const uint16_t* qkv, int ldq, int n_tokens, int
         !make_tmap_bf16(&tkv, qkv, n_tokens, ldq, ldq, BN, 64))
         return fail(JNX_ERR_CUDA, "attention: tensor map encode failed");
     AttnItems it;
-    it.S = S;
+    it.tiles = (max_seqlen + C::BM - 1) / C::BM;
     if (items) {
         it.list = items;
         it.n = n_items;
     } else {
         it.list = nullptr;
-        it.n = S * ((max_seqlen + C::BM - 1) / C::BM);
+        it.n = S * it.tiles;
     }
     if ((long long)it.n * H > 0x7FFFFFFFLL)
         return fail(JNX_ERR_UNSUPPORTED, "attention: too many work items");
     const int n_work = it.n * H;
     if (n_work == 0) return JNX_OK;
-    const int grid = std::min((n_work + 1) / 2, num_sms());
+    const int grid = std::min((n_work + C::NST - 1) / C::NST, num_sms());
     const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)HD));
-    k_attn_ws<HD, BN><<<grid, 384, C::SMEM, s>>>(tq, tkv, cu, it, H, Hkv, scale_log2, out, ldo,
-                                                 status);
-    cudaError_t e = cudaGetLastError();
-    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
-}
-
-template <int HD, int BN>
-static jnx_status launch_attn_tc(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv,
-                                 const int* cu, int S, int max_seqlen, uint16_t* out, int ldo,
-                                 int* status, cudaStream_t s) {
-    using C = AttnTcCfg<HD, BN>;
-    static bool attr = false;
-    if (!attr) {
-        if (cudaFuncSetAttribute(k_attn_tc<HD, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 C::SMEM) != cudaSuccess)
-            return fail(JNX_ERR_CUDA, "attention: smem attribute");
-        attr = true;
-    }
-    CUtensorMap tq, tkv;
-    if (!make_tmap_bf16(&tq, qkv, n_tokens, ldq, ldq, attn_tc::BM, 64) ||
-        !make_tmap_bf16(&tkv, qkv, n_tokens, ldq, ldq, BN, 64))
-        return fail(JNX_ERR_CUDA, "attention: tensor map encode failed");
-    const int tps = (max_seqlen + attn_tc::BM - 1) / attn_tc::BM;
-    const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)HD));
-    dim3 grid(S * tps, H);
-    k_attn_tc<HD, BN><<<grid, 128, C::SMEM, s>>>(tq, tkv, cu, tps, H, Hkv, scale_log2, out, ldo,
+    k_attn_ws<HD, BN><<<grid, C::THREADS, C::SMEM, s>>>(tq, tkv, cu, it, H, Hkv, scale_log2, out, ldo,
                                                  status);
     cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
@@ -855,7 +601,7 @@ jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, i
                             uint16_t* out, int ldo, int* status, cudaStream_t s) {
     if (S == 0 || max_seqlen == 0) return JNX_OK;
     if (Hkv <= 0 || H % Hkv) return fail(JNX_ERR_UNSUPPORTED, "attention: H %% Hkv != 0");
-    if ((long long)S * ((max_seqlen + attn_tc::BM - 1) / attn_tc::BM) > 0x7FFFFFFFLL || H > 65535)
+    if ((long long)S * ((max_seqlen + attn_ws::BM - 1) / attn_ws::BM) > 0x7FFFFFFFLL || H > 65535)
         return fail(JNX_ERR_UNSUPPORTED, "attention: grid too large");
     switch (hd) {
         case 64:
@@ -865,8 +611,8 @@ jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, i
             return launch_attn_ws<128, 64>(qkv, ldq, n_tokens, H, Hkv, cu, S, max_seqlen, items,
                                            n_items, out, ldo, status, s);
         case 256:
-            return launch_attn_tc<256, 64>(qkv, ldq, n_tokens, H, Hkv, cu, S, max_seqlen, out,
-                                           ldo, status, s);
+            return launch_attn_ws<256, 64>(qkv, ldq, n_tokens, H, Hkv, cu, S, max_seqlen, items,
+                                           n_items, out, ldo, status, s);
         default:
             return fail(JNX_ERR_UNSUPPORTED, "attention: head_dim %d not in {64,128,256}", hd);
     }
