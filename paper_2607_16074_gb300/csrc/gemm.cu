@@ -132,6 +132,17 @@ __device__ __forceinline__ void stg_store_bf16(uint8_t* stg, int lane, const uin
     __syncwarp();
 }
 
+// RMSNorm factor of a row whose A row is y = bf16(x * gamma) (folded norm):
+// rsqrt(mean(x^2) + eps) from the row's partial sums of squares, added in a
+// fixed order; 1 without a folded norm.
+__device__ __forceinline__ float row_norm_scale(const GemmParams& p, int row, bool valid) {
+    if (p.ss_in == nullptr || !valid) return 1.f;
+    const float* sp = p.ss_in + (size_t)row * p.ss_parts;
+    float t = 0.f;
+    for (int i = 0; i < p.ss_parts; ++i) t += sp[i];
+    return rsqrtf(t / (float)p.ss_cols + p.ss_eps);
+}
+
 // The accumulator tile at tbase (this warp's 32 TMEM lanes = rows
 // row_base..row_base+31, 256 fp32 columns) -> the epilogue's output.
 template <int EPI>
@@ -176,6 +187,10 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
 #pragma unroll
             for (int q = 0; q < RD - 1; ++q) load_resid(q, xr[q]);
         }
+        // folded RMSNorm (EPI_RESID with norm_gamma): y = bf16(x * gamma) and
+        // the sum of x^2 of each of this lane's four rows over its columns
+        const bool norm = EPI == EPI_RESID && p.norm_gamma != nullptr;
+        float ssq[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
             uint32_t r[32];
@@ -212,11 +227,32 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                                           make_uint4(__float_as_uint(o.x), __float_as_uint(o.y),
                                                      __float_as_uint(o.z), __float_as_uint(o.w)),
                                           pol);
+                    if (EPI == EPI_RESID && norm) {
+                        const uint2 g = *reinterpret_cast<const uint2*>(p.norm_gamma + col);
+                        ssq[i] += o.x * o.x + o.y * o.y + o.z * o.z + o.w * o.w;
+                        if (row < row_end)
+                            *reinterpret_cast<uint2*>(p.norm_out + (size_t)row * p.N + col) =
+                                make_uint2(pack_bf2(o.x * bf2f(g.x & 0xFFFF), o.y * bf2f(g.x >> 16)),
+                                           pack_bf2(o.z * bf2f(g.y & 0xFFFF), o.w * bf2f(g.y >> 16)));
+                    }
                 }
                 __syncwarp();
             }
         }
+        if (norm) {
+            // the four lanes of a row hold its 256 columns between them
+            const int parts = p.N / 256;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                float t = ssq[i];
+                t += __shfl_xor_sync(0xffffffffu, t, 1);
+                t += __shfl_xor_sync(0xffffffffu, t, 2);
+                const int row = row_base + 8 * i + (lane >> 2);
+                if ((lane & 3) == 0 && row < row_end) p.ss_out[(size_t)row * parts + n0 / 256] = t;
+            }
+        }
     } else if constexpr (EPI == EPI_GLU) {
+        const float rs = row_norm_scale(p, my_row, valid);
 #pragma unroll 1
         for (int c = 0; c < 4; ++c) {
             uint32_t g[32], u[32];
@@ -229,8 +265,8 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                 float o[8];
 #pragma unroll
                 for (int e = 0; e < 8; ++e)
-                    o[e] = act_fn(__uint_as_float(g[8 * q + e]), p.act) *
-                           __uint_as_float(u[8 * q + e]);
+                    o[e] = act_fn(rs * __uint_as_float(g[8 * q + e]), p.act) *
+                           (rs * __uint_as_float(u[8 * q + e]));
                 v[q] = pack8_bf16(o);
             }
             stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
@@ -240,6 +276,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
         const int hc = p.hd / 64;  // 32-column chunks in half a head
         const int half = p.hd / 2;
         const int pos = valid ? p.pos[my_row] : 0;
+        const float rs = row_norm_scale(p, my_row, valid);
 #pragma unroll 1
         for (int c = 0; c < 8; ++c) {
             const int hchunk = c % (2 * hc);
@@ -263,8 +300,8 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
             float a[32], b[32];
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
-                a[e] = __uint_as_float(lo[e]);
-                b[e] = __uint_as_float(hi[e]);
+                a[e] = rs * __uint_as_float(lo[e]);
+                b[e] = rs * __uint_as_float(hi[e]);
             }
             if (rot) {
 #pragma unroll

@@ -25,6 +25,19 @@ struct GemmParams {
     int act;              // EPI_GLU: JNX_GLU_*
     int group_m;          // tile-order group size (row blocks)
     int* status;          // device status word
+    // RMSNorm folded across two GEMMs.  EPI_RESID with norm_gamma set also
+    // writes y = bf16(x_new * gamma[col]) to norm_out [M, N] and, per row and
+    // 256-column block, the partial sum of x_new^2 to ss_out [M, N / 256].
+    const uint16_t* norm_gamma;
+    uint16_t* norm_out;
+    float* ss_out;
+    // EPI_ROPE / EPI_GLU with ss_in set: the A rows are such y, and each
+    // output row is first scaled by rsqrt(sum of ss_in[row][0, ss_parts) /
+    // ss_cols + ss_eps), the RMSNorm factor of the row (a per-row scale
+    // commutes with the product).
+    const float* ss_in;
+    int ss_parts, ss_cols;
+    float ss_eps;
 };
 
 // LoRA: rank and the number of tenant segments one launch describes.
@@ -94,6 +107,11 @@ jnx_status rmsnorm_launch(const float* x, const uint16_t* gamma, float eps, int 
 // Final RMSNorm fused with the per-sample mean pool.
 jnx_status final_pool_launch(const float* x, const uint16_t* gamma, float eps, const int* cu,
                              int S, int d, float* pooled, uint16_t* hidden, cudaStream_t s);
+
+// Folded RMSNorm, first half: y = bf16(x * gamma) [M, d] and per row and
+// 256-column block the sum of x^2 (ss [M, d / 256]).
+jnx_status rms_prep_launch(const float* x, const uint16_t* gamma, int M, int d, uint16_t* y,
+                           float* ss, cudaStream_t s);
 
 // (cos, sin) table for positions [0, max_pos) of head dim hd.
 jnx_status rope_table_launch(float2* tab, int max_pos, int hd, float theta, cudaStream_t s);

@@ -100,6 +100,60 @@ __global__ void __launch_bounds__(256) k_rmsnorm(const float* __restrict__ x,
     }
 }
 
+// First half of a folded RMSNorm (the residual GEMM epilogue does the same for
+// every later norm): y = bf16(x * gamma) and, per row and 256-column block,
+// the sum of x^2; the consuming GEMM scales its output rows by
+// rsqrt(sum / d + eps).  One warp per row.
+template <int V>
+__global__ void __launch_bounds__(256) k_rms_prep(const float* __restrict__ x,
+                                                  const uint16_t* __restrict__ gamma, int M,
+                                                  uint16_t* __restrict__ y, float* __restrict__ ss) {
+    constexpr int D = V * 128;
+    constexpr int P = D / 256;  // 256-column blocks: lane float4s i = 2b, 2b + 1
+    const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (row >= M) return;
+    const float4* xr = reinterpret_cast<const float4*>(x + (size_t)row * D);
+    float4 v[V];
+#pragma unroll
+    for (int i = 0; i < V; ++i) v[i] = __ldg(xr + lane + 32 * i);
+#pragma unroll
+    for (int b = 0; b < P; ++b) {
+        float t = 0.f;
+#pragma unroll
+        for (int i = 2 * b; i < 2 * b + 2; ++i)
+            t += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+        t = warp_sum(t);
+        if (lane == 0) ss[(size_t)row * P + b] = t;
+    }
+    uint2* orow = reinterpret_cast<uint2*>(y + (size_t)row * D);
+    const uint2* g2 = reinterpret_cast<const uint2*>(gamma);
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+        const uint2 gg = __ldg(g2 + lane + 32 * i);
+        uint2 o;
+        o.x = pack_bf2(v[i].x * bf2f(gg.x & 0xFFFF), v[i].y * bf2f(gg.x >> 16));
+        o.y = pack_bf2(v[i].z * bf2f(gg.y & 0xFFFF), v[i].w * bf2f(gg.y >> 16));
+        orow[lane + 32 * i] = o;
+    }
+}
+
+jnx_status rms_prep_launch(const float* x, const uint16_t* gamma, int M, int d, uint16_t* y,
+                           float* ss, cudaStream_t s) {
+    if (M == 0) return JNX_OK;
+    const int grid = (M + 7) / 8;
+    switch (d) {
+        case 256: k_rms_prep<2><<<grid, 256, 0, s>>>(x, gamma, M, y, ss); break;
+        case 512: k_rms_prep<4><<<grid, 256, 0, s>>>(x, gamma, M, y, ss); break;
+        case 1024: k_rms_prep<8><<<grid, 256, 0, s>>>(x, gamma, M, y, ss); break;
+        case 2048: k_rms_prep<16><<<grid, 256, 0, s>>>(x, gamma, M, y, ss); break;
+        case 4096: k_rms_prep<32><<<grid, 256, 0, s>>>(x, gamma, M, y, ss); break;
+        default: return fail(JNX_ERR_UNSUPPORTED, "rms prep: d=%d not in {256..4096}", d);
+    }
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "rms prep: %s", cudaGetErrorString(e));
+}
+
 jnx_status rmsnorm_launch(const float* x, const uint16_t* gamma, float eps, int M, int d,
                           uint16_t* out, cudaStream_t s) {
     if (M == 0) return JNX_OK;
