@@ -149,6 +149,44 @@ jnx_status jnx_group_plan(const jnx_schema* schemas, int32_t n_schemas,
                           const jnx_limits* lim, jnx_plan* out);
 
 /* ------------------------------------------------------------------------
+ * Inference scheduler (host only; callable without a GPU)
+ * ------------------------------------------------------------------------ */
+
+/* §3.3: the inference service has a maximum waiting time T and a target
+ * batch size B; it builds a batch from requests in FIFO order and starts it
+ * when the waiting time reaches T or the batch size reaches B. */
+typedef struct {
+    double timeout;         /* T, seconds the oldest queued request may wait */
+    int32_t batch_samples;  /* B, in samples: a batch this large starts at once;
+                               also the batch's sample limit */
+    int32_t max_tokens;     /* packed-token limit of one batch */
+    int32_t skip_ahead;     /* 0: stop at the first request incompatible with the
+                               oldest (App. A prefix); 1: pass over such requests,
+                               which stay queued, and take later compatible ones */
+    int32_t reserved;
+} jnx_sched_policy;
+
+/* The scheduler's decision at time `now` over a queue of n_reqs requests in
+ * arrival order (arrival[i] in seconds, any common origin).  It collects a
+ * batch as jnx_group_plan does (requests compatible with the oldest one,
+ * whole requests within batch_samples and max_tokens, the oldest always
+ * taken) and fires when the batch holds >= batch_samples samples, when it
+ * cannot grow (the next compatible request does not fit), or when the
+ * oldest request has waited >= timeout.  Firing: *n_take > 0 and take[0..
+ * *n_take) are the ascending queue indices to run (the caller removes them
+ * from its queue and plans them with jnx_group_plan, which accepts them
+ * all); *wake = now.  Not firing: *n_take = 0 and *wake = arrival[0] +
+ * timeout, the time to poll again (HUGE_VAL for an empty queue).  take[]
+ * holds n_reqs entries (caller-owned).  Errors: JNX_ERR_INVALID_ARG (null
+ * pointer, a policy with batch_samples < 1, max_tokens < 1, timeout < 0 or
+ * skip_ahead not 0/1, or a malformed request as jnx_group_plan rejects it),
+ * JNX_ERR_OVERFLOW as jnx_group_plan; nothing is written on error. */
+jnx_status jnx_sched_poll(const jnx_schema* schemas, int32_t n_schemas,
+                          const jnx_request* reqs, const double* arrival, int32_t n_reqs,
+                          int32_t n_tenants, double now, const jnx_sched_policy* pol,
+                          int32_t* take, int32_t* n_take, double* wake);
+
+/* ------------------------------------------------------------------------
  * Device-side view of a plan
  * ------------------------------------------------------------------------ */
 
@@ -267,7 +305,9 @@ size_t jnx_heads_workspace_bytes(const jnx_head* heads, int32_t n_tenants, const
  * array indexed by tenant.  Writes preds at each sample's target offset
  * (arrival layout, fp32) and loss[tenant] = mean squared error over the
  * tenant's samples and outputs, for the tenants in the group only.  The
- * activations the backward needs are kept in `workspace`. */
+ * activations the backward needs are kept in `workspace`.  targets and loss
+ * may both be NULL (inference: predictions only; a jnx_heads_backward then
+ * needs a forward with targets first). */
 jnx_status jnx_heads_forward(const jnx_head* heads, int32_t n_tenants, const jnx_group* g,
                              const float* pooled, const uint16_t* hidden,
                              const float* targets, float* preds, float* loss,

@@ -574,7 +574,7 @@ extern "C" jnx_status jnx_heads_forward(const jnx_head* heads, int32_t n_tenants
     jnx_status st;
     if ((st = check_heads(heads, n_tenants, g, false, nullptr, pooled, hidden))) return st;
     if (g->n_slots == 0) return JNX_OK;
-    if (!targets || !preds || !loss || !workspace)
+    if (!preds || !workspace || (!targets) != (!loss))
         return fail(JNX_ERR_INVALID_ARG, "heads forward: null buffer");
     HeadsWs w = carve_heads(heads, g, workspace);
     if (ws_bytes < w.bytes)

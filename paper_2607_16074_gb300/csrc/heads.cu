@@ -589,7 +589,8 @@ jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const 
     k_head_lin<2><<<dim3(b.n, (b.max_width + 7) / 8), 256, 0, s>>>(tab, ws.h, ws.ld_h, ws.y,
                                                                    nullptr, ws.ld_y,
                                                                    sample_target, preds);
-    k_l2_loss<<<b.n, 256, 0, s>>>(tab, ws.y, ws.ld_y, targets, sample_target, ws.dy, loss);
+    if (targets)  // without targets (inference) there is no loss
+        k_l2_loss<<<b.n, 256, 0, s>>>(tab, ws.y, ws.ld_y, targets, sample_target, ws.dy, loss);
     return cuda_ok("heads forward");
 }
 

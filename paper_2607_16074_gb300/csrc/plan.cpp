@@ -7,6 +7,7 @@
 // back.  §3.3: the canonical VLAFeature is where tenants' samples are
 // concatenated.  Packing is varlen (no padding) so grouped results equal
 // per-sample results.
+#include <cmath>
 #include <cstring>
 #include <mutex>
 #include <string>
@@ -40,22 +41,10 @@ static int64_t sample_len(const jnx_schema& sc, const jnx_sample& s) {
     return (int64_t)s.n_img * sc.vision_tokens + s.text_len;
 }
 
-}  // namespace jnx
-
-using namespace jnx;
-
-extern "C" const char* jnx_last_error(void) { return g_last_error.c_str(); }
-
-extern "C" int32_t jnx_version(void) { return 1; }
-
-extern "C" jnx_status jnx_group_plan(const jnx_schema* schemas, int32_t n_schemas,
-                                     const jnx_request* reqs, int32_t n_reqs, int32_t n_tenants,
-                                     const jnx_limits* lim, jnx_plan* out) {
-    clear_error();
-    if (!out || !lim || n_reqs < 0 || n_tenants < 0 || (n_reqs > 0 && (!reqs || !schemas)))
-        return fail(JNX_ERR_INVALID_ARG, "jnx_group_plan: null argument or negative count");
-
-    // Validate every request in the queue before deciding anything.
+// Every request of a queue well formed (tenant, schema, sample shapes and
+// offsets within int32).
+static jnx_status validate_requests(const jnx_schema* schemas, int32_t n_schemas,
+                                    const jnx_request* reqs, int32_t n_reqs, int32_t n_tenants) {
     for (int32_t i = 0; i < n_reqs; ++i) {
         const jnx_request& r = reqs[i];
         if (r.tenant < 0 || r.tenant >= n_tenants)
@@ -84,6 +73,26 @@ extern "C" jnx_status jnx_group_plan(const jnx_schema* schemas, int32_t n_schema
                 return fail(JNX_ERR_OVERFLOW, "request %d sample %d: offset beyond int32", i, j);
         }
     }
+    return JNX_OK;
+}
+
+}  // namespace jnx
+
+using namespace jnx;
+
+extern "C" const char* jnx_last_error(void) { return g_last_error.c_str(); }
+
+extern "C" int32_t jnx_version(void) { return 1; }
+
+extern "C" jnx_status jnx_group_plan(const jnx_schema* schemas, int32_t n_schemas,
+                                     const jnx_request* reqs, int32_t n_reqs, int32_t n_tenants,
+                                     const jnx_limits* lim, jnx_plan* out) {
+    clear_error();
+    if (!out || !lim || n_reqs < 0 || n_tenants < 0 || (n_reqs > 0 && (!reqs || !schemas)))
+        return fail(JNX_ERR_INVALID_ARG, "jnx_group_plan: null argument or negative count");
+
+    // Validate every request in the queue before deciding anything.
+    if (jnx_status st = validate_requests(schemas, n_schemas, reqs, n_reqs, n_tenants)) return st;
 
     // Largest FIFO-compatible prefix under the limits (whole requests).
     int32_t k = 0;
@@ -167,5 +176,63 @@ extern "C" jnx_status jnx_group_plan(const jnx_schema* schemas, int32_t n_schema
         out->seg_offsets[g + 1] = S;
     }
     out->max_seqlen = maxlen;
+    return JNX_OK;
+}
+
+// jnx_sched_poll: the inference scheduler's decision at time `now`.
+//
+// §3.3: the inference service keeps a maximum waiting time T and a target
+// batch size B, builds a batch from requests in FIFO order and starts it
+// when the waiting time reaches T or the batch size reaches B.  App. A: the
+// batch is the largest FIFO-compatible prefix the limits allow.  The batch
+// is collected as jnx_group_plan collects it (compatibility with the oldest
+// request, whole requests, the oldest always taken); it also fires when the
+// batch cannot grow because the next compatible request does not fit.  The
+// skip-ahead mode passes over incompatible requests, which stay queued.
+extern "C" jnx_status jnx_sched_poll(const jnx_schema* schemas, int32_t n_schemas,
+                                     const jnx_request* reqs, const double* arrival,
+                                     int32_t n_reqs, int32_t n_tenants, double now,
+                                     const jnx_sched_policy* pol, int32_t* take, int32_t* n_take,
+                                     double* wake) {
+    clear_error();
+    if (!pol || !n_take || !wake || n_reqs < 0 || n_tenants < 0 ||
+        (n_reqs > 0 && (!reqs || !schemas || !arrival || !take)))
+        return fail(JNX_ERR_INVALID_ARG, "jnx_sched_poll: null argument or negative count");
+    if (pol->batch_samples < 1 || pol->max_tokens < 1 || !(pol->timeout >= 0.0) ||
+        (pol->skip_ahead != 0 && pol->skip_ahead != 1))
+        return fail(JNX_ERR_INVALID_ARG, "jnx_sched_poll: bad policy");
+    if (jnx_status st = validate_requests(schemas, n_schemas, reqs, n_reqs, n_tenants)) return st;
+    *n_take = 0;
+    if (n_reqs == 0) {
+        *wake = HUGE_VAL;
+        return JNX_OK;
+    }
+    const jnx_schema& key = schemas[reqs[0].schema];
+    int32_t k = 0;
+    int64_t n_s = 0, n_t = 0;
+    bool full = false;
+    for (int32_t i = 0; i < n_reqs; ++i) {
+        const jnx_request& r = reqs[i];
+        const jnx_schema& sc = schemas[r.schema];
+        if (!same_prefix(sc, key)) {
+            if (pol->skip_ahead) continue;
+            break;
+        }
+        int64_t rt = 0;
+        for (int32_t j = 0; j < r.n_samples; ++j) rt += sample_len(sc, r.samples[j]);
+        if (k > 0 && (n_s + r.n_samples > pol->batch_samples || n_t + rt > pol->max_tokens)) {
+            full = true;
+            break;
+        }
+        take[k++] = i;
+        n_s += r.n_samples;
+        n_t += rt;
+    }
+    if (n_s >= pol->batch_samples || full || now - arrival[0] >= pol->timeout) {
+        *n_take = k;
+        *wake = now;
+    } else {
+        *wake = arrival[0] + pol->timeout;
+    }
     return JNX_OK;
 }

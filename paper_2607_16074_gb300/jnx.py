@@ -67,6 +67,11 @@ class jnx_plan(C.Structure):
                 ("slot_tenant", P32), ("gather_src", P32), ("pos_ids", P32)]
 
 
+class jnx_sched_policy(C.Structure):
+    _fields_ = [("timeout", C.c_double), ("batch_samples", C.c_int32), ("max_tokens", C.c_int32),
+                ("skip_ahead", C.c_int32), ("reserved", C.c_int32)]
+
+
 class jnx_group(C.Structure):
     _fields_ = [("n_samples", C.c_int32), ("n_tokens", C.c_int32), ("n_slots", C.c_int32),
                 ("max_seqlen", C.c_int32),
@@ -110,7 +115,7 @@ EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_work
            "jnx_heads_backward", "jnx_check_status", "jnx_pack_gate_up", "jnx_op_pack",
            "jnx_op_rmsnorm", "jnx_op_gemm_workspace_bytes", "jnx_op_gemm", "jnx_op_attention",
            "jnx_op_final_pool", "jnx_trace_enable", "jnx_trace_disable", "jnx_trace_count",
-           "jnx_trace_read", "jnx_op_gemm_rope_noalloc")
+           "jnx_trace_read", "jnx_op_gemm_rope_noalloc", "jnx_sched_poll")
 
 
 def lib() -> C.CDLL:
@@ -128,6 +133,10 @@ def lib() -> C.CDLL:
         "jnx_version": (i32, []),
         "jnx_group_plan": (i32, [C.POINTER(jnx_schema), i32, C.POINTER(jnx_request), i32, i32,
                                  C.POINTER(jnx_limits), C.POINTER(jnx_plan)]),
+        "jnx_sched_poll": (i32, [C.POINTER(jnx_schema), i32, C.POINTER(jnx_request),
+                                 C.POINTER(C.c_double), i32, i32, C.c_double,
+                                 C.POINTER(jnx_sched_policy), P32, C.POINTER(C.c_int32),
+                                 C.POINTER(C.c_double)]),
         "jnx_backbone_workspace_bytes": (sz, [C.POINTER(jnx_backbone), i32]),
         "jnx_backbone_forward": (i32, [C.POINTER(jnx_backbone), C.POINTER(jnx_group), vp, i64,
                                        vp, i64, vp, vp, vp, sz, vp]),
@@ -218,8 +227,8 @@ def make_requests(requests: Sequence[dict]):
     for i, r in enumerate(requests):
         ss = (jnx_sample * max(1, len(r["samples"])))()
         for j, s in enumerate(r["samples"]):
-            ss[j] = jnx_sample(s["n_img"], s["text_len"], s["vision_row"], s["text_pos"],
-                               s["target_off"])
+            ss[j] = jnx_sample(s["n_img"], s["text_len"], s.get("vision_row", 0),
+                               s.get("text_pos", 0), s.get("target_off", 0))
         keep.append(ss)
         arr[i] = jnx_request(r["tenant"], r["schema"], len(r["samples"]), 0,
                              C.cast(ss, C.POINTER(jnx_sample)))
@@ -250,6 +259,26 @@ def jnx_group_plan(schemas: Sequence[dict], requests: Sequence[dict], n_tenants:
         check(rc)
         return Plan(raw, arrays)
     raise JnxError(JNX_ERR_CAPACITY, "plan capacity")
+
+
+def jnx_sched_poll(schemas: Sequence[dict], requests: Sequence[dict], arrival: Sequence[float],
+                   n_tenants: int, now: float, timeout: float, batch_samples: int,
+                   max_tokens: int, skip_ahead: bool = False):
+    """The inference scheduler's decision at `now`: (take, wake) with take
+    the ascending queue indices to run now (empty: not yet) and wake the
+    time to poll again when not firing (`now` when firing, inf when empty)."""
+    L = lib()
+    sch = make_schemas(schemas)
+    req, keep = make_requests(requests)
+    n = len(requests)
+    arr = (C.c_double * max(1, n))(*[float(a) for a in arrival])
+    take = np.zeros(max(1, n), np.int32)
+    n_take, wake = C.c_int32(0), C.c_double(0.0)
+    pol = jnx_sched_policy(float(timeout), min(int(batch_samples), 2**31 - 1),
+                           min(int(max_tokens), 2**31 - 1), int(bool(skip_ahead)), 0)
+    check(L.jnx_sched_poll(sch, len(schemas), req, arr, n, n_tenants, float(now), C.byref(pol),
+                           take.ctypes.data_as(P32), C.byref(n_take), C.byref(wake)))
+    return take[:n_take.value].tolist(), wake.value
 
 
 # ---------------------------------------------------------------------------

@@ -113,3 +113,34 @@ def test_gpu_calls_reject_bad_arguments_without_a_gpu():
     assert "backbone" in J.jnx_last_error()
     rc = L.jnx_op_gemm(None, None, 1, 256, 64, 0, None, 256, None, 0, 0, 0, 0.0, 0, None, 0, None)
     assert rc == J.JNX_ERR_INVALID_ARG
+
+
+def test_scheduler_bit_exact_vs_oracle_random_queues():
+    # jnx_sched_poll (C++) against the scheduler oracle: same queue indices
+    # to take and the same wake time, on both collection modes
+    from oracle import sched as OS
+    from tests.test_oracle_sched import _random_queue as sched_queue
+    rng = random.Random(11)
+    for _ in range(1500):
+        schemas, reqs = sched_queue(rng, rng.randint(0, 8))
+        arrival = sorted(rng.uniform(0, 2) for _ in reqs)
+        now = (arrival[-1] if arrival else 0.0) + rng.uniform(0, 1.5)
+        T, Bs, mt = rng.uniform(0.0, 1.5), rng.randint(1, 12), rng.randint(1, 90)
+        skip = rng.random() < 0.5
+        want = OS.poll(schemas, reqs, arrival, now, T, Bs, mt, skip)
+        got = J.jnx_sched_poll(schemas, reqs, arrival, 4, now, T, Bs, mt, skip)
+        assert got == want
+
+
+def test_scheduler_rejects_bad_policies_and_requests():
+    from tests.test_oracle_sched import _random_queue as sched_queue
+    schemas, reqs = sched_queue(random.Random(3), 3)
+    for kw in (dict(batch_samples=0), dict(max_tokens=0), dict(timeout=-1.0)):
+        args = dict(timeout=1.0, batch_samples=4, max_tokens=64)
+        args.update(kw)
+        with pytest.raises(J.JnxError) as e:
+            J.jnx_sched_poll(schemas, reqs, [0.0, 0.1, 0.2], 4, 0.5, **args)
+        assert e.value.code == J.JNX_ERR_INVALID_ARG
+    bad = [dict(reqs[0], tenant=9)] + reqs[1:]
+    with pytest.raises(J.JnxError):
+        J.jnx_sched_poll(schemas, bad, [0.0, 0.1, 0.2], 4, 0.5, 1.0, 4, 64)
