@@ -519,6 +519,98 @@ def run_kernel(args):
                 times_ms=[round(t, 4) for t in times])
 
 
+def run_grid(args):
+    """Grouped vs serial inference (backbone forward + head forward, no
+    targets) on the grid of tenants {2, 4, 6, 8} x local batch {1, 2, 4, 8}
+    samples per tenant, the grid of the paper's group-execution study
+    (§4.2).  2B-class backbone (18 blocks, d=2048, 8x256 query heads, one KV
+    head, GeGLU 16384), MLP heads, each sample one 256-row image plus 16..64
+    text tokens.  Grouped: one plan over all tenants' requests (what
+    jnx_sched_poll hands over once the batch reaches B = tenants x local
+    batch); serial: each tenant's request planned and run alone, back to
+    back.  Speedup = serial time / grouped time (CUDA events, medians)."""
+    import dataclasses
+
+    import torch
+
+    import synth
+    from paper_2607_16074_gb300 import build as B
+    from paper_2607_16074_gb300 import jnx as J
+    from paper_2607_16074_gb300 import runtime as R
+
+    B.build()
+    J.lib()
+    dev = torch.device("cuda", 0)
+    bb = synth.Backbone(n_layers=18, d=2048, n_heads=8, n_kv_heads=1, head_dim=256, d_ff=16384,
+                        glu=synth.GLU_GEGLU)
+    T_max, b_max = 8, 8
+    tenants = [synth.Tenant(synth.HEAD_MLP, chunk=16, action_dim=7, d_hidden=1024, max_images=1)
+               for _ in range(T_max)]
+    rng = np.random.default_rng(42)
+    lens = rng.integers(16, 65, size=(T_max, b_max))
+
+    def workload(T, b):
+        per = [[synth.Sample(1, int(lens[t, i])) for i in range(b)] for t in range(T)]
+        w = synth.custom_workload(bb, tenants[:T], per, req_batch=b, seed=42, name=f"grid{T}x{b}")
+        return dataclasses.replace(w, tenants=tenants)
+
+    wmax = workload(T_max, b_max)
+    bw = synth.make_backbone_weights(wmax, device=dev)
+    hw = synth.make_head_weights(wmax, device=dev)
+    backbone = R.DeviceBackbone(bb, bw, n_tenants=T_max)
+    heads = R.DeviceHeads(tenants, bb.d, hw, device=dev)
+    s = torch.cuda.current_stream()
+
+    def timed(fns):
+        for _ in range(args.warmup):
+            for f in fns:
+                f()
+        ts = []
+        for _ in range(args.steps):
+            a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(s)
+            for f in fns:
+                f()
+            e.record(s)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(e))
+        return float(np.median(ts))
+
+    grid = {}
+    for T in (2, 4, 6, 8):
+        for b in (1, 2, 4, 8):
+            w = workload(T, b)
+            inp = synth.make_inputs(w, device=dev)
+            preds = torch.zeros_like(inp["targets"])
+            plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), T_max, w.max_samples,
+                                    w.max_tokens)
+            g = R.GroupedStep(backbone, heads, R.DeviceGroup(plan, device=dev), device=dev)
+            grouped = timed([lambda g=g: g.infer(inp["vision"], inp["text_ids"], preds)])
+            serial_steps = []
+            for t in range(T):
+                sub = w.subset([t])
+                p1 = J.jnx_group_plan(sub.schemas(), oracle_requests(sub), T_max, w.max_samples,
+                                      w.max_tokens)
+                serial_steps.append(R.GroupedStep(backbone, heads, R.DeviceGroup(p1, device=dev),
+                                                  device=dev))
+            serial = timed([lambda st=st: st.infer(inp["vision"], inp["text_ids"], preds)
+                            for st in serial_steps])
+            R.check_status(g.ws_bb)
+            grid[f"{T}x{b}"] = dict(tenants=T, local_batch=b, tokens=plan.n_tokens,
+                                    grouped_ms=round(grouped, 3), serial_ms=round(serial, 3),
+                                    speedup=round(serial / grouped, 3),
+                                    grouped_tokens_per_s=round(plan.n_tokens / grouped * 1e3, 1))
+            del g, serial_steps, inp, preds
+            torch.cuda.empty_cache()
+    return dict(metric="grouped vs serial inference forward speedup, tenants x local batch",
+                unit="x", higher_is_better=True, n_gpus=1, steps=args.steps,
+                warmup=args.warmup, data="synthetic",
+                config={"workload": "2B-class backbone (18 blocks, d=2048, MQA 8x256, GeGLU "
+                                    "16384), MLP heads; samples = 1 image (256 rows) + 16..64 "
+                                    "text tokens"},
+                grid=grid)
+
+
 def dataclass_layers(w, n_layers):
     """The workload with only its first n_layers blocks (weights of the other
     blocks are not needed by a bounded oracle sample)."""
@@ -544,7 +636,12 @@ def main():
     ap.add_argument("--subset", type=int, default=0,
                     help="keep only the first K tenants' requests (a smaller case for profilers)")
     ap.add_argument("--layers", type=int, default=0, help="override the number of blocks")
+    ap.add_argument("--grid", default=None, choices=["e4"],
+                    help="grouped vs serial inference on the tenants x local batch grid")
     args = ap.parse_args()
+    if args.grid:
+        print(json.dumps(run_grid(args)), flush=True)
+        return
     if args.kernel:
         print(json.dumps(run_kernel(args)), flush=True)
         return

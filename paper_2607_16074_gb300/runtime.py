@@ -133,9 +133,10 @@ class DeviceHeads:
 
     def forward(self, group: DeviceGroup, pooled, hidden, targets, preds, loss, ws,
                 stream=None) -> None:
+        """targets and loss may both be None (inference: predictions only)."""
         J.check(J.lib().jnx_heads_forward(
-            self.arr, self.n, group.ref, _ptr(pooled), _ptr(hidden), targets.data_ptr(),
-            preds.data_ptr(), loss.data_ptr(), ws.data_ptr(), ws.numel() * ws.element_size(),
+            self.arr, self.n, group.ref, _ptr(pooled), _ptr(hidden), _ptr(targets),
+            preds.data_ptr(), _ptr(loss), ws.data_ptr(), ws.numel() * ws.element_size(),
             _stream(stream)))
 
     def backward(self, group: DeviceGroup, pooled, hidden, targets, ws, stream=None) -> None:
@@ -175,6 +176,14 @@ class GroupedStep:
         self.heads.forward(self.group, self.pooled, self.hidden, targets, preds, self.loss,
                            self.ws_h, stream)
         self.heads.backward(self.group, self.pooled, self.hidden, targets, self.ws_h, stream)
+
+    def infer(self, vision, text_ids, preds, stream=None) -> None:
+        """Inference: the shared backbone forward and every group tenant's
+        head forward (predictions only; no targets, loss or backward)."""
+        self.bb.forward(self.group, vision, text_ids,
+                        self.pooled if self.need_pooled else None, self.hidden, self.ws_bb, stream)
+        self.heads.forward(self.group, self.pooled, self.hidden, None, preds, None, self.ws_h,
+                           stream)
 
 
 class StepPipeline:

@@ -402,3 +402,29 @@ def test_step_pipeline_matches_plain_steps():
         else:
             for t in set(sub_plan.slot_tenant.tolist()):
                 assert torch.equal(loss[t], sub_loss[t]), (i, t)
+
+
+def test_inference_path_matches_training_forward_and_is_grouping_invariant():
+    # the inference step (backbone + head forward, no targets) predicts what
+    # the training step's forward predicts, and a tenant's predictions are
+    # the same in the group as alone (bit for bit: same kernels, same order)
+    w = synth.make_workload("small")
+    s = Setup(w)
+    plan, step, preds_train = s.run()
+    preds = torch.full_like(preds_train, float("nan"))
+    step.infer(s.inp_d["vision"], s.inp_d["text_ids"], preds)
+    R.check_status(step.ws_bb)
+    torch.cuda.synchronize()
+    assert torch.equal(preds, preds_train)
+    for t in (0, 5):
+        wsub = w.subset([t])
+        p1 = J.jnx_group_plan(wsub.schemas(), oracle_requests(wsub), len(w.tenants),
+                              w.max_samples, w.max_tokens)
+        st1 = R.GroupedStep(s.bb, s.heads, R.DeviceGroup(p1))
+        pr1 = torch.full_like(preds, float("nan"))
+        st1.infer(s.inp_d["vision"], s.inp_d["text_ids"], pr1)
+        torch.cuda.synchronize()
+        offs = [int(o) for o in p1.sample_target]
+        width = w.tenants[t].width
+        for o in offs:
+            assert torch.equal(pr1.view(-1)[o:o + width], preds.view(-1)[o:o + width]), (t, o)
