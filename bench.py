@@ -523,7 +523,7 @@ def run_grid(args):
     """Grouped vs serial inference (backbone forward + head forward, no
     targets) on the grid of tenants {2, 4, 6, 8} x local batch {1, 2, 4, 8}
     samples per tenant, the grid of the paper's group-execution study
-    (§4.2).  2B-class backbone (18 blocks, d=2048, 8x256 query heads, one KV
+    (§5.2).  2B-class backbone (18 blocks, d=2048, 8x256 query heads, one KV
     head, GeGLU 16384), MLP heads, each sample one 256-row image plus 16..64
     text tokens.  Grouped: one plan over all tenants' requests (what
     jnx_sched_poll hands over once the batch reaches B = tenants x local

@@ -7,17 +7,17 @@
  *   jnx_group_plan        collect the largest FIFO-compatible prefix of
  *                         requests and canonicalise it into one packed varlen
  *                         batch with its slices (App. A, "Inference Queue
- *                         Composition"; §3.3, "Multi-Tenant Group Batching").
+ *                         Composition"; §4.3, "Multi-Tenant Group Batching").
  *   jnx_backbone_forward  one shared frozen backbone forward over the packed
- *                         batch (the `encode` of App. A; §4.2 group execution).
+ *                         batch (the `encode` of App. A; §5.2 group execution).
  *   jnx_heads_forward     split the features by the recorded slices and run
  *                         each tenant's own action head and L2 loss on that
  *                         tenant's samples only (App. A `split`/`decode`;
- *                         §4.2 tenant-private loss).
+ *                         §5.2 tenant-private loss).
  *   jnx_heads_backward    gradients of each tenant's loss into that tenant's
  *                         slot only; nothing is summed across tenants
  *                         (App. A, "Actor Consumption and Version
- *                         Consistency"; §4.2 tenant-private backward).
+ *                         Consistency"; §5.2 tenant-private backward).
  *
  * Conventions for every call:
  *   - All pointers are borrowed.  The library allocates no device memory and
@@ -152,7 +152,7 @@ jnx_status jnx_group_plan(const jnx_schema* schemas, int32_t n_schemas,
  * Inference scheduler (host only; callable without a GPU)
  * ------------------------------------------------------------------------ */
 
-/* §3.3: the inference service has a maximum waiting time T and a target
+/* §4.3: the inference service has a maximum waiting time T and a target
  * batch size B; it builds a batch from requests in FIFO order and starts it
  * when the waiting time reaches T or the batch size reaches B. */
 typedef struct {

@@ -22,7 +22,7 @@ extern "C" {
 #define JNX_EPI_ROPE 4  /* out bf16 [M, ldo] = C with rotate-half RoPE at
                            position pos[row] on columns < rope_cols */
 
-/* The canonical packing step (§3.3: the VLAFeature is where the tenants'
+/* The canonical packing step (§4.3: the VLAFeature is where the tenants'
  * samples are concatenated): x[t, :] = fp32 of vision[gather_src[t]] or of
  * text_table[text_ids[-gather_src[t] - 1]].  x is [n_tokens, d] fp32.  A
  * source index outside its buffer or a text id outside [0, vocab) writes a

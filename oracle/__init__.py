@@ -12,11 +12,11 @@ What it computes, and where the paper defines it:
   canonical packed batch with its slices (App. A, "Inference Queue
   Composition": requests examined in arrival order, the largest compatible
   prefix under the batch limits, compatibility decided at the shared
-  frozen-prefix boundary; §3.3 "Multi-Tenant Group Batching": the canonical
+  frozen-prefix boundary; §4.3 "Multi-Tenant Group Batching": the canonical
   VLAFeature is the concatenation point).
 * ``model``  — the shared frozen backbone forward, the tenant-private action
   heads, the per-tenant L2 loss and the head gradients.  The grouped method
-  must reach exactly what isolated per-tenant execution computes (§4.2: group
+  must reach exactly what isolated per-tenant execution computes (§5.2: group
   execution concatenates compatible inputs for one shared forward and then
   splits features for tenant-private loss and backward; App. A: nothing is
   averaged across tenants).  So the oracle is that plain definition: every
@@ -24,7 +24,7 @@ What it computes, and where the paper defines it:
   gradient see only that tenant's samples.
 
 The paper prints no layer equations, no head definition and no numeric
-result for this path (its §4.2 figures carry no numbers in the text).  The
+result for this path (its §5.2 figures carry no numbers in the text).  The
 readings taken where it is silent are listed in the header of ``model``.
 Each function is pinned by something other than itself — closed forms,
 special cases that reduce to a textbook result, brute force on tiny inputs,

@@ -7,7 +7,7 @@ is the textbook formula, with numpy's matmul as the only library step.
 
 Where the paper is silent, these readings are taken (the paper fixes only
 that a frozen VLM backbone is shared and tenant action modules, losses and
-gradients stay private — §2.1, §3.3, §4.2, App. A):
+gradients stay private — §3.1, §4.3, §5.2, App. A):
 
   R1  pre-norm decoder block without biases:
         x <- x + W_o . Attn(RoPE(W_q n1), RoPE(W_k n1), W_v n1),  n1 = RMSNorm(x)

@@ -10,7 +10,7 @@ Paper passages followed:
   interface (same base-model interface, same model-specific shape
   constraints), not of tenant identity; canonicalisation then yields one
   physical encoder batch together with the slices that route features back.
-* §3.3, "Multi-Tenant Group Batching": the canonical VLAFeature is where
+* §4.3, "Multi-Tenant Group Batching": the canonical VLAFeature is where
   samples of different tenants are concatenated; features are afterwards
   partitioned to each tenant's action module.
 

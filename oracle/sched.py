@@ -4,7 +4,7 @@ Test infrastructure only (see the package docstring).
 
 Paper passages followed:
 
-* §3.3, "Multi-Tenant Group Batching" (its scheduling paragraph): the
+* §4.3, "Multi-Tenant Group Batching" (its scheduling paragraph): the
   inference service keeps a maximum waiting time T and a target batch size
   B; it takes samples from requests in FIFO order to build a batch and
   starts inference when the waiting time reaches T or the batch size

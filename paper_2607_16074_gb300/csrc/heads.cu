@@ -2,7 +2,7 @@
 //
 // After the shared forward the features are split by the plan's slices and
 // each tenant's own module runs on that tenant's samples only (App. A
-// `split` / `decode`; §4.2 tenant-private loss and backward).  Samples are
+// `split` / `decode`; §5.2 tenant-private loss and backward).  Samples are
 // packed tenant by tenant, so group slot g owns packed samples [s0, s1) and
 // token rows [r0, r1); every kernel takes a table of per-slot descriptors
 // (that tenant's weights and gradient buffers) and walks the segments.

@@ -10,7 +10,7 @@ namespace jnx {
 // K1 packer.  One warp per packed token; 16-byte loads of the bf16 source
 // row (a vision row or the text-embedding row of the token's id), widened to
 // the fp32 residual stream.  The canonical packed batch is where the samples
-// of all tenants are concatenated (§3.3); gather_src comes from the plan.
+// of all tenants are concatenated (§4.3); gather_src comes from the plan.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_pack(const int32_t* __restrict__ gather, int n_tokens,
                                               const uint16_t* __restrict__ vision, int64_t n_vision,

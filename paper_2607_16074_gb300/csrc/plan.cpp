@@ -4,7 +4,7 @@
 // order; the scheduler keeps the largest prefix that is compatible at the
 // shared frozen-prefix boundary and fits the batch limits; canonicalisation
 // produces one physical encoder batch and the slices that route features
-// back.  §3.3: the canonical VLAFeature is where tenants' samples are
+// back.  §4.3: the canonical VLAFeature is where tenants' samples are
 // concatenated.  Packing is varlen (no padding) so grouped results equal
 // per-sample results.
 #include <cmath>
@@ -181,7 +181,7 @@ extern "C" jnx_status jnx_group_plan(const jnx_schema* schemas, int32_t n_schema
 
 // jnx_sched_poll: the inference scheduler's decision at time `now`.
 //
-// §3.3: the inference service keeps a maximum waiting time T and a target
+// §4.3: the inference service keeps a maximum waiting time T and a target
 // batch size B, builds a batch from requests in FIFO order and starts it
 // when the waiting time reaches T or the batch size reaches B.  App. A: the
 // batch is the largest FIFO-compatible prefix the limits allow.  The batch

@@ -5,7 +5,7 @@ none of the method's arithmetic: no planning, no packing, no model math.  Both
 the fp64 oracle (through the tests) and the CUDA path receive the arrays made
 here, so the two sides always see identical inputs.
 
-The five workloads follow the shapes of the group-batching experiment (§4.2)
+The five workloads follow the shapes of the group-batching experiment (§5.2)
 and of the model families the paper runs there (a QwenOFT-like linear head, a
 PaliGemma-2B-like MQA backbone with a query head, a 7B Llama-like backbone):
 
