@@ -324,6 +324,54 @@ jnx_status jnx_heads_backward(const jnx_head* heads, int32_t n_tenants, const jn
                               const float* targets, const jnx_head_grads* grads,
                               void* workspace, size_t ws_bytes, void* stream);
 
+/* Same, but adds the gradients into grads[tenant] (gradient accumulation
+ * over successive groups before an optimizer step) instead of overwriting. */
+jnx_status jnx_heads_backward_accumulate(const jnx_head* heads, int32_t n_tenants,
+                                         const jnx_group* g, const float* pooled,
+                                         const uint16_t* hidden, const float* targets,
+                                         const jnx_head_grads* grads, void* workspace,
+                                         size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Tenant-private optimizer step
+ * ------------------------------------------------------------------------ */
+
+/* One tenant's head optimizer state (App. A, "Actor Consumption and Version
+ * Consistency": only that tenant's optimizer runs on its microbatch and only
+ * its policy version increments; nothing is shared across tenants).  Device
+ * fp32 arrays with the shapes of the head's parameters, indexed in the order
+ * w1, b1, w2, b2, q, wk, wv, wout, bout (NULL for the parameters the head's
+ * kind does not have): the master copy the updates act on, and AdamW's first
+ * and second moments (zero before the first step).  step and version are
+ * host counters that jnx_heads_adamw increments. */
+typedef struct {
+    float* master[9];
+    float* m[9];
+    float* v[9];
+    int32_t step;     /* AdamW steps taken */
+    int32_t version;  /* policy version */
+} jnx_head_opt;
+
+typedef struct {
+    float lr, beta1, beta2, eps, weight_decay;
+} jnx_adamw;
+
+/* One AdamW step (decoupled weight decay) on the head of every tenant in the
+ * group, from its fp32 gradients: per element, with t = opt[tenant].step + 1,
+ *   m <- b1 m + (1 - b1) g,  v <- b2 v + (1 - b2) g^2,
+ *   master <- master - lr ((m / (1 - b1^t)) / (sqrt(v / (1 - b2^t)) + eps)
+ *                          + weight_decay master),
+ * then the head's bf16 parameter (written in place through the jnx_head
+ * pointers) = master rounded to nearest even; opt[tenant].step and .version
+ * increment.  fp32 arithmetic.  Tenants outside the group are not touched.
+ * heads[] and opt[] are HOST arrays indexed by tenant.  Errors:
+ * JNX_ERR_INVALID_ARG (null state for a parameter the head has, lr < 0,
+ * b1 or b2 outside [0, 1), eps < 0, weight_decay < 0); nothing is written
+ * on error. */
+jnx_status jnx_heads_adamw(const jnx_head* heads, const jnx_head_grads* grads,
+                           jnx_head_opt* opt, int32_t n_tenants, const jnx_group* g,
+                           const jnx_adamw* hp, void* stream);
+
 /* ------------------------------------------------------------------------
  * Status and helpers
  * ------------------------------------------------------------------------ */
@@ -356,6 +404,7 @@ jnx_status jnx_pack_gate_up(const uint16_t* w_gate, const uint16_t* w_up, int32_
 #define JNX_K_HEADS_BWD 11 /* work = FLOPs */
 #define JNX_K_GEMM 12      /* jnx_op_gemm; work = FLOPs */
 #define JNX_K_LORA 13      /* LoRA row tenants / down-projections; work = FLOPs */
+#define JNX_K_ADAMW 14     /* tenant-private head optimizer step; work = HBM bytes */
 
 /* While enabled on the calling thread, each kernel launch of the library is
  * bracketed by two CUDA events on its stream (up to `capacity` launches are

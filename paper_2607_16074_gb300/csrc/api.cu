@@ -480,7 +480,7 @@ jnx_status check_heads(const jnx_head* heads, int32_t n_tenants, const jnx_group
 
 // Fill the per-slot table for group slots [g0, g0 + n) and describe the batch.
 HeadBatch fill_table(HeadTable& tab, const jnx_head* heads, const jnx_head_grads* grads,
-                     const jnx_group* g, int g0, int n) {
+                     const jnx_group* g, int g0, int n, bool accum = false) {
     HeadBatch b{};
     b.g0 = g0;
     b.n = n;
@@ -491,6 +491,7 @@ HeadBatch fill_table(HeadTable& tab, const jnx_head* heads, const jnx_head_grads
         const jnx_head& h = heads[t];
         HeadSlot& hs = tab.slot[i];
         hs = HeadSlot{};
+        hs.accum = accum ? 1 : 0;
         hs.kind = h.kind;
         hs.tenant = t;
         hs.s0 = g->h_seg_offsets[g0 + i];
@@ -611,12 +612,10 @@ extern "C" jnx_status jnx_heads_forward(const jnx_head* heads, int32_t n_tenants
     return JNX_OK;
 }
 
-extern "C" jnx_status jnx_heads_backward(const jnx_head* heads, int32_t n_tenants,
-                                         const jnx_group* g, const float* pooled,
-                                         const uint16_t* hidden, const float* targets,
-                                         const jnx_head_grads* grads, void* workspace,
-                                         size_t ws_bytes, void* stream) {
-    clear_error();
+static jnx_status heads_backward(const jnx_head* heads, int32_t n_tenants, const jnx_group* g,
+                                 const float* pooled, const uint16_t* hidden,
+                                 const jnx_head_grads* grads, void* workspace, size_t ws_bytes,
+                                 void* stream, bool accum) {
     jnx_status st;
     if (!grads && g && g->n_slots > 0)
         return fail(JNX_ERR_INVALID_ARG, "heads backward: null grads");
@@ -632,13 +631,35 @@ extern "C" jnx_status jnx_heads_backward(const jnx_head* heads, int32_t n_tenant
     HeadTable tab;
     for (int g0 = 0; g0 < g->n_slots; g0 += kMaxSlots) {
         const int n = std::min(kMaxSlots, g->n_slots - g0);
-        HeadBatch b = fill_table(tab, heads, grads, g, g0, n);
+        HeadBatch b = fill_table(tab, heads, grads, g, g0, n, accum);
         TraceScope ts(JNX_K_HEADS_BWD, heads_flops(tab, n, true), s);
         if ((st = heads_backward_launch(tab, b, w.sc, pooled, d, hidden, g->cu_seqlens,
                                         g->sample_slot, s)))
             return st;
     }
     return JNX_OK;
+}
+
+extern "C" jnx_status jnx_heads_backward(const jnx_head* heads, int32_t n_tenants,
+                                         const jnx_group* g, const float* pooled,
+                                         const uint16_t* hidden, const float* targets,
+                                         const jnx_head_grads* grads, void* workspace,
+                                         size_t ws_bytes, void* stream) {
+    clear_error();
+    (void)targets;  // the loss gradient dy was kept by the forward
+    return heads_backward(heads, n_tenants, g, pooled, hidden, grads, workspace, ws_bytes, stream,
+                          false);
+}
+
+extern "C" jnx_status jnx_heads_backward_accumulate(const jnx_head* heads, int32_t n_tenants,
+                                                    const jnx_group* g, const float* pooled,
+                                                    const uint16_t* hidden, const float* targets,
+                                                    const jnx_head_grads* grads, void* workspace,
+                                                    size_t ws_bytes, void* stream) {
+    clear_error();
+    (void)targets;
+    return heads_backward(heads, n_tenants, g, pooled, hidden, grads, workspace, ws_bytes, stream,
+                          true);
 }
 
 // ---------------------------------------------------------------------------

@@ -157,8 +157,8 @@ __global__ void __launch_bounds__(256) k_head_dw_out(const __grid_constant__ Hea
         acc += g * h[(size_t)s * ld_h + j];
         accb += g;
     }
-    hs.g_w2[idx] = acc;
-    if (j == 0) hs.g_b2[o] = accb;
+    hs.g_w2[idx] = hs.accum ? hs.g_w2[idx] + acc : acc;
+    if (j == 0) hs.g_b2[o] = hs.accum ? hs.g_b2[o] + accb : accb;
 }
 
 // Gradient into the output layer's input: dh[s, j] = (sum_o dy[s, o] W[o, j])
@@ -211,12 +211,20 @@ __global__ void __launch_bounds__(256) k_mlp_dw1(const __grid_constant__ HeadTab
             acc.z += g * x.z;
             acc.w += g * x.w;
         }
-        *reinterpret_cast<float4*>(hs.g_w1 + (size_t)j * hs.d_in + k4 * 4) = acc;
+        float4* dst = reinterpret_cast<float4*>(hs.g_w1 + (size_t)j * hs.d_in + k4 * 4);
+        if (hs.accum) {
+            const float4 old = *dst;
+            acc.x += old.x;
+            acc.y += old.y;
+            acc.z += old.z;
+            acc.w += old.w;
+        }
+        *dst = acc;
     }
     if (blockIdx.z == 0 && threadIdx.x == 0) {
         float accb = 0.f;
         for (int s = hs.s0; s < hs.s1; ++s) accb += dz[(size_t)s * ld + j];
-        hs.g_b1[j] = accb;
+        hs.g_b1[j] = hs.accum ? hs.g_b1[j] + accb : accb;
     }
 }
 
@@ -413,7 +421,7 @@ __global__ void __launch_bounds__(256) k_xattn_dq(const __grid_constant__ HeadTa
     if (i >= hs.nq * hs.dq) return;
     float acc = 0.f;
     for (int s = hs.s0; s < hs.s1; ++s) acc += dQs[(size_t)s * ld_h + i];
-    hs.g_q[i] = acc;
+    hs.g_q[i] = hs.accum ? hs.g_q[i] + acc : acc;
 }
 
 // dW[c, e] = sum over the slot's token rows r of g[r, c] * X[r, e], for
@@ -556,10 +564,19 @@ __global__ void __launch_bounds__(128) k_xattn_wgrad(const __grid_constant__ Hea
         for (int j = 0; j < 8; ++j) {
             const int c = c0 + wm * 32 + im * 16 + g;
             const int e = e0 + wn * 64 + j * 8 + 2 * t;
-            *reinterpret_cast<float2*>(out + (size_t)c * hs.d_in + e) =
-                make_float2(acc[im][j][0], acc[im][j][1]);
-            *reinterpret_cast<float2*>(out + (size_t)(c + 8) * hs.d_in + e) =
-                make_float2(acc[im][j][2], acc[im][j][3]);
+            float2* d0 = reinterpret_cast<float2*>(out + (size_t)c * hs.d_in + e);
+            float2* d1 = reinterpret_cast<float2*>(out + (size_t)(c + 8) * hs.d_in + e);
+            float2 v0 = make_float2(acc[im][j][0], acc[im][j][1]);
+            float2 v1 = make_float2(acc[im][j][2], acc[im][j][3]);
+            if (hs.accum) {
+                const float2 o0 = *d0, o1 = *d1;
+                v0.x += o0.x;
+                v0.y += o0.y;
+                v1.x += o1.x;
+                v1.y += o1.y;
+            }
+            *d0 = v0;
+            *d1 = v1;
         }
     }
 }

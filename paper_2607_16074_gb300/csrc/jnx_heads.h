@@ -18,7 +18,7 @@ struct HeadSlot {
     int hid;         // input width of the output layer: MLP d_hidden, query head nq * dq
     int width;       // outputs per sample
     int nq, dq;      // query head
-    int pad_;
+    int accum;       // add into the gradient buffers instead of overwriting them
     const uint16_t *w1, *b1;   // MLP first layer
     const uint16_t *w2, *b2;   // output layer: MLP W2/b2 or query-head Wout/bout
     const uint16_t *q, *wk, *wv;

@@ -108,6 +108,19 @@ class jnx_head_grads(C.Structure):
                                           "bout")]
 
 
+HEAD_PARAMS = ("w1", "b1", "w2", "b2", "q", "wk", "wv", "wout", "bout")
+
+
+class jnx_head_opt(C.Structure):
+    _fields_ = [("master", C.c_void_p * 9), ("m", C.c_void_p * 9), ("v", C.c_void_p * 9),
+                ("step", C.c_int32), ("version", C.c_int32)]
+
+
+class jnx_adamw(C.Structure):
+    _fields_ = [("lr", C.c_float), ("beta1", C.c_float), ("beta2", C.c_float),
+                ("eps", C.c_float), ("weight_decay", C.c_float)]
+
+
 _LIB: Optional[C.CDLL] = None
 
 EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_workspace_bytes",
@@ -115,7 +128,8 @@ EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_work
            "jnx_heads_backward", "jnx_check_status", "jnx_pack_gate_up", "jnx_op_pack",
            "jnx_op_rmsnorm", "jnx_op_gemm_workspace_bytes", "jnx_op_gemm", "jnx_op_attention",
            "jnx_op_final_pool", "jnx_trace_enable", "jnx_trace_disable", "jnx_trace_count",
-           "jnx_trace_read", "jnx_op_gemm_rope_noalloc", "jnx_sched_poll")
+           "jnx_trace_read", "jnx_op_gemm_rope_noalloc", "jnx_sched_poll",
+           "jnx_heads_backward_accumulate", "jnx_heads_adamw")
 
 
 def lib() -> C.CDLL:
@@ -145,6 +159,12 @@ def lib() -> C.CDLL:
                                     vp, vp, vp, sz, vp]),
         "jnx_heads_backward": (i32, [C.POINTER(jnx_head), i32, C.POINTER(jnx_group), vp, vp, vp,
                                      C.POINTER(jnx_head_grads), vp, sz, vp]),
+        "jnx_heads_backward_accumulate": (i32, [C.POINTER(jnx_head), i32, C.POINTER(jnx_group),
+                                                vp, vp, vp, C.POINTER(jnx_head_grads), vp, sz,
+                                                vp]),
+        "jnx_heads_adamw": (i32, [C.POINTER(jnx_head), C.POINTER(jnx_head_grads),
+                                  C.POINTER(jnx_head_opt), i32, C.POINTER(jnx_group),
+                                  C.POINTER(jnx_adamw), vp]),
         "jnx_check_status": (i32, [vp, vp]),
         "jnx_pack_gate_up": (i32, [vp, vp, i32, i32, vp, vp]),
         "jnx_op_pack": (i32, [C.POINTER(jnx_group), vp, i64, vp, i64, vp, i32, i32, vp, vp, vp]),
@@ -286,7 +306,8 @@ def jnx_sched_poll(schemas: Sequence[dict], requests: Sequence[dict], arrival: S
 # ---------------------------------------------------------------------------
 KERNEL_NAMES = {1: "pack", 2: "rmsnorm", 3: "gemm_qkv_rope", 4: "attention", 5: "gemm_o_resid",
                 6: "gemm_gate_up_glu", 7: "gemm_down_resid", 8: "final_norm_pool",
-                9: "rope_table", 10: "heads_fwd", 11: "heads_bwd", 12: "gemm", 13: "lora_down"}
+                9: "rope_table", 10: "heads_fwd", 11: "heads_bwd", 12: "gemm", 13: "lora_down",
+                14: "heads_adamw"}
 TENSOR_KERNELS = (3, 4, 5, 6, 7, 12, 13)
 
 

@@ -139,10 +139,44 @@ class DeviceHeads:
             preds.data_ptr(), _ptr(loss), ws.data_ptr(), ws.numel() * ws.element_size(),
             _stream(stream)))
 
-    def backward(self, group: DeviceGroup, pooled, hidden, targets, ws, stream=None) -> None:
-        J.check(J.lib().jnx_heads_backward(
-            self.arr, self.n, group.ref, _ptr(pooled), _ptr(hidden), targets.data_ptr(),
-            self.garr, ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)))
+    def backward(self, group: DeviceGroup, pooled, hidden, targets, ws, stream=None,
+                 accumulate: bool = False) -> None:
+        """Gradients into each group tenant's slot: overwritten, or added to
+        what is there (gradient accumulation) with accumulate=True."""
+        fn = J.lib().jnx_heads_backward_accumulate if accumulate else J.lib().jnx_heads_backward
+        J.check(fn(self.arr, self.n, group.ref, _ptr(pooled), _ptr(hidden), targets.data_ptr(),
+                   self.garr, ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)))
+
+    def init_optimizer(self) -> None:
+        """Tenant-private AdamW state: an fp32 master copy of every head
+        parameter (from its bf16 value) and zero moments, per tenant."""
+        self.opt = (J.jnx_head_opt * max(1, self.n))()
+        self.opt_state: List[Dict[str, Dict[str, torch.Tensor]]] = []
+        for t, hw in enumerate(self.keep):
+            st = {}
+            for k, name in enumerate(J.HEAD_PARAMS):
+                if name not in hw:
+                    continue
+                p = hw[name]
+                st[name] = dict(master=p.float().clone(), m=torch.zeros_like(p, dtype=torch.float32),
+                                v=torch.zeros_like(p, dtype=torch.float32))
+                self.opt[t].master[k] = st[name]["master"].data_ptr()
+                self.opt[t].m[k] = st[name]["m"].data_ptr()
+                self.opt[t].v[k] = st[name]["v"].data_ptr()
+            self.opt_state.append(st)
+
+    def adamw_step(self, group: DeviceGroup, lr: float, beta1: float = 0.9,
+                   beta2: float = 0.999, eps: float = 1e-8, weight_decay: float = 0.0,
+                   stream=None) -> None:
+        """One AdamW step on every group tenant's head from its gradients
+        (bf16 parameters updated in place; the tenant's step and policy
+        version counters increment)."""
+        hp = J.jnx_adamw(lr, beta1, beta2, eps, weight_decay)
+        J.check(J.lib().jnx_heads_adamw(self.arr, self.garr, self.opt, self.n, group.ref,
+                                        C.byref(hp), _stream(stream)))
+
+    def version(self, t: int) -> int:
+        return int(self.opt[t].version)
 
 
 def check_status(ws: torch.Tensor, stream=None) -> None:
