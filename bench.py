@@ -493,6 +493,24 @@ def run_kernel(args):
                                           len(lens), max(lens), out.data_ptr(), None,
                                           s.cuda_stream)
         work, unit = sum(4.0 * l * l * Hq * hdq for l in lens), "TFLOP/s"
+    elif k == "heads_adamw":
+        # the 7B-class group's 32 MLP heads (4096 -> 1024 -> 56): one AdamW
+        # step over all of them, 30 bytes per parameter element
+        import synth
+        from paper_2607_16074_gb300 import runtime as R
+        w = synth.make_workload("llama7b")
+        hw = synth.make_head_weights(w, device=dev)
+        heads = R.DeviceHeads(w.tenants, w.backbone.d, hw, device=dev)
+        heads.init_optimizer()
+        for gr in heads.grads:
+            for v in gr.values():
+                v.normal_(generator=g)
+        plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), len(w.tenants), w.max_samples,
+                                w.max_tokens)
+        grp = R.DeviceGroup(plan, device=dev)
+        n_el = sum(v.numel() for gr in heads.grads for v in gr.values())
+        call = lambda: (heads.adamw_step(grp, lr=1e-4, weight_decay=0.01), 0)[1]
+        work, unit = 30.0 * n_el, "GB/s"
     elif k == "rmsnorm":
         x = torch.randn(M, d, generator=g, device=dev)
         gam = rnd(d)
@@ -631,7 +649,8 @@ def main():
     ap.add_argument("--reference-layers", type=int, default=1)
     ap.add_argument("--kernel", default=None,
                     help="time one kernel alone (gemm_gu, gemm_qkv, gemm_o, gemm_down, "
-                         "attention, rmsnorm) on 7B-class shapes with --tokens rows")
+                         "attention, attention_mqa, rmsnorm, heads_adamw) on 7B-class shapes "
+                         "with --tokens rows")
     ap.add_argument("--tokens", type=int, default=8192)
     ap.add_argument("--subset", type=int, default=0,
                     help="keep only the first K tenants' requests (a smaller case for profilers)")

@@ -6,7 +6,7 @@
 // averaged across tenants.  Here one launch steps every tenant of a group,
 // each on its own parameters, gradients and moments.
 //
-// AdamW with decoupled weight decay, fp32, one thread per parameter element:
+// AdamW with decoupled weight decay, fp32, four parameter elements a thread:
 // the kernel streams the gradient, the two moments and the fp32 master once
 // and writes the moments, the master and the bf16 parameter the forward
 // reads (30 bytes per element; HBM-bound).
@@ -36,16 +36,43 @@ struct AdamTable {
     AdamSeg seg[kMaxSeg];
 };
 
+__device__ __forceinline__ float adamw_elem(float g, float& m, float& v, float p, float c1,
+                                            float c2, float lr, float b1, float b2, float eps,
+                                            float wd) {
+    m = b1 * m + (1.f - b1) * g;
+    v = b2 * v + (1.f - b2) * g * g;
+    return p - lr * ((m * c1) / (sqrtf(v * c2) + eps) + wd * p);
+}
+
+// Four elements per thread (16-byte loads) where the segment's arrays allow
+// it, then a scalar tail.
 __global__ void __launch_bounds__(256) k_adamw(const __grid_constant__ AdamTable tab, float lr,
                                                float b1, float b2, float eps, float wd) {
     const AdamSeg& s = tab.seg[blockIdx.y];
-    for (long long i = (long long)blockIdx.x * 256 + threadIdx.x; i < s.n;
-         i += (long long)gridDim.x * 256) {
-        const float g = s.g[i];
-        const float m = b1 * s.m[i] + (1.f - b1) * g;
-        const float v = b2 * s.v[i] + (1.f - b2) * g * g;
-        float p = s.master[i];
-        p = p - lr * ((m * s.c1) / (sqrtf(v * s.c2) + eps) + wd * p);
+    const long long stride = (long long)gridDim.x * 256;
+    const long long t0 = (long long)blockIdx.x * 256 + threadIdx.x;
+    const bool vec = ((reinterpret_cast<uintptr_t>(s.g) | reinterpret_cast<uintptr_t>(s.m) |
+                       reinterpret_cast<uintptr_t>(s.v) | reinterpret_cast<uintptr_t>(s.master)) &
+                      15) == 0 &&
+                     (reinterpret_cast<uintptr_t>(s.p) & 7) == 0;
+    const long long n4 = vec ? s.n / 4 : 0;
+    for (long long i = t0; i < n4; i += stride) {
+        const float4 g = reinterpret_cast<const float4*>(s.g)[i];
+        float4 m = reinterpret_cast<float4*>(s.m)[i];
+        float4 v = reinterpret_cast<float4*>(s.v)[i];
+        float4 p = reinterpret_cast<float4*>(s.master)[i];
+        p.x = adamw_elem(g.x, m.x, v.x, p.x, s.c1, s.c2, lr, b1, b2, eps, wd);
+        p.y = adamw_elem(g.y, m.y, v.y, p.y, s.c1, s.c2, lr, b1, b2, eps, wd);
+        p.z = adamw_elem(g.z, m.z, v.z, p.z, s.c1, s.c2, lr, b1, b2, eps, wd);
+        p.w = adamw_elem(g.w, m.w, v.w, p.w, s.c1, s.c2, lr, b1, b2, eps, wd);
+        reinterpret_cast<float4*>(s.m)[i] = m;
+        reinterpret_cast<float4*>(s.v)[i] = v;
+        reinterpret_cast<float4*>(s.master)[i] = p;
+        reinterpret_cast<uint2*>(s.p)[i] = make_uint2(pack_bf2(p.x, p.y), pack_bf2(p.z, p.w));
+    }
+    for (long long i = 4 * n4 + t0; i < s.n; i += stride) {
+        float m = s.m[i], v = s.v[i];
+        const float p = adamw_elem(s.g[i], m, v, s.master[i], s.c1, s.c2, lr, b1, b2, eps, wd);
         s.m[i] = m;
         s.v[i] = v;
         s.master[i] = p;
@@ -120,7 +147,7 @@ extern "C" jnx_status jnx_heads_adamw(const jnx_head* heads, const jnx_head_grad
                 tab.seg[k] = segs[a + k];
                 mx = std::max(mx, segs[a + k].n);
             }
-            const int bx = (int)std::min<long long>((mx + 255) / 256, 1024);
+            const int bx = (int)std::min<long long>((mx / 4 + 255) / 256 + 1, 1024);
             k_adamw<<<dim3(bx, ns), 256, 0, s>>>(tab, hp->lr, hp->beta1, hp->beta2, hp->eps,
                                                  hp->weight_decay);
             cudaError_t e = cudaGetLastError();
