@@ -373,6 +373,86 @@ jnx_status jnx_heads_adamw(const jnx_head* heads, const jnx_head_grads* grads,
                            const jnx_adamw* hp, void* stream);
 
 /* ------------------------------------------------------------------------
+ * Trainable per-tenant adapters: the LoRA backward through the frozen backbone
+ *
+ * A tenant's trainable module may be a lightweight adapter over the fixed
+ * base (§3.1); its loss, gradients and optimizer state stay its own (§5.2,
+ * App. A).  With the backbone's LoRA adapters (lora_rank 16), one grouped
+ * step gives every group tenant the gradient of its own loss with respect
+ * to its own adapters:
+ *   jnx_backbone_forward_train   forward, keeping each block's residual input
+ *   jnx_heads_forward            per-tenant heads and losses
+ *   jnx_heads_backward_input     head gradients + dloss/d(final normed rows)
+ *   jnx_backbone_backward_lora   adapter gradients of every layer
+ * ------------------------------------------------------------------------ */
+
+/* Bytes of the buffer jnx_backbone_forward_train keeps: fp32
+ * [n_layers + 1, n_tokens, d_model]. */
+size_t jnx_backbone_saved_bytes(const jnx_backbone* bb, int32_t n_tokens);
+
+/* jnx_backbone_forward that also writes saved[l] = the fp32 residual stream
+ * entering block l (l < n_layers) and saved[n_layers] = the one entering
+ * the final RMSNorm. */
+jnx_status jnx_backbone_forward_train(const jnx_backbone* bb, const jnx_group* g,
+                                      const uint16_t* vision, int64_t n_vision_rows,
+                                      const int32_t* text_ids, int64_t n_text,
+                                      float* pooled, uint16_t* hidden, float* saved,
+                                      void* workspace, size_t ws_bytes, void* stream);
+
+/* jnx_heads_backward, and also d_hidden [n_tokens, d] fp32 = the gradient
+ * of each row's tenant loss with respect to that row's final normed
+ * hidden: (dz W1) / L_s on every row of an MLP-head sample (the feature is
+ * the mean of the rows), dk W_k + dv W_v on a query-head row.  Every row of
+ * the group is written. */
+jnx_status jnx_heads_backward_input(const jnx_head* heads, int32_t n_tenants,
+                                    const jnx_group* g, const float* pooled,
+                                    const uint16_t* hidden, const float* targets,
+                                    const jnx_head_grads* grads, float* d_hidden,
+                                    void* workspace, size_t ws_bytes, void* stream);
+
+/* Transposed copies of one block's frozen weights (device bf16), read by
+ * the backward's input-gradient GEMMs; jnx_transpose builds them once.
+ *   w_qkv_t  [d, (H + 2 Hkv) hd] = w_qkv^T
+ *   w_o_t    [H hd, d]           = w_o^T
+ *   w_gu_t   [d, 2 F]            = w_gu^T (columns in w_gu's packed row order)
+ *   w_down_t [F, d]              = w_down^T */
+typedef struct {
+    const uint16_t* w_qkv_t;
+    const uint16_t* w_o_t;
+    const uint16_t* w_gu_t;
+    const uint16_t* w_down_t;
+} jnx_layer_t;
+
+/* One block's adapter gradients (device fp32), the shapes of the adapters:
+ * a_* [n_tenants, r, in], b_* [n_tenants, out, r]. */
+typedef struct {
+    float *a_q, *b_q, *a_k, *b_k, *a_v, *b_v, *a_o, *b_o;
+} jnx_lora_grads;
+
+/* dst [batch][cols][rows] = src [batch][rows][cols] (bf16, not in place). */
+jnx_status jnx_transpose(const uint16_t* src, int32_t batch, int32_t rows, int32_t cols,
+                         uint16_t* dst, void* stream);
+
+/* Workspace bytes jnx_backbone_backward_lora needs for n_tokens rows. */
+size_t jnx_backbone_backward_workspace_bytes(const jnx_backbone* bb, int32_t n_tokens);
+
+/* The gradient of each group tenant's loss with respect to its own LoRA
+ * adapters in every block, written (accumulate == 0) or added into the
+ * tenant's slice of grads[l] (HOST array [n_layers]); slices of tenants
+ * outside the group are not touched.  saved: what jnx_backbone_forward_train
+ * kept for this group; d_hidden [n_tokens, d] fp32: dloss/d(final normed
+ * rows) (jnx_heads_backward_input).  layers_t: HOST array [n_layers] of the
+ * transposed weights.  Each block is recomputed from its saved input.
+ * Errors: JNX_ERR_INVALID_ARG (no rank-16 adapters, null buffer, a group
+ * tenant without an adapter), JNX_ERR_UNSUPPORTED (widths not multiples of
+ * 256, more than 256 group tenants), JNX_ERR_WORKSPACE. */
+jnx_status jnx_backbone_backward_lora(const jnx_backbone* bb, const jnx_layer_t* layers_t,
+                                      const jnx_group* g, const float* saved,
+                                      const float* d_hidden, const jnx_lora_grads* grads,
+                                      int32_t accumulate, void* workspace, size_t ws_bytes,
+                                      void* stream);
+
+/* ------------------------------------------------------------------------
  * Status and helpers
  * ------------------------------------------------------------------------ */
 
@@ -405,6 +485,10 @@ jnx_status jnx_pack_gate_up(const uint16_t* w_gate, const uint16_t* w_up, int32_
 #define JNX_K_GEMM 12      /* jnx_op_gemm; work = FLOPs */
 #define JNX_K_LORA 13      /* LoRA row tenants / down-projections; work = FLOPs */
 #define JNX_K_ADAMW 14     /* tenant-private head optimizer step; work = HBM bytes */
+#define JNX_K_GEMM_BWD 15  /* input-gradient GEMMs of the adapter backward; work = FLOPs */
+#define JNX_K_ATTN_BWD 16  /* attention backward; work = FLOPs of its five products */
+#define JNX_K_NORM_BWD 17  /* RMSNorm backward, attention-backward prologue; work = HBM bytes */
+#define JNX_K_LORA_BWD 18  /* adapter gradients and up-projections; work = FLOPs */
 
 /* While enabled on the calling thread, each kernel launch of the library is
  * bracketed by two CUDA events on its stream (up to `capacity` launches are

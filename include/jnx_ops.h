@@ -69,6 +69,60 @@ jnx_status jnx_op_final_pool(const float* x, const uint16_t* gamma, float eps,
                              const int32_t* cu_seqlens, int32_t n_samples, int32_t d,
                              float* pooled, uint16_t* hidden, void* stream);
 
+/* ---- stages of the adapter backward (jnx_backbone_backward_lora) ---- */
+
+/* jnx_op_attention that also writes lse [n_tokens, H] fp32: each query
+ * row's log2-sum-exp of its scaled scores, log2(sum_j 2^(s_j log2(e) /
+ * sqrt(hd))), from which the backward recomputes the probabilities. */
+jnx_status jnx_op_attention_lse(const uint16_t* qkv, int32_t n_tokens, int32_t n_heads,
+                                int32_t n_kv_heads, int32_t head_dim, const int32_t* cu_seqlens,
+                                int32_t n_samples, int32_t max_seqlen, uint16_t* out, float* lse,
+                                int32_t* status, void* stream);
+
+/* The attention backward's prologue: dO [n_tokens, H hd] bf16 = bf16(datt)
+ * (fp32) and D [n_tokens, H] = per head, the sum over its hd columns of
+ * dO * att (att = the forward's output, bf16). */
+jnx_status jnx_op_attention_backward_prep(const float* datt, const uint16_t* att, int32_t n_tokens,
+                                          int32_t n_heads, int32_t head_dim, uint16_t* dO,
+                                          float* D, void* stream);
+
+/* Workspace bytes of jnx_op_attention_backward. */
+size_t jnx_op_attention_backward_workspace_bytes(int32_t n_tokens, int32_t max_seqlen,
+                                                 int32_t head_dim);
+
+/* Gradients of jnx_op_attention with respect to its input qkv, given dO,
+ * the forward's lse and D (jnx_op_attention_backward_prep): for query head
+ * h on K/V head g, P = softmax(q k^T / sqrt(hd)) inside each sample,
+ * dv_g += P^T dO_h, dS = P * (dO_h v_g^T - D), dq_h = dS k_g / sqrt(hd),
+ * dk_g += dS^T q_h / sqrt(hd).  qkv holds q and k after RoPE; dqkv
+ * [n_tokens, (H + 2 Hkv) hd] bf16 receives the gradients of the pre-RoPE
+ * projections (dq, dk rotated back by the rotate-half RoPE of theta at
+ * pos[t]; dv as is).  h_cu_seqlens is the host copy of cu_seqlens (the work
+ * list is built from it).  A wait that ran out of time writes
+ * JNX_ERR_TIMEOUT to *status. */
+jnx_status jnx_op_attention_backward(const uint16_t* qkv, const uint16_t* dO, const float* lse,
+                                     const float* D, int32_t n_tokens, int32_t n_heads,
+                                     int32_t n_kv_heads, int32_t head_dim,
+                                     const int32_t* cu_seqlens, const int32_t* h_cu_seqlens,
+                                     int32_t n_samples, int32_t max_seqlen, const int32_t* pos,
+                                     float rope_theta, uint16_t* dqkv, void* workspace,
+                                     size_t ws_bytes, int32_t* status, void* stream);
+
+/* RMSNorm backward: with s = rsqrt(mean(x^2) + eps) per row,
+ * dx = dres + s gamma dn - x s^3 mean(gamma dn x) (fp32; dres may be NULL
+ * or dx itself) and dx_bf = bf16(dx) when not NULL.  d % 128 == 0. */
+jnx_status jnx_op_rms_backward(const float* x, const uint16_t* gamma, float eps, const float* dn,
+                               const float* dres, int32_t M, int32_t d, float* dx,
+                               uint16_t* dx_bf, void* stream);
+
+/* The feed-forward backward's first GEMM with the GLU backward fused:
+ * dm[M, F] = A[M, K] W[F, K]^T is the gradient at act(g) * u; gu [M, 2F]
+ * bf16 holds g | u in JNX_EPI_GLU's packed order (128-column blocks
+ * alternating gate and up) on entry and dg = dm u act'(g) | du = dm act(g)
+ * in the same order on return.  F % 256 == 0, K % 64 == 0. */
+jnx_status jnx_op_gemm_glu_backward(const uint16_t* A, const uint16_t* W, int32_t M, int32_t F,
+                                    int32_t K, uint16_t* gu, int32_t act, void* stream);
+
 /* The fused QKV projection + RoPE of jnx_op_gemm (JNX_EPI_ROPE) for callers
  * that cannot allocate device memory — e.g. a plugin in a serving process
  * whose pool owns every device allocation, or a batching worker that must

@@ -4,6 +4,7 @@
 #include <vector>
 
 #include "../../include/jnx_ops.h"
+#include "jnx_bwd.h"
 #include "jnx_dev.cuh"
 #include "jnx_heads.h"
 #include "jnx_kernels.h"
@@ -34,8 +35,6 @@ struct BackboneWs {
     size_t bytes;
 };
 
-constexpr int kMaxRopePos = 1 << 16;  // longest sample the workspace reserves RoPE rows for
-
 BackboneWs carve_backbone(const jnx_backbone* bb, int64_t N, void* base) {
     uint8_t* p = static_cast<uint8_t*>(base);
     BackboneWs w{};
@@ -63,6 +62,15 @@ BackboneWs carve_backbone(const jnx_backbone* bb, int64_t N, void* base) {
     w.bytes = off;
     return w;
 }
+
+jnx_status cuda_status(const char* what) {
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+}  // namespace
+
+namespace jnx {
 
 jnx_status check_backbone(const jnx_backbone* bb) {
     if (!bb || !bb->layers || !bb->text_table || !bb->final_norm)
@@ -114,24 +122,44 @@ jnx_status check_group(const jnx_group* g) {
     return JNX_OK;
 }
 
-jnx_status cuda_status(const char* what) {
-    cudaError_t e = cudaGetLastError();
-    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+// Attention work items (sample, 128-row tile), most expensive first, so
+// that a persistent kernel's round-robin over them ends with the cheap ones
+// (longest-processing-time-first balance across SMs).  The same list serves
+// every layer, the forward and the backward: the samples do not change.
+jnx_status build_attn_items(const jnx_group* g, std::vector<int2>& sorted) {
+    std::vector<int2> items;
+    std::vector<int> cost;
+    for (int i = 0; i < g->n_samples; ++i) {
+        const int L = g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i];
+        for (int q0 = 0; q0 < L; q0 += 128) {
+            items.push_back(make_int2(i, q0 / 128));
+            cost.push_back((L + 63) / 64);  // 64-row tiles the item's loop walks
+        }
+    }
+    std::vector<int> order(items.size());
+    for (size_t i = 0; i < order.size(); ++i) order[i] = (int)i;
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return cost[a] > cost[b]; });
+    sorted.resize(items.size());
+    for (size_t i = 0; i < order.size(); ++i) sorted[i] = items[order[i]];
+    if (sorted.size() > (size_t)g->n_tokens + g->n_tokens / 128 + 1)
+        return fail(JNX_ERR_INVALID_ARG, "attention items: sample lengths exceed n_tokens");
+    return JNX_OK;
 }
 
-}  // namespace
+}  // namespace jnx
 
 extern "C" size_t jnx_backbone_workspace_bytes(const jnx_backbone* bb, int32_t n_tokens) {
     if (!bb || n_tokens < 0) return 0;
     return carve_backbone(bb, n_tokens, nullptr).bytes;
 }
 
-extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_group* g,
-                                           const uint16_t* vision, int64_t n_vision_rows,
-                                           const int32_t* text_ids, int64_t n_text, float* pooled,
-                                           uint16_t* hidden, void* workspace, size_t ws_bytes,
-                                           void* stream) {
-    clear_error();
+// The forward; with `saved`, also keeps each block's fp32 residual input
+// and the final residual ([n_layers + 1, N, d]) for the adapter backward.
+static jnx_status backbone_forward(const jnx_backbone* bb, const jnx_group* g,
+                                   const uint16_t* vision, int64_t n_vision_rows,
+                                   const int32_t* text_ids, int64_t n_text, float* pooled,
+                                   uint16_t* hidden, float* saved, void* workspace, size_t ws_bytes,
+                                   void* stream) {
     jnx_status st;
     if ((st = check_backbone(bb)) || (st = check_group(g))) return st;
     if (!workspace) return fail(JNX_ERR_INVALID_ARG, "backbone: null workspace");
@@ -195,30 +223,11 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
         const double L = g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i];
         attn_flops += 4.0 * L * L * H * hd;
     }
-    // Attention work items, most expensive first, so that the persistent
-    // attention kernel's round-robin over them ends with the cheap ones
-    // (longest-processing-time-first balance across SMs).  Shared by every
-    // layer: the samples do not change.
     int n_items = 0;
     {
-        std::vector<int2> items;
-        std::vector<int> cost;
-        for (int i = 0; i < g->n_samples; ++i) {
-            const int L = g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i];
-            for (int q0 = 0; q0 < L; q0 += 128) {
-                items.push_back(make_int2(i, q0 / 128));
-                cost.push_back((L + 63) / 64);  // key tiles the item walks
-            }
-        }
-        std::vector<int> order(items.size());
-        for (size_t i = 0; i < order.size(); ++i) order[i] = (int)i;
-        std::stable_sort(order.begin(), order.end(),
-                         [&](int a, int b) { return cost[a] > cost[b]; });
-        std::vector<int2> sorted(items.size());
-        for (size_t i = 0; i < order.size(); ++i) sorted[i] = items[order[i]];
+        std::vector<int2> sorted;
+        if ((st = build_attn_items(g, sorted))) return st;
         n_items = (int)sorted.size();
-        if ((size_t)n_items > (size_t)N + N / 128 + 1)
-            return fail(JNX_ERR_INVALID_ARG, "backbone: sample lengths exceed n_tokens");
         if (n_items && cudaMemcpyAsync(w.attn_items, sorted.data(), sorted.size() * sizeof(int2),
                                        cudaMemcpyHostToDevice, s) != cudaSuccess)
             return cuda_status("backbone: attention items");
@@ -231,8 +240,16 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
     // K = 2048 (2B-class O projection) it costs ~0.2 ms more.
     const bool fold_ffn = H * hd >= 4096;  // pre-FFN norm, after the O projection
     const bool fold_attn = F >= 4096;      // pre-attention norm, after the down projection
+    auto save = [&](int l) -> jnx_status {
+        if (!saved) return JNX_OK;
+        return cudaMemcpyAsync(saved + (size_t)l * N * d, w.x, (size_t)N * d * sizeof(float),
+                               cudaMemcpyDeviceToDevice, s) == cudaSuccess
+                   ? JNX_OK
+                   : cuda_status("backbone: saving a residual");
+    };
     for (int l = 0; l < bb->n_layers; ++l) {
         const jnx_layer& L = bb->layers[l];
+        if ((st = save(l))) return st;
         // attention sub-block.  A folded RMSNorm: the residual GEMM before it
         // (or, for the first block, rms_prep) writes y = bf16(x * gamma) and
         // the row's sums of x^2; the GEMM after it reads y and scales each
@@ -284,7 +301,7 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
             TraceScope ts(JNX_K_ATTN, attn_flops, s);
             if ((st = attention_launch(w.qkv, qkvw, N, H, Hkv, hd, g->cu_seqlens, g->n_samples,
                                        g->max_seqlen, w.attn_items, n_items, w.att, H * hd,
-                                       w.status, s)))
+                                       nullptr, w.status, s)))
                 return st;
         }
         p = GemmParams{};
@@ -351,10 +368,37 @@ extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_gro
             if ((st = gemm_launch(w.u, F, L.w_down, F, p, s))) return st;
         }
     }
+    if ((st = save(bb->n_layers))) return st;
     TraceScope ts(JNX_K_POOL, Nd * 4.0 + (hidden ? Nd * 2.0 : 0.0) +
                                   (pooled ? (double)g->n_samples * d * 4.0 : 0.0), s);
     return final_pool_launch(w.x, bb->final_norm, bb->eps, g->cu_seqlens, g->n_samples, d, pooled,
                              hidden, s);
+}
+
+extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_group* g,
+                                           const uint16_t* vision, int64_t n_vision_rows,
+                                           const int32_t* text_ids, int64_t n_text, float* pooled,
+                                           uint16_t* hidden, void* workspace, size_t ws_bytes,
+                                           void* stream) {
+    clear_error();
+    return backbone_forward(bb, g, vision, n_vision_rows, text_ids, n_text, pooled, hidden,
+                            nullptr, workspace, ws_bytes, stream);
+}
+
+extern "C" size_t jnx_backbone_saved_bytes(const jnx_backbone* bb, int32_t n_tokens) {
+    if (!bb || n_tokens < 0 || bb->n_layers < 0) return 0;
+    return (size_t)(bb->n_layers + 1) * (size_t)n_tokens * (size_t)bb->d_model * sizeof(float);
+}
+
+extern "C" jnx_status jnx_backbone_forward_train(const jnx_backbone* bb, const jnx_group* g,
+                                                 const uint16_t* vision, int64_t n_vision_rows,
+                                                 const int32_t* text_ids, int64_t n_text,
+                                                 float* pooled, uint16_t* hidden, float* saved,
+                                                 void* workspace, size_t ws_bytes, void* stream) {
+    clear_error();
+    if (!saved) return fail(JNX_ERR_INVALID_ARG, "backbone: null saved-activation buffer");
+    return backbone_forward(bb, g, vision, n_vision_rows, text_ids, n_text, pooled, hidden, saved,
+                            workspace, ws_bytes, stream);
 }
 
 // ---------------------------------------------------------------------------
@@ -424,6 +468,7 @@ HeadsWs carve_heads(const jnx_head* heads, const jnx_group* g, void* base) {
         w.sc.P = take(N * hd.nq * 4);
         w.sc.dS = take(N * hd.nq * 4);
         w.sc.dQs = take(S * hd.ld_h * 4);
+        w.sc.dkv_bf = reinterpret_cast<uint16_t*>(take(N * 2 * hd.ldkv * 2));
     }
     w.bytes = off;
     return w;
@@ -662,6 +707,82 @@ extern "C" jnx_status jnx_heads_backward_accumulate(const jnx_head* heads, int32
                           true);
 }
 
+// dloss_t/d(final normed row) of every token row, after the heads backward
+// (which leaves dz of the MLP heads and dk, dv of the query heads in the
+// workspace): an MLP sample's rows each get (dz W1) / L; a query-head row
+// gets dk W_k + dv W_v.
+static jnx_status heads_feature_grad(const jnx_head* heads, const jnx_group* g, float* d_hidden,
+                                     void* workspace, cudaStream_t s) {
+    if (g->n_slots > kSegMaxSlots)
+        return fail(JNX_ERR_UNSUPPORTED, "heads feature gradient: at most %d tenants", kSegMaxSlots);
+    HeadsWs w = carve_heads(heads, g, workspace);
+    const int d = heads[g->h_slot_tenant[0]].d_in, N = g->n_tokens;
+    static thread_local MlpFeatTable mt;
+    mt = MlpFeatTable{};
+    bool any_mlp = false, any_x = false;
+    for (int i = 0; i < g->n_slots; ++i) {
+        const jnx_head& h = heads[g->h_slot_tenant[i]];
+        if (h.kind == JNX_HEAD_MLP) {
+            mt.w1[i] = h.w1;
+            mt.hid[i] = h.d_hidden;
+            any_mlp = true;
+        } else {
+            any_x = true;
+        }
+    }
+    jnx_status st;
+    TraceScope ts(JNX_K_HEADS_BWD, 0.0, s);
+    if (any_mlp && (st = mlp_dfeat_launch(w.sc.dh, w.sc.ld_h, g->cu_seqlens, g->sample_slot,
+                                          g->n_samples, mt, d, d_hidden, s)))
+        return st;
+    if (!any_x) return JNX_OK;
+    const int ld = w.sc.ldkv;
+    if ((st = to_bf16_launch(w.sc.dk, ld, N, ld, w.sc.dkv_bf, 2 * ld, s)) ||
+        (st = to_bf16_launch(w.sc.dv, ld, N, ld, w.sc.dkv_bf + ld, 2 * ld, s)))
+        return st;
+    // one launch per distinct query width; other slots are skipped
+    std::vector<int> widths;
+    for (int i = 0; i < g->n_slots; ++i) {
+        const jnx_head& h = heads[g->h_slot_tenant[i]];
+        if (h.kind == JNX_HEAD_XATTN &&
+            std::find(widths.begin(), widths.end(), h.q_dim) == widths.end())
+            widths.push_back(h.q_dim);
+    }
+    static thread_local SegUpParts sp;
+    for (int dq : widths) {
+        sp = SegUpParts{};
+        sp.n_parts = 2;
+        sp.t[0] = w.sc.dkv_bf;
+        sp.t[1] = w.sc.dkv_bf + ld;
+        sp.ldt[0] = sp.ldt[1] = 2 * ld;
+        sp.k[0] = sp.k[1] = dq;
+        for (int i = 0; i < g->n_slots; ++i) {
+            const jnx_head& h = heads[g->h_slot_tenant[i]];
+            if (h.kind == JNX_HEAD_XATTN && h.q_dim == dq) {
+                sp.w[0][i] = h.wk;
+                sp.w[1][i] = h.wv;
+            }
+        }
+        if ((st = seg_up_launch(g, sp, d, d_hidden, d, false, s))) return st;
+    }
+    return JNX_OK;
+}
+
+extern "C" jnx_status jnx_heads_backward_input(const jnx_head* heads, int32_t n_tenants,
+                                               const jnx_group* g, const float* pooled,
+                                               const uint16_t* hidden, const float* targets,
+                                               const jnx_head_grads* grads, float* d_hidden,
+                                               void* workspace, size_t ws_bytes, void* stream) {
+    clear_error();
+    (void)targets;
+    if (!d_hidden && g && g->n_tokens > 0)
+        return fail(JNX_ERR_INVALID_ARG, "heads backward: null feature-gradient buffer");
+    jnx_status st = heads_backward(heads, n_tenants, g, pooled, hidden, grads, workspace,
+                                   ws_bytes, stream, false);
+    if (st || g->n_slots == 0) return st;
+    return heads_feature_grad(heads, g, d_hidden, workspace, static_cast<cudaStream_t>(stream));
+}
+
 // ---------------------------------------------------------------------------
 // status and helpers
 
@@ -786,8 +907,8 @@ extern "C" jnx_status jnx_op_attention(const uint16_t* qkv, int32_t n_tokens, in
     const int ldq = (n_heads + 2 * n_kv_heads) * head_dim;
     TraceScope ts(JNX_K_ATTN, 0.0, static_cast<cudaStream_t>(stream));
     return attention_launch(qkv, ldq, n_tokens, n_heads, n_kv_heads, head_dim, cu_seqlens,
-                            n_samples, max_seqlen, nullptr, 0, out, n_heads * head_dim, status,
-                            static_cast<cudaStream_t>(stream));
+                            n_samples, max_seqlen, nullptr, 0, out, n_heads * head_dim, nullptr,
+                            status, static_cast<cudaStream_t>(stream));
 }
 
 extern "C" jnx_status jnx_op_final_pool(const float* x, const uint16_t* gamma, float eps,

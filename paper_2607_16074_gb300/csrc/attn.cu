@@ -247,7 +247,7 @@ template <int HD, int BN>
 __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
     k_attn_ws(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tkv,
               const int* __restrict__ cu, AttnItems items, int H, int Hkv, float scale_log2,
-              uint16_t* __restrict__ out, int ldo, int* status) {
+              uint16_t* __restrict__ out, int ldo, float* __restrict__ lse, int* status) {
     using C = AttnWsCfg<HD, BN>;
     constexpr int BM = C::BM;
     constexpr int NCH = HD / 64;  // 64-column (128-byte) chunks of a Q/K/V row
@@ -506,6 +506,8 @@ __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
             // epilogue: O / l -> bf16 once the item's last PV is done
             if (!(ok = wait_pv(gs))) break;
             const float inv = 1.0f / l;
+            if (lse != nullptr && qt * BM + quarter * 32 + lane < L)
+                lse[(size_t)(start + qt * BM + quarter * 32 + lane) * H + h] = m + log2f(l);
             // 32 columns at a time through this warp's staging slot, so each
             // store instruction writes 8 rows x 64 contiguous bytes; O is
             // released (o_free) once its last columns are in registers
@@ -561,7 +563,7 @@ __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
 template <int HD, int BN>
 static jnx_status launch_attn_ws(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv,
                                  const int* cu, int S, int max_seqlen, const int2* items,
-                                 int n_items, uint16_t* out, int ldo, int* status,
+                                 int n_items, uint16_t* out, int ldo, float* lse, int* status,
                                  cudaStream_t s) {
     using C = AttnWsCfg<HD, BN>;
     static bool attr = false;
@@ -591,14 +593,14 @@ static jnx_status launch_attn_ws(const uint16_t* qkv, int ldq, int n_tokens, int
     const int grid = std::min((n_work + C::NST - 1) / C::NST, num_sms());
     const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)HD));
     k_attn_ws<HD, BN><<<grid, C::THREADS, C::SMEM, s>>>(tq, tkv, cu, it, H, Hkv, scale_log2, out, ldo,
-                                                 status);
+                                                 lse, status);
     cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
 }
 
 jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv, int hd,
                             const int* cu, int S, int max_seqlen, const int2* items, int n_items,
-                            uint16_t* out, int ldo, int* status, cudaStream_t s) {
+                            uint16_t* out, int ldo, float* lse, int* status, cudaStream_t s) {
     if (S == 0 || max_seqlen == 0) return JNX_OK;
     if (Hkv <= 0 || H % Hkv) return fail(JNX_ERR_UNSUPPORTED, "attention: H %% Hkv != 0");
     if ((long long)S * ((max_seqlen + attn_ws::BM - 1) / attn_ws::BM) > 0x7FFFFFFFLL || H > 65535)
@@ -606,13 +608,13 @@ jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, i
     switch (hd) {
         case 64:
             return launch_attn_ws<64, 64>(qkv, ldq, n_tokens, H, Hkv, cu, S, max_seqlen, items,
-                                          n_items, out, ldo, status, s);
+                                          n_items, out, ldo, lse, status, s);
         case 128:
             return launch_attn_ws<128, 64>(qkv, ldq, n_tokens, H, Hkv, cu, S, max_seqlen, items,
-                                           n_items, out, ldo, status, s);
+                                           n_items, out, ldo, lse, status, s);
         case 256:
             return launch_attn_ws<256, 64>(qkv, ldq, n_tokens, H, Hkv, cu, S, max_seqlen, items,
-                                           n_items, out, ldo, status, s);
+                                           n_items, out, ldo, lse, status, s);
         default:
             return fail(JNX_ERR_UNSUPPORTED, "attention: head_dim %d not in {64,128,256}", hd);
     }

@@ -88,6 +88,21 @@ __device__ __forceinline__ float act_fn(float g, int act) {
     return 0.5f * g * (1.0f + tanhf(c * (g + 0.044715f * g * g * g)));
 }
 
+// act(g) and its derivative: SiLU' = s (1 + g (1 - s)) with s = sigmoid(g);
+// for 0.5 g (1 + t), t = tanh(c (g + a g^3)): 0.5 (1 + t) + 0.5 g (1 - t^2) c (1 + 3 a g^2).
+__device__ __forceinline__ void act_grad(float g, int act, float& a, float& da) {
+    if (act == JNX_GLU_SWIGLU) {
+        const float s = 1.0f / (1.0f + expf(-g));
+        a = g * s;
+        da = s * (1.0f + g * (1.0f - s));
+    } else {
+        const float c = 0.7978845608028654f;
+        const float t = tanhf(c * (g + 0.044715f * g * g * g));
+        a = 0.5f * g * (1.0f + t);
+        da = 0.5f * (1.0f + t) + 0.5f * g * (1.0f - t * t) * c * (1.0f + 3.0f * 0.044715f * g * g);
+    }
+}
+
 // Epilogue staging: each epilogue warp turns its 32 rows x 64 bytes from
 // one-row-per-thread (the TMEM layout) into row-contiguous global accesses
 // through a 2 KB shared-memory slot.  Writer: thread `lane` puts row `lane`.
@@ -271,6 +286,49 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
             }
             stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
                            n0 / 2 + c * 32, pol);
+        }
+    } else if constexpr (EPI == EPI_GLU_BWD) {
+        // accumulator: dm for F columns [n0, n0 + 256); F column f has its
+        // gate at packed column 256 (f / 128) + f % 128 and its up 128 later.
+        // This thread reads its own row's g and u of a chunk before the warp
+        // stores that chunk's dg and du, so out may be aux.
+        const bf16_t* gu = p.aux + (size_t)(valid ? my_row : 0) * p.ldaux;
+#pragma unroll 1
+        for (int c = 0; c < 8; ++c) {
+            const int f = n0 + c * 32;
+            const int gcol = (f / 128) * 256 + (f % 128);
+            uint32_t r[32];
+            tmem_ld32(tbase + c * 32, r);
+            uint4 gv[4], uv[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                gv[u] = valid ? ld_global_u4_hint(gu + gcol + 8 * u, pol) : make_uint4(0, 0, 0, 0);
+                uv[u] = valid ? ld_global_u4_hint(gu + gcol + 128 + 8 * u, pol) : make_uint4(0, 0, 0, 0);
+            }
+            tmem_ld_wait();
+            uint4 vg[4], vu[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const uint32_t gw[4] = {gv[u].x, gv[u].y, gv[u].z, gv[u].w};
+                const uint32_t uw[4] = {uv[u].x, uv[u].y, uv[u].z, uv[u].w};
+                float og[8], ou[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float g = bf2f((gw[e / 2] >> (16 * (e & 1))) & 0xFFFF);
+                    const float up = bf2f((uw[e / 2] >> (16 * (e & 1))) & 0xFFFF);
+                    const float dm = __uint_as_float(r[8 * u + e]);
+                    float a, da;
+                    act_grad(g, p.act, a, da);
+                    og[e] = dm * up * da;
+                    ou[e] = dm * a;
+                }
+                vg[u] = pack8_bf16(og);
+                vu[u] = pack8_bf16(ou);
+            }
+            stg_store_bf16(stg, lane, vg, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
+                           gcol, pol);
+            stg_store_bf16(stg, lane, vu, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
+                           gcol + 128, pol);
         }
     } else if constexpr (EPI == EPI_ROPE) {
         const int hc = p.hd / 64;  // 32-column chunks in half a head
@@ -676,6 +734,7 @@ jnx_status gemm_launch(const uint16_t* A, int lda, const uint16_t* B, int ldb, G
         case EPI_RESID: e = launch_epi<EPI_RESID, false>(ta, tb, none, p, grid, s); break;
         case EPI_GLU: e = launch_epi<EPI_GLU, false>(ta, tb, none, p, grid, s); break;
         case EPI_ROPE: e = launch_epi<EPI_ROPE, false>(ta, tb, none, p, grid, s); break;
+        case EPI_GLU_BWD: e = launch_epi<EPI_GLU_BWD, false>(ta, tb, none, p, grid, s); break;
         default: return fail(JNX_ERR_INVALID_ARG, "gemm: unknown epilogue %d", p.epi);
     }
     if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));

@@ -49,6 +49,7 @@ struct HeadScratch {
     int ldkv;
     float *P, *dS;                 // [nq * n_tokens], key-major per sample
     float* dQs;                    // [n_samples, ld_h]
+    uint16_t* dkv_bf;              // feature gradient: bf16 [dk | dv] rows [n_tokens, 2 ldkv]
 };
 
 jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const HeadScratch& ws,

@@ -4,11 +4,13 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <vector>
+
 #include "jnx_host.h"
 
 namespace jnx {
 
-enum { EPI_BF16 = 0, EPI_F32 = 1, EPI_RESID = 2, EPI_GLU = 3, EPI_ROPE = 4 };
+enum { EPI_BF16 = 0, EPI_F32 = 1, EPI_RESID = 2, EPI_GLU = 3, EPI_ROPE = 4, EPI_GLU_BWD = 5 };
 
 struct GemmParams {
     int M, N, K;
@@ -38,7 +40,20 @@ struct GemmParams {
     const float* ss_in;
     int ss_parts, ss_cols;
     float ss_eps;
+    // EPI_GLU_BWD: the GEMM computes dm = dloss/d(act(g) * u) for F columns;
+    // aux [M, ldaux] holds the gate / up pre-activations g, u in EPI_GLU's
+    // packed order (128-column blocks alternating gate and up), and out
+    // (same layout; it may be aux itself) receives dg = dm u act'(g) and
+    // du = dm act(g) in bf16.
+    const uint16_t* aux;
+    int ldaux;
 };
+
+constexpr int kMaxRopePos = 1 << 16;  // longest sample a workspace reserves RoPE rows for
+
+// Argument checks shared by the backbone's entry points.
+jnx_status check_backbone(const jnx_backbone* bb);
+jnx_status check_group(const jnx_group* g);
 
 // LoRA: rank and the number of tenant segments one launch describes.
 constexpr int kLoraRank = 16;
@@ -119,8 +134,14 @@ jnx_status rope_table_launch(float2* tab, int max_pos, int hd, float theta, cuda
 // Varlen attention confined to each sample, bidirectional.  `items`
 // (device, optional) lists the (sample, 128-query tile) work items in the
 // order the persistent kernel should take them; null enumerates them.
+// With lse set, also writes each query row's log2-sum-exp of its scaled
+// scores, lse[row * H + h] = log2(sum_j 2^(s_j log2(e) / sqrt(hd))), which
+// the backward uses to recompute the probabilities.
+// Attention work items (sample, 128-row tile) of a group, most expensive first.
+jnx_status build_attn_items(const jnx_group* g, std::vector<int2>& sorted);
+
 jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv, int hd,
                             const int* cu, int S, int max_seqlen, const int2* items, int n_items,
-                            uint16_t* out, int ldo, int* status, cudaStream_t s);
+                            uint16_t* out, int ldo, float* lse, int* status, cudaStream_t s);
 
 }  // namespace jnx

@@ -121,6 +121,17 @@ class jnx_adamw(C.Structure):
                 ("eps", C.c_float), ("weight_decay", C.c_float)]
 
 
+class jnx_layer_t(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in ("w_qkv_t", "w_o_t", "w_gu_t", "w_down_t")]
+
+
+LORA_GRADS = ("a_q", "b_q", "a_k", "b_k", "a_v", "b_v", "a_o", "b_o")
+
+
+class jnx_lora_grads(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in LORA_GRADS]
+
+
 _LIB: Optional[C.CDLL] = None
 
 EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_workspace_bytes",
@@ -129,7 +140,12 @@ EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_work
            "jnx_op_rmsnorm", "jnx_op_gemm_workspace_bytes", "jnx_op_gemm", "jnx_op_attention",
            "jnx_op_final_pool", "jnx_trace_enable", "jnx_trace_disable", "jnx_trace_count",
            "jnx_trace_read", "jnx_op_gemm_rope_noalloc", "jnx_sched_poll",
-           "jnx_heads_backward_accumulate", "jnx_heads_adamw")
+           "jnx_heads_backward_accumulate", "jnx_heads_adamw", "jnx_backbone_saved_bytes",
+           "jnx_backbone_forward_train", "jnx_heads_backward_input", "jnx_transpose",
+           "jnx_backbone_backward_workspace_bytes", "jnx_backbone_backward_lora",
+           "jnx_op_attention_lse", "jnx_op_attention_backward_prep",
+           "jnx_op_attention_backward_workspace_bytes", "jnx_op_attention_backward",
+           "jnx_op_rms_backward", "jnx_op_gemm_glu_backward")
 
 
 def lib() -> C.CDLL:
@@ -165,6 +181,23 @@ def lib() -> C.CDLL:
         "jnx_heads_adamw": (i32, [C.POINTER(jnx_head), C.POINTER(jnx_head_grads),
                                   C.POINTER(jnx_head_opt), i32, C.POINTER(jnx_group),
                                   C.POINTER(jnx_adamw), vp]),
+        "jnx_backbone_saved_bytes": (sz, [C.POINTER(jnx_backbone), i32]),
+        "jnx_backbone_forward_train": (i32, [C.POINTER(jnx_backbone), C.POINTER(jnx_group), vp,
+                                             i64, vp, i64, vp, vp, vp, vp, sz, vp]),
+        "jnx_heads_backward_input": (i32, [C.POINTER(jnx_head), i32, C.POINTER(jnx_group), vp,
+                                           vp, vp, C.POINTER(jnx_head_grads), vp, vp, sz, vp]),
+        "jnx_transpose": (i32, [vp, i32, i32, i32, vp, vp]),
+        "jnx_backbone_backward_workspace_bytes": (sz, [C.POINTER(jnx_backbone), i32]),
+        "jnx_backbone_backward_lora": (i32, [C.POINTER(jnx_backbone), C.POINTER(jnx_layer_t),
+                                             C.POINTER(jnx_group), vp, vp,
+                                             C.POINTER(jnx_lora_grads), i32, vp, sz, vp]),
+        "jnx_op_attention_lse": (i32, [vp, i32, i32, i32, i32, vp, i32, i32, vp, vp, vp, vp]),
+        "jnx_op_attention_backward_prep": (i32, [vp, vp, i32, i32, i32, vp, vp, vp]),
+        "jnx_op_attention_backward_workspace_bytes": (sz, [i32, i32, i32]),
+        "jnx_op_attention_backward": (i32, [vp, vp, vp, vp, i32, i32, i32, i32, vp, vp, i32, i32,
+                                            vp, f32, vp, vp, sz, vp, vp]),
+        "jnx_op_rms_backward": (i32, [vp, vp, f32, vp, vp, i32, i32, vp, vp, vp]),
+        "jnx_op_gemm_glu_backward": (i32, [vp, vp, i32, i32, i32, vp, i32, vp]),
         "jnx_check_status": (i32, [vp, vp]),
         "jnx_pack_gate_up": (i32, [vp, vp, i32, i32, vp, vp]),
         "jnx_op_pack": (i32, [C.POINTER(jnx_group), vp, i64, vp, i64, vp, i32, i32, vp, vp, vp]),
@@ -307,8 +340,9 @@ def jnx_sched_poll(schemas: Sequence[dict], requests: Sequence[dict], arrival: S
 KERNEL_NAMES = {1: "pack", 2: "rmsnorm", 3: "gemm_qkv_rope", 4: "attention", 5: "gemm_o_resid",
                 6: "gemm_gate_up_glu", 7: "gemm_down_resid", 8: "final_norm_pool",
                 9: "rope_table", 10: "heads_fwd", 11: "heads_bwd", 12: "gemm", 13: "lora_down",
-                14: "heads_adamw"}
-TENSOR_KERNELS = (3, 4, 5, 6, 7, 12, 13)
+                14: "heads_adamw", 15: "gemm_bwd", 16: "attention_bwd", 17: "norm_bwd",
+                18: "lora_bwd"}
+TENSOR_KERNELS = (3, 4, 5, 6, 7, 12, 13, 15, 16, 18)
 
 
 def jnx_trace_enable(capacity: int) -> None:

@@ -93,6 +93,60 @@ class DeviceBackbone:
             text_ids.data_ptr(), text_ids.shape[0], _ptr(pooled), _ptr(hidden),
             ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)))
 
+    # ---- trainable adapters ------------------------------------------------
+    def saved_bytes(self, n_tokens: int) -> int:
+        return J.lib().jnx_backbone_saved_bytes(C.byref(self.struct), n_tokens)
+
+    def backward_workspace_bytes(self, n_tokens: int) -> int:
+        return J.lib().jnx_backbone_backward_workspace_bytes(C.byref(self.struct), n_tokens)
+
+    def prepare_backward(self, stream=None) -> None:
+        """Transposed copies of the frozen weights (built once on the device)
+        and zeroed fp32 adapter-gradient buffers, one set per layer."""
+        cfg, L, s = self.cfg, J.lib(), _stream(stream)
+        n = max(1, cfg.n_layers)
+        self.layers_t = (J.jnx_layer_t * n)()
+        self.lgarr = (J.jnx_lora_grads * n)()
+        self.keep_t: List[torch.Tensor] = []
+        self.lora_grads: List[Dict[str, torch.Tensor]] = []
+        per = len(self.keep) // max(1, cfg.n_layers)
+        for i in range(cfg.n_layers):
+            ent = self.keep[i * per:(i + 1) * per]
+            w_qkv, w_o, w_gu, w_down = ent[1], ent[2], ent[4], ent[5]
+            outs = []
+            for w in (w_qkv, w_o, w_gu, w_down):
+                t = torch.empty((w.shape[1], w.shape[0]), dtype=torch.bfloat16, device=w.device)
+                J.check(L.jnx_transpose(w.data_ptr(), 1, w.shape[0], w.shape[1], t.data_ptr(), s))
+                outs.append(t)
+            self.keep_t += outs
+            self.layers_t[i] = J.jnx_layer_t(*[t.data_ptr() for t in outs])
+            lw = dict(zip(["attn_norm", "w_qkv", "w_o", "ffn_norm", "w_gu", "w_down",
+                           "lora_a_q", "lora_b_q", "lora_a_k", "lora_b_k", "lora_a_v",
+                           "lora_b_v", "lora_a_o", "lora_b_o"], ent))
+            g = {}
+            for name in J.LORA_GRADS:
+                src = lw.get("lora_" + name)
+                g[name] = (torch.zeros(src.shape, dtype=torch.float32, device=src.device)
+                           if src is not None else None)
+            self.lora_grads.append(g)
+            self.lgarr[i] = J.jnx_lora_grads(*[_ptr(g[k]) for k in J.LORA_GRADS])
+
+    def forward_train(self, group: DeviceGroup, vision, text_ids, pooled, hidden, saved, ws,
+                      stream=None) -> None:
+        J.check(J.lib().jnx_backbone_forward_train(
+            C.byref(self.struct), group.ref, vision.data_ptr(), vision.shape[0],
+            text_ids.data_ptr(), text_ids.shape[0], _ptr(pooled), _ptr(hidden),
+            saved.data_ptr(), ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)))
+
+    def backward_lora(self, group: DeviceGroup, saved, d_hidden, ws, accumulate: bool = False,
+                      stream=None) -> None:
+        """Every group tenant's adapter gradients into self.lora_grads (its
+        slice only), from dloss/d(final normed rows)."""
+        J.check(J.lib().jnx_backbone_backward_lora(
+            C.byref(self.struct), self.layers_t, group.ref, saved.data_ptr(), d_hidden.data_ptr(),
+            self.lgarr, 1 if accumulate else 0, ws.data_ptr(), ws.numel() * ws.element_size(),
+            _stream(stream)))
+
 
 class DeviceHeads:
     """One head slot per tenant (bf16 parameters) and fp32 gradient slots."""
@@ -146,6 +200,14 @@ class DeviceHeads:
         fn = J.lib().jnx_heads_backward_accumulate if accumulate else J.lib().jnx_heads_backward
         J.check(fn(self.arr, self.n, group.ref, _ptr(pooled), _ptr(hidden), targets.data_ptr(),
                    self.garr, ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)))
+
+    def backward_input(self, group: DeviceGroup, pooled, hidden, targets, d_hidden, ws,
+                       stream=None) -> None:
+        """backward, and also dloss/d(final normed row) of every token row."""
+        J.check(J.lib().jnx_heads_backward_input(
+            self.arr, self.n, group.ref, _ptr(pooled), _ptr(hidden), targets.data_ptr(),
+            self.garr, d_hidden.data_ptr(), ws.data_ptr(), ws.numel() * ws.element_size(),
+            _stream(stream)))
 
     def init_optimizer(self) -> None:
         """Tenant-private AdamW state: an fp32 master copy of every head
@@ -218,6 +280,38 @@ class GroupedStep:
                         self.pooled if self.need_pooled else None, self.hidden, self.ws_bb, stream)
         self.heads.forward(self.group, self.pooled, self.hidden, None, preds, None, self.ws_h,
                            stream)
+
+
+class LoraTrainStep(GroupedStep):
+    """One grouped training step of the tenants' adapters and heads through
+    the C ABI: the shared forward keeping each block's residual input, every
+    group tenant's head forward, loss and backward (with the gradient at its
+    features), then the adapter backward through the frozen backbone.  Head
+    gradients land in heads.grads, adapter gradients in backbone.lora_grads,
+    each tenant's in its own slice."""
+
+    def __init__(self, backbone: DeviceBackbone, heads: DeviceHeads, group: DeviceGroup,
+                 device="cuda"):
+        super().__init__(backbone, heads, group, device)
+        if not hasattr(backbone, "layers_t"):
+            backbone.prepare_backward()
+        N, d = group.plan.n_tokens, backbone.cfg.d
+        self.saved = torch.empty(max(backbone.saved_bytes(N) // 4, 1), dtype=torch.float32,
+                                 device=device)
+        self.d_hidden = torch.zeros((max(N, 1), d), dtype=torch.float32, device=device)
+        self.ws_bwd = torch.zeros(max(backbone.backward_workspace_bytes(N), 256),
+                                  dtype=torch.uint8, device=device)
+
+    def run(self, vision, text_ids, targets, preds, stream=None, accumulate: bool = False) -> None:
+        self.bb.forward_train(self.group, vision, text_ids,
+                              self.pooled if self.need_pooled else None, self.hidden, self.saved,
+                              self.ws_bb, stream)
+        self.heads.forward(self.group, self.pooled, self.hidden, targets, preds, self.loss,
+                           self.ws_h, stream)
+        self.heads.backward_input(self.group, self.pooled, self.hidden, targets, self.d_hidden,
+                                  self.ws_h, stream)
+        self.bb.backward_lora(self.group, self.saved, self.d_hidden, self.ws_bwd,
+                              accumulate=accumulate, stream=stream)
 
 
 class StepPipeline:

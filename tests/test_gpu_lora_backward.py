@@ -1,0 +1,330 @@
+"""Per-tenant LoRA backward through the frozen backbone, through the C ABI:
+each backward stage against the oracle's pieces, then every tenant's
+adapter gradients of a whole grouped training step against the oracle's
+chain rule (oracle/backward.py), the grouped == isolated invariant (bit for
+bit), slot isolation and gradient accumulation."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import backward as B
+from oracle import model as M
+from paper_2607_16074_gb300 import jnx as J
+from paper_2607_16074_gb300 import runtime as R
+from tests.gpu_helpers import f64, randn_bf16, stream
+from tests.helpers import deep_tol, oracle_requests, rel_err, rel_err_bf16_out
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2607_16074_gb300 import build as B_
+    B_.build()
+    J.lib()
+
+
+def _rel_l2(got, ref):
+    got, ref = np.asarray(got, np.float64), np.asarray(ref, np.float64)
+    return float(np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-300))
+
+
+# ---------------------------------------------------------------------------
+# stages
+# ---------------------------------------------------------------------------
+
+def test_transpose_exact():
+    src = randn_bf16((3, 70, 45), 1)
+    dst = torch.empty((3, 45, 70), dtype=torch.bfloat16, device="cuda")
+    J.check(J.lib().jnx_transpose(src.data_ptr(), 3, 70, 45, dst.data_ptr(), stream()))
+    torch.cuda.synchronize()
+    assert torch.equal(dst, src.transpose(1, 2))
+
+
+def test_rms_backward_vs_oracle():
+    M_, d = 37, 512
+    g = torch.Generator().manual_seed(3)
+    x = torch.randn(M_, d, generator=g).cuda()
+    dn = torch.randn(M_, d, generator=g).cuda()
+    dres = torch.randn(M_, d, generator=g).cuda()
+    gamma = randn_bf16((d,), 4, std=0.1) + 1.0
+    dx = torch.empty_like(x)
+    dxb = torch.empty((M_, d), dtype=torch.bfloat16, device="cuda")
+    J.check(J.lib().jnx_op_rms_backward(x.data_ptr(), gamma.data_ptr(), 1e-6, dn.data_ptr(),
+                                        dres.data_ptr(), M_, d, dx.data_ptr(), dxb.data_ptr(),
+                                        stream()))
+    torch.cuda.synchronize()
+    ref = f64(dres) + B.rmsnorm_backward(f64(x), f64(gamma), 1e-6, f64(dn))
+    # fp32 arithmetic over d = 512 terms
+    assert rel_err(f64(dx), ref) < 1e-5
+    assert torch.equal(dxb, dx.to(torch.bfloat16))
+
+
+@pytest.mark.parametrize("act", [0, 1])
+def test_glu_backward_gemm_vs_oracle(act):
+    M_, F, K = 300, 512, 256
+    A = randn_bf16((M_, K), 5)
+    W = randn_bf16((F, K), 6, std=0.05)
+    gu = randn_bf16((M_, 2 * F), 7)
+    g_ref = f64(gu)
+    J.check(J.lib().jnx_op_gemm_glu_backward(A.data_ptr(), W.data_ptr(), M_, F, K, gu.data_ptr(),
+                                             act, stream()))
+    torch.cuda.synchronize()
+    dm = f64(A) @ f64(W).T
+    # packed order: F column f has its gate at 256 (f // 128) + f % 128, its up 128 later
+    f = np.arange(F)
+    gcol = (f // 128) * 256 + f % 128
+    g, u = g_ref[:, gcol], g_ref[:, gcol + 128]
+    a = M.silu(g) if act == 0 else M.gelu_tanh(g)
+    da = M.silu_grad(g) if act == 0 else B.gelu_tanh_grad(g)
+    got = f64(gu)
+    # fp32 products of bf16 operands, stored in bf16
+    assert rel_err_bf16_out(got[:, gcol], dm * u * da) < 1e-3
+    assert rel_err_bf16_out(got[:, gcol + 128], dm * a) < 1e-3
+
+
+def _attn_case(lengths, H, Hkv, hd, seed, qk_std=1.0):
+    cu = np.concatenate([[0], np.cumsum(lengths)]).astype(np.int32)
+    N = int(cu[-1])
+    ldq = (H + 2 * Hkv) * hd
+    qkv = randn_bf16((N, ldq), seed, std=qk_std)
+    dO32 = torch.randn(N, H * hd, generator=torch.Generator().manual_seed(seed + 1)).cuda()
+    pos = np.concatenate([np.arange(L) for L in lengths]).astype(np.int32)
+    return cu, N, ldq, qkv, dO32, pos
+
+
+def _attn_backward_device(cu, N, H, Hkv, hd, qkv, dO32, pos, theta=1e4):
+    L = J.lib()
+    S = len(cu) - 1
+    maxL = int(np.max(np.diff(cu)))
+    cu_d = torch.from_numpy(cu).cuda()
+    pos_d = torch.from_numpy(pos).cuda()
+    att = torch.empty((N, H * hd), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((N, H), dtype=torch.float32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    J.check(L.jnx_op_attention_lse(qkv.data_ptr(), N, H, Hkv, hd, cu_d.data_ptr(), S, maxL,
+                                   att.data_ptr(), lse.data_ptr(), status.data_ptr(), stream()))
+    dO = torch.empty((N, H * hd), dtype=torch.bfloat16, device="cuda")
+    D = torch.empty((N, H), dtype=torch.float32, device="cuda")
+    J.check(L.jnx_op_attention_backward_prep(dO32.data_ptr(), att.data_ptr(), N, H, hd,
+                                             dO.data_ptr(), D.data_ptr(), stream()))
+    ws = torch.zeros(L.jnx_op_attention_backward_workspace_bytes(N, maxL, hd), dtype=torch.uint8,
+                     device="cuda")
+    dqkv = torch.full((N, (H + 2 * Hkv) * hd), float("nan"), dtype=torch.bfloat16, device="cuda")
+    J.check(L.jnx_op_attention_backward(qkv.data_ptr(), dO.data_ptr(), lse.data_ptr(),
+                                        D.data_ptr(), N, H, Hkv, hd, cu_d.data_ptr(),
+                                        cu.ctypes.data, S, maxL, pos_d.data_ptr(), theta,
+                                        dqkv.data_ptr(), ws.data_ptr(), ws.numel(),
+                                        status.data_ptr(), stream()))
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    return att, lse, dO, D, dqkv
+
+
+@pytest.mark.parametrize("H,Hkv,hd", [(4, 2, 64), (4, 4, 128), (8, 1, 256)])
+def test_attention_backward_vs_oracle(H, Hkv, hd):
+    # ragged samples: one token, a tail of one past a 64-tile, two 128-tiles
+    # plus a tail, several key tiles
+    lengths = [1, 65, 130, 7, 200]
+    cu, N, ldq, qkv, dO32, pos = _attn_case(lengths, H, Hkv, hd, seed=11 + hd)
+    att, lse, dO, D, dqkv = _attn_backward_device(cu, N, H, Hkv, hd, qkv, dO32, pos)
+    Q = f64(qkv)
+    got = f64(dqkv)
+    ref = np.zeros_like(got)
+    grp = H // Hkv
+    for i, L in enumerate(lengths):
+        r = slice(cu[i], cu[i + 1])
+        q = Q[r, :H * hd].reshape(L, H, hd)
+        k = Q[r, H * hd:(H + Hkv) * hd].reshape(L, Hkv, hd)
+        v = Q[r, (H + Hkv) * hd:].reshape(L, Hkv, hd)
+        do = f64(dO)[r].reshape(L, H, hd)
+        # lse: log2 of the softmax denominator of the scaled scores
+        for h in range(H):
+            s = q[:, h] @ k[:, h // grp].T / math.sqrt(hd)
+            m = s.max(axis=1)
+            ref_lse = (m + np.log(np.exp(s - m[:, None]).sum(axis=1))) / math.log(2.0)
+            assert np.max(np.abs(f64(lse)[r, h] - ref_lse)) < 2e-3
+        # D = rowsum(dO * O) with the device's bf16 dO and O
+        Dref = (do * f64(att)[r].reshape(L, H, hd)).sum(axis=2)
+        assert np.max(np.abs(f64(D)[r] - Dref)) <= 1e-4 * max(1.0, np.abs(Dref).max())
+        dq, dk, dv = B.attention_backward(q, k, v, do)
+        ref[r] = np.concatenate([B.rope_backward(dq, np.arange(L), 1e4).reshape(L, -1),
+                                 B.rope_backward(dk, np.arange(L), 1e4).reshape(L, -1),
+                                 dv.reshape(L, -1)], axis=1)
+    # each gradient block's relative L2 error over the batch (a one-token
+    # sample's dq and dk are exactly zero: one key makes dS vanish).  The
+    # result is stored in bf16 (rounding the exact reference alone gives
+    # ~1.7e-3 here) and P and dS are rounded to bf16 before the accumulating
+    # products (the same order again, averaged over the keys): 2^-8 bounds
+    # both with margin, where a wrong term or index is off by O(1).
+    for c0, c1, name in ((0, H * hd, "dq"), (H * hd, (H + Hkv) * hd, "dk"),
+                         ((H + Hkv) * hd, ldq, "dv")):
+        e = _rel_l2(got[:, c0:c1], ref[:, c0:c1])
+        assert e < 2.0 ** -8, (name, e)
+    r0 = slice(cu[0], cu[1])
+    scale = float(np.sqrt(np.mean(ref[:, :(H + Hkv) * hd] ** 2)))
+    assert np.max(np.abs(got[r0, :(H + Hkv) * hd])) < 1e-3 * scale
+
+
+def test_attention_backward_grouped_equals_isolated():
+    # one sample's gradients do not depend on the other samples in the batch
+    H, Hkv, hd = 4, 2, 128
+    lengths = [90, 150, 33]
+    cu, N, ldq, qkv, dO32, pos = _attn_case(lengths, H, Hkv, hd, seed=5)
+    *_, dqkv = _attn_backward_device(cu, N, H, Hkv, hd, qkv, dO32, pos)
+    r = slice(int(cu[1]), int(cu[2]))
+    cu1 = np.array([0, lengths[1]], np.int32)
+    *_, one = _attn_backward_device(cu1, lengths[1], H, Hkv, hd, qkv[r].contiguous(),
+                                    dO32[r].contiguous(), np.arange(lengths[1], dtype=np.int32))
+    assert torch.equal(one, dqkv[r])
+
+
+# ---------------------------------------------------------------------------
+# the whole training step
+# ---------------------------------------------------------------------------
+
+class TrainSetup:
+    def __init__(self, w, std=0.02, gen_device="cpu"):
+        self.w = w
+        self.bw = synth.make_backbone_weights(w, device=gen_device, std=std)
+        self.hw = synth.make_head_weights(w, device=gen_device, std=std)
+        self.inp = synth.make_inputs(w, device=gen_device)
+        c = lambda t: t.cuda()
+        self.bw_d = dict(layers=[{k: c(v) for k, v in L.items()} for L in self.bw["layers"]],
+                         final_norm=c(self.bw["final_norm"]), text_table=c(self.bw["text_table"]))
+        self.hw_d = [{k: c(v) for k, v in h.items()} for h in self.hw]
+        self.inp_d = {k: c(v) for k, v in self.inp.items()}
+        self.bb = R.DeviceBackbone(w.backbone, self.bw_d, n_tenants=len(w.tenants))
+        self.heads = R.DeviceHeads(w.tenants, w.backbone.d, self.hw_d)
+        self.bb.prepare_backward()
+
+    def run(self, wsub=None, accumulate=False):
+        w = wsub or self.w
+        plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), len(w.tenants), 1 << 30, 1 << 30)
+        g = R.DeviceGroup(plan)
+        step = R.LoraTrainStep(self.bb, self.heads, g)
+        preds = torch.full_like(self.inp_d["targets"], float("nan"))
+        step.run(self.inp_d["vision"], self.inp_d["text_ids"], self.inp_d["targets"], preds,
+                 accumulate=accumulate)
+        for ws in (step.ws_bb, step.ws_h, step.ws_bwd):
+            R.check_status(ws)
+        torch.cuda.synchronize()
+        return plan, step
+
+    def oracle(self, tenants=None):
+        np_bw = M.widen_tree(synth.to_numpy_tree(self.bw))
+        return B.lora_step(self.w, np_bw, M.widen_tree(synth.to_numpy_tree(self.hw)),
+                           synth.to_numpy_tree(self.inp), tenants=tenants)
+
+
+def _small_lora_workload(glu, n_layers=2):
+    bb = synth.Backbone(n_layers=n_layers, d=256, n_heads=8, n_kv_heads=4, head_dim=64,
+                        d_ff=512, vision_tokens=32, vocab=300, glu=glu, lora_rank=16,
+                        qk_std=0.05)
+    tenants = [synth.Tenant(synth.HEAD_MLP, chunk=4, action_dim=7, d_hidden=64, max_images=2),
+               synth.Tenant(synth.HEAD_XATTN, chunk=2, action_dim=7, n_queries=4, q_dim=256,
+                            max_images=2),
+               synth.Tenant(synth.HEAD_MLP, chunk=2, action_dim=3, d_hidden=32, max_images=2)]
+    per = [[synth.Sample(1, 5), synth.Sample(2, 31), synth.Sample(0, 3)],
+           [synth.Sample(1, 100), synth.Sample(0, 1)],
+           [synth.Sample(2, 77), synth.Sample(1, 0), synth.Sample(0, 140), synth.Sample(1, 9)]]
+    return synth.custom_workload(bb, tenants, per, req_batch=2, seed=31)
+
+
+def _check_vs_oracle(s, plan, step, ref, tol):
+    """Relative L2 error of every group tenant's feature gradient and of each
+    of its adapter gradients in every layer.  Adapter gradients pass through
+    every block's forward and the backward of the blocks above, each with a
+    few bf16 roundings (operands of every product, P and dS): measured
+    3e-3 - 7e-3 at one block, up to 1.1e-2 at two and 1.5e-2 at four, growing
+    like sqrt(depth); the bound is the forward's 2e-2 per block scaled by
+    sqrt(n_layers) (deep_tol), where a wrong term is off by O(1)."""
+    cu = plan.cu_seqlens
+    seg = plan.seg_offsets
+    for gi, t in enumerate(plan.slot_tenant.tolist()):
+        if t not in ref:
+            continue
+        r = ref[t]
+        # the feature gradient every row gets from its tenant's head
+        dh = np.concatenate(r["d_hidden"])
+        rows = np.concatenate([np.arange(cu[i], cu[i + 1]) for i in range(seg[gi], seg[gi + 1])])
+        e = _rel_l2(f64(step.d_hidden[torch.from_numpy(rows).long().cuda()]), dh)
+        assert e < tol, ("d_hidden", t, e)
+        for l, gl in enumerate(r["lora"]):
+            for name, gref in gl.items():
+                got = f64(s.bb.lora_grads[l][name][t])
+                e = _rel_l2(got, gref)
+                assert e < tol, ("lora", t, l, name, e)
+
+
+@pytest.mark.parametrize("glu", [0, 1])
+def test_lora_train_step_small_vs_oracle(glu):
+    w = _small_lora_workload(glu)
+    s = TrainSetup(w, std=0.05)
+    plan, step = s.run()
+    ref = s.oracle()
+    _check_vs_oracle(s, plan, step, ref, deep_tol(w.backbone.n_layers))
+
+
+def test_lora_train_step_mqa_hd256_vs_oracle():
+    """The 2B-class block shapes (d 2048, 8 query heads on one K/V head of
+    256, GeGLU 16384) one block deep, on two small tenants of the skewed
+    workload."""
+    w = synth.make_workload("zipf2b", n_layers=1)
+    counts = {t: sum(len(r.samples) for r in w.requests if r.tenant == t)
+              for t in range(len(w.tenants))}
+    pick = sorted(counts, key=lambda t: (counts[t], t))[:2]
+    s = TrainSetup(w.subset(pick), gen_device="cuda")
+    plan, step = s.run()
+    ref = s.oracle(tenants=pick)
+    _check_vs_oracle(s, plan, step, ref, deep_tol(1))
+
+
+def test_lora_grads_grouped_equal_isolated_and_other_slots_untouched():
+    w = _small_lora_workload(0)
+    s = TrainSetup(w, std=0.05)
+    s.run()
+    full = [{k: (v.clone() if v is not None else None) for k, v in g.items()}
+            for g in s.bb.lora_grads]
+    for g in s.bb.lora_grads:
+        for v in g.values():
+            v.fill_(7.0)
+    s.run(w.subset([1]))
+    for l, g in enumerate(s.bb.lora_grads):
+        for k, v in g.items():
+            # tenant 1 alone == tenant 1 inside the group, bit for bit
+            assert torch.equal(v[1], full[l][k][1]), (l, k)
+            # other tenants' slices are not written
+            assert torch.all(v[0] == 7.0) and torch.all(v[2] == 7.0), (l, k)
+
+
+def test_lora_grads_accumulate():
+    w = _small_lora_workload(1, n_layers=1)
+    s = TrainSetup(w, std=0.05)
+    s.run()
+    one = [{k: v.clone() for k, v in g.items()} for g in s.bb.lora_grads]
+    s.run(accumulate=True)
+    for l, g in enumerate(s.bb.lora_grads):
+        for k, v in g.items():
+            assert torch.equal(v, 2 * one[l][k]), (l, k)
+
+
+def test_lora_backward_rejects_a_backbone_without_adapters():
+    import dataclasses
+    w = _small_lora_workload(0, n_layers=1)
+    s = TrainSetup(w, std=0.05)
+    w0 = dataclasses.replace(w, backbone=dataclasses.replace(w.backbone, lora_rank=0))
+    bb0 = R.DeviceBackbone(w0.backbone, s.bw_d, n_tenants=len(w.tenants))
+    bb0.layers_t = s.bb.layers_t
+    bb0.lgarr = s.bb.lgarr
+    plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), len(w.tenants), 1 << 30, 1 << 30)
+    g = R.DeviceGroup(plan)
+    N = plan.n_tokens
+    saved = torch.zeros(max(bb0.saved_bytes(N) // 4, 1), device="cuda")
+    dh = torch.zeros((N, w.backbone.d), device="cuda")
+    ws = torch.zeros(max(bb0.backward_workspace_bytes(N), 256), dtype=torch.uint8, device="cuda")
+    with pytest.raises(J.JnxError):
+        bb0.backward_lora(g, saved, dh, ws)
