@@ -206,6 +206,145 @@ class ClockSampler:
 # our arm
 # ---------------------------------------------------------------------------
 
+def kernel_breakdown(J, kinds, ms, work):
+    """Per traced kernel kind: launches, total ms, share of the traced time
+    and its rate (TFLOP/s for tensor-core kinds, GB/s otherwise)."""
+    per_kernel = {}
+    tot_ms = float(ms.sum())
+    for k in sorted(set(kinds.tolist())):
+        m = kinds == k
+        name = J.KERNEL_NAMES.get(k, str(k))
+        kms = float(ms[m].sum())
+        wk = float(work[m].sum())
+        rate = wk / (kms / 1e3) if kms > 0 else 0.0
+        per_kernel[name] = dict(launches=int(m.sum()), ms=round(kms, 3),
+                                share=round(kms / tot_ms, 4) if tot_ms else None,
+                                **({"tflops": round(rate / 1e12, 1)} if k in J.TENSOR_KERNELS
+                                   else {"gbs": round(rate / 1e9, 1)}))
+    return per_kernel
+
+
+def run_train(args):
+    """One grouped training step of every tenant's LoRA adapters and head on
+    the skewed 64-tenant 2B-class workload (rank-16 adapters on Q/K/V/O):
+    the shared forward keeping each block's residual input, the tenants'
+    heads, losses and feature gradients, then the adapter backward through
+    the frozen backbone (each block recomputed from its saved input).
+    Tokens/s of the whole step, device-resident inputs, with the per-kernel
+    breakdown and the grouped vs per-tenant isolated speedup."""
+    import torch
+
+    import synth
+    from paper_2607_16074_gb300 import build as B
+    from paper_2607_16074_gb300 import jnx as J
+    from paper_2607_16074_gb300 import runtime as R
+
+    B.build()
+    J.lib()
+    dev = torch.device("cuda", 0)
+    w = make_bench_workload(args)
+    if not w.backbone.lora_rank:
+        raise SystemExit(f"--train-lora needs a workload with adapters (zipf2b), not {w.name}")
+    bw = synth.make_backbone_weights(w, device=dev)
+    hw = synth.make_head_weights(w, device=dev)
+    inp = synth.make_inputs(w, device=dev)
+    reqs = oracle_requests(w)
+    plan = J.jnx_group_plan(w.schemas(), reqs, len(w.tenants), w.max_samples, w.max_tokens)
+    backbone = R.DeviceBackbone(w.backbone, bw, n_tenants=len(w.tenants))
+    heads = R.DeviceHeads(w.tenants, w.backbone.d, hw, device=dev)
+    backbone.prepare_backward()
+    step = R.LoraTrainStep(backbone, heads, R.DeviceGroup(plan, device=dev), device=dev)
+    preds = torch.zeros_like(inp["targets"])
+    stream = torch.cuda.current_stream()
+    run = lambda st: st.run(inp["vision"], inp["text_ids"], inp["targets"], preds)
+    for _ in range(max(args.warmup, 3)):
+        run(step)
+    for ws in (step.ws_bb, step.ws_h, step.ws_bwd):
+        R.check_status(ws)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(0)
+    clocks.start()
+    cap = 8192 * max(1, args.steps)
+    J.jnx_trace_enable(cap)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        run(step)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    launches = J.jnx_trace_count()
+    kinds, ms, work = J.jnx_trace_read(cap)
+    J.jnx_trace_disable()
+    clk = clocks.stop()
+    t_ms = e0.elapsed_time(e1)
+    tokens = plan.n_tokens
+    per_kernel = kernel_breakdown(J, kinds, ms, work)
+    peaks = load_peaks()
+    # the dominant kernel kind of the step and its roofline
+    shares = {k: float(ms[kinds == k].sum()) for k in set(kinds.tolist())}
+    top = max(shares, key=shares.get)
+    m = kinds == top
+    top_rate = float(work[m].sum()) / (float(ms[m].sum()) / 1e3) / 1e12
+    roofline = dict(kernel=J.KERNEL_NAMES.get(top, str(top)), bound="tensor",
+                    achieved=round(top_rate, 1), peak=peaks["bf16_sustained"], unit="TFLOP/s",
+                    frac=round(top_rate / peaks["bf16_sustained"], 4),
+                    share_of_step=round(shares[top] / float(ms.sum()), 4),
+                    launches_per_step=int(m.sum()) // max(args.steps, 1),
+                    peak_note=f"bf16_tflops_sustained of {peaks['source']} peaks")
+    # the backward's four input-gradient GEMMs, told apart by their FLOPs per launch
+    gb = kinds == 15
+    by_shape = {}
+    for fl in sorted(set(work[gb].tolist()), reverse=True):
+        mm = gb & (work == fl)
+        kms = float(ms[mm].sum())
+        by_shape["%.3g TFLOP" % (fl / 1e12)] = dict(
+            launches=int(mm.sum()), ms=round(kms, 3),
+            tflops=round(fl * int(mm.sum()) / (kms / 1e3) / 1e12, 1))
+    roofline["gemm_bwd_by_shape"] = by_shape
+    bwd_mask = np.isin(kinds, (15, 16, 18))
+    bwd_tf = float(work[bwd_mask].sum()) / (float(ms[bwd_mask].sum()) / 1e3) / 1e12
+    step_flops = float(work[np.isin(kinds, J.TENSOR_KERNELS)].sum()) / args.steps
+    speed = None
+    if not args.no_per_tenant:
+        del step
+        torch.cuda.empty_cache()
+        iso = []
+        for t in range(len(w.tenants)):
+            sub = w.subset([t])
+            p = J.jnx_group_plan(sub.schemas(), oracle_requests(sub), len(w.tenants),
+                                 w.max_samples, w.max_tokens)
+            if p.n_samples:
+                iso.append(R.LoraTrainStep(backbone, heads, R.DeviceGroup(p, device=dev),
+                                           device=dev))
+        for st in iso:
+            run(st)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for st in iso:
+            run(st)
+        b.record(stream)
+        torch.cuda.synchronize()
+        t_iso = a.elapsed_time(b)
+        speed = dict(per_tenant_ms=round(t_iso, 3), grouped_ms=round(t_ms / args.steps, 3),
+                     speedup=round(t_iso / (t_ms / args.steps), 4),
+                     per_tenant_tokens_per_s=round(tokens / (t_iso / 1e3), 1))
+    return dict(metric="lora_train_tokens_per_s", value=round(tokens * args.steps / (t_ms / 1e3), 1),
+                unit="tokens/s", steps=args.steps, ms_per_step=round(t_ms / args.steps, 3),
+                higher_is_better=True, dtype="bf16", data="synthetic",
+                config=dict(workload=workload_desc(w), tokens=tokens, samples=plan.n_samples,
+                            tenants=len(w.tenants), lora_rank=w.backbone.lora_rank,
+                            step="forward (saving block inputs) + heads + feature gradient + "
+                                 "adapter backward (blocks recomputed)"),
+                clocks=clk, gpu_launches=int(launches), roofline=roofline,
+                backward_tensor=dict(kernels="gemm_bwd + attention_bwd + lora_bwd",
+                                     achieved=round(bwd_tf, 1), unit="TFLOP/s",
+                                     frac=round(bwd_tf / peaks["bf16_sustained"], 4)),
+                step_tensor=dict(achieved=round(step_flops / (t_ms / args.steps / 1e3) / 1e12, 1),
+                                 unit="TFLOP/s"),
+                per_tenant=speed, kernels=per_kernel)
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
 
@@ -325,18 +464,7 @@ def run_ours(args, rank, world, local_rank):
     gemm_mask = np.isin(kinds, (3, 5, 6, 7))
     g_flops, g_ms = float(work[gemm_mask].sum()), float(ms[gemm_mask].sum())
     g_tf = g_flops / (g_ms / 1e3) / 1e12 if g_ms > 0 else 0.0
-    per_kernel = {}
-    tot_ms = float(ms.sum())
-    for k in sorted(set(kinds.tolist())):
-        m = kinds == k
-        name = J.KERNEL_NAMES.get(k, str(k))
-        kms = float(ms[m].sum())
-        wk = float(work[m].sum())
-        rate = wk / (kms / 1e3) if kms > 0 else 0.0
-        per_kernel[name] = dict(launches=int(m.sum()), ms=round(kms, 3),
-                                share=round(kms / tot_ms, 4) if tot_ms else None,
-                                **({"tflops": round(rate / 1e12, 1)} if k in J.TENSOR_KERNELS
-                                   else {"gbs": round(rate / 1e9, 1)}))
+    per_kernel = kernel_breakdown(J, kinds, ms, work)
     step_flops = float(work[np.isin(kinds, J.TENSOR_KERNELS + (10, 11))].sum()) / args.steps
     step_tf = step_flops / (t_ms / args.steps / 1e3) / 1e12
     # the dominant kernel: the gate/up projection GEMM (largest share of the step)
@@ -657,7 +785,12 @@ def main():
     ap.add_argument("--layers", type=int, default=0, help="override the number of blocks")
     ap.add_argument("--grid", default=None, choices=["e4"],
                     help="grouped vs serial inference on the tenants x local batch grid")
+    ap.add_argument("--train-lora", action="store_true",
+                    help="time the per-tenant LoRA training step (use with --workload zipf2b)")
     args = ap.parse_args()
+    if args.train_lora:
+        print(json.dumps(run_train(args)), flush=True)
+        return
     if args.grid:
         print(json.dumps(run_grid(args)), flush=True)
         return
