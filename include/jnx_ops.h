@@ -21,6 +21,9 @@ extern "C" {
                            out bf16 [M, ldo] columns j < N/2 = act(C_gate) * C_up */
 #define JNX_EPI_ROPE 4  /* out bf16 [M, ldo] = C with rotate-half RoPE at
                            position pos[row] on columns < rope_cols */
+#define JNX_EPI_GLU_SAVE 6 /* W as for JNX_EPI_GLU; out bf16 [M, ldo], N columns in W's
+                              packed order: u act'(g) in each gate column, act(g) in each
+                              up column (the GLU backward's multipliers) */
 
 /* The canonical packing step (§4.3: the VLAFeature is where the tenants'
  * samples are concatenated): x[t, :] = fp32 of vision[gather_src[t]] or of
@@ -117,9 +120,11 @@ jnx_status jnx_op_rms_backward(const float* x, const uint16_t* gamma, float eps,
 
 /* The feed-forward backward's first GEMM with the GLU backward fused:
  * dm[M, F] = A[M, K] W[F, K]^T is the gradient at act(g) * u; gu [M, 2F]
- * bf16 holds g | u in JNX_EPI_GLU's packed order (128-column blocks
- * alternating gate and up) on entry and dg = dm u act'(g) | du = dm act(g)
- * in the same order on return.  F % 256 == 0, K % 64 == 0. */
+ * bf16 holds on entry what JNX_EPI_GLU_SAVE wrote (u act'(g) in the gate
+ * columns, act(g) in the up columns of the packed order, 128-column blocks
+ * alternating gate and up) and on return dg = dm u act'(g) in the gate
+ * columns, du = dm act(g) in the up columns.  F % 256 == 0, K % 64 == 0.
+ * act is not read (the multipliers already hold the activation). */
 jnx_status jnx_op_gemm_glu_backward(const uint16_t* A, const uint16_t* W, int32_t M, int32_t F,
                                     int32_t K, uint16_t* gu, int32_t act, void* stream);
 

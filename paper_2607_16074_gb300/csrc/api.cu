@@ -854,8 +854,11 @@ extern "C" jnx_status jnx_op_gemm(const uint16_t* A, const uint16_t* W, int32_t 
                                   void* workspace, size_t ws_bytes, void* stream) {
     clear_error();
     if (!A || !W || !out || M < 0) return fail(JNX_ERR_INVALID_ARG, "gemm: null argument");
-    if (epilogue < EPI_BF16 || epilogue > EPI_ROPE)
+    if ((epilogue < EPI_BF16 || epilogue > EPI_ROPE) && epilogue != EPI_GLU_SAVE)
         return fail(JNX_ERR_INVALID_ARG, "gemm: unknown epilogue %d", epilogue);
+    if ((epilogue == EPI_GLU || epilogue == EPI_GLU_SAVE) && act != JNX_GLU_SWIGLU &&
+        act != JNX_GLU_GEGLU_TANH)
+        return fail(JNX_ERR_INVALID_ARG, "gemm: unknown activation %d", act);
     {
         // the epilogues write (and the residual one reads) 16-byte vectors
         const int esz = (epilogue == EPI_F32 || epilogue == EPI_RESID) ? 4 : 2;

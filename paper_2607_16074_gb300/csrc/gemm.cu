@@ -287,48 +287,101 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
             stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
                            n0 / 2 + c * 32, pol);
         }
-    } else if constexpr (EPI == EPI_GLU_BWD) {
-        // accumulator: dm for F columns [n0, n0 + 256); F column f has its
-        // gate at packed column 256 (f / 128) + f % 128 and its up 128 later.
-        // This thread reads its own row's g and u of a chunk before the warp
-        // stores that chunk's dg and du, so out may be aux.
-        const bf16_t* gu = p.aux + (size_t)(valid ? my_row : 0) * p.ldaux;
+    } else if constexpr (EPI == EPI_GLU_SAVE) {
+        const float rs = row_norm_scale(p, my_row, valid);
 #pragma unroll 1
-        for (int c = 0; c < 8; ++c) {
-            const int f = n0 + c * 32;
-            const int gcol = (f / 128) * 256 + (f % 128);
-            uint32_t r[32];
-            tmem_ld32(tbase + c * 32, r);
-            uint4 gv[4], uv[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                gv[u] = valid ? ld_global_u4_hint(gu + gcol + 8 * u, pol) : make_uint4(0, 0, 0, 0);
-                uv[u] = valid ? ld_global_u4_hint(gu + gcol + 128 + 8 * u, pol) : make_uint4(0, 0, 0, 0);
-            }
+        for (int c = 0; c < 4; ++c) {
+            uint32_t g[32], u[32];
+            tmem_ld32(tbase + c * 32, g);
+            tmem_ld32(tbase + (c + 4) * 32, u);
             tmem_ld_wait();
             uint4 vg[4], vu[4];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const uint32_t gw[4] = {gv[u].x, gv[u].y, gv[u].z, gv[u].w};
-                const uint32_t uw[4] = {uv[u].x, uv[u].y, uv[u].z, uv[u].w};
+            for (int q = 0; q < 4; ++q) {
                 float og[8], ou[8];
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
-                    const float g = bf2f((gw[e / 2] >> (16 * (e & 1))) & 0xFFFF);
-                    const float up = bf2f((uw[e / 2] >> (16 * (e & 1))) & 0xFFFF);
-                    const float dm = __uint_as_float(r[8 * u + e]);
                     float a, da;
-                    act_grad(g, p.act, a, da);
-                    og[e] = dm * up * da;
-                    ou[e] = dm * a;
+                    act_grad(rs * __uint_as_float(g[8 * q + e]), p.act, a, da);
+                    og[e] = rs * __uint_as_float(u[8 * q + e]) * da;
+                    ou[e] = a;
                 }
-                vg[u] = pack8_bf16(og);
-                vu[u] = pack8_bf16(ou);
+                vg[q] = pack8_bf16(og);
+                vu[q] = pack8_bf16(ou);
             }
             stg_store_bf16(stg, lane, vg, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
-                           gcol, pol);
+                           n0 + c * 32, pol);
             stg_store_bf16(stg, lane, vu, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
-                           gcol + 128, pol);
+                           n0 + 128 + c * 32, pol);
+        }
+    } else if constexpr (EPI == EPI_GLU_BWD) {
+        // accumulator: dm for F columns [n0, n0 + 256); F column f has its
+        // gate slot at packed column 256 (f / 128) + f % 128 and its up slot
+        // 128 later.  As EPI_RESID: 16 columns per pass, dm staged through
+        // shared memory so lane handles 4 columns of rows 8 i + lane / 4 (its
+        // loads and stores cover 8 rows x 32 contiguous bytes per
+        // instruction), the multipliers of pass + RD - 1 in flight.  Each
+        // element is read before the same lane writes it, so out may be aux.
+        constexpr int RD = 4;
+        auto pcol = [&](int pass) {
+            const int f = n0 + pass * 16 + (lane & 3) * 4;
+            return (f / 128) * 256 + (f % 128);
+        };
+        uint2 mg[RD][4], mu[RD][4];
+        auto load_m = [&](int pass, uint2 (&g)[4], uint2 (&u)[4]) {
+            const int pc = pcol(pass);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int row = row_base + 8 * i + (lane >> 2);
+                g[i] = u[i] = make_uint2(0u, 0u);
+                if (row < row_end) {
+                    const bf16_t* src = p.aux + (size_t)row * p.ldaux + pc;
+                    g[i] = ld_global_u2_hint(src, pol);
+                    u[i] = ld_global_u2_hint(src + 128, pol);
+                }
+            }
+        };
+#pragma unroll
+        for (int q = 0; q < RD - 1; ++q) load_m(q, mg[q], mu[q]);
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            uint32_t r[32];
+            tmem_ld32(tbase + c * 32, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int pass = 2 * c + h;
+                if (pass + RD - 1 < 16) load_m(pass + RD - 1, mg[(pass + RD - 1) % RD],
+                                                mu[(pass + RD - 1) % RD]);
+                uint4 v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    v[u] = make_uint4(r[16 * h + 4 * u], r[16 * h + 4 * u + 1],
+                                      r[16 * h + 4 * u + 2], r[16 * h + 4 * u + 3]);
+                stg_put(stg, lane, v);
+                __syncwarp();
+                const int pc = pcol(pass);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const uint4 wv = stg_get(stg, lane, i);
+                    const int row = row_base + 8 * i + (lane >> 2);
+                    const float dm[4] = {__uint_as_float(wv.x), __uint_as_float(wv.y),
+                                         __uint_as_float(wv.z), __uint_as_float(wv.w)};
+                    const uint2 gm = mg[pass % RD][i], um = mu[pass % RD][i];
+                    const uint2 og = make_uint2(
+                        pack_bf2(dm[0] * bf2f(gm.x & 0xFFFF), dm[1] * bf2f(gm.x >> 16)),
+                        pack_bf2(dm[2] * bf2f(gm.y & 0xFFFF), dm[3] * bf2f(gm.y >> 16)));
+                    const uint2 ou = make_uint2(
+                        pack_bf2(dm[0] * bf2f(um.x & 0xFFFF), dm[1] * bf2f(um.x >> 16)),
+                        pack_bf2(dm[2] * bf2f(um.y & 0xFFFF), dm[3] * bf2f(um.y >> 16)));
+                    if (row < row_end) {
+                        bf16_t* dst = static_cast<bf16_t*>(p.out) + (size_t)row * p.ldo + pc;
+                        st_global_u2_hint(dst, og, pol);
+                        st_global_u2_hint(dst + 128, ou, pol);
+                    }
+                }
+                __syncwarp();
+            }
         }
     } else if constexpr (EPI == EPI_ROPE) {
         const int hc = p.hd / 64;  // 32-column chunks in half a head
@@ -735,6 +788,7 @@ jnx_status gemm_launch(const uint16_t* A, int lda, const uint16_t* B, int ldb, G
         case EPI_GLU: e = launch_epi<EPI_GLU, false>(ta, tb, none, p, grid, s); break;
         case EPI_ROPE: e = launch_epi<EPI_ROPE, false>(ta, tb, none, p, grid, s); break;
         case EPI_GLU_BWD: e = launch_epi<EPI_GLU_BWD, false>(ta, tb, none, p, grid, s); break;
+        case EPI_GLU_SAVE: e = launch_epi<EPI_GLU_SAVE, false>(ta, tb, none, p, grid, s); break;
         default: return fail(JNX_ERR_INVALID_ARG, "gemm: unknown epilogue %d", p.epi);
     }
     if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));

@@ -149,6 +149,22 @@ __device__ __forceinline__ void st_global_u4_hint(void* p, uint4 v, uint64_t pol
                  : "memory");
 }
 
+// 8-byte global load / store under an L2 cache policy (the load does not
+// allocate in L1).
+__device__ __forceinline__ uint2 ld_global_u2_hint(const void* p, uint64_t pol) {
+    uint2 v;
+    asm volatile("ld.global.L1::no_allocate.L2::cache_hint.v2.b32 {%0,%1}, [%2], %3;"
+                 : "=r"(v.x), "=r"(v.y)
+                 : "l"((uint64_t)p), "l"(pol));
+    return v;
+}
+
+__device__ __forceinline__ void st_global_u2_hint(void* p, uint2 v, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.v2.b32 [%0], {%1,%2}, %3;" ::"l"((uint64_t)p),
+                 "r"(v.x), "r"(v.y), "l"(pol)
+                 : "memory");
+}
+
 // 2D tiled load: box at (x = inner element index, y = row) into smem,
 // completion signalled on `bar` as transaction bytes.
 __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, int32_t x,

@@ -10,7 +10,8 @@
 
 namespace jnx {
 
-enum { EPI_BF16 = 0, EPI_F32 = 1, EPI_RESID = 2, EPI_GLU = 3, EPI_ROPE = 4, EPI_GLU_BWD = 5 };
+enum { EPI_BF16 = 0, EPI_F32 = 1, EPI_RESID = 2, EPI_GLU = 3, EPI_ROPE = 4, EPI_GLU_BWD = 5,
+       EPI_GLU_SAVE = 6 };
 
 struct GemmParams {
     int M, N, K;
@@ -40,11 +41,14 @@ struct GemmParams {
     const float* ss_in;
     int ss_parts, ss_cols;
     float ss_eps;
+    // EPI_GLU_SAVE: over the gate/up weights (as EPI_GLU), writes bf16
+    // u act'(g) in the gate columns and act(g) in the up columns of out
+    // [M, N] (EPI_GLU's packed order: 128-column blocks alternating gate and
+    // up): what the GLU backward multiplies the incoming gradient by.
     // EPI_GLU_BWD: the GEMM computes dm = dloss/d(act(g) * u) for F columns;
-    // aux [M, ldaux] holds the gate / up pre-activations g, u in EPI_GLU's
-    // packed order (128-column blocks alternating gate and up), and out
-    // (same layout; it may be aux itself) receives dg = dm u act'(g) and
-    // du = dm act(g) in bf16.
+    // aux [M, ldaux] holds what EPI_GLU_SAVE wrote, and out (same layout; it
+    // may be aux itself) receives dg = dm u act'(g) in the gate columns and
+    // du = dm act(g) in the up columns, bf16.
     const uint16_t* aux;
     int ldaux;
 };

@@ -12,9 +12,10 @@
 // Per block, with dy = dloss/d(block output) (fp32) and its bf16 copy:
 //   recompute   n1 = RMSNorm(x), t = n1 A^T, q|k|v = RoPE(n1 W_qkv^T + t B^T),
 //               O = Attn (+ its log2-sum-exp), h = x + O W_o^T (+ adapter),
-//               n2 = RMSNorm(h), g|u = n2 W_gu^T  (bf16, packed order)
-//   FFN         [dg|du] = GLU'(dy W_down)  (one GEMM, GLU backward fused in
-//               its epilogue, in place over g|u); dn2 = [dg|du] W_gu;
+//               n2 = RMSNorm(h); the gate/up GEMM's epilogue keeps the GLU
+//               backward's multipliers u act'(g) | act(g) (bf16, packed order)
+//   FFN         dm = dy W_down; dg|du = dm * multipliers (one GEMM, in place
+//               over the multipliers); dn2 = [dg|du] W_gu;
 //               dh = dy + RMSNorm'(h; dn2)
 //   O           dO = dh W_o + (dh B_o) A_o;  dB_o = dh^T t_o, dA_o = (dh B_o)^T O
 //   attention   dq, dk, dv (tcgen05 passes, inverse RoPE on dq, dk)
@@ -282,9 +283,10 @@ extern "C" jnx_status jnx_backbone_backward_lora(const jnx_backbone* bb, const j
         p.M = N;
         p.N = 2 * F;
         p.K = d;
-        p.epi = EPI_BF16;
+        p.epi = EPI_GLU_SAVE;  // u act'(g) | act(g): the GLU backward's multipliers
         p.out = w.gu;
         p.ldo = 2 * F;
+        p.act = bb->glu;
         p.status = w.status;
         {
             TraceScope ts(JNX_K_GEMM_GU, 2.0 * N * 2.0 * F * d, s);
@@ -516,8 +518,7 @@ extern "C" jnx_status jnx_op_gemm_glu_backward(const uint16_t* A, const uint16_t
                                                void* stream) {
     clear_error();
     if (M > 0 && (!A || !W || !gu)) return fail(JNX_ERR_INVALID_ARG, "glu backward: null argument");
-    if (act != JNX_GLU_SWIGLU && act != JNX_GLU_GEGLU_TANH)
-        return fail(JNX_ERR_INVALID_ARG, "glu backward: unknown activation %d", act);
+    (void)act;
     if ((reinterpret_cast<uintptr_t>(gu) & 15) || F % 256)
         return fail(JNX_ERR_INVALID_ARG, "glu backward: gu alignment or F %% 256");
     GemmParams p{};

@@ -25,6 +25,7 @@ JNX_ERR_UNSUPPORTED, JNX_ERR_WORKSPACE = -9, -10
 JNX_GLU_SWIGLU, JNX_GLU_GEGLU_TANH = 0, 1
 JNX_HEAD_MLP, JNX_HEAD_XATTN = 0, 1
 JNX_EPI_BF16, JNX_EPI_F32, JNX_EPI_RESID, JNX_EPI_GLU, JNX_EPI_ROPE = 0, 1, 2, 3, 4
+JNX_EPI_GLU_SAVE = 6
 JNX_NOALLOC_MAX_ROPE_ENTRIES = 1 << 19
 
 

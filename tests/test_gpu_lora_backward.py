@@ -64,26 +64,40 @@ def test_rms_backward_vs_oracle():
 
 
 @pytest.mark.parametrize("act", [0, 1])
-def test_glu_backward_gemm_vs_oracle(act):
-    M_, F, K = 300, 512, 256
+def test_glu_backward_gemms_vs_oracle(act):
+    # the recompute's gate/up GEMM keeps the multipliers u act'(g) | act(g),
+    # then the backward GEMM dm = A W_down^T finishes dg | du in place
+    M_, F, K, d = 300, 512, 256, 256
+    n2 = randn_bf16((M_, d), 8)
+    wg, wu = randn_bf16((F, d), 9, std=0.05), randn_bf16((F, d), 10, std=0.05)
+    w_gu = torch.empty((2 * F, d), dtype=torch.bfloat16, device="cuda")
+    J.check(J.lib().jnx_pack_gate_up(wg.data_ptr(), wu.data_ptr(), F, d, w_gu.data_ptr(),
+                                     stream()))
+    gu = torch.empty((M_, 2 * F), dtype=torch.bfloat16, device="cuda")
+    J.check(J.lib().jnx_op_gemm(n2.data_ptr(), w_gu.data_ptr(), M_, 2 * F, d,
+                                J.JNX_EPI_GLU_SAVE, gu.data_ptr(), 2 * F, None, 0, 0, 0, 0.0, act,
+                                None, 0, stream()))
+    torch.cuda.synchronize()
+    g = f64(n2) @ f64(wg).T
+    u = f64(n2) @ f64(wu).T
+    a = M.silu(g) if act == 0 else M.gelu_tanh(g)
+    da = M.silu_grad(g) if act == 0 else B.gelu_tanh_grad(g)
+    f = np.arange(F)
+    gcol = (f // 128) * 256 + f % 128   # F column f: gate slot, its up slot 128 later
+    saved = f64(gu)
+    # fp32 products of bf16 operands, stored in bf16
+    assert rel_err_bf16_out(saved[:, gcol], u * da) < 1e-3
+    assert rel_err_bf16_out(saved[:, gcol + 128], a) < 1e-3
     A = randn_bf16((M_, K), 5)
     W = randn_bf16((F, K), 6, std=0.05)
-    gu = randn_bf16((M_, 2 * F), 7)
-    g_ref = f64(gu)
     J.check(J.lib().jnx_op_gemm_glu_backward(A.data_ptr(), W.data_ptr(), M_, F, K, gu.data_ptr(),
                                              act, stream()))
     torch.cuda.synchronize()
     dm = f64(A) @ f64(W).T
-    # packed order: F column f has its gate at 256 (f // 128) + f % 128, its up 128 later
-    f = np.arange(F)
-    gcol = (f // 128) * 256 + f % 128
-    g, u = g_ref[:, gcol], g_ref[:, gcol + 128]
-    a = M.silu(g) if act == 0 else M.gelu_tanh(g)
-    da = M.silu_grad(g) if act == 0 else B.gelu_tanh_grad(g)
     got = f64(gu)
-    # fp32 products of bf16 operands, stored in bf16
-    assert rel_err_bf16_out(got[:, gcol], dm * u * da) < 1e-3
-    assert rel_err_bf16_out(got[:, gcol + 128], dm * a) < 1e-3
+    # against the multipliers as stored (the bf16 they were rounded to)
+    assert rel_err_bf16_out(got[:, gcol], dm * saved[:, gcol]) < 1e-3
+    assert rel_err_bf16_out(got[:, gcol + 128], dm * saved[:, gcol + 128]) < 1e-3
 
 
 def _attn_case(lengths, H, Hkv, hd, seed, qk_std=1.0):
