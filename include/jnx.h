@@ -453,6 +453,96 @@ jnx_status jnx_backbone_backward_lora(const jnx_backbone* bb, const jnx_layer_t*
                                       void* stream);
 
 /* ------------------------------------------------------------------------
+ * Flow-matching action expert (a DiT head) as the tenant's private module
+ *
+ * §3.1 names diffusion / flow-matching action experts among the action
+ * modules; §5.2 trains QwenGR00T's GR00T-style flow-matching head (and
+ * pi-0.5's) as the tenant-private module over the shared VLM.  The paper
+ * gives no equations; the expert here (per sample s of tenant t, context
+ * X = the sample's final normed backbone rows [L, d]):
+ *   x = tau a + (1 - tau) eps  (a: target chunk [C, D], eps: noise, tau in [0, 1]
+ *                               drawn by the caller), u = a - eps
+ *   phi = T2 SiLU(T1 s(tau) + tb1) + tb2, s(tau) = [sin(1000 tau w_i) | cos(...)],
+ *         w_i = 10000^(-i / (dm/2))
+ *   h = x W_in^T + b_in + pos + phi                                     [C, dm]
+ *   per block: q|k_a|v_a = n(h) W_qkv^T, k_c|v_c = X W_kvc^T,
+ *              h += MHA(q; [k_c; k_a], [v_c; v_a]) W_o^T   (heads of 64)
+ *              h += W_d (SiLU(n(h) W_g^T) * (n(h) W_u^T))
+ *   v = n(h) W_out^T + b_out,  n(h) = h / sqrt(mean(h^2) + 1e-6)
+ *   loss_t = mean over the tenant's samples and chunk elements of (v - u)^2
+ * Every tenant of a call has the same dimensions; parameters are stacked
+ * over tenants (bf16, tenant t's slice at t times the per-tenant size).
+ * ------------------------------------------------------------------------ */
+
+typedef struct {
+    const uint16_t* w_qkv;  /* [T, 3 dm, dm]: rows of W_q, W_k (action), W_v (action) */
+    const uint16_t* w_kvc;  /* [T, 2 dm, d]: rows of W_k, W_v over the context */
+    const uint16_t* w_o;    /* [T, dm, dm] */
+    const uint16_t* w_gu;   /* [T, 2 F, dm]: W_g, W_u in jnx_pack_gate_up's packed order */
+    const uint16_t* w_d;    /* [T, dm, F] */
+} jnx_flow_block;
+
+typedef struct {
+    int32_t d_model;     /* dm: 256, 512 or 1024 (heads of 64) */
+    int32_t d_ff;        /* F: a multiple of 128 */
+    int32_t n_blocks;
+    int32_t chunk;       /* C: 1..64 action steps */
+    int32_t action_dim;  /* D: 1..64 */
+    int32_t d_in;        /* the backbone width d (a multiple of 128) */
+    int32_t n_tenants;   /* T: tenants the stacked arrays hold */
+    const uint16_t* w_in;   /* [T, dm, D] */
+    const uint16_t* b_in;   /* [T, dm] */
+    const uint16_t* pos;    /* [T, C, dm] */
+    const uint16_t* t1;     /* [T, dm, dm] */
+    const uint16_t* tb1;    /* [T, dm] */
+    const uint16_t* t2;     /* [T, dm, dm] */
+    const uint16_t* tb2;    /* [T, dm] */
+    const uint16_t* w_out;  /* [T, D, dm] */
+    const uint16_t* b_out;  /* [T, D] */
+    const jnx_flow_block* blocks;  /* HOST array [n_blocks] */
+} jnx_flow_head;
+
+/* Gradients (device fp32), the shapes of the stacked parameters. */
+typedef struct {
+    float *w_qkv, *w_kvc, *w_o, *w_gu, *w_d;
+} jnx_flow_block_grads;
+
+typedef struct {
+    float *w_in, *b_in, *pos, *t1, *tb1, *t2, *tb2, *w_out, *b_out;
+    const jnx_flow_block_grads* blocks;  /* HOST array [n_blocks] */
+} jnx_flow_grads;
+
+/* Workspace bytes of jnx_flow_forward / jnx_flow_backward / jnx_flow_sample. */
+size_t jnx_flow_workspace_bytes(const jnx_flow_head* fh, const jnx_group* g);
+
+/* Training forward of every group tenant's expert over its samples.
+ * hidden [n_tokens, d] bf16: the backbone's final normed rows.  actions,
+ * noise [n_samples, C, D] fp32 and tau [n_samples] fp32 in the group's
+ * packed sample order; velocity [n_samples, C, D] fp32 (out);
+ * loss[tenant] fp32 for the group's tenants.  Keeps the activations the
+ * backward needs in `workspace`.  Every group tenant must be < n_tenants. */
+jnx_status jnx_flow_forward(const jnx_flow_head* fh, const jnx_group* g, const uint16_t* hidden,
+                            const float* actions, const float* noise, const float* tau,
+                            float* velocity, float* loss, void* workspace, size_t ws_bytes,
+                            void* stream);
+
+/* Gradients of each group tenant's loss with respect to its own expert
+ * parameters, written (accumulate == 0) or added into the tenant's slices
+ * of `grads`; other tenants' slices are not touched.  Must follow
+ * jnx_flow_forward with the same group, hidden rows and workspace. */
+jnx_status jnx_flow_backward(const jnx_flow_head* fh, const jnx_group* g, const uint16_t* hidden,
+                             const jnx_flow_grads* grads, int32_t accumulate, void* workspace,
+                             size_t ws_bytes, void* stream);
+
+/* Inference: from x = noise at tau = 0, n_steps Euler steps of
+ * x += v(x, tau) / n_steps up to tau = 1 (the context's K/V projections are
+ * computed once and reused by every step).  actions [n_samples, C, D] fp32
+ * (out), packed sample order. */
+jnx_status jnx_flow_sample(const jnx_flow_head* fh, const jnx_group* g, const uint16_t* hidden,
+                           const float* noise, int32_t n_steps, float* actions, void* workspace,
+                           size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
  * Status and helpers
  * ------------------------------------------------------------------------ */
 
@@ -489,6 +579,10 @@ jnx_status jnx_pack_gate_up(const uint16_t* w_gate, const uint16_t* w_up, int32_
 #define JNX_K_ATTN_BWD 16  /* attention backward; work = FLOPs of its five products */
 #define JNX_K_NORM_BWD 17  /* RMSNorm backward, attention-backward prologue; work = HBM bytes */
 #define JNX_K_LORA_BWD 18  /* adapter gradients and up-projections; work = FLOPs */
+#define JNX_K_FLOW_GEMM 19 /* flow expert: segmented projections; work = FLOPs */
+#define JNX_K_FLOW_ATTN 20 /* flow expert: attention forward / backward; work = FLOPs */
+#define JNX_K_FLOW_MISC 21 /* flow expert: time / embedding / output / norms / reductions */
+#define JNX_K_FLOW_WGRAD 22 /* flow expert: weight gradients; work = FLOPs */
 
 /* While enabled on the calling thread, each kernel launch of the library is
  * bracketed by two CUDA events on its stream (up to `capacity` launches are

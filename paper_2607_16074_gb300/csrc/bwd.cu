@@ -451,6 +451,125 @@ jnx_status seg_tn_launch(const jnx_group* g, const uint16_t* U, int ldu, const u
 }
 
 // ---------------------------------------------------------------------------
+// Weight gradient of a per-tenant linear layer: for every group tenant t,
+//   G[t][m, n] (+)= sum over the tenant's rows of U[row, m] V[row, n]
+// (U = the output gradient, V = the layer's input, both bf16).  One CTA per
+// (segment, 64 x 128 tile of G) walks all of the segment's rows in order
+// (no split over rows, so no partial sums and a fixed order); 4 warps as
+// 2 (m) x 2 (n), 32 x 64 each; rows in steps of 32, double-buffered.
+// ---------------------------------------------------------------------------
+namespace seg {
+constexpr int WG_BM = 64, WG_BN = 128, WG_ROWS = 32;
+}
+
+__global__ void __launch_bounds__(128) k_seg_wgrad(const __grid_constant__ SegRows sr,
+                                                   const uint16_t* __restrict__ U, int ldu,
+                                                   const uint16_t* __restrict__ V, int ldv,
+                                                   int m, int n, float* __restrict__ grad,
+                                                   long long gstride, int add) {
+    using namespace seg;
+    __shared__ __align__(128) uint8_t sU[2][WG_ROWS * 128];
+    __shared__ __align__(128) uint8_t sV[2][WG_ROWS * 256];
+    const int sg = blockIdx.z;
+    const int r0 = sr.r0[sg], r1 = sr.r1[sg];
+    const int m0 = blockIdx.y * WG_BM, n0 = blockIdx.x * WG_BN;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int wm = warp & 1, wn = warp >> 1;
+    const uint32_t ua = smem_u32(sU), va = smem_u32(sV);
+    const int nsteps = (r1 - r0 + WG_ROWS - 1) / WG_ROWS;
+    auto load = [&](int st, int buf) {
+        const int rb = r0 + st * WG_ROWS;
+        for (int i = tid; i < WG_ROWS * 8; i += 128) {  // U: 32 rows x 8 units (64 m)
+            const int r = i >> 3, u = i & 7;
+            const bool ok = rb + r < r1;
+            cp_async16(ua + buf * WG_ROWS * 128 + r * 128 + ((u ^ (r & 7)) << 4),
+                       U + (size_t)(ok ? rb + r : r0) * ldu + m0 + u * 8, ok);
+        }
+        for (int i = tid; i < WG_ROWS * 16; i += 128) {  // V: 32 rows x 16 units (128 n)
+            const int r = i >> 4, u = i & 15;
+            const bool ok = rb + r < r1;
+            cp_async16(va + buf * WG_ROWS * 256 + r * 256 + ((u ^ (r & 7)) << 4),
+                       V + (size_t)(ok ? rb + r : r0) * ldv + n0 + u * 8, ok);
+        }
+    };
+    float acc[2][8][4];
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j][0] = acc[i][j][1] = acc[i][j][2] = acc[i][j][3] = 0.f;
+    const int mi = lane >> 3, rr = lane & 7;
+    if (nsteps > 0) load(0, 0);
+    cp_async_commit();
+    for (int st = 0; st < nsteps; ++st) {
+        const int buf = st & 1;
+        if (st + 1 < nsteps) load(st + 1, buf ^ 1);
+        cp_async_commit();
+        cp_async_wait<1>();
+        __syncthreads();
+        const uint32_t ub = ua + buf * WG_ROWS * 128, vb = va + buf * WG_ROWS * 256;
+#pragma unroll
+        for (int ks = 0; ks < 2; ++ks) {
+            // A = U^T: transposed 8x8 blocks of U (rows = k, columns = m)
+            uint32_t a[2][4];
+#pragma unroll
+            for (int mt = 0; mt < 2; ++mt) {
+                const int r = ks * 16 + rr + 8 * (mi >> 1);
+                const int u = wm * 4 + mt * 2 + (mi & 1);
+                ldsm_x4_t(ub + r * 128 + ((u ^ (r & 7)) << 4), a[mt][0], a[mt][1], a[mt][2],
+                          a[mt][3]);
+            }
+#pragma unroll
+            for (int nb = 0; nb < 4; ++nb) {
+                const int r = ks * 16 + rr + 8 * (mi & 1), u = wn * 8 + nb * 2 + (mi >> 1);
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4_t(vb + r * 256 + ((u ^ (r & 7)) << 4), b0, b1, b2, b3);
+#pragma unroll
+                for (int mt = 0; mt < 2; ++mt) {
+                    mma_bf16(acc[mt][2 * nb], a[mt][0], a[mt][1], a[mt][2], a[mt][3], b0, b1);
+                    mma_bf16(acc[mt][2 * nb + 1], a[mt][0], a[mt][1], a[mt][2], a[mt][3], b2, b3);
+                }
+            }
+        }
+        __syncthreads();
+    }
+    const int g = lane >> 2, q = lane & 3;
+    float* gt = grad + (size_t)sr.tenant[sg] * gstride;
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int row = m0 + wm * 32 + mt * 16 + g + 8 * h;
+            float* o = gt + (size_t)row * n + n0 + wn * 64 + 2 * q;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                float2 v = make_float2(acc[mt][j][2 * h], acc[mt][j][2 * h + 1]);
+                if (add) {
+                    const float2 old = *reinterpret_cast<const float2*>(o + j * 8);
+                    v.x += old.x;
+                    v.y += old.y;
+                }
+                *reinterpret_cast<float2*>(o + j * 8) = v;
+            }
+        }
+}
+
+jnx_status seg_wgrad_launch(const SegRows& sr, const uint16_t* U, int ldu, const uint16_t* V,
+                            int ldv, int m, int n, float* grad, long long gstride, bool add,
+                            cudaStream_t s) {
+    if (m % seg::WG_BM || n % seg::WG_BN || ldu % 8 || ldv % 8)
+        return fail(JNX_ERR_UNSUPPORTED, "weight gradient: %d x %d", m, n);
+    if (sr.n <= 0) return JNX_OK;
+    if (m / seg::WG_BM > 65535 || sr.n > 65535)
+        return fail(JNX_ERR_UNSUPPORTED, "weight gradient: grid too large");
+    k_seg_wgrad<<<dim3(n / seg::WG_BN, m / seg::WG_BM, sr.n), 128, 0, s>>>(sr, U, ldu, V, ldv, m,
+                                                                          n, grad, gstride,
+                                                                          add ? 1 : 0);
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? JNX_OK
+                            : fail(JNX_ERR_CUDA, "weight gradient: %s", cudaGetErrorString(e));
+}
+
+// ---------------------------------------------------------------------------
 // MLP heads: d hidden[row] = (dz[s] W1) / L_s for every row of sample s.
 // One CTA per (sample, 256-column block); dz [n_samples, ldz] fp32.
 // ---------------------------------------------------------------------------

@@ -551,7 +551,10 @@ __global__ void __launch_bounds__(192, 1)
                     mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
                     uint8_t* sa = smem + stage * STAGE_BYTES;
                     tma_load_2d(sa, &ta, kb * BK, g.row0, &full[stage]);
-                    tma_load_2d(sa + A_BYTES, &tb, kb * BK, g.nb * BN, &full[stage]);
+                    int brow = g.nb * BN;
+                    if constexpr (LORA)
+                        if (lg.seg_b) brow += lg.seg_tenant[g.seg] * p.N;
+                    tma_load_2d(sa + A_BYTES, &tb, kb * BK, brow, &full[stage]);
                     ++issued;
                     if (++stage == STAGES) {
                         stage = 0;
@@ -560,6 +563,7 @@ __global__ void __launch_bounds__(192, 1)
                 }
                 if constexpr (LORA) {
                     if (*abort_flag) break;
+                    if (lg.n_parts == 0) continue;  // segmented weights only
                     // this tile's t rows (its part) and its tenant's B rows
                     if (!mbar_wait(&lempty[lj], lphase ^ 1)) {
                         *abort_flag = 1;
@@ -620,17 +624,21 @@ __global__ void __launch_bounds__(192, 1)
                     }
                 }
                 if constexpr (LORA) {
-                    // D += t[rows, part] . B_part[tenant][cols]^T (one K = 16 step)
-                    if (ok && !mbar_wait(&lfull[lj], lphase)) ok = false;
-                    if (ok) {
-                        *lconsumed = *lconsumed + 1;
-                        tc_fence_after();
-                        const uint32_t la = smem_u32(lsm + lj * LSTAGE);
-                        tc_mma_f16(d, sw32_desc(la), sw32_desc(la + LT_BYTES), IDESC, 1);
-                        tc_commit(&lempty[lj]);
-                        if (++lj == 2) {
-                            lj = 0;
-                            lphase ^= 1;
+                    // D += t[rows, part] . B_part[tenant][cols]^T (one K = 16 step);
+                    // none with segmented weights only (n_parts == 0)
+                    if (ok && lg.n_parts > 0) {
+                        if (!mbar_wait(&lfull[lj], lphase)) {
+                            ok = false;
+                        } else {
+                            *lconsumed = *lconsumed + 1;
+                            tc_fence_after();
+                            const uint32_t la = smem_u32(lsm + lj * LSTAGE);
+                            tc_mma_f16(d, sw32_desc(la), sw32_desc(la + LT_BYTES), IDESC, 1);
+                            tc_commit(&lempty[lj]);
+                            if (++lj == 2) {
+                                lj = 0;
+                                lphase ^= 1;
+                            }
                         }
                     }
                 }
@@ -790,6 +798,54 @@ jnx_status gemm_launch(const uint16_t* A, int lda, const uint16_t* B, int ldb, G
         case EPI_GLU_BWD: e = launch_epi<EPI_GLU_BWD, false>(ta, tb, none, p, grid, s); break;
         case EPI_GLU_SAVE: e = launch_epi<EPI_GLU_SAVE, false>(ta, tb, none, p, grid, s); break;
         default: return fail(JNX_ERR_INVALID_ARG, "gemm: unknown epilogue %d", p.epi);
+    }
+    if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));
+    return JNX_OK;
+}
+
+jnx_status gemm_launch_seg(const uint16_t* A, int lda, const uint16_t* B, int ldb, int n_tenants,
+                           GemmParams p, int n_seg, const int* seg_r0, const int* seg_r1,
+                           const int* seg_tenant, cudaStream_t s) {
+    jnx_status st = gemm_check(p.M, p.N, p.K);
+    if (st != JNX_OK) return st;
+    if (n_seg < 0 || n_seg > kLoraMaxSlots || n_tenants <= 0)
+        return fail(JNX_ERR_UNSUPPORTED, "gemm: bad segment description");
+    if (p.M == 0 || n_seg == 0) return JNX_OK;
+    static thread_local LoraGemm lg;  // staging of the kernel argument (copied at launch)
+    lg = LoraGemm{};
+    lg.n_parts = 0;
+    lg.seg_b = 1;
+    lg.n_seg = n_seg;
+    int tiles = 0;
+    for (int i = 0; i < n_seg; ++i) {
+        if (seg_r0[i] < 0 || seg_r1[i] < seg_r0[i] || seg_r1[i] > p.M || seg_tenant[i] < 0 ||
+            seg_tenant[i] >= n_tenants)
+            return fail(JNX_ERR_INVALID_ARG, "gemm: bad segment %d", i);
+        lg.seg_r0[i] = seg_r0[i];
+        lg.seg_r1[i] = seg_r1[i];
+        lg.seg_tenant[i] = seg_tenant[i];
+        lg.seg_tile0[i] = tiles;
+        tiles += (seg_r1[i] - seg_r0[i] + gemm::BM - 1) / gemm::BM;
+    }
+    lg.seg_tile0[n_seg] = tiles;
+    CUtensorMap ta, tb;
+    if (!make_tmap_bf16(&ta, A, p.M, p.K, lda, gemm::BM, gemm::BK) ||
+        !make_tmap_bf16(&tb, B, (uint64_t)n_tenants * p.N, p.K, ldb, gemm::BN, gemm::BK))
+        return fail(JNX_ERR_CUDA, "gemm: tensor map encode failed (alignment or driver)");
+    const int total = tiles * (p.N / gemm::BN);
+    if (total == 0) return JNX_OK;
+    int grid = num_sms();
+    if (total < grid) grid = total;
+    if (p.group_m <= 0) p.group_m = default_group_m(p.K);
+    cudaError_t e;
+    switch (p.epi) {
+        case EPI_BF16: e = launch_epi<EPI_BF16, true>(ta, tb, lg, p, grid, s); break;
+        case EPI_F32: e = launch_epi<EPI_F32, true>(ta, tb, lg, p, grid, s); break;
+        case EPI_RESID: e = launch_epi<EPI_RESID, true>(ta, tb, lg, p, grid, s); break;
+        case EPI_GLU: e = launch_epi<EPI_GLU, true>(ta, tb, lg, p, grid, s); break;
+        case EPI_GLU_SAVE: e = launch_epi<EPI_GLU_SAVE, true>(ta, tb, lg, p, grid, s); break;
+        case EPI_GLU_BWD: e = launch_epi<EPI_GLU_BWD, true>(ta, tb, lg, p, grid, s); break;
+        default: return fail(JNX_ERR_INVALID_ARG, "gemm: epilogue %d unsupported here", p.epi);
     }
     if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));
     return JNX_OK;

@@ -69,6 +69,11 @@ size_t seg_tn_part_floats(int n_tokens, int n_slots, int n);
 jnx_status seg_tn_launch(const jnx_group* g, const uint16_t* U, int ldu, const uint16_t* V,
                          int ldv, int n, float* part, size_t part_floats, float* grad,
                          long long gstride, bool trans, bool add, cudaStream_t s);
+// For every segment i of sr (rows [r0, r1), tenant): G[tenant][m, n] = (or
+// +=) sum over the rows of U[row, m] V[row, n]; m % 64 == 0, n % 128 == 0.
+jnx_status seg_wgrad_launch(const SegRows& sr, const uint16_t* U, int ldu, const uint16_t* V,
+                            int ldv, int m, int n, float* grad, long long gstride, bool add,
+                            cudaStream_t s);
 jnx_status mlp_dfeat_launch(const float* dz, int ldz, const int* cu, const int* sample_slot,
                             int n_samples, const MlpFeatTable& tab, int d, float* dh,
                             cudaStream_t s);

@@ -73,7 +73,9 @@ struct LoraGemm {
     CUtensorMap tt;          // t [M, ldt] bf16, box 16 x 128, 32-byte swizzle
     CUtensorMap tb[3];       // B_p viewed as [n_tenants * cols_p, 16], box 16 x 256
     int part_cols[3];        // output columns of each part (multiples of 256)
-    int n_parts, n_seg;
+    int n_parts, n_seg;      // n_parts = 0: no up-projection (gemm_launch_seg)
+    int seg_b;               // B holds every tenant's [N, K] weights stacked: a
+                             // segment's tiles read rows seg_tenant * N + ...
     int seg_r0[kLoraMaxSlots], seg_r1[kLoraMaxSlots], seg_tenant[kLoraMaxSlots];
     int seg_tile0[kLoraMaxSlots + 1];  // first 128-row tile of each segment
 };
@@ -93,6 +95,14 @@ struct LoraSpec {
 
 jnx_status gemm_launch_lora(const uint16_t* A, int lda, const uint16_t* B, int ldb, GemmParams p,
                             const LoraSpec& ls, cudaStream_t s);
+
+// Segmented GEMM with per-tenant weights: for every segment i (rows
+// [seg_r0[i], seg_r1[i]) of A and C, host arrays), C = A . B_t^T with B_t the
+// [N, K] slice of tenant seg_tenant[i] in B = [n_tenants * N, K] (row stride
+// ldb).  Output tiles never straddle two segments.  Any epilogue.
+jnx_status gemm_launch_seg(const uint16_t* A, int lda, const uint16_t* B, int ldb, int n_tenants,
+                           GemmParams p, int n_seg, const int* seg_r0, const int* seg_r1,
+                           const int* seg_tenant, cudaStream_t s);
 struct LoraSlots {
     int g0, n, sample0, pad_;
     int tenant[kLoraMaxSlots];

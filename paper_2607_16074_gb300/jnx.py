@@ -133,6 +133,31 @@ class jnx_lora_grads(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in LORA_GRADS]
 
 
+class jnx_flow_block(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in ("w_qkv", "w_kvc", "w_o", "w_gu", "w_d")]
+
+
+class jnx_flow_head(C.Structure):
+    _fields_ = [(n, C.c_int32) for n in ("d_model", "d_ff", "n_blocks", "chunk", "action_dim",
+                                         "d_in", "n_tenants")] + \
+               [(n, C.c_void_p) for n in ("w_in", "b_in", "pos", "t1", "tb1", "t2", "tb2",
+                                          "w_out", "b_out")] + \
+               [("blocks", C.POINTER(jnx_flow_block))]
+
+
+FLOW_PARAMS = ("w_in", "b_in", "pos", "t1", "tb1", "t2", "tb2", "w_out", "b_out")
+FLOW_BLOCK_PARAMS = ("w_qkv", "w_kvc", "w_o", "w_gu", "w_d")
+
+
+class jnx_flow_block_grads(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in FLOW_BLOCK_PARAMS]
+
+
+class jnx_flow_grads(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in FLOW_PARAMS] + \
+               [("blocks", C.POINTER(jnx_flow_block_grads))]
+
+
 _LIB: Optional[C.CDLL] = None
 
 EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_workspace_bytes",
@@ -146,7 +171,8 @@ EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_work
            "jnx_backbone_backward_workspace_bytes", "jnx_backbone_backward_lora",
            "jnx_op_attention_lse", "jnx_op_attention_backward_prep",
            "jnx_op_attention_backward_workspace_bytes", "jnx_op_attention_backward",
-           "jnx_op_rms_backward", "jnx_op_gemm_glu_backward")
+           "jnx_op_rms_backward", "jnx_op_gemm_glu_backward", "jnx_flow_workspace_bytes",
+           "jnx_flow_forward", "jnx_flow_backward", "jnx_flow_sample")
 
 
 def lib() -> C.CDLL:
@@ -199,6 +225,13 @@ def lib() -> C.CDLL:
                                             vp, f32, vp, vp, sz, vp, vp]),
         "jnx_op_rms_backward": (i32, [vp, vp, f32, vp, vp, i32, i32, vp, vp, vp]),
         "jnx_op_gemm_glu_backward": (i32, [vp, vp, i32, i32, i32, vp, i32, vp]),
+        "jnx_flow_workspace_bytes": (sz, [C.POINTER(jnx_flow_head), C.POINTER(jnx_group)]),
+        "jnx_flow_forward": (i32, [C.POINTER(jnx_flow_head), C.POINTER(jnx_group), vp, vp, vp,
+                                   vp, vp, vp, vp, sz, vp]),
+        "jnx_flow_backward": (i32, [C.POINTER(jnx_flow_head), C.POINTER(jnx_group), vp,
+                                    C.POINTER(jnx_flow_grads), i32, vp, sz, vp]),
+        "jnx_flow_sample": (i32, [C.POINTER(jnx_flow_head), C.POINTER(jnx_group), vp, vp, i32,
+                                  vp, vp, sz, vp]),
         "jnx_check_status": (i32, [vp, vp]),
         "jnx_pack_gate_up": (i32, [vp, vp, i32, i32, vp, vp]),
         "jnx_op_pack": (i32, [C.POINTER(jnx_group), vp, i64, vp, i64, vp, i32, i32, vp, vp, vp]),
@@ -342,8 +375,9 @@ KERNEL_NAMES = {1: "pack", 2: "rmsnorm", 3: "gemm_qkv_rope", 4: "attention", 5: 
                 6: "gemm_gate_up_glu", 7: "gemm_down_resid", 8: "final_norm_pool",
                 9: "rope_table", 10: "heads_fwd", 11: "heads_bwd", 12: "gemm", 13: "lora_down",
                 14: "heads_adamw", 15: "gemm_bwd", 16: "attention_bwd", 17: "norm_bwd",
-                18: "lora_bwd"}
-TENSOR_KERNELS = (3, 4, 5, 6, 7, 12, 13, 15, 16, 18)
+                18: "lora_bwd", 19: "flow_gemm", 20: "flow_attention", 21: "flow_misc",
+                22: "flow_wgrad"}
+TENSOR_KERNELS = (3, 4, 5, 6, 7, 12, 13, 15, 16, 18, 19, 20, 22)
 
 
 def jnx_trace_enable(capacity: int) -> None:

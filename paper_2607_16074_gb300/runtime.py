@@ -241,6 +241,67 @@ class DeviceHeads:
         return int(self.opt[t].version)
 
 
+class DeviceFlowHeads:
+    """Flow-matching action experts (DiT heads) of n_tenants tenants with the
+    same dimensions: stacked bf16 parameters (the gate/up pair of each block
+    packed by jnx_pack_gate_up) and fp32 gradient buffers of the same shapes."""
+
+    def __init__(self, dims: Dict, weights: Dict, stream=None):
+        L, s = J.lib(), _stream(stream)
+        self.dims = dims
+        T, dm, F = dims["n_tenants"], dims["d_model"], dims["d_ff"]
+        self.keep = {k: weights[k].contiguous() for k in J.FLOW_PARAMS}
+        self.blocks = []
+        for B in weights["blocks"]:
+            w_gu = torch.empty((T, 2 * F, dm), dtype=torch.bfloat16, device=B["wg"].device)
+            for t in range(T):
+                J.check(L.jnx_pack_gate_up(B["wg"][t].contiguous().data_ptr(),
+                                           B["wu"][t].contiguous().data_ptr(), F, dm,
+                                           w_gu[t].data_ptr(), s))
+            self.blocks.append(dict(w_qkv=B["w_qkv"].contiguous(), w_kvc=B["w_kvc"].contiguous(),
+                                    w_o=B["w_o"].contiguous(), w_gu=w_gu,
+                                    w_d=B["w_d"].contiguous()))
+        nb = max(1, len(self.blocks))
+        self.barr = (J.jnx_flow_block * nb)(*[J.jnx_flow_block(
+            *[b[k].data_ptr() for k in J.FLOW_BLOCK_PARAMS]) for b in self.blocks])
+        self.struct = J.jnx_flow_head(
+            dm, F, len(self.blocks), dims["chunk"], dims["action_dim"], dims["d_in"], T,
+            *[self.keep[k].data_ptr() for k in J.FLOW_PARAMS],
+            C.cast(self.barr, C.POINTER(J.jnx_flow_block)))
+        dev = self.keep["w_in"].device
+        self.grads = {k: torch.zeros(self.keep[k].shape, dtype=torch.float32, device=dev)
+                      for k in J.FLOW_PARAMS}
+        self.block_grads = [{k: torch.zeros(b[k].shape, dtype=torch.float32, device=dev)
+                             for k in J.FLOW_BLOCK_PARAMS} for b in self.blocks]
+        self.bgarr = (J.jnx_flow_block_grads * nb)(*[J.jnx_flow_block_grads(
+            *[g[k].data_ptr() for k in J.FLOW_BLOCK_PARAMS]) for g in self.block_grads])
+        self.gstruct = J.jnx_flow_grads(*[self.grads[k].data_ptr() for k in J.FLOW_PARAMS],
+                                        C.cast(self.bgarr, C.POINTER(J.jnx_flow_block_grads)))
+
+    def workspace_bytes(self, group: DeviceGroup) -> int:
+        return J.lib().jnx_flow_workspace_bytes(C.byref(self.struct), group.ref)
+
+    def forward(self, group: DeviceGroup, hidden, actions, noise, tau, velocity, loss, ws,
+                stream=None) -> None:
+        J.check(J.lib().jnx_flow_forward(
+            C.byref(self.struct), group.ref, hidden.data_ptr(), actions.data_ptr(),
+            noise.data_ptr(), tau.data_ptr(), velocity.data_ptr(), loss.data_ptr(),
+            ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)))
+
+    def backward(self, group: DeviceGroup, hidden, ws, accumulate: bool = False,
+                 stream=None) -> None:
+        J.check(J.lib().jnx_flow_backward(
+            C.byref(self.struct), group.ref, hidden.data_ptr(), C.byref(self.gstruct),
+            1 if accumulate else 0, ws.data_ptr(), ws.numel() * ws.element_size(),
+            _stream(stream)))
+
+    def sample(self, group: DeviceGroup, hidden, noise, n_steps: int, actions, ws,
+               stream=None) -> None:
+        J.check(J.lib().jnx_flow_sample(
+            C.byref(self.struct), group.ref, hidden.data_ptr(), noise.data_ptr(), n_steps,
+            actions.data_ptr(), ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)))
+
+
 def check_status(ws: torch.Tensor, stream=None) -> None:
     J.check(J.lib().jnx_check_status(ws.data_ptr(), _stream(stream)))
 

@@ -346,6 +346,37 @@ def make_head_weights(w: Workload, device="cpu", std: float = 0.02) -> List[Dict
     return out
 
 
+def make_flow_weights(n_tenants: int, d_model: int, d_ff: int, n_blocks: int, chunk: int,
+                      action_dim: int, d_in: int, seed: int, device="cpu",
+                      std: float = 0.02) -> Dict:
+    """Flow-matching action experts of n_tenants tenants, stacked over
+    tenants: bf16 N(0, std) projections [T, out, in] (the gate and up rows
+    of each block separately), N(0, std) biases and positions."""
+    T, dm, F = n_tenants, d_model, d_ff
+    r = lambda shape, *key: _normal((T,) + shape, std, device, seed, 70, *key)
+    out = dict(w_in=r((dm, action_dim), 0), b_in=r((dm,), 1), pos=r((chunk, dm), 2),
+               t1=r((dm, dm), 3), tb1=r((dm,), 4), t2=r((dm, dm), 5), tb2=r((dm,), 6),
+               w_out=r((action_dim, dm), 7), b_out=r((action_dim,), 8), blocks=[])
+    for b in range(n_blocks):
+        out["blocks"].append(dict(w_qkv=r((3 * dm, dm), 10, b), w_kvc=r((2 * dm, d_in), 11, b),
+                                  w_o=r((dm, dm), 12, b), wg=r((F, dm), 13, b),
+                                  wu=r((F, dm), 14, b), w_d=r((dm, F), 15, b)))
+    return out
+
+
+def make_flow_inputs(n_samples: int, chunk: int, action_dim: int, seed: int, device="cpu"):
+    """Per sample (packed order): target chunk U(-1, 1), noise N(0, 1), time
+    U(0, 1) (the flow-matching draws, made here and passed in)."""
+    import torch
+    g = _gen(device, seed, 80)
+    actions = torch.rand(n_samples, chunk, action_dim, generator=g, device=device) * 2 - 1
+    g = _gen(device, seed, 81)
+    noise = torch.randn(n_samples, chunk, action_dim, generator=g, device=device)
+    g = _gen(device, seed, 82)
+    tau = torch.rand(n_samples, generator=g, device=device)
+    return dict(actions=actions, noise=noise, tau=tau)
+
+
 def make_inputs(w: Workload, device="cpu") -> Dict:
     """Per-sample observations: vision rows N(0,1) bf16, text ids uniform in
     [0, vocab) (int32), action targets uniform in (-1, 1) (fp32), all laid out
