@@ -665,6 +665,108 @@ def run_kernel(args):
                 times_ms=[round(t, 4) for t in times])
 
 
+def run_flow(args):
+    """Flow-matching action experts (DiT heads) as the tenants' modules over
+    the shared 2B-class backbone (18 blocks, d=2048, 8x256 query heads on
+    one KV head, GeGLU 16384): `--flow-tenants` tenants x `--flow-batch`
+    samples (one 256-row image + 16..64 text tokens each; the paper's
+    forward breakdown uses 8 x 4), each tenant with a DiT expert of width
+    1024, 4 blocks, SwiGLU 4096, chunk 16 x 32.  One training step = the
+    shared backbone forward + every tenant's expert forward, rectified-flow
+    loss and backward; grouped (one plan) vs serial (each tenant alone, back
+    to back).  CUDA events, medians; the tracer gives the breakdown."""
+    import dataclasses
+
+    import torch
+
+    import synth
+    from paper_2607_16074_gb300 import build as B
+    from paper_2607_16074_gb300 import jnx as J
+    from paper_2607_16074_gb300 import runtime as R
+
+    B.build()
+    J.lib()
+    dev = torch.device("cuda", 0)
+    T, b = args.flow_tenants, args.flow_batch
+    bb = synth.Backbone(n_layers=18, d=2048, n_heads=8, n_kv_heads=1, head_dim=256, d_ff=16384,
+                        glu=synth.GLU_GEGLU)
+    dims = dict(n_tenants=T, d_model=1024, d_ff=4096, chunk=16, action_dim=32, d_in=bb.d)
+    tenants = [synth.Tenant(synth.HEAD_MLP, chunk=16, action_dim=32, d_hidden=1024, max_images=1)
+               for _ in range(T)]
+    rng = np.random.default_rng(43)
+    per = [[synth.Sample(1, int(rng.integers(16, 65))) for _ in range(b)] for _ in range(T)]
+    w = synth.custom_workload(bb, tenants, per, req_batch=b, seed=43, name=f"flow{T}x{b}")
+    bw = synth.make_backbone_weights(w, device=dev)
+    backbone = R.DeviceBackbone(bb, bw, n_tenants=T)
+    fw = synth.make_flow_weights(T, dims["d_model"], dims["d_ff"], 4, dims["chunk"],
+                                 dims["action_dim"], bb.d, 43, device=dev)
+    experts = R.DeviceFlowHeads(dims, fw)
+    inp = synth.make_inputs(w, device=dev)
+    s = torch.cuda.current_stream()
+
+    class Step:
+        def __init__(self, wsub):
+            plan = J.jnx_group_plan(wsub.schemas(), oracle_requests(wsub), T, 1 << 30, 1 << 30)
+            self.plan, self.g = plan, R.DeviceGroup(plan, device=dev)
+            self.ws_bb = torch.zeros(backbone.workspace_bytes(plan.n_tokens), dtype=torch.uint8,
+                                     device=dev)
+            self.ws_f = torch.zeros(experts.workspace_bytes(self.g), dtype=torch.uint8, device=dev)
+            self.hidden = torch.zeros((plan.n_tokens, bb.d), dtype=torch.bfloat16, device=dev)
+            self.fi = synth.make_flow_inputs(plan.n_samples, 16, 32, 44, device=dev)
+            self.vel = torch.zeros_like(self.fi["actions"])
+            self.loss = torch.zeros(T, device=dev)
+
+        def backbone(self):
+            backbone.forward(self.g, inp["vision"], inp["text_ids"], None, self.hidden, self.ws_bb)
+
+        def expert(self):
+            experts.forward(self.g, self.hidden, self.fi["actions"], self.fi["noise"],
+                            self.fi["tau"], self.vel, self.loss, self.ws_f)
+            experts.backward(self.g, self.hidden, self.ws_f)
+
+    def timed(fns):
+        for _ in range(max(args.warmup, 3)):
+            for f in fns:
+                f()
+        ts = []
+        for _ in range(args.steps):
+            a, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(s)
+            for f in fns:
+                f()
+            e.record(s)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(e))
+        return float(np.median(ts))
+
+    grouped = Step(w)
+    t_bb = timed([grouped.backbone])
+    t_ex = timed([grouped.expert])
+    t_step = timed([grouped.backbone, grouped.expert])
+    R.check_status(grouped.ws_bb)
+    R.check_status(grouped.ws_f)
+    # the expert's kernels in one traced step
+    J.jnx_trace_enable(8192)
+    grouped.expert()
+    torch.cuda.synchronize()
+    kinds, ms, work = J.jnx_trace_read(8192)
+    J.jnx_trace_disable()
+    expert_kernels = kernel_breakdown(J, kinds, ms, work)
+    serial = [Step(w.subset([t])) for t in range(T)]
+    t_serial = timed([f for st in serial for f in (st.backbone, st.expert)])
+    tokens = grouped.plan.n_tokens
+    return dict(metric="flow_expert_train_tokens_per_s",
+                value=round(tokens / (t_step / 1e3), 1), unit="tokens/s",
+                config=dict(workload=f"{T} tenants x {b} samples ({tokens} tokens) on a 2B-class "
+                                     "backbone (18 blocks, d=2048, MQA 8x256, GeGLU 16384)",
+                            expert="DiT: width 1024, 4 blocks, 16 heads, SwiGLU 4096, chunk 16 x 32"),
+                ms=dict(backbone_forward=round(t_bb, 3), expert_forward_backward=round(t_ex, 3),
+                        step=round(t_step, 3), serial_step=round(t_serial, 3)),
+                backbone_share_of_step=round(t_bb / t_step, 4),
+                speedup_vs_serial=round(t_serial / t_step, 4),
+                expert_kernels=expert_kernels)
+
+
 def run_grid(args):
     """Grouped vs serial inference (backbone forward + head forward, no
     targets) on the grid of tenants {2, 4, 6, 8} x local batch {1, 2, 4, 8}
@@ -787,7 +889,14 @@ def main():
                     help="grouped vs serial inference on the tenants x local batch grid")
     ap.add_argument("--train-lora", action="store_true",
                     help="time the per-tenant LoRA training step (use with --workload zipf2b)")
+    ap.add_argument("--flow", action="store_true",
+                    help="time flow-matching DiT experts as the tenants' modules")
+    ap.add_argument("--flow-tenants", type=int, default=8)
+    ap.add_argument("--flow-batch", type=int, default=4)
     args = ap.parse_args()
+    if args.flow:
+        print(json.dumps(run_flow(args)), flush=True)
+        return
     if args.train_lora:
         print(json.dumps(run_train(args)), flush=True)
         return

@@ -122,7 +122,9 @@ def test_flow_train_step_vs_oracle(dm, C, D):
     inp = _inputs(plan, C, D)
     g, vel, loss, ws = s.run(plan, hidden, inp)
     # bf16 operands of every projection and of the attention inputs, fp32
-    # residual stream, two blocks: a few 2^-9 roundings per block
+    # residual stream and attention, two blocks: a few 2^-9 roundings per
+    # block.  Measured relative L2 errors 1.2e-3 - 6.0e-3 over every
+    # parameter, tenant and both sizes; a wrong term or index is off by O(1).
     _check(s, plan, hidden, inp, vel, loss, 3e-2)
 
 
