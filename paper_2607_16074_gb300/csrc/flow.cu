@@ -168,19 +168,24 @@ __device__ __forceinline__ void stage_keys(float (*sk)[kHd + 1], float (*sv)[kHd
     }
 }
 
+// One CTA per (sample, head); each query's keys are split among KS = 64 / C
+// threads (thread t: query t % C, keys j = t / C (mod KS) of every staged
+// tile), whose partial (max, sum, accumulator) are merged at the end.
 __global__ void __launch_bounds__(64) k_flow_attn_fwd(const uint16_t* __restrict__ qkv,
                                                       const uint16_t* __restrict__ kvc,
                                                       const int* __restrict__ cu, FlowDims dd,
                                                       uint16_t* __restrict__ o,
                                                       float* __restrict__ lse) {
     __shared__ float sk[kKT][kHd + 1], sv[kKT][kHd + 1];
+    __shared__ float part[64][kHd + 2];  // per thread: accumulator, max, sum
     const int s = blockIdx.x, h = blockIdx.y, C = dd.C, dm = dd.dm;
-    const int c = threadIdx.x;
+    const int KS = min(8, 64 / C);  // key splits per query
+    const int c = threadIdx.x % C, ks = threadIdx.x / C;
     const int ctx0 = cu[s], L = cu[s + 1] - ctx0, act0 = s * C;
     const float sc = kLog2e / sqrtf((float)kHd);
     float q[kHd], acc[kHd];
     float m = -INFINITY, l = 0.f;
-    const bool act = c < C;
+    const bool act = ks < KS;
     if (act) {
         const uint16_t* qr = qkv + (size_t)(act0 + c) * 3 * dm + h * kHd;
 #pragma unroll
@@ -196,56 +201,72 @@ __global__ void __launch_bounds__(64) k_flow_attn_fwd(const uint16_t* __restrict
         stage_keys(sk, sv, j0, nk, L, kvc, ctx0, qkv, act0, dm, h);
         __syncthreads();
         if (!act) continue;
-        // the tile's scores (keys past nk are -inf, probability 0)
-        float sj[kKT];
-        float mt = m;
-#pragma unroll
-        for (int jj = 0; jj < kKT; ++jj) {
+        for (int jj = ks; jj < nk; jj += KS) {
             float a = 0.f;
 #pragma unroll
             for (int e = 0; e < kHd; ++e) a += q[e] * sk[jj][e];
-            sj[jj] = jj < nk ? a : -INFINITY;
-            mt = fmaxf(mt, sj[jj]);
-        }
-        const float alpha = exp2f(m - mt);
-        l *= alpha;
+            if (a > m) {
+                const float alpha = exp2f(m - a);
+                l *= alpha;
 #pragma unroll
-        for (int e = 0; e < kHd; ++e) acc[e] *= alpha;
-#pragma unroll
-        for (int jj = 0; jj < kKT; ++jj) {
-            const float p = exp2f(sj[jj] - mt);
+                for (int e = 0; e < kHd; ++e) acc[e] *= alpha;
+                m = a;
+            }
+            const float p = exp2f(a - m);
             l += p;
 #pragma unroll
             for (int e = 0; e < kHd; ++e) acc[e] += p * sv[jj][e];
         }
-        m = mt;
     }
     if (act) {
-        const float inv = 1.f / l;
-        uint16_t* orow = o + (size_t)(act0 + c) * dm + h * kHd;
 #pragma unroll
-        for (int e = 0; e < kHd; e += 2)
-            *reinterpret_cast<uint32_t*>(orow + e) = pack_bf2(acc[e] * inv, acc[e + 1] * inv);
-        lse[(size_t)(act0 + c) * dd.nh + h] = m + log2f(l);
+        for (int e = 0; e < kHd; ++e) part[threadIdx.x][e] = acc[e];
+        part[threadIdx.x][kHd] = m;
+        part[threadIdx.x][kHd + 1] = l;
+    }
+    __syncthreads();
+    if (act && ks == 0) {
+        float M = -INFINITY;
+        for (int k = 0; k < KS; ++k) M = fmaxf(M, part[k * C + c][kHd]);
+        float Ls = 0.f;
+        float w[8];
+        for (int k = 0; k < KS && k < 8; ++k) {
+            const float mk = part[k * C + c][kHd];
+            w[k] = mk == -INFINITY ? 0.f : exp2f(mk - M);
+            Ls += part[k * C + c][kHd + 1] * w[k];
+        }
+        const float inv = 1.f / Ls;
+        uint16_t* orow = o + (size_t)(act0 + c) * dm + h * kHd;
+        for (int e = 0; e < kHd; e += 2) {
+            float v0 = 0.f, v1 = 0.f;
+            for (int k = 0; k < KS && k < 8; ++k) {
+                v0 += part[k * C + c][e] * w[k];
+                v1 += part[k * C + c][e + 1] * w[k];
+            }
+            *reinterpret_cast<uint32_t*>(orow + e) = pack_bf2(v0 * inv, v1 * inv);
+        }
+        lse[(size_t)(act0 + c) * dd.nh + h] = M + log2f(Ls);
     }
 }
 
 // Backward, query side: dq_c = scale sum_j dS_cj k_j with dS = P (dP - D_c),
-// dP_cj = dO_c . v_j, D_c = dO_c . o_c.  One thread per query.
+// dP_cj = dO_c . v_j, D_c = dO_c . o_c.  Keys split among 64 / C threads per
+// query as in the forward; the partial dq are summed at the end.
 __global__ void __launch_bounds__(64) k_flow_attn_bwd_q(
     const uint16_t* __restrict__ qkv, const uint16_t* __restrict__ kvc, const int* __restrict__ cu,
     FlowDims dd, const uint16_t* __restrict__ o, const float* __restrict__ dO,
     const float* __restrict__ lse, uint16_t* __restrict__ dqkv) {
     __shared__ float sk[kKT][kHd + 1], sv[kKT][kHd + 1];
-    __shared__ float sq[64][kHd + 1];  // each thread's own (scaled) query row
+    __shared__ float sq[64][kHd + 1];  // each thread's own (scaled) query row, then its dq
     const int s = blockIdx.x, h = blockIdx.y, C = dd.C, dm = dd.dm;
-    const int c = threadIdx.x;
+    const int KS = min(8, 64 / C);  // key splits per query
+    const int c = threadIdx.x % C, ks = threadIdx.x / C;
     const int ctx0 = cu[s], L = cu[s + 1] - ctx0, act0 = s * C;
     const float sc = 1.f / sqrtf((float)kHd);
     float g[kHd], dq[kHd];
     float Dc = 0.f, lc = 0.f;
-    const bool act = c < C;
-    float* q = sq[c];
+    const bool act = ks < KS;
+    float* q = sq[threadIdx.x];
     if (act) {
         const size_t r = (size_t)(act0 + c);
         const uint16_t* qr = qkv + r * 3 * dm + h * kHd;
@@ -267,7 +288,7 @@ __global__ void __launch_bounds__(64) k_flow_attn_bwd_q(
         stage_keys(sk, sv, j0, nk, L, kvc, ctx0, qkv, act0, dm, h);
         __syncthreads();
         if (!act) continue;
-        for (int jj = 0; jj < nk; ++jj) {
+        for (int jj = ks; jj < nk; jj += KS) {
             float a = 0.f, dp = 0.f;
 #pragma unroll
             for (int e = 0; e < kHd; ++e) {
@@ -279,11 +300,22 @@ __global__ void __launch_bounds__(64) k_flow_attn_bwd_q(
             for (int e = 0; e < kHd; ++e) dq[e] += ds * sk[jj][e];
         }
     }
+    __syncthreads();  // every thread is done with its query row: reuse it for dq
     if (act) {
-        uint16_t* dr = dqkv + (size_t)(act0 + c) * 3 * dm + h * kHd;
 #pragma unroll
-        for (int e = 0; e < kHd; e += 2)
-            *reinterpret_cast<uint32_t*>(dr + e) = pack_bf2(dq[e] * sc, dq[e + 1] * sc);
+        for (int e = 0; e < kHd; ++e) q[e] = dq[e];
+    }
+    __syncthreads();
+    if (act && ks == 0) {
+        uint16_t* dr = dqkv + (size_t)(act0 + c) * 3 * dm + h * kHd;
+        for (int e = 0; e < kHd; e += 2) {
+            float v0 = 0.f, v1 = 0.f;
+            for (int k = 0; k < KS; ++k) {
+                v0 += sq[k * C + c][e];
+                v1 += sq[k * C + c][e + 1];
+            }
+            *reinterpret_cast<uint32_t*>(dr + e) = pack_bf2(v0 * sc, v1 * sc);
+        }
     }
 }
 
