@@ -37,8 +37,11 @@ constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 512;  // two 256-column fp32 accumulators
-constexpr int STG_BYTES = 4 * 2048;  // epilogue staging, 2 KB per epilogue warp
+constexpr int STG_BYTES = 4 * 2048;  // epilogue staging, 2 KB per epilogue warp (4 warps)
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/ + STG_BYTES;
+// with eight epilogue warps (two per TMEM lane quarter, each taking half of
+// a tile's columns) for the epilogues whose column halves are independent
+constexpr int SMEM_BYTES_EW8 = SMEM_BYTES + STG_BYTES;
 constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 // LoRA operands of one tile (K = 16, 32-byte rows): t rows and B rows, a
 // 2-deep ring after the main stages.
@@ -160,16 +163,20 @@ __device__ __forceinline__ float row_norm_scale(const GemmParams& p, int row, bo
 
 // The accumulator tile at tbase (this warp's 32 TMEM lanes = rows
 // row_base..row_base+31, 256 fp32 columns) -> the epilogue's output.
-template <int EPI>
+// NC, cb: the 32-column chunks [cb, cb + NC) of the tile this warp handles
+// (all 8, or one half of 4 with eight epilogue warps: EPI_BF16, EPI_F32,
+// EPI_RESID without a folded norm and EPI_GLU_BWD only).  Ring slots are
+// indexed by the pass within this warp's range, so they stay compile-time.
+template <int EPI, int NC = 8>
 __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int lane,
                                               int row_base, int row_end, int n0,
-                                              const GemmParams& p) {
+                                              const GemmParams& p, int cb = 0) {
     const int my_row = row_base + lane;
     const bool valid = my_row < row_end;
     const uint64_t pol = l2_evict_first_policy();  // outputs and residual are streamed
     if constexpr (EPI == EPI_BF16) {
 #pragma unroll 1
-        for (int c = 0; c < 8; ++c) {
+        for (int c = cb; c < cb + NC; ++c) {
             uint32_t r[32];
             tmem_ld32(tbase + c * 32, r);
             tmem_ld_wait();
@@ -198,24 +205,29 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                                    __uint_as_float(u.z), __uint_as_float(u.w));
             }
         };
+        constexpr int NP = 2 * NC;  // staging passes of this warp
+        const int pb = 2 * cb;
         if constexpr (EPI == EPI_RESID) {
 #pragma unroll
-            for (int q = 0; q < RD - 1; ++q) load_resid(q, xr[q]);
+            for (int q = 0; q < RD - 1; ++q) load_resid(pb + q, xr[q]);
         }
         // folded RMSNorm (EPI_RESID with norm_gamma): y = bf16(x * gamma) and
         // the sum of x^2 of each of this lane's four rows over its columns
-        const bool norm = EPI == EPI_RESID && p.norm_gamma != nullptr;
+        // (never with half-tile warps: a row's sums span the whole tile)
+        const bool norm = EPI == EPI_RESID && NC == 8 && p.norm_gamma != nullptr;
         float ssq[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
+        for (int lc = 0; lc < NC; ++lc) {
+            const int c = cb + lc;
             uint32_t r[32];
             tmem_ld32(tbase + c * 32, r);
             tmem_ld_wait();
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-                const int pass = 2 * c + h;
+                const int lp = 2 * lc + h;  // pass within this warp's range
+                const int pass = pb + lp;
                 if constexpr (EPI == EPI_RESID)
-                    if (pass + RD - 1 < 16) load_resid(pass + RD - 1, xr[(pass + RD - 1) % RD]);
+                    if (lp + RD - 1 < NP) load_resid(pass + RD - 1, xr[(lp + RD - 1) % RD]);
                 uint4 v[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u)
@@ -231,7 +243,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                     float4 o = make_float4(__uint_as_float(w.x), __uint_as_float(w.y),
                                            __uint_as_float(w.z), __uint_as_float(w.w));
                     if constexpr (EPI == EPI_RESID) {
-                        const float4 x = xr[pass % RD][i];
+                        const float4 x = xr[lp % RD][i];
                         o.x += x.x;
                         o.y += x.y;
                         o.z += x.z;
@@ -341,18 +353,22 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                 }
             }
         };
+        constexpr int NP = 2 * NC;  // staging passes of this warp
+        const int pb = 2 * cb;
 #pragma unroll
-        for (int q = 0; q < RD - 1; ++q) load_m(q, mg[q], mu[q]);
+        for (int q = 0; q < RD - 1; ++q) load_m(pb + q, mg[q], mu[q]);
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
+        for (int lc = 0; lc < NC; ++lc) {
+            const int c = cb + lc;
             uint32_t r[32];
             tmem_ld32(tbase + c * 32, r);
             tmem_ld_wait();
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-                const int pass = 2 * c + h;
-                if (pass + RD - 1 < 16) load_m(pass + RD - 1, mg[(pass + RD - 1) % RD],
-                                                mu[(pass + RD - 1) % RD]);
+                const int lp = 2 * lc + h;  // pass within this warp's range
+                const int pass = pb + lp;
+                if (lp + RD - 1 < NP) load_m(pass + RD - 1, mg[(lp + RD - 1) % RD],
+                                             mu[(lp + RD - 1) % RD]);
                 uint4 v[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u)
@@ -367,7 +383,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                     const int row = row_base + 8 * i + (lane >> 2);
                     const float dm[4] = {__uint_as_float(wv.x), __uint_as_float(wv.y),
                                          __uint_as_float(wv.z), __uint_as_float(wv.w)};
-                    const uint2 gm = mg[pass % RD][i], um = mu[pass % RD][i];
+                    const uint2 gm = mg[lp % RD][i], um = mu[lp % RD][i];
                     const uint2 og = make_uint2(
                         pack_bf2(dm[0] * bf2f(gm.x & 0xFFFF), dm[1] * bf2f(gm.x >> 16)),
                         pack_bf2(dm[2] * bf2f(gm.y & 0xFFFF), dm[3] * bf2f(gm.y >> 16)));
@@ -468,8 +484,8 @@ __device__ __forceinline__ void lora_part(const LoraGemm& lg, int nb, int& part,
     c0 = c;
 }
 
-template <int EPI, bool LORA>
-__global__ void __launch_bounds__(192, 1)
+template <int EPI, bool LORA, int EW>
+__global__ void __launch_bounds__(64 + 32 * EW, 1)
     k_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
            const __grid_constant__ typename std::conditional<LORA, LoraGemm, NoLora>::type lg,
            GemmParams p) {
@@ -500,7 +516,7 @@ __global__ void __launch_bounds__(192, 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
-            mbar_init(&tempty[a], 128);
+            mbar_init(&tempty[a], 32 * EW);
             mbar_init(&lfull[a], 1);
             mbar_init(&lempty[a], 1);
         }
@@ -655,6 +671,9 @@ __global__ void __launch_bounds__(192, 1)
         }
     } else {
         const int q = warp & 3;  // TMEM lane quarter this warp may access
+        // with eight epilogue warps, warps 2-5 take chunks 0-3 of a tile and
+        // warps 6-9 chunks 4-7 (the same lane quarters)
+        const int cb = EW == 8 ? ((warp - 2) >> 2) * 4 : 0;
         // this warp's staging slot, after the barrier block
         uint8_t* stg = reinterpret_cast<uint8_t*>(full) + 256 + (warp - 2) * 2048;
         int local = 0;
@@ -669,8 +688,8 @@ __global__ void __launch_bounds__(192, 1)
                 break;
             }
             tc_fence_after();
-            epilogue_tile<EPI>(tmem_base + acc * BN + ((uint32_t)(q * 32) << 16), stg, lane,
-                               row_base, g.row_end, g.nb * BN, p);
+            epilogue_tile<EPI, EW == 8 ? 4 : 8>(tmem_base + acc * BN + ((uint32_t)(q * 32) << 16),
+                                                stg, lane, row_base, g.row_end, g.nb * BN, p, cb);
             tc_fence_before();
             mbar_arrive(&tempty[acc]);
         }
@@ -740,18 +759,23 @@ int num_sms() {
     return n > 0 ? n : 1;
 }
 
-template <int EPI, bool LORA, class LG>
+template <int EPI, bool LORA, class LG, int EW = 4>
 static cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const LG& lg,
                               const GemmParams& p, int grid, cudaStream_t s) {
-    constexpr int smem = LORA ? gemm::SMEM_BYTES_LORA : gemm::SMEM_BYTES;
+    static_assert(EW == 4 || (EW == 8 && !LORA &&
+                              (EPI == EPI_BF16 || EPI == EPI_F32 || EPI == EPI_RESID ||
+                               EPI == EPI_GLU_BWD)),
+                  "eight epilogue warps: column-splittable epilogues without LoRA only");
+    constexpr int smem = LORA ? gemm::SMEM_BYTES_LORA
+                              : (EW == 8 ? gemm::SMEM_BYTES_EW8 : gemm::SMEM_BYTES);
     static bool attr_done = false;  // per instantiation; idempotent if raced
     if (!attr_done) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm<EPI, LORA>,
+        cudaError_t e = cudaFuncSetAttribute(k_gemm<EPI, LORA, EW>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         attr_done = true;
     }
-    k_gemm<EPI, LORA><<<grid, 192, smem, s>>>(ta, tb, lg, p);
+    k_gemm<EPI, LORA, EW><<<grid, 64 + 32 * EW, smem, s>>>(ta, tb, lg, p);
     return cudaGetLastError();
 }
 
@@ -791,11 +815,18 @@ jnx_status gemm_launch(const uint16_t* A, int lda, const uint16_t* B, int ldb, G
     const NoLora none{};
     switch (p.epi) {
         case EPI_BF16: e = launch_epi<EPI_BF16, false>(ta, tb, none, p, grid, s); break;
-        case EPI_F32: e = launch_epi<EPI_F32, false>(ta, tb, none, p, grid, s); break;
-        case EPI_RESID: e = launch_epi<EPI_RESID, false>(ta, tb, none, p, grid, s); break;
+        case EPI_F32: e = launch_epi<EPI_F32, false, NoLora, 8>(ta, tb, none, p, grid, s); break;
+        case EPI_RESID:
+            // eight epilogue warps unless an RMSNorm is folded in (its per-row
+            // sums span the whole tile)
+            e = p.norm_gamma ? launch_epi<EPI_RESID, false>(ta, tb, none, p, grid, s)
+                             : launch_epi<EPI_RESID, false, NoLora, 8>(ta, tb, none, p, grid, s);
+            break;
         case EPI_GLU: e = launch_epi<EPI_GLU, false>(ta, tb, none, p, grid, s); break;
         case EPI_ROPE: e = launch_epi<EPI_ROPE, false>(ta, tb, none, p, grid, s); break;
-        case EPI_GLU_BWD: e = launch_epi<EPI_GLU_BWD, false>(ta, tb, none, p, grid, s); break;
+        case EPI_GLU_BWD:
+            e = launch_epi<EPI_GLU_BWD, false, NoLora, 8>(ta, tb, none, p, grid, s);
+            break;
         case EPI_GLU_SAVE: e = launch_epi<EPI_GLU_SAVE, false>(ta, tb, none, p, grid, s); break;
         default: return fail(JNX_ERR_INVALID_ARG, "gemm: unknown epilogue %d", p.epi);
     }
