@@ -40,8 +40,11 @@ constexpr int TMEM_COLS = 512;  // two 256-column fp32 accumulators
 constexpr int STG_BYTES = 4 * 2048;  // epilogue staging, 2 KB per epilogue warp (4 warps)
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/ + STG_BYTES;
 // with eight epilogue warps (two per TMEM lane quarter, each taking half of
-// a tile's columns) for the epilogues whose column halves are independent
-constexpr int SMEM_BYTES_EW8 = SMEM_BYTES + STG_BYTES;
+// a tile's columns) for the epilogues whose column halves are independent;
+// their staging slots are 4 KB (32 rows x 32 fp32 columns)
+constexpr int STG_SLOT_EW8 = 4096;
+constexpr int SMEM_BYTES_EW8 = SMEM_BYTES - STG_BYTES + 8 * STG_SLOT_EW8;
+static_assert(SMEM_BYTES_EW8 <= 227 * 1024, "shared memory per CTA");
 constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 // LoRA operands of one tile (K = 16, 32-byte rows): t rows and B rows, a
 // 2-deep ring after the main stages.
@@ -325,6 +328,77 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                            n0 + c * 32, pol);
             stg_store_bf16(stg, lane, vu, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
                            n0 + 128 + c * 32, pol);
+        }
+    } else if constexpr (EPI == EPI_GLU_BWD && NC == 4) {
+        // half-tile warps (4 KB staging slot): one staging round per 32-column
+        // chunk, so each lane takes 8 contiguous columns of rows 8 i + lane / 4
+        // and its multiplier loads and result stores are 16 bytes; the next
+        // chunk's multipliers are in flight while one is finished.  F column f
+        // has its gate slot at packed column 256 (f / 128) + f % 128, its up
+        // slot 128 later; a lane reads each element before it writes it, so
+        // out may be aux.
+        auto pcol = [&](int c) {
+            const int f = n0 + c * 32 + (lane & 3) * 8;
+            return (f / 128) * 256 + (f % 128);
+        };
+        uint4 mg[2][4], mu[2][4];
+        auto load_m = [&](int c, uint4 (&g)[4], uint4 (&u)[4]) {
+            const int pc = pcol(c);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int row = row_base + 8 * i + (lane >> 2);
+                g[i] = u[i] = make_uint4(0u, 0u, 0u, 0u);
+                if (row < row_end) {
+                    const bf16_t* src = p.aux + (size_t)row * p.ldaux + pc;
+                    g[i] = ld_global_u4_hint(src, pol);
+                    u[i] = ld_global_u4_hint(src + 128, pol);
+                }
+            }
+        };
+        load_m(cb, mg[0], mu[0]);
+#pragma unroll
+        for (int lc = 0; lc < NC; ++lc) {
+            const int c = cb + lc;
+            if (lc + 1 < NC) load_m(c + 1, mg[(lc + 1) & 1], mu[(lc + 1) & 1]);
+            uint32_t r[32];
+            tmem_ld32(tbase + c * 32, r);
+            tmem_ld_wait();
+            // row `lane` puts its 32 fp32 (8 units of 16 bytes, XOR-swizzled
+            // by row % 8)
+            uint8_t* rowp = stg + lane * 128;
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                *reinterpret_cast<uint4*>(rowp + ((j ^ (lane & 7)) << 4)) =
+                    make_uint4(r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
+            __syncwarp();
+            const int pc = pcol(c);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int rr = 8 * i + (lane >> 2), u0 = (lane & 3) * 2;
+                const uint8_t* rp = stg + rr * 128;
+                const uint4 a = *reinterpret_cast<const uint4*>(rp + ((u0 ^ (rr & 7)) << 4));
+                const uint4 b = *reinterpret_cast<const uint4*>(rp + (((u0 + 1) ^ (rr & 7)) << 4));
+                const float dm[8] = {__uint_as_float(a.x), __uint_as_float(a.y),
+                                     __uint_as_float(a.z), __uint_as_float(a.w),
+                                     __uint_as_float(b.x), __uint_as_float(b.y),
+                                     __uint_as_float(b.z), __uint_as_float(b.w)};
+                const uint4 gm = mg[lc & 1][i], um = mu[lc & 1][i];
+                const uint32_t gw[4] = {gm.x, gm.y, gm.z, gm.w};
+                const uint32_t uw[4] = {um.x, um.y, um.z, um.w};
+                float og[8], ou[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    og[e] = dm[e] * bf2f((gw[e / 2] >> (16 * (e & 1))) & 0xFFFF);
+                    ou[e] = dm[e] * bf2f((uw[e / 2] >> (16 * (e & 1))) & 0xFFFF);
+                }
+                const int row = row_base + rr;
+                if (row < row_end) {
+                    bf16_t* dst = static_cast<bf16_t*>(p.out) + (size_t)row * p.ldo + pc;
+                    st_global_u4_hint(dst, pack8_bf16(og), pol);
+                    st_global_u4_hint(dst + 128, pack8_bf16(ou), pol);
+                }
+            }
+            __syncwarp();
         }
     } else if constexpr (EPI == EPI_GLU_BWD) {
         // accumulator: dm for F columns [n0, n0 + 256); F column f has its
@@ -675,7 +749,8 @@ __global__ void __launch_bounds__(64 + 32 * EW, 1)
         // warps 6-9 chunks 4-7 (the same lane quarters)
         const int cb = EW == 8 ? ((warp - 2) >> 2) * 4 : 0;
         // this warp's staging slot, after the barrier block
-        uint8_t* stg = reinterpret_cast<uint8_t*>(full) + 256 + (warp - 2) * 2048;
+        uint8_t* stg = reinterpret_cast<uint8_t*>(full) + 256 +
+                       (warp - 2) * (EW == 8 ? gemm::STG_SLOT_EW8 : 2048);
         int local = 0;
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
             const int acc = local & 1;
