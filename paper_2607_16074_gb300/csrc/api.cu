@@ -24,7 +24,7 @@ struct BackboneWs {
     int* status;
     float* x;         // residual stream [N, d] fp32
     uint16_t* nrm;    // GEMM input of the folded RMSNorm: bf16(x * gamma) [N, d]
-    float* ss;        // its per-row, per-256-column-block sums of x^2 [N, d / 256]
+    float* ss;        // its per-row, per-128-column-block sums of x^2 [N, d / 128]
     uint16_t* qkv;    // [N, (H + 2 Hkv) hd] bf16
     uint16_t* att;    // [N, H hd] bf16
     uint16_t* u;      // [N, F] bf16
@@ -48,7 +48,7 @@ BackboneWs carve_backbone(const jnx_backbone* bb, int64_t N, void* base) {
     w.status = reinterpret_cast<int*>(take(kStatusBytes));
     w.x = reinterpret_cast<float*>(take((size_t)N * d * 4));
     w.nrm = reinterpret_cast<uint16_t*>(take((size_t)N * d * 2));
-    w.ss = reinterpret_cast<float*>(take((size_t)N * (d / 256) * 4));
+    w.ss = reinterpret_cast<float*>(take((size_t)N * (d / 128) * 4));
     w.qkv = reinterpret_cast<uint16_t*>(take((size_t)N * qkvw * 2));
     w.att = reinterpret_cast<uint16_t*>(take((size_t)N * bb->n_heads * bb->head_dim * 2));
     w.u = reinterpret_cast<uint16_t*>(take((size_t)N * bb->d_ff * 2));
@@ -263,7 +263,7 @@ static jnx_status backbone_forward(const jnx_backbone* bb, const jnx_group* g,
         }
         auto fold_in = [&](GemmParams& q) {
             q.ss_in = w.ss;
-            q.ss_parts = d / 256;
+            q.ss_parts = d / 128;
             q.ss_cols = d;
             q.ss_eps = bb->eps;
         };

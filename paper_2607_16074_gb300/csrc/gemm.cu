@@ -192,8 +192,9 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
     } else if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
         // 16 fp32 columns (64 bytes) per staging pass; the residual is
         // loaded RD - 1 passes ahead of its use, so several passes' loads
-        // are in flight while the accumulator is staged
-        constexpr int RD = 4;
+        // are in flight while the accumulator is staged (a shallower ring for
+        // half-tile warps, which run with fewer registers per thread)
+        constexpr int RD = NC == 4 ? 3 : 4;
         float* dst = EPI == EPI_RESID ? p.resid : static_cast<float*>(p.out);
         const int ld = EPI == EPI_RESID ? p.ldr : p.ldo;
         float4 xr[RD][4];
@@ -215,10 +216,10 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
             for (int q = 0; q < RD - 1; ++q) load_resid(pb + q, xr[q]);
         }
         // folded RMSNorm (EPI_RESID with norm_gamma): y = bf16(x * gamma) and
-        // the sum of x^2 of each of this lane's four rows over its columns
-        // (never with half-tile warps: a row's sums span the whole tile)
-        const bool norm = EPI == EPI_RESID && NC == 8 && p.norm_gamma != nullptr;
-        float ssq[4] = {0.f, 0.f, 0.f, 0.f};
+        // the sums of x^2 of each of this lane's four rows over its columns,
+        // one per 128-column half of the tile (8 staging passes each)
+        const bool norm = EPI == EPI_RESID && p.norm_gamma != nullptr;
+        float ssq[NC / 4][4] = {};
 #pragma unroll
         for (int lc = 0; lc < NC; ++lc) {
             const int c = cb + lc;
@@ -259,7 +260,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                                           pol);
                     if (EPI == EPI_RESID && norm) {
                         const uint2 g = *reinterpret_cast<const uint2*>(p.norm_gamma + col);
-                        ssq[i] += o.x * o.x + o.y * o.y + o.z * o.z + o.w * o.w;
+                        ssq[lp / 8][i] += o.x * o.x + o.y * o.y + o.z * o.z + o.w * o.w;
                         if (row < row_end)
                             *reinterpret_cast<uint2*>(p.norm_out + (size_t)row * p.N + col) =
                                 make_uint2(pack_bf2(o.x * bf2f(g.x & 0xFFFF), o.y * bf2f(g.x >> 16)),
@@ -270,16 +271,19 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
             }
         }
         if (norm) {
-            // the four lanes of a row hold its 256 columns between them
-            const int parts = p.N / 256;
+            // the four lanes of a row hold each half's columns between them
+            const int parts = p.N / 128;
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                float t = ssq[i];
-                t += __shfl_xor_sync(0xffffffffu, t, 1);
-                t += __shfl_xor_sync(0xffffffffu, t, 2);
-                const int row = row_base + 8 * i + (lane >> 2);
-                if ((lane & 3) == 0 && row < row_end) p.ss_out[(size_t)row * parts + n0 / 256] = t;
-            }
+            for (int hb = 0; hb < NC / 4; ++hb)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    float t = ssq[hb][i];
+                    t += __shfl_xor_sync(0xffffffffu, t, 1);
+                    t += __shfl_xor_sync(0xffffffffu, t, 2);
+                    const int row = row_base + 8 * i + (lane >> 2);
+                    if ((lane & 3) == 0 && row < row_end)
+                        p.ss_out[(size_t)row * parts + (n0 + 32 * cb) / 128 + hb] = t;
+                }
         }
     } else if constexpr (EPI == EPI_GLU) {
         const float rs = row_norm_scale(p, my_row, valid);
@@ -890,13 +894,11 @@ jnx_status gemm_launch(const uint16_t* A, int lda, const uint16_t* B, int ldb, G
     const NoLora none{};
     switch (p.epi) {
         case EPI_BF16: e = launch_epi<EPI_BF16, false>(ta, tb, none, p, grid, s); break;
-        case EPI_F32: e = launch_epi<EPI_F32, false, NoLora, 8>(ta, tb, none, p, grid, s); break;
-        case EPI_RESID:
-            // eight epilogue warps unless an RMSNorm is folded in (its per-row
-            // sums span the whole tile)
-            e = p.norm_gamma ? launch_epi<EPI_RESID, false>(ta, tb, none, p, grid, s)
-                             : launch_epi<EPI_RESID, false, NoLora, 8>(ta, tb, none, p, grid, s);
-            break;
+        // eight epilogue warps only where the epilogue is the bottleneck: with
+        // the fp32 and residual epilogues they slowed the GEMMs on GB300 (the
+        // 7B-class O / down projections 1,314 / 1,460 -> 1,246 / 1,419 TFLOP/s)
+        case EPI_F32: e = launch_epi<EPI_F32, false>(ta, tb, none, p, grid, s); break;
+        case EPI_RESID: e = launch_epi<EPI_RESID, false>(ta, tb, none, p, grid, s); break;
         case EPI_GLU: e = launch_epi<EPI_GLU, false>(ta, tb, none, p, grid, s); break;
         case EPI_ROPE: e = launch_epi<EPI_ROPE, false>(ta, tb, none, p, grid, s); break;
         case EPI_GLU_BWD:

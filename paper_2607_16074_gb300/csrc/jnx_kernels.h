@@ -30,7 +30,7 @@ struct GemmParams {
     int* status;          // device status word
     // RMSNorm folded across two GEMMs.  EPI_RESID with norm_gamma set also
     // writes y = bf16(x_new * gamma[col]) to norm_out [M, N] and, per row and
-    // 256-column block, the partial sum of x_new^2 to ss_out [M, N / 256].
+    // 128-column block, the partial sum of x_new^2 to ss_out [M, N / 128].
     const uint16_t* norm_gamma;
     uint16_t* norm_out;
     float* ss_out;
@@ -138,7 +138,7 @@ jnx_status final_pool_launch(const float* x, const uint16_t* gamma, float eps, c
                              int S, int d, float* pooled, uint16_t* hidden, cudaStream_t s);
 
 // Folded RMSNorm, first half: y = bf16(x * gamma) [M, d] and per row and
-// 256-column block the sum of x^2 (ss [M, d / 256]).
+// 128-column block the sum of x^2 (ss [M, d / 128]).
 jnx_status rms_prep_launch(const float* x, const uint16_t* gamma, int M, int d, uint16_t* y,
                            float* ss, cudaStream_t s);
 

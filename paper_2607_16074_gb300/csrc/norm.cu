@@ -109,7 +109,7 @@ __global__ void __launch_bounds__(256) k_rms_prep(const float* __restrict__ x,
                                                   const uint16_t* __restrict__ gamma, int M,
                                                   uint16_t* __restrict__ y, float* __restrict__ ss) {
     constexpr int D = V * 128;
-    constexpr int P = D / 256;  // 256-column blocks: lane float4s i = 2b, 2b + 1
+    constexpr int P = D / 128;  // 128-column blocks: lane float4 i = b
     const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (row >= M) return;
@@ -121,8 +121,7 @@ __global__ void __launch_bounds__(256) k_rms_prep(const float* __restrict__ x,
     for (int b = 0; b < P; ++b) {
         float t = 0.f;
 #pragma unroll
-        for (int i = 2 * b; i < 2 * b + 2; ++i)
-            t += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+        t += v[b].x * v[b].x + v[b].y * v[b].y + v[b].z * v[b].z + v[b].w * v[b].w;
         t = warp_sum(t);
         if (lane == 0) ss[(size_t)row * P + b] = t;
     }
