@@ -54,8 +54,8 @@ def workload_desc(w):
 # command are in profiles/), valid only for the GEMM source it was taken on.
 RECORDED_TRAFFIC = {
     # workload: (sha256 of csrc/gemm.cu, bytes per launch, profile)
-    "llama7b": ("53b6844e9af1004cc4be22948c8c6d683c8c9846040c420e5bae98210ada0a2b",
-                3.01e9 + 1.44e9, "profiles/gemm_gate_up_glu_llama7b_dram.md"),
+    "llama7b": ("c51437a803d1cb100b10081d1d06002dc8f3bc9a80e54031f9ca5b791ce0992f",
+                3.09e9 + 1.44e9, "profiles/gemm_gate_up_glu_llama7b_dram.md"),
 }
 
 
