@@ -256,7 +256,16 @@ def run_train(args):
     step = R.LoraTrainStep(backbone, heads, R.DeviceGroup(plan, device=dev), device=dev)
     preds = torch.zeros_like(inp["targets"])
     stream = torch.cuda.current_stream()
-    run = lambda st: st.run(inp["vision"], inp["text_ids"], inp["targets"], preds)
+    # every group tenant's optimizer step on its own adapters and head
+    opt = R.TenantAdamW(backbone.lora_pairs())
+    heads.init_optimizer()
+    group_tenants = sorted(set(plan.slot_tenant.tolist()))
+
+    def run(st):
+        st.run(inp["vision"], inp["text_ids"], inp["targets"], preds)
+        tenants = sorted(set(st.group.plan.slot_tenant.tolist()))
+        opt.step(tenants, lr=1e-4, weight_decay=0.01)
+        heads.adamw_step(st.group, lr=1e-4, weight_decay=0.01)
     for _ in range(max(args.warmup, 3)):
         run(step)
     for ws in (step.ws_bb, step.ws_h, step.ws_bwd):
@@ -335,7 +344,9 @@ def run_train(args):
                 config=dict(workload=workload_desc(w), tokens=tokens, samples=plan.n_samples,
                             tenants=len(w.tenants), lora_rank=w.backbone.lora_rank,
                             step="forward (saving block inputs) + heads + feature gradient + "
-                                 "adapter backward (blocks recomputed)"),
+                                 "adapter backward (blocks recomputed) + every group tenant's "
+                                 "AdamW step on its adapters and head",
+                            group_tenants=len(group_tenants)),
                 clocks=clk, gpu_launches=int(launches), roofline=roofline,
                 backward_tensor=dict(kernels="gemm_bwd + attention_bwd + lora_bwd",
                                      achieved=round(bwd_tf, 1), unit="TFLOP/s",
@@ -673,8 +684,8 @@ def run_flow(args):
     forward breakdown uses 8 x 4), each tenant with a DiT expert of width
     1024, 4 blocks, SwiGLU 4096, chunk 16 x 32.  One training step = the
     shared backbone forward + every tenant's expert forward, rectified-flow
-    loss and backward; grouped (one plan) vs serial (each tenant alone, back
-    to back).  CUDA events, medians; the tracer gives the breakdown."""
+    loss, backward and AdamW step; grouped (one plan) vs serial (each tenant
+    alone, back to back).  CUDA events, medians; the tracer gives the breakdown."""
     import dataclasses
 
     import torch
@@ -701,6 +712,7 @@ def run_flow(args):
     fw = synth.make_flow_weights(T, dims["d_model"], dims["d_ff"], 4, dims["chunk"],
                                  dims["action_dim"], bb.d, 43, device=dev)
     experts = R.DeviceFlowHeads(dims, fw)
+    opt = R.TenantAdamW(experts.param_pairs())  # each tenant's expert optimizer
     inp = synth.make_inputs(w, device=dev)
     s = torch.cuda.current_stream()
 
@@ -715,6 +727,7 @@ def run_flow(args):
             self.fi = synth.make_flow_inputs(plan.n_samples, 16, 32, 44, device=dev)
             self.vel = torch.zeros_like(self.fi["actions"])
             self.loss = torch.zeros(T, device=dev)
+            self.tenants = sorted(set(plan.slot_tenant.tolist()))
 
         def backbone(self):
             backbone.forward(self.g, inp["vision"], inp["text_ids"], None, self.hidden, self.ws_bb)
@@ -723,6 +736,7 @@ def run_flow(args):
             experts.forward(self.g, self.hidden, self.fi["actions"], self.fi["noise"],
                             self.fi["tau"], self.vel, self.loss, self.ws_f)
             experts.backward(self.g, self.hidden, self.ws_f)
+            opt.step(self.tenants, lr=1e-4, weight_decay=0.01)
 
     def timed(fns):
         for _ in range(max(args.warmup, 3)):

@@ -543,6 +543,32 @@ jnx_status jnx_flow_sample(const jnx_flow_head* fh, const jnx_group* g, const ui
                            size_t ws_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
+ * Tenant-private optimizer step on any trainable tensors
+ * ------------------------------------------------------------------------ */
+
+/* One tenant-private parameter tensor (device): its bf16 value the kernels
+ * read (written in place), fp32 master copy, AdamW moments (zero before the
+ * first step), fp32 gradient, element count, and the number of steps this
+ * tensor has taken (a host counter the call increments).  A LoRA adapter's
+ * or a flow expert's slice of one tenant is one such tensor. */
+typedef struct {
+    uint16_t* param;
+    float* master;
+    float* m;
+    float* v;
+    const float* grad;
+    int64_t n;
+    int32_t* step;
+} jnx_adam_tensor;
+
+/* One AdamW step (the update of jnx_heads_adamw) on each tensor, with
+ * t = *step + 1 for that tensor; then each *step increments.  Errors:
+ * JNX_ERR_INVALID_ARG (null buffer, n < 0, hyperparameters as for
+ * jnx_heads_adamw); nothing is written on error. */
+jnx_status jnx_adamw_tensors(const jnx_adam_tensor* tensors, int32_t n_tensors,
+                             const jnx_adamw* hp, void* stream);
+
+/* ------------------------------------------------------------------------
  * Status and helpers
  * ------------------------------------------------------------------------ */
 

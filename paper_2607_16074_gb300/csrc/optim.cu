@@ -85,15 +85,70 @@ __global__ void __launch_bounds__(256) k_adamw(const __grid_constant__ AdamTable
 
 using namespace jnx;
 
+static jnx_status check_hp(const jnx_adamw* hp) {
+    if (!(hp->lr >= 0.f) || !(hp->beta1 >= 0.f && hp->beta1 < 1.f) ||
+        !(hp->beta2 >= 0.f && hp->beta2 < 1.f) || !(hp->eps >= 0.f) || !(hp->weight_decay >= 0.f))
+        return fail(JNX_ERR_INVALID_ARG, "adamw: hyperparameter out of range");
+    return JNX_OK;
+}
+
+static jnx_status launch_segments(const std::vector<AdamSeg>& segs, const jnx_adamw* hp,
+                                  cudaStream_t s) {
+    for (size_t a = 0; a < segs.size(); a += kMaxSeg) {
+        AdamTable tab;
+        const int ns = (int)std::min<size_t>(kMaxSeg, segs.size() - a);
+        long long mx = 0;
+        for (int k = 0; k < ns; ++k) {
+            tab.seg[k] = segs[a + k];
+            mx = std::max(mx, segs[a + k].n);
+        }
+        if (mx == 0) continue;
+        const int bx = (int)std::min<long long>((mx / 4 + 255) / 256 + 1, 1024);
+        k_adamw<<<dim3(bx, ns), 256, 0, s>>>(tab, hp->lr, hp->beta1, hp->beta2, hp->eps,
+                                             hp->weight_decay);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "adamw: %s", cudaGetErrorString(e));
+    }
+    return JNX_OK;
+}
+
+extern "C" jnx_status jnx_adamw_tensors(const jnx_adam_tensor* tensors, int32_t n_tensors,
+                                        const jnx_adamw* hp, void* stream) {
+    clear_error();
+    if (!hp || n_tensors < 0 || (n_tensors > 0 && !tensors))
+        return fail(JNX_ERR_INVALID_ARG, "adamw: null argument");
+    jnx_status st;
+    if ((st = check_hp(hp))) return st;
+    std::vector<AdamSeg> segs;
+    double bytes = 0.0;
+    for (int i = 0; i < n_tensors; ++i) {
+        const jnx_adam_tensor& t = tensors[i];
+        if (t.n < 0 || !t.step) return fail(JNX_ERR_INVALID_ARG, "adamw: tensor %d", i);
+        if (t.n > 0 && (!t.param || !t.master || !t.m || !t.v || !t.grad))
+            return fail(JNX_ERR_INVALID_ARG, "adamw: tensor %d has a null buffer", i);
+        const int step = *t.step + 1;
+        const float c1 = (float)(1.0 / (1.0 - std::pow((double)hp->beta1, step)));
+        const float c2 = (float)(1.0 / (1.0 - std::pow((double)hp->beta2, step)));
+        segs.push_back(AdamSeg{t.param, t.master, t.m, t.v, t.grad, t.n, c1, c2});
+        bytes += 30.0 * (double)t.n;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    {
+        TraceScope ts(JNX_K_ADAMW, bytes, s);
+        if ((st = launch_segments(segs, hp, s))) return st;
+    }
+    for (int i = 0; i < n_tensors; ++i) ++*tensors[i].step;
+    return JNX_OK;
+}
+
 extern "C" jnx_status jnx_heads_adamw(const jnx_head* heads, const jnx_head_grads* grads,
                                       jnx_head_opt* opt, int32_t n_tenants, const jnx_group* g,
                                       const jnx_adamw* hp, void* stream) {
     clear_error();
     if (!heads || !grads || !opt || !g || !hp || n_tenants < 0)
         return fail(JNX_ERR_INVALID_ARG, "adamw: null argument");
-    if (!(hp->lr >= 0.f) || !(hp->beta1 >= 0.f && hp->beta1 < 1.f) ||
-        !(hp->beta2 >= 0.f && hp->beta2 < 1.f) || !(hp->eps >= 0.f) || !(hp->weight_decay >= 0.f))
-        return fail(JNX_ERR_INVALID_ARG, "adamw: hyperparameter out of range");
+    jnx_status st;
+    if ((st = check_hp(hp))) return st;
     if (g->n_slots == 0) return JNX_OK;
     if (!g->h_slot_tenant) return fail(JNX_ERR_INVALID_ARG, "adamw: null slot tenants");
 
@@ -139,20 +194,7 @@ extern "C" jnx_status jnx_heads_adamw(const jnx_head* heads, const jnx_head_grad
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     {
         TraceScope ts(JNX_K_ADAMW, bytes, s);
-        for (size_t a = 0; a < segs.size(); a += kMaxSeg) {
-            AdamTable tab;
-            const int ns = (int)std::min<size_t>(kMaxSeg, segs.size() - a);
-            long long mx = 0;
-            for (int k = 0; k < ns; ++k) {
-                tab.seg[k] = segs[a + k];
-                mx = std::max(mx, segs[a + k].n);
-            }
-            const int bx = (int)std::min<long long>((mx / 4 + 255) / 256 + 1, 1024);
-            k_adamw<<<dim3(bx, ns), 256, 0, s>>>(tab, hp->lr, hp->beta1, hp->beta2, hp->eps,
-                                                 hp->weight_decay);
-            cudaError_t e = cudaGetLastError();
-            if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "adamw: %s", cudaGetErrorString(e));
-        }
+        if ((st = launch_segments(segs, hp, s))) return st;
     }
     for (int i = 0; i < g->n_slots; ++i) {
         jnx_head_opt& o = opt[g->h_slot_tenant[i]];

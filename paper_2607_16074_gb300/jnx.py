@@ -158,6 +158,12 @@ class jnx_flow_grads(C.Structure):
                [("blocks", C.POINTER(jnx_flow_block_grads))]
 
 
+class jnx_adam_tensor(C.Structure):
+    _fields_ = [("param", C.c_void_p), ("master", C.c_void_p), ("m", C.c_void_p),
+                ("v", C.c_void_p), ("grad", C.c_void_p), ("n", C.c_int64),
+                ("step", C.POINTER(C.c_int32))]
+
+
 _LIB: Optional[C.CDLL] = None
 
 EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_workspace_bytes",
@@ -172,7 +178,7 @@ EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_work
            "jnx_op_attention_lse", "jnx_op_attention_backward_prep",
            "jnx_op_attention_backward_workspace_bytes", "jnx_op_attention_backward",
            "jnx_op_rms_backward", "jnx_op_gemm_glu_backward", "jnx_flow_workspace_bytes",
-           "jnx_flow_forward", "jnx_flow_backward", "jnx_flow_sample")
+           "jnx_flow_forward", "jnx_flow_backward", "jnx_flow_sample", "jnx_adamw_tensors")
 
 
 def lib() -> C.CDLL:
@@ -232,6 +238,7 @@ def lib() -> C.CDLL:
                                     C.POINTER(jnx_flow_grads), i32, vp, sz, vp]),
         "jnx_flow_sample": (i32, [C.POINTER(jnx_flow_head), C.POINTER(jnx_group), vp, vp, i32,
                                   vp, vp, sz, vp]),
+        "jnx_adamw_tensors": (i32, [C.POINTER(jnx_adam_tensor), i32, C.POINTER(jnx_adamw), vp]),
         "jnx_check_status": (i32, [vp, vp]),
         "jnx_pack_gate_up": (i32, [vp, vp, i32, i32, vp, vp]),
         "jnx_op_pack": (i32, [C.POINTER(jnx_group), vp, i64, vp, i64, vp, i32, i32, vp, vp, vp]),

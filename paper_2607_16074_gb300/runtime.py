@@ -131,6 +131,17 @@ class DeviceBackbone:
             self.lora_grads.append(g)
             self.lgarr[i] = J.jnx_lora_grads(*[_ptr(g[k]) for k in J.LORA_GRADS])
 
+    def lora_pairs(self):
+        """(adapter [n_tenants, ...] bf16, its gradient buffer) of every layer,
+        for TenantAdamW (the adapters are updated in place)."""
+        per = len(self.keep) // max(1, self.cfg.n_layers)
+        out = []
+        for i in range(self.cfg.n_layers):
+            ent = self.keep[i * per:(i + 1) * per][6:]
+            for name, p in zip(J.LORA_GRADS, ent):
+                out.append((p, self.lora_grads[i][name]))
+        return out
+
     def forward_train(self, group: DeviceGroup, vision, text_ids, pooled, hidden, saved, ws,
                       stream=None) -> None:
         J.check(J.lib().jnx_backbone_forward_train(
@@ -281,6 +292,14 @@ class DeviceFlowHeads:
     def workspace_bytes(self, group: DeviceGroup) -> int:
         return J.lib().jnx_flow_workspace_bytes(C.byref(self.struct), group.ref)
 
+    def param_pairs(self):
+        """(stacked parameter, its gradient buffer) of every expert tensor
+        (the packed gate/up pair as one), for TenantAdamW."""
+        out = [(self.keep[k], self.grads[k]) for k in J.FLOW_PARAMS]
+        for b, g in zip(self.blocks, self.block_grads):
+            out += [(b[k], g[k]) for k in J.FLOW_BLOCK_PARAMS]
+        return out
+
     def forward(self, group: DeviceGroup, hidden, actions, noise, tau, velocity, loss, ws,
                 stream=None) -> None:
         J.check(J.lib().jnx_flow_forward(
@@ -300,6 +319,38 @@ class DeviceFlowHeads:
         J.check(J.lib().jnx_flow_sample(
             C.byref(self.struct), group.ref, hidden.data_ptr(), noise.data_ptr(), n_steps,
             actions.data_ptr(), ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)))
+
+
+class TenantAdamW:
+    """Tenant-private AdamW over stacked per-tenant parameters: for every
+    (parameter [n_tenants, ...] bf16, gradient [n_tenants, ...] fp32) pair an
+    fp32 master copy and zero moments; step(tenants) updates only those
+    tenants' slices, each slice with its own step counter
+    (jnx_adamw_tensors)."""
+
+    def __init__(self, pairs):
+        self.pairs = [(p, g) for p, g in pairs]
+        self.master = [p.float().clone() for p, _ in self.pairs]
+        self.m = [torch.zeros_like(x) for x in self.master]
+        self.v = [torch.zeros_like(x) for x in self.master]
+        self.counts: Dict = {}
+
+    def steps(self, i: int, t: int) -> int:
+        c = self.counts.get((i, t))
+        return int(c.value) if c is not None else 0
+
+    def step(self, tenants, lr: float, beta1: float = 0.9, beta2: float = 0.999,
+             eps: float = 1e-8, weight_decay: float = 0.0, stream=None) -> None:
+        arr = []
+        for i, (p, g) in enumerate(self.pairs):
+            for t in tenants:
+                cnt = self.counts.setdefault((i, t), C.c_int32(0))
+                arr.append(J.jnx_adam_tensor(p[t].data_ptr(), self.master[i][t].data_ptr(),
+                                             self.m[i][t].data_ptr(), self.v[i][t].data_ptr(),
+                                             g[t].data_ptr(), p[t].numel(), C.pointer(cnt)))
+        tab = (J.jnx_adam_tensor * max(1, len(arr)))(*arr)
+        hp = J.jnx_adamw(lr, beta1, beta2, eps, weight_decay)
+        J.check(J.lib().jnx_adamw_tensors(tab, len(arr), C.byref(hp), _stream(stream)))
 
 
 def check_status(ws: torch.Tensor, stream=None) -> None:

@@ -148,3 +148,49 @@ def test_adamw_rejects_bad_hyperparameters():
         with pytest.raises(J.JnxError):
             heads.adamw_step(g, **dict(HP, **bad))
     assert heads.version(0) == 0
+
+
+def test_tenant_adamw_on_stacked_slices_only_the_named_tenants_move():
+    # the generic entry point (jnx_adamw_tensors) on stacked per-tenant
+    # tensors, as the LoRA adapters and flow experts hold them
+    g = torch.Generator().manual_seed(12)
+    params = [torch.randn(3, 40, 24, generator=g).to(torch.bfloat16).cuda(),
+              torch.randn(3, 7, generator=g).to(torch.bfloat16).cuda()]
+    grads = [torch.randn(p.shape, generator=g).cuda() for p in params]
+    p0 = [p.clone() for p in params]
+    opt = R.TenantAdamW(list(zip(params, grads)))
+    ref = {(i, t): (f64(params[i][t]), np.zeros(params[i][t].shape), np.zeros(params[i][t].shape))
+           for i in range(2) for t in (0, 2)}
+    for step in (1, 2, 3):
+        opt.step([0, 2], **HP)
+        torch.cuda.synchronize()
+        for (i, t), (p, m, v) in ref.items():
+            p, m, v = O.adamw_step(p, f64(grads[i][t]), m, v, step, **HP32)
+            ref[(i, t)] = (p, m, v)
+            assert opt.steps(i, t) == step
+            assert _close(f64(opt.m[i][t]), m, 4e-6)
+            assert _close(f64(opt.v[i][t]), v, 4e-6)
+            assert _close(f64(opt.master[i][t]), p, 1e-6, 1e-7)
+            assert torch.equal(params[i][t], opt.master[i][t].to(torch.bfloat16))
+    for i in range(2):
+        assert torch.equal(params[i][1], p0[i][1])  # tenant 1 not named: untouched
+        assert opt.steps(i, 1) == 0
+
+
+def test_flow_expert_and_adapter_parameter_pairs():
+    # the accessors pair every trainable tensor with a gradient of its shape
+    w = synth.make_workload("zipf2b", n_layers=1)
+    bw = synth.make_backbone_weights(w.subset([0]), device="cuda")
+    bb = R.DeviceBackbone(w.backbone, bw, n_tenants=len(w.tenants))
+    bb.prepare_backward()
+    pairs = bb.lora_pairs()
+    assert len(pairs) == 8
+    for p, gr in pairs:
+        assert p.shape == gr.shape and p.dtype == torch.bfloat16 and gr.dtype == torch.float32
+    dims = dict(n_tenants=2, d_model=256, d_ff=256, chunk=4, action_dim=3, d_in=256)
+    fw = synth.make_flow_weights(2, 256, 256, 2, 4, 3, 256, 5, device="cuda")
+    fh = R.DeviceFlowHeads(dims, fw)
+    fp = fh.param_pairs()
+    assert len(fp) == 9 + 2 * 5
+    for p, gr in fp:
+        assert p.shape == gr.shape
