@@ -512,7 +512,9 @@ typedef struct {
     const jnx_flow_block_grads* blocks;  /* HOST array [n_blocks] */
 } jnx_flow_grads;
 
-/* Workspace bytes of jnx_flow_forward / jnx_flow_backward / jnx_flow_sample. */
+/* Workspace bytes of jnx_flow_forward / jnx_flow_backward / jnx_flow_sample.
+ * The workspace must be 256-byte aligned and the t1, t2 and w_out weights
+ * 16-byte aligned (JNX_ERR_INVALID_ARG otherwise). */
 size_t jnx_flow_workspace_bytes(const jnx_flow_head* fh, const jnx_group* g);
 
 /* Training forward of every group tenant's expert over its samples.

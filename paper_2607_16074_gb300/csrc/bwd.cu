@@ -28,21 +28,49 @@ namespace jnx {
 // ---------------------------------------------------------------------------
 // transpose
 // ---------------------------------------------------------------------------
+// 64 x 64 tiles through shared memory, 16-byte loads along the source rows
+// and 16-byte stores along the destination rows when the buffers are 16-byte
+// aligned (vec), element by element at the edges and otherwise.
 __global__ void __launch_bounds__(256) k_transpose(const uint16_t* __restrict__ src, int rows,
-                                                   int cols, uint16_t* __restrict__ dst) {
-    __shared__ uint16_t tile[32][34];
+                                                   int cols, uint16_t* __restrict__ dst, int vec) {
+    __shared__ uint16_t tile[64][64 + 2];
     const size_t plane = (size_t)rows * cols;
     src += (size_t)blockIdx.z * plane;
     dst += (size_t)blockIdx.z * plane;
-    const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
-    for (int i = threadIdx.y; i < 32; i += 8) {
-        const int r = r0 + i, c = c0 + threadIdx.x;
-        if (r < rows && c < cols) tile[i][threadIdx.x] = src[(size_t)r * cols + c];
+    const int r0 = blockIdx.y * 64, c0 = blockIdx.x * 64;
+    const bool vec_in = vec && (cols % 8) == 0 && c0 + 64 <= cols;
+    for (int i = threadIdx.x; i < 64 * 8; i += 256) {
+        const int r = i / 8, u = i % 8;  // 8 elements at columns c0 + 8 u
+        if (r0 + r >= rows) continue;
+        if (vec_in) {
+            const uint4 v = *reinterpret_cast<const uint4*>(src + (size_t)(r0 + r) * cols + c0 + 8 * u);
+            const uint16_t* e = reinterpret_cast<const uint16_t*>(&v);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) tile[r][8 * u + k] = e[k];
+        } else {
+            for (int k = 0; k < 8; ++k) {
+                const int c = c0 + 8 * u + k;
+                if (c < cols) tile[r][8 * u + k] = src[(size_t)(r0 + r) * cols + c];
+            }
+        }
     }
     __syncthreads();
-    for (int i = threadIdx.y; i < 32; i += 8) {
-        const int c = c0 + i, r = r0 + threadIdx.x;
-        if (c < cols && r < rows) dst[(size_t)c * rows + r] = tile[threadIdx.x][i];
+    const bool vec_out = vec && (rows % 8) == 0 && r0 + 64 <= rows;
+    for (int i = threadIdx.x; i < 64 * 8; i += 256) {
+        const int c = i / 8, u = i % 8;  // destination row c0 + c, columns r0 + 8 u
+        if (c0 + c >= cols) continue;
+        if (vec_out) {
+            uint16_t e[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) e[k] = tile[8 * u + k][c];
+            *reinterpret_cast<uint4*>(dst + (size_t)(c0 + c) * rows + r0 + 8 * u) =
+                *reinterpret_cast<const uint4*>(e);
+        } else {
+            for (int k = 0; k < 8; ++k) {
+                const int r = r0 + 8 * u + k;
+                if (r < rows) dst[(size_t)(c0 + c) * rows + r] = tile[8 * u + k][c];
+            }
+        }
     }
 }
 
@@ -50,10 +78,11 @@ jnx_status transpose_launch(const uint16_t* src, int batch, int rows, int cols, 
                             cudaStream_t s) {
     if (batch < 0 || rows < 0 || cols < 0) return fail(JNX_ERR_INVALID_ARG, "transpose: sizes");
     if (batch == 0 || rows == 0 || cols == 0) return JNX_OK;
-    if ((rows + 31) / 32 > 65535 || batch > 65535)
+    if ((rows + 63) / 64 > 65535 || batch > 65535)
         return fail(JNX_ERR_UNSUPPORTED, "transpose: too many rows or planes");
-    k_transpose<<<dim3((cols + 31) / 32, (rows + 31) / 32, batch), dim3(32, 8), 0, s>>>(src, rows,
-                                                                                     cols, dst);
+    const int vec = ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0;
+    k_transpose<<<dim3((cols + 63) / 64, (rows + 63) / 64, batch), 256, 0, s>>>(src, rows, cols,
+                                                                             dst, vec);
     cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "transpose: %s", cudaGetErrorString(e));
 }

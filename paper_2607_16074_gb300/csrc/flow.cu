@@ -48,19 +48,40 @@ __device__ __forceinline__ float silu_grad_f(float z) {
 }
 
 // ---------------------------------------------------------------------------
-// time embedding: s(tau), z1 = T1 s + tb1, phi = T2 SiLU(z1) + tb2 (one CTA
-// per sample; one warp per output row, lanes along the dot product)
+// time embedding: s(tau), z1 = T1 s + tb1, phi = T2 SiLU(z1) + tb2.  Each
+// layer is one launch over (sample, block of 32 output rows): one warp per
+// row, lanes along the dot product with 16-byte weight loads (dm is a
+// multiple of 256), the row sum in a fixed butterfly order.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_flow_time(const float* __restrict__ tau,
-                                                   const int* __restrict__ sample_slot,
-                                                   const __grid_constant__ FlowSlots fs, FlowDims dd,
-                                                   const uint16_t* __restrict__ t1,
-                                                   const uint16_t* __restrict__ tb1,
-                                                   const uint16_t* __restrict__ t2,
-                                                   const uint16_t* __restrict__ tb2,
-                                                   float* __restrict__ sfeat,
-                                                   float* __restrict__ z1, float* __restrict__ phi) {
-    extern __shared__ float sh[];  // s(tau) [dm], SiLU(z1) [dm]
+constexpr int kTimeRows = 32;
+
+// dot product of the bf16 row w [dm] with the fp32 vector v [dm] in shared
+// memory, summed over the warp (every lane returns the sum)
+__device__ __forceinline__ float warp_row_dot(const uint16_t* __restrict__ w,
+                                              const float* __restrict__ v, int dm, int lane) {
+    float acc = 0.f;
+    for (int k = 8 * lane; k < dm; k += 256) {
+        const uint4 q = *reinterpret_cast<const uint4*>(w + k);
+        const uint32_t u[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            acc = fmaf(__uint_as_float(u[e] << 16), v[k + 2 * e], acc);
+            acc = fmaf(__uint_as_float(u[e] & 0xffff0000u), v[k + 2 * e + 1], acc);
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    return acc;
+}
+
+__global__ void __launch_bounds__(256) k_flow_time1(const float* __restrict__ tau,
+                                                    const int* __restrict__ sample_slot,
+                                                    const __grid_constant__ FlowSlots fs,
+                                                    FlowDims dd, const uint16_t* __restrict__ t1,
+                                                    const uint16_t* __restrict__ tb1,
+                                                    float* __restrict__ sfeat,
+                                                    float* __restrict__ z1) {
+    extern __shared__ float sh[];  // s(tau) [dm]
     const int s = blockIdx.x, dm = dd.dm, half = dm / 2;
     const int t = fs.tenant[sample_slot[s]];
     const float tv = tau[s];
@@ -70,29 +91,32 @@ __global__ void __launch_bounds__(256) k_flow_time(const float* __restrict__ tau
         const float a = 1000.f * tv * w;
         const float v = i < half ? sinf(a) : cosf(a);
         sh[i] = v;
-        sfeat[(size_t)s * dm + i] = v;
+        if (blockIdx.y == 0) sfeat[(size_t)s * dm + i] = v;
     }
     __syncthreads();
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint16_t* T1 = t1 + (size_t)t * dm * dm;
-    for (int j = warp; j < dm; j += nw) {
-        float acc = 0.f;
-        for (int k = lane; k < dm; k += 32) acc += bf2f(T1[(size_t)j * dm + k]) * sh[k];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-        if (lane == 0) {
-            const float z = acc + bf2f(tb1[(size_t)t * dm + j]);
-            z1[(size_t)s * dm + j] = z;
-            sh[dm + j] = silu_f(z);
-        }
+    for (int j = blockIdx.y * kTimeRows + warp; j < (blockIdx.y + 1) * kTimeRows; j += 8) {
+        const float acc = warp_row_dot(T1 + (size_t)j * dm, sh, dm, lane);
+        if (lane == 0) z1[(size_t)s * dm + j] = acc + bf2f(tb1[(size_t)t * dm + j]);
     }
+}
+
+__global__ void __launch_bounds__(256) k_flow_time2(const int* __restrict__ sample_slot,
+                                                    const __grid_constant__ FlowSlots fs,
+                                                    FlowDims dd, const uint16_t* __restrict__ t2,
+                                                    const uint16_t* __restrict__ tb2,
+                                                    const float* __restrict__ z1,
+                                                    float* __restrict__ phi) {
+    extern __shared__ float sh[];  // SiLU(z1) [dm]
+    const int s = blockIdx.x, dm = dd.dm;
+    const int t = fs.tenant[sample_slot[s]];
+    for (int i = threadIdx.x; i < dm; i += blockDim.x) sh[i] = silu_f(z1[(size_t)s * dm + i]);
     __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint16_t* T2 = t2 + (size_t)t * dm * dm;
-    for (int j = warp; j < dm; j += nw) {
-        float acc = 0.f;
-        for (int k = lane; k < dm; k += 32) acc += bf2f(T2[(size_t)j * dm + k]) * sh[dm + k];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    for (int j = blockIdx.y * kTimeRows + warp; j < (blockIdx.y + 1) * kTimeRows; j += 8) {
+        const float acc = warp_row_dot(T2 + (size_t)j * dm, sh, dm, lane);
         if (lane == 0) phi[(size_t)s * dm + j] = acc + bf2f(tb2[(size_t)t * dm + j]);
     }
 }
@@ -136,269 +160,536 @@ __global__ void __launch_bounds__(256) k_flow_embed(
 }
 
 // ---------------------------------------------------------------------------
-// attention: per (sample, head) the C action queries against the sample's L
-// context keys then its C action keys, online softmax in fp32 (log2 units).
-// One thread per query; keys staged 32 at a time in shared memory.
+// attention on the warp-level bf16 tensor-core path (mma.sync m16n8k16, fp32
+// accumulation).  Per (sample, head): the C action queries against the
+// sample's L context keys then its C action keys, bidirectional.  Keys are
+// staged 64 at a time by cp.async into shared-memory rows of 64 bf16 (128
+// bytes, the 16-byte units XOR-swizzled by the row's low three bits, so the
+// ldmatrix row gathers hit distinct banks).  Query rows past C are zero and
+// never stored; key rows past L + C are zero and masked.
 //   qkv [M_a, 3 dm] bf16 (q | k_a | v_a), kvc [N, 2 dm] bf16 (k_c | v_c),
-//   o [M_a, dm] bf16, lse [M_a, nh] fp32 (log2 of the softmax denominator
-//   of the log2e-scaled scores).
+//   o [M_a, dm] bf16, lse [M_a, nh] fp32: the log2 of the softmax
+//   denominator of the log2e-scaled scores, their maximum included.
 // ---------------------------------------------------------------------------
-constexpr int kKT = 32;  // keys per staged tile
+constexpr int kKT = 64;          // keys per staged tile
+constexpr int kRowB = kHd * 2;   // bytes per staged row
+constexpr int kTileB = kKT * kRowB;
 
-__device__ __forceinline__ void stage_keys(float (*sk)[kHd + 1], float (*sv)[kHd + 1], int j0,
-                                           int nk, int L, const uint16_t* __restrict__ kvc,
-                                           int ctx0, const uint16_t* __restrict__ qkv, int act0,
-                                           int dm, int h) {
-    for (int i = threadIdx.x; i < kKT * kHd; i += blockDim.x) {
-        const int jj = i / kHd, e = i % kHd, j = j0 + jj;
-        float kv = 0.f, vv = 0.f;
-        if (jj < nk) {
-            if (j < L) {
-                const uint16_t* row = kvc + (size_t)(ctx0 + j) * 2 * dm;
-                kv = bf2f(row[h * kHd + e]);
-                vv = bf2f(row[dm + h * kHd + e]);
-            } else {
-                const uint16_t* row = qkv + (size_t)(act0 + j - L) * 3 * dm;
-                kv = bf2f(row[dm + h * kHd + e]);
-                vv = bf2f(row[2 * dm + h * kHd + e]);
-            }
-        }
-        sk[jj][e] = kv;
-        sv[jj][e] = vv;
+__device__ __forceinline__ uint32_t swz(int row, int unit) {
+    return (uint32_t)(row * kRowB + ((unit ^ (row & 7)) << 4));
+}
+
+// Key j of the sample (context rows first, then its action rows): its K row;
+// the V row follows dm elements later in both buffers.
+__device__ __forceinline__ const uint16_t* key_row(int j, int L, const uint16_t* kvc, int ctx0,
+                                                   const uint16_t* qkv, int act0, int dm, int h) {
+    return j < L ? kvc + (size_t)(ctx0 + j) * 2 * dm + h * kHd
+                 : qkv + (size_t)(act0 + j - L) * 3 * dm + dm + h * kHd;
+}
+
+// cp.async of keys j0 .. j0 + 63 into the K tile at sk and the V tile at sv.
+__device__ __forceinline__ void load_kv_tile(uint32_t sk, uint32_t sv, int j0, int nkeys, int L,
+                                             const uint16_t* kvc, int ctx0, const uint16_t* qkv,
+                                             int act0, int dm, int h) {
+    for (int i = threadIdx.x; i < kKT * 8; i += blockDim.x) {
+        const int r = i >> 3, u = i & 7, j = j0 + r;
+        const bool ok = j < nkeys;
+        const uint16_t* kr = ok ? key_row(j, L, kvc, ctx0, qkv, act0, dm, h) : qkv;
+        cp_async16(sk + swz(r, u), kr + 8 * u, ok);
+        cp_async16(sv + swz(r, u), kr + dm + 8 * u, ok);
     }
 }
 
-// One CTA per (sample, head); each query's keys are split among KS = 64 / C
-// threads (thread t: query t % C, keys j = t / C (mod KS) of every staged
-// tile), whose partial (max, sum, accumulator) are merged at the end.
-__global__ void __launch_bounds__(64) k_flow_attn_fwd(const uint16_t* __restrict__ qkv,
-                                                      const uint16_t* __restrict__ kvc,
-                                                      const int* __restrict__ cu, FlowDims dd,
-                                                      uint16_t* __restrict__ o,
-                                                      float* __restrict__ lse) {
-    __shared__ float sk[kKT][kHd + 1], sv[kKT][kHd + 1];
-    __shared__ float part[64][kHd + 2];  // per thread: accumulator, max, sum
+// cp.async of the bf16 rows 0 .. C - 1 (row stride ld) into a tile of `rows`
+// rows at dst; rows C .. rows - 1 zero.
+__device__ __forceinline__ void load_rows(uint32_t dst, const uint16_t* src, size_t ld, int C,
+                                          int rows) {
+    for (int i = threadIdx.x; i < rows * 8; i += blockDim.x) {
+        const int r = i >> 3, u = i & 7;
+        const bool ok = r < C;
+        cp_async16(dst + swz(r, u), ok ? src + (size_t)r * ld + 8 * u : src, ok);
+    }
+}
+
+// The fp32 rows 0 .. C - 1 (row stride ld) as bf16 into a tile of `rows` rows
+// at dst (generic pointer); rows C .. rows - 1 zero.
+__device__ __forceinline__ void store_rows_bf16(uint8_t* dst, const float* src, size_t ld, int C,
+                                                int rows) {
+    for (int i = threadIdx.x; i < rows * 8; i += blockDim.x) {
+        const int r = i >> 3, u = i & 7;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (r < C) {
+            const float4 a = *reinterpret_cast<const float4*>(src + (size_t)r * ld + 8 * u);
+            const float4 b = *reinterpret_cast<const float4*>(src + (size_t)r * ld + 8 * u + 4);
+            v = make_uint4(pack_bf2(a.x, a.y), pack_bf2(a.z, a.w), pack_bf2(b.x, b.y),
+                           pack_bf2(b.z, b.w));
+        }
+        *reinterpret_cast<uint4*>(dst + swz(r, u)) = v;
+    }
+}
+
+// A operand (16 rows from row0, k16 step kk) from a swizzled row tile.
+__device__ __forceinline__ void ld_a(uint32_t base, int row0, int kk, int lane, uint32_t (&a)[4]) {
+    const int mi = lane >> 3, rr = lane & 7;
+    ldsm_x4(base + swz(row0 + rr + 8 * (mi & 1), kk * 2 + (mi >> 1)), a[0], a[1], a[2], a[3]);
+}
+// B operand of two n8 tiles (rows n0 .. n0 + 15 hold n, their columns k;
+// k16 step kk): b0, b1 for the first tile, b2, b3 for the second.
+__device__ __forceinline__ void ld_b(uint32_t base, int n0, int kk, int lane, uint32_t (&b)[4]) {
+    const int mi = lane >> 3, rr = lane & 7;
+    ldsm_x4(base + swz(n0 + rr + 8 * (mi >> 1), kk * 2 + (mi & 1)), b[0], b[1], b[2], b[3]);
+}
+// B operand of two n8 tiles (columns 16 dn .. 16 dn + 15 hold n, rows
+// k0 .. k0 + 15 hold k).
+__device__ __forceinline__ void ld_bt(uint32_t base, int k0, int dn, int lane, uint32_t (&b)[4]) {
+    const int mi = lane >> 3, rr = lane & 7;
+    ldsm_x4_t(base + swz(k0 + rr + 8 * (mi & 1), dn * 2 + (mi >> 1)), b[0], b[1], b[2], b[3]);
+}
+// Two n8 accumulator tiles (16 rows x 16 columns) as the bf16 A operand of
+// the next product (its k = their columns).
+__device__ __forceinline__ void acc_to_a(const float (&c0)[4], const float (&c1)[4],
+                                         uint32_t (&a)[4]) {
+    a[0] = pack_bf2(c0[0], c0[1]);
+    a[1] = pack_bf2(c0[2], c0[3]);
+    a[2] = pack_bf2(c1[0], c1[1]);
+    a[3] = pack_bf2(c1[2], c1[3]);
+}
+__device__ __forceinline__ void mma4(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
+                                     uint32_t b1) {
+    mma_bf16(c, a[0], a[1], a[2], a[3], b0, b1);
+}
+
+// Forward.  One CTA of four warps per (sample, head); warp w takes query
+// tile w / KS (16 rows) and the w % KS-th of the 64 / KS-key slices of every
+// staged tile, with its own running maximum and sum; the KS slices are
+// merged at the end in slice order.
+template <int KS>
+__global__ void __launch_bounds__(128) k_flow_attn_fwd(const uint16_t* __restrict__ qkv,
+                                                       const uint16_t* __restrict__ kvc,
+                                                       const int* __restrict__ cu, FlowDims dd,
+                                                       uint16_t* __restrict__ o,
+                                                       float* __restrict__ lse) {
+    constexpr int NK = kKT / KS, NT = NK / 8;
+    __shared__ __align__(128) uint8_t sbuf[4 * kTileB];  // (K, V) x 2 buffers
     const int s = blockIdx.x, h = blockIdx.y, C = dd.C, dm = dd.dm;
-    const int KS = min(8, 64 / C);  // key splits per query
-    const int c = threadIdx.x % C, ks = threadIdx.x / C;
-    const int ctx0 = cu[s], L = cu[s + 1] - ctx0, act0 = s * C;
-    const float sc = kLog2e / sqrtf((float)kHd);
-    float q[kHd], acc[kHd];
-    float m = -INFINITY, l = 0.f;
-    const bool act = ks < KS;
-    if (act) {
-        const uint16_t* qr = qkv + (size_t)(act0 + c) * 3 * dm + h * kHd;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, tq = lane & 3;
+    const int MT = (C + 15) >> 4, mt = warp / KS, ks = warp % KS;
+    const bool active = mt < MT;
+    const int ctx0 = cu[s], L = cu[s + 1] - ctx0, act0 = s * C, nkeys = L + C;
+    const uint32_t sb = smem_u32(sbuf);
+    load_rows(sb, qkv + (size_t)act0 * 3 * dm + h * kHd, 3 * dm, C, MT * 16);
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
+    uint32_t qa[4][4];
+    if (active)
 #pragma unroll
-        for (int e = 0; e < kHd; ++e) {
-            q[e] = bf2f(qr[e]) * sc;
-            acc[e] = 0.f;
+        for (int kk = 0; kk < 4; ++kk) ld_a(sb, mt * 16, kk, lane, qa[kk]);
+    __syncthreads();
+    float oacc[8][4];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) oacc[i][0] = oacc[i][1] = oacc[i][2] = oacc[i][3] = 0.f;
+    float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+    const float sc2 = kLog2e / sqrtf((float)kHd);
+    const int ntiles = (nkeys + kKT - 1) / kKT;
+    load_kv_tile(sb, sb + kTileB, 0, nkeys, L, kvc, ctx0, qkv, act0, dm, h);
+    cp_async_commit();
+    for (int t = 0; t < ntiles; ++t) {
+        const uint32_t kb = sb + (t & 1) * 2 * kTileB, vb = kb + kTileB;
+        if (t + 1 < ntiles) {
+            const uint32_t nk = sb + ((t + 1) & 1) * 2 * kTileB;
+            load_kv_tile(nk, nk + kTileB, (t + 1) * kKT, nkeys, L, kvc, ctx0, qkv, act0, dm, h);
         }
-    }
-    const int nkeys = L + C;
-    for (int j0 = 0; j0 < nkeys; j0 += kKT) {
-        const int nk = min(kKT, nkeys - j0);
+        cp_async_commit();
+        cp_async_wait<1>();
         __syncthreads();
-        stage_keys(sk, sv, j0, nk, L, kvc, ctx0, qkv, act0, dm, h);
-        __syncthreads();
-        if (!act) continue;
-        for (int jj = ks; jj < nk; jj += KS) {
-            float a = 0.f;
+        if (active) {
+            float sacc[NT][4];
 #pragma unroll
-            for (int e = 0; e < kHd; ++e) a += q[e] * sk[jj][e];
-            if (a > m) {
-                const float alpha = exp2f(m - a);
-                l *= alpha;
+            for (int i = 0; i < NT; ++i) sacc[i][0] = sacc[i][1] = sacc[i][2] = sacc[i][3] = 0.f;
 #pragma unroll
-                for (int e = 0; e < kHd; ++e) acc[e] *= alpha;
-                m = a;
+            for (int kk = 0; kk < 4; ++kk)
+#pragma unroll
+                for (int nb = 0; nb < NT / 2; ++nb) {
+                    uint32_t b[4];
+                    ld_b(kb, ks * NK + nb * 16, kk, lane, b);
+                    mma4(sacc[2 * nb], qa[kk], b[0], b[1]);
+                    mma4(sacc[2 * nb + 1], qa[kk], b[2], b[3]);
+                }
+            float mx[2] = {mrow[0], mrow[1]};
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int j = t * kKT + ks * NK + nt * 8 + 2 * tq + (e & 1);
+                    const float v = j < nkeys ? sacc[nt][e] * sc2 : -INFINITY;
+                    sacc[nt][e] = v;
+                    mx[e >> 1] = fmaxf(mx[e >> 1], v);
+                }
+            float alpha[2];
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                mx[i] = fmaxf(mx[i], __shfl_xor_sync(0xffffffffu, mx[i], 1));
+                mx[i] = fmaxf(mx[i], __shfl_xor_sync(0xffffffffu, mx[i], 2));
+                alpha[i] = mx[i] == -INFINITY ? 1.f : exp2f(mrow[i] - mx[i]);
+                mrow[i] = mx[i];
+                lrow[i] *= alpha[i];
             }
-            const float p = exp2f(a - m);
-            l += p;
 #pragma unroll
-            for (int e = 0; e < kHd; ++e) acc[e] += p * sv[jj][e];
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float m = mx[e >> 1];
+                    const float p = m == -INFINITY ? 0.f : exp2f(sacc[nt][e] - m);
+                    sacc[nt][e] = p;
+                    lrow[e >> 1] += p;
+                }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                oacc[i][0] *= alpha[0];
+                oacc[i][1] *= alpha[0];
+                oacc[i][2] *= alpha[1];
+                oacc[i][3] *= alpha[1];
+            }
+#pragma unroll
+            for (int k2 = 0; k2 < NK / 16; ++k2) {
+                uint32_t pa[4];
+                acc_to_a(sacc[2 * k2], sacc[2 * k2 + 1], pa);
+#pragma unroll
+                for (int dn = 0; dn < 4; ++dn) {
+                    uint32_t b[4];
+                    ld_bt(vb, ks * NK + k2 * 16, dn, lane, b);
+                    mma4(oacc[2 * dn], pa, b[0], b[1]);
+                    mma4(oacc[2 * dn + 1], pa, b[2], b[3]);
+                }
+            }
         }
+        __syncthreads();
     }
-    if (act) {
 #pragma unroll
-        for (int e = 0; e < kHd; ++e) part[threadIdx.x][e] = acc[e];
-        part[threadIdx.x][kHd] = m;
-        part[threadIdx.x][kHd + 1] = l;
+    for (int i = 0; i < 2; ++i) {
+        lrow[i] += __shfl_xor_sync(0xffffffffu, lrow[i], 1);
+        lrow[i] += __shfl_xor_sync(0xffffffffu, lrow[i], 2);
+    }
+    if (KS == 1) {
+        if (!active) return;
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const int c = mt * 16 + g + 8 * i;
+            if (c >= C) continue;
+            const float inv = 1.f / lrow[i];
+            uint16_t* orow = o + (size_t)(act0 + c) * dm + h * kHd;
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt)
+                *reinterpret_cast<uint32_t*>(orow + nt * 8 + 2 * tq) =
+                    pack_bf2(oacc[nt][2 * i] * inv, oacc[nt][2 * i + 1] * inv);
+            if (tq == 0) lse[(size_t)(act0 + c) * dd.nh + h] = mrow[i] + log2f(lrow[i]);
+        }
+        return;
+    }
+    // merge the KS slices: per warp its 16 x 64 partial output, maximum and sum
+    float* mo = reinterpret_cast<float*>(sbuf);  // [4][16][kHd + 1]
+    float* mm = mo + 4 * 16 * (kHd + 1);         // [4][16]
+    float* ml = mm + 4 * 16;                     // [4][16]
+    if (active) {
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const int r = g + 8 * i;
+            float* row = mo + (warp * 16 + r) * (kHd + 1);
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                row[nt * 8 + 2 * tq] = oacc[nt][2 * i];
+                row[nt * 8 + 2 * tq + 1] = oacc[nt][2 * i + 1];
+            }
+            if (tq == 0) {
+                mm[warp * 16 + r] = mrow[i];
+                ml[warp * 16 + r] = lrow[i];
+            }
+        }
     }
     __syncthreads();
-    if (act && ks == 0) {
+    for (int i = threadIdx.x; i < MT * 16 * (kHd / 2); i += blockDim.x) {
+        const int r = i / (kHd / 2), e = 2 * (i % (kHd / 2));
+        if (r >= C) continue;
+        const int w0 = (r >> 4) * KS, rl = r & 15;
         float M = -INFINITY;
-        for (int k = 0; k < KS; ++k) M = fmaxf(M, part[k * C + c][kHd]);
-        float Ls = 0.f;
-        float w[8];
-        for (int k = 0; k < KS && k < 8; ++k) {
-            const float mk = part[k * C + c][kHd];
-            w[k] = mk == -INFINITY ? 0.f : exp2f(mk - M);
-            Ls += part[k * C + c][kHd + 1] * w[k];
+#pragma unroll
+        for (int k = 0; k < KS; ++k) M = fmaxf(M, mm[(w0 + k) * 16 + rl]);
+        float Ls = 0.f, v0 = 0.f, v1 = 0.f;
+#pragma unroll
+        for (int k = 0; k < KS; ++k) {
+            const float mk = mm[(w0 + k) * 16 + rl];
+            const float wk = mk == -INFINITY ? 0.f : exp2f(mk - M);
+            const float* row = mo + ((w0 + k) * 16 + rl) * (kHd + 1);
+            Ls += ml[(w0 + k) * 16 + rl] * wk;
+            v0 += row[e] * wk;
+            v1 += row[e + 1] * wk;
         }
         const float inv = 1.f / Ls;
-        uint16_t* orow = o + (size_t)(act0 + c) * dm + h * kHd;
-        for (int e = 0; e < kHd; e += 2) {
-            float v0 = 0.f, v1 = 0.f;
-            for (int k = 0; k < KS && k < 8; ++k) {
-                v0 += part[k * C + c][e] * w[k];
-                v1 += part[k * C + c][e + 1] * w[k];
-            }
-            *reinterpret_cast<uint32_t*>(orow + e) = pack_bf2(v0 * inv, v1 * inv);
-        }
-        lse[(size_t)(act0 + c) * dd.nh + h] = M + log2f(Ls);
+        *reinterpret_cast<uint32_t*>(o + (size_t)(act0 + r) * dm + h * kHd + e) =
+            pack_bf2(v0 * inv, v1 * inv);
+        if (e == 0) lse[(size_t)(act0 + r) * dd.nh + h] = M + log2f(Ls);
     }
 }
 
-// Backward, query side: dq_c = scale sum_j dS_cj k_j with dS = P (dP - D_c),
-// dP_cj = dO_c . v_j, D_c = dO_c . o_c.  Keys split among 64 / C threads per
-// query as in the forward; the partial dq are summed at the end.
-__global__ void __launch_bounds__(64) k_flow_attn_bwd_q(
+// Query-row prologue of the backward: q (and dO as bf16) into shared tiles,
+// D_c = dO_c . o_c (fp32) and the forward's lse per row; rows past C get
+// D = 0, lse = +inf (so their probabilities are 0).
+__device__ __forceinline__ void bwd_query_side(uint32_t sq, uint8_t* sg_gen, float* sD, float* sL,
+                                               const uint16_t* qkv, const uint16_t* o,
+                                               const float* dO, const float* lse, int act0, int C,
+                                               int rows, int dm, int nh, int h) {
+    load_rows(sq, qkv + (size_t)act0 * 3 * dm + h * kHd, 3 * dm, C, rows);
+    cp_async_commit();
+    store_rows_bf16(sg_gen, dO + (size_t)act0 * dm + h * kHd, dm, C, rows);
+    for (int c = threadIdx.x; c < rows; c += blockDim.x) {
+        float Dc = 0.f, lc = INFINITY;
+        if (c < C) {
+            const size_t r = (size_t)(act0 + c);
+            const float* gr = dO + r * dm + h * kHd;
+            const uint16_t* orow = o + r * dm + h * kHd;
+            for (int e = 0; e < kHd; ++e) Dc += gr[e] * bf2f(orow[e]);
+            lc = lse[r * nh + h];
+        }
+        sD[c] = Dc;
+        sL[c] = lc;
+    }
+    cp_async_wait<0>();
+    __syncthreads();
+}
+
+// Backward, query side: dq_c = scale sum_j dS_cj k_j, dS = P (dP - D_c),
+// dP_cj = dO_c . v_j, P from the forward's lse.  Warps split as the forward
+// (query tile, key slice); the KS partial dq are summed in slice order.
+template <int KS>
+__global__ void __launch_bounds__(128) k_flow_attn_bwd_q(
     const uint16_t* __restrict__ qkv, const uint16_t* __restrict__ kvc, const int* __restrict__ cu,
     FlowDims dd, const uint16_t* __restrict__ o, const float* __restrict__ dO,
     const float* __restrict__ lse, uint16_t* __restrict__ dqkv) {
-    __shared__ float sk[kKT][kHd + 1], sv[kKT][kHd + 1];
-    __shared__ float sq[64][kHd + 1];  // each thread's own (scaled) query row, then its dq
+    constexpr int NK = kKT / KS, NT = NK / 8;
+    __shared__ __align__(128) uint8_t sbuf[4 * kTileB];
+    __shared__ float sD[kMaxC], sL[kMaxC];
     const int s = blockIdx.x, h = blockIdx.y, C = dd.C, dm = dd.dm;
-    const int KS = min(8, 64 / C);  // key splits per query
-    const int c = threadIdx.x % C, ks = threadIdx.x / C;
-    const int ctx0 = cu[s], L = cu[s + 1] - ctx0, act0 = s * C;
-    const float sc = 1.f / sqrtf((float)kHd);
-    float g[kHd], dq[kHd];
-    float Dc = 0.f, lc = 0.f;
-    const bool act = ks < KS;
-    float* q = sq[threadIdx.x];
-    if (act) {
-        const size_t r = (size_t)(act0 + c);
-        const uint16_t* qr = qkv + r * 3 * dm + h * kHd;
-        const uint16_t* orow = o + r * dm + h * kHd;
-        const float* gr = dO + r * dm + h * kHd;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, tq = lane & 3;
+    const int MT = (C + 15) >> 4, mt = warp / KS, ks = warp % KS;
+    const bool active = mt < MT;
+    const int ctx0 = cu[s], L = cu[s + 1] - ctx0, act0 = s * C, nkeys = L + C;
+    const uint32_t sb = smem_u32(sbuf);
+    bwd_query_side(sb, sbuf + kTileB, sD, sL, qkv, o, dO, lse, act0, C, MT * 16, dm, dd.nh, h);
+    uint32_t qa[4][4], ga[4][4];
+    float lr[2] = {0.f, 0.f}, Dr[2] = {0.f, 0.f};
+    if (active) {
 #pragma unroll
-        for (int e = 0; e < kHd; ++e) {
-            q[e] = bf2f(qr[e]) * sc * kLog2e;
-            g[e] = gr[e];
-            Dc += g[e] * bf2f(orow[e]);
-            dq[e] = 0.f;
+        for (int kk = 0; kk < 4; ++kk) {
+            ld_a(sb, mt * 16, kk, lane, qa[kk]);
+            ld_a(sb + kTileB, mt * 16, kk, lane, ga[kk]);
         }
-        lc = lse[r * dd.nh + h];
-    }
-    const int nkeys = L + C;
-    for (int j0 = 0; j0 < nkeys; j0 += kKT) {
-        const int nk = min(kKT, nkeys - j0);
-        __syncthreads();
-        stage_keys(sk, sv, j0, nk, L, kvc, ctx0, qkv, act0, dm, h);
-        __syncthreads();
-        if (!act) continue;
-        for (int jj = ks; jj < nk; jj += KS) {
-            float a = 0.f, dp = 0.f;
 #pragma unroll
-            for (int e = 0; e < kHd; ++e) {
-                a += q[e] * sk[jj][e];
-                dp += g[e] * sv[jj][e];
-            }
-            const float ds = exp2f(a - lc) * (dp - Dc);
-#pragma unroll
-            for (int e = 0; e < kHd; ++e) dq[e] += ds * sk[jj][e];
+        for (int i = 0; i < 2; ++i) {
+            const int c = mt * 16 + g + 8 * i;
+            lr[i] = c < C ? sL[c] : 0.f;
+            Dr[i] = sD[c];
         }
-    }
-    __syncthreads();  // every thread is done with its query row: reuse it for dq
-    if (act) {
-#pragma unroll
-        for (int e = 0; e < kHd; ++e) q[e] = dq[e];
     }
     __syncthreads();
-    if (act && ks == 0) {
-        uint16_t* dr = dqkv + (size_t)(act0 + c) * 3 * dm + h * kHd;
-        for (int e = 0; e < kHd; e += 2) {
-            float v0 = 0.f, v1 = 0.f;
-            for (int k = 0; k < KS; ++k) {
-                v0 += sq[k * C + c][e];
-                v1 += sq[k * C + c][e + 1];
-            }
-            *reinterpret_cast<uint32_t*>(dr + e) = pack_bf2(v0 * sc, v1 * sc);
+    float dq[8][4];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) dq[i][0] = dq[i][1] = dq[i][2] = dq[i][3] = 0.f;
+    const float sc2 = kLog2e / sqrtf((float)kHd);
+    const int ntiles = (nkeys + kKT - 1) / kKT;
+    load_kv_tile(sb, sb + kTileB, 0, nkeys, L, kvc, ctx0, qkv, act0, dm, h);
+    cp_async_commit();
+    for (int t = 0; t < ntiles; ++t) {
+        const uint32_t kb = sb + (t & 1) * 2 * kTileB, vb = kb + kTileB;
+        if (t + 1 < ntiles) {
+            const uint32_t nk = sb + ((t + 1) & 1) * 2 * kTileB;
+            load_kv_tile(nk, nk + kTileB, (t + 1) * kKT, nkeys, L, kvc, ctx0, qkv, act0, dm, h);
         }
+        cp_async_commit();
+        cp_async_wait<1>();
+        __syncthreads();
+        if (active) {
+            float sacc[NT][4], dp[NT][4];
+#pragma unroll
+            for (int i = 0; i < NT; ++i)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) sacc[i][e] = dp[i][e] = 0.f;
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+#pragma unroll
+                for (int nb = 0; nb < NT / 2; ++nb) {
+                    uint32_t b[4];
+                    ld_b(kb, ks * NK + nb * 16, kk, lane, b);
+                    mma4(sacc[2 * nb], qa[kk], b[0], b[1]);
+                    mma4(sacc[2 * nb + 1], qa[kk], b[2], b[3]);
+                    ld_b(vb, ks * NK + nb * 16, kk, lane, b);
+                    mma4(dp[2 * nb], ga[kk], b[0], b[1]);
+                    mma4(dp[2 * nb + 1], ga[kk], b[2], b[3]);
+                }
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int j = t * kKT + ks * NK + nt * 8 + 2 * tq + (e & 1);
+                    const float p = j < nkeys ? exp2f(sacc[nt][e] * sc2 - lr[e >> 1]) : 0.f;
+                    sacc[nt][e] = p * (dp[nt][e] - Dr[e >> 1]);
+                }
+#pragma unroll
+            for (int k2 = 0; k2 < NK / 16; ++k2) {
+                uint32_t da[4];
+                acc_to_a(sacc[2 * k2], sacc[2 * k2 + 1], da);
+#pragma unroll
+                for (int dn = 0; dn < 4; ++dn) {
+                    uint32_t b[4];
+                    ld_bt(kb, ks * NK + k2 * 16, dn, lane, b);
+                    mma4(dq[2 * dn], da, b[0], b[1]);
+                    mma4(dq[2 * dn + 1], da, b[2], b[3]);
+                }
+            }
+        }
+        __syncthreads();
+    }
+    const float sc = 1.f / sqrtf((float)kHd);
+    if (KS == 1) {
+        if (!active) return;
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const int c = mt * 16 + g + 8 * i;
+            if (c >= C) continue;
+            uint16_t* dr = dqkv + (size_t)(act0 + c) * 3 * dm + h * kHd;
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt)
+                *reinterpret_cast<uint32_t*>(dr + nt * 8 + 2 * tq) =
+                    pack_bf2(dq[nt][2 * i] * sc, dq[nt][2 * i + 1] * sc);
+        }
+        return;
+    }
+    float* mo = reinterpret_cast<float*>(sbuf);  // [4][16][kHd + 1]
+    if (active) {
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            float* row = mo + (warp * 16 + g + 8 * i) * (kHd + 1);
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                row[nt * 8 + 2 * tq] = dq[nt][2 * i];
+                row[nt * 8 + 2 * tq + 1] = dq[nt][2 * i + 1];
+            }
+        }
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < MT * 16 * (kHd / 2); i += blockDim.x) {
+        const int r = i / (kHd / 2), e = 2 * (i % (kHd / 2));
+        if (r >= C) continue;
+        const int w0 = (r >> 4) * KS, rl = r & 15;
+        float v0 = 0.f, v1 = 0.f;
+#pragma unroll
+        for (int k = 0; k < KS; ++k) {
+            const float* row = mo + ((w0 + k) * 16 + rl) * (kHd + 1);
+            v0 += row[e];
+            v1 += row[e + 1];
+        }
+        *reinterpret_cast<uint32_t*>(dqkv + (size_t)(act0 + r) * 3 * dm + h * kHd + e) =
+            pack_bf2(v0 * sc, v1 * sc);
     }
 }
 
-// Backward, key side, one pass per gradient (DK: dk_j = scale sum_c dS_cj
-// q_c; otherwise dv_j = sum_c P_cj dO_c), so each thread keeps 64
-// accumulators.  One thread per key (context keys, then action keys); the
-// sample's query side for the head (q, dO, lse, D) in shared memory; each
-// thread's k_j (and v_j) in a padded shared row.
-template <bool DK>
+// Backward, key side: per key j, dv_j = sum_c P_cj dO_c and dk_j = scale
+// sum_c dS_cj q_c over the NQ x 16 (padded) queries.  One CTA of four warps
+// per (sample, head, key-tile stride): tiles blockIdx.z, blockIdx.z +
+// gridDim.z, ...; warp w owns keys 16 w .. 16 w + 15 of each tile.  Each key's
+// gradients are complete in one pass (no accumulation across CTAs).
+template <int NQ>
 __global__ void __launch_bounds__(128) k_flow_attn_bwd_kv(
     const uint16_t* __restrict__ qkv, const uint16_t* __restrict__ kvc, const int* __restrict__ cu,
     FlowDims dd, const uint16_t* __restrict__ o, const float* __restrict__ dO,
     const float* __restrict__ lse, uint16_t* __restrict__ dqkv, uint16_t* __restrict__ dkvc) {
-    extern __shared__ float fsm[];
-    float* sq = fsm;                      // [C][kHd + 1]
-    float* sg = sq + kMaxC * (kHd + 1);   // [C][kHd + 1]
-    float* sl = sg + kMaxC * (kHd + 1);   // [C]
-    float* sD = sl + kMaxC;               // [C]
-    float* skv = sD + kMaxC;              // [128][2 kHd + 1]
+    constexpr int NT = 2 * NQ;  // n8 query tiles
+    __shared__ __align__(128) uint8_t sbuf[4 * kTileB];  // q, dO, K, V
+    __shared__ float sD[kMaxC], sL[kMaxC];
     const int s = blockIdx.x, h = blockIdx.y, C = dd.C, dm = dd.dm;
-    const int ctx0 = cu[s], L = cu[s + 1] - ctx0, act0 = s * C;
-    const float sc = 1.f / sqrtf((float)kHd);
-    for (int i = threadIdx.x; i < C * kHd; i += blockDim.x) {
-        const int c = i / kHd, e = i % kHd;
-        const size_t r = (size_t)(act0 + c);
-        sq[c * (kHd + 1) + e] = bf2f(qkv[r * 3 * dm + h * kHd + e]) * sc * kLog2e;
-        sg[c * (kHd + 1) + e] = dO[r * dm + h * kHd + e];
-    }
-    __syncthreads();
-    if (threadIdx.x < C) {
-        const int c = threadIdx.x;
-        const size_t r = (size_t)(act0 + c);
-        float Dc = 0.f;
-        for (int e = 0; e < kHd; ++e) Dc += sg[c * (kHd + 1) + e] * bf2f(o[r * dm + h * kHd + e]);
-        sD[c] = Dc;
-        sl[c] = lse[r * dd.nh + h];
-    }
-    __syncthreads();
-    const int nkeys = L + C;
-    float* mykv = skv + threadIdx.x * (2 * kHd + 1);
-    for (int j = blockIdx.z * blockDim.x + threadIdx.x; j < nkeys; j += gridDim.z * blockDim.x) {
-        const uint16_t* kr;
-        if (j < L)
-            kr = kvc + (size_t)(ctx0 + j) * 2 * dm + h * kHd;
-        else
-            kr = qkv + (size_t)(act0 + j - L) * 3 * dm + dm + h * kHd;
-        const uint16_t* vr = kr + dm;
-        for (int e = 0; e < kHd; ++e) {
-            mykv[e] = bf2f(kr[e]);
-            if (DK) mykv[kHd + e] = bf2f(vr[e]);
-        }
-        float acc[kHd];
+    const int ctx0 = cu[s], L = cu[s + 1] - ctx0, act0 = s * C, nkeys = L + C;
+    const int ntiles = (nkeys + kKT - 1) / kKT;
+    if ((int)blockIdx.z >= ntiles) return;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, tq = lane & 3;
+    const uint32_t sq = smem_u32(sbuf), sg = sq + kTileB, kb = sq + 2 * kTileB, vb = kb + kTileB;
+    bwd_query_side(sq, sbuf + kTileB, sD, sL, qkv, o, dO, lse, act0, C, NQ * 16, dm, dd.nh, h);
+    const float sc2 = kLog2e / sqrtf((float)kHd), sc = 1.f / sqrtf((float)kHd);
+    for (int t = blockIdx.z; t < ntiles; t += gridDim.z) {
+        __syncthreads();  // the previous tile's readers are done
+        load_kv_tile(kb, vb, t * kKT, nkeys, L, kvc, ctx0, qkv, act0, dm, h);
+        cp_async_commit();
+        cp_async_wait<0>();
+        __syncthreads();
+        const int k0 = t * kKT + warp * 16;
+        if (k0 >= nkeys) continue;
+        float st[NT][4], dpt[NT][4];
 #pragma unroll
-        for (int e = 0; e < kHd; ++e) acc[e] = 0.f;
-        for (int c = 0; c < C; ++c) {
-            const float* qc = sq + c * (kHd + 1);
-            const float* gc = sg + c * (kHd + 1);
-            float a = 0.f;
+        for (int i = 0; i < NT; ++i)
 #pragma unroll
-            for (int e = 0; e < kHd; ++e) a += qc[e] * mykv[e];
-            const float p = exp2f(a - sl[c]);
-            if (DK) {
-                float dp = 0.f;
+            for (int e = 0; e < 4; ++e) st[i][e] = dpt[i][e] = 0.f;
 #pragma unroll
-                for (int e = 0; e < kHd; ++e) dp += gc[e] * mykv[kHd + e];
-                const float ds = p * (dp - sD[c]);
+        for (int kk = 0; kk < 4; ++kk) {
+            uint32_t ka[4], va[4];
+            ld_a(kb, warp * 16, kk, lane, ka);
+            ld_a(vb, warp * 16, kk, lane, va);
 #pragma unroll
-                for (int e = 0; e < kHd; ++e) acc[e] += ds * qc[e];
-            } else {
-#pragma unroll
-                for (int e = 0; e < kHd; ++e) acc[e] += p * gc[e];
+            for (int nb = 0; nb < NQ; ++nb) {
+                uint32_t b[4];
+                ld_b(sq, nb * 16, kk, lane, b);
+                mma4(st[2 * nb], ka, b[0], b[1]);
+                mma4(st[2 * nb + 1], ka, b[2], b[3]);
+                ld_b(sg, nb * 16, kk, lane, b);
+                mma4(dpt[2 * nb], va, b[0], b[1]);
+                mma4(dpt[2 * nb + 1], va, b[2], b[3]);
             }
         }
-        // (DK) the queries were scaled by sc log2e; dk needs sc alone
-        const float f = DK ? 1.f / kLog2e : 1.f;
-        uint16_t* dr;
-        if (j < L)
-            dr = dkvc + (size_t)(ctx0 + j) * 2 * dm + h * kHd + (DK ? 0 : dm);
-        else
-            dr = dqkv + (size_t)(act0 + j - L) * 3 * dm + dm + h * kHd + (DK ? 0 : dm);
+        // P^T and dS^T: rows are keys k0 + g (+ 8), columns queries
+        const bool kv0 = k0 + g < nkeys, kv1 = k0 + g + 8 < nkeys;
 #pragma unroll
-        for (int e = 0; e < kHd; e += 2)
-            *reinterpret_cast<uint32_t*>(dr + e) = pack_bf2(acc[e] * f, acc[e + 1] * f);
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int c = nt * 8 + 2 * tq + (e & 1);
+                const bool ok = (e >> 1) ? kv1 : kv0;
+                const float p = ok ? exp2f(st[nt][e] * sc2 - sL[c]) : 0.f;
+                st[nt][e] = p;
+                dpt[nt][e] = p * (dpt[nt][e] - sD[c]);
+            }
+        float dv[8][4], dk[8][4];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) dv[i][e] = dk[i][e] = 0.f;
+#pragma unroll
+        for (int kq = 0; kq < NQ; ++kq) {
+            uint32_t pa[4], da[4];
+            acc_to_a(st[2 * kq], st[2 * kq + 1], pa);
+            acc_to_a(dpt[2 * kq], dpt[2 * kq + 1], da);
+#pragma unroll
+            for (int dn = 0; dn < 4; ++dn) {
+                uint32_t b[4];
+                ld_bt(sg, kq * 16, dn, lane, b);
+                mma4(dv[2 * dn], pa, b[0], b[1]);
+                mma4(dv[2 * dn + 1], pa, b[2], b[3]);
+                ld_bt(sq, kq * 16, dn, lane, b);
+                mma4(dk[2 * dn], da, b[0], b[1]);
+                mma4(dk[2 * dn + 1], da, b[2], b[3]);
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const int j = k0 + g + 8 * i;
+            if (j >= nkeys) continue;
+            uint16_t* kr = j < L ? dkvc + (size_t)(ctx0 + j) * 2 * dm + h * kHd
+                                 : dqkv + (size_t)(act0 + j - L) * 3 * dm + dm + h * kHd;
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                *reinterpret_cast<uint32_t*>(kr + nt * 8 + 2 * tq) =
+                    pack_bf2(dk[nt][2 * i] * sc, dk[nt][2 * i + 1] * sc);
+                *reinterpret_cast<uint32_t*>(kr + dm + nt * 8 + 2 * tq) =
+                    pack_bf2(dv[nt][2 * i], dv[nt][2 * i + 1]);
+            }
+        }
     }
 }
 
@@ -420,12 +711,34 @@ __global__ void __launch_bounds__(256) k_flow_out(const uint16_t* __restrict__ n
     const int slot = sample_slot[r / C];
     const int t = fs.tenant[slot];
     const float nt = (float)(fs.s1[slot] - fs.s0[slot]) * C * D;
-    const uint16_t* x = nf + (size_t)r * dm;
+    // the row in registers: lane holds columns 8 lane + 256 i, i < dm / 256
+    float xr[4][8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        if (256 * i < dm) {
+            const uint4 q = *reinterpret_cast<const uint4*>(nf + (size_t)r * dm + 256 * i + 8 * lane);
+            const uint32_t w4[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                xr[i][2 * e] = __uint_as_float(w4[e] << 16);
+                xr[i][2 * e + 1] = __uint_as_float(w4[e] & 0xffff0000u);
+            }
+        }
     float sq = 0.f;
     for (int k = 0; k < D; ++k) {
-        const uint16_t* wr = w_out + ((size_t)t * D + k) * dm;
+        const uint16_t* wr = w_out + ((size_t)t * D + k) * dm + 8 * lane;
         float acc = 0.f;
-        for (int j = lane; j < dm; j += 32) acc += bf2f(x[j]) * bf2f(wr[j]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            if (256 * i < dm) {
+                const uint4 q = *reinterpret_cast<const uint4*>(wr + 256 * i);
+                const uint32_t w4[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    acc = fmaf(xr[i][2 * e], __uint_as_float(w4[e] << 16), acc);
+                    acc = fmaf(xr[i][2 * e + 1], __uint_as_float(w4[e] & 0xffff0000u), acc);
+                }
+            }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
         acc += bf2f(b_out[(size_t)t * D + k]);
@@ -548,30 +861,56 @@ __global__ void __launch_bounds__(256) k_flow_embed_wgrad(const float* __restric
     }
 }
 
-// dphi[s, j] = sum_c dh[s C + c, j]; then dz1[s, k] = (sum_j dphi[s, j]
-// T2[j, k]) SiLU'(z1[s, k]).  One CTA per sample.
-__global__ void __launch_bounds__(256) k_flow_time_bwd(const float* __restrict__ dh,
-                                                       const int* __restrict__ sample_slot,
+// dphi[s, j] = sum_c dh[s C + c, j] (the time embedding is added to every
+// action row of the sample), c in order.
+__global__ void __launch_bounds__(256) k_flow_dphi(const float* __restrict__ dh, FlowDims dd,
+                                                   float* __restrict__ dphi) {
+    const int s = blockIdx.x, dm = dd.dm, C = dd.C;
+    const int j = blockIdx.y * blockDim.x + threadIdx.x;
+    if (j >= dm) return;
+    float acc = 0.f;
+    for (int c = 0; c < C; ++c) acc += dh[((size_t)s * C + c) * dm + j];
+    dphi[(size_t)s * dm + j] = acc;
+}
+
+// dz1[s, k] = (sum_j dphi[s, j] T2[j, k]) SiLU'(z1[s, k]) over (sample, block
+// of 128 columns k).  Thread (jg, kq): 8 consecutive columns (one 16-byte load
+// per row), rows j = jg, jg + 16, ...; the 16 row groups are summed in order.
+__global__ void __launch_bounds__(256) k_flow_time_bwd(const int* __restrict__ sample_slot,
                                                        const __grid_constant__ FlowSlots fs,
                                                        FlowDims dd, const uint16_t* __restrict__ t2,
                                                        const float* __restrict__ z1,
-                                                       float* __restrict__ dphi,
+                                                       const float* __restrict__ dphi,
                                                        float* __restrict__ dz1) {
-    extern __shared__ float sh[];  // dphi [dm]
-    const int s = blockIdx.x, dm = dd.dm, C = dd.C;
+    extern __shared__ float sh[];  // dphi [dm], then partials [16][128]
+    const int s = blockIdx.x, dm = dd.dm, k0 = blockIdx.y * 128;
     const int t = fs.tenant[sample_slot[s]];
-    for (int j = threadIdx.x; j < dm; j += blockDim.x) {
-        float acc = 0.f;
-        for (int c = 0; c < C; ++c) acc += dh[((size_t)s * C + c) * dm + j];
-        sh[j] = acc;
-        dphi[(size_t)s * dm + j] = acc;
-    }
+    for (int j = threadIdx.x; j < dm; j += blockDim.x) sh[j] = dphi[(size_t)s * dm + j];
     __syncthreads();
-    const uint16_t* T2 = t2 + (size_t)t * dm * dm;
-    for (int k = threadIdx.x; k < dm; k += blockDim.x) {
-        float acc = 0.f;
-        for (int j = 0; j < dm; ++j) acc += sh[j] * bf2f(T2[(size_t)j * dm + k]);
-        dz1[(size_t)s * dm + k] = acc * silu_grad_f(z1[(size_t)s * dm + k]);
+    const int jg = threadIdx.x >> 4, kq = threadIdx.x & 15;
+    const uint16_t* T2 = t2 + (size_t)t * dm * dm + k0 + 8 * kq;
+    float acc[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+    for (int j = jg; j < dm; j += 16) {
+        const uint4 q = *reinterpret_cast<const uint4*>(T2 + (size_t)j * dm);
+        const uint32_t u[4] = {q.x, q.y, q.z, q.w};
+        const float g = sh[j];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            acc[2 * e] = fmaf(g, __uint_as_float(u[e] << 16), acc[2 * e]);
+            acc[2 * e + 1] = fmaf(g, __uint_as_float(u[e] & 0xffff0000u), acc[2 * e + 1]);
+        }
+    }
+    float* part = sh + dm;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) part[jg * 128 + 8 * kq + e] = acc[e];
+    __syncthreads();
+    if (threadIdx.x < 128) {
+        float v = 0.f;
+        for (int g = 0; g < 16; ++g) v += part[g * 128 + threadIdx.x];
+        const size_t o = (size_t)s * dm + k0 + threadIdx.x;
+        dz1[o] = v * silu_grad_f(z1[o]);
     }
 }
 
@@ -684,6 +1023,65 @@ FlowWs carve_flow(const FlowDims& d, int S, int N, void* base) {
     return w;
 }
 
+jnx_status last(const char* what) {
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Query tiles of 16 rows: one tile -> four key slices per tile of 64 keys,
+// two -> two, three or four -> one.
+jnx_status flow_attn_fwd_launch(const uint16_t* qkv, const uint16_t* kvc, const int* cu,
+                                const FlowDims& d, uint16_t* o, float* lse, int S,
+                                cudaStream_t s) {
+    if (S == 0) return JNX_OK;
+    const int MT = (d.C + 15) / 16;
+    const dim3 grid(S, d.nh);
+    if (MT == 1)
+        k_flow_attn_fwd<4><<<grid, 128, 0, s>>>(qkv, kvc, cu, d, o, lse);
+    else if (MT == 2)
+        k_flow_attn_fwd<2><<<grid, 128, 0, s>>>(qkv, kvc, cu, d, o, lse);
+    else
+        k_flow_attn_fwd<1><<<grid, 128, 0, s>>>(qkv, kvc, cu, d, o, lse);
+    return last("flow attention");
+}
+
+template <int NQ>
+void launch_bwd_kv(dim3 grid, const uint16_t* qkv, const uint16_t* kvc, const int* cu,
+                   const FlowDims& d, const uint16_t* o, const float* dO, const float* lse,
+                   uint16_t* dqkv, uint16_t* dkvc, cudaStream_t s) {
+    k_flow_attn_bwd_kv<NQ><<<grid, 128, 0, s>>>(qkv, kvc, cu, d, o, dO, lse, dqkv, dkvc);
+}
+
+// dq (query side), then dk / dv (key side: one CTA per sample, head and
+// key tile up to 16 tiles, striding beyond).
+jnx_status flow_attn_bwd_launch(const uint16_t* qkv, const uint16_t* kvc, const jnx_group* g,
+                                const FlowDims& d, const uint16_t* o, const float* dO,
+                                const float* lse, uint16_t* dqkv, uint16_t* dkvc,
+                                cudaStream_t s) {
+    const int S = g->n_samples;
+    if (S == 0) return JNX_OK;
+    const int MT = (d.C + 15) / 16;
+    const int* cu = g->cu_seqlens;
+    const dim3 grid(S, d.nh);
+    if (MT == 1)
+        k_flow_attn_bwd_q<4><<<grid, 128, 0, s>>>(qkv, kvc, cu, d, o, dO, lse, dqkv);
+    else if (MT == 2)
+        k_flow_attn_bwd_q<2><<<grid, 128, 0, s>>>(qkv, kvc, cu, d, o, dO, lse, dqkv);
+    else
+        k_flow_attn_bwd_q<1><<<grid, 128, 0, s>>>(qkv, kvc, cu, d, o, dO, lse, dqkv);
+    int tiles = 1;
+    for (int i = 0; i < S; ++i)
+        tiles = std::max(tiles, (g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i] + d.C + kKT - 1) / kKT);
+    const dim3 gkv(S, d.nh, std::min(tiles, 16));
+    switch (MT) {
+        case 1: launch_bwd_kv<1>(gkv, qkv, kvc, cu, d, o, dO, lse, dqkv, dkvc, s); break;
+        case 2: launch_bwd_kv<2>(gkv, qkv, kvc, cu, d, o, dO, lse, dqkv, dkvc, s); break;
+        case 3: launch_bwd_kv<3>(gkv, qkv, kvc, cu, d, o, dO, lse, dqkv, dkvc, s); break;
+        default: launch_bwd_kv<4>(gkv, qkv, kvc, cu, d, o, dO, lse, dqkv, dkvc, s); break;
+    }
+    return last("flow attention backward");
+}
+
 jnx_status check_flow(const jnx_flow_head* fh, const jnx_group* g, FlowDims& d) {
     jnx_status st;
     if ((st = check_group(g))) return st;
@@ -713,6 +1111,9 @@ jnx_status check_flow(const jnx_flow_head* fh, const jnx_group* g, FlowDims& d) 
         if (!B.w_qkv || !B.w_kvc || !B.w_o || !B.w_gu || !B.w_d)
             return fail(JNX_ERR_INVALID_ARG, "flow: block %d has a null weight", b);
     }
+    if ((reinterpret_cast<uintptr_t>(fh->t1) | reinterpret_cast<uintptr_t>(fh->t2) |
+         reinterpret_cast<uintptr_t>(fh->w_out)) & 15)
+        return fail(JNX_ERR_INVALID_ARG, "flow: t1, t2 and w_out must be 16-byte aligned");
     if ((long long)g->n_samples * d.C > 0x7FFFFFFF)
         return fail(JNX_ERR_UNSUPPORTED, "flow: too many action rows");
     return JNX_OK;
@@ -744,11 +1145,6 @@ Segs make_segs(const jnx_group* g, int C) {
         sg.ten.push_back(g->h_slot_tenant[i]);
     }
     return sg;
-}
-
-jnx_status last(const char* what) {
-    cudaError_t e = cudaGetLastError();
-    return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
 __global__ void k_fill_bf16(uint16_t* p, int n, uint16_t v) {
@@ -820,8 +1216,7 @@ jnx_status flow_network(const jnx_flow_head* fh, const FlowDims& d, const jnx_gr
             for (int i = 0; i < S; ++i)
                 fl += 4.0 * d.C * (double)(g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i] + d.C) * dm;
             TraceScope ts(JNX_K_FLOW_ATTN, fl, s);
-            k_flow_attn_fwd<<<dim3(S, d.nh), 64, 0, s>>>(qkv, kvc, g->cu_seqlens, d, o, lse);
-            if ((st = last("flow attention"))) return st;
+            if ((st = flow_attn_fwd_launch(qkv, kvc, g->cu_seqlens, d, o, lse, S, s))) return st;
         }
         p = GemmParams{};
         p.M = Ma;
@@ -907,6 +1302,8 @@ static jnx_status flow_begin(const jnx_flow_head* fh, const jnx_group* g, const 
     if ((st = check_flow(fh, g, d))) return st;
     if (!workspace || (g->n_tokens > 0 && !hidden))
         return fail(JNX_ERR_INVALID_ARG, "flow: null workspace or hidden rows");
+    if (reinterpret_cast<uintptr_t>(workspace) & 255)
+        return fail(JNX_ERR_INVALID_ARG, "flow: workspace must be 256-byte aligned");
     w = carve_flow(d, g->n_samples, g->n_tokens, workspace);
     if (ws_bytes < w.bytes)
         return fail(JNX_ERR_WORKSPACE, "flow: workspace %zu < %zu bytes", ws_bytes, w.bytes);
@@ -921,9 +1318,11 @@ static jnx_status flow_embed(const jnx_flow_head* fh, const FlowDims& d, const j
     const int S = g->n_samples, Ma = S * d.C;
     TraceScope ts(JNX_K_FLOW_MISC, (double)S * d.dm * d.dm * 4.0, s);
     k_fill_bf16<<<(d.dm + 255) / 256, 256, 0, s>>>(w.ones, d.dm, (uint16_t)0x3F80);
-    k_flow_time<<<S, 256, 2 * d.dm * sizeof(float), s>>>(tau, g->sample_slot, fs, d, fh->t1,
-                                                         fh->tb1, fh->t2, fh->tb2, w.sfeat, w.z1,
-                                                         w.phi);
+    const dim3 tg(S, d.dm / kTimeRows);
+    k_flow_time1<<<tg, 256, d.dm * sizeof(float), s>>>(tau, g->sample_slot, fs, d, fh->t1, fh->tb1,
+                                                       w.sfeat, w.z1);
+    k_flow_time2<<<tg, 256, d.dm * sizeof(float), s>>>(g->sample_slot, fs, d, fh->t2, fh->tb2,
+                                                       w.z1, w.phi);
     k_flow_embed<<<Ma, 256, 0, s>>>(actions, noise, tau, xin, g->sample_slot, fs, d, fh->w_in,
                                     fh->b_in, fh->pos, w.phi, w.x, w.u, w.h);
     return last("flow embedding");
@@ -1134,26 +1533,8 @@ extern "C" jnx_status jnx_flow_backward(const jnx_flow_head* fh, const jnx_group
             for (int i = 0; i < S; ++i)
                 fl += 8.0 * d.C * (double)(g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i] + d.C) * dm;
             TraceScope ts(JNX_K_FLOW_ATTN, fl, s);
-            k_flow_attn_bwd_q<<<dim3(S, d.nh), 64, 0, s>>>(qkv, kvc, g->cu_seqlens, d, o, w.dO,
-                                                           lse, w.dqkv);
-            const size_t smem = (size_t)(2 * kMaxC * (kHd + 1) + 2 * kMaxC + 128 * (2 * kHd + 1)) *
-                                sizeof(float);
-            static bool attr = false;
-            if (!attr) {
-                if (cudaFuncSetAttribute(k_flow_attn_bwd_kv<true>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem) != cudaSuccess ||
-                    cudaFuncSetAttribute(k_flow_attn_bwd_kv<false>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem) != cudaSuccess)
-                    return last("flow: smem attribute");
-                attr = true;
-            }
-            k_flow_attn_bwd_kv<true><<<dim3(S, d.nh, 4), 128, smem, s>>>(
-                qkv, kvc, g->cu_seqlens, d, o, w.dO, lse, w.dqkv, w.dkvc);
-            k_flow_attn_bwd_kv<false><<<dim3(S, d.nh, 4), 128, smem, s>>>(
-                qkv, kvc, g->cu_seqlens, d, o, w.dO, lse, w.dqkv, w.dkvc);
-            if ((st = last("flow attention backward"))) return st;
+            if ((st = flow_attn_bwd_launch(qkv, kvc, g, d, o, w.dO, lse, w.dqkv, w.dkvc, s)))
+                return st;
         }
         {
             TraceScope ts(JNX_K_FLOW_WGRAD,
@@ -1189,8 +1570,9 @@ extern "C" jnx_status jnx_flow_backward(const jnx_flow_head* fh, const jnx_group
     TraceScope ts(JNX_K_FLOW_MISC, (double)Ma * dm * 8.0 + (double)S * dm * dm * 8.0, s);
     k_flow_embed_wgrad<<<dim3(nsl, (dm + 255) / 256), 256, 0, s>>>(w.dh, w.x, fs, d, gr->w_in,
                                                                     gr->b_in, gr->pos, add);
-    k_flow_time_bwd<<<S, 256, dm * sizeof(float), s>>>(w.dh, g->sample_slot, fs, d, fh->t2, w.z1,
-                                                       w.dphi, w.dz1);
+    k_flow_dphi<<<dim3(S, (dm + 255) / 256), 256, 0, s>>>(w.dh, d, w.dphi);
+    k_flow_time_bwd<<<dim3(S, dm / 128), 256, (dm + 16 * 128) * sizeof(float), s>>>(
+        g->sample_slot, fs, d, fh->t2, w.z1, w.dphi, w.dz1);
     k_flow_outer<true><<<dim3(nsl, dm), 256, 0, s>>>(w.dphi, w.z1, fs, d, gr->t2, gr->tb2, add);
     k_flow_outer<false><<<dim3(nsl, dm), 256, 0, s>>>(w.dz1, w.sfeat, fs, d, gr->t1, gr->tb1, add);
     return last("flow embedding backward");
