@@ -566,13 +566,10 @@ static jnx_status launch_attn_ws(const uint16_t* qkv, int ldq, int n_tokens, int
                                  int n_items, uint16_t* out, int ldo, float* lse, int* status,
                                  cudaStream_t s) {
     using C = AttnWsCfg<HD, BN>;
-    static bool attr = false;
-    if (!attr) {
-        if (cudaFuncSetAttribute(k_attn_ws<HD, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 C::SMEM) != cudaSuccess)
-            return fail(JNX_ERR_CUDA, "attention: smem attribute");
-        attr = true;
-    }
+    static std::atomic<uint64_t> attr{0};
+    if (set_smem_limit(reinterpret_cast<const void*>(k_attn_ws<HD, BN>), C::SMEM, attr) !=
+        cudaSuccess)
+        return fail(JNX_ERR_CUDA, "attention: smem attribute");
     CUtensorMap tq, tkv;
     if (!make_tmap_bf16(&tq, qkv, n_tokens, ldq, ldq, C::BM, 64) ||
         !make_tmap_bf16(&tkv, qkv, n_tokens, ldq, ldq, BN, 64))

@@ -524,13 +524,10 @@ static jnx_status launch_bwd(const CUtensorMap (&maps)[4], const int* cu, const 
                              const float2* rope, int rope_ld, uint16_t* dqkv, int ldq, int* status,
                              cudaStream_t s) {
     using C = AttnBwdCfg<HD, MODE>;
-    static bool attr = false;
-    if (!attr) {
-        if (cudaFuncSetAttribute(k_attn_bwd<HD, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 C::SMEM) != cudaSuccess)
-            return fail(JNX_ERR_CUDA, "attention backward: smem attribute");
-        attr = true;
-    }
+    static std::atomic<uint64_t> attr{0};
+    if (set_smem_limit(reinterpret_cast<const void*>(k_attn_bwd<HD, MODE>), C::SMEM, attr) !=
+        cudaSuccess)
+        return fail(JNX_ERR_CUDA, "attention backward: smem attribute");
     const int HP = MODE == abwd::DQ ? H : Hkv;
     const long long n_work = (long long)it.n * HP;
     if (n_work > 0x7FFFFFFFLL) return fail(JNX_ERR_UNSUPPORTED, "attention backward: too many items");

@@ -838,6 +838,17 @@ int num_sms() {
     return n > 0 ? n : 1;
 }
 
+cudaError_t set_smem_limit(const void* fn, int bytes, std::atomic<uint64_t>& done) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = dev < 64 ? 1ull << dev : 0ull;
+    if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) done.fetch_or(bit, std::memory_order_acq_rel);
+    return e;
+}
+
 template <int EPI, bool LORA, class LG, int EW = 4>
 static cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const LG& lg,
                               const GemmParams& p, int grid, cudaStream_t s) {
@@ -847,13 +858,9 @@ static cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, cons
                   "eight epilogue warps: column-splittable epilogues without LoRA only");
     constexpr int smem = LORA ? gemm::SMEM_BYTES_LORA
                               : (EW == 8 ? gemm::SMEM_BYTES_EW8 : gemm::SMEM_BYTES);
-    static bool attr_done = false;  // per instantiation; idempotent if raced
-    if (!attr_done) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm<EPI, LORA, EW>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e != cudaSuccess) return e;
-        attr_done = true;
-    }
+    static std::atomic<uint64_t> attr{0};  // per instantiation, one bit per device
+    cudaError_t e = set_smem_limit(reinterpret_cast<const void*>(k_gemm<EPI, LORA, EW>), smem, attr);
+    if (e != cudaSuccess) return e;
     k_gemm<EPI, LORA, EW><<<grid, 64 + 32 * EW, smem, s>>>(ta, tb, lg, p);
     return cudaGetLastError();
 }

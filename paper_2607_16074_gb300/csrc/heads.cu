@@ -21,6 +21,7 @@
 // so a tenant's results are identical whether it runs grouped or alone.
 #include "jnx_dev.cuh"
 #include "jnx_heads.h"
+#include "jnx_kernels.h"
 
 namespace jnx {
 
@@ -636,15 +637,11 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
 }
 
 jnx_status heads_set_smem() {
-    static bool done = false;
-    if (done) return JNX_OK;
+    static std::atomic<uint64_t> fwd{0}, bwd{0};
     const int mx = 2 * kMaxQ * 512 * (int)sizeof(float);
-    if (cudaFuncSetAttribute(k_xattn_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, mx) !=
-            cudaSuccess ||
-        cudaFuncSetAttribute(k_xattn_bwd, cudaFuncAttributeMaxDynamicSharedMemorySize, mx) !=
-            cudaSuccess)
+    if (set_smem_limit(reinterpret_cast<const void*>(k_xattn_fwd), mx, fwd) != cudaSuccess ||
+        set_smem_limit(reinterpret_cast<const void*>(k_xattn_bwd), mx, bwd) != cudaSuccess)
         return cuda_ok("heads smem attribute");
-    done = true;
     return JNX_OK;
 }
 

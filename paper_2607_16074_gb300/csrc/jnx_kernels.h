@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <vector>
 
 #include "jnx_host.h"
@@ -123,6 +124,11 @@ bool make_tmap_bf16(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t col
                     uint64_t row_stride_elems, uint32_t box_rows, uint32_t box_cols,
                     int swizzle_bytes = 128);
 int num_sms();
+
+// Raise fn's dynamic shared-memory limit to `bytes` on the current device,
+// once per device (the attribute is per device; `done` holds one bit per
+// device ordinal < 64, and callers that race both set it, which is harmless).
+cudaError_t set_smem_limit(const void* fn, int bytes, std::atomic<uint64_t>& done);
 
 // Packer: x[N, d] fp32 = widened gather of vision rows / text-embedding rows.
 jnx_status pack_launch(const jnx_group* g, const uint16_t* vision, int64_t n_vision,

@@ -213,3 +213,18 @@ def test_flow_rejects_bad_dimensions():
     loss = torch.zeros(3, device="cuda")
     with pytest.raises(J.JnxError):
         s.heads.forward(g, hidden, inp["actions"], inp["noise"], inp["tau"], vel, loss, ws)
+
+
+def test_flow_rejects_misaligned_workspace():
+    s = FlowSetup()
+    plan = s.plan()
+    g = R.DeviceGroup(plan)
+    hidden = torch.zeros(plan.n_tokens, 256, dtype=torch.bfloat16, device="cuda")
+    ws = torch.zeros(max(s.heads.workspace_bytes(g), 256) + 512, dtype=torch.uint8, device="cuda")
+    inp = _inputs(plan, s.C, s.D)
+    vel = torch.full((plan.n_samples, s.C, s.D), -3.0, device="cuda")
+    loss = torch.full((3,), -3.0, device="cuda")
+    with pytest.raises(J.JnxError, match="aligned"):
+        s.heads.forward(g, hidden, inp["actions"], inp["noise"], inp["tau"], vel, loss, ws[16:])
+    torch.cuda.synchronize()
+    assert torch.all(vel == -3.0) and torch.all(loss == -3.0)  # rejected before any launch
