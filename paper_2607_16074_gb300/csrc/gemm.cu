@@ -198,7 +198,9 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
         float* dst = EPI == EPI_RESID ? p.resid : static_cast<float*>(p.out);
         const int ld = EPI == EPI_RESID ? p.ldr : p.ldo;
         float4 xr[RD][4];
-        auto load_resid = [&](int pass, float4 (&x)[4]) {
+        uint2 gr[RD];  // folded norm: this lane's four gamma values of each pass
+        const bool norm = EPI == EPI_RESID && p.norm_gamma != nullptr;
+        auto load_resid = [&](int pass, float4 (&x)[4], uint2& gq) {
             const int col = n0 + pass * 16 + (lane & 3) * 4;
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
@@ -208,17 +210,17 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                 x[i] = make_float4(__uint_as_float(u.x), __uint_as_float(u.y),
                                    __uint_as_float(u.z), __uint_as_float(u.w));
             }
+            if (norm) gq = *reinterpret_cast<const uint2*>(p.norm_gamma + col);
         };
         constexpr int NP = 2 * NC;  // staging passes of this warp
         const int pb = 2 * cb;
         if constexpr (EPI == EPI_RESID) {
 #pragma unroll
-            for (int q = 0; q < RD - 1; ++q) load_resid(pb + q, xr[q]);
+            for (int q = 0; q < RD - 1; ++q) load_resid(pb + q, xr[q], gr[q]);
         }
         // folded RMSNorm (EPI_RESID with norm_gamma): y = bf16(x * gamma) and
         // the sums of x^2 of each of this lane's four rows over its columns,
         // one per 128-column half of the tile (8 staging passes each)
-        const bool norm = EPI == EPI_RESID && p.norm_gamma != nullptr;
         float ssq[NC / 4][4] = {};
 #pragma unroll
         for (int lc = 0; lc < NC; ++lc) {
@@ -231,7 +233,8 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                 const int lp = 2 * lc + h;  // pass within this warp's range
                 const int pass = pb + lp;
                 if constexpr (EPI == EPI_RESID)
-                    if (lp + RD - 1 < NP) load_resid(pass + RD - 1, xr[(lp + RD - 1) % RD]);
+                    if (lp + RD - 1 < NP)
+                        load_resid(pass + RD - 1, xr[(lp + RD - 1) % RD], gr[(lp + RD - 1) % RD]);
                 uint4 v[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u)
@@ -240,6 +243,14 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                 stg_put(stg, lane, v);
                 __syncwarp();
                 const int col = n0 + pass * 16 + (lane & 3) * 4;
+                float gf[4] = {0.f, 0.f, 0.f, 0.f};
+                if (EPI == EPI_RESID && norm) {
+                    const uint2 g = gr[lp % RD];
+                    gf[0] = bf2f(g.x & 0xFFFF);
+                    gf[1] = bf2f(g.x >> 16);
+                    gf[2] = bf2f(g.y & 0xFFFF);
+                    gf[3] = bf2f(g.y >> 16);
+                }
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const uint4 w = stg_get(stg, lane, i);
@@ -259,12 +270,11 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                                                      __float_as_uint(o.z), __float_as_uint(o.w)),
                                           pol);
                     if (EPI == EPI_RESID && norm) {
-                        const uint2 g = *reinterpret_cast<const uint2*>(p.norm_gamma + col);
                         ssq[lp / 8][i] += o.x * o.x + o.y * o.y + o.z * o.z + o.w * o.w;
                         if (row < row_end)
                             *reinterpret_cast<uint2*>(p.norm_out + (size_t)row * p.N + col) =
-                                make_uint2(pack_bf2(o.x * bf2f(g.x & 0xFFFF), o.y * bf2f(g.x >> 16)),
-                                           pack_bf2(o.z * bf2f(g.y & 0xFFFF), o.w * bf2f(g.y >> 16)));
+                                make_uint2(pack_bf2(o.x * gf[0], o.y * gf[1]),
+                                           pack_bf2(o.z * gf[2], o.w * gf[3]));
                     }
                 }
                 __syncwarp();
