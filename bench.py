@@ -54,7 +54,7 @@ def workload_desc(w):
 # command are in profiles/), valid only for the GEMM source it was taken on.
 RECORDED_TRAFFIC = {
     # workload: (sha256 of csrc/gemm.cu, bytes per launch, profile)
-    "llama7b": ("c51437a803d1cb100b10081d1d06002dc8f3bc9a80e54031f9ca5b791ce0992f",
+    "llama7b": ("0e15caa660f37ae152e2b9071dce9f78b138a1c38379d3eaf71d7cebbc59e7bd",
                 3.09e9 + 1.44e9, "profiles/gemm_gate_up_glu_llama7b_dram.md"),
 }
 
