@@ -51,11 +51,13 @@ def workload_desc(w):
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one gate/up
 # GEMM launch from an ncu capture of the full-size benchmark (the summary and
-# command are in profiles/), valid only for the GEMM source it was taken on.
+# command are in profiles/), valid only for the GEMM source it was taken on
+# and the launch shape it was taken at (packed rows, width, FFN width).
 RECORDED_TRAFFIC = {
-    # workload: (sha256 of csrc/gemm.cu, bytes per launch, profile)
+    # workload: (sha256 of csrc/gemm.cu, (rows, d, F), bytes per launch, profile)
     "llama7b": ("0e15caa660f37ae152e2b9071dce9f78b138a1c38379d3eaf71d7cebbc59e7bd",
-                3.09e9 + 1.44e9, "profiles/gemm_gate_up_glu_llama7b_dram.md"),
+                (65817, 4096, 11008), 3.09e9 + 1.44e9,
+                "profiles/gemm_gate_up_glu_llama7b_dram.md"),
 }
 
 
@@ -66,11 +68,13 @@ def gemm_source_hash() -> str:
         return hashlib.sha256(f.read()).hexdigest()
 
 
-def recorded_traffic(workload: str):
+def recorded_traffic(workload: str, shape):
+    """The recorded traffic of the gate/up launch, or None when the GEMM
+    source or the launch shape (rows, d, F) differs from the capture's."""
     rec = RECORDED_TRAFFIC.get(workload)
-    if not rec or rec[0] != gemm_source_hash():
+    if not rec or rec[0] != gemm_source_hash() or tuple(rec[1]) != tuple(shape):
         return None
-    return dict(bytes_per_launch=rec[1], source=rec[2])
+    return dict(bytes_per_launch=rec[2], source=rec[3])
 
 
 def gu_algorithmic_bytes(w, n_tokens: int) -> int:
@@ -483,7 +487,7 @@ def run_ours(args, rank, world, local_rank):
     gu_n = int(gu.sum())
     gu_flops, gu_ms = float(work[gu].sum()), float(ms[gu].sum())
     gu_tf = gu_flops / (gu_ms / 1e3) / 1e12 if gu_ms > 0 else 0.0
-    tr = recorded_traffic(w.name)
+    tr = recorded_traffic(w.name, (plan.n_tokens, w.backbone.d, w.backbone.d_ff))
     roofline = dict(kernel="k_gemm<EPI_GLU> (tcgen05): gate/up projection + SwiGLU/GeGLU",
                     bound="tensor", achieved=round(gu_tf, 1), peak=peaks["bf16_sustained"],
                     unit="TFLOP/s", frac=round(gu_tf / peaks["bf16_sustained"], 4),
@@ -496,7 +500,7 @@ def run_ours(args, rank, world, local_rank):
                     traffic=tr["bytes_per_launch"] if tr else None,
                     algorithmic_bytes_per_launch=gu_algorithmic_bytes(w, plan.n_tokens),
                     traffic_source=tr["source"] if tr else
-                    "none recorded for this kernel source and workload")
+                    "none recorded for this kernel source and launch shape")
     roofline_all_gemm = dict(kernels="all backbone GEMM launches (QKV+RoPE, O+residual, "
                                      "gate/up+GLU, down+residual)",
                              achieved=round(g_tf, 1), unit="TFLOP/s",

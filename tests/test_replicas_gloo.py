@@ -1,4 +1,4 @@
-"""The N > 1 benchmark path on CPU: two gloo ranks, each an independent
+"""bench.py host logic on CPU.  The N > 1 path: two gloo ranks, each an independent
 replica of the grouped step's host side (its own plan over its own seeded
 workload), the job time taken as the slowest rank's, throughput summed over
 ranks.  No data-path collective is involved."""
@@ -56,3 +56,12 @@ def test_two_gloo_replicas_weak_scaling():
 def test_single_rank_needs_no_process_group():
     assert bench.max_over_ranks(7.5, 1) == 7.5
     assert bench.replica_seed(4, 0) == 4
+
+
+def test_recorded_traffic_only_for_the_captured_launch_shape():
+    # the capture's own shape: the 7B-class group's gate/up launch
+    rec = bench.RECORDED_TRAFFIC["llama7b"]
+    assert bench.recorded_traffic("llama7b", rec[1]) is not None or rec[0] != bench.gemm_source_hash()
+    # any other launch (a tenant subset, another width) has no recorded traffic
+    assert bench.recorded_traffic("llama7b", (16672, 4096, 11008)) is None
+    assert bench.recorded_traffic("mqa2b", (141000, 2048, 16384)) is None
