@@ -680,6 +680,28 @@ def run_kernel(args):
                 times_ms=[round(t, 4) for t in times])
 
 
+# The flow-expert bench's expert: width 1024, 4 blocks, SwiGLU 4096, chunk 16 x 32.
+FLOW_EXPERT = dict(d_model=1024, d_ff=4096, n_blocks=4, chunk=16, action_dim=32)
+
+
+def flow_workload(T: int, b: int):
+    """The flow bench's group on the 2B-class backbone: T tenants x b samples
+    of one 256-row image + 16..64 text tokens (seed 43); returns the workload
+    and the experts' dimensions (jnx_flow_head fields)."""
+    import synth
+    bb = synth.Backbone(n_layers=18, d=2048, n_heads=8, n_kv_heads=1, head_dim=256, d_ff=16384,
+                        glu=synth.GLU_GEGLU)
+    fe = FLOW_EXPERT
+    dims = dict(n_tenants=T, d_model=fe["d_model"], d_ff=fe["d_ff"], chunk=fe["chunk"],
+                action_dim=fe["action_dim"], d_in=bb.d)
+    tenants = [synth.Tenant(synth.HEAD_MLP, chunk=fe["chunk"], action_dim=fe["action_dim"],
+                            d_hidden=1024, max_images=1) for _ in range(T)]
+    rng = np.random.default_rng(43)
+    per = [[synth.Sample(1, int(rng.integers(16, 65))) for _ in range(b)] for _ in range(T)]
+    return synth.custom_workload(bb, tenants, per, req_batch=b, seed=43,
+                                 name=f"flow{T}x{b}"), dims
+
+
 def run_flow(args):
     """Flow-matching action experts (DiT heads) as the tenants' modules over
     the shared 2B-class backbone (18 blocks, d=2048, 8x256 query heads on
@@ -703,18 +725,12 @@ def run_flow(args):
     J.lib()
     dev = torch.device("cuda", 0)
     T, b = args.flow_tenants, args.flow_batch
-    bb = synth.Backbone(n_layers=18, d=2048, n_heads=8, n_kv_heads=1, head_dim=256, d_ff=16384,
-                        glu=synth.GLU_GEGLU)
-    dims = dict(n_tenants=T, d_model=1024, d_ff=4096, chunk=16, action_dim=32, d_in=bb.d)
-    tenants = [synth.Tenant(synth.HEAD_MLP, chunk=16, action_dim=32, d_hidden=1024, max_images=1)
-               for _ in range(T)]
-    rng = np.random.default_rng(43)
-    per = [[synth.Sample(1, int(rng.integers(16, 65))) for _ in range(b)] for _ in range(T)]
-    w = synth.custom_workload(bb, tenants, per, req_batch=b, seed=43, name=f"flow{T}x{b}")
+    w, dims = flow_workload(T, b)
+    bb = w.backbone
     bw = synth.make_backbone_weights(w, device=dev)
     backbone = R.DeviceBackbone(bb, bw, n_tenants=T)
-    fw = synth.make_flow_weights(T, dims["d_model"], dims["d_ff"], 4, dims["chunk"],
-                                 dims["action_dim"], bb.d, 43, device=dev)
+    fw = synth.make_flow_weights(T, dims["d_model"], dims["d_ff"], FLOW_EXPERT["n_blocks"],
+                                 dims["chunk"], dims["action_dim"], bb.d, 43, device=dev)
     experts = R.DeviceFlowHeads(dims, fw)
     opt = R.TenantAdamW(experts.param_pairs())  # each tenant's expert optimizer
     inp = synth.make_inputs(w, device=dev)
@@ -728,7 +744,8 @@ def run_flow(args):
                                      device=dev)
             self.ws_f = torch.zeros(experts.workspace_bytes(self.g), dtype=torch.uint8, device=dev)
             self.hidden = torch.zeros((plan.n_tokens, bb.d), dtype=torch.bfloat16, device=dev)
-            self.fi = synth.make_flow_inputs(plan.n_samples, 16, 32, 44, device=dev)
+            self.fi = synth.make_flow_inputs(plan.n_samples, dims["chunk"], dims["action_dim"], 44,
+                                             device=dev)
             self.vel = torch.zeros_like(self.fi["actions"])
             self.loss = torch.zeros(T, device=dev)
             self.tenants = sorted(set(plan.slot_tenant.tolist()))

@@ -29,16 +29,19 @@ def _rel_l2(got, ref):
 
 
 class FlowSetup:
-    def __init__(self, dm=256, F=256, nb=2, C=8, D=7, d=256, per=None, seed=3, std=0.05):
-        per = per or [[synth.Sample(1, 5), synth.Sample(0, 17)],
-                      [synth.Sample(2, 3)],
-                      [synth.Sample(0, 1), synth.Sample(1, 40), synth.Sample(0, 9)]]
-        bb = synth.Backbone(n_layers=0, d=d, n_heads=4, n_kv_heads=4, head_dim=64, d_ff=1024,
-                            vision_tokens=32, vocab=100)
-        tenants = [synth.Tenant(synth.HEAD_MLP, chunk=C, action_dim=D, d_hidden=64,
-                                max_images=2) for _ in per]
-        self.w = synth.custom_workload(bb, tenants, per, req_batch=1, seed=seed)
-        T = len(per)
+    def __init__(self, dm=256, F=256, nb=2, C=8, D=7, d=256, per=None, seed=3, std=0.05,
+                 workload=None):
+        if workload is None:
+            per = per or [[synth.Sample(1, 5), synth.Sample(0, 17)],
+                          [synth.Sample(2, 3)],
+                          [synth.Sample(0, 1), synth.Sample(1, 40), synth.Sample(0, 9)]]
+            bb = synth.Backbone(n_layers=0, d=d, n_heads=4, n_kv_heads=4, head_dim=64, d_ff=1024,
+                                vision_tokens=32, vocab=100)
+            tenants = [synth.Tenant(synth.HEAD_MLP, chunk=C, action_dim=D, d_hidden=64,
+                                    max_images=2) for _ in per]
+            workload = synth.custom_workload(bb, tenants, per, req_batch=1, seed=seed)
+        self.w = workload
+        T = len(self.w.tenants)
         self.dims = dict(n_tenants=T, d_model=dm, d_ff=F, chunk=C, action_dim=D, d_in=d)
         self.wt = synth.make_flow_weights(T, dm, F, nb, C, D, d, seed, device="cuda", std=std)
         self.heads = R.DeviceFlowHeads(self.dims, self.wt)
@@ -83,10 +86,12 @@ def _inputs(plan, C, D, seed=4):
     return inp
 
 
-def _check(s, plan, hidden, inp, vel, loss, tol):
+def _check(s, plan, hidden, inp, vel, loss, tol, only=None):
     H = f64(hidden)
     cu, seg = plan.cu_seqlens, plan.seg_offsets
     for gi, t in enumerate(plan.slot_tenant.tolist()):
+        if only is not None and t not in only:
+            continue
         ss = range(seg[gi], seg[gi + 1])
         ctx = [H[cu[i]:cu[i + 1]] for i in ss]
         acts = f64(inp["actions"][seg[gi]:seg[gi + 1]])
@@ -129,6 +134,27 @@ def test_flow_train_step_vs_oracle(dm, C, D):
     # block.  Measured relative L2 errors 1.2e-3 - 6.0e-3 over every
     # parameter, tenant and both sizes; a wrong term or index is off by O(1).
     _check(s, plan, hidden, inp, vel, loss, 3e-2)
+
+
+def test_flow_bench_size_sampled_tenant_vs_oracle():
+    """The launch configuration the flow bench times: 8 tenants x 4 samples
+    (one 256-row image + 16..64 text rows each) on 2048-wide context rows,
+    experts of width 1024, 4 blocks, SwiGLU 4096, chunk 16 x 32.  The whole
+    group runs; one seeded tenant's velocities, loss and every parameter
+    gradient are checked against the oracle."""
+    import bench
+    w, dims = bench.flow_workload(8, 4)
+    fe = bench.FLOW_EXPERT
+    s = FlowSetup(dm=fe["d_model"], F=fe["d_ff"], nb=fe["n_blocks"], C=fe["chunk"],
+                  D=fe["action_dim"], d=dims["d_in"], seed=43, std=0.02, workload=w)
+    plan = s.plan()
+    hidden = (torch.randn(plan.n_tokens, dims["d_in"], generator=torch.Generator().manual_seed(9))
+              .to(torch.bfloat16).cuda())
+    inp = synth.make_flow_inputs(plan.n_samples, s.C, s.D, 44, device="cuda")
+    g, vel, loss, ws = s.run(plan, hidden, inp)
+    assert torch.isfinite(vel).all() and torch.isfinite(loss[:8]).all()
+    t = int(np.random.default_rng(5).integers(8))
+    _check(s, plan, hidden, inp, vel, loss, 3e-2, only={t})
 
 
 def test_flow_sampling_vs_oracle():

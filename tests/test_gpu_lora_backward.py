@@ -315,6 +315,35 @@ def test_lora_grads_grouped_equal_isolated_and_other_slots_untouched():
             assert torch.all(v[0] == 7.0) and torch.all(v[2] == 7.0), (l, k)
 
 
+def test_lora_train_step_full_size_grouped_equals_isolated():
+    """The launch configuration the training bench times: the whole skewed
+    2B-class group (64 tenants, Zipf sample counts, 18 blocks, rank-16
+    adapters on Q/K/V/O).  The smallest tenant's feature gradient and every
+    adapter gradient in all 18 blocks are the same, bit for bit, grouped or
+    run alone (at this size the oracle cannot run the whole tenant; the
+    per-element checks run on one and two blocks above)."""
+    w = synth.make_workload("zipf2b")
+    counts = {t: sum(len(r.samples) for r in w.requests if r.tenant == t)
+              for t in range(len(w.tenants))}
+    t = min(counts, key=lambda k: (counts[k], k))
+    s = TrainSetup(w, gen_device="cuda")
+    plan, step = s.run()
+    gi = plan.slot_tenant.tolist().index(t)
+    cu, seg = plan.cu_seqlens, plan.seg_offsets
+    r0, r1 = int(cu[seg[gi]]), int(cu[seg[gi + 1]])
+    dh_group = step.d_hidden[r0:r1].clone()
+    assert torch.isfinite(step.d_hidden).all()
+    full = [{k: v[t].clone() for k, v in g.items()} for g in s.bb.lora_grads]
+    del step
+    torch.cuda.empty_cache()
+    _, step1 = s.run(w.subset([t]))
+    assert torch.equal(step1.d_hidden, dh_group)
+    for l, g in enumerate(s.bb.lora_grads):
+        for k, v in g.items():
+            assert torch.isfinite(full[l][k]).all(), (l, k)
+            assert torch.equal(v[t], full[l][k]), (l, k)
+
+
 def test_lora_grads_accumulate():
     w = _small_lora_workload(1, n_layers=1)
     s = TrainSetup(w, std=0.05)
