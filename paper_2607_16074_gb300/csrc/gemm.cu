@@ -88,24 +88,36 @@ __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int 
     nb = in / gm;
 }
 
-__device__ __forceinline__ float act_fn(float g, int act) {
-    if (act == JNX_GLU_SWIGLU) return g / (1.0f + expf(-g));
-    const float c = 0.7978845608028654f;  // sqrt(2/pi)
-    return 0.5f * g * (1.0f + tanhf(c * (g + 0.044715f * g * g * g)));
+// Both activations are g sigmoid(z): SiLU with z = g, and the tanh-form
+// GELU 0.5 g (1 + tanh(u)) with z = 2 u, u = sqrt(2/pi) (g + 0.044715 g^3),
+// since 0.5 (1 + tanh(u)) = sigmoid(2 u).  The sigmoid takes the fast
+// exponential and an approximate reciprocal (a few ulp, far below the bf16
+// rounding of every product that reads it); its limits are exact (an
+// overflowing exponential gives 0).
+__device__ __forceinline__ float sigmoid_fast(float z) {
+    return __fdividef(1.0f, 1.0f + __expf(-z));
+}
+__device__ __forceinline__ float gelu_arg(float g) {
+    return 1.5957691216057308f * (g + 0.044715f * g * g * g);  // 2 sqrt(2/pi) (g + a g^3)
 }
 
-// act(g) and its derivative: SiLU' = s (1 + g (1 - s)) with s = sigmoid(g);
-// for 0.5 g (1 + t), t = tanh(c (g + a g^3)): 0.5 (1 + t) + 0.5 g (1 - t^2) c (1 + 3 a g^2).
+__device__ __forceinline__ float act_fn(float g, int act) {
+    return g * sigmoid_fast(act == JNX_GLU_SWIGLU ? g : gelu_arg(g));
+}
+
+// act(g) and its derivative, s = sigmoid(z): SiLU' = s (1 + g (1 - s)); for
+// the GELU, with tanh(u) = 2 s - 1 and 1 - tanh(u)^2 = 4 s (1 - s),
+// d/dg [0.5 g (1 + tanh(u))] = s + 2 g s (1 - s) sqrt(2/pi) (1 + 3 a g^2).
 __device__ __forceinline__ void act_grad(float g, int act, float& a, float& da) {
     if (act == JNX_GLU_SWIGLU) {
-        const float s = 1.0f / (1.0f + expf(-g));
+        const float s = sigmoid_fast(g);
         a = g * s;
         da = s * (1.0f + g * (1.0f - s));
     } else {
-        const float c = 0.7978845608028654f;
-        const float t = tanhf(c * (g + 0.044715f * g * g * g));
-        a = 0.5f * g * (1.0f + t);
-        da = 0.5f * (1.0f + t) + 0.5f * g * (1.0f - t * t) * c * (1.0f + 3.0f * 0.044715f * g * g);
+        const float s = sigmoid_fast(gelu_arg(g));
+        a = g * s;
+        da = s + 2.0f * g * s * (1.0f - s) * 0.7978845608028654f *
+                     (1.0f + 3.0f * 0.044715f * g * g);
     }
 }
 
