@@ -55,8 +55,8 @@ def workload_desc(w):
 # and the launch shape it was taken at (packed rows, width, FFN width).
 RECORDED_TRAFFIC = {
     # workload: (sha256 of csrc/gemm.cu, (rows, d, F), bytes per launch, profile)
-    "llama7b": ("0e15caa660f37ae152e2b9071dce9f78b138a1c38379d3eaf71d7cebbc59e7bd",
-                (65817, 4096, 11008), 3.09e9 + 1.44e9,
+    "llama7b": ("5fd9e53974a1be9a3343dad5356d1f5639f680a646cd8383f40eafb3bdb628eb",
+                (65817, 4096, 11008), 3.07e9 + 1.44e9,
                 "profiles/gemm_gate_up_glu_llama7b_dram.md"),
 }
 
