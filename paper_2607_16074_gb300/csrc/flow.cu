@@ -10,7 +10,8 @@
 // rows times its slice of the stacked weights); weight gradients are
 // k_seg_wgrad (mma.sync, a tenant's rows in a fixed order); the attention
 // (C <= 64 queries per sample against its L context rows and C action rows)
-// and the small per-row / per-sample pieces run on CUDA cores in fp32.
+// runs on bf16 mma.sync tiles with fp32 softmax; the small per-row and
+// per-sample pieces run on CUDA cores in fp32.
 #include <algorithm>
 #include <cmath>
 #include <vector>
