@@ -413,7 +413,7 @@ struct HeadsWs {
 };
 
 struct HeadDims {
-    int ld_h = 8, ld_y = 8, ldkv = 256, nq = 4;
+    int ld_h = 8, ld_y = 8, ldkv = 256, nq = 4, d_in = 128;
     bool any_mlp = false, any_x = false;
 };
 
@@ -431,6 +431,7 @@ HeadDims head_dims(const jnx_head* heads, const jnx_group* g) {
             d.any_x = true;
             d.ldkv = std::max(d.ldkv, h.q_dim);
             d.nq = h.n_queries;
+            d.d_in = std::max(d.d_in, h.d_in);
         } else {
             d.any_mlp = true;
         }
@@ -469,6 +470,8 @@ HeadsWs carve_heads(const jnx_head* heads, const jnx_group* g, void* base) {
         w.sc.dS = take(N * hd.nq * 4);
         w.sc.dQs = take(S * hd.ld_h * 4);
         w.sc.dkv_bf = reinterpret_cast<uint16_t*>(take(N * 2 * hd.ldkv * 2));
+        w.sc.Gs = take(S * 32 * hd.d_in * 4);
+        w.sc.Hs = take(S * 32 * hd.d_in * 4);
     }
     w.bytes = off;
     return w;
@@ -488,6 +491,9 @@ jnx_status check_heads(const jnx_head* heads, int32_t n_tenants, const jnx_group
         const jnx_head& h = heads[t];
         if (h.width <= 0 || h.d_in <= 0 || h.d_in % 64)
             return fail(JNX_ERR_UNSUPPORTED, "heads: tenant %d needs width > 0, d_in %% 64 == 0", t);
+        if (h.d_in != heads[g->h_slot_tenant[0]].d_in)
+            return fail(JNX_ERR_UNSUPPORTED,
+                        "heads: the heads of one group read the same features (one d_in)");
         if (h.kind == JNX_HEAD_MLP) {
             if (h.d_hidden <= 0 || h.d_hidden % 8)
                 return fail(JNX_ERR_UNSUPPORTED, "heads: tenant %d d_hidden %% 8 != 0", t);
@@ -515,6 +521,18 @@ jnx_status check_heads(const jnx_head* heads, int32_t n_tenants, const jnx_group
                 return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null gradient buffer", t);
         } else {
             return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d unknown head kind %d", t, h.kind);
+        }
+        // weight rows are read, and the output layer's gradients written, with
+        // 16-byte accesses
+        auto a16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+        const uint16_t* w_out = h.kind == JNX_HEAD_MLP ? h.w2 : h.wout;
+        if (!a16(w_out) || (h.kind == JNX_HEAD_MLP && !a16(h.w1)))
+            return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d weights must be 16-byte aligned", t);
+        if (need_grads) {
+            const float* gw = h.kind == JNX_HEAD_MLP ? grads[t].w2 : grads[t].wout;
+            if (!a16(gw) || (h.kind == JNX_HEAD_XATTN && (!a16(grads[t].wk) || !a16(grads[t].wv))))
+                return fail(JNX_ERR_INVALID_ARG,
+                            "heads: tenant %d gradient buffers must be 16-byte aligned", t);
         }
         const int s0 = g->h_seg_offsets[i], s1 = g->h_seg_offsets[i + 1];
         if (s0 < 0 || s1 <= s0 || s1 > g->n_samples)
@@ -580,6 +598,7 @@ HeadBatch fill_table(HeadTable& tab, const jnx_head* heads, const jnx_head_grads
         }
         b.max_hid = std::max(b.max_hid, hs.hid);
         b.max_width = std::max(b.max_width, hs.width);
+        b.max_ns = std::max(b.max_ns, hs.s1 - hs.s0);
     }
     return b;
 }

@@ -55,64 +55,97 @@ __device__ __forceinline__ void bf8_to_f(const uint4 w, float (&f)[8]) {
 
 // ---------------------------------------------------------------------------
 // Segmented linear layer: out[s, j] = sum_k in[s, k] W[j, k] + b[j] over the
-// slot's samples.  One warp per output column j, 8 samples at a time; lanes
-// stride K in 8-element (16-byte) weight chunks.
+// slot's samples.  One CTA per (slot, 32 output columns, 8 samples): warp w
+// takes columns j0 + 4w .. j0 + 4w + 3, its lanes stride K in 8-element
+// (16-byte) weight chunks and keep 4 columns x 8 samples of partial sums;
+// the samples' input rows are staged 256 columns at a time in shared memory
+// (read once per CTA instead of once per column); each sum is closed by a
+// fixed butterfly over the lanes.
 //   LAYER 1: MLP first layer (W1, b1; in = pooled); stores z and h = SiLU(z).
 //   LAYER 2: output layer of either head (W2 or Wout; in = h); stores y and
 //            scatters it to the caller's predictions at each target offset.
 // ---------------------------------------------------------------------------
+constexpr int kLinCols = 32, kLinS = 8, kLinK = 256, kLinW = kLinCols / 8;  // columns per warp
+
 template <int LAYER>
-__global__ void __launch_bounds__(256) k_head_lin(const __grid_constant__ HeadTable tab,
+__global__ void __launch_bounds__(256, 2) k_head_lin(const __grid_constant__ HeadTable tab,
                                                   const float* __restrict__ in, int ld_in,
                                                   float* __restrict__ z_out, float* __restrict__ h_out,
                                                   int ld_out, const int* __restrict__ sample_target,
                                                   float* __restrict__ preds) {
+    __shared__ __align__(16) float sx[kLinS][kLinK];
     const HeadSlot& hs = tab.slot[blockIdx.x];
     if (LAYER == 1 && hs.kind != JNX_HEAD_MLP) return;
     const int J = LAYER == 1 ? hs.hid : hs.width;
     const int K = LAYER == 1 ? hs.d_in : hs.hid;
     const uint16_t* W = LAYER == 1 ? hs.w1 : hs.w2;
     const uint16_t* B = LAYER == 1 ? hs.b1 : hs.b2;
-    const int j = blockIdx.y * 8 + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
-    if (j >= J) return;
-    const uint4* wr = reinterpret_cast<const uint4*>(W + (size_t)j * K);
-    const float bj = bf2f(B[j]);
-    for (int s0 = hs.s0; s0 < hs.s1; s0 += 8) {
-        const int ns = min(8, hs.s1 - s0);
-        float acc[8];
+    const int j0 = blockIdx.y * kLinCols, s0 = hs.s0 + blockIdx.z * kLinS;
+    if (j0 >= J || s0 >= hs.s1) return;
+    const int ns = min(kLinS, hs.s1 - s0);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int jw = j0 + kLinW * warp;
+    float acc[kLinW][kLinS];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-        for (int c = lane; c < K / 8; c += 32) {
-            float wf[8];
-            bf8_to_f(__ldg(wr + c), wf);
+    for (int c = 0; c < kLinW; ++c)
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                if (i < ns) {
-                    const float4* xr =
-                        reinterpret_cast<const float4*>(in + (size_t)(s0 + i) * ld_in + c * 8);
-                    const float4 x0 = xr[0], x1 = xr[1];
-                    acc[i] += x0.x * wf[0] + x0.y * wf[1] + x0.z * wf[2] + x0.w * wf[3] +
-                              x1.x * wf[4] + x1.y * wf[5] + x1.z * wf[6] + x1.w * wf[7];
+        for (int i = 0; i < kLinS; ++i) acc[c][i] = 0.f;
+    for (int k0 = 0; k0 < K; k0 += kLinK) {
+        const int nk = min(kLinK, K - k0);  // a multiple of 8
+        __syncthreads();
+        for (int i = threadIdx.x; i < kLinS * (kLinK / 4); i += 256) {
+            const int r = i / (kLinK / 4), u = i % (kLinK / 4);
+            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (r < ns && 4 * u < nk)
+                v = *reinterpret_cast<const float4*>(in + (size_t)(s0 + r) * ld_in + k0 + 4 * u);
+            *reinterpret_cast<float4*>(&sx[r][4 * u]) = v;
+        }
+        __syncthreads();
+        if (8 * lane < nk) {
+            float x[kLinS][8];
+#pragma unroll
+            for (int i = 0; i < kLinS; ++i) {
+                const float4 a = *reinterpret_cast<const float4*>(&sx[i][8 * lane]);
+                const float4 c4 = *reinterpret_cast<const float4*>(&sx[i][8 * lane + 4]);
+                x[i][0] = a.x; x[i][1] = a.y; x[i][2] = a.z; x[i][3] = a.w;
+                x[i][4] = c4.x; x[i][5] = c4.y; x[i][6] = c4.z; x[i][7] = c4.w;
+            }
+#pragma unroll
+            for (int c = 0; c < kLinW; ++c) {
+                if (jw + c < J) {
+                    float wf[8];
+                    bf8_to_f(__ldg(reinterpret_cast<const uint4*>(W + (size_t)(jw + c) * K + k0) + lane),
+                             wf);
+#pragma unroll
+                    for (int i = 0; i < kLinS; ++i) {
+                        float t = acc[c][i];
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) t = fmaf(x[i][e], wf[e], t);
+                        acc[c][i] = t;
+                    }
                 }
             }
         }
-#pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = warp_sum_h(acc[i]);
-        if (lane < ns) {
-            float v = 0.f;
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-                if (i == lane) v = acc[i];
-            const int s = s0 + lane;
-            const float zz = v + bj;
-            z_out[(size_t)s * ld_out + j] = zz;
-            if (LAYER == 1)
-                h_out[(size_t)s * ld_out + j] = silu_f(zz);
-            else
-                preds[sample_target[s] + j] = zz;
-        }
     }
+#pragma unroll
+    for (int c = 0; c < kLinW; ++c)
+#pragma unroll
+        for (int i = 0; i < kLinS; ++i) acc[c][i] = warp_sum_h(acc[c][i]);
+#pragma unroll
+    for (int c = 0; c < kLinW; ++c)
+#pragma unroll
+        for (int i = 0; i < kLinS; ++i) {
+            const int j = jw + c;
+            if (lane == ((c * kLinS + i) & 31) && i < ns && j < J) {
+                const int s = s0 + i;
+                const float zz = acc[c][i] + bf2f(B[j]);
+                z_out[(size_t)s * ld_out + j] = zz;
+                if (LAYER == 1)
+                    h_out[(size_t)s * ld_out + j] = silu_f(zz);
+                else
+                    preds[sample_target[s] + j] = zz;
+            }
+        }
 }
 
 // Per-tenant loss and dy, one CTA per group slot, fixed-order reduction.
@@ -144,51 +177,130 @@ __global__ void __launch_bounds__(256) k_l2_loss(const __grid_constant__ HeadTab
 }
 
 // Output-layer weight gradient of either head: dW[o, j] = sum_s dy[s, o] h[s, j],
-// db[o] = sum_s dy[s, o].
+// db[o] = sum_s dy[s, o], over the slot's samples in order.  One CTA per
+// (slot, 16 outputs o, 256 columns j); a thread keeps 4 o x 4 j; the
+// samples' dy and h rows are staged 32 at a time in shared memory.
 __global__ void __launch_bounds__(256) k_head_dw_out(const __grid_constant__ HeadTable tab,
                                                      const float* __restrict__ dy, int ld_y,
                                                      const float* __restrict__ h, int ld_h) {
+    __shared__ __align__(16) float sh[32][256];
+    __shared__ __align__(16) float sd[32][16];
     const HeadSlot& hs = tab.slot[blockIdx.x];
-    const int idx = blockIdx.y * 256 + threadIdx.x;
-    if (idx >= hs.width * hs.hid) return;
-    const int o = idx / hs.hid, j = idx % hs.hid;
-    float acc = 0.f, accb = 0.f;
-    for (int s = hs.s0; s < hs.s1; ++s) {
-        const float g = dy[(size_t)s * ld_y + o];
-        acc += g * h[(size_t)s * ld_h + j];
-        accb += g;
+    const int o0 = blockIdx.y * 16, jb = blockIdx.z * 256;
+    if (o0 >= hs.width || jb >= hs.hid) return;
+    const int ty = threadIdx.x >> 6, tx = threadIdx.x & 63;
+    const int ob = o0 + 4 * ty, j0 = jb + 4 * tx;
+    float acc[4][4];
+#pragma unroll
+    for (int a = 0; a < 4; ++a) acc[a][0] = acc[a][1] = acc[a][2] = acc[a][3] = 0.f;
+    for (int sb = hs.s0; sb < hs.s1; sb += 32) {
+        const int nsb = min(32, hs.s1 - sb);
+        __syncthreads();
+        for (int i = threadIdx.x; i < 32 * 64; i += 256) {
+            const int r = i >> 6, u = i & 63;
+            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (r < nsb && jb + 4 * u < hs.hid)
+                v = *reinterpret_cast<const float4*>(h + (size_t)(sb + r) * ld_h + jb + 4 * u);
+            *reinterpret_cast<float4*>(&sh[r][4 * u]) = v;
+        }
+        for (int i = threadIdx.x; i < 32 * 16; i += 256) {
+            const int r = i >> 4, o = i & 15;
+            sd[r][o] = (r < nsb && o0 + o < hs.width) ? dy[(size_t)(sb + r) * ld_y + o0 + o] : 0.f;
+        }
+        __syncthreads();
+        for (int r = 0; r < nsb; ++r) {
+            const float4 d4 = *reinterpret_cast<const float4*>(&sd[r][4 * ty]);
+            const float4 x4 = *reinterpret_cast<const float4*>(&sh[r][4 * tx]);
+            const float d[4] = {d4.x, d4.y, d4.z, d4.w}, x[4] = {x4.x, x4.y, x4.z, x4.w};
+#pragma unroll
+            for (int a = 0; a < 4; ++a)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) acc[a][e] = fmaf(d[a], x[e], acc[a][e]);
+        }
     }
-    hs.g_w2[idx] = hs.accum ? hs.g_w2[idx] + acc : acc;
-    if (j == 0) hs.g_b2[o] = hs.accum ? hs.g_b2[o] + accb : accb;
+    if (j0 < hs.hid) {
+#pragma unroll
+        for (int a = 0; a < 4; ++a) {
+            const int o = ob + a;
+            if (o >= hs.width) break;
+            float4* dst = reinterpret_cast<float4*>(hs.g_w2 + (size_t)o * hs.hid + j0);
+            float4 v = make_float4(acc[a][0], acc[a][1], acc[a][2], acc[a][3]);
+            if (hs.accum) {
+                const float4 old = *dst;
+                v.x += old.x;
+                v.y += old.y;
+                v.z += old.z;
+                v.w += old.w;
+            }
+            *dst = v;
+        }
+    }
+    if (blockIdx.z == 0 && threadIdx.x < 16 && o0 + (int)threadIdx.x < hs.width) {
+        const int o = o0 + threadIdx.x;
+        float accb = 0.f;
+        for (int s = hs.s0; s < hs.s1; ++s) accb += dy[(size_t)s * ld_y + o];
+        hs.g_b2[o] = hs.accum ? hs.g_b2[o] + accb : accb;
+    }
 }
 
 // Gradient into the output layer's input: dh[s, j] = (sum_o dy[s, o] W[o, j])
 // times SiLU'(z[s, j]) for an MLP slot (dz), plain for a query head (dO).
-// One thread per column j, 8 samples at a time so W is read once per 8.
+// One CTA per (slot, 1024 columns j, 8 samples); a thread keeps 4
+// consecutive columns x 8 samples, so each weight row is read once per 8
+// samples (8-byte loads); dy is staged 64 outputs at a time in shared
+// memory; the outputs o are summed in order.
 __global__ void __launch_bounds__(256) k_head_back_in(const __grid_constant__ HeadTable tab,
                                                       const float* __restrict__ dy, int ld_y,
                                                       const float* __restrict__ z, int ld_h,
                                                       float* __restrict__ dh) {
+    __shared__ __align__(16) float sdy[64][8];
     const HeadSlot& hs = tab.slot[blockIdx.x];
-    const int j = blockIdx.y * 256 + threadIdx.x;
-    if (j >= hs.hid) return;
-    for (int s0 = hs.s0; s0 < hs.s1; s0 += 8) {
-        const int ns = min(8, hs.s1 - s0);
-        float acc[8];
+    const int s0 = hs.s0 + blockIdx.z * 8, jb = blockIdx.y * 1024;
+    if (s0 >= hs.s1 || jb >= hs.hid) return;
+    const int ns = min(8, hs.s1 - s0);
+    const int j0 = jb + 4 * threadIdx.x;
+    const bool colok = j0 < hs.hid;
+    float acc[8][4];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-        for (int o = 0; o < hs.width; ++o) {
-            const float w = bf2f(hs.w2[(size_t)o * hs.hid + j]);
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-                if (i < ns) acc[i] += dy[(size_t)(s0 + i) * ld_y + o] * w;
+    for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
+    for (int o0 = 0; o0 < hs.width; o0 += 64) {
+        const int no = min(64, hs.width - o0);
+        __syncthreads();
+        for (int i = threadIdx.x; i < 64 * 8; i += 256) {
+            const int si = i >> 6, o = i & 63;
+            sdy[o][si] = (o < no && si < ns) ? dy[(size_t)(s0 + si) * ld_y + o0 + o] : 0.f;
         }
+        __syncthreads();
+        if (colok) {
+            for (int o = 0; o < no; ++o) {
+                const uint2 wv =
+                    *reinterpret_cast<const uint2*>(hs.w2 + (size_t)(o0 + o) * hs.hid + j0);
+                const float w[4] = {__uint_as_float(wv.x << 16), __uint_as_float(wv.x & 0xFFFF0000u),
+                                    __uint_as_float(wv.y << 16), __uint_as_float(wv.y & 0xFFFF0000u)};
+                const float4 da = *reinterpret_cast<const float4*>(&sdy[o][0]);
+                const float4 db = *reinterpret_cast<const float4*>(&sdy[o][4]);
+                const float d[8] = {da.x, da.y, da.z, da.w, db.x, db.y, db.z, db.w};
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            if (i >= ns) break;
-            const size_t at = (size_t)(s0 + i) * ld_h + j;
-            dh[at] = hs.kind == JNX_HEAD_MLP ? acc[i] * silu_grad_f(z[at]) : acc[i];
+                for (int i = 0; i < 8; ++i)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) acc[i][e] = fmaf(d[i], w[e], acc[i][e]);
+            }
         }
+    }
+    if (!colok) return;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        if (i >= ns) break;
+        const size_t at = (size_t)(s0 + i) * ld_h + j0;
+        float4 v = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+        if (hs.kind == JNX_HEAD_MLP) {
+            const float4 zz = *reinterpret_cast<const float4*>(z + at);
+            v.x *= silu_grad_f(zz.x);
+            v.y *= silu_grad_f(zz.y);
+            v.z *= silu_grad_f(zz.z);
+            v.w *= silu_grad_f(zz.w);
+        }
+        *reinterpret_cast<float4*>(dh + at) = v;
     }
 }
 
@@ -425,160 +537,189 @@ __global__ void __launch_bounds__(256) k_xattn_dq(const __grid_constant__ HeadTa
     hs.g_q[i] = hs.accum ? hs.g_q[i] + acc : acc;
 }
 
-// dW[c, e] = sum over the slot's token rows r of g[r, c] * X[r, e], for
-// g = dk (-> dWk) and g = dv (-> dWv): a GEMM whose reduction runs over the
-// tenant's rows, on bf16 mma.sync (m16n8k16) with fp32 accumulation.  One
-// CTA per 64 x 128 output tile, 4 warps in a 2 x 2 layout (32 x 64 each);
-// rows stream through shared memory in chunks of 32.  The fp32 g is split
-// while staged into g_hi = bf16(g) and g_lo = bf16(g - g_hi) and both are
-// multiplied (X is exact in bf16), which keeps the result at fp32 accuracy;
-// both operands are row-major in r (MN-major) and are read with
-// ldmatrix.trans; X arrives by cp.async.  Fixed reduction order.
-namespace wg {
-constexpr int BMC = 64, BNE = 128, BR = 32;
-}
+// Query-head weight gradients, re-associated through the queries.  Per
+// sample, dk = scale dS^T Q and dv = P^T dO have rank <= nq (P, dS: [L, nq]
+// key-major), so
+//   dWk = sum_rows dk^T X = scale Q^T (sum_s G_s),  G_s = dS_s^T X_s  [nq, d]
+//   dWv = sum_rows dv^T X = sum_s dO_s^T H_s,       H_s = P_s^T X_s   [nq, d]
+// which takes 2 nq d flops per row and product instead of 2 dq d.  Both
+// steps run in fp32 on CUDA cores (X is exact in bf16), every sum in a fixed
+// order, so a tenant's gradients do not depend on the batch around it.
+//
+// k_xattn_gh: one CTA per (sample, 128 columns e of X); warp w takes
+// queries 4w..4w+3, a lane four consecutive columns; the sample's rows are
+// staged 32 at a time by cp.async (X rows, and the P / dS rows, nq floats
+// each, contiguous per sample).
+constexpr int kGhRows = 32;
 
-__global__ void __launch_bounds__(128) k_xattn_wgrad(const __grid_constant__ HeadTable tab,
-                                                     const float* __restrict__ dk,
-                                                     const float* __restrict__ dv, int ldkv,
-                                                     const uint16_t* __restrict__ X, int ldx) {
-    using namespace wg;
-    const HeadSlot& hs = tab.slot[blockIdx.x];
+__global__ void __launch_bounds__(256) k_xattn_gh(const __grid_constant__ HeadTable tab, int g0,
+                                                  const int* __restrict__ cu,
+                                                  const int* __restrict__ sample_slot,
+                                                  int sample0, const float* __restrict__ P,
+                                                  const float* __restrict__ dS,
+                                                  const uint16_t* __restrict__ X, int ldx,
+                                                  float* __restrict__ Gs, float* __restrict__ Hs,
+                                                  int ldg) {
+    __shared__ __align__(16) uint16_t sx[2][kGhRows][128];
+    __shared__ __align__(16) float sp[2][kGhRows * kMaxQ], sd[2][kGhRows * kMaxQ];
+    const int s = sample0 + blockIdx.x;
+    const HeadSlot& hs = tab.slot[sample_slot[s] - g0];
     if (hs.kind != JNX_HEAD_XATTN) return;
-    const int which = blockIdx.z & 1;
-    const int c0 = blockIdx.y * BMC;            // dq rows of the tile
-    const int e0 = (blockIdx.z >> 1) * BNE;     // d columns of the tile
-    if (c0 >= hs.dq || e0 >= hs.d_in) return;
-    const float* G = which ? dv : dk;
-    float* out = which ? hs.g_wv : hs.g_wk;
-    __shared__ __align__(128) uint8_t sA[2][2][BR * BMC * 2];  // [buf][hi/lo][r][c] bf16
-    __shared__ __align__(128) uint8_t sB[2][BR * BNE * 2];  // [r][e] bf16, 256-byte rows
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int wm = warp & 1, wn = warp >> 1;
-    const uint32_t aA = smem_u32(sA), aB = smem_u32(sB);
-    // row r, 16-byte chunk ch of a tile with `cpr` chunks per row, XOR-swizzled
-    auto swz = [](int r, int ch, int cpr) { return (uint32_t)(r * cpr * 16 + ((ch ^ (r & 7)) << 4)); };
-
-    float acc[2][8][4];
-#pragma unroll
-    for (int i = 0; i < 2; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j][0] = acc[i][j][1] = acc[i][j][2] = acc[i][j][3] = 0.f;
-
-    // A staging: thread -> (row = tid / 4, 16 consecutive c at (tid % 4) * 16)
-    const int ar = tid >> 2, ac = (tid & 3) * 16;
-    float4 areg[4];
-    auto load_a = [&](int r) {
-        const bool ok = r + ar < hs.r1;
-        const float4* src = reinterpret_cast<const float4*>(G + (size_t)(r + ar) * ldkv + c0 + ac);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) areg[i] = ok ? src[i] : make_float4(0.f, 0.f, 0.f, 0.f);
-    };
-    auto store_a = [&](int buf) {
-        uint8_t* hi_base = sA[buf][0];
-        uint8_t* lo_base = sA[buf][1];
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const float v[8] = {areg[2 * h].x,     areg[2 * h].y,     areg[2 * h].z,
-                                areg[2 * h].w,     areg[2 * h + 1].x, areg[2 * h + 1].y,
-                                areg[2 * h + 1].z, areg[2 * h + 1].w};
-            uint32_t hw[4], lw[4];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                hw[q] = pack_bf2(v[2 * q], v[2 * q + 1]);
-                const float h0 = __uint_as_float(hw[q] << 16);
-                const float h1 = __uint_as_float(hw[q] & 0xFFFF0000u);
-                lw[q] = pack_bf2(v[2 * q] - h0, v[2 * q + 1] - h1);
-            }
-            const uint32_t off = swz(ar, ac / 8 + h, BMC / 8);
-            *reinterpret_cast<uint4*>(hi_base + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-            *reinterpret_cast<uint4*>(lo_base + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-        }
-    };
-    auto load_b = [&](int r, int buf) {
-        for (int i = tid; i < BR * (BNE / 8); i += 128) {
-            const int rr = i / (BNE / 8), ch = i % (BNE / 8);
-            const bool ok = r + rr < hs.r1;
-            cp_async16(aB + buf * BR * BNE * 2 + swz(rr, ch, BNE / 8),
-                       ok ? (const void*)(X + (size_t)(r + rr) * ldx + e0 + ch * 8)
+    const int nq = hs.nq, e0 = blockIdx.y * 128;
+    if (e0 >= hs.d_in) return;
+    const int r0 = cu[s], L = cu[s + 1] - r0;
+    const float* Ps = P + (size_t)nq * r0;
+    const float* Ds = dS + (size_t)nq * r0;
+    auto load = [&](int j0, int buf) {
+        const int nr = min(kGhRows, L - j0);
+        for (int i = threadIdx.x; i < kGhRows * 16; i += 256) {
+            const int r = i >> 4, u = i & 15;
+            const bool ok = r < nr;
+            cp_async16(smem_u32(&sx[buf][r][8 * u]),
+                       ok ? (const void*)(X + (size_t)(r0 + j0 + r) * ldx + e0 + 8 * u)
                           : (const void*)X,
                        ok);
         }
-    };
-
-    const int mi = lane >> 3, rr8 = lane & 7;
-    int buf = 0;
-    if (hs.r0 < hs.r1) {
-        load_a(hs.r0);
-        load_b(hs.r0, 0);
-        cp_async_commit();
-        store_a(0);
-    }
-    for (int r = hs.r0; r < hs.r1; r += BR) {
-        const bool more = r + BR < hs.r1;
-        if (more) {
-            load_a(r + BR);
-            load_b(r + BR, buf ^ 1);
+        const int units = nr * nq / 4;  // nr rows of nq floats, contiguous
+        for (int i = threadIdx.x; i < kGhRows * kMaxQ / 4; i += 256) {
+            const bool ok = i < units;
+            cp_async16(smem_u32(&sp[buf][4 * i]), ok ? (const void*)(Ps + (size_t)j0 * nq + 4 * i)
+                                                     : (const void*)Ps, ok);
+            cp_async16(smem_u32(&sd[buf][4 * i]), ok ? (const void*)(Ds + (size_t)j0 * nq + 4 * i)
+                                                     : (const void*)Ds, ok);
         }
+    };
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool act = 4 * w < nq;
+    float g[4][4], h[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) g[i][e] = h[i][e] = 0.f;
+    const int nchunks = (L + kGhRows - 1) / kGhRows;
+    if (nchunks > 0) load(0, 0);
+    cp_async_commit();
+    for (int c = 0; c < nchunks; ++c) {
+        const int buf = c & 1;
+        if (c + 1 < nchunks) load((c + 1) * kGhRows, buf ^ 1);
         cp_async_commit();
         cp_async_wait<1>();
         __syncthreads();
-        const uint32_t a_base = aA + buf * 2 * BR * BMC * 2, b_base = aB + buf * BR * BNE * 2;
+        if (act) {
+            const int nr = min(kGhRows, L - c * kGhRows);
+            for (int r = 0; r < nr; ++r) {
+                const uint2 xv = *reinterpret_cast<const uint2*>(&sx[buf][r][4 * lane]);
+                const float x[4] = {__uint_as_float(xv.x << 16), __uint_as_float(xv.x & 0xFFFF0000u),
+                                    __uint_as_float(xv.y << 16), __uint_as_float(xv.y & 0xFFFF0000u)};
+                const float4 p4 = *reinterpret_cast<const float4*>(&sp[buf][r * nq + 4 * w]);
+                const float4 d4 = *reinterpret_cast<const float4*>(&sd[buf][r * nq + 4 * w]);
+                const float pq[4] = {p4.x, p4.y, p4.z, p4.w}, dq[4] = {d4.x, d4.y, d4.z, d4.w};
 #pragma unroll
-        for (int ks = 0; ks < BR / 16; ++ks) {
-            uint32_t af[2][2][4];  // [hi/lo][m-tile][regs]
+                for (int i = 0; i < 4; ++i)
 #pragma unroll
-            for (int part = 0; part < 2; ++part)
-#pragma unroll
-                for (int im = 0; im < 2; ++im) {
-                    // matrices (m 0-7, k 0-7), (m 8-15, k 0-7), (m 0-7, k 8-15), (m 8-15, k 8-15)
-                    const int kr = ks * 16 + rr8 + 8 * (mi >> 1);
-                    const int mch = (wm * 32 + im * 16) / 8 + (mi & 1);
-                    ldsm_x4_t(a_base + part * BR * BMC * 2 + swz(kr, mch, BMC / 8),
-                              af[part][im][0], af[part][im][1], af[part][im][2], af[part][im][3]);
-                }
-#pragma unroll
-            for (int np = 0; np < 4; ++np) {
-                // matrices (k 0-7, n 0-7), (k 8-15, n 0-7), (k 0-7, n 8-15), (k 8-15, n 8-15)
-                const int kr = ks * 16 + rr8 + 8 * (mi & 1);
-                const int nch = (wn * 64 + np * 16) / 8 + (mi >> 1);
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4_t(b_base + swz(kr, nch, BNE / 8), b0, b1, b2, b3);
-#pragma unroll
-                for (int part = 0; part < 2; ++part)
-#pragma unroll
-                    for (int im = 0; im < 2; ++im) {
-                        const uint32_t* a = af[part][im];
-                        mma_bf16(acc[im][2 * np], a[0], a[1], a[2], a[3], b0, b1);
-                        mma_bf16(acc[im][2 * np + 1], a[0], a[1], a[2], a[3], b2, b3);
+                    for (int e = 0; e < 4; ++e) {
+                        h[i][e] = fmaf(pq[i], x[e], h[i][e]);
+                        g[i][e] = fmaf(dq[i], x[e], g[i][e]);
                     }
             }
         }
         __syncthreads();
-        if (more) store_a(buf ^ 1);
-        buf ^= 1;
     }
-    const int g = lane >> 2, t = lane & 3;
+    if (!act) return;
 #pragma unroll
-    for (int im = 0; im < 2; ++im) {
+    for (int i = 0; i < 4; ++i) {
+        const size_t o = ((size_t)s * kMaxQ + 4 * w + i) * ldg + e0 + 4 * lane;
+        *reinterpret_cast<float4*>(Gs + o) = make_float4(g[i][0], g[i][1], g[i][2], g[i][3]);
+        *reinterpret_cast<float4*>(Hs + o) = make_float4(h[i][0], h[i][1], h[i][2], h[i][3]);
+    }
+}
+
+// k_xattn_wgrad: one CTA per (slot, 32 value columns c, 64 columns e); warp
+// w takes c = c0 + 4w..4w+3 (and the running sum of G_s over rows
+// q = 4w..4w+3), a lane two consecutive columns e.  The slot's samples in
+// order: dWv += dO_s^T H_s with dO_s [nq, 32] and H_s [nq, 64] staged; at the
+// end dWk = scale Q^T G_t with G_t staged.
+__global__ void __launch_bounds__(256) k_xattn_wgrad(const __grid_constant__ HeadTable tab,
+                                                     const float* __restrict__ Gs,
+                                                     const float* __restrict__ Hs, int ldg,
+                                                     const float* __restrict__ dO, int ld_h) {
+    __shared__ __align__(16) float sh[kMaxQ][64];
+    __shared__ __align__(16) float so[kMaxQ][32];
+    __shared__ __align__(16) float sg[kMaxQ][64];
+    const HeadSlot& hs = tab.slot[blockIdx.x];
+    if (hs.kind != JNX_HEAD_XATTN) return;
+    const int nq = hs.nq, dq = hs.dq, c0 = blockIdx.y * 32, e0 = blockIdx.z * 64;
+    if (c0 >= dq || e0 >= hs.d_in) return;
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float av[4][2], gt[4][2];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const int c = c0 + wm * 32 + im * 16 + g;
-            const int e = e0 + wn * 64 + j * 8 + 2 * t;
-            float2* d0 = reinterpret_cast<float2*>(out + (size_t)c * hs.d_in + e);
-            float2* d1 = reinterpret_cast<float2*>(out + (size_t)(c + 8) * hs.d_in + e);
-            float2 v0 = make_float2(acc[im][j][0], acc[im][j][1]);
-            float2 v1 = make_float2(acc[im][j][2], acc[im][j][3]);
-            if (hs.accum) {
-                const float2 o0 = *d0, o1 = *d1;
-                v0.x += o0.x;
-                v0.y += o0.y;
-                v1.x += o1.x;
-                v1.y += o1.y;
-            }
-            *d0 = v0;
-            *d1 = v1;
+    for (int i = 0; i < 4; ++i) av[i][0] = av[i][1] = gt[i][0] = gt[i][1] = 0.f;
+    for (int s = hs.s0; s < hs.s1; ++s) {
+        __syncthreads();  // the previous sample's staged rows are read
+        for (int i = threadIdx.x; i < nq * 16; i += 256) {  // H_s [nq, 64]: 16 float4 per row
+            const int q = i >> 4, u = i & 15;
+            *reinterpret_cast<float4*>(&sh[q][4 * u]) = *reinterpret_cast<const float4*>(
+                Hs + ((size_t)s * kMaxQ + q) * ldg + e0 + 4 * u);
         }
+        for (int i = threadIdx.x; i < nq * 8; i += 256) {  // dO_s [nq, 32]: 8 float4 per row
+            const int q = i >> 3, u = i & 7;
+            *reinterpret_cast<float4*>(&so[q][4 * u]) = *reinterpret_cast<const float4*>(
+                dO + (size_t)s * ld_h + (size_t)q * dq + c0 + 4 * u);
+        }
+        if (4 * w < nq) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float2 gv = *reinterpret_cast<const float2*>(
+                    Gs + ((size_t)s * kMaxQ + 4 * w + i) * ldg + e0 + 2 * lane);
+                gt[i][0] += gv.x;
+                gt[i][1] += gv.y;
+            }
+        }
+        __syncthreads();
+        for (int q = 0; q < nq; ++q) {
+            const float4 o4 = *reinterpret_cast<const float4*>(&so[q][4 * w]);
+            const float2 hv = *reinterpret_cast<const float2*>(&sh[q][2 * lane]);
+            const float o[4] = {o4.x, o4.y, o4.z, o4.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                av[i][0] = fmaf(o[i], hv.x, av[i][0]);
+                av[i][1] = fmaf(o[i], hv.y, av[i][1]);
+            }
+        }
+    }
+    __syncthreads();
+    if (4 * w < nq) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            *reinterpret_cast<float2*>(&sg[4 * w + i][2 * lane]) = make_float2(gt[i][0], gt[i][1]);
+    }
+    __syncthreads();
+    const float scale = rsqrtf((float)dq);
+    float ak[4][2] = {};
+    for (int q = 0; q < nq; ++q) {
+        const float2 gv = *reinterpret_cast<const float2*>(&sg[q][2 * lane]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float qv = bf2f(hs.q[(size_t)q * dq + c0 + 4 * w + i]);
+            ak[i][0] = fmaf(qv, gv.x, ak[i][0]);
+            ak[i][1] = fmaf(qv, gv.y, ak[i][1]);
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const size_t o = (size_t)(c0 + 4 * w + i) * hs.d_in + e0 + 2 * lane;
+        float2 vk = make_float2(ak[i][0] * scale, ak[i][1] * scale);
+        float2 vv = make_float2(av[i][0], av[i][1]);
+        if (hs.accum) {
+            const float2 ok = *reinterpret_cast<const float2*>(hs.g_wk + o);
+            const float2 ov = *reinterpret_cast<const float2*>(hs.g_wv + o);
+            vk.x += ok.x;
+            vk.y += ok.y;
+            vv.x += ov.x;
+            vv.y += ov.y;
+        }
+        *reinterpret_cast<float2*>(hs.g_wk + o) = vk;
+        *reinterpret_cast<float2*>(hs.g_wv + o) = vv;
     }
 }
 
@@ -596,7 +737,8 @@ jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const 
                                 float* loss, cudaStream_t s) {
     if (b.n == 0) return JNX_OK;
     if (b.any_mlp)
-        k_head_lin<1><<<dim3(b.n, (b.max_hid + 7) / 8), 256, 0, s>>>(
+        k_head_lin<1><<<dim3(b.n, (b.max_mlp_hid + kLinCols - 1) / kLinCols,
+                             (b.max_ns + kLinS - 1) / kLinS), 256, 0, s>>>(
             tab, pooled, d, ws.z, ws.h, ws.ld_h, sample_target, preds);
     if (b.any_xattn) {
         const size_t smem = (size_t)b.max_nq * b.max_dq * sizeof(float);
@@ -604,9 +746,9 @@ jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const 
                                                              b.sample0, ws.kbuf, ws.vbuf, ws.ldkv,
                                                              ws.P, ws.h, ws.ld_h);
     }
-    k_head_lin<2><<<dim3(b.n, (b.max_width + 7) / 8), 256, 0, s>>>(tab, ws.h, ws.ld_h, ws.y,
-                                                                   nullptr, ws.ld_y,
-                                                                   sample_target, preds);
+    k_head_lin<2><<<dim3(b.n, (b.max_width + kLinCols - 1) / kLinCols,
+                         (b.max_ns + kLinS - 1) / kLinS), 256, 0, s>>>(
+        tab, ws.h, ws.ld_h, ws.y, nullptr, ws.ld_y, sample_target, preds);
     if (targets)  // without targets (inference) there is no loss
         k_l2_loss<<<b.n, 256, 0, s>>>(tab, ws.y, ws.ld_y, targets, sample_target, ws.dy, loss);
     return cuda_ok("heads forward");
@@ -616,10 +758,10 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
                                  const float* pooled, int d, const uint16_t* hidden,
                                  const int* cu, const int* sample_slot, cudaStream_t s) {
     if (b.n == 0) return JNX_OK;
-    k_head_dw_out<<<dim3(b.n, (b.max_width * b.max_hid + 255) / 256), 256, 0, s>>>(
+    k_head_dw_out<<<dim3(b.n, (b.max_width + 15) / 16, (b.max_hid + 255) / 256), 256, 0, s>>>(
         tab, ws.dy, ws.ld_y, ws.h, ws.ld_h);
-    k_head_back_in<<<dim3(b.n, (b.max_hid + 255) / 256), 256, 0, s>>>(tab, ws.dy, ws.ld_y, ws.z,
-                                                                      ws.ld_h, ws.dh);
+    k_head_back_in<<<dim3(b.n, (b.max_hid + 1023) / 1024, (b.max_ns + 7) / 8), 256, 0, s>>>(
+        tab, ws.dy, ws.ld_y, ws.z, ws.ld_h, ws.dh);
     if (b.any_mlp)
         k_mlp_dw1<<<dim3(b.n, b.max_mlp_hid, (d / 4 + 255) / 256), 256, 0, s>>>(tab, ws.dh,
                                                                                ws.ld_h, pooled, d);
@@ -630,8 +772,10 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
             ws.ld_h, ws.dk, ws.dv, ws.dQs);
         k_xattn_dq<<<dim3(b.n, (b.max_nq * b.max_dq + 255) / 256), 256, 0, s>>>(tab, ws.dQs,
                                                                                  ws.ld_h);
-        k_xattn_wgrad<<<dim3(b.n, b.max_dq / wg::BMC, 2 * (d / wg::BNE)), 128, 0, s>>>(
-            tab, ws.dk, ws.dv, ws.ldkv, hidden, d);
+        k_xattn_gh<<<dim3(b.sample1 - b.sample0, d / 128), 256, 0, s>>>(
+            tab, b.g0, cu, sample_slot, b.sample0, ws.P, ws.dS, hidden, d, ws.Gs, ws.Hs, d);
+        k_xattn_wgrad<<<dim3(b.n, b.max_dq / 32, d / 64), 256, 0, s>>>(tab, ws.Gs, ws.Hs, d, ws.dh,
+                                                                       ws.ld_h);
     }
     return cuda_ok("heads backward");
 }

@@ -36,6 +36,7 @@ struct HeadBatch {
     int g0, n;                 // group slots [g0, g0 + n)
     int sample0, sample1;      // their packed samples
     int max_hid, max_mlp_hid, max_width, max_nq, max_dq;
+    int max_ns;                // most samples in one slot
     bool any_mlp, any_xattn;
 };
 
@@ -49,6 +50,7 @@ struct HeadScratch {
     int ldkv;
     float *P, *dS;                 // [nq * n_tokens], key-major per sample
     float* dQs;                    // [n_samples, ld_h]
+    float *Gs, *Hs;                // [n_samples, 32, d]: dS_s^T X_s and P_s^T X_s (32 query rows)
     uint16_t* dkv_bf;              // feature gradient: bf16 [dk | dv] rows [n_tokens, 2 ldkv]
 };
 
