@@ -115,6 +115,58 @@ def test_gpu_calls_reject_bad_arguments_without_a_gpu():
     assert rc == J.JNX_ERR_INVALID_ARG
 
 
+def _host_group(n_tokens=4):
+    """A one-sample, one-slot group whose device arrays are placeholders:
+    only its host arrays are read before a call's checks fail."""
+    import ctypes as C
+    keep = [(C.c_int32 * 2)(0, n_tokens), (C.c_int32 * 2)(0, 1), (C.c_int32 * 1)(0)]
+    fake = 1 << 20  # never dereferenced: the calls below return before any launch
+    g = J.jnx_group(1, n_tokens, 1, n_tokens, fake, fake, fake, fake, fake, fake,
+                    C.cast(keep[0], J.P32), C.cast(keep[1], J.P32), C.cast(keep[2], J.P32))
+    return g, keep
+
+
+def _host_flow_head(d_model):
+    import ctypes as C
+    fake = 1 << 20
+    blocks = (J.jnx_flow_block * 1)(J.jnx_flow_block(fake, fake, fake, fake, fake))
+    fh = J.jnx_flow_head(d_model, 256, 1, 8, 7, 256, 1, *([fake] * 9),
+                         C.cast(blocks, C.POINTER(J.jnx_flow_block)))
+    return fh, blocks
+
+
+def test_training_entry_points_reject_bad_arguments_without_a_gpu():
+    import ctypes as C
+    L = J.lib()
+    inv, uns = J.JNX_ERR_INVALID_ARG, J.JNX_ERR_UNSUPPORTED
+    # null descriptors and groups are rejected on the host before any launch
+    assert L.jnx_flow_forward(None, None, None, None, None, None, None, None, None, 0, None) == inv
+    assert L.jnx_flow_backward(None, None, None, None, 0, None, 0, None) == inv
+    assert L.jnx_flow_sample(None, None, None, None, 4, None, None, 0, None) == inv
+    assert L.jnx_flow_workspace_bytes(None, None) == 0
+    assert L.jnx_backbone_backward_lora(None, None, None, None, None, None, 0, None, 0,
+                                        None) == inv
+    assert L.jnx_heads_backward_input(None, 0, None, None, None, None, None, None, None, 0,
+                                      None) == inv
+    assert L.jnx_adamw_tensors(None, 1, None, None) == inv
+    assert L.jnx_transpose(None, 1, -1, 4, None, None) == inv
+    # a well-formed group: the expert's checks decide, still before any launch
+    g, keep = _host_group()
+    fh, blocks = _host_flow_head(384)  # width not in {256, 512, 1024}
+    fake = 1 << 20
+    rc = L.jnx_flow_forward(C.byref(fh), C.byref(g), fake, fake, fake, fake, fake, fake, fake,
+                            1 << 30, None)
+    assert rc == uns and "d_model" in J.jnx_last_error()
+    fh, blocks = _host_flow_head(256)
+    rc = L.jnx_flow_forward(C.byref(fh), C.byref(g), fake, fake, fake, fake, fake, fake,
+                            fake + 16, 1 << 30, None)  # workspace off a 256-byte boundary
+    assert rc == inv and "aligned" in J.jnx_last_error()
+    fh.t1 = fake + 2  # a time-MLP weight off a 16-byte boundary
+    rc = L.jnx_flow_forward(C.byref(fh), C.byref(g), fake, fake, fake, fake, fake, fake, fake,
+                            1 << 30, None)
+    assert rc == inv and "aligned" in J.jnx_last_error()
+
+
 def test_scheduler_bit_exact_vs_oracle_random_queues():
     # jnx_sched_poll (C++) against the scheduler oracle: same queue indices
     # to take and the same wake time, on both collection modes
