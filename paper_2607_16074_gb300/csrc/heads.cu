@@ -341,98 +341,193 @@ __global__ void __launch_bounds__(256) k_mlp_dw1(const __grid_constant__ HeadTab
     }
 }
 
+constexpr int kMaxQ = 32;
+constexpr int kXRows = 32;  // key rows staged at a time
+
+// Shared-memory layout of the per-sample query-head kernels (fp32, rows
+// padded by 4 floats so the rows a warp reads together fall in distinct
+// banks): A [kMaxQ][dq + 4] (the queries, or dO), R [kXRows][dq + 4] (a
+// tile of key rows of k or v), then a P chunk and a dS chunk of
+// [kXRows][kMaxQ] each.
+__host__ __device__ constexpr size_t xattn_smem_bytes(int dq) {
+    return ((size_t)(kMaxQ + kXRows) * (dq + 4) + 2 * kXRows * kMaxQ) * sizeof(float);
+}
+
+// The nq x dq rows of a bf16 (src16) or fp32 (src32) matrix into sA (padded).
+__device__ __forceinline__ void xattn_stage_a(float* sA, const uint16_t* src16, const float* src32,
+                                              int nq, int dq) {
+    const int ld = dq + 4;
+    for (int i = threadIdx.x; i < nq * dq; i += blockDim.x) {
+        const int q = i / dq, c = i % dq;
+        sA[q * ld + c] = src16 ? bf2f(src16[i]) : src32[i];
+    }
+}
+
+// Rows j0 .. j0 + nr - 1 of R (stride ldkv, from row r0) into the padded
+// tile sR by cp.async (rows past nr zero).  Caller commits and waits.
+__device__ __forceinline__ void xattn_stage_rows(float* sR, const float* __restrict__ R, int ldkv,
+                                                 int r0, int j0, int nr, int dq) {
+    const int ld = dq + 4, units = dq / 4;
+    for (int i = threadIdx.x; i < kXRows * units; i += blockDim.x) {
+        const int r = i / units, u = i % units;
+        const bool ok = r < nr;
+        cp_async16(smem_u32(sR + r * ld + 4 * u),
+                   ok ? (const void*)(R + (size_t)(r0 + j0 + r) * ldkv + 4 * u) : (const void*)R,
+                   ok);
+    }
+}
+
+// out[j * nq + q] = scale * (A[q, :] . R[r0 + j, :]) for the sample's L key
+// rows, key-major.  Key rows staged kXRows at a time; thread (jj = tid / 8,
+// g = tid % 8) takes row jj and queries g, g + 8, g + 16, g + 24 (strided so
+// the eight query rows a warp reads at once sit in distinct banks).  Ends
+// with a barrier.
+__device__ void xattn_rows_dot(const float* __restrict__ R, int ldkv, int r0, int L,
+                               const float* sA, float* sR, int nq, int dq, float scale,
+                               float* __restrict__ out) {
+    const int ld = dq + 4;
+    const int jj = threadIdx.x >> 3, g = threadIdx.x & 7;
+    for (int j0 = 0; j0 < L; j0 += kXRows) {
+        const int nr = min(kXRows, L - j0);
+        __syncthreads();  // the previous tile (or sA's writers) done
+        xattn_stage_rows(sR, R, ldkv, r0, j0, nr, dq);
+        cp_async_commit();
+        cp_async_wait<0>();
+        __syncthreads();
+        if (jj < nr) {
+            float acc[4] = {0.f, 0.f, 0.f, 0.f};
+            const float* rr = sR + jj * ld;
+            for (int c = 0; c < dq; c += 4) {
+                const float4 x = *reinterpret_cast<const float4*>(rr + c);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    if (g + 8 * i < nq) {
+                        const float4 a = *reinterpret_cast<const float4*>(sA + (g + 8 * i) * ld + c);
+                        acc[i] = fmaf(a.x, x.x, fmaf(a.y, x.y, fmaf(a.z, x.z, fmaf(a.w, x.w, acc[i]))));
+                    }
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                if (g + 8 * i < nq) out[(size_t)(j0 + jj) * nq + g + 8 * i] = acc[i] * scale;
+        }
+    }
+    __syncthreads();
+}
+
+// Per-query reductions over the sample's key-major [L, nq] block X (and Y):
+// thread (q = tid % 32, part = tid / 32) covers keys part, part + 8, ...;
+// the eight parts are combined in order.  red: 8 x 32 floats of shared
+// memory.  MAX: max_j X; otherwise sum_j X * Y (Y may be X's weights).
+template <bool MAX>
+__device__ float xattn_reduce_q(const float* __restrict__ X, const float* __restrict__ Y, int L,
+                                int nq, float* red) {
+    const int q = threadIdx.x & 31, part = threadIdx.x >> 5;
+    float v = MAX ? -INFINITY : 0.f;
+    if (q < nq)
+        for (int j = part; j < L; j += 8) {
+            const float x = X[(size_t)j * nq + q];
+            v = MAX ? fmaxf(v, x) : fmaf(x, Y[(size_t)j * nq + q], v);
+        }
+    red[part * 32 + q] = v;
+    __syncthreads();
+    float r = MAX ? -INFINITY : 0.f;
+    for (int p = 0; p < 8; ++p) r = MAX ? fmaxf(r, red[p * 32 + q]) : r + red[p * 32 + q];
+    __syncthreads();  // red is reused by the caller
+    return r;  // valid in threads with q < nq (every part holds the same value)
+}
+
 // ---------------------------------------------------------------------------
-// Query head, per sample.  One CTA per packed sample of a query-head slot;
-// the tenant's learned queries (nq <= 32 of width dq) sit in shared memory.
+// Query head, per sample.  One CTA per packed sample of a query-head slot.
 // P (normalised attention) for sample s is stored key-major at P + nq * cu[s]:
 // element (query q, key j) at j * nq + q (nq a multiple of 4).
 // ---------------------------------------------------------------------------
-constexpr int kMaxQ = 32;
-
-__global__ void __launch_bounds__(256, 1) k_xattn_fwd(const __grid_constant__ HeadTable tab, int g0,
+__global__ void __launch_bounds__(256) k_xattn_fwd(const __grid_constant__ HeadTable tab, int g0,
                                                    const int* __restrict__ cu,
                                                    const int* __restrict__ sample_slot,
                                                    int sample0, const float* __restrict__ kbuf,
                                                    const float* __restrict__ vbuf, int ldkv,
                                                    float* __restrict__ P, float* __restrict__ h,
                                                    int ld_h) {
-    extern __shared__ float xs[];  // Q [nq][dq]
+    extern __shared__ __align__(16) float xs[];
+    __shared__ float red[8 * 32];
     const int s = sample0 + blockIdx.x;
     const HeadSlot& hs = tab.slot[sample_slot[s] - g0];
     if (hs.kind != JNX_HEAD_XATTN) return;
-    const int nq = hs.nq, dq = hs.dq;
+    const int nq = hs.nq, dq = hs.dq, ld = dq + 4;
+    float* sA = xs;
+    float* sR = sA + kMaxQ * ld;
+    float* sP = sR + kXRows * ld;
     const int r0 = cu[s], L = cu[s + 1] - r0;
-    const float scale = rsqrtf((float)dq);
-    for (int i = threadIdx.x; i < nq * dq; i += 256) xs[i] = bf2f(hs.q[i]);
-    __syncthreads();
     float* Ps = P + (size_t)nq * r0;
-    // scores: one thread per key, all queries
-    for (int j = threadIdx.x; j < L; j += 256) {
-        float acc[kMaxQ];
-#pragma unroll
-        for (int q = 0; q < kMaxQ; ++q) acc[q] = 0.f;
-        const float4* kr = reinterpret_cast<const float4*>(kbuf + (size_t)(r0 + j) * ldkv);
-        for (int c4 = 0; c4 < dq / 4; ++c4) {
-            const float4 kv = kr[c4];
-#pragma unroll
-            for (int q = 0; q < kMaxQ; ++q) {
-                if (q < nq) {
-                    const float* qq = xs + q * dq + 4 * c4;
-                    acc[q] += qq[0] * kv.x + qq[1] * kv.y + qq[2] * kv.z + qq[3] * kv.w;
-                }
-            }
-        }
-#pragma unroll
-        for (int q = 0; q < kMaxQ; ++q)
-            if (q < nq) Ps[(size_t)j * nq + q] = acc[q] * scale;
-    }
-    __syncthreads();
-    // softmax per query (key-major storage: element (q, j) at j * nq + q);
-    // one warp per query
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int q = warp; q < nq; q += 8) {
-        float m = -INFINITY;
-        for (int j = lane; j < L; j += 32) m = fmaxf(m, Ps[(size_t)j * nq + q]);
-        m = warp_max_h(m);
+    xattn_stage_a(sA, hs.q, nullptr, nq, dq);
+    // scores S[j, q] = q_q . k_j / sqrt(dq)
+    xattn_rows_dot(kbuf, ldkv, r0, L, sA, sR, nq, dq, rsqrtf((float)dq), Ps);
+    // softmax over the keys of each query, in place
+    const float m = xattn_reduce_q<true>(Ps, nullptr, L, nq, red);
+    {
+        const int q = threadIdx.x & 31, part = threadIdx.x >> 5;
         float sum = 0.f;
-        for (int j = lane; j < L; j += 32) {
-            const float e = expf(Ps[(size_t)j * nq + q] - m);
-            Ps[(size_t)j * nq + q] = e;
-            sum += e;
-        }
-        sum = warp_sum_h(sum);
-        const float inv = 1.0f / sum;
-        for (int j = lane; j < L; j += 32) Ps[(size_t)j * nq + q] *= inv;
+        if (q < nq)
+            for (int j = part; j < L; j += 8) {
+                const float e = expf(Ps[(size_t)j * nq + q] - m);
+                Ps[(size_t)j * nq + q] = e;
+                sum += e;
+            }
+        red[part * 32 + q] = sum;
+        __syncthreads();
+        float tot = 0.f;
+        for (int p = 0; p < 8; ++p) tot += red[p * 32 + q];
+        const float inv = 1.0f / tot;
+        if (q < nq)
+            for (int j = part; j < L; j += 8) Ps[(size_t)j * nq + q] *= inv;
+        __syncthreads();
     }
-    __syncthreads();
-    // O = P v: one thread per value column c
-    for (int c = threadIdx.x; c < dq; c += 256) {
+    // O[q, c] = sum_j P[j, q] v[j, c]: a thread per value column, keys in
+    // order; P and v rows staged kXRows at a time
+    for (int c0 = 0; c0 < dq; c0 += 256) {
+        const int c = c0 + threadIdx.x;
         float acc[kMaxQ];
 #pragma unroll
         for (int q = 0; q < kMaxQ; ++q) acc[q] = 0.f;
-        for (int j = 0; j < L; ++j) {
-            const float vv = vbuf[(size_t)(r0 + j) * ldkv + c];
-            const float4* pj = reinterpret_cast<const float4*>(Ps + (size_t)j * nq);
+        for (int j0 = 0; j0 < L; j0 += kXRows) {
+            const int nr = min(kXRows, L - j0);
+            __syncthreads();
+            xattn_stage_rows(sR, vbuf, ldkv, r0, j0, nr, dq);
+            for (int i = threadIdx.x; i < nr * nq / 4; i += 256)
+                cp_async16(smem_u32(sP + 4 * i), Ps + (size_t)j0 * nq + 4 * i, true);
+            cp_async_commit();
+            cp_async_wait<0>();
+            __syncthreads();
+            if (c < dq)
+                for (int j = 0; j < nr; ++j) {
+                    const float vv = sR[j * ld + c];
 #pragma unroll
-            for (int q4 = 0; q4 < kMaxQ / 4; ++q4) {
-                if (4 * q4 < nq) {
-                    const float4 pp = pj[q4];
-                    acc[4 * q4 + 0] += pp.x * vv;
-                    acc[4 * q4 + 1] += pp.y * vv;
-                    acc[4 * q4 + 2] += pp.z * vv;
-                    acc[4 * q4 + 3] += pp.w * vv;
+                    for (int q4 = 0; q4 < kMaxQ / 4; ++q4) {
+                        if (4 * q4 < nq) {
+                            const float4 pp = *reinterpret_cast<const float4*>(sP + j * nq + 4 * q4);
+                            acc[4 * q4 + 0] = fmaf(pp.x, vv, acc[4 * q4 + 0]);
+                            acc[4 * q4 + 1] = fmaf(pp.y, vv, acc[4 * q4 + 1]);
+                            acc[4 * q4 + 2] = fmaf(pp.z, vv, acc[4 * q4 + 2]);
+                            acc[4 * q4 + 3] = fmaf(pp.w, vv, acc[4 * q4 + 3]);
+                        }
+                    }
                 }
-            }
         }
+        if (c < dq) {
 #pragma unroll
-        for (int q = 0; q < kMaxQ; ++q)
-            if (q < nq) h[(size_t)s * ld_h + q * dq + c] = acc[q];
+            for (int q = 0; q < kMaxQ; ++q)
+                if (q < nq) h[(size_t)s * ld_h + q * dq + c] = acc[q];
+        }
     }
 }
 
-// Backward per sample: dP, dS (stored over dPbuf), dv, dk rows, and this
-// sample's dQ contribution (summed per tenant later in sample order).
-__global__ void __launch_bounds__(256, 1) k_xattn_bwd(const __grid_constant__ HeadTable tab, int g0,
+// Backward per sample: dP = dO v^T (into dS), the per-query sums
+// D_q = sum_j dP P, dS = P (dP - D_q) in place, then per value column c
+// with dO[:, c] and Q[:, c] in registers: dv[j, c] = sum_q P dO,
+// dk[j, c] = scale sum_q dS Q, and this sample's dQ contribution
+// scale sum_j dS[j, q] k[j, c] (summed per tenant later in sample order).
+__global__ void __launch_bounds__(256) k_xattn_bwd(const __grid_constant__ HeadTable tab, int g0,
                                                    const int* __restrict__ cu,
                                                    const int* __restrict__ sample_slot,
                                                    int sample0, const float* __restrict__ kbuf,
@@ -442,86 +537,82 @@ __global__ void __launch_bounds__(256, 1) k_xattn_bwd(const __grid_constant__ He
                                                    const float* __restrict__ dO, int ld_h,
                                                    float* __restrict__ dk, float* __restrict__ dv,
                                                    float* __restrict__ dQs) {
-    extern __shared__ float xs[];  // Q [nq][dq], then dO [nq][dq]
+    extern __shared__ __align__(16) float xs[];
+    __shared__ float red[8 * 32];
     const int s = sample0 + blockIdx.x;
     const HeadSlot& hs = tab.slot[sample_slot[s] - g0];
     if (hs.kind != JNX_HEAD_XATTN) return;
-    const int nq = hs.nq, dq = hs.dq;
+    const int nq = hs.nq, dq = hs.dq, ld = dq + 4;
+    float* sA = xs;
+    float* sR = sA + kMaxQ * ld;
+    float* sP = sR + kXRows * ld;
+    float* sD = sP + kXRows * kMaxQ;
     const int r0 = cu[s], L = cu[s + 1] - r0;
     const float scale = rsqrtf((float)dq);
-    float* Qs = xs;
-    float* dOs = xs + nq * dq;
-    for (int i = threadIdx.x; i < nq * dq; i += 256) {
-        Qs[i] = bf2f(hs.q[i]);
-        dOs[i] = dO[(size_t)s * ld_h + i];
-    }
-    __syncthreads();
     const float* Ps = P + (size_t)nq * r0;
     float* dSs = dS + (size_t)nq * r0;
-    // dP[q, j] = dO[q, :] . v[j, :]
-    for (int j = threadIdx.x; j < L; j += 256) {
-        float acc[kMaxQ];
-#pragma unroll
-        for (int q = 0; q < kMaxQ; ++q) acc[q] = 0.f;
-        const float4* vr = reinterpret_cast<const float4*>(vbuf + (size_t)(r0 + j) * ldkv);
-        for (int c4 = 0; c4 < dq / 4; ++c4) {
-            const float4 vv = vr[c4];
-#pragma unroll
-            for (int q = 0; q < kMaxQ; ++q) {
-                if (q < nq) {
-                    const float* o = dOs + q * dq + 4 * c4;
-                    acc[q] += o[0] * vv.x + o[1] * vv.y + o[2] * vv.z + o[3] * vv.w;
-                }
+    xattn_stage_a(sA, nullptr, dO + (size_t)s * ld_h, nq, dq);
+    xattn_rows_dot(vbuf, ldkv, r0, L, sA, sR, nq, dq, 1.f, dSs);  // dP
+    const float Dq = xattn_reduce_q<false>(dSs, Ps, L, nq, red);
+    {
+        const int q = threadIdx.x & 31, part = threadIdx.x >> 5;
+        if (q < nq)
+            for (int j = part; j < L; j += 8) {
+                const size_t at = (size_t)j * nq + q;
+                dSs[at] = Ps[at] * (dSs[at] - Dq);
             }
-        }
-#pragma unroll
-        for (int q = 0; q < kMaxQ; ++q)
-            if (q < nq) dSs[(size_t)j * nq + q] = acc[q];
+        __syncthreads();
     }
-    __syncthreads();
-    // dS = P * (dP - sum_j dP * P), one warp per query (key-major storage)
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int q = warp; q < nq; q += 8) {
-        float t = 0.f;
-        for (int j = lane; j < L; j += 32) t += dSs[(size_t)j * nq + q] * Ps[(size_t)j * nq + q];
-        t = warp_sum_h(t);
-        for (int j = lane; j < L; j += 32) {
-            const size_t at = (size_t)j * nq + q;
-            dSs[at] = Ps[at] * (dSs[at] - t);
+    for (int c0 = 0; c0 < dq; c0 += 256) {
+        const int c = c0 + threadIdx.x;
+        const bool colok = c < dq;
+        float go[kMaxQ], qc[kMaxQ], dqa[kMaxQ];
+#pragma unroll
+        for (int q = 0; q < kMaxQ; ++q) {
+            go[q] = colok && q < nq ? sA[q * ld + c] : 0.f;
+            qc[q] = colok && q < nq ? bf2f(hs.q[(size_t)q * dq + c]) : 0.f;
+            dqa[q] = 0.f;
         }
-    }
-    __syncthreads();
-    // per value column c: dv[j, c], dk[j, c] for every key j, and dQ[:, c]
-    for (int c = threadIdx.x; c < dq; c += 256) {
-        float dq_acc[kMaxQ];
+        for (int j0 = 0; j0 < L; j0 += kXRows) {
+            const int nr = min(kXRows, L - j0);
+            __syncthreads();
+            xattn_stage_rows(sR, kbuf, ldkv, r0, j0, nr, dq);
+            for (int i = threadIdx.x; i < nr * nq / 4; i += 256) {
+                cp_async16(smem_u32(sP + 4 * i), Ps + (size_t)j0 * nq + 4 * i, true);
+                cp_async16(smem_u32(sD + 4 * i), dSs + (size_t)j0 * nq + 4 * i, true);
+            }
+            cp_async_commit();
+            cp_async_wait<0>();
+            __syncthreads();
+            if (!colok) continue;
+            for (int j = 0; j < nr; ++j) {
+                const float kk = sR[j * ld + c];
+                float a_v = 0.f, a_k = 0.f;
 #pragma unroll
-        for (int q = 0; q < kMaxQ; ++q) dq_acc[q] = 0.f;
-        for (int j = 0; j < L; ++j) {
-            float a_v = 0.f, a_k = 0.f;
-            const float kk = kbuf[(size_t)(r0 + j) * ldkv + c];
-            const float4* pj = reinterpret_cast<const float4*>(Ps + (size_t)j * nq);
-            const float4* dj = reinterpret_cast<const float4*>(dSs + (size_t)j * nq);
+                for (int q4 = 0; q4 < kMaxQ / 4; ++q4) {
+                    if (4 * q4 < nq) {
+                        const float4 p4 = *reinterpret_cast<const float4*>(sP + j * nq + 4 * q4);
+                        const float4 d4 = *reinterpret_cast<const float4*>(sD + j * nq + 4 * q4);
+                        const float pp[4] = {p4.x, p4.y, p4.z, p4.w};
+                        const float dd[4] = {d4.x, d4.y, d4.z, d4.w};
 #pragma unroll
-            for (int q4 = 0; q4 < kMaxQ / 4; ++q4) {
-                if (4 * q4 < nq) {
-                    const float4 p4 = pj[q4], d4 = dj[q4];
-                    const float pp[4] = {p4.x, p4.y, p4.z, p4.w};
-                    const float dd[4] = {d4.x, d4.y, d4.z, d4.w};
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int q = 4 * q4 + e;
-                        a_v += pp[e] * dOs[q * dq + c];
-                        a_k += dd[e] * Qs[q * dq + c];
-                        dq_acc[q] += dd[e] * kk;
+                        for (int e = 0; e < 4; ++e) {
+                            const int q = 4 * q4 + e;
+                            a_v = fmaf(pp[e], go[q], a_v);
+                            a_k = fmaf(dd[e], qc[q], a_k);
+                            dqa[q] = fmaf(dd[e], kk, dqa[q]);
+                        }
                     }
                 }
+                dv[(size_t)(r0 + j0 + j) * ldkv + c] = a_v;
+                dk[(size_t)(r0 + j0 + j) * ldkv + c] = a_k * scale;
             }
-            dv[(size_t)(r0 + j) * ldkv + c] = a_v;
-            dk[(size_t)(r0 + j) * ldkv + c] = a_k * scale;
         }
+        if (colok) {
 #pragma unroll
-        for (int q = 0; q < kMaxQ; ++q)
-            if (q < nq) dQs[(size_t)s * ld_h + q * dq + c] = dq_acc[q] * scale;
+            for (int q = 0; q < kMaxQ; ++q)
+                if (q < nq) dQs[(size_t)s * ld_h + q * dq + c] = dqa[q] * scale;
+        }
     }
 }
 
@@ -741,7 +832,7 @@ jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const 
                              (b.max_ns + kLinS - 1) / kLinS), 256, 0, s>>>(
             tab, pooled, d, ws.z, ws.h, ws.ld_h, sample_target, preds);
     if (b.any_xattn) {
-        const size_t smem = (size_t)b.max_nq * b.max_dq * sizeof(float);
+        const size_t smem = xattn_smem_bytes(b.max_dq);
         k_xattn_fwd<<<b.sample1 - b.sample0, 256, smem, s>>>(tab, b.g0, cu, sample_slot,
                                                              b.sample0, ws.kbuf, ws.vbuf, ws.ldkv,
                                                              ws.P, ws.h, ws.ld_h);
@@ -766,7 +857,7 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
         k_mlp_dw1<<<dim3(b.n, b.max_mlp_hid, (d / 4 + 255) / 256), 256, 0, s>>>(tab, ws.dh,
                                                                                ws.ld_h, pooled, d);
     if (b.any_xattn) {
-        const size_t smem = 2 * (size_t)b.max_nq * b.max_dq * sizeof(float);
+        const size_t smem = xattn_smem_bytes(b.max_dq);
         k_xattn_bwd<<<b.sample1 - b.sample0, 256, smem, s>>>(
             tab, b.g0, cu, sample_slot, b.sample0, ws.kbuf, ws.vbuf, ws.ldkv, ws.P, ws.dS, ws.dh,
             ws.ld_h, ws.dk, ws.dv, ws.dQs);
@@ -782,7 +873,7 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
 
 jnx_status heads_set_smem() {
     static std::atomic<uint64_t> fwd{0}, bwd{0};
-    const int mx = 2 * kMaxQ * 512 * (int)sizeof(float);
+    const int mx = (int)xattn_smem_bytes(512);
     if (set_smem_limit(reinterpret_cast<const void*>(k_xattn_fwd), mx, fwd) != cudaSuccess ||
         set_smem_limit(reinterpret_cast<const void*>(k_xattn_bwd), mx, bwd) != cudaSuccess)
         return cuda_ok("heads smem attribute");
