@@ -87,6 +87,62 @@ jnx_status transpose_launch(const uint16_t* src, int batch, int rows, int cols, 
     return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "transpose: %s", cudaGetErrorString(e));
 }
 
+// Segment-padded transpose: dst [cols][kpad] bf16 with dst[c][p] = src[r][c]
+// for the row r that padded position p stands for: segment i's rows
+// r0_i .. r1_i - 1 sit at positions off_i .. off_i + (r1_i - r0_i) - 1
+// (off_i = sr.tile_start[i], ascending, 64-aligned), every other position is
+// zero.  64 x 64 tiles as k_transpose (cols % 64 == 0, kpad % 64 == 0,
+// 16-byte aligned buffers and strides).
+__global__ void __launch_bounds__(256) k_transpose_seg(const uint16_t* __restrict__ src, int ld_src,
+                                                       const __grid_constant__ SegRows sr, int kpad,
+                                                       uint16_t* __restrict__ dst) {
+    __shared__ uint16_t tile[64][64 + 2];
+    __shared__ int srow[64];
+    const int p0 = blockIdx.y * 64, c0 = blockIdx.x * 64;
+    if (threadIdx.x < 64) {
+        const int p = p0 + threadIdx.x;
+        int lo = 0, hi = sr.n - 1;  // last segment with off <= p
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (sr.tile_start[mid] <= p) lo = mid; else hi = mid - 1;
+        }
+        const int r = sr.r0[lo] + (p - sr.tile_start[lo]);
+        srow[threadIdx.x] = (sr.n > 0 && p >= sr.tile_start[lo] && r < sr.r1[lo]) ? r : -1;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < 64 * 8; i += 256) {
+        const int rr = i / 8, u = i % 8;
+        const int r = srow[rr];
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (r >= 0) v = *reinterpret_cast<const uint4*>(src + (size_t)r * ld_src + c0 + 8 * u);
+        const uint16_t* e = reinterpret_cast<const uint16_t*>(&v);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) tile[rr][8 * u + k] = e[k];
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < 64 * 8; i += 256) {
+        const int c = i / 8, u = i % 8;
+        uint16_t e[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) e[k] = tile[8 * u + k][c];
+        *reinterpret_cast<uint4*>(dst + (size_t)(c0 + c) * kpad + p0 + 8 * u) =
+            *reinterpret_cast<const uint4*>(e);
+    }
+}
+
+jnx_status transpose_seg_launch(const uint16_t* src, int ld_src, int cols, const SegRows& sr,
+                                int kpad, uint16_t* dst, cudaStream_t s) {
+    if (cols <= 0 || cols % 64 || kpad % 64 || ld_src % 8 ||
+        ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15))
+        return fail(JNX_ERR_UNSUPPORTED, "segmented transpose: layout");
+    if (kpad == 0) return JNX_OK;
+    if (kpad / 64 > 65535) return fail(JNX_ERR_UNSUPPORTED, "segmented transpose: too many rows");
+    k_transpose_seg<<<dim3(cols / 64, kpad / 64), 256, 0, s>>>(src, ld_src, sr, kpad, dst);
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? JNX_OK
+                            : fail(JNX_ERR_CUDA, "segmented transpose: %s", cudaGetErrorString(e));
+}
+
 // ---------------------------------------------------------------------------
 // RMSNorm backward: with s = rsqrt(mean(x^2) + eps) and n = x s gamma,
 //   dx = dres + s (gamma dn) - x s^3 mean(gamma dn x)

@@ -965,6 +965,9 @@ struct FlowWs {
     float* lse;               // [nb][M_a, nh]
     uint16_t* m;              // [nb][M_a, F]
     uint16_t* kvc;            // [nb][N, 2 dm]
+    // the context weight gradient on the tensor cores: the hidden rows and
+    // dKV_c transposed, each tenant's rows at a 64-aligned column offset
+    uint16_t *xT, *dkT;       // [d, kpad], [2 dm, kpad]
     // backward scratch
     float *dh, *dn, *dO;      // [M_a, dm]
     uint16_t* dh_bf;          // [M_a, dm]
@@ -976,7 +979,7 @@ struct FlowWs {
     size_t bytes;
 };
 
-FlowWs carve_flow(const FlowDims& d, int S, int N, void* base) {
+FlowWs carve_flow(const FlowDims& d, int S, int N, int n_slots, void* base) {
     uint8_t* p = static_cast<uint8_t*>(base);
     FlowWs w{};
     size_t off = 0;
@@ -1020,6 +1023,9 @@ FlowWs carve_flow(const FlowDims& d, int S, int N, void* base) {
     w.wt = b16((size_t)d.T * std::max(3 * dm * dm, 2 * (size_t)d.F * dm));
     w.dphi = f32(s * dm);
     w.dz1 = f32(s * dm);
+    const size_t kpad = (n + 63) / 64 * 64 + 64 * (size_t)std::max(n_slots, 0);
+    w.xT = b16((size_t)d.d * kpad);
+    w.dkT = b16(2 * dm * kpad);
     w.bytes = off;
     return w;
 }
@@ -1294,7 +1300,7 @@ extern "C" size_t jnx_flow_workspace_bytes(const jnx_flow_head* fh, const jnx_gr
     if (!fh || !g) return 0;
     FlowDims d{fh->d_model, fh->d_ff, fh->n_blocks, fh->chunk, fh->action_dim, fh->d_in,
                fh->n_tenants, fh->d_model / kHd};
-    return carve_flow(d, g->n_samples, g->n_tokens, nullptr).bytes;
+    return carve_flow(d, g->n_samples, g->n_tokens, g->n_slots, nullptr).bytes;
 }
 
 static jnx_status flow_begin(const jnx_flow_head* fh, const jnx_group* g, const uint16_t* hidden,
@@ -1305,7 +1311,7 @@ static jnx_status flow_begin(const jnx_flow_head* fh, const jnx_group* g, const 
         return fail(JNX_ERR_INVALID_ARG, "flow: null workspace or hidden rows");
     if (reinterpret_cast<uintptr_t>(workspace) & 255)
         return fail(JNX_ERR_INVALID_ARG, "flow: workspace must be 256-byte aligned");
-    w = carve_flow(d, g->n_samples, g->n_tokens, workspace);
+    w = carve_flow(d, g->n_samples, g->n_tokens, g->n_slots, workspace);
     if (ws_bytes < w.bytes)
         return fail(JNX_ERR_WORKSPACE, "flow: workspace %zu < %zu bytes", ws_bytes, w.bytes);
     return JNX_OK;
@@ -1420,6 +1426,21 @@ extern "C" jnx_status jnx_flow_backward(const jnx_flow_head* fh, const jnx_group
         rt.r0[i] = sg.t0[i];
         rt.r1[i] = sg.t1[i];
     }
+    // the context weight gradient dW_kvc[t] = dKV_c^T X over tenant t's token
+    // rows runs as one tcgen05 GEMM per tenant (K = its rows, padded to 64)
+    // on transposed copies; widths that are not a multiple of 256 keep the
+    // mma.sync segmented kernel
+    const bool tc_kvc = d.d % 256 == 0;
+    static thread_local SegRows rp;  // token-row segments at padded offsets
+    rp = rt;
+    std::vector<int> kp(nsl);
+    int kpad = 0;
+    for (int i = 0; i < nsl; ++i) {
+        rp.tile_start[i] = kpad;
+        kp[i] = (rt.r1[i] - rt.r0[i] + 63) / 64 * 64;
+        kpad += kp[i];
+    }
+    if (tc_kvc && (st = transpose_seg_launch(hidden, d.d, d.d, rp, kpad, w.xT, s))) return st;
     // output layer
     {
         TraceScope ts(JNX_K_FLOW_MISC, (double)Ma * dm * d.D * 4.0, s);
@@ -1541,10 +1562,41 @@ extern "C" jnx_status jnx_flow_backward(const jnx_flow_head* fh, const jnx_group
             TraceScope ts(JNX_K_FLOW_WGRAD,
                           2.0 * Ma * 3 * dm * dm + 2.0 * g->n_tokens * 2 * dm * d.d, s);
             if ((st = seg_wgrad_launch(ra, w.dqkv, 3 * dm, n1, dm, 3 * dm, dm, G.w_qkv,
-                                       (long long)3 * dm * dm, add, s)) ||
-                (st = seg_wgrad_launch(rt, w.dkvc, 2 * dm, hidden, d.d, 2 * dm, d.d, G.w_kvc,
-                                       (long long)2 * dm * d.d, add, s)))
+                                       (long long)3 * dm * dm, add, s)))
                 return st;
+            if (!tc_kvc) {
+                if ((st = seg_wgrad_launch(rt, w.dkvc, 2 * dm, hidden, d.d, 2 * dm, d.d,
+                                           G.w_kvc, (long long)2 * dm * d.d, add, s)))
+                    return st;
+            } else {
+                if ((st = transpose_seg_launch(w.dkvc, 2 * dm, 2 * dm, rp, kpad, w.dkT, s)))
+                    return st;
+                for (int i = 0; i < nsl; ++i) {
+                    float* gw = G.w_kvc + (size_t)rt.tenant[i] * 2 * dm * d.d;
+                    if (kp[i] == 0) {  // no context rows: a zero gradient
+                        if (!add && cudaMemsetAsync(gw, 0, sizeof(float) * 2 * dm * d.d, s))
+                            return last("flow context weight gradient");
+                        continue;
+                    }
+                    GemmParams q{};
+                    q.M = 2 * dm;
+                    q.N = d.d;
+                    q.K = kp[i];
+                    q.status = w.status;
+                    if (add) {
+                        q.epi = EPI_RESID;
+                        q.resid = gw;
+                        q.ldr = d.d;
+                    } else {
+                        q.epi = EPI_F32;
+                        q.out = gw;
+                        q.ldo = d.d;
+                    }
+                    if ((st = gemm_launch(w.dkT + rp.tile_start[i], kpad, w.xT + rp.tile_start[i],
+                                          kpad, q, s)))
+                        return st;
+                }
+            }
         }
         {
             TraceScope ts(JNX_K_FLOW_GEMM, 2.0 * Ma * dm * 3 * dm, s);

@@ -71,6 +71,10 @@ jnx_status seg_tn_launch(const jnx_group* g, const uint16_t* U, int ldu, const u
                          long long gstride, bool trans, bool add, cudaStream_t s);
 // For every segment i of sr (rows [r0, r1), tenant): G[tenant][m, n] = (or
 // +=) sum over the rows of U[row, m] V[row, n]; m % 64 == 0, n % 128 == 0.
+// dst [cols][kpad] bf16: segment i's rows of src [*, ld_src] transposed to
+// columns sr.tile_start[i] .. (64-aligned, ascending), zero elsewhere.
+jnx_status transpose_seg_launch(const uint16_t* src, int ld_src, int cols, const SegRows& sr,
+                                int kpad, uint16_t* dst, cudaStream_t s);
 jnx_status seg_wgrad_launch(const SegRows& sr, const uint16_t* U, int ldu, const uint16_t* V,
                             int ldv, int m, int n, float* grad, long long gstride, bool add,
                             cudaStream_t s);
