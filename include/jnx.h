@@ -263,7 +263,11 @@ size_t jnx_backbone_workspace_bytes(const jnx_backbone* bb, int32_t n_tokens);
  * vision [n_vision_rows, d] bf16 and text_ids [n_text] int32 are the
  * caller's observation buffers that gather_src indexes.  A gather index
  * outside them, or a text id outside [0, vocab), sets
- * JNX_ERR_DEVICE_BOUNDS in the status word and the row is zero-filled. */
+ * JNX_ERR_DEVICE_BOUNDS in the status word and the row is zero-filled.
+ * The call uploads the group's attention work list from host memory, so it
+ * cannot be captured into a CUDA graph: on a capturing stream it returns
+ * JNX_ERR_UNSUPPORTED before any launch (as do jnx_backbone_forward_train,
+ * jnx_backbone_backward_lora and jnx_op_attention_backward). */
 jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_group* g,
                                 const uint16_t* vision, int64_t n_vision_rows,
                                 const int32_t* text_ids, int64_t n_text,

@@ -70,6 +70,22 @@ jnx_status cuda_status(const char* what) {
 
 }  // namespace
 
+// A call that uploads a per-group work list from host memory (the attention
+// items) cannot be captured into a CUDA graph: the graph would replay the
+// copy from a host buffer that is gone by then.  Refused before any launch.
+jnx_status jnx::refuse_capture(cudaStream_t s, const char* what) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(s, &cs) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(JNX_ERR_UNSUPPORTED, "%s: cannot tell whether the stream is capturing", what);
+    }
+    if (cs != cudaStreamCaptureStatusNone)
+        return fail(JNX_ERR_UNSUPPORTED,
+                    "%s: cannot be captured into a CUDA graph (it uploads a per-group work list "
+                    "from host memory)", what);
+    return JNX_OK;
+}
+
 namespace jnx {
 
 jnx_status check_backbone(const jnx_backbone* bb) {
@@ -175,6 +191,7 @@ static jnx_status backbone_forward(const jnx_backbone* bb, const jnx_group* g,
             return fail(JNX_ERR_INVALID_ARG, "backbone: tenant %d has no LoRA adapter",
                         g->h_slot_tenant[i]);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if ((st = refuse_capture(s, "backbone"))) return st;
     const int qkvw = (H + 2 * Hkv) * hd;
 
     const double Nd = (double)N * d;

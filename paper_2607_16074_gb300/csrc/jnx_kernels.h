@@ -159,6 +159,9 @@ jnx_status rope_table_launch(float2* tab, int max_pos, int hd, float theta, cuda
 // the backward uses to recompute the probabilities.
 // Attention work items (sample, 128-row tile) of a group, most expensive first.
 jnx_status build_attn_items(const jnx_group* g, std::vector<int2>& sorted);
+// JNX_ERR_UNSUPPORTED when s is capturing into a CUDA graph (for the calls
+// that upload a work list from host memory).
+jnx_status refuse_capture(cudaStream_t s, const char* what);
 
 jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv, int hd,
                             const int* cu, int S, int max_seqlen, const int2* items, int n_items,

@@ -156,6 +156,7 @@ extern "C" jnx_status jnx_backbone_backward_lora(const jnx_backbone* bb, const j
         return fail(JNX_ERR_WORKSPACE, "backward: workspace %zu < %zu bytes", ws_bytes, w.bytes);
     if (N == 0) return JNX_OK;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if ((st = refuse_capture(s, "backward"))) return st;
     const bool add = accumulate != 0;
     const double Nd = (double)N * d;
 
@@ -491,6 +492,7 @@ extern "C" jnx_status jnx_op_attention_backward(const uint16_t* qkv, const uint1
     g.h_cu_seqlens = h_cu_seqlens;
     std::vector<int2> items;
     jnx_status st;
+    if ((st = refuse_capture(s, "attention backward"))) return st;
     if ((st = build_attn_items(&g, items))) return st;
     if (!items.empty() && cudaMemcpyAsync(items_d, items.data(), items.size() * sizeof(int2),
                                           cudaMemcpyHostToDevice, s) != cudaSuccess)

@@ -428,3 +428,24 @@ def test_inference_path_matches_training_forward_and_is_grouping_invariant():
         width = w.tenants[t].width
         for o in offs:
             assert torch.equal(pr1.view(-1)[o:o + width], preds.view(-1)[o:o + width]), (t, o)
+
+
+@pytest.mark.filterwarnings("ignore:The CUDA Graph is empty")
+def test_backbone_forward_refuses_cuda_graph_capture():
+    """The backbone forward uploads its attention work list from host memory;
+    a CUDA graph would replay that copy from a freed host buffer, so a
+    capturing stream is refused before any launch (and nothing is replayed
+    here).  The same step still runs eagerly afterwards."""
+    s = Setup(synth.make_workload("tiny"))
+    plan, step, preds = s.run()
+    stream = torch.cuda.Stream()
+    graph = torch.cuda.CUDAGraph()
+    with pytest.raises(J.JnxError, match="CUDA graph"):
+        with torch.cuda.graph(graph, stream=stream):
+            step.run(s.inp_d["vision"], s.inp_d["text_ids"], s.inp_d["targets"], preds)
+    del graph
+    torch.cuda.synchronize()
+    preds2 = torch.full_like(preds, float("nan"))
+    step.run(s.inp_d["vision"], s.inp_d["text_ids"], s.inp_d["targets"], preds2)
+    torch.cuda.synchronize()
+    assert torch.equal(preds2, preds)
