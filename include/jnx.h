@@ -203,7 +203,21 @@ typedef struct {
     const int32_t* h_cu_seqlens;   /* host   [n_samples + 1] */
     const int32_t* h_seg_offsets;  /* host   [n_slots + 1] */
     const int32_t* h_slot_tenant;  /* host   [n_slots] */
+    /* Optional: the group's attention work list on the device, [n_attn_items]
+     * (sample, 128-row tile) int32 pairs exactly as jnx_group_attn_items
+     * writes them, 8-byte aligned.  When it is set, the backbone forward and
+     * backward read it instead of uploading their own copy, which makes them
+     * capturable into a CUDA graph; NULL (and 0) keeps the upload. */
+    const int32_t* attn_items;
+    int32_t n_attn_items;
 } jnx_group;
+
+/* The group's attention work list on the host: (sample, 128-row tile) pairs,
+ * the most expensive first, into out[2 * cap].  Returns the number of pairs;
+ * when out is NULL or cap is smaller, writes nothing and returns that number
+ * (call again with room); < 0 on an invalid group.  Needs n_samples,
+ * n_tokens and h_cu_seqlens only. */
+int32_t jnx_group_attn_items(const jnx_group* g, int32_t* out, int32_t cap);
 
 /* ------------------------------------------------------------------------
  * Shared frozen backbone
@@ -264,10 +278,12 @@ size_t jnx_backbone_workspace_bytes(const jnx_backbone* bb, int32_t n_tokens);
  * caller's observation buffers that gather_src indexes.  A gather index
  * outside them, or a text id outside [0, vocab), sets
  * JNX_ERR_DEVICE_BOUNDS in the status word and the row is zero-filled.
- * The call uploads the group's attention work list from host memory, so it
- * cannot be captured into a CUDA graph: on a capturing stream it returns
- * JNX_ERR_UNSUPPORTED before any launch (as do jnx_backbone_forward_train,
- * jnx_backbone_backward_lora and jnx_op_attention_backward). */
+ * Without the group's attn_items the call uploads the attention work list
+ * from host memory, which a CUDA graph cannot replay: on a capturing stream
+ * it then returns JNX_ERR_UNSUPPORTED before any launch (as do
+ * jnx_backbone_forward_train and jnx_backbone_backward_lora, and
+ * jnx_op_attention_backward always).  With attn_items set the forward and
+ * the backward are capturable. */
 jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_group* g,
                                 const uint16_t* vision, int64_t n_vision_rows,
                                 const int32_t* text_ids, int64_t n_text,

@@ -135,6 +135,34 @@ jnx_status check_group(const jnx_group* g) {
         return fail(JNX_ERR_INVALID_ARG, "group: null slot array");
     if (g->max_seqlen > kMaxRopePos)
         return fail(JNX_ERR_UNSUPPORTED, "group: sample longer than %d tokens", kMaxRopePos);
+    if (g->n_attn_items < 0 || (g->n_attn_items > 0 && !g->attn_items) ||
+        (reinterpret_cast<uintptr_t>(g->attn_items) & 7))
+        return fail(JNX_ERR_INVALID_ARG, "group: bad attention work list");
+    return JNX_OK;
+}
+
+// The work list the attention launches take: the group's own device copy
+// when it has one (checked against the plan), else `upload` (uploaded here
+// from host memory, which a capturing stream refuses).
+jnx_status attn_items_for(const jnx_group* g, int2* upload, cudaStream_t s, const char* what,
+                          const int2*& items, int& n_items) {
+    jnx_status st;
+    std::vector<int2> sorted;
+    if ((st = build_attn_items(g, sorted))) return st;
+    n_items = (int)sorted.size();
+    if (g->attn_items) {
+        if (g->n_attn_items != n_items)
+            return fail(JNX_ERR_INVALID_ARG, "%s: the group's work list has %d items, its plan %d",
+                        what, g->n_attn_items, n_items);
+        items = reinterpret_cast<const int2*>(g->attn_items);
+        return JNX_OK;
+    }
+    if ((st = refuse_capture(s, what))) return st;
+    if (n_items && cudaMemcpyAsync(upload, sorted.data(), sorted.size() * sizeof(int2),
+                                   cudaMemcpyHostToDevice, s) != cudaSuccess)
+        return fail(JNX_ERR_CUDA, "%s: attention items: %s", what,
+                    cudaGetErrorString(cudaGetLastError()));
+    items = upload;
     return JNX_OK;
 }
 
@@ -191,7 +219,9 @@ static jnx_status backbone_forward(const jnx_backbone* bb, const jnx_group* g,
             return fail(JNX_ERR_INVALID_ARG, "backbone: tenant %d has no LoRA adapter",
                         g->h_slot_tenant[i]);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if ((st = refuse_capture(s, "backbone"))) return st;
+    const int2* items = nullptr;
+    int n_items = 0;
+    if ((st = attn_items_for(g, w.attn_items, s, "backbone", items, n_items))) return st;
     const int qkvw = (H + 2 * Hkv) * hd;
 
     const double Nd = (double)N * d;
@@ -239,15 +269,6 @@ static jnx_status backbone_forward(const jnx_backbone* bb, const jnx_group* g,
     for (int i = 0; i < g->n_samples; ++i) {
         const double L = g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i];
         attn_flops += 4.0 * L * L * H * hd;
-    }
-    int n_items = 0;
-    {
-        std::vector<int2> sorted;
-        if ((st = build_attn_items(g, sorted))) return st;
-        n_items = (int)sorted.size();
-        if (n_items && cudaMemcpyAsync(w.attn_items, sorted.data(), sorted.size() * sizeof(int2),
-                                       cudaMemcpyHostToDevice, s) != cudaSuccess)
-            return cuda_status("backbone: attention items");
     }
 
     // Fold an RMSNorm into the residual GEMM before it only where that GEMM's
@@ -317,7 +338,7 @@ static jnx_status backbone_forward(const jnx_backbone* bb, const jnx_group* g,
         {
             TraceScope ts(JNX_K_ATTN, attn_flops, s);
             if ((st = attention_launch(w.qkv, qkvw, N, H, Hkv, hd, g->cu_seqlens, g->n_samples,
-                                       g->max_seqlen, w.attn_items, n_items, w.att, H * hd,
+                                       g->max_seqlen, items, n_items, w.att, H * hd,
                                        nullptr, w.status, s)))
                 return st;
         }
@@ -390,6 +411,24 @@ static jnx_status backbone_forward(const jnx_backbone* bb, const jnx_group* g,
                                   (pooled ? (double)g->n_samples * d * 4.0 : 0.0), s);
     return final_pool_launch(w.x, bb->final_norm, bb->eps, g->cu_seqlens, g->n_samples, d, pooled,
                              hidden, s);
+}
+
+extern "C" int32_t jnx_group_attn_items(const jnx_group* g, int32_t* out, int32_t cap) {
+    clear_error();
+    if (!g || g->n_samples < 0 || g->n_tokens < 0 || (g->n_samples > 0 && !g->h_cu_seqlens)) {
+        fail(JNX_ERR_INVALID_ARG, "group attention items: bad group");
+        return JNX_ERR_INVALID_ARG;
+    }
+    std::vector<int2> sorted;
+    jnx_status st = build_attn_items(g, sorted);
+    if (st) return st;
+    const int32_t n = (int32_t)sorted.size();
+    if (!out || cap < n) return n;
+    for (int32_t i = 0; i < n; ++i) {
+        out[2 * i] = sorted[i].x;
+        out[2 * i + 1] = sorted[i].y;
+    }
+    return n;
 }
 
 extern "C" jnx_status jnx_backbone_forward(const jnx_backbone* bb, const jnx_group* g,

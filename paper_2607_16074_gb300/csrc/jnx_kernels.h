@@ -162,6 +162,10 @@ jnx_status build_attn_items(const jnx_group* g, std::vector<int2>& sorted);
 // JNX_ERR_UNSUPPORTED when s is capturing into a CUDA graph (for the calls
 // that upload a work list from host memory).
 jnx_status refuse_capture(cudaStream_t s, const char* what);
+// The attention work list for g: its own device copy if it has one, else
+// uploaded into `upload` (refused on a capturing stream).
+jnx_status attn_items_for(const jnx_group* g, int2* upload, cudaStream_t s, const char* what,
+                          const int2*& items, int& n_items);
 
 jnx_status attention_launch(const uint16_t* qkv, int ldq, int n_tokens, int H, int Hkv, int hd,
                             const int* cu, int S, int max_seqlen, const int2* items, int n_items,

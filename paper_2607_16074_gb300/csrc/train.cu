@@ -156,7 +156,6 @@ extern "C" jnx_status jnx_backbone_backward_lora(const jnx_backbone* bb, const j
         return fail(JNX_ERR_WORKSPACE, "backward: workspace %zu < %zu bytes", ws_bytes, w.bytes);
     if (N == 0) return JNX_OK;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if ((st = refuse_capture(s, "backward"))) return st;
     const bool add = accumulate != 0;
     const double Nd = (double)N * d;
 
@@ -165,14 +164,8 @@ extern "C" jnx_status jnx_backbone_backward_lora(const jnx_backbone* bb, const j
         if ((st = rope_table_launch(w.rope, g->max_seqlen, hd, bb->rope_theta, s))) return st;
     }
     int n_items = 0;
-    {
-        std::vector<int2> items;
-        if ((st = build_attn_items(g, items))) return st;
-        n_items = (int)items.size();
-        if (n_items && cudaMemcpyAsync(w.items, items.data(), items.size() * sizeof(int2),
-                                       cudaMemcpyHostToDevice, s) != cudaSuccess)
-            return cuda_ok("backward: attention items");
-    }
+    const int2* items = nullptr;
+    if ((st = attn_items_for(g, w.items, s, "backward", items, n_items))) return st;
     double attn_flops = 0.0;
     for (int i = 0; i < g->n_samples; ++i) {
         const double L = g->h_cu_seqlens[i + 1] - g->h_cu_seqlens[i];
@@ -252,7 +245,7 @@ extern "C" jnx_status jnx_backbone_backward_lora(const jnx_backbone* bb, const j
         {
             TraceScope ts(JNX_K_ATTN, attn_flops, s);
             if ((st = attention_launch(w.qkv, qkvw, N, H, Hkv, hd, g->cu_seqlens, g->n_samples,
-                                       g->max_seqlen, w.items, n_items, w.att, Hhd, w.lse,
+                                       g->max_seqlen, items, n_items, w.att, Hhd, w.lse,
                                        w.status, s)))
                 return st;
         }
@@ -368,7 +361,7 @@ extern "C" jnx_status jnx_backbone_backward_lora(const jnx_backbone* bb, const j
             TraceScope ts(JNX_K_ATTN_BWD, 2.5 * attn_flops, s);
             if ((st = attention_bwd_launch(w.qkv, qkvw, w.dO, w.lse, w.Dsum, N, H, Hkv, hd,
                                            g->cu_seqlens, g->pos_ids, w.rope, g->max_seqlen,
-                                           w.items, n_items, w.dqkv, w.status, s)))
+                                           items, n_items, w.dqkv, w.status, s)))
                 return st;
         }
 

@@ -79,7 +79,8 @@ class jnx_group(C.Structure):
                 ("cu_seqlens", C.c_void_p), ("sample_slot", C.c_void_p),
                 ("sample_target", C.c_void_p), ("seg_offsets", C.c_void_p),
                 ("gather_src", C.c_void_p), ("pos_ids", C.c_void_p),
-                ("h_cu_seqlens", P32), ("h_seg_offsets", P32), ("h_slot_tenant", P32)]
+                ("h_cu_seqlens", P32), ("h_seg_offsets", P32), ("h_slot_tenant", P32),
+                ("attn_items", C.c_void_p), ("n_attn_items", C.c_int32)]
 
 
 class jnx_layer(C.Structure):
@@ -166,7 +167,8 @@ class jnx_adam_tensor(C.Structure):
 
 _LIB: Optional[C.CDLL] = None
 
-EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_backbone_workspace_bytes",
+EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_group_attn_items",
+           "jnx_backbone_workspace_bytes",
            "jnx_backbone_forward", "jnx_heads_workspace_bytes", "jnx_heads_forward",
            "jnx_heads_backward", "jnx_check_status", "jnx_pack_gate_up", "jnx_op_pack",
            "jnx_op_rmsnorm", "jnx_op_gemm_workspace_bytes", "jnx_op_gemm", "jnx_op_attention",
@@ -196,6 +198,7 @@ def lib() -> C.CDLL:
         "jnx_version": (i32, []),
         "jnx_group_plan": (i32, [C.POINTER(jnx_schema), i32, C.POINTER(jnx_request), i32, i32,
                                  C.POINTER(jnx_limits), C.POINTER(jnx_plan)]),
+        "jnx_group_attn_items": (i32, [C.POINTER(jnx_group), vp, i32]),
         "jnx_sched_poll": (i32, [C.POINTER(jnx_schema), i32, C.POINTER(jnx_request),
                                  C.POINTER(C.c_double), i32, i32, C.c_double,
                                  C.POINTER(jnx_sched_policy), P32, C.POINTER(C.c_int32),

@@ -41,7 +41,23 @@ class DeviceGroup:
         self.struct = J.jnx_group(
             plan.n_samples, plan.n_tokens, plan.n_slots, plan.max_seqlen,
             *[self.d[k].data_ptr() or None for k in self.DEV],
-            hp("cu_seqlens"), hp("seg_offsets"), hp("slot_tenant"))
+            hp("cu_seqlens"), hp("seg_offsets"), hp("slot_tenant"), None, 0)
+        # the attention work list on the device too, so the backbone's calls
+        # read it instead of uploading it (and can be captured into a graph)
+        L = J.lib()
+        n = L.jnx_group_attn_items(C.byref(self.struct), None, 0)
+        if n < 0:
+            J.check(n)
+        items = np.zeros(2 * max(n, 1), dtype=np.int32)
+        got = L.jnx_group_attn_items(C.byref(self.struct), items.ctypes.data, n)
+        if got != n:
+            J.check(got if got < 0 else J.JNX_ERR_INVALID_ARG)
+        t = torch.from_numpy(items)
+        if non_blocking:
+            t = t.pin_memory()
+        self.d["attn_items"] = t.to(device, non_blocking=non_blocking)
+        self.struct.attn_items = self.d["attn_items"].data_ptr() if n else None
+        self.struct.n_attn_items = n
 
     @property
     def ref(self):

@@ -135,6 +135,33 @@ def _host_flow_head(d_model):
     return fh, blocks
 
 
+def test_group_attention_work_list():
+    """jnx_group_attn_items: every (sample, 128-row tile) of the group once,
+    the most expensive first (a sample's cost is its 64-row key tiles), with
+    the two-call size query."""
+    import ctypes as C
+    L = J.lib()
+    w = synth.make_workload("small")
+    plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), len(w.tenants), w.max_samples,
+                            w.max_tokens)
+    cu = np.ascontiguousarray(plan.cu_seqlens, dtype=np.int32)
+    g = J.jnx_group(plan.n_samples, plan.n_tokens, 0, plan.max_seqlen, *([None] * 6),
+                    cu.ctypes.data_as(J.P32), None, None)
+    n = L.jnx_group_attn_items(C.byref(g), None, 0)
+    lens = np.diff(cu)
+    assert n == int(sum((l + 127) // 128 for l in lens))
+    out = np.full(2 * n, -1, dtype=np.int32)
+    assert L.jnx_group_attn_items(C.byref(g), out.ctypes.data, n - 1) == n  # too small: nothing
+    assert (out == -1).all()
+    assert L.jnx_group_attn_items(C.byref(g), out.ctypes.data, n) == n
+    pairs = out.reshape(n, 2)
+    want = sorted((i, t) for i, l in enumerate(lens) for t in range((l + 127) // 128))
+    assert sorted(map(tuple, pairs.tolist())) == want
+    cost = [(lens[i] + 63) // 64 for i, _ in pairs]
+    assert all(a >= b for a, b in zip(cost, cost[1:]))
+    assert L.jnx_group_attn_items(None, None, 0) == J.JNX_ERR_INVALID_ARG
+
+
 def test_training_entry_points_reject_bad_arguments_without_a_gpu():
     import ctypes as C
     L = J.lib()

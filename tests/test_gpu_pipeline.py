@@ -431,13 +431,15 @@ def test_inference_path_matches_training_forward_and_is_grouping_invariant():
 
 
 @pytest.mark.filterwarnings("ignore:The CUDA Graph is empty")
-def test_backbone_forward_refuses_cuda_graph_capture():
-    """The backbone forward uploads its attention work list from host memory;
-    a CUDA graph would replay that copy from a freed host buffer, so a
-    capturing stream is refused before any launch (and nothing is replayed
-    here).  The same step still runs eagerly afterwards."""
+def test_backbone_forward_without_a_device_work_list_refuses_graph_capture():
+    """Without the group's device copy of the attention work list the
+    backbone forward uploads it from host memory, which a CUDA graph would
+    replay from a freed buffer: a capturing stream is refused before any
+    launch (nothing is replayed here), and the step still runs eagerly."""
     s = Setup(synth.make_workload("tiny"))
     plan, step, preds = s.run()
+    step.group.struct.attn_items = None
+    step.group.struct.n_attn_items = 0
     stream = torch.cuda.Stream()
     graph = torch.cuda.CUDAGraph()
     with pytest.raises(J.JnxError, match="CUDA graph"):
@@ -449,3 +451,33 @@ def test_backbone_forward_refuses_cuda_graph_capture():
     step.run(s.inp_d["vision"], s.inp_d["text_ids"], s.inp_d["targets"], preds2)
     torch.cuda.synchronize()
     assert torch.equal(preds2, preds)
+
+
+@pytest.mark.parametrize("name", ["tiny", "mqa2b"])
+def test_grouped_step_replays_as_a_cuda_graph(name):
+    """With the group's work list on the device the whole grouped step
+    (backbone, heads forward, loss, heads backward) is captured once and
+    replayed; the replay gives the eager step's predictions, losses and head
+    gradients bit for bit."""
+    w = synth.make_workload(name, n_layers=1) if name != "tiny" else synth.make_workload(name)
+    s = Setup(w, gen_device="cuda")
+    plan, step, preds = s.run()
+    want_p, want_l = preds.clone(), step.loss.clone()
+    want_g = [{k: v.clone() for k, v in g.items()} for g in s.heads.grads]
+    stream = torch.cuda.Stream()
+    stream.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        step.run(s.inp_d["vision"], s.inp_d["text_ids"], s.inp_d["targets"], preds)
+    preds.fill_(float("nan"))
+    for g in s.heads.grads:
+        for v in g.values():
+            v.fill_(7.0)
+    graph.replay()
+    torch.cuda.synchronize()
+    R.check_status(step.ws_bb)
+    R.check_status(step.ws_h)
+    assert torch.equal(preds, want_p) and torch.equal(step.loss, want_l)
+    for g, wg in zip(s.heads.grads, want_g):
+        for k in g:
+            assert torch.equal(g[k], wg[k]), k
