@@ -474,6 +474,11 @@ def run_ours(args, rank, world, local_rank):
                      per_tenant_tokens_per_s=round(tokens / (t_iso / 1e3), 1))
         del iso
 
+    # ---- CUDA-graph replay (--graphs): the same steps captured once ---------
+    graphs = None
+    if args.graphs:
+        graphs = graph_timings(args, step, inp, preds, plan, backbone, heads, w, dev, stream)
+
     # ---- roofline of the dominant kernel (all backbone GEMM launches) ------
     peaks = load_peaks()
     gemm_mask = np.isin(kinds, (3, 5, 6, 7))
@@ -540,6 +545,69 @@ def run_ours(args, rank, world, local_rank):
         kernels=per_kernel,
         cpu_baseline=cpu,
     )
+    if graphs is not None:
+        out["graphs"] = graphs
+    return out
+
+
+def graph_timings(args, step, inp, preds, plan, backbone, heads, w, dev, stream):
+    """The grouped step, and the per-tenant steps back to back, each captured
+    once into a CUDA graph and replayed: K replays timed with CUDA events
+    (launch overheads gone from both arms), with the grouped replay's
+    predictions checked against the eager step's."""
+    import torch
+
+    from paper_2607_16074_gb300 import jnx as J
+    from paper_2607_16074_gb300 import runtime as R
+
+    def capture(fn):
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            fn()
+        torch.cuda.synchronize()
+        return g
+
+    def replay_ms(g):
+        for _ in range(max(args.warmup, 3)):
+            g.replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / args.steps
+
+    run = lambda st: st.run(inp["vision"], inp["text_ids"], inp["targets"], preds)
+    run(step)
+    torch.cuda.synchronize()
+    want = preds.clone()
+    g = capture(lambda: run(step))
+    t_g = replay_ms(g)
+    same = bool(torch.equal(preds, want))
+    out = dict(ms_per_step=round(t_g, 4),
+               value=round(plan.n_tokens / (t_g / 1e3), 1), unit="tokens/s",
+               replay_equals_eager=same)
+    del g
+    if not args.no_per_tenant:
+        iso = []
+        for t in range(len(w.tenants)):
+            sub = w.subset([t])
+            p = J.jnx_group_plan(sub.schemas(), oracle_requests(sub), len(w.tenants),
+                                 w.max_samples, w.max_tokens)
+            if p.n_samples:
+                iso.append(R.GroupedStep(backbone, heads, R.DeviceGroup(p, device=dev),
+                                         device=dev))
+        for st in iso:
+            run(st)
+        torch.cuda.synchronize()
+        gi = capture(lambda: [run(st) for st in iso])
+        t_i = replay_ms(gi)
+        del gi, iso
+        out.update(per_tenant_ms=round(t_i, 4), speedup=round(t_i / t_g, 4))
     return out
 
 
@@ -859,6 +927,26 @@ def run_grid(args):
             ts.append(a.elapsed_time(e))
         return float(np.median(ts))
 
+    def graph_timed(fns):
+        # the same launches captured once into a CUDA graph, then replayed
+        for f in fns:
+            f()
+        cs = torch.cuda.Stream()
+        cs.wait_stream(s)
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=cs):
+            for f in fns:
+                f()
+        torch.cuda.synchronize()
+        t = timed([gr.replay])
+        del gr
+        return t
+
+    if args.graphs:
+        timed_arm = graph_timed
+    else:
+        timed_arm = timed
+
     grid = {}
     for T in (2, 4, 6, 8):
         for b in (1, 2, 4, 8):
@@ -868,7 +956,7 @@ def run_grid(args):
             plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), T_max, w.max_samples,
                                     w.max_tokens)
             g = R.GroupedStep(backbone, heads, R.DeviceGroup(plan, device=dev), device=dev)
-            grouped = timed([lambda g=g: g.infer(inp["vision"], inp["text_ids"], preds)])
+            grouped = timed_arm([lambda g=g: g.infer(inp["vision"], inp["text_ids"], preds)])
             serial_steps = []
             for t in range(T):
                 sub = w.subset([t])
@@ -876,8 +964,8 @@ def run_grid(args):
                                       w.max_tokens)
                 serial_steps.append(R.GroupedStep(backbone, heads, R.DeviceGroup(p1, device=dev),
                                                   device=dev))
-            serial = timed([lambda st=st: st.infer(inp["vision"], inp["text_ids"], preds)
-                            for st in serial_steps])
+            serial = timed_arm([lambda st=st: st.infer(inp["vision"], inp["text_ids"], preds)
+                                for st in serial_steps])
             R.check_status(g.ws_bb)
             grid[f"{T}x{b}"] = dict(tenants=T, local_batch=b, tokens=plan.n_tokens,
                                     grouped_ms=round(grouped, 3), serial_ms=round(serial, 3),
@@ -887,7 +975,7 @@ def run_grid(args):
             torch.cuda.empty_cache()
     return dict(metric="grouped vs serial inference forward speedup, tenants x local batch",
                 unit="x", higher_is_better=True, n_gpus=1, steps=args.steps,
-                warmup=args.warmup, data="synthetic",
+                warmup=args.warmup, data="synthetic", cuda_graphs=bool(args.graphs),
                 config={"workload": "2B-class backbone (18 blocks, d=2048, MQA 8x256, GeGLU "
                                     "16384), MLP heads; samples = 1 image (256 rows) + 16..64 "
                                     "text tokens"},
@@ -924,6 +1012,8 @@ def main():
                     help="grouped vs serial inference on the tenants x local batch grid")
     ap.add_argument("--train-lora", action="store_true",
                     help="time the per-tenant LoRA training step (use with --workload zipf2b)")
+    ap.add_argument("--graphs", action="store_true",
+                    help="also time the grouped and per-tenant steps as CUDA-graph replays")
     ap.add_argument("--flow", action="store_true",
                     help="time flow-matching DiT experts as the tenants' modules")
     ap.add_argument("--flow-tenants", type=int, default=8)
