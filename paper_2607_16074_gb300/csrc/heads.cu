@@ -16,6 +16,8 @@
 //   dWout = dy^T h, dbout = sum dy, dO = dy Wout,
 //   dP = dO v^T, dS = P * (dP - rowsum(dP * P)), dv = P^T dO,
 //   dk = dS^T Q / sqrt(dq), dQ = sum_s dS k / sqrt(dq), dWk = dk^T X, dWv = dv^T X
+//   (the weight gradients formed through the queries per sample:
+//    dWk = Q^T (sum_s dS_s^T X_s) / sqrt(dq), dWv = sum_s dO_s^T (P_s^T X_s))
 // Loss (both): l_t = sum (y - t)^2 / (n_t * width), dy = 2 (y - t) / (n_t width).
 // All sums run in a fixed order inside one thread or one CTA (no atomics),
 // so a tenant's results are identical whether it runs grouped or alone.
