@@ -447,6 +447,8 @@ def run_ours(args, rank, world, local_rank):
     step.group = group
     e2e_plan_bytes = sum(a.nbytes for a in (plan.cu_seqlens, plan.sample_slot, plan.sample_target,
                                             plan.seg_offsets, plan.gather_src, plan.pos_ids))
+    # each step's group also uploads its attention work list
+    e2e_plan_bytes += group.d["attn_items"].numel() * 4
 
     # ---- per-tenant isolated execution (the speedup's baseline) -----------
     speed = None
