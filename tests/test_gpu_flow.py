@@ -118,10 +118,10 @@ def _check(s, plan, hidden, inp, vel, loss, tol, only=None):
             assert _rel_l2(gu, GB["wu"]) < tol, ("grad", t, b, "wu", _rel_l2(gu, GB["wu"]))
 
 
-# chunk 8 and 16: one 16-row query tile (four key slices per warp group);
-# 24: two tiles; 40: three (one warp idle); 64: four, the longest chunk.
+# chunk 1, 8 and 16: one 16-row query tile (four key slices per warp
+# group); 24: two tiles; 40: three (one warp idle); 64: four, the longest.
 @pytest.mark.parametrize("dm,C,D", [(256, 8, 7), (512, 16, 14), (256, 24, 7), (256, 40, 5),
-                                    (256, 64, 3)])
+                                    (256, 64, 3), (256, 1, 2)])
 def test_flow_train_step_vs_oracle(dm, C, D):
     s = FlowSetup(dm=dm, F=dm, C=C, D=D)
     plan = s.plan()

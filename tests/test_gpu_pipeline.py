@@ -234,11 +234,16 @@ def test_heads_stage_on_synthetic_features(name):
             assert e < 1e-4, (t, k, e)
 
 
-def test_query_heads_stage_on_synthetic_hidden_rows():
+@pytest.mark.parametrize("nq,dq", [(32, 256), (8, 512)])
+def test_query_heads_stage_on_synthetic_hidden_rows(nq, dq):
     """The cross-attention query head alone (2B-class head shapes: 32 queries
-    x 256, d = 2048, widths 350 / 700 / 1600) on seeded random hidden rows,
+    x 256, and 8 queries x 512 for the wide-query path with two value-column
+    passes; d = 2048, widths 350 / 700 / 1600) on seeded random hidden rows,
     for three tenants of the MQA workload, against the oracle."""
+    import dataclasses
     w = synth.make_workload("mqa2b").subset([0, 1, 2])
+    w = dataclasses.replace(w, tenants=[dataclasses.replace(tn, n_queries=nq, q_dim=dq)
+                                        for tn in w.tenants])
     hw = synth.make_head_weights(w)
     inp = synth.make_inputs(w)
     plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), len(w.tenants), 1 << 30, 1 << 30)
