@@ -48,7 +48,10 @@ size_t jnx_op_gemm_workspace_bytes(int32_t max_pos, int32_t head_dim);
  * ldo >= the output width (N, or N / 2 for JNX_EPI_GLU), 16-byte aligned
  * rows and base, else JNX_ERR_INVALID_ARG.
  * pos/max_pos/rope_cols/head_dim/rope_theta are read for JNX_EPI_ROPE only
- * (workspace then holds the status word and the RoPE table); act
+ * (workspace then holds the status word and the RoPE table; rope_cols a
+ * multiple of head_dim within [0, N]; a position outside [0, max_pos) leaves
+ * its row unrotated and records JNX_ERR_DEVICE_BOUNDS in the status word,
+ * read by jnx_check_status(workspace)); act
  * (JNX_GLU_*) for JNX_EPI_GLU only.  workspace may be NULL otherwise. */
 jnx_status jnx_op_gemm(const uint16_t* A, const uint16_t* W, int32_t M, int32_t N, int32_t K,
                        int32_t epilogue, void* out, int32_t ldo, const int32_t* pos,
@@ -137,7 +140,13 @@ jnx_status jnx_op_gemm_glu_backward(const uint16_t* A, const uint16_t* W, int32_
  * table live in a fixed file-scope device array inside the library (every
  * GPU that loads the library holds it until exit; nothing is allocated).
  * Limits: max_pos * head_dim / 2 <= JNX_NOALLOC_MAX_ROPE_ENTRIES, otherwise
- * JNX_ERR_UNSUPPORTED before any launch; positions must be < max_pos.
+ * JNX_ERR_UNSUPPORTED before any launch.  Host-detected errors (null
+ * pointers, head_dim not 64/128/256, rope_cols not a multiple of head_dim
+ * within [0, N], ldo < N, out or its rows not 16-byte aligned) return
+ * JNX_ERR_INVALID_ARG before any launch with nothing written.  A position
+ * outside [0, max_pos) is a device-detected error: its row is written
+ * unrotated and JNX_ERR_DEVICE_BOUNDS is recorded in the array's status
+ * word (read it with jnx_op_gemm_rope_noalloc_status).
  * The first call on a device looks up the array's address (make it before
  * any stream capture).  All calls on a device share the array: each clears
  * the status word and rewrites the table it reads, and calls that overlap on
@@ -147,6 +156,13 @@ jnx_status jnx_op_gemm_rope_noalloc(const uint16_t* A, const uint16_t* W, int32_
                                     int32_t K, uint16_t* out, int32_t ldo, const int32_t* pos,
                                     int32_t max_pos, int32_t rope_cols, int32_t head_dim,
                                     float rope_theta, void* stream);
+
+/* Reads and clears the status word of jnx_op_gemm_rope_noalloc's fixed
+ * array on the current device, after the work queued on `stream` (it
+ * synchronises the stream; allocates nothing).  Returns JNX_OK, or the
+ * first error a kernel recorded since the last read or call (a call clears
+ * it on entry): JNX_ERR_DEVICE_BOUNDS, JNX_ERR_TIMEOUT. */
+jnx_status jnx_op_gemm_rope_noalloc_status(void* stream);
 
 #ifdef __cplusplus
 }

@@ -16,7 +16,7 @@ Passages followed:
   over the fixed base VLM; §2 places LoRA adapters over one shared base
   among the prior systems.  The adapter's form is reading R5 of ``model``.
 
-Readings where the paper is silent (each is listed in the design doc):
+Readings where the paper is silent (each a choice, not a statement of the paper):
 
   L1  the backbone stays frozen: its projections, norms and the text
       embedding table get no gradient; the trainable backbone-side

@@ -14,7 +14,7 @@ Passages followed:
   the tenant-private module, the VLM the resident base; even a large DiT
   action head costs less than the base VLM's forward.
 
-The paper prints no equation of the expert.  Readings (listed in the design doc):
+The paper prints no equation of the expert.  Readings (each a choice, not a statement of the paper):
 
   F1  rectified-flow training: with the tenant's target chunk a [C, D],
       noise eps [C, D] and time tau in [0, 1] per sample (drawn by the

@@ -13,7 +13,7 @@ Paper passages followed:
 * §4.2, "Server Backend" (its Training Queue paragraph): training activates
   the action module and optimizer state of the job's tenant.
 
-Readings where the paper is silent (each is a choice, listed in the design doc):
+Readings where the paper is silent (each is a choice, not a statement of the paper):
 
 * the optimizer is AdamW (Adam moments with bias correction; weight decay
   decoupled from the gradient and applied to the parameter before the step);

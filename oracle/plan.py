@@ -14,7 +14,7 @@ Paper passages followed:
   samples of different tenants are concatenated; features are afterwards
   partitioned to each tenant's action module.
 
-Readings where the paper is silent (each is a choice, listed in the design doc):
+Readings where the paper is silent (each is a choice, not a statement of the paper):
 
 * compatibility = equality of the prefix signature (backbone id, width,
   vision tokens per image, embedding dtype, vocabulary id, RoPE id);

@@ -14,7 +14,7 @@ Paper passages followed:
   batching timeout and maximum batch size allow; compatibility is a property
   of the shared frozen-prefix interface, not of the tenant.
 
-Readings where the paper is silent (each is a choice, listed in the design doc):
+Readings where the paper is silent (each is a choice, not a statement of the paper):
 
 * the waiting time is that of the oldest queued request (now - arrival[0]);
 * batch size counts samples, and B is also the batch's sample limit; a

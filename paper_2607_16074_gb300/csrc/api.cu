@@ -958,6 +958,10 @@ extern "C" jnx_status jnx_op_gemm(const uint16_t* A, const uint16_t* W, int32_t 
         if (!pos || !workspace || (head_dim != 64 && head_dim != 128 && head_dim != 256) ||
             max_pos <= 0)
             return fail(JNX_ERR_INVALID_ARG, "gemm rope: need pos, workspace, head_dim");
+        if (rope_cols < 0 || rope_cols > N || rope_cols % head_dim)
+            return fail(JNX_ERR_INVALID_ARG,
+                        "gemm rope: rope_cols %d must be a multiple of head_dim %d within N %d",
+                        rope_cols, head_dim, N);
         if (ws_bytes < jnx_op_gemm_workspace_bytes(max_pos, head_dim))
             return fail(JNX_ERR_WORKSPACE, "gemm rope: workspace too small");
         float2* tab = reinterpret_cast<float2*>(static_cast<uint8_t*>(workspace) + kStatusBytes);

@@ -449,7 +449,13 @@ __global__ void __launch_bounds__(192, 1)
                 const float sc = is_v ? 1.f : scale;
                 const uint32_t ta = tacc + acc * HD;
                 if (!is_v) {
-                    const int pr = rv ? pos[grow] : 0;
+                    // a position outside the (cos, sin) table is reported
+                    // and read as position 0 (no rotation)
+                    int pr = rv ? pos[grow] : 0;
+                    if (pr < 0 || pr >= rope_ld) {
+                        if (rv) report(status, JNX_ERR_DEVICE_BOUNDS);
+                        pr = 0;
+                    }
 #pragma unroll 1
                     for (int c = 0; c < HD / 64; ++c) {
                         float2 cs[32];

@@ -502,14 +502,19 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
     } else if constexpr (EPI == EPI_ROPE) {
         const int hc = p.hd / 64;  // 32-column chunks in half a head
         const int half = p.hd / 2;
-        const int pos = valid ? p.pos[my_row] : 0;
+        // a position outside the (cos, sin) table is reported and its row
+        // is left unrotated (the table load is skipped)
+        int pos = valid ? p.pos[my_row] : 0;
+        const bool pos_ok = pos >= 0 && pos < p.rope_ld;
+        if (valid && !pos_ok) report(p.status, JNX_ERR_DEVICE_BOUNDS);
+        if (!pos_ok) pos = 0;
         const float rs = row_norm_scale(p, my_row, valid);
 #pragma unroll 1
         for (int c = 0; c < 8; ++c) {
             const int hchunk = c % (2 * hc);
             if (hchunk >= hc) continue;  // handled with its lower partner
             const int col = n0 + c * 32;
-            const bool rot = valid && col < p.rope_cols;
+            const bool rot = valid && pos_ok && col < p.rope_cols;
             // (cos, sin) of this row's position for the chunk's 32
             // frequencies, loaded before the TMEM read so their latency
             // overlaps it; the table is frequency-major, so the warp's rows

@@ -20,6 +20,10 @@
 //   - Every call on a device shares the one array.  Each call clears the
 //     status word and rewrites the table rows it reads; calls that overlap
 //     on the GPU (different streams, no ordering between them) race on it.
+//   - A kernel-detected error (a position outside [0, max_pos): that row is
+//     left unrotated; a wait that ran out of time) is recorded in the
+//     array's status word; jnx_op_gemm_rope_noalloc_status reads and clears
+//     it.
 //   - Nothing here calls cudaMalloc, cudaFree or any allocating routine.
 #include <mutex>
 
@@ -81,6 +85,14 @@ extern "C" jnx_status jnx_op_gemm_rope_noalloc(const uint16_t* A, const uint16_t
                          "gemm_rope_noalloc: max_pos %d x head_dim/2 %d exceeds the fixed scratch "
                          "of %zu table entries",
                          max_pos, head_dim / 2, kTableEntries);
+    if (rope_cols < 0 || rope_cols > N || rope_cols % head_dim)
+        return jnx::fail(JNX_ERR_INVALID_ARG,
+                         "gemm_rope_noalloc: rope_cols %d must be a multiple of head_dim %d "
+                         "within N %d", rope_cols, head_dim, N);
+    // the epilogue writes 16-byte vectors of whole rows
+    if (ldo < N || ((size_t)ldo * 2) % 16 || reinterpret_cast<uintptr_t>(out) % 16)
+        return jnx::fail(JNX_ERR_INVALID_ARG,
+                         "gemm_rope_noalloc: out needs 16-byte aligned rows of >= %d", N);
     jnx_status st = jnx::gemm_check(M, N, K);
     if (st) return st;
     uint8_t* scratch = nullptr;
@@ -105,4 +117,22 @@ extern "C" jnx_status jnx_op_gemm_rope_noalloc(const uint16_t* A, const uint16_t
     p.hd = head_dim;
     p.status = reinterpret_cast<int*>(scratch);
     return jnx::gemm_launch(A, K, W, K, p, s);
+}
+
+extern "C" jnx_status jnx_op_gemm_rope_noalloc_status(void* stream) {
+    jnx::clear_error();
+    uint8_t* scratch = nullptr;
+    jnx_status st = scratch_on_current_device(&scratch);
+    if (st) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int v = 0;
+    // a copy into this pageable host int and a clear of the word: nothing
+    // is allocated
+    if (cudaMemcpyAsync(&v, scratch, sizeof v, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaMemsetAsync(scratch, 0, sizeof v, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return jnx::fail(JNX_ERR_CUDA, "gemm_rope_noalloc_status: %s",
+                         cudaGetErrorString(cudaGetLastError()));
+    if (v != 0) return jnx::fail(v, "a kernel reported status %d", v);
+    return JNX_OK;
 }

@@ -173,7 +173,8 @@ EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_group_attn_it
            "jnx_heads_backward", "jnx_check_status", "jnx_pack_gate_up", "jnx_op_pack",
            "jnx_op_rmsnorm", "jnx_op_gemm_workspace_bytes", "jnx_op_gemm", "jnx_op_attention",
            "jnx_op_final_pool", "jnx_trace_enable", "jnx_trace_disable", "jnx_trace_count",
-           "jnx_trace_read", "jnx_op_gemm_rope_noalloc", "jnx_sched_poll",
+           "jnx_trace_read", "jnx_op_gemm_rope_noalloc", "jnx_op_gemm_rope_noalloc_status",
+           "jnx_sched_poll",
            "jnx_heads_backward_accumulate", "jnx_heads_adamw", "jnx_backbone_saved_bytes",
            "jnx_backbone_forward_train", "jnx_heads_backward_input", "jnx_transpose",
            "jnx_backbone_backward_workspace_bytes", "jnx_backbone_backward_lora",
@@ -257,6 +258,7 @@ def lib() -> C.CDLL:
         "jnx_trace_read": (i32, [vp, vp, vp, i32, P32]),
         "jnx_op_gemm_rope_noalloc": (i32, [vp, vp, i32, i32, i32, vp, i32, vp, i32, i32, i32, f32,
                                            vp]),
+        "jnx_op_gemm_rope_noalloc_status": (i32, [vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
