@@ -164,6 +164,26 @@ jnx_status jnx_op_gemm_rope_noalloc(const uint16_t* A, const uint16_t* W, int32_
  * it on entry): JNX_ERR_DEVICE_BOUNDS, JNX_ERR_TIMEOUT. */
 jnx_status jnx_op_gemm_rope_noalloc_status(void* stream);
 
+/* Diagnostics: two device routines of the hot path run on their own, so
+ * tests can pin them.  Neither is part of the grouped path.
+ *
+ * y[i] = 2^x[i] by the polynomial exponential that the varlen attention's
+ * softmax evaluates for one key pair in four (range reduction j = rint(x),
+ * f = x - j, 2^f by the degree-3 minimax polynomial on [-0.5, 0.5], x
+ * clamped at -126).  x, y: n device floats.  It stands for the softmax
+ * probabilities 2^(s - m) of §5.2's shared backbone attention. */
+jnx_status jnx_diag_ex2_poly(const float* x, float* y, int32_t n, void* stream);
+
+/* One thread waits, through the library's bounded mbarrier wait, on a
+ * barrier that completes (arrive != 0) or that nothing ever arrives on
+ * (arrive == 0), giving up after limit_cycles SM clocks (0 < limit <= 2^31,
+ * else JNX_ERR_INVALID_ARG before the launch).  A wait that gave up writes
+ * JNX_ERR_TIMEOUT to *status (a device int) and the kernel returns; every
+ * spin in the library's kernels behaves this way.  The paper has no
+ * counterpart (failure detection of the kernels themselves). */
+jnx_status jnx_diag_bounded_wait(int64_t limit_cycles, int32_t arrive, int32_t* status,
+                                 void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 OBJ = os.path.join(ROOT, "_build", "obj")
 LIB = os.path.join(HERE, "libjnx.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["plan.cpp", "api.cu", "gemm.cu", "attn.cu", "norm.cu", "heads.cu", "trace.cu", "noalloc.cu", "lora.cu", "optim.cu", "bwd.cu", "attn_bwd.cu", "train.cu", "flow.cu"]
+SOURCES = ["plan.cpp", "api.cu", "gemm.cu", "attn.cu", "norm.cu", "heads.cu", "trace.cu", "noalloc.cu", "lora.cu", "optim.cu", "bwd.cu", "attn_bwd.cu", "train.cu", "flow.cu", "diag.cu"]
 
 
 def _nvcc() -> str:

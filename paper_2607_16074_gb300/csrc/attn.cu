@@ -147,31 +147,7 @@ struct AttnWsCfg {
 // Softmax of one 128 x BN score tile for this thread's row: row max (pass
 // 1), then probabilities packed as bf16 pairs (pass 2).  FULL: every key of
 // the tile lies inside the sample (no mask).
-// 2^x for a pair of arguments on the FMA pipe instead of the MUFU pipe
-// (range reduction plus a polynomial, as in common libm exp2 designs):
-// j = rint(x) by adding 1.5 * 2^23, f = x - j in [-0.5, 0.5], 2^f by a
-// degree-3 polynomial fitted for minimum maximum relative error on that
-// interval (below 8e-5, under the 2^-9 rounding that P gets in bf16), and
-// j added into the exponent field.  x is clamped at -126 so the exponent
-// cannot wrap; such a p (below 2^-126) is negligible next to the row's
-// largest p (at least 2^-8).
-__device__ __forceinline__ void ex2_poly2(float x0, float x1, float& p0, float& p1) {
-    const uint64_t magic = f2_pack(12582912.f, 12582912.f);
-    const uint64_t nmagic = f2_pack(-12582912.f, -12582912.f);
-    const uint64_t x = f2_pack(fmaxf(x0, -126.f), fmaxf(x1, -126.f));
-    const uint64_t t = f2_add(x, magic);                            // j in the low mantissa bits
-    const uint64_t f = f2_fma(f2_add(t, nmagic), f2_pack(-1.f, -1.f), x);  // x - j
-    uint64_t q = f2_pack(0.055174146f, 0.055174146f);
-    q = f2_fma(q, f, f2_pack(0.24261758f, 0.24261758f));
-    q = f2_fma(q, f, f2_pack(0.69326109f, 0.69326109f));
-    q = f2_fma(q, f, f2_pack(0.99992758f, 0.99992758f));
-    float t0, t1, q0, q1;
-    f2_unpack(t, t0, t1);
-    f2_unpack(q, q0, q1);
-    p0 = __uint_as_float(__float_as_uint(q0) + (__float_as_uint(t0) << 23));
-    p1 = __uint_as_float(__float_as_uint(q1) + (__float_as_uint(t1) << 23));
-}
-
+// The exponential of one key pair in four: ex2_poly2 (jnx_dev.cuh).
 template <int BN, bool FULL>
 __device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float scale_log2,
                                                 bool first, float& m, float& alpha, float& rs,

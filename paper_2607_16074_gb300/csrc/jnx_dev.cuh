@@ -59,6 +59,38 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
     return d;
 }
 
+// 2^x for a pair of arguments on the FMA pipe instead of the MUFU pipe
+// (range reduction plus a polynomial, as in common libm exp2 designs):
+// j = rint(x) by adding 1.5 * 2^23, f = x - j in [-0.5, 0.5], 2^f by the
+// degree-3 polynomial of minimum maximum relative error on that interval
+// (Remez exchange, tests/fit_ex2_poly.py: 7.48e-5, under the 2^-9 rounding
+// that an attention probability gets in bf16), and j added into the
+// exponent field.  x is clamped at -126 so the exponent cannot wrap.  For
+// x in [-126, -125) a result below 2^-126 lands in the subnormal encoding
+// and keeps only an absolute accuracy of 2^-125; such a p is negligible
+// next to a softmax row's largest p (at least 2^-8).
+constexpr float kEx2C0 = 0.999928074f;
+constexpr float kEx2C1 = 0.693260985f;
+constexpr float kEx2C2 = 0.242611122f;
+constexpr float kEx2C3 = 0.0551716691f;
+
+__device__ __forceinline__ void ex2_poly2(float x0, float x1, float& p0, float& p1) {
+    const uint64_t magic = f2_pack(12582912.f, 12582912.f);
+    const uint64_t nmagic = f2_pack(-12582912.f, -12582912.f);
+    const uint64_t x = f2_pack(fmaxf(x0, -126.f), fmaxf(x1, -126.f));
+    const uint64_t t = f2_add(x, magic);                            // j in the low mantissa bits
+    const uint64_t f = f2_fma(f2_add(t, nmagic), f2_pack(-1.f, -1.f), x);  // x - j
+    uint64_t q = f2_pack(kEx2C3, kEx2C3);
+    q = f2_fma(q, f, f2_pack(kEx2C2, kEx2C2));
+    q = f2_fma(q, f, f2_pack(kEx2C1, kEx2C1));
+    q = f2_fma(q, f, f2_pack(kEx2C0, kEx2C0));
+    float t0, t1, q0, q1;
+    f2_unpack(t, t0, t1);
+    f2_unpack(q, q0, q1);
+    p0 = __uint_as_float(__float_as_uint(q0) + (__float_as_uint(t0) << 23));
+    p1 = __uint_as_float(__float_as_uint(q1) + (__float_as_uint(t1) << 23));
+}
+
 // Record the first device-side error in the status word (never traps).
 __device__ __forceinline__ void report(int* status, int code) {
     if (status) atomicCAS(status, 0, code);

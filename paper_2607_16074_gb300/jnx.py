@@ -174,7 +174,7 @@ EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_group_attn_it
            "jnx_op_rmsnorm", "jnx_op_gemm_workspace_bytes", "jnx_op_gemm", "jnx_op_attention",
            "jnx_op_final_pool", "jnx_trace_enable", "jnx_trace_disable", "jnx_trace_count",
            "jnx_trace_read", "jnx_op_gemm_rope_noalloc", "jnx_op_gemm_rope_noalloc_status",
-           "jnx_sched_poll",
+           "jnx_sched_poll", "jnx_diag_ex2_poly", "jnx_diag_bounded_wait",
            "jnx_heads_backward_accumulate", "jnx_heads_adamw", "jnx_backbone_saved_bytes",
            "jnx_backbone_forward_train", "jnx_heads_backward_input", "jnx_transpose",
            "jnx_backbone_backward_workspace_bytes", "jnx_backbone_backward_lora",
@@ -259,6 +259,8 @@ def lib() -> C.CDLL:
         "jnx_op_gemm_rope_noalloc": (i32, [vp, vp, i32, i32, i32, vp, i32, vp, i32, i32, i32, f32,
                                            vp]),
         "jnx_op_gemm_rope_noalloc_status": (i32, [vp]),
+        "jnx_diag_ex2_poly": (i32, [vp, vp, i32, vp]),
+        "jnx_diag_bounded_wait": (i32, [C.c_int64, i32, vp, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)

@@ -11,7 +11,7 @@ from oracle import flow as Fl
 from paper_2607_16074_gb300 import jnx as J
 from paper_2607_16074_gb300 import runtime as R
 from tests.gpu_helpers import f64
-from tests.helpers import oracle_requests
+from tests.helpers import BF16_TOL, oracle_requests, rel_err
 
 pytestmark = pytest.mark.gpu
 
@@ -23,9 +23,23 @@ def built():
     J.lib()
 
 
-def _rel_l2(got, ref):
-    got, ref = np.asarray(got, np.float64), np.asarray(ref, np.float64)
-    return float(np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-300))
+# Velocities, losses and Euler samples are held to the stated 2e-2
+# (measured on GB300 at most 0.017, 2.4e-3 and 4.3e-3).  The parameter
+# gradients are sums over the action rows of products of bf16-rounded
+# factors, and their max|err|/rms is ill-conditioned: perturbing the fp64
+# oracle's own parameters and context rows by relative noise of 2^-9 (2^-8)
+# moves its gradients by up to 0.094 (0.177) of rms.  Measured on GB300,
+# worst over every tenant and parameter: 0.054 - 0.156 (the training-step
+# cases), 0.174 (the flow bench's launch configuration); the bound is 1.5x
+# the worst (relative L2 of the same gradients: 1.2e-3 - 6.2e-3).
+FLOW_GRAD_TOL = 0.26
+
+
+def _err(what, got, ref, tol, worst):
+    e = rel_err(got, ref)
+    print(f"{what}: max|err|/rms {e:.4e}")
+    worst[0] = max(worst[0], e)
+    assert e < tol, (what, e, tol)
 
 
 class FlowSetup:
@@ -89,6 +103,7 @@ def _inputs(plan, C, D, seed=4):
 def _check(s, plan, hidden, inp, vel, loss, tol, only=None):
     H = f64(hidden)
     cu, seg = plan.cu_seqlens, plan.seg_offsets
+    worst = [0.0]
     for gi, t in enumerate(plan.slot_tenant.tolist()):
         if only is not None and t not in only:
             continue
@@ -99,23 +114,22 @@ def _check(s, plan, hidden, inp, vel, loss, tol, only=None):
         taus = f64(inp["tau"][seg[gi]:seg[gi + 1]])
         p = s.oracle_params(t)
         ref_loss, V, G = Fl.tenant_step(p, s.nh, ctx, acts, noise, taus)
-        e = _rel_l2(f64(vel[seg[gi]:seg[gi + 1]]), V)
-        assert e < tol, ("velocity", t, e)
-        assert abs(float(loss[t]) - ref_loss) <= tol * ref_loss, ("loss", t)
+        _err(f"tenant {t} velocity", f64(vel[seg[gi]:seg[gi + 1]]), V, BF16_TOL, [0.0])
+        e = abs(float(loss[t]) - ref_loss) / ref_loss
+        print(f"tenant {t} loss: relative {e:.4e}")
+        assert e <= BF16_TOL, ("loss", t, e)
         for k in J.FLOW_PARAMS:
-            ref = G[k]
-            got = f64(s.heads.grads[k][t])
-            assert _rel_l2(got, ref) < tol, ("grad", t, k, _rel_l2(got, ref))
+            _err(f"tenant {t} grad {k}", f64(s.heads.grads[k][t]), G[k], tol, worst)
         for b, GB in enumerate(G["blocks"]):
             dg = s.heads.block_grads[b]
             pairs = [("w_qkv", GB["wqkv"]), ("w_kvc", GB["wkvc"]), ("w_o", GB["wo"]),
                      ("w_d", GB["wd"])]
             for name, ref in pairs:
-                e = _rel_l2(f64(dg[name][t]), ref)
-                assert e < tol, ("grad", t, b, name, e)
+                _err(f"tenant {t} block {b} grad {name}", f64(dg[name][t]), ref, tol, worst)
             gg, gu = s.unpack_gu(f64(dg["w_gu"][t]))
-            assert _rel_l2(gg, GB["wg"]) < tol, ("grad", t, b, "wg", _rel_l2(gg, GB["wg"]))
-            assert _rel_l2(gu, GB["wu"]) < tol, ("grad", t, b, "wu", _rel_l2(gu, GB["wu"]))
+            _err(f"tenant {t} block {b} grad wg", gg, GB["wg"], tol, worst)
+            _err(f"tenant {t} block {b} grad wu", gu, GB["wu"], tol, worst)
+    print(f"largest max|err|/rms {worst[0]:.4e} (bound {tol})")
 
 
 # chunk 1, 8 and 16: one 16-row query tile (four key slices per warp
@@ -131,9 +145,8 @@ def test_flow_train_step_vs_oracle(dm, C, D):
     g, vel, loss, ws = s.run(plan, hidden, inp)
     # bf16 operands of every projection and of the attention inputs, fp32
     # residual stream and attention, two blocks: a few 2^-9 roundings per
-    # block.  Measured relative L2 errors 1.2e-3 - 6.0e-3 over every
-    # parameter, tenant and both sizes; a wrong term or index is off by O(1).
-    _check(s, plan, hidden, inp, vel, loss, 3e-2)
+    # block; a wrong term or index is off by O(1)
+    _check(s, plan, hidden, inp, vel, loss, FLOW_GRAD_TOL)
 
 
 def test_flow_bench_size_sampled_tenant_vs_oracle():
@@ -154,7 +167,7 @@ def test_flow_bench_size_sampled_tenant_vs_oracle():
     g, vel, loss, ws = s.run(plan, hidden, inp)
     assert torch.isfinite(vel).all() and torch.isfinite(loss[:8]).all()
     t = int(np.random.default_rng(5).integers(8))
-    _check(s, plan, hidden, inp, vel, loss, 3e-2, only={t})
+    _check(s, plan, hidden, inp, vel, loss, FLOW_GRAD_TOL, only={t})
 
 
 def test_flow_sampling_vs_oracle():
@@ -174,8 +187,9 @@ def test_flow_sampling_vs_oracle():
         p = s.oracle_params(t)
         for i in range(seg[gi], seg[gi + 1]):
             ref = Fl.sample(p, s.nh, H[cu[i]:cu[i + 1]], f64(noise[i]), 4)
-            e = _rel_l2(f64(out[i]), ref)
-            assert e < 3e-2, (t, i, e)
+            e = rel_err(f64(out[i]), ref)
+            print(f"tenant {t} sample {i} Euler sample: max|err|/rms {e:.4e}")
+            assert e < BF16_TOL, (t, i, e)
 
 
 def test_flow_grouped_equals_isolated_and_other_slots_untouched():

@@ -14,8 +14,9 @@ from oracle import backward as B
 from oracle import model as M
 from paper_2607_16074_gb300 import jnx as J
 from paper_2607_16074_gb300 import runtime as R
+from tests import bf16_emulation as E
 from tests.gpu_helpers import f64, randn_bf16, stream
-from tests.helpers import deep_tol, oracle_requests, rel_err, rel_err_bf16_out
+from tests.helpers import BF16_TOL, check_bf16_out, oracle_requests, rel_err
 
 pytestmark = pytest.mark.gpu
 
@@ -27,9 +28,15 @@ def built():
     J.lib()
 
 
-def _rel_l2(got, ref):
-    got, ref = np.asarray(got, np.float64), np.asarray(ref, np.float64)
-    return float(np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-300))
+# max|err|/rms(ref) bounds of every adapter and feature gradient of the
+# whole training step against the oracle, by block depth.  These gradients
+# sum outer products over a sample's rows through several bf16 roundings
+# (operands of every product, P and dS), and their max|err|/rms is far more
+# sensitive than their relative L2: measured on GB300, worst over every
+# tenant, layer and adapter tensor, 0.035 at one block (d 2048, MQA hd 256)
+# and 0.083 / 0.139 at two (SwiGLU / GeGLU, d 256); the bounds are 1.5x
+# those (relative L2 of the same gradients: 3e-3 - 1.1e-2).
+LORA_GRAD_TOL = {1: 0.053, 2: 0.21}
 
 
 # ---------------------------------------------------------------------------
@@ -86,8 +93,8 @@ def test_glu_backward_gemms_vs_oracle(act):
     gcol = (f // 128) * 256 + f % 128   # F column f: gate slot, its up slot 128 later
     saved = f64(gu)
     # fp32 products of bf16 operands, stored in bf16
-    assert rel_err_bf16_out(saved[:, gcol], u * da) < 1e-3
-    assert rel_err_bf16_out(saved[:, gcol + 128], a) < 1e-3
+    check_bf16_out(saved[:, gcol], u * da, 1e-3, f"glu save u act' {act}")
+    check_bf16_out(saved[:, gcol + 128], a, 1e-3, f"glu save act {act}")
     A = randn_bf16((M_, K), 5)
     W = randn_bf16((F, K), 6, std=0.05)
     J.check(J.lib().jnx_op_gemm_glu_backward(A.data_ptr(), W.data_ptr(), M_, F, K, gu.data_ptr(),
@@ -96,8 +103,8 @@ def test_glu_backward_gemms_vs_oracle(act):
     dm = f64(A) @ f64(W).T
     got = f64(gu)
     # against the multipliers as stored (the bf16 they were rounded to)
-    assert rel_err_bf16_out(got[:, gcol], dm * saved[:, gcol]) < 1e-3
-    assert rel_err_bf16_out(got[:, gcol + 128], dm * saved[:, gcol + 128]) < 1e-3
+    check_bf16_out(got[:, gcol], dm * saved[:, gcol], 1e-3, f"glu backward dg {act}")
+    check_bf16_out(got[:, gcol + 128], dm * saved[:, gcol + 128], 1e-3, f"glu backward du {act}")
 
 
 def _attn_case(lengths, H, Hkv, hd, seed, qk_std=1.0):
@@ -148,6 +155,7 @@ def test_attention_backward_vs_oracle(H, Hkv, hd):
     Q = f64(qkv)
     got = f64(dqkv)
     ref = np.zeros_like(got)
+    emu = np.zeros_like(got)  # the same with the kernel's bf16 rounding points
     grp = H // Hkv
     for i, L in enumerate(lengths):
         r = slice(cu[i], cu[i + 1])
@@ -164,20 +172,21 @@ def test_attention_backward_vs_oracle(H, Hkv, hd):
         # D = rowsum(dO * O) with the device's bf16 dO and O
         Dref = (do * f64(att)[r].reshape(L, H, hd)).sum(axis=2)
         assert np.max(np.abs(f64(D)[r] - Dref)) <= 1e-4 * max(1.0, np.abs(Dref).max())
-        dq, dk, dv = B.attention_backward(q, k, v, do)
-        ref[r] = np.concatenate([B.rope_backward(dq, np.arange(L), 1e4).reshape(L, -1),
-                                 B.rope_backward(dk, np.arange(L), 1e4).reshape(L, -1),
-                                 dv.reshape(L, -1)], axis=1)
-    # each gradient block's relative L2 error over the batch (a one-token
-    # sample's dq and dk are exactly zero: one key makes dS vanish).  The
-    # result is stored in bf16 (rounding the exact reference alone gives
-    # ~1.7e-3 here) and P and dS are rounded to bf16 before the accumulating
-    # products (the same order again, averaged over the keys): 2^-8 bounds
-    # both with margin, where a wrong term or index is off by O(1).
+        for dst, grads in ((ref, B.attention_backward(q, k, v, do)),
+                           (emu, E.attention_backward(q, k, v, do))):
+            dq, dk, dv = grads
+            dst[r] = np.concatenate([B.rope_backward(dq, np.arange(L), 1e4).reshape(L, -1),
+                                     B.rope_backward(dk, np.arange(L), 1e4).reshape(L, -1),
+                                     dv.reshape(L, -1)], axis=1)
+    # each gradient block over the batch (a one-token sample's dq and dk are
+    # exactly zero: one key makes dS vanish).  The result is stored in bf16
+    # and P and dS are rounded to bf16 before the accumulating products: the
+    # floor is the emulated gradients' distance from the oracle's
+    emu = E.bf16(emu)
     for c0, c1, name in ((0, H * hd, "dq"), (H * hd, (H + Hkv) * hd, "dk"),
                          ((H + Hkv) * hd, ldq, "dv")):
-        e = _rel_l2(got[:, c0:c1], ref[:, c0:c1])
-        assert e < 2.0 ** -8, (name, e)
+        fl = rel_err(emu[:, c0:c1], ref[:, c0:c1])
+        check_bf16_out(got[:, c0:c1], ref[:, c0:c1], BF16_TOL, f"attention backward {name}", fl)
     r0 = slice(cu[0], cu[1])
     scale = float(np.sqrt(np.mean(ref[:, :(H + Hkv) * hd] ** 2)))
     assert np.max(np.abs(got[r0, :(H + Hkv) * hd])) < 1e-3 * scale
@@ -249,15 +258,14 @@ def _small_lora_workload(glu, n_layers=2):
 
 
 def _check_vs_oracle(s, plan, step, ref, tol):
-    """Relative L2 error of every group tenant's feature gradient and of each
-    of its adapter gradients in every layer.  Adapter gradients pass through
-    every block's forward and the backward of the blocks above, each with a
-    few bf16 roundings (operands of every product, P and dS): measured
-    3e-3 - 7e-3 at one block, up to 1.1e-2 at two and 1.5e-2 at four, growing
-    like sqrt(depth); the bound is the forward's 2e-2 per block scaled by
-    sqrt(n_layers) (deep_tol), where a wrong term is off by O(1)."""
+    """max|err|/rms(ref) of every group tenant's feature gradient and of each
+    of its adapter gradients in every layer, printed and held to tol.
+    Adapter gradients pass through every block's forward and the backward of
+    the blocks above, each with several bf16 roundings (operands of every
+    product, P and dS)."""
     cu = plan.cu_seqlens
     seg = plan.seg_offsets
+    worst = 0.0
     for gi, t in enumerate(plan.slot_tenant.tolist()):
         if t not in ref:
             continue
@@ -265,13 +273,17 @@ def _check_vs_oracle(s, plan, step, ref, tol):
         # the feature gradient every row gets from its tenant's head
         dh = np.concatenate(r["d_hidden"])
         rows = np.concatenate([np.arange(cu[i], cu[i + 1]) for i in range(seg[gi], seg[gi + 1])])
-        e = _rel_l2(f64(step.d_hidden[torch.from_numpy(rows).long().cuda()]), dh)
+        e = rel_err(f64(step.d_hidden[torch.from_numpy(rows).long().cuda()]), dh)
+        print(f"tenant {t} d_hidden: max|err|/rms {e:.4e}")
+        worst = max(worst, e)
         assert e < tol, ("d_hidden", t, e)
         for l, gl in enumerate(r["lora"]):
             for name, gref in gl.items():
-                got = f64(s.bb.lora_grads[l][name][t])
-                e = _rel_l2(got, gref)
+                e = rel_err(f64(s.bb.lora_grads[l][name][t]), gref)
+                print(f"tenant {t} layer {l} {name}: max|err|/rms {e:.4e}")
+                worst = max(worst, e)
                 assert e < tol, ("lora", t, l, name, e)
+    print(f"largest max|err|/rms {worst:.4e} (bound {tol})")
 
 
 @pytest.mark.parametrize("glu", [0, 1])
@@ -280,7 +292,7 @@ def test_lora_train_step_small_vs_oracle(glu):
     s = TrainSetup(w, std=0.05)
     plan, step = s.run()
     ref = s.oracle()
-    _check_vs_oracle(s, plan, step, ref, deep_tol(w.backbone.n_layers))
+    _check_vs_oracle(s, plan, step, ref, LORA_GRAD_TOL[w.backbone.n_layers])
 
 
 def test_lora_train_step_mqa_hd256_vs_oracle():
@@ -294,7 +306,7 @@ def test_lora_train_step_mqa_hd256_vs_oracle():
     s = TrainSetup(w.subset(pick), gen_device="cuda")
     plan, step = s.run()
     ref = s.oracle(tenants=pick)
-    _check_vs_oracle(s, plan, step, ref, deep_tol(1))
+    _check_vs_oracle(s, plan, step, ref, LORA_GRAD_TOL[1])
 
 
 def test_lora_grads_grouped_equal_isolated_and_other_slots_untouched():

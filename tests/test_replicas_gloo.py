@@ -74,14 +74,18 @@ def test_reference_arm_prints_the_contract_line():
     import subprocess
     import sys
     r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--steps", "1",
-                        "--warmup", "3"], capture_output=True, text=True, timeout=600,
+                        "--warmup", "1"], capture_output=True, text=True, timeout=600,
                        cwd=os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
     assert r.returncode == 0, r.stderr[-2000:]
     lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
     assert len(lines) == 1
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["metric"] == bench.METRIC
-    assert d["value"] > 0 and d["steps"] == 1 and d["warmup"] == 3
+    assert d["value"] > 0 and d["steps"] == 1 and d["warmup"] == 1
+    # what was timed: one whole tenant through two blocks, scaled to depth
+    tm = d["timed"]
+    assert tm["blocks"] == 2 and tm["scale"] == 16 and tm["tokens"] > 0
+    assert tm["full_depth_ms_per_step"] > d["ms_per_step"]
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"] and cb["value"] == d["value"]
     e = d["e2e"]
