@@ -25,8 +25,9 @@ Rounding points (the switch names):
             projection (K = H hd) before the pre-FFN norm.  Elsewhere the
             operand is bf16(x rsqrt(mean(x^2) + eps) gamma).
   qkv       q and k after RoPE, and v, stored in bf16.
-  p         the attention probabilities as the P V operand, in bf16.  The
-            row sums use the unrounded values.
+  p         the attention probabilities as the P V operand, in bf16,
+            relative to the kernel's lazy running max (attention()); the row
+            sums use the unrounded values.
   attn_out  the attention output, stored in bf16.
   u         the GLU product act(g) * u, stored in bf16.
   lora_t    the adapter down-projection x A^T, stored in bf16.  Its input is
@@ -182,20 +183,45 @@ def _rounder(rounding):
     return lambda name, a: bf16(a) if name in rounding else a
 
 
+KEY_TILE = 64    # keys per tile of the forward attention kernel
+LAZY_LOG2 = 8.0  # its running max is raised only past this growth (log2 units)
+
+
 def attention(q, k, v, rounding: Sequence[str] = ALL) -> np.ndarray:
     """One sample's attention (bidirectional, scale 1/sqrt(hd), K/V head
     h // (H / Hkv)) with the rounding points 'p' and 'attn_out'.
-    q: [L, H, hd], k/v: [L, Hkv, hd] -> [L, H hd]."""
+    q: [L, H, hd], k/v: [L, Hkv, hd] -> [L, H hd].
+
+    P is formed as the kernel forms it, which decides what its bf16 rounding
+    sees: over tiles of KEY_TILE keys, relative to a running max m taken from
+    the first tile and raised (with O and the row sum rescaled) only when a
+    tile's max exceeds it by more than LAZY_LOG2, so P = 2^(s log2(e) - m)
+    can reach 2^8 and the row's largest P is in general not exactly 1; the
+    row sum adds the unrounded values.  Without rounding this is the
+    softmax of the oracle up to reassociation."""
     rd = _rounder(rounding)
     L, H, hd = q.shape
     grp = H // k.shape[1]
+    c = math.log2(math.e) / math.sqrt(hd)
     o = np.empty_like(q)
     for h in range(H):
         g = h // grp
-        s = q[:, h, :] @ k[:, g, :].T / math.sqrt(hd)
-        p = np.exp(s - np.max(s, axis=1, keepdims=True))
-        l = np.sum(p, axis=1, keepdims=True)
-        o[:, h, :] = (rd("p", p) @ v[:, g, :]) / l
+        s = (q[:, h, :] @ k[:, g, :].T) * c
+        m = l = O = None
+        for k0 in range(0, L, KEY_TILE):
+            st = s[:, k0:k0 + KEY_TILE]
+            mx = np.max(st, axis=1)
+            if m is None:
+                m, alpha = mx, np.ones(L)
+                l, O = np.zeros(L), np.zeros((L, hd))
+            else:
+                up = mx > m + LAZY_LOG2
+                alpha = np.where(up, np.exp2(m - mx), 1.0)
+                m = np.where(up, mx, m)
+            p = np.exp2(st - m[:, None])
+            O = O * alpha[:, None] + rd("p", p) @ v[k0:k0 + KEY_TILE, g, :]
+            l = l * alpha + np.sum(p, axis=1)
+        o[:, h, :] = O / l[:, None]
     return rd("attn_out", o.reshape(L, H * hd))
 
 
