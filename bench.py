@@ -50,14 +50,17 @@ def workload_desc(w):
 
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one gate/up
-# GEMM launch from an ncu capture of the full-size benchmark (the summary and
-# command are in profiles/), valid only for the GEMM source it was taken on
-# and the launch shape it was taken at (packed rows, width, FFN width).
+# GEMM launch: captured by ncu on a small launch of the same kernel whose
+# row blocks fill whole tile groups, as the full launch's do (10,240 rows),
+# and scaled by rows to the full launch (the traffic per row is the same:
+# A once, the weight once per tile group, u once; the summary and command
+# are in profiles/).  Valid only for the GEMM source it was taken on and the
+# launch shape it is scaled to (packed rows, width, FFN width).
 RECORDED_TRAFFIC = {
     # workload: (sha256 of csrc/gemm.cu, (rows, d, F), bytes per launch, profile)
-    "llama7b": ("5fd9e53974a1be9a3343dad5356d1f5639f680a646cd8383f40eafb3bdb628eb",
-                (65817, 4096, 11008), 3.07e9 + 1.44e9,
-                "profiles/gemm_gate_up_glu_llama7b_dram.md"),
+    "llama7b": ("8ae0084ca22eba83c00bdc18a9ece2d9956dbc2873b4f8142777cc187087ec5e",
+                (65817, 4096, 11008), (465.714176e6 + 215.440640e6) * 65817 / 10240,
+                "profiles/gemm_gate_up_glu_10240_dram.md (10,240 rows, scaled by rows)"),
 }
 
 
@@ -821,6 +824,76 @@ def run_kernel(args):
         n_el = sum(v.numel() for gr in heads.grads for v in gr.values())
         call = lambda: (heads.adamw_step(grp, lr=1e-4, weight_decay=0.01), 0)[1]
         work, unit = 30.0 * n_el, "GB/s"
+    elif k in ("heads_bwd_adamw", "heads_bwd_then_adamw"):
+        # the 7B-class group's 32 MLP heads: the heads backward with the
+        # AdamW step fused into it, or the backward then the separate step;
+        # both rated on the fused step's algorithmic bytes (weights read for
+        # the input gradient, features, moments and masters read and written,
+        # bf16 parameters written: 26 bytes per parameter element)
+        import synth
+        from paper_2607_16074_gb300 import runtime as R
+        w = synth.make_workload("llama7b")
+        hw = synth.make_head_weights(w, device=dev)
+        heads = R.DeviceHeads(w.tenants, w.backbone.d, hw, device=dev)
+        heads.init_optimizer()
+        plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), len(w.tenants), w.max_samples,
+                                w.max_tokens)
+        grp = R.DeviceGroup(plan, device=dev)
+        pooled = torch.randn(plan.n_samples, w.backbone.d, generator=g, device=dev)
+        tg = synth.make_inputs(w, device=dev)["targets"]
+        ws = torch.zeros(heads.workspace_bytes(grp), dtype=torch.uint8, device=dev)
+        heads.forward(grp, pooled, None, tg, torch.zeros_like(tg),
+                      torch.zeros(len(w.tenants), device=dev), ws)
+        n_el = sum(v.numel() for gr in heads.grads for v in gr.values())
+        hb = head_bytes(w, plan)[1] - 4 * n_el  # the backward's bytes without its stores
+        if k == "heads_bwd_adamw":
+            call = lambda: (heads.backward_adamw(grp, pooled, None, tg, ws, lr=1e-4), 0)[1]
+        else:
+            call = lambda: (heads.backward(grp, pooled, None, tg, ws),
+                            heads.adamw_step(grp, lr=1e-4), 0)[2]
+        work, unit = hb + 26.0 * n_el, "GB/s"
+    elif k == "heads_fwd":
+        # the 7B-class group's 32 MLP heads forward and loss on random pooled
+        # features, rated on its algorithmic bytes (head_bytes)
+        import synth
+        from paper_2607_16074_gb300 import runtime as R
+        w = synth.make_workload("llama7b")
+        hw = synth.make_head_weights(w, device=dev)
+        heads = R.DeviceHeads(w.tenants, w.backbone.d, hw, device=dev)
+        plan = J.jnx_group_plan(w.schemas(), oracle_requests(w), len(w.tenants), w.max_samples,
+                                w.max_tokens)
+        grp = R.DeviceGroup(plan, device=dev)
+        pooled = torch.randn(plan.n_samples, w.backbone.d, generator=g, device=dev)
+        tg = synth.make_inputs(w, device=dev)["targets"]
+        ws = torch.zeros(heads.workspace_bytes(grp), dtype=torch.uint8, device=dev)
+        preds, lossb = torch.zeros_like(tg), torch.zeros(len(w.tenants), device=dev)
+        call = lambda: (heads.forward(grp, pooled, None, tg, preds, lossb, ws), 0)[1]
+        work, unit = head_bytes(w, plan)[0], "GB/s"
+    elif k == "pack":
+        # the packer over whole 7B-class tenants until --tokens rows: bf16
+        # rows read, fp32 rows written (6 bytes per element)
+        import synth
+        from paper_2607_16074_gb300 import runtime as R
+        w = synth.make_workload("llama7b")
+        tok, keep = 0, []
+        for t in range(len(w.tenants)):
+            keep.append(t)
+            tok += sum(smp.length(w.backbone.vision_tokens) for r in w.requests if r.tenant == t
+                       for smp in r.samples)
+            if tok >= M:
+                break
+        ws_ = w.subset(keep)
+        plan = J.jnx_group_plan(ws_.schemas(), oracle_requests(ws_), len(w.tenants), 1 << 30,
+                                1 << 30)
+        grp = R.DeviceGroup(plan, device=dev)
+        inp = synth.make_inputs(w, device=dev)
+        tab = rnd(w.backbone.vocab, d)
+        x = torch.empty(plan.n_tokens, d, dtype=torch.float32, device=dev)
+        call = lambda: L.jnx_op_pack(grp.ref, inp["vision"].data_ptr(), inp["vision"].shape[0],
+                                     inp["text_ids"].data_ptr(), inp["text_ids"].shape[0],
+                                     tab.data_ptr(), w.backbone.vocab, d, x.data_ptr(), None,
+                                     s.cuda_stream)
+        work, unit = plan.n_tokens * d * 6.0, "GB/s"
     elif k == "rmsnorm":
         x = torch.randn(M, d, generator=g, device=dev)
         gam = rnd(d)
@@ -1101,7 +1174,8 @@ def main():
     ap.add_argument("--reference-layers", type=int, default=2)
     ap.add_argument("--kernel", default=None,
                     help="time one kernel alone (gemm_gu, gemm_qkv, gemm_o, gemm_down, "
-                         "attention, attention_mqa, rmsnorm, heads_adamw) on 7B-class shapes "
+                         "attention, attention_mqa, rmsnorm, heads_adamw, heads_bwd_adamw, "
+                         "heads_bwd_then_adamw, pack, heads_fwd) on 7B-class shapes "
                          "with --tokens rows")
     ap.add_argument("--tokens", type=int, default=8192)
     ap.add_argument("--subset", type=int, default=0,

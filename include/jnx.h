@@ -395,6 +395,30 @@ jnx_status jnx_heads_adamw(const jnx_head* heads, const jnx_head_grads* grads,
                            jnx_head_opt* opt, int32_t n_tenants, const jnx_group* g,
                            const jnx_adamw* hp, void* stream);
 
+/* The heads backward with each group tenant's AdamW step fused into it
+ * (App. A "Actor Consumption and Version Consistency": a microbatch steps
+ * only its own tenant's optimizer and policy version; nothing is shared or
+ * averaged across tenants).  The result equals jnx_heads_backward (or, with
+ * accumulate != 0, jnx_heads_backward_accumulate) followed by
+ * jnx_heads_adamw, but no gradient is stored: each gradient element goes
+ * straight into its parameter's update, which saves writing and re-reading
+ * the fp32 gradients.  accumulate != 0 adds grads[tenant] (the earlier
+ * microbatches' sum, read, not written) to this backward's gradient before
+ * the step; accumulate == 0 never touches grads (may be NULL).  d_hidden
+ * (optional, [n_tokens, d] fp32, as jnx_heads_backward_input) receives the
+ * gradient at the final normed rows, formed from the parameters before
+ * their update.  Every parameter is read before it is updated.  On success
+ * opt[tenant].step and .version are incremented for the group's tenants.
+ * Errors as jnx_heads_backward and jnx_heads_adamw (null or misaligned
+ * optimizer state: JNX_ERR_INVALID_ARG before any launch).  A capturing
+ * stream is accepted (nothing is uploaded from host memory). */
+jnx_status jnx_heads_backward_adamw(const jnx_head* heads, int32_t n_tenants,
+                                    const jnx_group* g, const float* pooled,
+                                    const uint16_t* hidden, const float* targets,
+                                    const jnx_head_grads* grads, int32_t accumulate,
+                                    jnx_head_opt* opt, const jnx_adamw* hp, float* d_hidden,
+                                    void* workspace, size_t ws_bytes, void* stream);
+
 /* ------------------------------------------------------------------------
  * Trainable per-tenant adapters: the LoRA backward through the frozen backbone
  *

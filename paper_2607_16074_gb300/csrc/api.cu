@@ -1,6 +1,7 @@
 // C-ABI entry points: the shared backbone forward, the tenant heads, status
 // and helpers, plus the stage-level entry points of jnx_ops.h.
 #include <algorithm>
+#include <cmath>
 #include <vector>
 
 #include "../../include/jnx_ops.h"
@@ -856,6 +857,108 @@ extern "C" jnx_status jnx_heads_backward_input(const jnx_head* heads, int32_t n_
                                    ws_bytes, stream, false);
     if (st || g->n_slots == 0) return st;
     return heads_feature_grad(heads, g, d_hidden, workspace, static_cast<cudaStream_t>(stream));
+}
+
+// The heads backward with every group tenant's AdamW step fused into it
+// (App. A "Actor Consumption and Version Consistency": the step of one
+// tenant's own optimizer, nothing shared or averaged across tenants).
+extern "C" jnx_status jnx_heads_backward_adamw(const jnx_head* heads, int32_t n_tenants,
+                                               const jnx_group* g, const float* pooled,
+                                               const uint16_t* hidden, const float* targets,
+                                               const jnx_head_grads* grads, int32_t accumulate,
+                                               jnx_head_opt* opt, const jnx_adamw* hp,
+                                               float* d_hidden, void* workspace, size_t ws_bytes,
+                                               void* stream) {
+    clear_error();
+    (void)targets;  // the loss gradient dy was kept by the forward
+    if (!opt || !hp) return fail(JNX_ERR_INVALID_ARG, "heads backward adamw: null argument");
+    if (!(hp->lr >= 0.f) || !(hp->beta1 >= 0.f && hp->beta1 < 1.f) ||
+        !(hp->beta2 >= 0.f && hp->beta2 < 1.f) || !(hp->eps >= 0.f) || !(hp->weight_decay >= 0.f))
+        return fail(JNX_ERR_INVALID_ARG, "heads backward adamw: hyperparameter out of range");
+    if (accumulate && !grads && g && g->n_slots > 0)
+        return fail(JNX_ERR_INVALID_ARG, "heads backward adamw: accumulating needs grads");
+    jnx_status st;
+    if ((st = check_heads(heads, n_tenants, g, accumulate != 0, grads, pooled, hidden))) return st;
+    if (g->n_slots == 0) return JNX_OK;
+    if (!workspace) return fail(JNX_ERR_INVALID_ARG, "heads backward adamw: null workspace");
+    // every group tenant's optimizer state, checked before anything is written
+    auto al = [](const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; };
+    for (int i = 0; i < g->n_slots; ++i) {
+        const int t = g->h_slot_tenant[i];
+        const jnx_head& h = heads[t];
+        const jnx_head_opt& o = opt[t];
+        const bool mlp = h.kind == JNX_HEAD_MLP;
+        const int ks[5] = {mlp ? 0 : 4, mlp ? 1 : 5, mlp ? 2 : 6, mlp ? 3 : 7, mlp ? -1 : 8};
+        for (int k : ks) {
+            if (k < 0) continue;
+            if (!o.master[k] || !o.m[k] || !o.v[k])
+                return fail(JNX_ERR_INVALID_ARG,
+                            "heads backward adamw: tenant %d: null state for tensor %d", t, k);
+        }
+        // the weight tensors' state is updated with 16-byte (W1, W2, Wout)
+        // or 8-byte (Wk, Wv) accesses
+        const int vec[3] = {mlp ? 0 : 7, mlp ? 2 : 5, mlp ? -1 : 6};
+        for (int k : vec) {
+            if (k < 0) continue;
+            const uintptr_t a = (k == 5 || k == 6) ? 8 : 16;
+            if (!al(o.master[k], a) || !al(o.m[k], a) || !al(o.v[k], a))
+                return fail(JNX_ERR_INVALID_ARG,
+                            "heads backward adamw: tenant %d: tensor %d state misaligned", t, k);
+        }
+        if (!mlp && (!al(h.wk, 4) || !al(h.wv, 4)))
+            return fail(JNX_ERR_INVALID_ARG, "heads backward adamw: tenant %d: Wk/Wv misaligned", t);
+    }
+    HeadsWs w = carve_heads(heads, g, workspace);
+    if (ws_bytes < w.bytes)
+        return fail(JNX_ERR_WORKSPACE, "heads: workspace %zu < %zu bytes", ws_bytes, w.bytes);
+    if ((st = heads_set_smem())) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int d = heads[g->h_slot_tenant[0]].d_in;
+    const AdamHp ahp{hp->lr, hp->beta1, hp->beta2, hp->eps, hp->weight_decay};
+    static thread_local HeadTable tab;
+    static thread_local HeadOptTable otab;
+    {
+        TraceScope ts(JNX_K_HEADS_BWD, 0.0, s);
+        for (int g0 = 0; g0 < g->n_slots; g0 += kMaxSlots) {
+            const int n = std::min(kMaxSlots, g->n_slots - g0);
+            HeadBatch b = fill_table(tab, heads, grads, g, g0, n, accumulate != 0);
+            if ((st = heads_backward_front_launch(tab, b, w.sc, d, hidden, g->cu_seqlens,
+                                                  g->sample_slot, s)))
+                return st;
+        }
+    }
+    if (d_hidden && (st = heads_feature_grad(heads, g, d_hidden, workspace, s))) return st;
+    double fl = 0.0;
+    for (int g0 = 0; g0 < g->n_slots; g0 += kMaxSlots) {
+        const int n = std::min(kMaxSlots, g->n_slots - g0);
+        HeadBatch b = fill_table(tab, heads, grads, g, g0, n, accumulate != 0);
+        fl += heads_flops(tab, n, true);
+        otab = HeadOptTable{};
+        for (int i = 0; i < n; ++i) {
+            const int t = g->h_slot_tenant[g0 + i];
+            const jnx_head& h = heads[t];
+            const jnx_head_opt& o = opt[t];
+            HeadOpt& ho = otab.slot[i];
+            const uint16_t* p[9] = {h.w1, h.b1, h.w2, h.b2, h.q, h.wk, h.wv, h.wout, h.bout};
+            for (int k = 0; k < 9; ++k) {
+                ho.master[k] = o.master[k];
+                ho.m[k] = o.m[k];
+                ho.v[k] = o.v[k];
+                ho.p[k] = const_cast<uint16_t*>(p[k]);
+            }
+            const int step = o.step + 1;
+            ho.c1 = (float)(1.0 / (1.0 - std::pow((double)hp->beta1, step)));
+            ho.c2 = (float)(1.0 / (1.0 - std::pow((double)hp->beta2, step)));
+        }
+        TraceScope ts(JNX_K_HEADS_BWD, heads_flops(tab, n, true), s);
+        if ((st = heads_backward_step_launch(tab, otab, ahp, b, w.sc, pooled, d, s))) return st;
+    }
+    for (int i = 0; i < g->n_slots; ++i) {
+        jnx_head_opt& o = opt[g->h_slot_tenant[i]];
+        ++o.step;
+        ++o.version;
+    }
+    return JNX_OK;
 }
 
 // ---------------------------------------------------------------------------

@@ -21,6 +21,8 @@
 // Loss (both): l_t = sum (y - t)^2 / (n_t * width), dy = 2 (y - t) / (n_t width).
 // All sums run in a fixed order inside one thread or one CTA (no atomics),
 // so a tenant's results are identical whether it runs grouped or alone.
+#include <type_traits>
+
 #include "jnx_dev.cuh"
 #include "jnx_heads.h"
 #include "jnx_kernels.h"
@@ -55,6 +57,56 @@ __device__ __forceinline__ void bf8_to_f(const uint4 w, float (&f)[8]) {
     f[7] = __uint_as_float(w.w & 0xFFFF0000u);
 }
 
+// Where a gradient kernel finishes a parameter's gradient element.  With
+// NoOpt it is stored into the slot's gradient buffer (added to it when the
+// slot accumulates); with HeadOptTable the element (plus the buffer's
+// accumulated value) goes straight into the tenant's AdamW update, and the
+// moments, fp32 master and bf16 parameter are rewritten instead.
+struct NoOpt {};
+template <class OT>
+constexpr bool kFused = std::is_same<OT, HeadOptTable>::value;
+
+__device__ __forceinline__ void opt_step1(const HeadOpt& o, int k, size_t i, float g,
+                                          const AdamHp& hp) {
+    float m = o.m[k][i], v = o.v[k][i];
+    const float p = adamw_elem(g, m, v, o.master[k][i], o.c1, o.c2, hp.lr, hp.b1, hp.b2, hp.eps,
+                               hp.wd);
+    o.m[k][i] = m;
+    o.v[k][i] = v;
+    o.master[k][i] = p;
+    o.p[k][i] = f2bf(p);
+}
+
+// four consecutive elements i .. i + 3 (i a multiple of 4; 16-byte state)
+__device__ __forceinline__ void opt_step4(const HeadOpt& o, int k, size_t i, float4 g,
+                                          const AdamHp& hp) {
+    float4 m = *reinterpret_cast<const float4*>(o.m[k] + i);
+    float4 v = *reinterpret_cast<const float4*>(o.v[k] + i);
+    float4 p = *reinterpret_cast<const float4*>(o.master[k] + i);
+    p.x = adamw_elem(g.x, m.x, v.x, p.x, o.c1, o.c2, hp.lr, hp.b1, hp.b2, hp.eps, hp.wd);
+    p.y = adamw_elem(g.y, m.y, v.y, p.y, o.c1, o.c2, hp.lr, hp.b1, hp.b2, hp.eps, hp.wd);
+    p.z = adamw_elem(g.z, m.z, v.z, p.z, o.c1, o.c2, hp.lr, hp.b1, hp.b2, hp.eps, hp.wd);
+    p.w = adamw_elem(g.w, m.w, v.w, p.w, o.c1, o.c2, hp.lr, hp.b1, hp.b2, hp.eps, hp.wd);
+    *reinterpret_cast<float4*>(o.m[k] + i) = m;
+    *reinterpret_cast<float4*>(o.v[k] + i) = v;
+    *reinterpret_cast<float4*>(o.master[k] + i) = p;
+    *reinterpret_cast<uint2*>(o.p[k] + i) = make_uint2(pack_bf2(p.x, p.y), pack_bf2(p.z, p.w));
+}
+
+// two consecutive elements i, i + 1 (i even; 8-byte state)
+__device__ __forceinline__ void opt_step2(const HeadOpt& o, int k, size_t i, float2 g,
+                                          const AdamHp& hp) {
+    float2 m = *reinterpret_cast<const float2*>(o.m[k] + i);
+    float2 v = *reinterpret_cast<const float2*>(o.v[k] + i);
+    float2 p = *reinterpret_cast<const float2*>(o.master[k] + i);
+    p.x = adamw_elem(g.x, m.x, v.x, p.x, o.c1, o.c2, hp.lr, hp.b1, hp.b2, hp.eps, hp.wd);
+    p.y = adamw_elem(g.y, m.y, v.y, p.y, o.c1, o.c2, hp.lr, hp.b1, hp.b2, hp.eps, hp.wd);
+    *reinterpret_cast<float2*>(o.m[k] + i) = m;
+    *reinterpret_cast<float2*>(o.v[k] + i) = v;
+    *reinterpret_cast<float2*>(o.master[k] + i) = p;
+    *reinterpret_cast<uint32_t*>(o.p[k] + i) = pack_bf2(p.x, p.y);
+}
+
 // ---------------------------------------------------------------------------
 // Segmented linear layer: out[s, j] = sum_k in[s, k] W[j, k] + b[j] over the
 // slot's samples.  One CTA per (slot, 32 output columns, 8 samples): warp w
@@ -75,7 +127,7 @@ __global__ void __launch_bounds__(256, 2) k_head_lin(const __grid_constant__ Hea
                                                   float* __restrict__ z_out, float* __restrict__ h_out,
                                                   int ld_out, const int* __restrict__ sample_target,
                                                   float* __restrict__ preds) {
-    __shared__ __align__(16) float sx[kLinS][kLinK];
+    __shared__ __align__(16) float sx[2][kLinS][kLinK];
     const HeadSlot& hs = tab.slot[blockIdx.x];
     if (LAYER == 1 && hs.kind != JNX_HEAD_MLP) return;
     const int J = LAYER == 1 ? hs.hid : hs.width;
@@ -92,41 +144,67 @@ __global__ void __launch_bounds__(256, 2) k_head_lin(const __grid_constant__ Hea
     for (int c = 0; c < kLinW; ++c)
 #pragma unroll
         for (int i = 0; i < kLinS; ++i) acc[c][i] = 0.f;
-    for (int k0 = 0; k0 < K; k0 += kLinK) {
-        const int nk = min(kLinK, K - k0);  // a multiple of 8
-        __syncthreads();
+    // the samples' input rows of one K chunk into staging buffer b
+    auto stage = [&](int b, int k0) {
+        const int nk = min(kLinK, K - k0);
         for (int i = threadIdx.x; i < kLinS * (kLinK / 4); i += 256) {
             const int r = i / (kLinK / 4), u = i % (kLinK / 4);
             float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
             if (r < ns && 4 * u < nk)
                 v = *reinterpret_cast<const float4*>(in + (size_t)(s0 + r) * ld_in + k0 + 4 * u);
-            *reinterpret_cast<float4*>(&sx[r][4 * u]) = v;
+            *reinterpret_cast<float4*>(&sx[b][r][4 * u]) = v;
         }
-        __syncthreads();
-        if (8 * lane < nk) {
+    };
+    // this lane's 16-byte weight chunks of a K chunk (zero past K or J)
+    auto load_w = [&](int k0, uint4 (&wv)[kLinW]) {
+        const bool in_k = 8 * lane < K - k0;
+#pragma unroll
+        for (int c = 0; c < kLinW; ++c)
+            wv[c] = (in_k && jw + c < J)
+                        ? __ldg(reinterpret_cast<const uint4*>(W + (size_t)(jw + c) * K + k0) + lane)
+                        : make_uint4(0, 0, 0, 0);
+    };
+    // the weights stream through registers one chunk ahead and the inputs
+    // through two staging buffers, so each chunk's loads are in flight
+    // during the previous chunk's arithmetic and one barrier closes a chunk
+    uint4 wv[kLinW];
+    load_w(0, wv);
+    stage(0, 0);
+    __syncthreads();
+    const int nch = (K + kLinK - 1) / kLinK;
+    for (int kc = 0; kc < nch; ++kc) {
+        const int b = kc & 1, k0 = kc * kLinK;
+        uint4 wn[kLinW];
+        if (kc + 1 < nch) {
+            load_w(k0 + kLinK, wn);
+            stage(b ^ 1, k0 + kLinK);
+        }
+        if (8 * lane < K - k0) {
             float x[kLinS][8];
 #pragma unroll
             for (int i = 0; i < kLinS; ++i) {
-                const float4 a = *reinterpret_cast<const float4*>(&sx[i][8 * lane]);
-                const float4 c4 = *reinterpret_cast<const float4*>(&sx[i][8 * lane + 4]);
+                const float4 a = *reinterpret_cast<const float4*>(&sx[b][i][8 * lane]);
+                const float4 c4 = *reinterpret_cast<const float4*>(&sx[b][i][8 * lane + 4]);
                 x[i][0] = a.x; x[i][1] = a.y; x[i][2] = a.z; x[i][3] = a.w;
                 x[i][4] = c4.x; x[i][5] = c4.y; x[i][6] = c4.z; x[i][7] = c4.w;
             }
 #pragma unroll
             for (int c = 0; c < kLinW; ++c) {
-                if (jw + c < J) {
-                    float wf[8];
-                    bf8_to_f(__ldg(reinterpret_cast<const uint4*>(W + (size_t)(jw + c) * K + k0) + lane),
-                             wf);
+                float wf[8];
+                bf8_to_f(wv[c], wf);
 #pragma unroll
-                    for (int i = 0; i < kLinS; ++i) {
-                        float t = acc[c][i];
+                for (int i = 0; i < kLinS; ++i) {
+                    float t = acc[c][i];
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) t = fmaf(x[i][e], wf[e], t);
-                        acc[c][i] = t;
-                    }
+                    for (int e = 0; e < 8; ++e) t = fmaf(x[i][e], wf[e], t);
+                    acc[c][i] = t;
                 }
             }
+        }
+        __syncthreads();
+        if (kc + 1 < nch) {
+#pragma unroll
+            for (int c = 0; c < kLinW; ++c) wv[c] = wn[c];
         }
     }
 #pragma unroll
@@ -182,7 +260,9 @@ __global__ void __launch_bounds__(256) k_l2_loss(const __grid_constant__ HeadTab
 // db[o] = sum_s dy[s, o], over the slot's samples in order.  One CTA per
 // (slot, 16 outputs o, 256 columns j); a thread keeps 4 o x 4 j; the
 // samples' dy and h rows are staged 32 at a time in shared memory.
+template <class OT>
 __global__ void __launch_bounds__(256) k_head_dw_out(const __grid_constant__ HeadTable tab,
+                                                     const __grid_constant__ OT opt, AdamHp hp,
                                                      const float* __restrict__ dy, int ld_y,
                                                      const float* __restrict__ h, int ld_h) {
     __shared__ __align__(16) float sh[32][256];
@@ -234,14 +314,22 @@ __global__ void __launch_bounds__(256) k_head_dw_out(const __grid_constant__ Hea
                 v.z += old.z;
                 v.w += old.w;
             }
-            *dst = v;
+            if constexpr (kFused<OT>)
+                opt_step4(opt.slot[blockIdx.x], hs.kind == JNX_HEAD_MLP ? 2 : 7,
+                          (size_t)o * hs.hid + j0, v, hp);
+            else
+                *dst = v;
         }
     }
     if (blockIdx.z == 0 && threadIdx.x < 16 && o0 + (int)threadIdx.x < hs.width) {
         const int o = o0 + threadIdx.x;
         float accb = 0.f;
         for (int s = hs.s0; s < hs.s1; ++s) accb += dy[(size_t)s * ld_y + o];
-        hs.g_b2[o] = hs.accum ? hs.g_b2[o] + accb : accb;
+        const float gb = hs.accum ? hs.g_b2[o] + accb : accb;
+        if constexpr (kFused<OT>)
+            opt_step1(opt.slot[blockIdx.x], hs.kind == JNX_HEAD_MLP ? 3 : 8, o, gb, hp);
+        else
+            hs.g_b2[o] = gb;
     }
 }
 
@@ -308,7 +396,9 @@ __global__ void __launch_bounds__(256) k_head_back_in(const __grid_constant__ He
 
 // MLP first-layer gradient: dW1[j, k] = sum_s dz[s, j] p[s, k]; db1[j] = sum_s dz[s, j].
 // One CTA per (slot, j, 1024-column block); float4 columns.
+template <class OT>
 __global__ void __launch_bounds__(256) k_mlp_dw1(const __grid_constant__ HeadTable tab,
+                                                 const __grid_constant__ OT opt, AdamHp hp,
                                                  const float* __restrict__ dz, int ld,
                                                  const float* __restrict__ p, int ld_p) {
     const HeadSlot& hs = tab.slot[blockIdx.x];
@@ -334,12 +424,19 @@ __global__ void __launch_bounds__(256) k_mlp_dw1(const __grid_constant__ HeadTab
             acc.z += old.z;
             acc.w += old.w;
         }
-        *dst = acc;
+        if constexpr (kFused<OT>)
+            opt_step4(opt.slot[blockIdx.x], 0, (size_t)j * hs.d_in + k4 * 4, acc, hp);
+        else
+            *dst = acc;
     }
     if (blockIdx.z == 0 && threadIdx.x == 0) {
         float accb = 0.f;
         for (int s = hs.s0; s < hs.s1; ++s) accb += dz[(size_t)s * ld + j];
-        hs.g_b1[j] = hs.accum ? hs.g_b1[j] + accb : accb;
+        const float gb = hs.accum ? hs.g_b1[j] + accb : accb;
+        if constexpr (kFused<OT>)
+            opt_step1(opt.slot[blockIdx.x], 1, j, gb, hp);
+        else
+            hs.g_b1[j] = gb;
     }
 }
 
@@ -619,7 +716,9 @@ __global__ void __launch_bounds__(256) k_xattn_bwd(const __grid_constant__ HeadT
 }
 
 // dQ_t = sum over the slot's samples (in order) of their contributions.
+template <class OT>
 __global__ void __launch_bounds__(256) k_xattn_dq(const __grid_constant__ HeadTable tab,
+                                                  const __grid_constant__ OT opt, AdamHp hp,
                                                   const float* __restrict__ dQs, int ld_h) {
     const HeadSlot& hs = tab.slot[blockIdx.x];
     if (hs.kind != JNX_HEAD_XATTN) return;
@@ -627,7 +726,11 @@ __global__ void __launch_bounds__(256) k_xattn_dq(const __grid_constant__ HeadTa
     if (i >= hs.nq * hs.dq) return;
     float acc = 0.f;
     for (int s = hs.s0; s < hs.s1; ++s) acc += dQs[(size_t)s * ld_h + i];
-    hs.g_q[i] = hs.accum ? hs.g_q[i] + acc : acc;
+    const float g = hs.accum ? hs.g_q[i] + acc : acc;
+    if constexpr (kFused<OT>)
+        opt_step1(opt.slot[blockIdx.x], 4, i, g, hp);
+    else
+        hs.g_q[i] = g;
 }
 
 // Query-head weight gradients, re-associated through the queries.  Per
@@ -639,11 +742,20 @@ __global__ void __launch_bounds__(256) k_xattn_dq(const __grid_constant__ HeadTa
 // steps run in fp32 on CUDA cores (X is exact in bf16), every sum in a fixed
 // order, so a tenant's gradients do not depend on the batch around it.
 //
-// k_xattn_gh: one CTA per (sample, 128 columns e of X); warp w takes
-// queries 4w..4w+3, a lane four consecutive columns; the sample's rows are
-// staged 32 at a time by cp.async (X rows, and the P / dS rows, nq floats
-// each, contiguous per sample).
-constexpr int kGhRows = 32;
+// k_xattn_gh: one CTA per (sample, 128 columns e of X), on the bf16 tensor
+// cores (mma.sync m16n8k16, fp32 accumulation).  X is bf16 already; P and dS
+// are fp32 and enter as two bf16 operands each, hi = bf16(P) and lo =
+// bf16(P - hi), so P X = hi X + lo X to about 2^-17 of P, i.e. within the
+// fp32 path's accuracy for these sums.  The sample's rows are staged 32 keys
+// at a time by cp.async (X rows into padded rows; the P / dS rows, nq
+// floats each, contiguous per sample), then split and transposed into
+// [query][key] operands in shared memory by all threads.  Warp w computes
+// columns e0 + 16 w .. + 15 (two 8-column tiles) for all 32 query rows (two
+// 16-row tiles; rows past nq are zero) of both products.  The key order of
+// the sums is fixed, so a sample's result does not depend on the group.
+constexpr int kGhRows = 32;       // keys per staged chunk
+constexpr int kGhXPad = 136;      // X row stride (bf16): conflict-free ldmatrix
+constexpr int kGhAPad = 40;       // [query][key] operand row stride (bf16)
 
 __global__ void __launch_bounds__(256) k_xattn_gh(const __grid_constant__ HeadTable tab, int g0,
                                                   const int* __restrict__ cu,
@@ -653,8 +765,11 @@ __global__ void __launch_bounds__(256) k_xattn_gh(const __grid_constant__ HeadTa
                                                   const uint16_t* __restrict__ X, int ldx,
                                                   float* __restrict__ Gs, float* __restrict__ Hs,
                                                   int ldg) {
-    __shared__ __align__(16) uint16_t sx[2][kGhRows][128];
+    static_assert(kMaxQ == 32, "two 16-row query tiles");
+    __shared__ __align__(16) uint16_t sx[2][kGhRows][kGhXPad];
     __shared__ __align__(16) float sp[2][kGhRows * kMaxQ], sd[2][kGhRows * kMaxQ];
+    // split operands: [P hi, P lo, dS hi, dS lo][query][key]
+    __shared__ __align__(16) uint16_t sa[4][kMaxQ][kGhAPad];
     const int s = sample0 + blockIdx.x;
     const HeadSlot& hs = tab.slot[sample_slot[s] - g0];
     if (hs.kind != JNX_HEAD_XATTN) return;
@@ -683,12 +798,16 @@ __global__ void __launch_bounds__(256) k_xattn_gh(const __grid_constant__ HeadTa
         }
     };
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const bool act = 4 * w < nq;
-    float g[4][4], h[4][4];
+    // acc[product: 0 = H (P), 1 = G (dS)][query tile][column tile][4]
+    float acc[2][2][2][4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int a = 0; a < 2; ++a)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) g[i][e] = h[i][e] = 0.f;
+        for (int m = 0; m < 2; ++m)
+#pragma unroll
+            for (int n = 0; n < 2; ++n)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) acc[a][m][n][e] = 0.f;
     const int nchunks = (L + kGhRows - 1) / kGhRows;
     if (nchunks > 0) load(0, 0);
     cp_async_commit();
@@ -698,33 +817,62 @@ __global__ void __launch_bounds__(256) k_xattn_gh(const __grid_constant__ HeadTa
         cp_async_commit();
         cp_async_wait<1>();
         __syncthreads();
-        if (act) {
-            const int nr = min(kGhRows, L - c * kGhRows);
-            for (int r = 0; r < nr; ++r) {
-                const uint2 xv = *reinterpret_cast<const uint2*>(&sx[buf][r][4 * lane]);
-                const float x[4] = {__uint_as_float(xv.x << 16), __uint_as_float(xv.x & 0xFFFF0000u),
-                                    __uint_as_float(xv.y << 16), __uint_as_float(xv.y & 0xFFFF0000u)};
-                const float4 p4 = *reinterpret_cast<const float4*>(&sp[buf][r * nq + 4 * w]);
-                const float4 d4 = *reinterpret_cast<const float4*>(&sd[buf][r * nq + 4 * w]);
-                const float pq[4] = {p4.x, p4.y, p4.z, p4.w}, dq[4] = {d4.x, d4.y, d4.z, d4.w};
+        // split and transpose: key j, query q of this chunk (rows past the
+        // sample's keys or queries past nq are zero); 4 elements a thread
+        const int nr = min(kGhRows, L - c * kGhRows);
+        for (int i = threadIdx.x; i < kGhRows * kMaxQ; i += 256) {
+            const int q = i >> 5, j = i & 31;
+            const bool ok = j < nr && q < nq;
+            const float pv = ok ? sp[buf][j * nq + q] : 0.f;
+            const float dv = ok ? sd[buf][j * nq + q] : 0.f;
+            const uint16_t ph = f2bf(pv), dh = f2bf(dv);
+            sa[0][q][j] = ph;
+            sa[1][q][j] = f2bf(pv - bf2f(ph));
+            sa[2][q][j] = dh;
+            sa[3][q][j] = f2bf(dv - bf2f(dh));
+        }
+        __syncthreads();
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
+        for (int k0 = 0; k0 < kGhRows; k0 += 16) {
+            // B: X rows k0..k0+15, this warp's 16 columns (two 8-column tiles)
+            uint32_t b[4];
+            {
+                const int kr = k0 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                const int col = 16 * w + (lane >> 4) * 8;
+                ldsm_x4_t(smem_u32(&sx[buf][kr][col]), b[0], b[1], b[2], b[3]);
+            }
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        h[i][e] = fmaf(pq[i], x[e], h[i][e]);
-                        g[i][e] = fmaf(dq[i], x[e], g[i][e]);
-                    }
+            for (int op = 0; op < 4; ++op) {  // P hi, P lo, dS hi, dS lo
+#pragma unroll
+                for (int m = 0; m < 2; ++m) {
+                    uint32_t a[4];
+                    const int qr = 16 * m + (lane & 7) + ((lane >> 3) & 1) * 8;
+                    const int kc = k0 + (lane >> 4) * 8;
+                    ldsm_x4(smem_u32(&sa[op][qr][kc]), a[0], a[1], a[2], a[3]);
+                    mma_bf16(acc[op >> 1][m][0], a[0], a[1], a[2], a[3], b[0], b[1]);
+                    mma_bf16(acc[op >> 1][m][1], a[0], a[1], a[2], a[3], b[2], b[3]);
+                }
             }
         }
         __syncthreads();
     }
-    if (!act) return;
+    // accumulator element e of tile (m, n): query 16 m + lane / 4 (+ 8 for
+    // e >= 2), column 16 w + 8 n + 2 (lane % 4) (+ 1 for odd e)
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const size_t o = ((size_t)s * kMaxQ + 4 * w + i) * ldg + e0 + 4 * lane;
-        *reinterpret_cast<float4*>(Gs + o) = make_float4(g[i][0], g[i][1], g[i][2], g[i][3]);
-        *reinterpret_cast<float4*>(Hs + o) = make_float4(h[i][0], h[i][1], h[i][2], h[i][3]);
-    }
+    for (int m = 0; m < 2; ++m)
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int q = 16 * m + (lane >> 2) + 8 * half;
+            if (q >= nq) continue;
+#pragma unroll
+            for (int n = 0; n < 2; ++n) {
+                const size_t o = ((size_t)s * kMaxQ + q) * ldg + e0 + 16 * w + 8 * n + 2 * (lane & 3);
+                *reinterpret_cast<float2*>(Hs + o) =
+                    make_float2(acc[0][m][n][2 * half], acc[0][m][n][2 * half + 1]);
+                *reinterpret_cast<float2*>(Gs + o) =
+                    make_float2(acc[1][m][n][2 * half], acc[1][m][n][2 * half + 1]);
+            }
+        }
 }
 
 // k_xattn_wgrad: one CTA per (slot, 32 value columns c, 64 columns e); warp
@@ -732,7 +880,9 @@ __global__ void __launch_bounds__(256) k_xattn_gh(const __grid_constant__ HeadTa
 // q = 4w..4w+3), a lane two consecutive columns e.  The slot's samples in
 // order: dWv += dO_s^T H_s with dO_s [nq, 32] and H_s [nq, 64] staged; at the
 // end dWk = scale Q^T G_t with G_t staged.
+template <class OT>
 __global__ void __launch_bounds__(256) k_xattn_wgrad(const __grid_constant__ HeadTable tab,
+                                                     const __grid_constant__ OT opt, AdamHp hp,
                                                      const float* __restrict__ Gs,
                                                      const float* __restrict__ Hs, int ldg,
                                                      const float* __restrict__ dO, int ld_h) {
@@ -811,8 +961,13 @@ __global__ void __launch_bounds__(256) k_xattn_wgrad(const __grid_constant__ Hea
             vv.x += ov.x;
             vv.y += ov.y;
         }
-        *reinterpret_cast<float2*>(hs.g_wk + o) = vk;
-        *reinterpret_cast<float2*>(hs.g_wv + o) = vv;
+        if constexpr (kFused<OT>) {
+            opt_step2(opt.slot[blockIdx.x], 5, o, vk, hp);
+            opt_step2(opt.slot[blockIdx.x], 6, o, vv, hp);
+        } else {
+            *reinterpret_cast<float2*>(hs.g_wk + o) = vk;
+            *reinterpret_cast<float2*>(hs.g_wv + o) = vv;
+        }
     }
 }
 
@@ -851,26 +1006,67 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
                                  const float* pooled, int d, const uint16_t* hidden,
                                  const int* cu, const int* sample_slot, cudaStream_t s) {
     if (b.n == 0) return JNX_OK;
-    k_head_dw_out<<<dim3(b.n, (b.max_width + 15) / 16, (b.max_hid + 255) / 256), 256, 0, s>>>(
-        tab, ws.dy, ws.ld_y, ws.h, ws.ld_h);
+    const NoOpt no{};
+    const AdamHp nh{};
+    k_head_dw_out<NoOpt>
+        <<<dim3(b.n, (b.max_width + 15) / 16, (b.max_hid + 255) / 256), 256, 0, s>>>(
+            tab, no, nh, ws.dy, ws.ld_y, ws.h, ws.ld_h);
     k_head_back_in<<<dim3(b.n, (b.max_hid + 1023) / 1024, (b.max_ns + 7) / 8), 256, 0, s>>>(
         tab, ws.dy, ws.ld_y, ws.z, ws.ld_h, ws.dh);
     if (b.any_mlp)
-        k_mlp_dw1<<<dim3(b.n, b.max_mlp_hid, (d / 4 + 255) / 256), 256, 0, s>>>(tab, ws.dh,
-                                                                               ws.ld_h, pooled, d);
+        k_mlp_dw1<NoOpt><<<dim3(b.n, b.max_mlp_hid, (d / 4 + 255) / 256), 256, 0, s>>>(
+            tab, no, nh, ws.dh, ws.ld_h, pooled, d);
     if (b.any_xattn) {
         const size_t smem = xattn_smem_bytes(b.max_dq);
         k_xattn_bwd<<<b.sample1 - b.sample0, 256, smem, s>>>(
             tab, b.g0, cu, sample_slot, b.sample0, ws.kbuf, ws.vbuf, ws.ldkv, ws.P, ws.dS, ws.dh,
             ws.ld_h, ws.dk, ws.dv, ws.dQs);
-        k_xattn_dq<<<dim3(b.n, (b.max_nq * b.max_dq + 255) / 256), 256, 0, s>>>(tab, ws.dQs,
-                                                                                 ws.ld_h);
+        k_xattn_dq<NoOpt><<<dim3(b.n, (b.max_nq * b.max_dq + 255) / 256), 256, 0, s>>>(
+            tab, no, nh, ws.dQs, ws.ld_h);
         k_xattn_gh<<<dim3(b.sample1 - b.sample0, d / 128), 256, 0, s>>>(
             tab, b.g0, cu, sample_slot, b.sample0, ws.P, ws.dS, hidden, d, ws.Gs, ws.Hs, d);
-        k_xattn_wgrad<<<dim3(b.n, b.max_dq / 32, d / 64), 256, 0, s>>>(tab, ws.Gs, ws.Hs, d, ws.dh,
-                                                                       ws.ld_h);
+        k_xattn_wgrad<NoOpt><<<dim3(b.n, b.max_dq / 32, d / 64), 256, 0, s>>>(
+            tab, no, nh, ws.Gs, ws.Hs, d, ws.dh, ws.ld_h);
     }
     return cuda_ok("heads backward");
+}
+
+jnx_status heads_backward_front_launch(const HeadTable& tab, const HeadBatch& b,
+                                       const HeadScratch& ws, int d, const uint16_t* hidden,
+                                       const int* cu, const int* sample_slot, cudaStream_t s) {
+    if (b.n == 0) return JNX_OK;
+    k_head_back_in<<<dim3(b.n, (b.max_hid + 1023) / 1024, (b.max_ns + 7) / 8), 256, 0, s>>>(
+        tab, ws.dy, ws.ld_y, ws.z, ws.ld_h, ws.dh);
+    if (b.any_xattn) {
+        const size_t smem = xattn_smem_bytes(b.max_dq);
+        k_xattn_bwd<<<b.sample1 - b.sample0, 256, smem, s>>>(
+            tab, b.g0, cu, sample_slot, b.sample0, ws.kbuf, ws.vbuf, ws.ldkv, ws.P, ws.dS, ws.dh,
+            ws.ld_h, ws.dk, ws.dv, ws.dQs);
+        k_xattn_gh<<<dim3(b.sample1 - b.sample0, d / 128), 256, 0, s>>>(
+            tab, b.g0, cu, sample_slot, b.sample0, ws.P, ws.dS, hidden, d, ws.Gs, ws.Hs, d);
+    }
+    return cuda_ok("heads backward");
+}
+
+jnx_status heads_backward_step_launch(const HeadTable& tab, const HeadOptTable& opt,
+                                      const AdamHp& hp, const HeadBatch& b,
+                                      const HeadScratch& ws, const float* pooled, int d,
+                                      cudaStream_t s) {
+    if (b.n == 0) return JNX_OK;
+    k_head_dw_out<HeadOptTable>
+        <<<dim3(b.n, (b.max_width + 15) / 16, (b.max_hid + 255) / 256), 256, 0, s>>>(
+            tab, opt, hp, ws.dy, ws.ld_y, ws.h, ws.ld_h);
+    if (b.any_mlp)
+        k_mlp_dw1<HeadOptTable><<<dim3(b.n, b.max_mlp_hid, (d / 4 + 255) / 256), 256, 0, s>>>(
+            tab, opt, hp, ws.dh, ws.ld_h, pooled, d);
+    if (b.any_xattn) {
+        // wgrad reads the learned queries, which dq then updates
+        k_xattn_wgrad<HeadOptTable><<<dim3(b.n, b.max_dq / 32, d / 64), 256, 0, s>>>(
+            tab, opt, hp, ws.Gs, ws.Hs, d, ws.dh, ws.ld_h);
+        k_xattn_dq<HeadOptTable><<<dim3(b.n, (b.max_nq * b.max_dq + 255) / 256), 256, 0, s>>>(
+            tab, opt, hp, ws.dQs, ws.ld_h);
+    }
+    return cuda_ok("heads backward step");
 }
 
 jnx_status heads_set_smem() {

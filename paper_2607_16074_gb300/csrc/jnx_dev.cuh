@@ -91,6 +91,24 @@ __device__ __forceinline__ void ex2_poly2(float x0, float x1, float& p0, float& 
     p1 = __uint_as_float(__float_as_uint(q1) + (__float_as_uint(t1) << 23));
 }
 
+// One AdamW update of a parameter element (bias-corrected moments, weight
+// decay decoupled from the gradient and applied to the parameter before the
+// step): updates the moments in place and returns the new fp32 parameter.
+// c1 = 1 / (1 - beta1^t), c2 = 1 / (1 - beta2^t).  Shared by the optimizer
+// kernel and the heads backward's fused step.  Every operation is an
+// explicitly rounded one (no contraction into fused multiply-adds, whose
+// choice the compiler may make differently at each inlined copy), so every
+// copy gives the same bits.
+__device__ __forceinline__ float adamw_elem(float g, float& m, float& v, float p, float c1,
+                                            float c2, float lr, float b1, float b2, float eps,
+                                            float wd) {
+    m = __fadd_rn(__fmul_rn(b1, m), __fmul_rn(__fsub_rn(1.f, b1), g));
+    v = __fadd_rn(__fmul_rn(b2, v), __fmul_rn(__fmul_rn(__fsub_rn(1.f, b2), g), g));
+    const float den = __fadd_rn(__fsqrt_rn(__fmul_rn(v, c2)), eps);
+    const float upd = __fadd_rn(__fdiv_rn(__fmul_rn(m, c1), den), __fmul_rn(wd, p));
+    return __fsub_rn(p, __fmul_rn(lr, upd));
+}
+
 // Record the first device-side error in the status word (never traps).
 __device__ __forceinline__ void report(int* status, int code) {
     if (status) atomicCAS(status, 0, code);

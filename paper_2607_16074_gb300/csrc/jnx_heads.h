@@ -31,6 +31,25 @@ struct HeadTable {
     HeadSlot slot[kMaxSlots];
 };
 
+// The fused optimizer step of the heads backward: per slot, the AdamW state
+// of its 9 possible parameter tensors (jnx_head_opt order: w1, b1, w2, b2,
+// q, wk, wv, wout, bout; the output layer's are 2, 3 for an MLP head and
+// 7, 8 for a query head), the bf16 parameters it rewrites and the bias
+// corrections of this step.
+struct HeadOpt {
+    float* master[9];
+    float* m[9];
+    float* v[9];
+    uint16_t* p[9];
+    float c1, c2;
+};
+struct HeadOptTable {
+    HeadOpt slot[kMaxSlots];
+};
+struct AdamHp {
+    float lr, b1, b2, eps, wd;
+};
+
 // What one launch batch of slots holds.
 struct HeadBatch {
     int g0, n;                 // group slots [g0, g0 + n)
@@ -61,6 +80,22 @@ jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const 
 jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const HeadScratch& ws,
                                  const float* pooled, int d, const uint16_t* hidden,
                                  const int* cu, const int* sample_slot, cudaStream_t s);
+// The backward with the tenant-private AdamW step fused into it, in two
+// launches so that nothing updates a parameter before every read of it:
+// front: the output layer's input gradient (reads W2 / Wout) and the query
+// heads' attention backward (reads the learned queries); the caller may
+// then form the feature gradient (reads W1, Wk, Wv); step: every
+// parameter's gradient element goes straight into its AdamW update (plus
+// the accumulated gradient buffer when the slots accumulate) and is not
+// stored; the query heads' Wk/Wv kernel (reads the queries) runs before
+// the queries' own update.
+jnx_status heads_backward_front_launch(const HeadTable& tab, const HeadBatch& b,
+                                       const HeadScratch& ws, int d, const uint16_t* hidden,
+                                       const int* cu, const int* sample_slot, cudaStream_t s);
+jnx_status heads_backward_step_launch(const HeadTable& tab, const HeadOptTable& opt,
+                                      const AdamHp& hp, const HeadBatch& b,
+                                      const HeadScratch& ws, const float* pooled, int d,
+                                      cudaStream_t s);
 jnx_status heads_set_smem();
 
 }  // namespace jnx

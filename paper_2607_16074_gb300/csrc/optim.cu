@@ -36,14 +36,6 @@ struct AdamTable {
     AdamSeg seg[kMaxSeg];
 };
 
-__device__ __forceinline__ float adamw_elem(float g, float& m, float& v, float p, float c1,
-                                            float c2, float lr, float b1, float b2, float eps,
-                                            float wd) {
-    m = b1 * m + (1.f - b1) * g;
-    v = b2 * v + (1.f - b2) * g * g;
-    return p - lr * ((m * c1) / (sqrtf(v * c2) + eps) + wd * p);
-}
-
 // Four elements per thread (16-byte loads) where the segment's arrays allow
 // it, then a scalar tail.
 __global__ void __launch_bounds__(256) k_adamw(const __grid_constant__ AdamTable tab, float lr,

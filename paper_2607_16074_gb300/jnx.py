@@ -175,7 +175,8 @@ EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_group_attn_it
            "jnx_op_final_pool", "jnx_trace_enable", "jnx_trace_disable", "jnx_trace_count",
            "jnx_trace_read", "jnx_op_gemm_rope_noalloc", "jnx_op_gemm_rope_noalloc_status",
            "jnx_sched_poll", "jnx_diag_ex2_poly", "jnx_diag_bounded_wait",
-           "jnx_heads_backward_accumulate", "jnx_heads_adamw", "jnx_backbone_saved_bytes",
+           "jnx_heads_backward_accumulate", "jnx_heads_adamw", "jnx_heads_backward_adamw",
+           "jnx_backbone_saved_bytes",
            "jnx_backbone_forward_train", "jnx_heads_backward_input", "jnx_transpose",
            "jnx_backbone_backward_workspace_bytes", "jnx_backbone_backward_lora",
            "jnx_op_attention_lse", "jnx_op_attention_backward_prep",
@@ -218,6 +219,10 @@ def lib() -> C.CDLL:
         "jnx_heads_adamw": (i32, [C.POINTER(jnx_head), C.POINTER(jnx_head_grads),
                                   C.POINTER(jnx_head_opt), i32, C.POINTER(jnx_group),
                                   C.POINTER(jnx_adamw), vp]),
+        "jnx_heads_backward_adamw": (i32, [C.POINTER(jnx_head), i32, C.POINTER(jnx_group), vp, vp,
+                                           vp, C.POINTER(jnx_head_grads), i32,
+                                           C.POINTER(jnx_head_opt), C.POINTER(jnx_adamw), vp, vp,
+                                           sz, vp]),
         "jnx_backbone_saved_bytes": (sz, [C.POINTER(jnx_backbone), i32]),
         "jnx_backbone_forward_train": (i32, [C.POINTER(jnx_backbone), C.POINTER(jnx_group), vp,
                                              i64, vp, i64, vp, vp, vp, vp, sz, vp]),

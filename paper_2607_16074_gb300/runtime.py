@@ -264,6 +264,21 @@ class DeviceHeads:
         J.check(J.lib().jnx_heads_adamw(self.arr, self.garr, self.opt, self.n, group.ref,
                                         C.byref(hp), _stream(stream)))
 
+    def backward_adamw(self, group: DeviceGroup, pooled, hidden, targets, ws, lr: float,
+                       beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8,
+                       weight_decay: float = 0.0, accumulate: bool = False, d_hidden=None,
+                       stream=None) -> None:
+        """The heads backward with every group tenant's AdamW step fused into
+        it: the same result as backward() then adamw_step(), without storing
+        the gradients (with accumulate=True the gradients already in the
+        slots are added first).  d_hidden, if given, receives the gradient at
+        the final normed rows (as backward_input)."""
+        hp = J.jnx_adamw(lr, beta1, beta2, eps, weight_decay)
+        J.check(J.lib().jnx_heads_backward_adamw(
+            self.arr, self.n, group.ref, _ptr(pooled), _ptr(hidden), _ptr(targets), self.garr,
+            1 if accumulate else 0, self.opt, C.byref(hp), _ptr(d_hidden), ws.data_ptr(),
+            ws.numel() * ws.element_size(), _stream(stream)))
+
     def version(self, t: int) -> int:
         return int(self.opt[t].version)
 

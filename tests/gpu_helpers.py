@@ -6,7 +6,7 @@ import synth
 from oracle import model as M
 from paper_2607_16074_gb300 import jnx as J
 from paper_2607_16074_gb300 import runtime as R
-from tests.helpers import BF16_TOL, gate, oracle_requests, rel_err
+from tests.helpers import SAMPLE_FLOOR_FACTOR, gate, oracle_requests, rel_err
 
 
 def dev():
@@ -127,9 +127,10 @@ def check_tenants(name, setup, plan, step, preds, pick):
     gated by gate(floor): the stated 2e-2, or FLOOR_FACTOR times the floor
     that the CUDA path's own roundings set (the emulated forward's distance
     from the oracle, and the oracle's head step on the emulated features).
-    Checks every sample's features (pooled, or final normed rows for a
-    query head), each tenant's predictions, loss and head gradients; prints
-    every number.  Returns the largest ratio of GPU error to floor."""
+    Checks each tenant's features (pooled, or final normed rows for a query
+    head) as a whole and every sample's (at SAMPLE_FLOOR_FACTOR), each
+    tenant's predictions, loss and head gradients; prints every number.
+    Returns the largest ratio of GPU error to floor at FLOOR_FACTOR gates."""
     w = setup.w
     feats = oracle_and_floor(setup, pick)
     idx = packed_index(plan, w)
@@ -139,21 +140,28 @@ def check_tenants(name, setup, plan, step, preds, pick):
     loss = step.loss.cpu().numpy()
     worst = 0.0
 
-    def one(what, e, fl):
+    def one(what, e, fl, factor=None):
         nonlocal worst
-        worst = max(worst, e / max(fl, 1e-300))
-        print(f"{name} {what}: gpu {e:.4e}  floor {fl:.4e}  gate {gate(fl):.4e}")
-        assert e <= gate(fl), (name, what, e, fl)
+        gt = gate(fl) if factor is None else gate(fl, factor)
+        if factor is None:
+            worst = max(worst, e / max(fl, 1e-300))
+        print(f"{name} {what}: gpu {e:.4e}  floor {fl:.4e}  ratio {e / max(fl, 1e-300):.3f}  "
+              f"gate {gt:.4e}")
+        assert e <= gt, (name, what, e, fl)
 
     for t in pick:
         tn = w.tenants[t]
         mlp = tn.head_kind == synth.HEAD_MLP
         samples = tenant_samples(w, t)
-        for k, i in enumerate(idx[t]):
-            g = pooled[i] if mlp else hid[cu[i]:cu[i + 1]]
+        kind = "pooled" if mlp else "rows"
+        gs = [pooled[i] if mlp else hid[cu[i]:cu[i + 1]] for i in idx[t]]
+        for k, g in enumerate(gs):
             r, e = feats[t]["ref"][k], feats[t]["emu"][k]
-            one(f"tenant {t} sample {k} {'pooled' if mlp else 'rows'}", rel_err(g, r),
-                rel_err(e, r))
+            one(f"tenant {t} sample {k} {kind}", rel_err(g, r), rel_err(e, r),
+                SAMPLE_FLOOR_FACTOR)
+        cat = lambda xs: np.concatenate([np.ravel(x) for x in xs])
+        R_, E_ = cat(feats[t]["ref"]), cat(feats[t]["emu"])
+        one(f"tenant {t} all samples' {kind}", rel_err(cat(gs), R_), rel_err(E_, R_))
         hw = M.widen_tree(synth.to_numpy_tree(setup.hw[t]))
         T = np.stack([setup.inp["targets"][smp.target_off:smp.target_off + tn.width]
                       .double().cpu().numpy() for smp in samples])

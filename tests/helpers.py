@@ -27,12 +27,17 @@ GROUPED_TOL = 1e-3   # GPU grouped vs GPU per-tenant isolated
 # BF16_TOL from the fp64 oracle, the GPU may be at most this factor beyond
 # the floor those formats alone set (computed in fp64, never on the GPU).
 FLOOR_FACTOR = 1.3
+# One sample's max|err|/rms is set by a few elements, and at shallow depth
+# by where the bf16 output rounding of the GPU and of the emulation happen
+# to land; it is gated at this wider factor, the tenant's results as a whole
+# at FLOOR_FACTOR.
+SAMPLE_FLOOR_FACTOR = 1.5
 
 
-def gate(floor: float) -> float:
+def gate(floor: float, factor: float = FLOOR_FACTOR) -> float:
     """The bound a floating-point result is held to: the stated BF16_TOL, or
-    FLOOR_FACTOR times the floor its storage formats set, if that is larger."""
-    return max(BF16_TOL, FLOOR_FACTOR * floor)
+    factor times the floor its storage formats set, if that is larger."""
+    return max(BF16_TOL, factor * floor)
 
 
 def rel_err_bf16_out(got, ref):
