@@ -105,19 +105,21 @@ __device__ __forceinline__ AttnWork attn_fetch(const AttnItems& it, const int* _
     return a;
 }
 
-// Epilogue staging (as in the GEMM epilogue): thread `lane` puts its row's
-// 64 bytes; in step i thread `lane` gets row 8 i + lane / 4, 16-byte unit
-// lane % 4.  Units are XOR-swizzled by (row / 2) % 4 (no bank conflicts).
-__device__ __forceinline__ void attn_stg_put(uint8_t* stg, int lane, const uint4 (&v)[4]) {
-    uint8_t* rowp = stg + lane * 64;
-    const int sw = (lane >> 1) & 3;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) *reinterpret_cast<uint4*>(rowp + ((j ^ sw) << 4)) = v[j];
+// Epilogue staging of 16 output columns (32 bytes a row) through a 1 KB
+// slot per softmax warp: thread `lane` puts its row's two 16-byte units;
+// in round i thread `lane` gets row 16 i + lane / 2, unit lane % 2, so each
+// store instruction writes 16 rows x 32 contiguous bytes.  Units are
+// XOR-swizzled by (row / 4) % 2 (no bank conflicts either way).
+__device__ __forceinline__ void attn_stg_put(uint8_t* stg, int lane, const uint4 (&v)[2]) {
+    uint8_t* rowp = stg + lane * 32;
+    const int sw = (lane >> 2) & 1;
+    *reinterpret_cast<uint4*>(rowp + ((0 ^ sw) << 4)) = v[0];
+    *reinterpret_cast<uint4*>(rowp + ((1 ^ sw) << 4)) = v[1];
 }
 
 __device__ __forceinline__ uint4 attn_stg_get(const uint8_t* stg, int lane, int i) {
-    const int r = 8 * i + (lane >> 2), j = lane & 3;
-    return *reinterpret_cast<const uint4*>(stg + r * 64 + ((j ^ ((r >> 1) & 3)) << 4));
+    const int r = 16 * i + (lane >> 1), j = lane & 1;
+    return *reinterpret_cast<const uint4*>(stg + r * 32 + ((j ^ ((r >> 2) & 1)) << 4));
 }
 
 template <int HD, int BN>
@@ -127,7 +129,12 @@ struct AttnWsCfg {
     // streams per CTA: a stream holds two BN-column score buffers and an
     // HD-column O in TMEM (512 columns), so head dim 256 runs one stream
     static constexpr int NST = HD == 256 ? 1 : 2;
-    static constexpr int THREADS = 128 + 128 * NST;
+    // softmax warpgroups per stream: each takes half of a tile's columns
+    // (and half of O's columns in the epilogue) for all 128 rows
+    static constexpr int SPLIT = 2;
+    static constexpr int HCOLS = BN / SPLIT;   // score columns per softmax thread
+    static constexpr int SMW = 4 * SPLIT * NST;  // softmax warps
+    static constexpr int THREADS = 128 + 32 * SMW;
     static constexpr uint32_t TSTRIDE = 256;  // TMEM columns between streams
     static constexpr int BM = attn_ws::BM;
     static constexpr int QB = BM * HD * 2;  // Q tile
@@ -135,84 +142,69 @@ struct AttnWsCfg {
     static constexpr int OFF_K = QB;
     static constexpr int OFF_V = OFF_K + 2 * KB;
     static constexpr int STREAM = OFF_V + 2 * KB;  // bytes per stream (multiple of 1024)
-    static constexpr int OFF_STG = NST * STREAM;  // epilogue staging, 2 KB per softmax warp
-    static constexpr int OFF_BAR = OFF_STG + 4 * NST * 2048;
-    static constexpr int SMEM = OFF_BAR + NST * attn_ws::kBars * 8 + 16 + 1024;
+    static constexpr int OFF_STG = NST * STREAM;  // epilogue staging, 1 KB per softmax warp
+    // row-max / row-sum exchange between a stream's two halves:
+    // [stream][slot 0/1][half][BM] floats
+    static constexpr int OFF_XM = OFF_STG + SMW * 1024;
+    static constexpr int OFF_BAR = OFF_XM + NST * 2 * SPLIT * BM * 4;
+    static constexpr int NBAR = attn_ws::kBars + 8;  // + exchange barriers [quarter][slot]
+    static constexpr int SMEM = OFF_BAR + NST * NBAR * 8 + 16 + 1024;
     static_assert(STREAM % 1024 == 0, "128B-swizzled tiles need 1024-byte alignment");
     static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
     static constexpr uint32_t O_COL = 2 * BN;  // within the stream's 256 columns
     static_assert(O_COL + HD <= (NST == 2 ? TSTRIDE : 512), "TMEM columns per stream");
 };
 
-// Softmax of one 128 x BN score tile for this thread's row: row max (pass
-// 1), then probabilities packed as bf16 pairs (pass 2).  FULL: every key of
-// the tile lies inside the sample (no mask).
-// The exponential of one key pair in four: ex2_poly2 (jnx_dev.cuh).
-template <int BN, bool FULL>
-__device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float scale_log2,
-                                                bool first, float& m, float& alpha, float& rs,
-                                                uint32_t (&pk)[BN / 2]) {
-    static_assert(BN == 64, "one S row is two 32-column TMEM loads");
-    // the whole S row in one TMEM round trip
-    uint32_t v[2][32];
-    tmem_ld32(tS, v[0]);
-    tmem_ld32(tS + 32, v[1]);
-    tmem_ld_wait();
-    // row max into 4 independent partial results (then a tree), so it is not
-    // one 64-long dependent chain; full tiles take two keys per instruction
+// Softmax of one 128 x 64 score tile, split between two threads per row:
+// this thread holds 32 of the row's scores (v) and kvalid of them lie in
+// the sample (FULL: all 32).  attn_half_max: the raw max of the valid ones;
+// attn_half_exp: p = 2^(s scale - m) packed as bf16 pairs, and their sum.
+// The exponential of one key pair in four: ex2_poly2 (jnx_dev.cuh), which
+// takes load off the MUFU pipe the softmax warps share.
+template <bool FULL>
+__device__ __forceinline__ float attn_half_max(const uint32_t (&v)[32], int kvalid) {
     float mx4[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) mx4[j] = -INFINITY;
 #pragma unroll
-    for (int c = 0; c < 2; ++c)
-#pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-            const float a0 = __uint_as_float(v[c][e]), a1 = __uint_as_float(v[c][e + 1]);
-            float& acc = mx4[(e >> 1) & 3];
-            if (FULL) {
-                acc = fmax3(acc, a0, a1);
-            } else {
-                if (c * 32 + e < kvalid) acc = fmaxf(acc, a0);
-                if (c * 32 + e + 1 < kvalid) acc = fmaxf(acc, a1);
-            }
+    for (int e = 0; e < 32; e += 2) {
+        const float a0 = __uint_as_float(v[e]), a1 = __uint_as_float(v[e + 1]);
+        float& acc = mx4[(e >> 1) & 3];
+        if (FULL) {
+            acc = fmax3(acc, a0, a1);
+        } else {
+            if (e < kvalid) acc = fmaxf(acc, a0);
+            if (e + 1 < kvalid) acc = fmaxf(acc, a1);
         }
-    float mx = fmax3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3]));
-    mx *= scale_log2;
-    alpha = 1.f;
-    if (first) {
-        m = mx;
-    } else if (mx > m + attn_ws::kLazy) {
-        alpha = ex2_approx(m - mx);
-        m = mx;
     }
-    // p = 2^(s scale - m): the argument of two keys per packed FMA, the row
-    // sum in two packed partial sums
+    return fmax3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3]));
+}
+
+template <bool FULL>
+__device__ __forceinline__ void attn_half_exp(const uint32_t (&v)[32], int kvalid,
+                                              float scale_log2, float m, float& rs,
+                                              uint32_t (&pk)[16]) {
     const uint64_t sc2 = f2_pack(scale_log2, scale_log2), nm2 = f2_pack(-m, -m);
     uint64_t rs2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
 #pragma unroll
-    for (int c = 0; c < 2; ++c)
-#pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-            float x0, x1;
-            f2_unpack(f2_fma(f2_pack(__uint_as_float(v[c][e]), __uint_as_float(v[c][e + 1])), sc2,
-                             nm2),
-                      x0, x1);
-            float p0, p1;
-            // on full tiles one pair in four goes to the FMA pipe, which
-            // relieves the MUFU pipe the two streams' softmax warps share
-            if (FULL && ((e >> 1) & 3) == 3) {
-                ex2_poly2(x0, x1, p0, p1);
-            } else {
-                p0 = ex2_approx(x0);
-                p1 = ex2_approx(x1);
-            }
-            if (!FULL) {
-                if (c * 32 + e >= kvalid) p0 = 0.f;
-                if (c * 32 + e + 1 >= kvalid) p1 = 0.f;
-            }
-            rs2[(e >> 1) & 1] = f2_add(rs2[(e >> 1) & 1], f2_pack(p0, p1));
-            pk[c * 16 + e / 2] = pack_bf2(p0, p1);
+    for (int e = 0; e < 32; e += 2) {
+        float x0, x1;
+        f2_unpack(f2_fma(f2_pack(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), sc2, nm2),
+                  x0, x1);
+        float p0, p1;
+        if (FULL && ((e >> 1) & 3) == 3) {
+            ex2_poly2(x0, x1, p0, p1);
+        } else {
+            p0 = ex2_approx(x0);
+            p1 = ex2_approx(x1);
         }
+        if (!FULL) {
+            if (e >= kvalid) p0 = 0.f;
+            if (e + 1 >= kvalid) p1 = 0.f;
+        }
+        rs2[(e >> 1) & 1] = f2_add(rs2[(e >> 1) & 1], f2_pack(p0, p1));
+        pk[e / 2] = pack_bf2(p0, p1);
+    }
     float r0, r1, r2, r3;
     f2_unpack(rs2[0], r0, r1);
     f2_unpack(rs2[1], r2, r3);
@@ -220,7 +212,7 @@ __device__ __forceinline__ void attn_ws_softmax(uint32_t tS, int kvalid, float s
 }
 
 template <int HD, int BN>
-__global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
+__global__ void __launch_bounds__(HD == 256 ? 384 : 640, 1)
     k_attn_ws(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tkv,
               const int* __restrict__ cu, AttnItems items, int H, int Hkv, float scale_log2,
               uint16_t* __restrict__ out, int ldo, float* __restrict__ lse, int* status) {
@@ -230,17 +222,19 @@ __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + C::OFF_BAR + C::NST * attn_ws::kBars * 8);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + C::OFF_BAR + C::NST * C::NBAR * 8);
     volatile int* fail_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    // stream of this warp: producers 0/1, MMA issuers 2/3, softmax 4-7 / 8-11
-    const int t = warp < 4 ? (warp & 1) : (warp - 4) >> 2;
+    // stream of this warp: producers 0/1, MMA issuers 2/3, then per stream
+    // 4 SPLIT softmax warps (stream t, half h, lane quarter q: warp
+    // 4 + 4 SPLIT t + 4 h + q, so warp % 4 = q)
+    const int t = warp < 4 ? (warp & 1) : (warp - 4) / (4 * C::SPLIT);
     uint8_t* st = sm + t * C::STREAM;
     uint8_t* sQ = st;
     auto sK = [&](int b) { return st + C::OFF_K + b * C::KB; };
     auto sV = [&](int b) { return st + C::OFF_V + b * C::KB; };
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR) + t * attn_ws::kBars;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR) + t * C::NBAR;
     uint64_t* q_full = bars + 0;
     uint64_t* q_empty = bars + 1;
     uint64_t* k_full = bars + 2;   // [2]
@@ -252,17 +246,21 @@ __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
     uint64_t* o_done = bars + 14;  // [2]
     uint64_t* o_free = bars + 16;
     uint64_t* drain = bars + 17;
+    uint64_t* xbar = bars + attn_ws::kBars;  // [quarter][slot]: the halves' exchanges
 
     const int n_work = items.n * H;
     const int group = H / Hkv;
     const int w0 = C::NST * blockIdx.x + t, dw = C::NST * gridDim.x;
     if (tid == 0) {
         // both streams' barriers: one arrival each, but p_full[] and o_free,
-        // which every softmax thread of the stream arrives on
+        // which every softmax thread of the stream arrives on, and the
+        // exchange barriers, which the 64 threads of a warp pair arrive on
         uint64_t* all = reinterpret_cast<uint64_t*>(sm + C::OFF_BAR);
-        for (int i = 0; i < C::NST * attn_ws::kBars; ++i) {
-            const int k = i % attn_ws::kBars;
-            mbar_init(&all[i], (k == 12 || k == 13 || k == 16) ? BM : 1);
+        for (int i = 0; i < C::NST * C::NBAR; ++i) {
+            const int k = i % C::NBAR;
+            mbar_init(&all[i], k >= attn_ws::kBars                  ? 64
+                               : (k == 12 || k == 13 || k == 16) ? C::SPLIT * BM
+                                                                 : 1);
         }
         *fail_flag = 0;
         fence_barrier_init();
@@ -410,11 +408,18 @@ __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
         }
     } else {
         // ---------------- softmax + epilogue of stream t ----------------
+        // This thread: row quarter * 32 + lane of the item's query tile,
+        // score columns [32 half, 32 half + 32) of each key tile, O columns
+        // [HD/2 half, HD/2 half + HD/2) in the epilogue.
         const int quarter = warp & 3;  // TMEM lanes this warp may access
+        const int half = ((warp - 4) >> 2) % C::SPLIT;
+        const int row = quarter * 32 + lane;
         const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-        const uint32_t tO = tbase + lane_base + C::O_COL;
+        const uint32_t tO = tbase + lane_base + C::O_COL + half * (HD / 2);
+        float* xm = reinterpret_cast<float*>(sm + C::OFF_XM) + t * 2 * C::SPLIT * BM;
         uint32_t gs = 0;  // S tiles consumed
         uint32_t nw = 0;  // PVs this thread has seen complete (in order)
+        uint32_t xg = 0;  // exchanges with the other half
         // wait until PV(0 .. upto-1) of this stream have completed
         auto wait_pv = [&](uint32_t upto) -> bool {
             for (; nw < upto; ++nw)
@@ -422,6 +427,25 @@ __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
                     return false;
             tc_fence_after();
             return true;
+        };
+        // exchange a value with the thread of the other half that holds the
+        // same row (slot xg % 2 of the shared array, a 64-arrival barrier of
+        // the warp pair; the slot is rewritten two exchanges later, after
+        // the partner has passed the next exchange, i.e. read this one).
+        // The fences order this thread's TMEM loads before the partner's
+        // stores past the barrier (the partner's P overwrites scores).
+        auto exchange = [&](float mine, float& other) -> bool {
+            const int slot = xg & 1;
+            float* x = xm + slot * C::SPLIT * BM;
+            x[half * BM + row] = mine;
+            tc_fence_before();
+            mbar_arrive(&xbar[quarter * 2 + slot]);
+            const bool got =
+                __all_sync(0xffffffffu, mbar_wait(&xbar[quarter * 2 + slot], (xg >> 1) & 1));
+            tc_fence_after();
+            other = x[(half ^ 1) * BM + row];
+            ++xg;
+            return got;
         };
         bool ok = true;
         AttnWork nxt = attn_fetch(items, cu, H, w0, n_work);
@@ -434,7 +458,7 @@ __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
             }
             const int start = a.start, L = a.L, qt = a.qt, h = a.h;
             const int n_kt = (L + BN - 1) / BN;
-            float m = 0.f, l = 0.f;
+            float m = 0.f, l = 0.f;  // running max (shared by the halves); this half's row sum
             for (int kt = 0; kt < n_kt; ++kt) {
                 // waits are made warp-uniform: TMEM loads are warp-collective
                 if (!(ok = __all_sync(0xffffffffu, mbar_wait(&s_full[gs & 1], (gs >> 1) & 1))))
@@ -442,35 +466,50 @@ __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
                 tc_fence_after();
                 const uint32_t tS = tbase + lane_base + (gs & 1) * BN;
                 const uint32_t g = gs++;  // stream-wide index of this tile
-                const int kvalid = L - kt * BN;  // keys of this tile inside the sample
-                uint32_t pk[BN / 2];
-                float alpha, rs;
-                if (kvalid >= BN)
-                    attn_ws_softmax<BN, true>(tS, kvalid, scale_log2, kt == 0, m, alpha, rs, pk);
+                const int kvalid = L - kt * BN - half * C::HCOLS;  // of this half's keys
+                const bool full = L - kt * BN >= BN;
+                uint32_t v[32];
+                tmem_ld32(tS + half * C::HCOLS, v);
+                tmem_ld_wait();
+                float mine = full ? attn_half_max<true>(v, kvalid) : attn_half_max<false>(v, kvalid);
+                float theirs;
+                if (!(ok = exchange(mine, theirs))) break;
+                const float mx = fmaxf(mine, theirs) * scale_log2;
+                float alpha = 1.f;
+                if (kt == 0) {
+                    m = mx;
+                } else if (mx > m + attn_ws::kLazy) {
+                    alpha = ex2_approx(m - mx);
+                    m = mx;
+                }
+                uint32_t pk[16];
+                float rs;
+                if (full)
+                    attn_half_exp<true>(v, kvalid, scale_log2, m, rs, pk);
                 else
-                    attn_ws_softmax<BN, false>(tS, kvalid, scale_log2, kt == 0, m, alpha, rs, pk);
+                    attn_half_exp<false>(v, kvalid, scale_log2, m, rs, pk);
                 if (kt > 0 && __any_sync(0xffffffffu, alpha < 1.f)) {
-                    // rescaling O needs every earlier PV of the item done
+                    // rescaling O needs every earlier PV of the item done;
+                    // each half rescales its half of O's columns
                     if (!(ok = wait_pv(g))) break;
-                    {
 #pragma unroll 1
-                        for (int c = 0; c < HD / 32; ++c) {
-                            uint32_t v[32];
-                            tmem_ld32(tO + c * 32, v);
-                            tmem_ld_wait();
+                    for (int c = 0; c < HD / 2 / 16; ++c) {
+                        uint32_t o16[16];
+                        tmem_ld16(tO + c * 16, o16);
+                        tmem_ld_wait();
 #pragma unroll
-                            for (int e = 0; e < 32; ++e)
-                                v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
-                            tmem_st32(tO + c * 32, v);
-                        }
-                        tmem_st_wait();
+                        for (int e = 0; e < 16; ++e)
+                            o16[e] = __float_as_uint(__uint_as_float(o16[e]) * alpha);
+                        tmem_st16(tO + c * 16, o16);
                     }
+                    tmem_st_wait();
                 }
                 l = l * alpha + rs;
                 // keeps o_done[b] within one phase of this thread's waits
                 if (g >= 2 && !(ok = wait_pv(g - 1))) break;
-                static_assert(BN / 2 == 32, "P of one row is one 32-column TMEM store");
-                tmem_st32(tS, pk);
+                // P of this half's 32 keys: 16 columns of bf16 pairs, over
+                // the score buffer's first 32 columns (keys in order)
+                tmem_st16(tS + half * (C::HCOLS / 2), pk);
                 tmem_st_wait();
                 tc_fence_before();
                 mbar_arrive(&p_full[g & 1]);
@@ -479,34 +518,36 @@ __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
             // the next item's loads overlap this epilogue (fetched here, not
             // at the top, so they hold no registers during the key loop)
             nxt = attn_fetch(items, cu, H, w + dw, n_work);
-            // epilogue: O / l -> bf16 once the item's last PV is done
+            // epilogue: O / l -> bf16 once the item's last PV is done; the
+            // row sum is the two halves' sums, added in half order
             if (!(ok = wait_pv(gs))) break;
-            const float inv = 1.0f / l;
-            if (lse != nullptr && qt * BM + quarter * 32 + lane < L)
-                lse[(size_t)(start + qt * BM + quarter * 32 + lane) * H + h] = m + log2f(l);
-            // 32 columns at a time through this warp's staging slot, so each
-            // store instruction writes 8 rows x 64 contiguous bytes; O is
+            float lo;
+            if (!(ok = exchange(l, lo))) break;
+            const float ltot = half == 0 ? l + lo : lo + l;
+            const float inv = 1.0f / ltot;
+            if (half == 0 && lse != nullptr && qt * BM + row < L)
+                lse[(size_t)(start + qt * BM + row) * H + h] = m + log2f(ltot);
+            // 16 columns at a time through this warp's staging slot; O is
             // released (o_free) once its last columns are in registers
-            uint8_t* stg = sm + C::OFF_STG + (warp - 4) * 2048;
+            uint8_t* stg = sm + C::OFF_STG + (warp - 4) * 1024;
             const int row0 = qt * BM + quarter * 32;  // first row of this warp
-            // the TMEM load of chunk c + 1 is in flight while chunk c is
-            // converted and stored
-            uint32_t ov[2][32];
-            tmem_ld32(tO, ov[0]);
+            constexpr int NCK = HD / 2 / 16;            // 16-column chunks of this half
+            uint32_t ov[2][16];
+            tmem_ld16(tO, ov[0]);
 #pragma unroll
-            for (int c = 0; c < HD / 32; ++c) {
-                uint32_t(&v)[32] = ov[c & 1];
-                tmem_ld_wait_regs(v);
-                if (c + 1 < HD / 32) {
-                    tmem_ld32(tO + (c + 1) * 32, ov[(c + 1) & 1]);
+            for (int c = 0; c < NCK; ++c) {
+                uint32_t(&v)[16] = ov[c & 1];
+                tmem_ld_wait_regs16(v);
+                if (c + 1 < NCK) {
+                    tmem_ld16(tO + (c + 1) * 16, ov[(c + 1) & 1]);
                 } else {
                     tc_fence_before();
                     mbar_arrive(o_free);
                 }
-                uint4 q4[4];
+                uint4 q2[2];
 #pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    q4[u] = make_uint4(pack_bf2(__uint_as_float(v[8 * u]) * inv,
+                for (int u = 0; u < 2; ++u)
+                    q2[u] = make_uint4(pack_bf2(__uint_as_float(v[8 * u]) * inv,
                                                 __uint_as_float(v[8 * u + 1]) * inv),
                                        pack_bf2(__uint_as_float(v[8 * u + 2]) * inv,
                                                 __uint_as_float(v[8 * u + 3]) * inv),
@@ -514,15 +555,15 @@ __global__ void __launch_bounds__(HD == 256 ? 256 : 384, 1)
                                                 __uint_as_float(v[8 * u + 5]) * inv),
                                        pack_bf2(__uint_as_float(v[8 * u + 6]) * inv,
                                                 __uint_as_float(v[8 * u + 7]) * inv));
-                attn_stg_put(stg, lane, q4);
+                attn_stg_put(stg, lane, q2);
                 __syncwarp();
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int rr = 8 * i + (lane >> 2);
+                for (int i = 0; i < 2; ++i) {
+                    const int rr = 16 * i + (lane >> 1);
                     const uint4 w4 = attn_stg_get(stg, lane, i);
                     if (row0 + rr < L)
                         *reinterpret_cast<uint4*>(out + (size_t)(start + row0 + rr) * ldo + h * HD +
-                                                  c * 32 + (lane & 3) * 8) = w4;
+                                                  half * (HD / 2) + c * 16 + (lane & 1) * 8) = w4;
                 }
                 __syncwarp();
             }
