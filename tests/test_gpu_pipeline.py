@@ -111,7 +111,7 @@ def test_llama7b_shapes_one_block_whole_tenants():
     plan, step, preds = s.run()
     counts = {t: sum(len(r.samples) for r in w.requests if r.tenant == t) for t in range(32)}
     pick = sorted(counts, key=lambda t: (counts[t], t))[:2]
-    _compare(s, plan, step, preds, pick)
+    _compare(s, plan, step, preds, pick, name="llama7b 1 block")
 
 
 @pytest.mark.parametrize("name", ["small", "llama7b"])

@@ -91,3 +91,24 @@ def test_reference_arm_prints_the_contract_line():
     e = d["e2e"]
     assert e["value"] == d["value"] and e["unit"] == d["unit"]
     assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
+
+
+def test_oracle_timing_subset_is_whole_tenants_largest_and_smallest():
+    """The CPU baseline times whole tenants: every tenant of the one- and
+    six-block workloads; otherwise the two with the most tokens and the two
+    with the fewest."""
+    import synth
+    assert bench.oracle_tenant_subset(synth.make_workload("tiny")) == [0, 1]
+    assert bench.oracle_tenant_subset(synth.make_workload("small")) == list(range(8))
+    for name in ("mqa2b", "zipf2b", "llama7b"):
+        w = synth.make_workload(name)
+        v = w.backbone.vision_tokens
+        tok = {t: sum(s.length(v) for r in w.requests if r.tenant == t for s in r.samples)
+               for t in range(len(w.tenants))}
+        sub = bench.oracle_tenant_subset(w)
+        assert len(sub) == 4
+        rest = [t for t in tok if t not in sub]
+        lo = sorted(sub, key=lambda t: (tok[t], t))[:2]
+        hi = sorted(sub, key=lambda t: (tok[t], t))[2:]
+        assert all(tok[t] >= max(tok[x] for x in lo) for t in rest)
+        assert all(tok[t] <= min(tok[x] for x in hi) for t in rest)
