@@ -144,16 +144,20 @@ __global__ void __launch_bounds__(256, 2) k_head_lin(const __grid_constant__ Hea
     for (int c = 0; c < kLinW; ++c)
 #pragma unroll
         for (int i = 0; i < kLinS; ++i) acc[c][i] = 0.f;
-    // the samples' input rows of one K chunk into staging buffer b
+    // the samples' input rows of one K chunk into staging buffer b, by
+    // cp.async (zero-filled past the slot's samples or past K), so the copy
+    // of the next chunk is in flight while this one is computed
     auto stage = [&](int b, int k0) {
         const int nk = min(kLinK, K - k0);
         for (int i = threadIdx.x; i < kLinS * (kLinK / 4); i += 256) {
             const int r = i / (kLinK / 4), u = i % (kLinK / 4);
-            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (r < ns && 4 * u < nk)
-                v = *reinterpret_cast<const float4*>(in + (size_t)(s0 + r) * ld_in + k0 + 4 * u);
-            *reinterpret_cast<float4*>(&sx[b][r][4 * u]) = v;
+            const bool ok = r < ns && 4 * u < nk;
+            cp_async16(smem_u32(&sx[b][r][4 * u]),
+                       ok ? (const void*)(in + (size_t)(s0 + r) * ld_in + k0 + 4 * u)
+                          : (const void*)in,
+                       ok);
         }
+        cp_async_commit();
     };
     // this lane's 16-byte weight chunks of a K chunk (zero past K or J)
     auto load_w = [&](int k0, uint4 (&wv)[kLinW]) {
@@ -170,6 +174,7 @@ __global__ void __launch_bounds__(256, 2) k_head_lin(const __grid_constant__ Hea
     uint4 wv[kLinW];
     load_w(0, wv);
     stage(0, 0);
+    cp_async_wait<0>();
     __syncthreads();
     const int nch = (K + kLinK - 1) / kLinK;
     for (int kc = 0; kc < nch; ++kc) {
@@ -201,6 +206,9 @@ __global__ void __launch_bounds__(256, 2) k_head_lin(const __grid_constant__ Hea
                 }
             }
         }
+        // the next chunk's inputs have landed (this thread's copies), and
+        // every warp is done with this buffer before it is refilled
+        cp_async_wait<0>();
         __syncthreads();
         if (kc + 1 < nch) {
 #pragma unroll
