@@ -32,7 +32,13 @@ namespace jnx {
 //                 buffers, O += P(kt) V(kt) into the TMEM accumulator; S runs
 //                 two tiles ahead of PV, so the tensor core computes the next
 //                 scores while the softmax warps work on the current ones
-//   warps 4+4t..  online softmax and epilogue, one query row per thread
+//   warps 4 + 8t + 4h + q (h = 0, 1; q = 0..3)
+//                 online softmax and epilogue: two warpgroups, each thread
+//                 holding one query row (lane 32 q + lane) and half of each
+//                 64-key score tile (columns 32 h .. 32 h + 31); the two
+//                 threads of a row exchange their half-row max every tile and
+//                 their partial row sums in the epilogue, and each normalises
+//                 and stores half of O's columns
 // and TMEM columns from 256 t: S buffers at +0 and +BN, O (HD columns) at
 // +2 BN.  P (bf16, two per 32-bit column) overwrites the first BN / 2
 // columns of the score buffer it was computed from and is the TMEM A
@@ -41,7 +47,9 @@ namespace jnx {
 // of tile kt does not wait for PV(kt-1) (only a rare rescale of O does).
 // The two streams share nothing but the tensor core, so one stream's
 // softmax overlaps the other's MMAs and copies, and a short tail tile costs
-// only its own stream.
+// only its own stream.  P of half 1 (keys 32..63) lands in score columns
+// 16..31, which hold half 0's scores: it is written only after the row's
+// exchange, which half 0 reaches after its scores are in registers.
 //
 // The running max is lazy: a row raises the max m it subtracts only when a
 // new tile's max exceeds it by more than 8 (log2 units), so O is rarely
@@ -53,13 +61,20 @@ namespace jnx {
 //   v_full[2], v_empty[2]    V ring (a slot frees when its PV MMA completes)
 //   s_full[2]                score buffer b holds a new S
 //   p_full[2]                P of a tile written over its S in score
-//                            buffer b (128 arrivals)
+//                            buffer b (256 arrivals: both halves)
 //   o_done[2]                PV of a tile with score buffer b completed; a
 //                            softmax thread waits for PV(g-2) before it
 //                            arrives for tile g, so neither barrier runs two
 //                            phases ahead of a waiter
-//   o_free                   the epilogue has read O (128 arrivals)
+//   o_free                   the epilogue has read O (256 arrivals)
 //   drain                    all MMAs of the stream completed (teardown)
+//   xbar[4][2]               exchange between the two threads of each row:
+//                            per lane quarter q and slot (exchange count % 2),
+//                            64 arrivals (the warp pair); the exchanged
+//                            values live in a [slot][half][row] array, a slot
+//                            reused two exchanges later, after the partner
+//                            has passed the next exchange (every wait, as
+//                            all of them, bounded)
 // ---------------------------------------------------------------------------
 namespace attn_ws {
 constexpr int BM = 128;        // query rows per item
