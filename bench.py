@@ -275,9 +275,9 @@ def head_bytes(w, plan):
 
 def kernel_breakdown(J, kinds, ms, work, bytes_per_launch=None):
     """Per traced kernel kind: launches, total ms, share of the traced time
-    and its rate: TFLOP/s for tensor-core kinds, GFLOP/s for the CUDA-core
-    head kinds (plus GB/s from bytes_per_launch[kind] where given), GB/s of
-    the traced bytes otherwise."""
+    and its rate: TFLOP/s for the tcgen05 kinds, GFLOP/s for the head kinds
+    (plus GB/s from bytes_per_launch[kind] where given), GB/s of the traced
+    bytes otherwise."""
     per_kernel = {}
     tot_ms = float(ms.sum())
     for k in sorted(set(kinds.tolist())):

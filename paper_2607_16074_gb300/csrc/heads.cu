@@ -109,17 +109,31 @@ __device__ __forceinline__ void opt_step2(const HeadOpt& o, int k, size_t i, flo
 
 // ---------------------------------------------------------------------------
 // Segmented linear layer: out[s, j] = sum_k in[s, k] W[j, k] + b[j] over the
-// slot's samples.  One CTA per (slot, 32 output columns, 8 samples): warp w
-// takes columns j0 + 4w .. j0 + 4w + 3, its lanes stride K in 8-element
-// (16-byte) weight chunks and keep 4 columns x 8 samples of partial sums;
-// the samples' input rows are staged 256 columns at a time in shared memory
-// (read once per CTA instead of once per column); each sum is closed by a
-// fixed butterfly over the lanes.
+// slot's samples, on the bf16 tensor cores (mma.sync m16n8k16, fp32
+// accumulation).  One CTA per (8 samples, 32 output columns, slot); the
+// sample block varies fastest in the grid, so the CTAs that read one weight
+// tile run together and share it through L2.  K is streamed in 256-column
+// chunks through a ring of kLinStages shared-memory slots (the block's 32
+// weight rows and its samples' input rows, by cp.async, kLinStages - 1
+// chunks ahead of the arithmetic).  W is bf16 already; the fp32 inputs enter
+// as two bf16 operands, hi = bf16(x) and lo = bf16(x - hi), so W x = W hi +
+// W lo to about 2^-17 of x.  Warp w takes the chunk's columns 32 w .. + 31
+// (two 16-deep steps) for all 32 output columns (two 16-row tiles) and the 8
+// samples; the 8 warps' partial sums are added in warp order at the end, so
+// the result does not depend on the group around the slot.
 //   LAYER 1: MLP first layer (W1, b1; in = pooled); stores z and h = SiLU(z).
 //   LAYER 2: output layer of either head (W2 or Wout; in = h); stores y and
 //            scatters it to the caller's predictions at each target offset.
 // ---------------------------------------------------------------------------
-constexpr int kLinCols = 32, kLinS = 8, kLinK = 256, kLinW = kLinCols / 8;  // columns per warp
+constexpr int kLinCols = 32, kLinS = 8, kLinK = 256;
+constexpr int kLinStages = 4;
+constexpr int kLinWPad = kLinK + 8;  // weight row stride (bf16): conflict-free ldmatrix
+constexpr int kLinXPad = kLinK + 8;  // input row stride (fp32): conflict-free 8-byte loads
+constexpr int kLinWBytes = kLinCols * kLinWPad * 2;
+constexpr int kLinXBytes = kLinS * kLinXPad * 4;
+constexpr int kLinSmem = kLinStages * (kLinWBytes + kLinXBytes);
+constexpr int kLinRedPad = kLinCols + 4;  // [warp][sample][column] partial sums
+static_assert(8 * kLinS * kLinRedPad * 4 <= kLinSmem, "partial sums reuse the ring");
 
 template <int LAYER>
 __global__ void __launch_bounds__(256, 2) k_head_lin(const __grid_constant__ HeadTable tab,
@@ -127,113 +141,111 @@ __global__ void __launch_bounds__(256, 2) k_head_lin(const __grid_constant__ Hea
                                                   float* __restrict__ z_out, float* __restrict__ h_out,
                                                   int ld_out, const int* __restrict__ sample_target,
                                                   float* __restrict__ preds) {
-    __shared__ __align__(16) float sx[2][kLinS][kLinK];
-    const HeadSlot& hs = tab.slot[blockIdx.x];
+    extern __shared__ __align__(16) uint8_t lin_smem[];
+    const HeadSlot& hs = tab.slot[blockIdx.z];
     if (LAYER == 1 && hs.kind != JNX_HEAD_MLP) return;
     const int J = LAYER == 1 ? hs.hid : hs.width;
     const int K = LAYER == 1 ? hs.d_in : hs.hid;
     const uint16_t* W = LAYER == 1 ? hs.w1 : hs.w2;
     const uint16_t* B = LAYER == 1 ? hs.b1 : hs.b2;
-    const int j0 = blockIdx.y * kLinCols, s0 = hs.s0 + blockIdx.z * kLinS;
+    const int j0 = blockIdx.y * kLinCols, s0 = hs.s0 + blockIdx.x * kLinS;
     if (j0 >= J || s0 >= hs.s1) return;
     const int ns = min(kLinS, hs.s1 - s0);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int jw = j0 + kLinW * warp;
-    float acc[kLinW][kLinS];
-#pragma unroll
-    for (int c = 0; c < kLinW; ++c)
-#pragma unroll
-        for (int i = 0; i < kLinS; ++i) acc[c][i] = 0.f;
-    // the samples' input rows of one K chunk into staging buffer b, by
-    // cp.async (zero-filled past the slot's samples or past K), so the copy
-    // of the next chunk is in flight while this one is computed
-    auto stage = [&](int b, int k0) {
-        const int nk = min(kLinK, K - k0);
-        for (int i = threadIdx.x; i < kLinS * (kLinK / 4); i += 256) {
-            const int r = i / (kLinK / 4), u = i % (kLinK / 4);
-            const bool ok = r < ns && 4 * u < nk;
-            cp_async16(smem_u32(&sx[b][r][4 * u]),
-                       ok ? (const void*)(in + (size_t)(s0 + r) * ld_in + k0 + 4 * u)
-                          : (const void*)in,
-                       ok);
+    auto sw = [&](int b) { return reinterpret_cast<uint16_t*>(lin_smem + b * kLinWBytes); };
+    auto sx = [&](int b) {
+        return reinterpret_cast<float*>(lin_smem + kLinStages * kLinWBytes + b * kLinXBytes);
+    };
+    const int nch = (K + kLinK - 1) / kLinK;
+    // chunk kc into ring slot kc % kLinStages, zero-filled past J, K or the
+    // slot's samples; one commit group per chunk (empty past the last one)
+    auto stage = [&](int kc) {
+        if (kc < nch) {
+            const int b = kc % kLinStages, k0 = kc * kLinK, nk = min(kLinK, K - k0);
+            uint16_t* w = sw(b);
+            for (int i = threadIdx.x; i < kLinCols * (kLinK / 8); i += 256) {
+                const int c = i / (kLinK / 8), u = i % (kLinK / 8);
+                const bool ok = j0 + c < J && 8 * u < nk;
+                cp_async16(smem_u32(w + c * kLinWPad + 8 * u),
+                           ok ? (const void*)(W + (size_t)(j0 + c) * K + k0 + 8 * u)
+                              : (const void*)W,
+                           ok);
+            }
+            float* x = sx(b);
+            for (int i = threadIdx.x; i < kLinS * (kLinK / 4); i += 256) {
+                const int r = i / (kLinK / 4), u = i % (kLinK / 4);
+                const bool ok = r < ns && 4 * u < nk;
+                cp_async16(smem_u32(x + r * kLinXPad + 4 * u),
+                           ok ? (const void*)(in + (size_t)(s0 + r) * ld_in + k0 + 4 * u)
+                              : (const void*)in,
+                           ok);
+            }
         }
         cp_async_commit();
     };
-    // this lane's 16-byte weight chunks of a K chunk (zero past K or J)
-    auto load_w = [&](int k0, uint4 (&wv)[kLinW]) {
-        const bool in_k = 8 * lane < K - k0;
+    // acc[row tile m][e]: output column j0 + 16 m + lane / 4 (+ 8 for e >= 2),
+    // sample 2 (lane % 4) (+ 1 for odd e)
+    float acc[2][4];
 #pragma unroll
-        for (int c = 0; c < kLinW; ++c)
-            wv[c] = (in_k && jw + c < J)
-                        ? __ldg(reinterpret_cast<const uint4*>(W + (size_t)(jw + c) * K + k0) + lane)
-                        : make_uint4(0, 0, 0, 0);
-    };
-    // the weights stream through registers one chunk ahead and the inputs
-    // through two staging buffers, so each chunk's loads are in flight
-    // during the previous chunk's arithmetic and one barrier closes a chunk
-    uint4 wv[kLinW];
-    load_w(0, wv);
-    stage(0, 0);
-    cp_async_wait<0>();
-    __syncthreads();
-    const int nch = (K + kLinK - 1) / kLinK;
+    for (int m = 0; m < 2; ++m)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) acc[m][e] = 0.f;
+    const int g = lane >> 2, q = lane & 3;
+#pragma unroll
+    for (int kc = 0; kc < kLinStages - 1; ++kc) stage(kc);
     for (int kc = 0; kc < nch; ++kc) {
-        const int b = kc & 1, k0 = kc * kLinK;
-        uint4 wn[kLinW];
-        if (kc + 1 < nch) {
-            load_w(k0 + kLinK, wn);
-            stage(b ^ 1, k0 + kLinK);
-        }
-        if (8 * lane < K - k0) {
-            float x[kLinS][8];
-#pragma unroll
-            for (int i = 0; i < kLinS; ++i) {
-                const float4 a = *reinterpret_cast<const float4*>(&sx[b][i][8 * lane]);
-                const float4 c4 = *reinterpret_cast<const float4*>(&sx[b][i][8 * lane + 4]);
-                x[i][0] = a.x; x[i][1] = a.y; x[i][2] = a.z; x[i][3] = a.w;
-                x[i][4] = c4.x; x[i][5] = c4.y; x[i][6] = c4.z; x[i][7] = c4.w;
-            }
-#pragma unroll
-            for (int c = 0; c < kLinW; ++c) {
-                float wf[8];
-                bf8_to_f(wv[c], wf);
-#pragma unroll
-                for (int i = 0; i < kLinS; ++i) {
-                    float t = acc[c][i];
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) t = fmaf(x[i][e], wf[e], t);
-                    acc[c][i] = t;
-                }
-            }
-        }
-        // the next chunk's inputs have landed (this thread's copies), and
-        // every warp is done with this buffer before it is refilled
-        cp_async_wait<0>();
+        // chunk kc landed (kLinStages - 1 groups were committed after it), and
+        // every warp is done with chunk kc - 1, whose slot is refilled next
+        cp_async_wait<kLinStages - 2>();
         __syncthreads();
-        if (kc + 1 < nch) {
+        stage(kc + kLinStages - 1);
+        const int b = kc % kLinStages;
+        const uint16_t* ws = sw(b);
+        const float* xs = sx(b);
 #pragma unroll
-            for (int c = 0; c < kLinW; ++c) wv[c] = wn[c];
+        for (int st = 0; st < 2; ++st) {
+            const int kb = 32 * warp + 16 * st;
+            // B (16 deep x 8 samples): sample g, depths 2q, 2q + 1 and 2q + 8, 2q + 9
+            const float2 x0 = *reinterpret_cast<const float2*>(xs + g * kLinXPad + kb + 2 * q);
+            const float2 x1 = *reinterpret_cast<const float2*>(xs + g * kLinXPad + kb + 2 * q + 8);
+            const uint32_t h0 = pack_bf2(x0.x, x0.y), h1 = pack_bf2(x1.x, x1.y);
+            const uint32_t l0 = pack_bf2(x0.x - bf2f((uint16_t)(h0 & 0xffff)),
+                                         x0.y - bf2f((uint16_t)(h0 >> 16)));
+            const uint32_t l1 = pack_bf2(x1.x - bf2f((uint16_t)(h1 & 0xffff)),
+                                         x1.y - bf2f((uint16_t)(h1 >> 16)));
+#pragma unroll
+            for (int m = 0; m < 2; ++m) {
+                uint32_t a[4];
+                const int r = 16 * m + (lane & 7) + ((lane >> 3) & 1) * 8;
+                ldsm_x4(smem_u32(ws + r * kLinWPad + kb + (lane >> 4) * 8), a[0], a[1], a[2], a[3]);
+                mma_bf16(acc[m], a[0], a[1], a[2], a[3], h0, h1);
+                mma_bf16(acc[m], a[0], a[1], a[2], a[3], l0, l1);
+            }
         }
     }
+    cp_async_wait<0>();
+    __syncthreads();  // the ring is free: it takes the warps' partial sums
+    float* red = reinterpret_cast<float*>(lin_smem);
 #pragma unroll
-    for (int c = 0; c < kLinW; ++c)
+    for (int m = 0; m < 2; ++m)
 #pragma unroll
-        for (int i = 0; i < kLinS; ++i) acc[c][i] = warp_sum_h(acc[c][i]);
+        for (int e = 0; e < 4; ++e)
+            red[(warp * kLinS + 2 * q + (e & 1)) * kLinRedPad + 16 * m + g + 8 * (e >> 1)] =
+                acc[m][e];
+    __syncthreads();
+    const int i = threadIdx.x >> 5, j = j0 + lane;  // sample s0 + i, column j
+    if (i < ns && j < J) {
+        float sum = 0.f;
 #pragma unroll
-    for (int c = 0; c < kLinW; ++c)
-#pragma unroll
-        for (int i = 0; i < kLinS; ++i) {
-            const int j = jw + c;
-            if (lane == ((c * kLinS + i) & 31) && i < ns && j < J) {
-                const int s = s0 + i;
-                const float zz = acc[c][i] + bf2f(B[j]);
-                z_out[(size_t)s * ld_out + j] = zz;
-                if (LAYER == 1)
-                    h_out[(size_t)s * ld_out + j] = silu_f(zz);
-                else
-                    preds[sample_target[s] + j] = zz;
-            }
-        }
+        for (int w = 0; w < 8; ++w) sum += red[(w * kLinS + i) * kLinRedPad + lane];
+        const int s = s0 + i;
+        const float zz = sum + bf2f(B[j]);
+        z_out[(size_t)s * ld_out + j] = zz;
+        if (LAYER == 1)
+            h_out[(size_t)s * ld_out + j] = silu_f(zz);
+        else
+            preds[sample_target[s] + j] = zz;
+    }
 }
 
 // Per-tenant loss and dy, one CTA per group slot, fixed-order reduction.
@@ -993,8 +1005,9 @@ jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const 
                                 float* loss, cudaStream_t s) {
     if (b.n == 0) return JNX_OK;
     if (b.any_mlp)
-        k_head_lin<1><<<dim3(b.n, (b.max_mlp_hid + kLinCols - 1) / kLinCols,
-                             (b.max_ns + kLinS - 1) / kLinS), 256, 0, s>>>(
+        k_head_lin<1><<<dim3((b.max_ns + kLinS - 1) / kLinS,
+                             (b.max_mlp_hid + kLinCols - 1) / kLinCols, b.n),
+                        256, kLinSmem, s>>>(
             tab, pooled, d, ws.z, ws.h, ws.ld_h, sample_target, preds);
     if (b.any_xattn) {
         const size_t smem = xattn_smem_bytes(b.max_dq);
@@ -1002,8 +1015,9 @@ jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const 
                                                              b.sample0, ws.kbuf, ws.vbuf, ws.ldkv,
                                                              ws.P, ws.h, ws.ld_h);
     }
-    k_head_lin<2><<<dim3(b.n, (b.max_width + kLinCols - 1) / kLinCols,
-                         (b.max_ns + kLinS - 1) / kLinS), 256, 0, s>>>(
+    k_head_lin<2><<<dim3((b.max_ns + kLinS - 1) / kLinS,
+                         (b.max_width + kLinCols - 1) / kLinCols, b.n),
+                    256, kLinSmem, s>>>(
         tab, ws.h, ws.ld_h, ws.y, nullptr, ws.ld_y, sample_target, preds);
     if (targets)  // without targets (inference) there is no loss
         k_l2_loss<<<b.n, 256, 0, s>>>(tab, ws.y, ws.ld_y, targets, sample_target, ws.dy, loss);
@@ -1078,10 +1092,14 @@ jnx_status heads_backward_step_launch(const HeadTable& tab, const HeadOptTable& 
 }
 
 jnx_status heads_set_smem() {
-    static std::atomic<uint64_t> fwd{0}, bwd{0};
+    static std::atomic<uint64_t> fwd{0}, bwd{0}, lin1{0}, lin2{0};
     const int mx = (int)xattn_smem_bytes(512);
     if (set_smem_limit(reinterpret_cast<const void*>(k_xattn_fwd), mx, fwd) != cudaSuccess ||
-        set_smem_limit(reinterpret_cast<const void*>(k_xattn_bwd), mx, bwd) != cudaSuccess)
+        set_smem_limit(reinterpret_cast<const void*>(k_xattn_bwd), mx, bwd) != cudaSuccess ||
+        set_smem_limit(reinterpret_cast<const void*>(k_head_lin<1>), kLinSmem, lin1) !=
+            cudaSuccess ||
+        set_smem_limit(reinterpret_cast<const void*>(k_head_lin<2>), kLinSmem, lin2) !=
+            cudaSuccess)
         return cuda_ok("heads smem attribute");
     return JNX_OK;
 }
