@@ -312,9 +312,9 @@ typedef struct {
     const uint16_t *q, *wk, *wv, *wout, *bout;
 } jnx_head;
 
-/* Per-slot fp32 gradient buffers, same shapes as the parameters.  w1 and
- * w2 / wout (parameters), and the gradients' w2 / wout, wk and wv, must be
- * 16-byte aligned, and the heads of one group share d_in
+/* Per-slot fp32 gradient buffers, same shapes as the parameters.  w1,
+ * w2 / wout and q (parameters), and the gradients' w2 / wout, wk and wv,
+ * must be 16-byte aligned, and the heads of one group share d_in
  * (JNX_ERR_INVALID_ARG / JNX_ERR_UNSUPPORTED otherwise). */
 typedef struct {
     float *w1, *b1, *w2, *b2;

@@ -570,6 +570,9 @@ jnx_status check_heads(const jnx_head* heads, int32_t n_tenants, const jnx_group
             nq = h.n_queries;
             if (!h.q || !h.wk || !h.wv || !h.wout || !h.bout)
                 return fail(JNX_ERR_INVALID_ARG, "heads: tenant %d null parameter", t);
+            if (reinterpret_cast<uintptr_t>(h.q) & 15)
+                return fail(JNX_ERR_INVALID_ARG,
+                            "heads: tenant %d learned queries must be 16-byte aligned", t);
             if (!hidden) return fail(JNX_ERR_INVALID_ARG, "heads: query heads need hidden rows");
             if (h.d_in % 128)
                 return fail(JNX_ERR_UNSUPPORTED, "heads: query heads need d_in %% 128 == 0");
@@ -736,7 +739,7 @@ extern "C" jnx_status jnx_heads_forward(const jnx_head* heads, int32_t n_tenants
 static jnx_status heads_backward(const jnx_head* heads, int32_t n_tenants, const jnx_group* g,
                                  const float* pooled, const uint16_t* hidden,
                                  const jnx_head_grads* grads, void* workspace, size_t ws_bytes,
-                                 void* stream, bool accum) {
+                                 void* stream, bool accum, bool kv_grads = false) {
     jnx_status st;
     if (!grads && g && g->n_slots > 0)
         return fail(JNX_ERR_INVALID_ARG, "heads backward: null grads");
@@ -755,7 +758,7 @@ static jnx_status heads_backward(const jnx_head* heads, int32_t n_tenants, const
         HeadBatch b = fill_table(tab, heads, grads, g, g0, n, accum);
         TraceScope ts(JNX_K_HEADS_BWD, heads_flops(tab, n, true), s);
         if ((st = heads_backward_launch(tab, b, w.sc, pooled, d, hidden, g->cu_seqlens,
-                                        g->sample_slot, s)))
+                                        g->sample_slot, kv_grads, s)))
             return st;
     }
     return JNX_OK;
@@ -854,7 +857,7 @@ extern "C" jnx_status jnx_heads_backward_input(const jnx_head* heads, int32_t n_
     if (!d_hidden && g && g->n_tokens > 0)
         return fail(JNX_ERR_INVALID_ARG, "heads backward: null feature-gradient buffer");
     jnx_status st = heads_backward(heads, n_tenants, g, pooled, hidden, grads, workspace,
-                                   ws_bytes, stream, false);
+                                   ws_bytes, stream, false, true);
     if (st || g->n_slots == 0) return st;
     return heads_feature_grad(heads, g, d_hidden, workspace, static_cast<cudaStream_t>(stream));
 }
@@ -923,7 +926,7 @@ extern "C" jnx_status jnx_heads_backward_adamw(const jnx_head* heads, int32_t n_
             const int n = std::min(kMaxSlots, g->n_slots - g0);
             HeadBatch b = fill_table(tab, heads, grads, g, g0, n, accumulate != 0);
             if ((st = heads_backward_front_launch(tab, b, w.sc, d, hidden, g->cu_seqlens,
-                                                  g->sample_slot, s)))
+                                                  g->sample_slot, d_hidden != nullptr, s)))
                 return st;
         }
     }

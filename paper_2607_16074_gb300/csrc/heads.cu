@@ -19,8 +19,9 @@
 //   (the weight gradients formed through the queries per sample:
 //    dWk = Q^T (sum_s dS_s^T X_s) / sqrt(dq), dWv = sum_s dO_s^T (P_s^T X_s))
 // Loss (both): l_t = sum (y - t)^2 / (n_t * width), dy = 2 (y - t) / (n_t width).
-// All sums run in a fixed order inside one thread or one CTA (no atomics),
-// so a tenant's results are identical whether it runs grouped or alone.
+// All sums run in a fixed order inside one thread, one CTA or one
+// tensor-core instruction sequence (no atomics), so a tenant's results are
+// identical whether it runs grouped or alone.
 #include <type_traits>
 
 #include "jnx_dev.cuh"
@@ -461,77 +462,164 @@ __global__ void __launch_bounds__(256) k_mlp_dw1(const __grid_constant__ HeadTab
 }
 
 constexpr int kMaxQ = 32;
-constexpr int kXRows = 32;  // key rows staged at a time
+constexpr int kXRows = 32;   // key rows staged at a time
+constexpr int kXCols = 256;  // columns per pass of the products over keys
+constexpr int kXPad = 40;    // row stride (bf16) of the [query][key] / [key][query] tiles
 
-// Shared-memory layout of the per-sample query-head kernels (fp32, rows
-// padded by 4 floats so the rows a warp reads together fall in distinct
-// banks): A [kMaxQ][dq + 4] (the queries, or dO), R [kXRows][dq + 4] (a
-// tile of key rows of k or v), then a P chunk and a dS chunk of
-// [kXRows][kMaxQ] each.
-__host__ __device__ constexpr size_t xattn_smem_bytes(int dq) {
-    return ((size_t)(kMaxQ + kXRows) * (dq + 4) + 2 * kXRows * kMaxQ) * sizeof(float);
+// Shared memory of the per-sample query-head kernels: bf16 operand tiles of
+// the bf16 tensor cores (mma.sync m16n8k16, fp32 accumulation), rows padded
+// by 8 elements (16 bytes) so that the eight rows one ldmatrix reads fall in
+// distinct banks.  fp32 operands enter as two bf16 planes, hi = bf16(x) and
+// lo = bf16(x - hi) (x = hi + lo to about 2^-17 of x); a product of two split
+// operands takes hi hi + hi lo + lo hi, of a split and a bf16 one hi + lo.
+//   sQ [kMaxQ][dq + 8]        the learned queries (bf16, rows past nq zero)
+//   sA [2][kMaxQ][dq + 8]     dO, hi and lo (backward)
+//   sR [2][kXRows][dq + 8]    a chunk of key or value rows, hi and lo
+//   sT [2][2][kMaxQ][kXPad]   a chunk of P / dS, query-major, hi and lo
+//   sU [2][2][kXRows][kXPad]  the same chunk key-major (backward)
+__host__ __device__ constexpr size_t xattn_smem_bytes(int dq, bool bwd) {
+    return ((size_t)(bwd ? 3 : 1) * kMaxQ * (dq + 8) + (size_t)2 * kXRows * (dq + 8) +
+            (size_t)(bwd ? 8 : 4) * kMaxQ * kXPad) *
+           2;
 }
 
-// The nq x dq rows of a bf16 (src16) or fp32 (src32) matrix into sA (padded).
-__device__ __forceinline__ void xattn_stage_a(float* sA, const uint16_t* src16, const float* src32,
-                                              int nq, int dq) {
-    const int ld = dq + 4;
-    for (int i = threadIdx.x; i < nq * dq; i += blockDim.x) {
-        const int q = i / dq, c = i % dq;
-        sA[q * ld + c] = src16 ? bf2f(src16[i]) : src32[i];
-    }
+// hi and lo planes of four fp32 values, packed in bf16 pairs.
+__device__ __forceinline__ void split4(const float4 v, uint2& hi, uint2& lo) {
+    hi = make_uint2(pack_bf2(v.x, v.y), pack_bf2(v.z, v.w));
+    lo = make_uint2(pack_bf2(v.x - bf2f((uint16_t)(hi.x & 0xffff)),
+                             v.y - bf2f((uint16_t)(hi.x >> 16))),
+                    pack_bf2(v.z - bf2f((uint16_t)(hi.y & 0xffff)),
+                             v.w - bf2f((uint16_t)(hi.y >> 16))));
 }
 
-// Rows j0 .. j0 + nr - 1 of R (stride ldkv, from row r0) into the padded
-// tile sR by cp.async (rows past nr zero).  Caller commits and waits.
-__device__ __forceinline__ void xattn_stage_rows(float* sR, const float* __restrict__ R, int ldkv,
-                                                 int r0, int j0, int nr, int dq) {
-    const int ld = dq + 4, units = dq / 4;
-    for (int i = threadIdx.x; i < kXRows * units; i += blockDim.x) {
+// Rows [row0, row0 + nr) x columns [c0, c0 + nc) of the fp32 matrix R
+// (stride ld) into the hi plane dst and the lo plane dst + rows * ldt (row
+// stride ldt); rows nr .. rows - 1 are zero.  16-byte loads: R, ld and c0
+// 16-byte aligned.
+__device__ __forceinline__ void xattn_split_rows(uint16_t* dst, int rows, int ldt,
+                                                 const float* __restrict__ R, int ld, size_t row0,
+                                                 int nr, int c0, int nc) {
+    const int units = nc / 4;
+    for (int i = threadIdx.x; i < rows * units; i += blockDim.x) {
         const int r = i / units, u = i % units;
-        const bool ok = r < nr;
-        cp_async16(smem_u32(sR + r * ld + 4 * u),
-                   ok ? (const void*)(R + (size_t)(r0 + j0 + r) * ldkv + 4 * u) : (const void*)R,
-                   ok);
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (r < nr) v = *reinterpret_cast<const float4*>(R + (row0 + r) * ld + c0 + 4 * u);
+        uint2 hi, lo;
+        split4(v, hi, lo);
+        *reinterpret_cast<uint2*>(dst + (size_t)r * ldt + 4 * u) = hi;
+        *reinterpret_cast<uint2*>(dst + (size_t)(rows + r) * ldt + 4 * u) = lo;
     }
 }
 
-// out[j * nq + q] = scale * (A[q, :] . R[r0 + j, :]) for the sample's L key
-// rows, key-major.  Key rows staged kXRows at a time; thread (jj = tid / 8,
-// g = tid % 8) takes row jj and queries g, g + 8, g + 16, g + 24 (strided so
-// the eight query rows a warp reads at once sit in distinct banks).  Ends
-// with a barrier.
-__device__ void xattn_rows_dot(const float* __restrict__ R, int ldkv, int r0, int L,
-                               const float* sA, float* sR, int nq, int dq, float scale,
-                               float* __restrict__ out) {
-    const int ld = dq + 4;
-    const int jj = threadIdx.x >> 3, g = threadIdx.x & 7;
+// Keys [j0, j0 + nr) of the key-major [L][nq] block X (P or dS) into hi / lo
+// planes of a query-major tile tq[plane][q][j] and, if tk, a key-major tile
+// tk[plane][j][q]; entries past nr or nq are zero.
+__device__ __forceinline__ void xattn_split_chunk(uint16_t* tq, uint16_t* tk,
+                                                  const float* __restrict__ X, int j0, int nr,
+                                                  int nq) {
+    for (int i = threadIdx.x; i < kMaxQ * kXRows; i += blockDim.x) {
+        const int q = i & 31, j = i >> 5;  // a key's nq values are contiguous
+        const bool ok = j < nr && q < nq;
+        const float x = ok ? X[(size_t)(j0 + j) * nq + q] : 0.f;
+        const uint16_t hi = f2bf(x), lo = f2bf(x - bf2f(hi));
+        if (tq) {
+            tq[q * kXPad + j] = hi;
+            tq[(kMaxQ + q) * kXPad + j] = lo;
+        }
+        if (tk) {
+            tk[j * kXPad + q] = hi;
+            tk[(kXRows + j) * kXPad + q] = lo;
+        }
+    }
+}
+
+// The learned queries (bf16 [nq][dq], 16-byte aligned) into sQ.
+__device__ __forceinline__ void xattn_stage_q(uint16_t* sQ, int ldr, const uint16_t* __restrict__ q,
+                                              int nq, int dq) {
+    const int units = dq / 8;
+    for (int i = threadIdx.x; i < kMaxQ * units; i += blockDim.x) {
+        const int r = i / units, u = i % units;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (r < nq) v = *reinterpret_cast<const uint4*>(q + (size_t)r * dq + 8 * u);
+        *reinterpret_cast<uint4*>(sQ + (size_t)r * ldr + 8 * u) = v;
+    }
+}
+
+// out[j * nq + q] = scale * sum_c A[q, c] R[r0 + j, c] over the sample's L
+// key rows, key-major: A = (ahi, alo) split, or bf16 ahi alone (alo null).
+// Per 32-key chunk (rows split into sR), warp w takes query tile w % 2 and
+// keys 8 (w / 2) .. + 7, over all dq.  Ends with a barrier.
+__device__ void xattn_scores(const uint16_t* ahi, const uint16_t* alo, int ldr, uint16_t* sR,
+                             const float* __restrict__ R, int ldkv, int r0, int L, int nq, int dq,
+                             float scale, float* __restrict__ out) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m = warp & 1, nt = warp >> 1, g = lane >> 2, t = lane & 3;
+    const int arow = 16 * m + (lane & 7) + ((lane >> 3) & 1) * 8, acol = (lane >> 4) * 8;
+    // B (8 keys x 16 deep): matrices hi / k 0-7, hi / k 8-15, lo / k 0-7, lo / k 8-15
+    const int brow = 8 * nt + (lane & 7), bcol = ((lane >> 3) & 1) * 8;
+    const uint16_t* bsrc = sR + (size_t)(lane >> 4) * kXRows * ldr + (size_t)brow * ldr + bcol;
     for (int j0 = 0; j0 < L; j0 += kXRows) {
         const int nr = min(kXRows, L - j0);
-        __syncthreads();  // the previous tile (or sA's writers) done
-        xattn_stage_rows(sR, R, ldkv, r0, j0, nr, dq);
-        cp_async_commit();
-        cp_async_wait<0>();
+        __syncthreads();  // the previous chunk's readers (or the A tiles' writers) done
+        xattn_split_rows(sR, kXRows, ldr, R, ldkv, (size_t)r0 + j0, nr, 0, dq);
         __syncthreads();
-        if (jj < nr) {
-            float acc[4] = {0.f, 0.f, 0.f, 0.f};
-            const float* rr = sR + jj * ld;
-            for (int c = 0; c < dq; c += 4) {
-                const float4 x = *reinterpret_cast<const float4*>(rr + c);
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    if (g + 8 * i < nq) {
-                        const float4 a = *reinterpret_cast<const float4*>(sA + (g + 8 * i) * ld + c);
-                        acc[i] = fmaf(a.x, x.x, fmaf(a.y, x.y, fmaf(a.z, x.z, fmaf(a.w, x.w, acc[i]))));
-                    }
-                }
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int kc = 0; kc < dq; kc += 16) {
+            uint32_t a[4], b[4];
+            ldsm_x4(smem_u32(ahi + (size_t)arow * ldr + kc + acol), a[0], a[1], a[2], a[3]);
+            ldsm_x4(smem_u32(bsrc + kc), b[0], b[1], b[2], b[3]);
+            mma_bf16(acc, a[0], a[1], a[2], a[3], b[0], b[1]);
+            mma_bf16(acc, a[0], a[1], a[2], a[3], b[2], b[3]);
+            if (alo) {
+                ldsm_x4(smem_u32(alo + (size_t)arow * ldr + kc + acol), a[0], a[1], a[2], a[3]);
+                mma_bf16(acc, a[0], a[1], a[2], a[3], b[0], b[1]);
             }
+        }
+        // element e: query 16 m + g (+ 8 for e >= 2), key 8 nt + 2 t (+ 1 for odd e)
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
-                if (g + 8 * i < nq) out[(size_t)(j0 + jj) * nq + g + 8 * i] = acc[i] * scale;
+        for (int e = 0; e < 4; ++e) {
+            const int q = 16 * m + g + 8 * (e >> 1), key = 8 * nt + 2 * t + (e & 1);
+            if (key < nr && q < nq) out[(size_t)(j0 + key) * nq + q] = acc[e] * scale;
         }
     }
     __syncthreads();
+}
+
+// acc[m][n] += X R over one staged 32-key chunk: X the query-major split
+// tile tq (hi, lo planes), R the key-row split tile sR (row stride
+// kXCols + 8); warp w takes columns 32 w .. + 31 (four 8-column tiles n)
+// of both query tiles m.
+__device__ __forceinline__ void xattn_chunk_xr(float (&acc)[2][4][4], const uint16_t* tq,
+                                               const uint16_t* sR) {
+    constexpr int ldt = kXCols + 8;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int kr = (lane & 7) + ((lane >> 3) & 1) * 8, arow = kr, acol = (lane >> 4) * 8;
+#pragma unroll
+    for (int k0 = 0; k0 < kXRows; k0 += 16) {
+        uint32_t ah[2][4], al[2][4];
+#pragma unroll
+        for (int m = 0; m < 2; ++m) {
+            const uint16_t* a = tq + (size_t)(16 * m + arow) * kXPad + k0 + acol;
+            ldsm_x4(smem_u32(a), ah[m][0], ah[m][1], ah[m][2], ah[m][3]);
+            ldsm_x4(smem_u32(a + kMaxQ * kXPad), al[m][0], al[m][1], al[m][2], al[m][3]);
+        }
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+            const uint16_t* b = sR + (size_t)(k0 + kr) * ldt + 32 * warp + 16 * hf + acol;
+            uint32_t bh[4], bl[4];
+            ldsm_x4_t(smem_u32(b), bh[0], bh[1], bh[2], bh[3]);
+            ldsm_x4_t(smem_u32(b + kXRows * ldt), bl[0], bl[1], bl[2], bl[3]);
+#pragma unroll
+            for (int m = 0; m < 2; ++m)
+#pragma unroll
+                for (int n = 0; n < 2; ++n) {
+                    float(&c)[4] = acc[m][2 * hf + n];
+                    mma_bf16(c, ah[m][0], ah[m][1], ah[m][2], ah[m][3], bh[2 * n], bh[2 * n + 1]);
+                    mma_bf16(c, ah[m][0], ah[m][1], ah[m][2], ah[m][3], bl[2 * n], bl[2 * n + 1]);
+                    mma_bf16(c, al[m][0], al[m][1], al[m][2], al[m][3], bh[2 * n], bh[2 * n + 1]);
+                }
+        }
+    }
 }
 
 // Per-query reductions over the sample's key-major [L, nq] block X (and Y):
@@ -559,7 +647,10 @@ __device__ float xattn_reduce_q(const float* __restrict__ X, const float* __rest
 // ---------------------------------------------------------------------------
 // Query head, per sample.  One CTA per packed sample of a query-head slot.
 // P (normalised attention) for sample s is stored key-major at P + nq * cu[s]:
-// element (query q, key j) at j * nq + q (nq a multiple of 4).
+// element (query q, key j) at j * nq + q (nq a multiple of 4).  The
+// products run on the bf16 tensor cores with split fp32 operands (see
+// xattn_smem_bytes); every sum runs in a fixed order, so a sample's result
+// does not depend on the batch around it.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_xattn_fwd(const __grid_constant__ HeadTable tab, int g0,
                                                    const int* __restrict__ cu,
@@ -568,20 +659,21 @@ __global__ void __launch_bounds__(256) k_xattn_fwd(const __grid_constant__ HeadT
                                                    const float* __restrict__ vbuf, int ldkv,
                                                    float* __restrict__ P, float* __restrict__ h,
                                                    int ld_h) {
-    extern __shared__ __align__(16) float xs[];
+    static_assert(kMaxQ == 32 && kXRows == 32, "two 16-row tiles of queries and of keys");
+    extern __shared__ __align__(16) uint8_t xsm[];
     __shared__ float red[8 * 32];
     const int s = sample0 + blockIdx.x;
     const HeadSlot& hs = tab.slot[sample_slot[s] - g0];
     if (hs.kind != JNX_HEAD_XATTN) return;
-    const int nq = hs.nq, dq = hs.dq, ld = dq + 4;
-    float* sA = xs;
-    float* sR = sA + kMaxQ * ld;
-    float* sP = sR + kXRows * ld;
+    const int nq = hs.nq, dq = hs.dq, ldr = dq + 8;
+    uint16_t* sQ = reinterpret_cast<uint16_t*>(xsm);
+    uint16_t* sR = sQ + kMaxQ * ldr;
+    uint16_t* sT = sR + 2 * kXRows * ldr;
     const int r0 = cu[s], L = cu[s + 1] - r0;
     float* Ps = P + (size_t)nq * r0;
-    xattn_stage_a(sA, hs.q, nullptr, nq, dq);
-    // scores S[j, q] = q_q . k_j / sqrt(dq)
-    xattn_rows_dot(kbuf, ldkv, r0, L, sA, sR, nq, dq, rsqrtf((float)dq), Ps);
+    xattn_stage_q(sQ, ldr, hs.q, nq, dq);
+    // scores S[j, q] = Q_q . k_j / sqrt(dq) into Ps
+    xattn_scores(sQ, nullptr, ldr, sR, kbuf, ldkv, r0, L, nq, dq, rsqrtf((float)dq), Ps);
     // softmax over the keys of each query, in place
     const float m = xattn_reduce_q<true>(Ps, nullptr, L, nq, red);
     {
@@ -602,50 +694,40 @@ __global__ void __launch_bounds__(256) k_xattn_fwd(const __grid_constant__ HeadT
             for (int j = part; j < L; j += 8) Ps[(size_t)j * nq + q] *= inv;
         __syncthreads();
     }
-    // O[q, c] = sum_j P[j, q] v[j, c]: a thread per value column, keys in
-    // order; P and v rows staged kXRows at a time
-    for (int c0 = 0; c0 < dq; c0 += 256) {
-        const int c = c0 + threadIdx.x;
-        float acc[kMaxQ];
-#pragma unroll
-        for (int q = 0; q < kMaxQ; ++q) acc[q] = 0.f;
+    // O = P v, kXCols value columns at a time, keys in 32-key chunks
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+    for (int c0 = 0; c0 < dq; c0 += kXCols) {
+        float acc[2][4][4] = {};
         for (int j0 = 0; j0 < L; j0 += kXRows) {
             const int nr = min(kXRows, L - j0);
             __syncthreads();
-            xattn_stage_rows(sR, vbuf, ldkv, r0, j0, nr, dq);
-            for (int i = threadIdx.x; i < nr * nq / 4; i += 256)
-                cp_async16(smem_u32(sP + 4 * i), Ps + (size_t)j0 * nq + 4 * i, true);
-            cp_async_commit();
-            cp_async_wait<0>();
+            xattn_split_rows(sR, kXRows, kXCols + 8, vbuf, ldkv, (size_t)r0 + j0, nr, c0, kXCols);
+            xattn_split_chunk(sT, nullptr, Ps, j0, nr, nq);
             __syncthreads();
-            if (c < dq)
-                for (int j = 0; j < nr; ++j) {
-                    const float vv = sR[j * ld + c];
-#pragma unroll
-                    for (int q4 = 0; q4 < kMaxQ / 4; ++q4) {
-                        if (4 * q4 < nq) {
-                            const float4 pp = *reinterpret_cast<const float4*>(sP + j * nq + 4 * q4);
-                            acc[4 * q4 + 0] = fmaf(pp.x, vv, acc[4 * q4 + 0]);
-                            acc[4 * q4 + 1] = fmaf(pp.y, vv, acc[4 * q4 + 1]);
-                            acc[4 * q4 + 2] = fmaf(pp.z, vv, acc[4 * q4 + 2]);
-                            acc[4 * q4 + 3] = fmaf(pp.w, vv, acc[4 * q4 + 3]);
-                        }
-                    }
-                }
+            xattn_chunk_xr(acc, sT, sR);
         }
-        if (c < dq) {
+        // element e of tile (m, n): query 16 m + g (+ 8 for e >= 2), column
+        // c0 + 32 w + 8 n + 2 t (+ 1 for odd e)
 #pragma unroll
-            for (int q = 0; q < kMaxQ; ++q)
-                if (q < nq) h[(size_t)s * ld_h + q * dq + c] = acc[q];
-        }
+        for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+            for (int hf = 0; hf < 2; ++hf) {
+                const int q = 16 * mt + g + 8 * hf;
+                if (q >= nq) continue;
+#pragma unroll
+                for (int n = 0; n < 4; ++n)
+                    *reinterpret_cast<float2*>(h + (size_t)s * ld_h + (size_t)q * dq + c0 +
+                                               32 * warp + 8 * n + 2 * t) =
+                        make_float2(acc[mt][n][2 * hf], acc[mt][n][2 * hf + 1]);
+            }
     }
 }
 
 // Backward per sample: dP = dO v^T (into dS), the per-query sums
-// D_q = sum_j dP P, dS = P (dP - D_q) in place, then per value column c
-// with dO[:, c] and Q[:, c] in registers: dv[j, c] = sum_q P dO,
-// dk[j, c] = scale sum_q dS Q, and this sample's dQ contribution
-// scale sum_j dS[j, q] k[j, c] (summed per tenant later in sample order).
+// D_q = sum_j dP P, dS = P (dP - D_q) in place, this sample's dQ
+// contribution scale dS k (summed per tenant later in sample order), and,
+// when kv_grads is set (the feature gradient needs them), the key rows'
+// dv = P^T dO and dk = scale dS^T Q.
 __global__ void __launch_bounds__(256) k_xattn_bwd(const __grid_constant__ HeadTable tab, int g0,
                                                    const int* __restrict__ cu,
                                                    const int* __restrict__ sample_slot,
@@ -655,23 +737,25 @@ __global__ void __launch_bounds__(256) k_xattn_bwd(const __grid_constant__ HeadT
                                                    float* __restrict__ dS,
                                                    const float* __restrict__ dO, int ld_h,
                                                    float* __restrict__ dk, float* __restrict__ dv,
-                                                   float* __restrict__ dQs) {
-    extern __shared__ __align__(16) float xs[];
+                                                   float* __restrict__ dQs, int kv_grads) {
+    extern __shared__ __align__(16) uint8_t xsm[];
     __shared__ float red[8 * 32];
     const int s = sample0 + blockIdx.x;
     const HeadSlot& hs = tab.slot[sample_slot[s] - g0];
     if (hs.kind != JNX_HEAD_XATTN) return;
-    const int nq = hs.nq, dq = hs.dq, ld = dq + 4;
-    float* sA = xs;
-    float* sR = sA + kMaxQ * ld;
-    float* sP = sR + kXRows * ld;
-    float* sD = sP + kXRows * kMaxQ;
+    const int nq = hs.nq, dq = hs.dq, ldr = dq + 8;
+    uint16_t* sQ = reinterpret_cast<uint16_t*>(xsm);
+    uint16_t* sA = sQ + kMaxQ * ldr;
+    uint16_t* sR = sA + 2 * kMaxQ * ldr;
+    uint16_t* sT = sR + 2 * kXRows * ldr;
+    uint16_t* sU = sT + 4 * kMaxQ * kXPad;
     const int r0 = cu[s], L = cu[s + 1] - r0;
     const float scale = rsqrtf((float)dq);
     const float* Ps = P + (size_t)nq * r0;
     float* dSs = dS + (size_t)nq * r0;
-    xattn_stage_a(sA, nullptr, dO + (size_t)s * ld_h, nq, dq);
-    xattn_rows_dot(vbuf, ldkv, r0, L, sA, sR, nq, dq, 1.f, dSs);  // dP
+    xattn_stage_q(sQ, ldr, hs.q, nq, dq);
+    xattn_split_rows(sA, kMaxQ, ldr, dO + (size_t)s * ld_h, dq, 0, nq, 0, dq);
+    xattn_scores(sA, sA + kMaxQ * ldr, ldr, sR, vbuf, ldkv, r0, L, nq, dq, 1.f, dSs);  // dP
     const float Dq = xattn_reduce_q<false>(dSs, Ps, L, nq, red);
     {
         const int q = threadIdx.x & 31, part = threadIdx.x >> 5;
@@ -682,56 +766,89 @@ __global__ void __launch_bounds__(256) k_xattn_bwd(const __grid_constant__ HeadT
             }
         __syncthreads();
     }
-    for (int c0 = 0; c0 < dq; c0 += 256) {
-        const int c = c0 + threadIdx.x;
-        const bool colok = c < dq;
-        float go[kMaxQ], qc[kMaxQ], dqa[kMaxQ];
-#pragma unroll
-        for (int q = 0; q < kMaxQ; ++q) {
-            go[q] = colok && q < nq ? sA[q * ld + c] : 0.f;
-            qc[q] = colok && q < nq ? bf2f(hs.q[(size_t)q * dq + c]) : 0.f;
-            dqa[q] = 0.f;
-        }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+    const int kr = (lane & 7) + ((lane >> 3) & 1) * 8, acol = (lane >> 4) * 8;
+    // sT: dS query-major (hi, lo); sU: P key-major (hi, lo), then dS key-major (hi, lo)
+    uint16_t* uP = sU;
+    uint16_t* uD = sU + 2 * kXRows * kXPad;
+    for (int c0 = 0; c0 < dq; c0 += kXCols) {
+        float aq[2][4][4] = {};
         for (int j0 = 0; j0 < L; j0 += kXRows) {
             const int nr = min(kXRows, L - j0);
             __syncthreads();
-            xattn_stage_rows(sR, kbuf, ldkv, r0, j0, nr, dq);
-            for (int i = threadIdx.x; i < nr * nq / 4; i += 256) {
-                cp_async16(smem_u32(sP + 4 * i), Ps + (size_t)j0 * nq + 4 * i, true);
-                cp_async16(smem_u32(sD + 4 * i), dSs + (size_t)j0 * nq + 4 * i, true);
-            }
-            cp_async_commit();
-            cp_async_wait<0>();
+            xattn_split_rows(sR, kXRows, kXCols + 8, kbuf, ldkv, (size_t)r0 + j0, nr, c0, kXCols);
+            xattn_split_chunk(sT, kv_grads ? uD : nullptr, dSs, j0, nr, nq);
+            if (kv_grads) xattn_split_chunk(nullptr, uP, Ps, j0, nr, nq);
             __syncthreads();
-            if (!colok) continue;
-            for (int j = 0; j < nr; ++j) {
-                const float kk = sR[j * ld + c];
-                float a_v = 0.f, a_k = 0.f;
+            xattn_chunk_xr(aq, sT, sR);  // dQ += dS k
+            if (!kv_grads) continue;
+            // dv[j, c] = sum_q P[q, j] dO[q, c], dk[j, c] = scale sum_q dS[q, j] Q[q, c]:
+            // key tiles m of the chunk, columns c0 + 32 w + 8 n, queries as the depth
+            float av[2][4][4] = {}, ak[2][4][4] = {};
 #pragma unroll
-                for (int q4 = 0; q4 < kMaxQ / 4; ++q4) {
-                    if (4 * q4 < nq) {
-                        const float4 p4 = *reinterpret_cast<const float4*>(sP + j * nq + 4 * q4);
-                        const float4 d4 = *reinterpret_cast<const float4*>(sD + j * nq + 4 * q4);
-                        const float pp[4] = {p4.x, p4.y, p4.z, p4.w};
-                        const float dd[4] = {d4.x, d4.y, d4.z, d4.w};
+            for (int k0 = 0; k0 < kMaxQ; k0 += 16) {
+                uint32_t ph[2][4], pl[2][4], dh[2][4], dl[2][4];
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const int q = 4 * q4 + e;
-                            a_v = fmaf(pp[e], go[q], a_v);
-                            a_k = fmaf(dd[e], qc[q], a_k);
-                            dqa[q] = fmaf(dd[e], kk, dqa[q]);
+                for (int m = 0; m < 2; ++m) {
+                    const size_t o = (size_t)(16 * m + kr) * kXPad + k0 + acol;
+                    ldsm_x4(smem_u32(uP + o), ph[m][0], ph[m][1], ph[m][2], ph[m][3]);
+                    ldsm_x4(smem_u32(uP + kXRows * kXPad + o), pl[m][0], pl[m][1], pl[m][2],
+                            pl[m][3]);
+                    ldsm_x4(smem_u32(uD + o), dh[m][0], dh[m][1], dh[m][2], dh[m][3]);
+                    ldsm_x4(smem_u32(uD + kXRows * kXPad + o), dl[m][0], dl[m][1], dl[m][2],
+                            dl[m][3]);
+                }
+#pragma unroll
+                for (int hf = 0; hf < 2; ++hf) {
+                    const size_t o = (size_t)(k0 + kr) * ldr + c0 + 32 * warp + 16 * hf + acol;
+                    uint32_t oh[4], ol[4], qb[4];
+                    ldsm_x4_t(smem_u32(sA + o), oh[0], oh[1], oh[2], oh[3]);
+                    ldsm_x4_t(smem_u32(sA + (size_t)kMaxQ * ldr + o), ol[0], ol[1], ol[2], ol[3]);
+                    ldsm_x4_t(smem_u32(sQ + o), qb[0], qb[1], qb[2], qb[3]);
+#pragma unroll
+                    for (int m = 0; m < 2; ++m)
+#pragma unroll
+                        for (int n = 0; n < 2; ++n) {
+                            float(&v)[4] = av[m][2 * hf + n];
+                            mma_bf16(v, ph[m][0], ph[m][1], ph[m][2], ph[m][3], oh[2 * n], oh[2 * n + 1]);
+                            mma_bf16(v, ph[m][0], ph[m][1], ph[m][2], ph[m][3], ol[2 * n], ol[2 * n + 1]);
+                            mma_bf16(v, pl[m][0], pl[m][1], pl[m][2], pl[m][3], oh[2 * n], oh[2 * n + 1]);
+                            float(&k)[4] = ak[m][2 * hf + n];
+                            mma_bf16(k, dh[m][0], dh[m][1], dh[m][2], dh[m][3], qb[2 * n], qb[2 * n + 1]);
+                            mma_bf16(k, dl[m][0], dl[m][1], dl[m][2], dl[m][3], qb[2 * n], qb[2 * n + 1]);
                         }
+                }
+            }
+            // element e of tile (m, n): key j0 + 16 m + g (+ 8 for e >= 2),
+            // column c0 + 32 w + 8 n + 2 t (+ 1 for odd e)
+#pragma unroll
+            for (int m = 0; m < 2; ++m)
+#pragma unroll
+                for (int hf = 0; hf < 2; ++hf) {
+                    const int j = 16 * m + g + 8 * hf;
+                    if (j >= nr) continue;
+                    const size_t row = (size_t)(r0 + j0 + j) * ldkv + c0 + 32 * warp + 2 * t;
+#pragma unroll
+                    for (int n = 0; n < 4; ++n) {
+                        *reinterpret_cast<float2*>(dv + row + 8 * n) =
+                            make_float2(av[m][n][2 * hf], av[m][n][2 * hf + 1]);
+                        *reinterpret_cast<float2*>(dk + row + 8 * n) =
+                            make_float2(ak[m][n][2 * hf] * scale, ak[m][n][2 * hf + 1] * scale);
                     }
                 }
-                dv[(size_t)(r0 + j0 + j) * ldkv + c] = a_v;
-                dk[(size_t)(r0 + j0 + j) * ldkv + c] = a_k * scale;
-            }
         }
-        if (colok) {
 #pragma unroll
-            for (int q = 0; q < kMaxQ; ++q)
-                if (q < nq) dQs[(size_t)s * ld_h + q * dq + c] = dqa[q] * scale;
-        }
+        for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+            for (int hf = 0; hf < 2; ++hf) {
+                const int q = 16 * mt + g + 8 * hf;
+                if (q >= nq) continue;
+#pragma unroll
+                for (int n = 0; n < 4; ++n)
+                    *reinterpret_cast<float2*>(dQs + (size_t)s * ld_h + (size_t)q * dq + c0 +
+                                               32 * warp + 8 * n + 2 * t) =
+                        make_float2(aq[mt][n][2 * hf] * scale, aq[mt][n][2 * hf + 1] * scale);
+            }
     }
 }
 
@@ -1010,7 +1127,7 @@ jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const 
                         256, kLinSmem, s>>>(
             tab, pooled, d, ws.z, ws.h, ws.ld_h, sample_target, preds);
     if (b.any_xattn) {
-        const size_t smem = xattn_smem_bytes(b.max_dq);
+        const size_t smem = xattn_smem_bytes(b.max_dq, false);
         k_xattn_fwd<<<b.sample1 - b.sample0, 256, smem, s>>>(tab, b.g0, cu, sample_slot,
                                                              b.sample0, ws.kbuf, ws.vbuf, ws.ldkv,
                                                              ws.P, ws.h, ws.ld_h);
@@ -1026,7 +1143,8 @@ jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const 
 
 jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const HeadScratch& ws,
                                  const float* pooled, int d, const uint16_t* hidden,
-                                 const int* cu, const int* sample_slot, cudaStream_t s) {
+                                 const int* cu, const int* sample_slot, bool kv_grads,
+                                 cudaStream_t s) {
     if (b.n == 0) return JNX_OK;
     const NoOpt no{};
     const AdamHp nh{};
@@ -1039,10 +1157,10 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
         k_mlp_dw1<NoOpt><<<dim3(b.n, b.max_mlp_hid, (d / 4 + 255) / 256), 256, 0, s>>>(
             tab, no, nh, ws.dh, ws.ld_h, pooled, d);
     if (b.any_xattn) {
-        const size_t smem = xattn_smem_bytes(b.max_dq);
+        const size_t smem = xattn_smem_bytes(b.max_dq, true);
         k_xattn_bwd<<<b.sample1 - b.sample0, 256, smem, s>>>(
             tab, b.g0, cu, sample_slot, b.sample0, ws.kbuf, ws.vbuf, ws.ldkv, ws.P, ws.dS, ws.dh,
-            ws.ld_h, ws.dk, ws.dv, ws.dQs);
+            ws.ld_h, ws.dk, ws.dv, ws.dQs, kv_grads ? 1 : 0);
         k_xattn_dq<NoOpt><<<dim3(b.n, (b.max_nq * b.max_dq + 255) / 256), 256, 0, s>>>(
             tab, no, nh, ws.dQs, ws.ld_h);
         k_xattn_gh<<<dim3(b.sample1 - b.sample0, d / 128), 256, 0, s>>>(
@@ -1055,15 +1173,16 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
 
 jnx_status heads_backward_front_launch(const HeadTable& tab, const HeadBatch& b,
                                        const HeadScratch& ws, int d, const uint16_t* hidden,
-                                       const int* cu, const int* sample_slot, cudaStream_t s) {
+                                       const int* cu, const int* sample_slot, bool kv_grads,
+                                       cudaStream_t s) {
     if (b.n == 0) return JNX_OK;
     k_head_back_in<<<dim3(b.n, (b.max_hid + 1023) / 1024, (b.max_ns + 7) / 8), 256, 0, s>>>(
         tab, ws.dy, ws.ld_y, ws.z, ws.ld_h, ws.dh);
     if (b.any_xattn) {
-        const size_t smem = xattn_smem_bytes(b.max_dq);
+        const size_t smem = xattn_smem_bytes(b.max_dq, true);
         k_xattn_bwd<<<b.sample1 - b.sample0, 256, smem, s>>>(
             tab, b.g0, cu, sample_slot, b.sample0, ws.kbuf, ws.vbuf, ws.ldkv, ws.P, ws.dS, ws.dh,
-            ws.ld_h, ws.dk, ws.dv, ws.dQs);
+            ws.ld_h, ws.dk, ws.dv, ws.dQs, kv_grads ? 1 : 0);
         k_xattn_gh<<<dim3(b.sample1 - b.sample0, d / 128), 256, 0, s>>>(
             tab, b.g0, cu, sample_slot, b.sample0, ws.P, ws.dS, hidden, d, ws.Gs, ws.Hs, d);
     }
@@ -1093,9 +1212,10 @@ jnx_status heads_backward_step_launch(const HeadTable& tab, const HeadOptTable& 
 
 jnx_status heads_set_smem() {
     static std::atomic<uint64_t> fwd{0}, bwd{0}, lin1{0}, lin2{0};
-    const int mx = (int)xattn_smem_bytes(512);
-    if (set_smem_limit(reinterpret_cast<const void*>(k_xattn_fwd), mx, fwd) != cudaSuccess ||
-        set_smem_limit(reinterpret_cast<const void*>(k_xattn_bwd), mx, bwd) != cudaSuccess ||
+    if (set_smem_limit(reinterpret_cast<const void*>(k_xattn_fwd),
+                       (int)xattn_smem_bytes(512, false), fwd) != cudaSuccess ||
+        set_smem_limit(reinterpret_cast<const void*>(k_xattn_bwd),
+                       (int)xattn_smem_bytes(512, true), bwd) != cudaSuccess ||
         set_smem_limit(reinterpret_cast<const void*>(k_head_lin<1>), kLinSmem, lin1) !=
             cudaSuccess ||
         set_smem_limit(reinterpret_cast<const void*>(k_head_lin<2>), kLinSmem, lin2) !=

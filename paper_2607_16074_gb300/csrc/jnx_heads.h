@@ -77,9 +77,12 @@ jnx_status heads_forward_launch(const HeadTable& tab, const HeadBatch& b, const 
                                 const float* pooled, int d, const int* cu, const int* sample_slot,
                                 const int* sample_target, const float* targets, float* preds,
                                 float* loss, cudaStream_t s);
+// kv_grads: also write the query heads' per-row dk, dv (read by the feature
+// gradient only).
 jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const HeadScratch& ws,
                                  const float* pooled, int d, const uint16_t* hidden,
-                                 const int* cu, const int* sample_slot, cudaStream_t s);
+                                 const int* cu, const int* sample_slot, bool kv_grads,
+                                 cudaStream_t s);
 // The backward with the tenant-private AdamW step fused into it, in two
 // launches so that nothing updates a parameter before every read of it:
 // front: the output layer's input gradient (reads W2 / Wout) and the query
@@ -91,7 +94,8 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
 // the queries' own update.
 jnx_status heads_backward_front_launch(const HeadTable& tab, const HeadBatch& b,
                                        const HeadScratch& ws, int d, const uint16_t* hidden,
-                                       const int* cu, const int* sample_slot, cudaStream_t s);
+                                       const int* cu, const int* sample_slot, bool kv_grads,
+                                       cudaStream_t s);
 jnx_status heads_backward_step_launch(const HeadTable& tab, const HeadOptTable& opt,
                                       const AdamHp& hp, const HeadBatch& b,
                                       const HeadScratch& ws, const float* pooled, int d,

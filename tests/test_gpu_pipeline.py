@@ -186,9 +186,12 @@ def test_query_heads_stage_on_synthetic_hidden_rows(nq, dq):
         lo, Y, gr = M.tenant_step(1, M.widen_tree(synth.to_numpy_tree(hw[t])), feats, T)
         assert abs(float(loss[t]) - lo) < 1e-4 * abs(lo)
         got = np.stack([f64(preds[s.target_off:s.target_off + tn.width]) for s in samples])
-        assert rel_err(got, Y) < 1e-4
-        for k, v in gr.items():
-            e = rel_err(f64(heads.grads[t][k]), v)
+        e_y = rel_err(got, Y)
+        e_g = {k: rel_err(f64(heads.grads[t][k]), v) for k, v in gr.items()}
+        print(f"query head nq={nq} dq={dq} tenant {t}: preds {e_y:.2e}, grads "
+              + ", ".join(f"{k} {e:.2e}" for k, e in e_g.items()))
+        assert e_y < 1e-4
+        for k, e in e_g.items():
             assert e < 1e-3, (t, k, e)
 
 
