@@ -625,7 +625,7 @@ def run_ours(args, rank, world, local_rank):
         step_tensor=dict(achieved=round(step_tf, 1), unit="TFLOP/s",
                          frac_of_burst=round(step_tf / peaks["bf16"], 4),
                          frac_of_sustained=round(step_tf / peaks["bf16_sustained"], 4),
-                         note="algorithmic FLOPs of one step (tensor-core GEMMs and attention, plus the heads CUDA-core FLOPs, under 0.01 %) / step time"),
+                         note="algorithmic FLOPs of one step (tensor-core GEMMs and attention, plus the heads' FLOPs, under 0.01 %) / step time"),
         per_tenant=speed,
         plan_ms=round(plan_ms, 3),
         kernels=per_kernel,
