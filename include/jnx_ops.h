@@ -131,6 +131,19 @@ jnx_status jnx_op_rms_backward(const float* x, const uint16_t* gamma, float eps,
 jnx_status jnx_op_gemm_glu_backward(const uint16_t* A, const uint16_t* W, int32_t M, int32_t F,
                                     int32_t K, uint16_t* gu, int32_t act, void* stream);
 
+/* The feed-forward backward's GLU step with the gate/up GEMM recomputed
+ * (what jnx_backbone_backward_lora runs per block): dm[M, F] = dy[M, d]
+ * w_down_t[F, d]^T is the gradient at act(g) * u; it is stored bf16 in the
+ * up columns of gu [M, 2F] (packed order: 128-column blocks alternating
+ * gate and up), then the gate/up GEMM g|u = n2[M, d] w_gu[2F, d]^T (w_gu in
+ * the packed order of jnx_pack_gate_up) leaves dg = dm u act'(g) in the gate
+ * columns and du = dm act(g) in the up columns, bf16.  gu needs no content
+ * on entry.  F % 256 == 0 (the GEMM's 256-column tiles), d % 64 == 0, gu
+ * 16-byte aligned, act a JNX_GLU_* value (JNX_ERR_INVALID_ARG otherwise). */
+jnx_status jnx_op_ffn_glu_backward(const uint16_t* dy, const uint16_t* w_down_t,
+                                   const uint16_t* n2, const uint16_t* w_gu, int32_t M, int32_t F,
+                                   int32_t d, int32_t act, uint16_t* gu, void* stream);
+
 /* The fused QKV projection + RoPE of jnx_op_gemm (JNX_EPI_ROPE) for callers
  * that cannot allocate device memory — e.g. a plugin in a serving process
  * whose pool owns every device allocation, or a batching worker that must

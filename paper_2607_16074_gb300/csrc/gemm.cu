@@ -20,6 +20,10 @@
 //              act(C_gate) * C_up -> bf16   (SwiGLU / tanh-GeGLU)
 //   EPI_ROPE   the fused Q|K|V projection: rotate-half RoPE at each row's
 //              position on columns < rope_cols, then bf16
+// and by the training paths (the GLU's backward, with the gate/up GEMM
+// recomputed): EPI_GLU_SAVE (the multipliers u act'(g) | act(g)),
+// EPI_GLU_BWD (dm times those multipliers), EPI_GLU_DM (the gate/up
+// product times a dm already stored in the up columns).
 // Every output element's K reduction runs in the same order whatever M is
 // or where the row sits, so packed (grouped) and per-tenant runs agree
 // bit for bit.
@@ -180,7 +184,7 @@ __device__ __forceinline__ float row_norm_scale(const GemmParams& p, int row, bo
 // row_base..row_base+31, 256 fp32 columns) -> the epilogue's output.
 // NC, cb: the 32-column chunks [cb, cb + NC) of the tile this warp handles
 // (all 8, or one half of 4 with eight epilogue warps: EPI_BF16, EPI_F32,
-// EPI_RESID without a folded norm and EPI_GLU_BWD only).  Ring slots are
+// EPI_RESID without a folded norm, EPI_GLU_BWD and EPI_GLU_DM only).  Ring slots are
 // indexed by the pass within this warp's range, so they stay compile-time.
 template <int EPI, int NC = 8>
 __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int lane,
@@ -198,8 +202,11 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
             uint4 v[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) v[u] = pack8_bf16(reinterpret_cast<const float*>(r) + 8 * u);
+            // a 32-column chunk never straddles a 128-column block
+            const int n = n0 + c * 32;
+            const int col = p.pack_up ? 256 * (n / 128) + 128 + n % 128 : n;
             stg_store_bf16(stg, lane, v, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
-                           n0 + c * 32, pol);
+                           col, pol);
         }
     } else if constexpr (EPI == EPI_F32 || EPI == EPI_RESID) {
         // 16 fp32 columns (64 bytes) per staging pass; the residual is
@@ -346,6 +353,55 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tbase, uint8_t* stg, int 
                     act_grad(rs * __uint_as_float(g[8 * q + e]), p.act, a, da);
                     og[e] = rs * __uint_as_float(u[8 * q + e]) * da;
                     ou[e] = a;
+                }
+                vg[q] = pack8_bf16(og);
+                vu[q] = pack8_bf16(ou);
+            }
+            stg_store_bf16(stg, lane, vg, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
+                           n0 + c * 32, pol);
+            stg_store_bf16(stg, lane, vu, static_cast<bf16_t*>(p.out), p.ldo, row_base, row_end,
+                           n0 + 128 + c * 32, pol);
+        }
+    } else if constexpr (EPI == EPI_GLU_DM) {
+        // as EPI_GLU_SAVE over the chunk pairs (gate c, up c + 4) of this
+        // warp's range (all four, or two of them with eight epilogue warps),
+        // with dm (this thread's row, the chunk's 32 F columns: 64
+        // contiguous bytes of the up slot, through L1 so each 32-byte sector
+        // is fetched once) loaded one chunk ahead; every lane of the warp has
+        // its chunk's dm in registers before any lane's stores reach that
+        // chunk's columns, so out may be aux
+        const int c0 = cb / 2, nc = NC / 2;
+        const float rs = row_norm_scale(p, my_row, valid);
+        const bf16_t* dmrow = p.aux + (size_t)my_row * p.ldaux + n0 + 128;
+        uint4 dmv[2][4];
+        auto load_dm = [&](int c, uint4 (&v)[4]) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                v[q] = valid ? *reinterpret_cast<const uint4*>(dmrow + c * 32 + 8 * q)
+                             : make_uint4(0u, 0u, 0u, 0u);
+        };
+        load_dm(c0, dmv[0]);
+#pragma unroll
+        for (int lc = 0; lc < nc; ++lc) {
+            const int c = c0 + lc;
+            uint32_t g[32], u[32];
+            tmem_ld32(tbase + c * 32, g);
+            tmem_ld32(tbase + (c + 4) * 32, u);
+            if (lc + 1 < nc) load_dm(c + 1, dmv[(lc + 1) & 1]);
+            tmem_ld_wait();
+            uint4 vg[4], vu[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint4 m4 = dmv[lc & 1][q];
+                const uint32_t mw[4] = {m4.x, m4.y, m4.z, m4.w};
+                float og[8], ou[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    float a, da;
+                    act_grad(rs * __uint_as_float(g[8 * q + e]), p.act, a, da);
+                    const float dm = bf2f((mw[e / 2] >> (16 * (e & 1))) & 0xFFFF);
+                    og[e] = dm * (rs * __uint_as_float(u[8 * q + e]) * da);
+                    ou[e] = dm * a;
                 }
                 vg[q] = pack8_bf16(og);
                 vu[q] = pack8_bf16(ou);
@@ -788,6 +844,17 @@ __global__ void __launch_bounds__(64 + 32 * EW, 1)
             const uint32_t acc_phase = (local >> 1) & 1;
             const TileGeo g = tile_geo<LORA>(tile, num_m, num_n, p, lg);
             const int row_base = g.row0 + q * 32;
+            if constexpr (EPI == EPI_GLU_DM) {
+                // this thread's dm for the tile (its row, its chunks of the
+                // up slot) into L2 while the tile's K loop runs
+                const int row = row_base + lane;
+                const int nbytes = (EW == 8 ? 2 : 4) * 64;
+                if (row < g.row_end)
+                    for (int b = 0; b < nbytes; b += 128)
+                        prefetch_l2(reinterpret_cast<const uint8_t*>(
+                                        p.aux + (size_t)row * p.ldaux + g.nb * BN + 128 + cb * 16) +
+                                    b);
+            }
             if (!mbar_wait(&tfull[acc], acc_phase) || *abort_flag) {
                 *abort_flag = 1;
                 report(p.status, JNX_ERR_TIMEOUT);
@@ -881,7 +948,7 @@ static cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, cons
                               const GemmParams& p, int grid, cudaStream_t s) {
     static_assert(EW == 4 || (EW == 8 && !LORA &&
                               (EPI == EPI_BF16 || EPI == EPI_F32 || EPI == EPI_RESID ||
-                               EPI == EPI_GLU_BWD)),
+                               EPI == EPI_GLU_BWD || EPI == EPI_GLU_DM)),
                   "eight epilogue warps: column-splittable epilogues without LoRA only");
     constexpr int smem = LORA ? gemm::SMEM_BYTES_LORA
                               : (EW == 8 ? gemm::SMEM_BYTES_EW8 : gemm::SMEM_BYTES);
@@ -939,6 +1006,9 @@ jnx_status gemm_launch(const uint16_t* A, int lda, const uint16_t* B, int ldb, G
             e = launch_epi<EPI_GLU_BWD, false, NoLora, 8>(ta, tb, none, p, grid, s);
             break;
         case EPI_GLU_SAVE: e = launch_epi<EPI_GLU_SAVE, false>(ta, tb, none, p, grid, s); break;
+        case EPI_GLU_DM:
+            e = launch_epi<EPI_GLU_DM, false, NoLora, 8>(ta, tb, none, p, grid, s);
+            break;
         default: return fail(JNX_ERR_INVALID_ARG, "gemm: unknown epilogue %d", p.epi);
     }
     if (e != cudaSuccess) return fail(JNX_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));

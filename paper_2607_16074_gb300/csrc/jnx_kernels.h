@@ -12,7 +12,7 @@
 namespace jnx {
 
 enum { EPI_BF16 = 0, EPI_F32 = 1, EPI_RESID = 2, EPI_GLU = 3, EPI_ROPE = 4, EPI_GLU_BWD = 5,
-       EPI_GLU_SAVE = 6 };
+       EPI_GLU_SAVE = 6, EPI_GLU_DM = 7 };
 
 struct GemmParams {
     int M, N, K;
@@ -52,6 +52,14 @@ struct GemmParams {
     // du = dm act(g) in the up columns, bf16.
     const uint16_t* aux;
     int ldaux;
+    // EPI_GLU_DM: over the gate/up weights (as EPI_GLU); aux [M, ldaux]
+    // holds dm = dloss/d(act(g) * u) in the up columns of the packed order
+    // (F column f at packed column 256 (f / 128) + 128 + f % 128), and out
+    // (same layout; it may be aux itself) receives dg = dm u act'(g) in the
+    // gate columns and du = dm act(g) in the up columns, bf16.
+    // EPI_BF16 with pack_up set writes output column n to packed column
+    // 256 (n / 128) + 128 + n % 128 (dm into the up columns for EPI_GLU_DM).
+    int pack_up;
 };
 
 constexpr int kMaxRopePos = 1 << 16;  // longest sample a workspace reserves RoPE rows for

@@ -12,11 +12,11 @@
 // Per block, with dy = dloss/d(block output) (fp32) and its bf16 copy:
 //   recompute   n1 = RMSNorm(x), t = n1 A^T, q|k|v = RoPE(n1 W_qkv^T + t B^T),
 //               O = Attn (+ its log2-sum-exp), h = x + O W_o^T (+ adapter),
-//               n2 = RMSNorm(h); the gate/up GEMM's epilogue keeps the GLU
-//               backward's multipliers u act'(g) | act(g) (bf16, packed order)
-//   FFN         dm = dy W_down; dg|du = dm * multipliers (one GEMM, in place
-//               over the multipliers); dn2 = [dg|du] W_gu;
-//               dh = dy + RMSNorm'(h; dn2)
+//               n2 = RMSNorm(h)
+//   FFN         dm = dy W_down (bf16, into the up columns of the packed
+//               gate/up buffer); the gate/up GEMM recomputed from n2 with
+//               dg = dm u act'(g), du = dm act(g) in its epilogue (in place
+//               over dm); dn2 = [dg|du] W_gu; dh = dy + RMSNorm'(h; dn2)
 //   O           dO = dh W_o + (dh B_o) A_o;  dB_o = dh^T t_o, dA_o = (dh B_o)^T O
 //   attention   dq, dk, dv (tcgen05 passes, inverse RoPE on dq, dk)
 //   Q/K/V       dB = dY^T t, dA = (dY B)^T n1, dn1 = dqkv W_qkv + sum (dY B) A;
@@ -49,6 +49,45 @@ struct BwdWs {
     size_t part_floats;
     size_t bytes;
 };
+
+// The GLU's backward with its gate/up GEMM recomputed: dm [M, F] = dy
+// W_down^T (W_down^T stored as wdt [F, d]) goes, bf16, into the up columns
+// of gu [M, 2F] (packed order: 128-column blocks alternating gate and up);
+// the gate/up GEMM over the normed rows n2 [M, d] then leaves dg = dm u
+// act'(g) in the gate columns and du = dm act(g) in the up columns.  Each
+// up column is read by the tile that writes it, so no other buffer is
+// needed.
+static jnx_status ffn_glu_backward(const uint16_t* dy_bf, const uint16_t* wdt, const uint16_t* n2,
+                                   const uint16_t* w_gu, int64_t M, int64_t F, int64_t d, int act,
+                                   uint16_t* gu, int* status, cudaStream_t s) {
+    jnx_status st;
+    GemmParams p{};
+    p.M = (int)M;
+    p.N = (int)F;
+    p.K = (int)d;
+    p.epi = EPI_BF16;
+    p.pack_up = 1;
+    p.out = gu;
+    p.ldo = (int)(2 * F);
+    p.status = status;
+    {
+        TraceScope ts(JNX_K_GEMM_BWD, 2.0 * M * F * d, s);
+        if ((st = gemm_launch(dy_bf, (int)d, wdt, (int)d, p, s))) return st;
+    }
+    p = GemmParams{};
+    p.M = (int)M;
+    p.N = (int)(2 * F);
+    p.K = (int)d;
+    p.epi = EPI_GLU_DM;
+    p.out = gu;
+    p.ldo = (int)(2 * F);
+    p.aux = gu;
+    p.ldaux = (int)(2 * F);
+    p.act = act;
+    p.status = status;
+    TraceScope ts(JNX_K_GEMM_GU, 2.0 * M * 2.0 * F * d, s);
+    return gemm_launch(n2, (int)d, w_gu, (int)d, p, s);
+}
 
 BwdWs carve_bwd(const jnx_backbone* bb, int64_t N, void* base) {
     uint8_t* p = static_cast<uint8_t*>(base);
@@ -273,36 +312,13 @@ extern "C" jnx_status jnx_backbone_backward_lora(const jnx_backbone* bb, const j
             TraceScope ts(JNX_K_RMSNORM, Nd * 6.0, s);
             if ((st = rmsnorm_launch(w.xh, L.ffn_norm, bb->eps, N, d, w.n2, s))) return st;
         }
-        p = GemmParams{};
-        p.M = N;
-        p.N = 2 * F;
-        p.K = d;
-        p.epi = EPI_GLU_SAVE;  // u act'(g) | act(g): the GLU backward's multipliers
-        p.out = w.gu;
-        p.ldo = 2 * F;
-        p.act = bb->glu;
-        p.status = w.status;
-        {
-            TraceScope ts(JNX_K_GEMM_GU, 2.0 * N * 2.0 * F * d, s);
-            if ((st = gemm_launch(w.n2, d, L.w_gu, d, p, s))) return st;
-        }
-
         // ---------------- feed-forward backward ----------------
-        p = GemmParams{};
-        p.M = N;
-        p.N = F;
-        p.K = d;
-        p.epi = EPI_GLU_BWD;
-        p.out = w.gu;
-        p.ldo = 2 * F;
-        p.aux = w.gu;
-        p.ldaux = 2 * F;
-        p.act = bb->glu;
-        p.status = w.status;
-        {
-            TraceScope ts(JNX_K_GEMM_BWD, 2.0 * N * F * d, s);
-            if ((st = gemm_launch(w.dy_bf, d, Lt.w_down_t, d, p, s))) return st;
-        }
+        // dm = dy W_down (the gradient at act(g) * u) into the up columns of
+        // gu, then the gate/up GEMM recomputed from the normed rows n2 with
+        // dg = dm u act'(g) and du = dm act(g) formed in its epilogue
+        if ((st = ffn_glu_backward(w.dy_bf, Lt.w_down_t, w.n2, L.w_gu, N, F, d, bb->glu, w.gu,
+                                   w.status, s)))
+            return st;
         p = GemmParams{};
         p.M = N;
         p.N = d;
@@ -506,6 +522,23 @@ extern "C" jnx_status jnx_op_rms_backward(const float* x, const uint16_t* gamma,
         return fail(JNX_ERR_INVALID_ARG, "rms backward: null argument");
     return rms_bwd_launch(x, gamma, eps, dn, dres, M, d, dx, dx_bf,
                           static_cast<cudaStream_t>(stream));
+}
+
+extern "C" jnx_status jnx_op_ffn_glu_backward(const uint16_t* dy, const uint16_t* w_down_t,
+                                              const uint16_t* n2, const uint16_t* w_gu, int32_t M,
+                                              int32_t F, int32_t d, int32_t act, uint16_t* gu,
+                                              void* stream) {
+    clear_error();
+    if (M < 0 || F <= 0 || d <= 0)
+        return fail(JNX_ERR_INVALID_ARG, "ffn glu backward: bad sizes");
+    if (M > 0 && (!dy || !w_down_t || !n2 || !w_gu || !gu))
+        return fail(JNX_ERR_INVALID_ARG, "ffn glu backward: null argument");
+    if ((reinterpret_cast<uintptr_t>(gu) & 15) || F % 256 || d % 64)
+        return fail(JNX_ERR_INVALID_ARG, "ffn glu backward: gu alignment, F %% 256 or d %% 64");
+    if (act != JNX_GLU_SWIGLU && act != JNX_GLU_GEGLU_TANH)
+        return fail(JNX_ERR_INVALID_ARG, "ffn glu backward: unknown activation %d", act);
+    return ffn_glu_backward(dy, w_down_t, n2, w_gu, M, F, d, act, gu, nullptr,
+                            static_cast<cudaStream_t>(stream));
 }
 
 extern "C" jnx_status jnx_op_gemm_glu_backward(const uint16_t* A, const uint16_t* W, int32_t M,

@@ -181,7 +181,7 @@ EXPORTS = ("jnx_last_error", "jnx_version", "jnx_group_plan", "jnx_group_attn_it
            "jnx_backbone_backward_workspace_bytes", "jnx_backbone_backward_lora",
            "jnx_op_attention_lse", "jnx_op_attention_backward_prep",
            "jnx_op_attention_backward_workspace_bytes", "jnx_op_attention_backward",
-           "jnx_op_rms_backward", "jnx_op_gemm_glu_backward", "jnx_flow_workspace_bytes",
+           "jnx_op_rms_backward", "jnx_op_gemm_glu_backward", "jnx_op_ffn_glu_backward", "jnx_flow_workspace_bytes",
            "jnx_flow_forward", "jnx_flow_backward", "jnx_flow_sample", "jnx_adamw_tensors")
 
 
@@ -240,6 +240,7 @@ def lib() -> C.CDLL:
                                             vp, f32, vp, vp, sz, vp, vp]),
         "jnx_op_rms_backward": (i32, [vp, vp, f32, vp, vp, i32, i32, vp, vp, vp]),
         "jnx_op_gemm_glu_backward": (i32, [vp, vp, i32, i32, i32, vp, i32, vp]),
+        "jnx_op_ffn_glu_backward": (i32, [vp, vp, vp, vp, i32, i32, i32, i32, vp, vp]),
         "jnx_flow_workspace_bytes": (sz, [C.POINTER(jnx_flow_head), C.POINTER(jnx_group)]),
         "jnx_flow_forward": (i32, [C.POINTER(jnx_flow_head), C.POINTER(jnx_group), vp, vp, vp,
                                    vp, vp, vp, vp, sz, vp]),

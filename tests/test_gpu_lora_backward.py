@@ -16,7 +16,8 @@ from paper_2607_16074_gb300 import jnx as J
 from paper_2607_16074_gb300 import runtime as R
 from tests import bf16_emulation as E
 from tests.gpu_helpers import f64, randn_bf16, stream
-from tests.helpers import BF16_TOL, check_bf16_out, gate, oracle_requests, rel_err
+from tests.helpers import (BF16_TOL, check_bf16_out, gate, oracle_requests, rel_err,
+                           rel_err_bf16_out)
 
 pytestmark = pytest.mark.gpu
 
@@ -105,6 +106,44 @@ def test_glu_backward_gemms_vs_oracle(act):
     # against the multipliers as stored (the bf16 they were rounded to)
     check_bf16_out(got[:, gcol], dm * saved[:, gcol], 1e-3, f"glu backward dg {act}")
     check_bf16_out(got[:, gcol + 128], dm * saved[:, gcol + 128], 1e-3, f"glu backward du {act}")
+
+
+@pytest.mark.parametrize("act", [0, 1])
+def test_ffn_glu_backward_vs_oracle(act):
+    # the GLU step as the LoRA backward runs it: dm = dy W_down goes, bf16,
+    # into the up columns of gu, then the recomputed gate/up GEMM forms
+    # dg = dm u act'(g) and du = dm act(g) from it in place (gu starts as NaN:
+    # nothing is read before it is written).  Gated at the floor of the
+    # stage's own rounding points (dm stored in bf16, outputs in bf16),
+    # emulated in fp64.
+    bf16 = E.bf16
+    M_, F, d = 300, 512, 256
+    n2 = randn_bf16((M_, d), 8)
+    wg, wu = randn_bf16((F, d), 9, std=0.05), randn_bf16((F, d), 10, std=0.05)
+    w_gu = torch.empty((2 * F, d), dtype=torch.bfloat16, device="cuda")
+    J.check(J.lib().jnx_pack_gate_up(wg.data_ptr(), wu.data_ptr(), F, d, w_gu.data_ptr(),
+                                     stream()))
+    dy = randn_bf16((M_, d), 5)
+    wdt = randn_bf16((F, d), 6, std=0.05)
+    gu = torch.full((M_, 2 * F), float("nan"), dtype=torch.bfloat16, device="cuda")
+    J.check(J.lib().jnx_op_ffn_glu_backward(dy.data_ptr(), wdt.data_ptr(), n2.data_ptr(),
+                                            w_gu.data_ptr(), M_, F, d, act, gu.data_ptr(),
+                                            stream()))
+    torch.cuda.synchronize()
+    g = f64(n2) @ f64(wg).T
+    u = f64(n2) @ f64(wu).T
+    a = M.silu(g) if act == 0 else M.gelu_tanh(g)
+    da = M.silu_grad(g) if act == 0 else B.gelu_tanh_grad(g)
+    dm = f64(dy) @ f64(wdt).T
+    f = np.arange(F)
+    gcol = (f // 128) * 256 + f % 128
+    got = f64(gu)
+    assert np.isfinite(got).all()
+    for name, cols, ref, emu in (("dg", gcol, dm * u * da, bf16(bf16(dm) * u * da)),
+                                 ("du", gcol + 128, dm * a, bf16(bf16(dm) * a))):
+        floor = rel_err(emu, ref)
+        tol = max(1e-3, 1.5 * rel_err_bf16_out(emu, ref))
+        check_bf16_out(got[:, cols], ref, tol, f"ffn glu backward {name} {act}", floor=floor)
 
 
 def _attn_case(lengths, H, Hkv, hd, seed, qk_std=1.0):
