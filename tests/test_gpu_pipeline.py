@@ -72,6 +72,40 @@ def test_grouped_equals_isolated_on_gpu():
         assert torch.equal(st1.pooled[:len(idx[t])], full_pooled[idx[t]])
 
 
+def test_empty_plan_and_zero_sizes_write_nothing():
+    """Degenerate inputs: a GEMM of zero rows, attention over zero samples,
+    and a whole grouped step (backbone, heads forward, loss, heads backward)
+    over the plan of an empty request queue all return JNX_OK and leave
+    every output as it was."""
+    from tests.gpu_helpers import randn_bf16, stream
+    L = J.lib()
+    A = randn_bf16((1, 256), 1)
+    W = randn_bf16((256, 256), 2, 0.05)
+    out = torch.full((1, 256), 7.0, device="cuda")
+    J.check(L.jnx_op_gemm(A.data_ptr(), W.data_ptr(), 0, 256, 256, J.JNX_EPI_F32,
+                          out.data_ptr(), 256, None, 0, 0, 0, 0.0, 0, None, 0, stream()))
+    qkv = randn_bf16((1, 3 * 128), 3)
+    o = torch.full((1, 128), 7.0, dtype=torch.bfloat16, device="cuda")
+    cu = torch.zeros(1, dtype=torch.int32, device="cuda")
+    J.check(L.jnx_op_attention(qkv.data_ptr(), 0, 1, 1, 128, cu.data_ptr(), 0, 0, o.data_ptr(),
+                               None, stream()))
+    w = synth.make_workload("tiny")
+    s = Setup(w)
+    plan = J.jnx_group_plan(w.schemas(), [], len(w.tenants), w.max_samples, w.max_tokens)
+    assert plan.n_samples == 0 and plan.n_tokens == 0 and plan.n_slots == 0
+    g = R.DeviceGroup(plan)
+    step = R.GroupedStep(s.bb, s.heads, g)
+    preds = torch.full_like(s.inp_d["targets"], 7.0)
+    grads_before = [v.clone() for gr in s.heads.grads for v in gr.values()]
+    step.run(s.inp_d["vision"], s.inp_d["text_ids"], s.inp_d["targets"], preds)
+    R.check_status(step.ws_bb)
+    R.check_status(step.ws_h)
+    torch.cuda.synchronize()
+    assert (out == 7).all() and (o == 7).all() and (preds == 7).all()
+    for a, b in zip(grads_before, [v for gr in s.heads.grads for v in gr.values()]):
+        assert torch.equal(a, b)
+
+
 def test_slots_outside_the_group_are_not_touched():
     w = synth.make_workload("small")
     s = Setup(w)
