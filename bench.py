@@ -273,6 +273,17 @@ def head_bytes(w, plan):
     return fwd, bwd
 
 
+def attention_executed_flops(cu_seqlens, H, hd):
+    """FLOPs one attention launch executes on the tensor cores: per sample
+    of L tokens and query head, ceil(L / 128) query tiles of 128 rows times
+    ceil(L / 64) key tiles of 64, for both products (S = Q K^T, O += P V),
+    masked entries included."""
+    L = np.diff(np.asarray(cu_seqlens, dtype=np.int64))
+    rows = -(-L // 128) * 128
+    keys = -(-L // 64) * 64
+    return float(4.0 * H * hd * np.sum(rows * keys))
+
+
 def kernel_breakdown(J, kinds, ms, work, bytes_per_launch=None):
     """Per traced kernel kind: launches, total ms, share of the traced time
     and its rate: TFLOP/s for the tcgen05 kinds, GFLOP/s for the head kinds
@@ -562,6 +573,14 @@ def run_ours(args, rank, world, local_rank):
     g_tf = g_flops / (g_ms / 1e3) / 1e12 if g_ms > 0 else 0.0
     hb = head_bytes(w, plan)
     per_kernel = kernel_breakdown(J, kinds, ms, work, {10: hb[0], 11: hb[1]} if hb else None)
+    att = kinds == 4
+    if att.any() and "attention" in per_kernel:
+        # the attention row's rate counts 4 L^2 H hd per sample; the kernel
+        # also computes the masked parts of its 128-query and 64-key tiles
+        ex = attention_executed_flops(plan.cu_seqlens, w.backbone.n_heads, w.backbone.head_dim)
+        a_ms = float(ms[att].sum())
+        per_kernel["attention"]["tflops_executed"] = round(
+            ex * int(att.sum()) / (a_ms / 1e3) / 1e12, 1)
     step_flops = float(work[np.isin(kinds, J.TENSOR_KERNELS + (10, 11))].sum()) / args.steps
     step_tf = step_flops / (t_ms / args.steps / 1e3) / 1e12
     # the dominant kernel: the gate/up projection GEMM (largest share of the step)
