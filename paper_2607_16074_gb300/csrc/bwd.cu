@@ -4,7 +4,9 @@
 //   k_transpose     bf16 [batch][rows][cols] -> [batch][cols][rows] (the
 //                   frozen weights' transposes, read by the input-gradient
 //                   GEMMs; the adapters' B^T each step)
-//   k_rms_bwd       RMSNorm backward with the residual gradient added
+//   k_rms_bwd       RMSNorm backward with the residual gradient added (one
+//                   warp per row; k_rms_bwd_row, one CTA per row with the
+//                   row in registers, for 1024 <= d <= 4096)
 //   k_attn_bwd_prep attention's dO in bf16 and D = rowsum(dO * O) per head
 //   k_seg_up        per tenant segment  out[rows] (+)= sum_p T_p W_p[t]
 //                   (LoRA up-projections of gradients; the query heads'
@@ -190,12 +192,87 @@ __global__ void __launch_bounds__(256) k_rms_bwd(const float* __restrict__ x,
     }
 }
 
+// The same for 1024 <= d <= 4096: one 256-thread CTA per row, each thread
+// holding NU float4 units of x and dn (units tid, tid + 256, ...) in
+// registers, so every input byte is read once; the row sums are combined
+// over the warps in a fixed order.
+template <int NU>
+__global__ void __launch_bounds__(256) k_rms_bwd_row(const float* __restrict__ x,
+                                                     const uint16_t* __restrict__ gamma, float eps,
+                                                     const float* __restrict__ dn, const float* dres,
+                                                     int d, float* dx, uint16_t* dx_bf) {
+    __shared__ float red[2][8];
+    const size_t row = blockIdx.x;
+    const int units = d / 4, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const float* xr = x + row * d;
+    const float* dr = dn + row * d;
+    float4 xv[NU], dv[NU];
+    uint2 gv[NU];
+    float ss = 0.f, sd = 0.f;
+#pragma unroll
+    for (int i = 0; i < NU; ++i) {
+        const int u = threadIdx.x + 256 * i;
+        xv[i] = dv[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        gv[i] = make_uint2(0u, 0u);
+        if (u < units) {
+            xv[i] = *reinterpret_cast<const float4*>(xr + 4 * u);
+            dv[i] = *reinterpret_cast<const float4*>(dr + 4 * u);
+            gv[i] = *reinterpret_cast<const uint2*>(gamma + 4 * u);
+        }
+        ss += xv[i].x * xv[i].x + xv[i].y * xv[i].y + xv[i].z * xv[i].z + xv[i].w * xv[i].w;
+        sd += bf2f(gv[i].x & 0xFFFF) * dv[i].x * xv[i].x + bf2f(gv[i].x >> 16) * dv[i].y * xv[i].y +
+              bf2f(gv[i].y & 0xFFFF) * dv[i].z * xv[i].z + bf2f(gv[i].y >> 16) * dv[i].w * xv[i].w;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        sd += __shfl_xor_sync(0xffffffffu, sd, o);
+    }
+    if (lane == 0) {
+        red[0][warp] = ss;
+        red[1][warp] = sd;
+    }
+    __syncthreads();
+    ss = sd = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) {
+        ss += red[0][w];
+        sd += red[1][w];
+    }
+    const float s = rsqrtf(ss / (float)d + eps);
+    const float k = s * s * s * sd / (float)d;
+#pragma unroll
+    for (int i = 0; i < NU; ++i) {
+        const int u = threadIdx.x + 256 * i;
+        if (u >= units) continue;
+        float4 r = dres ? *reinterpret_cast<const float4*>(dres + row * d + 4 * u)
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+        r.x += s * bf2f(gv[i].x & 0xFFFF) * dv[i].x - xv[i].x * k;
+        r.y += s * bf2f(gv[i].x >> 16) * dv[i].y - xv[i].y * k;
+        r.z += s * bf2f(gv[i].y & 0xFFFF) * dv[i].z - xv[i].z * k;
+        r.w += s * bf2f(gv[i].y >> 16) * dv[i].w - xv[i].w * k;
+        *reinterpret_cast<float4*>(dx + row * d + 4 * u) = r;
+        if (dx_bf)
+            *reinterpret_cast<uint2*>(dx_bf + row * d + 4 * u) =
+                make_uint2(pack_bf2(r.x, r.y), pack_bf2(r.z, r.w));
+    }
+}
+
 jnx_status rms_bwd_launch(const float* x, const uint16_t* gamma, float eps, const float* dn,
                           const float* dres, int M, int d, float* dx, uint16_t* dx_bf,
                           cudaStream_t s) {
     if (d % 128) return fail(JNX_ERR_UNSUPPORTED, "rms backward: d %% 128 != 0");
     if (M <= 0) return JNX_OK;
-    k_rms_bwd<<<(M + 7) / 8, 256, 0, s>>>(x, gamma, eps, dn, dres, M, d, dx, dx_bf);
+    if (d >= 1024 && d <= 4096) {
+        if (d <= 1024)
+            k_rms_bwd_row<1><<<M, 256, 0, s>>>(x, gamma, eps, dn, dres, d, dx, dx_bf);
+        else if (d <= 2048)
+            k_rms_bwd_row<2><<<M, 256, 0, s>>>(x, gamma, eps, dn, dres, d, dx, dx_bf);
+        else
+            k_rms_bwd_row<4><<<M, 256, 0, s>>>(x, gamma, eps, dn, dres, d, dx, dx_bf);
+    } else {
+        k_rms_bwd<<<(M + 7) / 8, 256, 0, s>>>(x, gamma, eps, dn, dres, M, d, dx, dx_bf);
+    }
     cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? JNX_OK : fail(JNX_ERR_CUDA, "rms backward: %s", cudaGetErrorString(e));
 }

@@ -52,21 +52,28 @@ def test_transpose_exact():
     assert torch.equal(dst, src.transpose(1, 2))
 
 
-def test_rms_backward_vs_oracle():
-    M_, d = 37, 512
+@pytest.mark.parametrize("d,mode", [(512, "dres"), (1024, "none"), (2048, "dres"),
+                                    (2048, "in place"), (3072, "dres"), (4096, "dres")])
+def test_rms_backward_vs_oracle(d, mode):
+    # d = 512: one warp per row; 1024..4096: one CTA per row (3072 leaves part
+    # of the last register slot of each thread unused); dres absent, separate
+    # or dx itself
+    M_ = 37
     g = torch.Generator().manual_seed(3)
     x = torch.randn(M_, d, generator=g).cuda()
     dn = torch.randn(M_, d, generator=g).cuda()
     dres = torch.randn(M_, d, generator=g).cuda()
     gamma = randn_bf16((d,), 4, std=0.1) + 1.0
-    dx = torch.empty_like(x)
+    dx = dres.clone() if mode == "in place" else torch.empty_like(x)
     dxb = torch.empty((M_, d), dtype=torch.bfloat16, device="cuda")
+    src = {"dres": dres.data_ptr(), "none": None, "in place": dx.data_ptr()}[mode]
     J.check(J.lib().jnx_op_rms_backward(x.data_ptr(), gamma.data_ptr(), 1e-6, dn.data_ptr(),
-                                        dres.data_ptr(), M_, d, dx.data_ptr(), dxb.data_ptr(),
-                                        stream()))
+                                        src, M_, d, dx.data_ptr(), dxb.data_ptr(), stream()))
     torch.cuda.synchronize()
-    ref = f64(dres) + B.rmsnorm_backward(f64(x), f64(gamma), 1e-6, f64(dn))
-    # fp32 arithmetic over d = 512 terms
+    ref = B.rmsnorm_backward(f64(x), f64(gamma), 1e-6, f64(dn))
+    if mode != "none":
+        ref = ref + f64(dres)
+    # fp32 arithmetic over d terms
     assert rel_err(f64(dx), ref) < 1e-5
     assert torch.equal(dxb, dx.to(torch.bfloat16))
 
