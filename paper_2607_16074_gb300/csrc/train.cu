@@ -57,7 +57,7 @@ struct BwdWs {
 // act'(g) in the gate columns and du = dm act(g) in the up columns.  Each
 // up column is read by the tile that writes it, so no other buffer is
 // needed.
-static jnx_status ffn_glu_backward(const uint16_t* dy_bf, const uint16_t* wdt, const uint16_t* n2,
+jnx_status ffn_glu_backward(const uint16_t* dy_bf, const uint16_t* wdt, const uint16_t* n2,
                                    const uint16_t* w_gu, int64_t M, int64_t F, int64_t d, int act,
                                    uint16_t* gu, int* status, cudaStream_t s) {
     jnx_status st;
