@@ -416,7 +416,12 @@ __global__ void __launch_bounds__(256) k_head_back_in(const __grid_constant__ He
 }
 
 // MLP first-layer gradient: dW1[j, k] = sum_s dz[s, j] p[s, k]; db1[j] = sum_s dz[s, j].
-// One CTA per (slot, j, 1024-column block); float4 columns.
+// One CTA per (slot, kDw1Rows rows j, 1024-column block); a thread holds
+// float4 columns of the block's rows, so each feature load serves all of
+// them, and the loop over the slot's samples (in order, per element) is
+// unrolled so that several samples' loads are in flight.
+constexpr int kDw1Rows = 8;
+
 template <class OT>
 __global__ void __launch_bounds__(256) k_mlp_dw1(const __grid_constant__ HeadTable tab,
                                                  const __grid_constant__ OT opt, AdamHp hp,
@@ -424,33 +429,47 @@ __global__ void __launch_bounds__(256) k_mlp_dw1(const __grid_constant__ HeadTab
                                                  const float* __restrict__ p, int ld_p) {
     const HeadSlot& hs = tab.slot[blockIdx.x];
     if (hs.kind != JNX_HEAD_MLP) return;
-    const int j = blockIdx.y;
-    if (j >= hs.hid) return;
+    const int j0 = blockIdx.y * kDw1Rows;
+    if (j0 >= hs.hid) return;
+    const int nj = min(kDw1Rows, hs.hid - j0);
     const int k4 = blockIdx.z * 256 + threadIdx.x;
     if (k4 * 4 < hs.d_in) {
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 acc[kDw1Rows];
+#pragma unroll
+        for (int r = 0; r < kDw1Rows; ++r) acc[r] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
         for (int s = hs.s0; s < hs.s1; ++s) {
-            const float g = dz[(size_t)s * ld + j];
             const float4 x = *reinterpret_cast<const float4*>(p + (size_t)s * ld_p + k4 * 4);
-            acc.x += g * x.x;
-            acc.y += g * x.y;
-            acc.z += g * x.z;
-            acc.w += g * x.w;
+            const float* g = dz + (size_t)s * ld + j0;
+#pragma unroll
+            for (int r = 0; r < kDw1Rows; ++r) {
+                const float gr = r < nj ? g[r] : 0.f;
+                acc[r].x += gr * x.x;
+                acc[r].y += gr * x.y;
+                acc[r].z += gr * x.z;
+                acc[r].w += gr * x.w;
+            }
         }
-        float4* dst = reinterpret_cast<float4*>(hs.g_w1 + (size_t)j * hs.d_in + k4 * 4);
-        if (hs.accum) {
-            const float4 old = *dst;
-            acc.x += old.x;
-            acc.y += old.y;
-            acc.z += old.z;
-            acc.w += old.w;
+#pragma unroll
+        for (int r = 0; r < kDw1Rows; ++r) {
+            if (r >= nj) break;
+            const size_t at = (size_t)(j0 + r) * hs.d_in + k4 * 4;
+            float4 a = acc[r];
+            if (hs.accum) {
+                const float4 old = *reinterpret_cast<const float4*>(hs.g_w1 + at);
+                a.x += old.x;
+                a.y += old.y;
+                a.z += old.z;
+                a.w += old.w;
+            }
+            if constexpr (kFused<OT>)
+                opt_step4(opt.slot[blockIdx.x], 0, at, a, hp);
+            else
+                *reinterpret_cast<float4*>(hs.g_w1 + at) = a;
         }
-        if constexpr (kFused<OT>)
-            opt_step4(opt.slot[blockIdx.x], 0, (size_t)j * hs.d_in + k4 * 4, acc, hp);
-        else
-            *dst = acc;
     }
-    if (blockIdx.z == 0 && threadIdx.x == 0) {
+    if (blockIdx.z == 0 && threadIdx.x < nj) {
+        const int j = j0 + threadIdx.x;
         float accb = 0.f;
         for (int s = hs.s0; s < hs.s1; ++s) accb += dz[(size_t)s * ld + j];
         const float gb = hs.accum ? hs.g_b1[j] + accb : accb;
@@ -1154,7 +1173,8 @@ jnx_status heads_backward_launch(const HeadTable& tab, const HeadBatch& b, const
     k_head_back_in<<<dim3(b.n, (b.max_hid + 1023) / 1024, (b.max_ns + 7) / 8), 256, 0, s>>>(
         tab, ws.dy, ws.ld_y, ws.z, ws.ld_h, ws.dh);
     if (b.any_mlp)
-        k_mlp_dw1<NoOpt><<<dim3(b.n, b.max_mlp_hid, (d / 4 + 255) / 256), 256, 0, s>>>(
+        k_mlp_dw1<NoOpt><<<dim3(b.n, (b.max_mlp_hid + kDw1Rows - 1) / kDw1Rows, (d / 4 + 255) / 256),
+                           256, 0, s>>>(
             tab, no, nh, ws.dh, ws.ld_h, pooled, d);
     if (b.any_xattn) {
         const size_t smem = xattn_smem_bytes(b.max_dq, true);
@@ -1198,7 +1218,9 @@ jnx_status heads_backward_step_launch(const HeadTable& tab, const HeadOptTable& 
         <<<dim3(b.n, (b.max_width + 15) / 16, (b.max_hid + 255) / 256), 256, 0, s>>>(
             tab, opt, hp, ws.dy, ws.ld_y, ws.h, ws.ld_h);
     if (b.any_mlp)
-        k_mlp_dw1<HeadOptTable><<<dim3(b.n, b.max_mlp_hid, (d / 4 + 255) / 256), 256, 0, s>>>(
+        k_mlp_dw1<HeadOptTable>
+            <<<dim3(b.n, (b.max_mlp_hid + kDw1Rows - 1) / kDw1Rows, (d / 4 + 255) / 256), 256, 0,
+               s>>>(
             tab, opt, hp, ws.dh, ws.ld_h, pooled, d);
     if (b.any_xattn) {
         // wgrad reads the learned queries, which dq then updates
